@@ -1,0 +1,216 @@
+"""Seeded synthetic workloads for the homogenized StackLSTM step.
+
+This module draws the inputs that both the CUDA path and the fp64 oracle consume:
+the discrete op streams, x, W, bias and the initial state. It holds none of the
+StackLSTM arithmetic -- only random draws, the op-stream generators (which track the
+stack depth solely to keep every stream valid) and the round-to-nearest-even
+rounding of inputs to bf16, so that both sides see bit-identical input values.
+
+Op encoding follows the unified pointer update of Sec. 3 (p <- p + op): push = +1,
+pop = -1, hold = 0 (the hold op is introduced for arc-eager / arc-hybrid, Sec. 3,
+last paragraph). The arc-standard stream generator flattens each transition of
+Table 1 into primitive stack ops: Shift -> push, Left-Arc -> pop, pop, push,
+Right-Arc -> pop.
+
+Random draws use numpy's PCG64 (``numpy.random.default_rng(seed)``) in this fixed
+order: (1) per-instance lengths and op choices, instance-major then time;
+(2) x in [T, B, I] C order; (3) W; (4) bias, h0 and c0 when a variant asks for them
+(zeros otherwise).
+"""
+from __future__ import annotations
+
+import dataclasses
+import math
+from typing import Optional, Sequence
+
+import numpy as np
+
+PUSH, POP, HOLD = 1, -1, 0
+
+
+# ----------------------------------------------------------------------------- bf16
+def to_bf16_bits(a: np.ndarray) -> np.ndarray:
+    """Round float32 values to bf16 (round to nearest, ties to even); return the bits."""
+    u = np.ascontiguousarray(a, dtype=np.float32).view(np.uint32)
+    bias = ((u >> np.uint32(16)) & np.uint32(1)) + np.uint32(0x7FFF)
+    return ((u + bias) >> np.uint32(16)).astype(np.uint16)
+
+
+def bf16_bits_to_f32(bits: np.ndarray) -> np.ndarray:
+    """Widen bf16 bit patterns exactly to float32."""
+    return (np.ascontiguousarray(bits, dtype=np.uint16).astype(np.uint32) << np.uint32(16)).view(np.float32)
+
+
+def round_to_bf16(a: np.ndarray) -> np.ndarray:
+    """float32 array holding the bf16-rounded values of ``a``."""
+    return bf16_bits_to_f32(to_bf16_bits(a))
+
+
+# ------------------------------------------------------------------------ op streams
+def ops_random_walk(rng: np.random.Generator, B: int, T: int,
+                    probs: Sequence[float], lengths: Optional[np.ndarray] = None) -> np.ndarray:
+    """Ops [T, B] int8 drawn per step with probabilities (push, pop, hold).
+
+    A pop is never drawn at depth 0: there the pop weight is dropped and the push and
+    hold weights are renormalised. Steps at or beyond an instance's length are holds.
+    One uniform per (instance, step) is drawn, instance-major.
+    """
+    w_push, w_pop, w_hold = (float(v) for v in probs)
+    u = rng.random((B, T))  # instance-major draw order
+    ops = np.zeros((T, B), dtype=np.int8)
+    depth = np.zeros(B, dtype=np.int64)
+    lim = np.full(B, T, dtype=np.int64) if lengths is None else np.asarray(lengths, dtype=np.int64)
+    tot = w_push + w_pop + w_hold
+    t_push, t_pop = w_push / tot, (w_push + w_pop) / tot
+    t_push0 = w_push / (w_push + w_hold)
+    for t in range(T):
+        ut = u[:, t]
+        at_bottom = depth == 0
+        op = np.where(ut < t_push, PUSH, np.where(ut < t_pop, POP, HOLD))
+        op0 = np.where(ut < t_push0, PUSH, HOLD)
+        op = np.where(at_bottom, op0, op)
+        op = np.where(t < lim, op, HOLD)
+        ops[t] = op
+        depth += op
+    return ops
+
+
+def arc_standard_transitions(rng: np.random.Generator, n: int) -> list:
+    """One uniformly random valid arc-standard transition sequence over n tokens.
+
+    At each parser state the next transition is chosen uniformly among the valid ones:
+    Shift while the buffer is non-empty, Left-Arc and Right-Arc while the token stack
+    holds at least two tokens. The sequence ends with an empty buffer and one token on
+    the stack, so it has 2n - 1 transitions.
+    """
+    buf, stack, seq = n, 0, []
+    while buf > 0 or stack > 1:
+        valid = []
+        if buf > 0:
+            valid.append("S")
+        if stack >= 2:
+            valid += ["LA", "RA"]
+        tr = valid[int(rng.integers(len(valid)))]
+        seq.append(tr)
+        if tr == "S":
+            buf -= 1
+            stack += 1
+        else:
+            stack -= 1
+    return seq
+
+
+ARC_STANDARD_OPS = {"S": (PUSH,), "LA": (POP, POP, PUSH), "RA": (POP,)}
+
+
+def ops_arc_standard(rng: np.random.Generator, B: int, n_range=(10, 60)):
+    """Per instance: n ~ U{n_lo..n_hi}, a random valid arc-standard sequence, flattened
+    to primitive ops (Table 1) and padded with holds to the batch maximum.
+    Returns (ops [T, B] int8, lengths [B] int32)."""
+    streams = []
+    for _ in range(B):
+        n = int(rng.integers(n_range[0], n_range[1] + 1))
+        flat = []
+        for tr in arc_standard_transitions(rng, n):
+            flat.extend(ARC_STANDARD_OPS[tr])
+        streams.append(flat)
+    T = max(len(s) for s in streams)
+    ops = np.zeros((T, B), dtype=np.int8)
+    for b, s in enumerate(streams):
+        ops[: len(s), b] = s
+    return ops, np.array([len(s) for s in streams], dtype=np.int32)
+
+
+# ------------------------------------------------------------------------- workload
+@dataclasses.dataclass
+class Workload:
+    """One batch of synthetic input. Float arrays are float32; for the bf16 path they
+    already hold bf16-representable values (x, W, h0), so the oracle and the kernels
+    consume bit-identical inputs. c0, bias and the loss seed stay float32."""
+
+    name: str
+    T: int
+    B: int
+    I: int
+    H: int
+    dtype: str  # "fp32" or "bf16"
+    seed: int
+    ops: np.ndarray  # [T, B] int8 in {-1, 0, 1}
+    lengths: np.ndarray  # [B] int32, real (non-padding) steps per instance
+    x: np.ndarray  # [T, B, I]
+    W: np.ndarray  # [I + H, 4H], gate column blocks i, f, g, o
+    bias: np.ndarray  # [4H]
+    h0: np.ndarray  # [B, H]
+    c0: np.ndarray  # [B, H]
+    d_top_h: np.ndarray  # [B, H] gradient of the loss w.r.t. the final top h
+    dy: Optional[np.ndarray] = None  # [T, B, H] gradient w.r.t. y_t, or None
+
+    @property
+    def real_step_share(self) -> float:
+        return float(self.lengths.sum()) / float(self.T * self.B)
+
+    def bits(self, name: str) -> np.ndarray:
+        """bf16 bit pattern of x, W or h0 (bf16 workloads only)."""
+        assert self.dtype == "bf16"
+        return to_bf16_bits(getattr(self, name))
+
+
+def make_workload(name: str, T: Optional[int], B: int, I: int, H: int, dtype: str, seed: int,
+                  ops_kind: str, probs=(1 / 3, 1 / 3, 1 / 3), len_range=None,
+                  bias_scale: float = 0.0, h0_scale: float = 0.0, c0_scale: float = 0.0,
+                  dy_scale: float = 0.0, n_range=(10, 60)) -> Workload:
+    """Draw one workload. ``ops_kind`` is "random_walk" (needs T and probs, optional
+    len_range for ragged hold-padded lengths) or "arc_standard" (T = batch maximum)."""
+    rng = np.random.default_rng(seed)
+    if ops_kind == "arc_standard":
+        ops, lengths = ops_arc_standard(rng, B, n_range)
+        T = ops.shape[0]
+    elif ops_kind == "random_walk":
+        if len_range is not None:
+            lengths = rng.integers(len_range[0], len_range[1] + 1, size=B).astype(np.int32)
+        else:
+            lengths = np.full(B, T, dtype=np.int32)
+        ops = ops_random_walk(rng, B, T, probs, lengths)
+    else:
+        raise ValueError(ops_kind)
+    x = rng.standard_normal((T, B, I), dtype=np.float32)
+    r = 1.0 / math.sqrt(H)
+    W = rng.uniform(-r, r, size=(I + H, 4 * H)).astype(np.float32)
+    bias = (rng.uniform(-bias_scale, bias_scale, size=4 * H) if bias_scale else np.zeros(4 * H)).astype(np.float32)
+    h0 = (rng.uniform(-h0_scale, h0_scale, size=(B, H)) if h0_scale else np.zeros((B, H))).astype(np.float32)
+    c0 = (rng.uniform(-c0_scale, c0_scale, size=(B, H)) if c0_scale else np.zeros((B, H))).astype(np.float32)
+    dy = rng.standard_normal((T, B, H), dtype=np.float32) * np.float32(dy_scale) if dy_scale else None
+    if dtype == "bf16":
+        x, W, h0 = round_to_bf16(x), round_to_bf16(W), round_to_bf16(h0)
+    elif dtype != "fp32":
+        raise ValueError(dtype)
+    return Workload(name=name, T=int(T), B=B, I=I, H=H, dtype=dtype, seed=seed, ops=ops,
+                    lengths=lengths, x=x, W=W, bias=bias, h0=h0, c0=c0,
+                    d_top_h=np.ones((B, H), dtype=np.float32), dy=dy)
+
+
+# The five synthetic workloads, shaped like the parsing workloads of Sec. 4.1
+# (hidden size 200) and like larger string-to-tree decoders.
+CONFIGS = {
+    "tiny": dict(T=12, B=4, I=16, H=16, dtype="fp32", seed=0, ops_kind="random_walk",
+                 probs=(1 / 3, 1 / 3, 1 / 3)),
+    "parser64": dict(T=None, B=64, I=200, H=200, dtype="bf16", seed=1, ops_kind="arc_standard"),
+    "sweep": dict(T=None, B=(1, 8, 32, 128, 512, 1024), I=200, H=200, dtype="bf16", seed=2,
+                  ops_kind="arc_standard"),
+    "large": dict(T=256, B=256, I=512, H=1024, dtype="bf16", seed=3, ops_kind="random_walk",
+                  probs=(0.5, 0.3, 0.2), len_range=(64, 256)),
+    "stress": dict(T=512, B=4096, I=256, H=256, dtype="bf16", seed=4, ops_kind="random_walk",
+                   probs=(0.6, 0.3, 0.1)),
+}
+
+
+def config_workload(name: str, B: Optional[int] = None) -> Workload:
+    """The named workload. ``sweep`` needs B (one of its batch sizes)."""
+    cfg = dict(CONFIGS[name])
+    if name == "sweep":
+        if B is None or B not in cfg["B"]:
+            raise ValueError("sweep needs B in %s" % (cfg["B"],))
+        cfg["B"] = B
+    elif B is not None and B != cfg["B"]:
+        raise ValueError("%s has fixed B=%d" % (name, cfg["B"]))
+    return make_workload(name=name, **cfg)
