@@ -1,0 +1,142 @@
+/*
+ * stacklstm.h -- C ABI of the GB300 (sm_103a) homogenized StackLSTM step.
+ *
+ * The library runs the minibatched, homogenized StackLSTM of Ding & Koehn,
+ * "Parallelizable Stack Long Short-Term Memory" (arXiv:1904.03409), forward and
+ * backward, on one GPU:
+ *   - every step, every instance b reads the (h, c) state at its stack-top pointer p[b],
+ *     computes the LSTM gates from [x_t ; h_p] with one fused gate contraction, writes
+ *     the new state to stack slot p[b] + 1 and moves p[b] by its op (push +1, pop -1,
+ *     hold 0), whatever the op is (Algorithm 1; unified pointer update, Sec. 3);
+ *   - the step output is the top after the pointer update (Algorithm 1, return value);
+ *   - cell states move with hidden states (footnote to Sec. 2);
+ *   - the backward runs in reverse time and routes gradients to every state a step read,
+ *     including states later popped or overwritten (Sec. 5).
+ *
+ * LSTM cell (the paper names only "LSTM"): z = [x ; h] W + bias with W of shape
+ * [I + H, 4H], row-major, gate column blocks in the order i, f, g, o;
+ * i, f, o = sigmoid, g = tanh; c' = f c + i g; h' = o tanh(c').
+ *
+ * Conventions for every call below:
+ *   - All tensor pointers are DEVICE pointers on the handle's device, C-ordered
+ *     (row-major, last index fastest), owned by the caller, and must be 16-byte aligned.
+ *   - Calls are asynchronous with respect to the GPU and ordered on the handle's stream.
+ *     In the default synchronous mode, forward and backward synchronize the stream before
+ *     returning and report device-detected errors (bad op, underflow); in async mode
+ *     (stacklstm_set_async) they return after enqueueing and stacklstm_status reports.
+ *   - No call aborts, traps or prints. Each returns a status; stacklstm_last_error gives
+ *     a one-line message for the last failure on a handle.
+ *   - Device-detected errors never cause out-of-bounds accesses: a bad op or a pop at
+ *     depth 0 is recorded and then treated as a hold, so every index stays in range.
+ *
+ * Element types by dtype:
+ *   SL_FP32: x, h0, W, h_stack, y are float; every computation in fp32 on CUDA cores
+ *            (no tensor cores, no TF32).
+ *   SL_BF16: x, h0, W, h_stack, y are bf16 (uint16 bit patterns); the gate contractions
+ *            run on tcgen05 tensor cores with fp32 accumulation; cell states, gradients
+ *            and all accumulations are fp32. Requires I % 8 == 0 and H % 8 == 0.
+ *   c0, c_stack, bias and every gradient are float in both modes.
+ */
+#ifndef STACKLSTM_H
+#define STACKLSTM_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct stacklstm *stacklstm_t;
+
+typedef enum {
+    SL_OK = 0,
+    SL_ERR_ARG = 1,         /* null handle or pointer, size out of range, misaligned pointer */
+    SL_ERR_OP = 2,          /* an op outside {-1, 0, +1} (the op set of Sec. 3)            */
+    SL_ERR_UNDERFLOW = 3,   /* a pop at stack depth 0 (undefined in the paper)             */
+    SL_ERR_STATE = 4,       /* backward without a completed forward on the handle          */
+    SL_ERR_CUDA = 5,        /* a CUDA runtime error (message in stacklstm_last_error)       */
+    SL_ERR_TIMEOUT = 6,     /* a bounded device-side wait ran out; the context stays usable */
+    SL_ERR_UNSUPPORTED = 7, /* sizes or device this build's kernels do not support         */
+    SL_ERR_OOM = 8          /* device workspace allocation failed                          */
+} sl_status;
+
+typedef enum { SL_FP32 = 0, SL_BF16 = 1 } sl_dtype;
+
+/*
+ * stacklstm_create -- allocate a handle and its device workspace for one problem size.
+ *   T      time steps (>= 1); the stack has T + 1 slots, so it can never overflow
+ *          (the paper fixes 150 slots, Sec. 4.1; here capacity follows T).
+ *   B      batch instances (>= 1); I input width (>= 1); H hidden width (>= 1).
+ *   dtype  SL_FP32 or SL_BF16 (see above).
+ *   device CUDA device ordinal; stream: a cudaStream_t (NULL = legacy default stream).
+ * The workspace (state history, saved gates, gradient history, indices) is owned by the
+ * handle until stacklstm_destroy. Returns SL_ERR_ARG, SL_ERR_UNSUPPORTED or SL_ERR_OOM
+ * on failure, leaving *out NULL.
+ */
+sl_status stacklstm_create(stacklstm_t *out, int T, int B, int I, int H, sl_dtype dtype,
+                           int device, void *stream);
+
+/* Replace the stream later calls are ordered on. */
+sl_status stacklstm_set_stream(stacklstm_t s, void *stream);
+
+/* async != 0: forward/backward return after enqueueing; stacklstm_status reports. */
+sl_status stacklstm_set_async(stacklstm_t s, int async);
+
+/*
+ * stacklstm_forward -- T homogenized steps (Algorithm 1) for all B instances.
+ * Inputs:
+ *   x     [T, B, I]  input vectors x_t (dtype)
+ *   ops   [T, B]     int8 ops in {-1, 0, +1}; a pop needs depth > 0
+ *   h0    [B, H]     initial hidden state, stack slot 0 (dtype)
+ *   c0    [B, H]     initial cell state (float)
+ *   W     [I+H, 4H]  gate weights (dtype); rows 0..I-1 act on x, rows I.. on h
+ *   bias  [4H]       gate bias (float)
+ * Outputs (all nullable except p_final):
+ *   h_stack [T+1, B, H] final slot-indexed stack, hidden part (dtype); slot 0 is h0,
+ *                       slots no step wrote are 0. Slots above the top hold what
+ *                       Algorithm 1 last wrote there.
+ *   c_stack [T+1, B, H] the same for cell states (float)
+ *   p_final [B]         final stack pointers
+ *   p_traj  [T+1, B]    pointer before each step and after the last (p_traj[0] = 0);
+ *                       step t reads slot p_traj[t] and writes slot p_traj[t] + 1
+ *   src     [T+1, B]    provenance of the top at each time: 0 is the initial state,
+ *                       t + 1 is the state written at step t; src[t] is what step t read
+ *   y       [T, B, H]   step outputs: h at the top after step t's pointer move (dtype)
+ * The handle keeps what backward needs (a packed copy of W, the states read, the gates),
+ * so x and W may change after forward returns.
+ */
+sl_status stacklstm_forward(stacklstm_t s, const void *x, const int8_t *ops, const void *h0,
+                            const float *c0, const void *W, const float *bias, void *h_stack,
+                            float *c_stack, int32_t *p_final, int32_t *p_traj, int32_t *src,
+                            void *y);
+
+/*
+ * stacklstm_backward -- reverse-time backward of the last forward on this handle for the
+ * loss L = sum(d_top_h * h_top_final) + sum_t sum(dy_t * y_t).
+ * Inputs (nullable; NULL means zero): d_top_h [B, H], dy [T, B, H] (float).
+ * Outputs (float; each nullable): dx [T, B, I], dh0 [B, H], dc0 [B, H],
+ * dW [I+H, 4H], dbias [4H]. Gradients are overwritten, not accumulated.
+ * Every reduction runs in a fixed order with no atomics, so results are bitwise
+ * reproducible run to run. Returns SL_ERR_STATE without a preceding forward.
+ */
+sl_status stacklstm_backward(stacklstm_t s, const float *d_top_h, const float *dy, float *dx,
+                             float *dh0, float *dc0, float *dW, float *dbias);
+
+/* Synchronize the handle's stream and return (then clear) any device-detected error. */
+sl_status stacklstm_status(stacklstm_t s);
+
+/* Free the handle and its workspace (synchronizes its stream first). NULL is a no-op. */
+sl_status stacklstm_destroy(stacklstm_t s);
+
+/* Static, human-readable name of a status code. */
+const char *stacklstm_status_string(sl_status st);
+
+/* One-line message for the last failure on the handle ("" if none). Valid until the
+ * next call on the handle. */
+const char *stacklstm_last_error(stacklstm_t s);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* STACKLSTM_H */

@@ -1,0 +1,170 @@
+"""Thin ctypes binding of libstacklstm.so (include/stacklstm.h).
+
+Argument marshalling only: every computation runs in the library's CUDA kernels.
+PyTorch supplies device memory and the stream. Functions keep the C names; tensors are
+passed as torch tensors (device, dtype and shape are checked here, then only their data
+pointers cross the boundary). If the library is missing this module raises; there is no
+fallback.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import re
+from typing import Optional
+
+from . import build as _build
+
+SL_FP32, SL_BF16 = 0, 1
+STATUS = {0: "SL_OK", 1: "SL_ERR_ARG", 2: "SL_ERR_OP", 3: "SL_ERR_UNDERFLOW", 4: "SL_ERR_STATE",
+          5: "SL_ERR_CUDA", 6: "SL_ERR_TIMEOUT", 7: "SL_ERR_UNSUPPORTED", 8: "SL_ERR_OOM"}
+HEADER = os.path.join(_build.ROOT, "include", "stacklstm.h")
+
+_lib = None
+
+
+class StackLSTMError(RuntimeError):
+    def __init__(self, status: int, where: str, message: str = ""):
+        super().__init__("%s: %s%s" % (where, STATUS.get(status, status), (" (%s)" % message) if message else ""))
+        self.status = status
+
+
+def header_functions():
+    """Names of the functions include/stacklstm.h declares."""
+    with open(HEADER) as f:
+        text = f.read()
+    return sorted(set(re.findall(r"^\s*(?:const\s+)?\w+\s*\*?\s*(stacklstm_\w+)\s*\(", text, re.M)))
+
+
+def load(path: Optional[str] = None):
+    """Load the library (built in-tree by ``build.build()``); raise if it is missing."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    path = path or _build.LIB
+    if not os.path.exists(path):
+        raise RuntimeError("libstacklstm.so is not built (%s); run paper_1904_03409_gb300.build.build()" % path)
+    lib = ctypes.CDLL(path)
+    vp, i, i32p = ctypes.c_void_p, ctypes.c_int, ctypes.c_void_p
+    lib.stacklstm_create.argtypes = [ctypes.POINTER(vp), i, i, i, i, i, i, vp]
+    lib.stacklstm_forward.argtypes = [vp] * 13
+    lib.stacklstm_backward.argtypes = [vp] * 8
+    lib.stacklstm_set_stream.argtypes = [vp, vp]
+    lib.stacklstm_set_async.argtypes = [vp, i]
+    lib.stacklstm_status.argtypes = [vp]
+    lib.stacklstm_destroy.argtypes = [vp]
+    lib.stacklstm_status_string.argtypes = [i]
+    lib.stacklstm_status_string.restype = ctypes.c_char_p
+    lib.stacklstm_last_error.argtypes = [vp]
+    lib.stacklstm_last_error.restype = ctypes.c_char_p
+    for fn in ("stacklstm_create", "stacklstm_forward", "stacklstm_backward", "stacklstm_set_stream",
+               "stacklstm_set_async", "stacklstm_status", "stacklstm_destroy"):
+        getattr(lib, fn).restype = ctypes.c_int
+    _lib = lib
+    return lib
+
+
+def _check(handle, st: int, where: str):
+    if st != 0:
+        msg = load().stacklstm_last_error(handle).decode() if handle else ""
+        raise StackLSTMError(st, where, msg)
+
+
+def _ptr(t, device=None, dtype=None, shape=None, name="tensor"):
+    if t is None:
+        return None
+    import torch
+    if not isinstance(t, torch.Tensor):
+        raise TypeError("%s must be a torch tensor" % name)
+    if not t.is_cuda or (device is not None and t.device.index != device):
+        raise ValueError("%s must live on cuda:%s" % (name, device))
+    if dtype is not None and t.dtype != dtype:
+        raise ValueError("%s must be %s, got %s" % (name, dtype, t.dtype))
+    if shape is not None and tuple(t.shape) != tuple(shape):
+        raise ValueError("%s must have shape %s, got %s" % (name, tuple(shape), tuple(t.shape)))
+    if not t.is_contiguous():
+        raise ValueError("%s must be contiguous" % name)
+    return ctypes.c_void_p(t.data_ptr())
+
+
+def stacklstm_status_string(st: int) -> str:
+    return load().stacklstm_status_string(int(st)).decode()
+
+
+def stacklstm_create(T: int, B: int, I: int, H: int, dtype: int, device: int = 0, stream=None):
+    """Create a handle. ``stream`` is a torch.cuda.Stream, a raw cudaStream_t int, or None
+    (the current torch stream of ``device``)."""
+    import torch
+    if stream is None:
+        stream = torch.cuda.current_stream(device)
+    raw = stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream)
+    h = ctypes.c_void_p()
+    _check(None, load().stacklstm_create(ctypes.byref(h), T, B, I, H, dtype, device, ctypes.c_void_p(raw)),
+           "stacklstm_create")
+    return StackLSTMHandle(h, T, B, I, H, dtype, device)
+
+
+class StackLSTMHandle:
+    """Owns one library handle; ``destroy`` (or garbage collection) frees it."""
+
+    def __init__(self, h, T, B, I, H, dtype, device):
+        self.h, self.T, self.B, self.I, self.H, self.dtype, self.device = h, T, B, I, H, dtype, device
+
+    @property
+    def tdtype(self):
+        import torch
+        return torch.bfloat16 if self.dtype == SL_BF16 else torch.float32
+
+    def destroy(self):
+        if self.h is not None and _lib is not None:
+            _lib.stacklstm_destroy(self.h)
+        self.h = None
+
+    def __del__(self):
+        try:
+            self.destroy()
+        except Exception:
+            pass
+
+
+def stacklstm_set_stream(hd: StackLSTMHandle, stream):
+    raw = stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream)
+    _check(hd.h, load().stacklstm_set_stream(hd.h, ctypes.c_void_p(raw)), "stacklstm_set_stream")
+
+
+def stacklstm_set_async(hd: StackLSTMHandle, on: bool):
+    _check(hd.h, load().stacklstm_set_async(hd.h, int(bool(on))), "stacklstm_set_async")
+
+
+def stacklstm_status(hd: StackLSTMHandle):
+    _check(hd.h, load().stacklstm_status(hd.h), "stacklstm_status")
+
+
+def stacklstm_forward(hd: StackLSTMHandle, x, ops, h0, c0, W, bias, h_stack=None, c_stack=None, p_final=None,
+                      p_traj=None, src=None, y=None):
+    """Forward over all T steps; see include/stacklstm.h for the layout of each tensor."""
+    import torch
+    T, B, I, H, d, dt = hd.T, hd.B, hd.I, hd.H, hd.device, hd.tdtype
+    args = [
+        _ptr(x, d, dt, (T, B, I), "x"), _ptr(ops, d, torch.int8, (T, B), "ops"), _ptr(h0, d, dt, (B, H), "h0"),
+        _ptr(c0, d, torch.float32, (B, H), "c0"), _ptr(W, d, dt, (I + H, 4 * H), "W"),
+        _ptr(bias, d, torch.float32, (4 * H,), "bias"), _ptr(h_stack, d, dt, (T + 1, B, H), "h_stack"),
+        _ptr(c_stack, d, torch.float32, (T + 1, B, H), "c_stack"), _ptr(p_final, d, torch.int32, (B,), "p_final"),
+        _ptr(p_traj, d, torch.int32, (T + 1, B), "p_traj"), _ptr(src, d, torch.int32, (T + 1, B), "src"),
+        _ptr(y, d, dt, (T, B, H), "y")]
+    _check(hd.h, load().stacklstm_forward(hd.h, *args), "stacklstm_forward")
+
+
+def stacklstm_backward(hd: StackLSTMHandle, d_top_h=None, dy=None, dx=None, dh0=None, dc0=None, dW=None,
+                       dbias=None):
+    """Backward of the last forward; gradients are overwritten."""
+    import torch
+    T, B, I, H, d, f = hd.T, hd.B, hd.I, hd.H, hd.device, torch.float32
+    args = [_ptr(d_top_h, d, f, (B, H), "d_top_h"), _ptr(dy, d, f, (T, B, H), "dy"),
+            _ptr(dx, d, f, (T, B, I), "dx"), _ptr(dh0, d, f, (B, H), "dh0"), _ptr(dc0, d, f, (B, H), "dc0"),
+            _ptr(dW, d, f, (I + H, 4 * H), "dW"), _ptr(dbias, d, f, (4 * H,), "dbias")]
+    _check(hd.h, load().stacklstm_backward(hd.h, *args), "stacklstm_backward")
+
+
+def stacklstm_destroy(hd: StackLSTMHandle):
+    hd.destroy()

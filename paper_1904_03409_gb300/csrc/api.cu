@@ -1,0 +1,263 @@
+// api.cu -- the C ABI (include/stacklstm.h): argument checks, workspace ownership and
+// the order of launches for forward and backward. All arithmetic runs in the kernels of
+// index_kernels.cu, fp32_path.cu and bf16_path.cu.
+#include <stdio.h>
+
+#include <algorithm>
+#include <new>
+
+#include "common.cuh"
+
+namespace {
+
+struct DeviceGuard {
+    int prev = -1;
+    explicit DeviceGuard(int dev)
+    {
+        if (cudaGetDevice(&prev) != cudaSuccess) prev = -1;
+        if (prev != dev) cudaSetDevice(dev);
+    }
+    ~DeviceGuard()
+    {
+        int cur = -1;
+        if (prev >= 0 && cudaGetDevice(&cur) == cudaSuccess && cur != prev) cudaSetDevice(prev);
+    }
+};
+
+sl_status fail(stacklstm *s, sl_status st, const char *msg)
+{
+    if (s) s->last_error = msg ? msg : "";
+    return st;
+}
+
+sl_status cuda_fail(stacklstm *s, cudaError_t e, const char *where)
+{
+    if (s) {
+        char buf[256];
+        snprintf(buf, sizeof buf, "%s: %s", where, cudaGetErrorString(e));
+        s->last_error = buf;
+    }
+    return SL_ERR_CUDA;
+}
+
+bool aligned16(const void *p) { return ((uintptr_t)p & 15u) == 0; }
+
+size_t elem_size(sl_dtype dt) { return dt == SL_BF16 ? 2 : 4; }
+
+void free_all(stacklstm *s)
+{
+    for (void *p : s->allocs) cudaFree(p);
+    s->allocs.clear();
+}
+
+template <typename P>
+bool alloc(stacklstm *s, P **out, size_t bytes)
+{
+    void *p = nullptr;
+    if (bytes == 0) bytes = 16;
+    if (cudaMalloc(&p, bytes) != cudaSuccess) {
+        cudaGetLastError();  // clear the sticky-free allocation error
+        return false;
+    }
+    s->allocs.push_back(p);
+    *out = (P *)p;
+    return true;
+}
+
+// Reads back the device error flag (synchronizing the stream) and clears it.
+sl_status read_status(stacklstm *s)
+{
+    int32_t h = 0;
+    cudaError_t e = cudaMemcpyAsync(&h, s->err, sizeof h, cudaMemcpyDeviceToHost, s->stream);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s->stream);
+    if (e != cudaSuccess) return cuda_fail(s, e, "synchronize");
+    if (h != SL_OK) {
+        e = cudaMemsetAsync(s->err, 0, sizeof(int32_t), s->stream);
+        if (e == cudaSuccess) e = cudaStreamSynchronize(s->stream);
+        if (e != cudaSuccess) return cuda_fail(s, e, "clear status");
+        const char *what = h == SL_ERR_OP ? "op outside {-1, 0, +1}"
+                           : h == SL_ERR_UNDERFLOW ? "pop at stack depth 0"
+                           : h == SL_ERR_TIMEOUT ? "device-side wait ran out"
+                           : "device error";
+        return fail(s, (sl_status)h, what);
+    }
+    return SL_OK;
+}
+
+}  // namespace
+
+namespace sl {
+cudaError_t configure_prepass(stacklstm *s);
+}
+
+extern "C" {
+
+const char *stacklstm_status_string(sl_status st)
+{
+    switch (st) {
+    case SL_OK: return "ok";
+    case SL_ERR_ARG: return "invalid argument";
+    case SL_ERR_OP: return "op outside {-1, 0, +1}";
+    case SL_ERR_UNDERFLOW: return "pop at stack depth 0";
+    case SL_ERR_STATE: return "backward without a forward";
+    case SL_ERR_CUDA: return "CUDA error";
+    case SL_ERR_TIMEOUT: return "device-side wait timed out";
+    case SL_ERR_UNSUPPORTED: return "unsupported sizes or device";
+    case SL_ERR_OOM: return "out of device memory";
+    }
+    return "unknown status";
+}
+
+const char *stacklstm_last_error(stacklstm_t s) { return s ? s->last_error.c_str() : "null handle"; }
+
+sl_status stacklstm_create(stacklstm_t *out, int T, int B, int I, int H, sl_dtype dtype, int device,
+                           void *stream)
+{
+    if (!out) return SL_ERR_ARG;
+    *out = nullptr;
+    if (T < 1 || B < 1 || I < 1 || H < 1 || (dtype != SL_FP32 && dtype != SL_BF16)) return SL_ERR_ARG;
+    // 32-bit launch-shape limits and int32 history indices
+    if (B > 65535 || (long long)T * B > (1LL << 31) - 1 || T > (1 << 30)) return SL_ERR_UNSUPPORTED;
+    if (dtype == SL_BF16 && sl::bf16_unsupported(T, B, I, H)) return SL_ERR_UNSUPPORTED;
+
+    int ndev = 0;
+    if (cudaGetDeviceCount(&ndev) != cudaSuccess || device < 0 || device >= ndev) {
+        cudaGetLastError();
+        return SL_ERR_ARG;
+    }
+    DeviceGuard g(device);
+    stacklstm *s = new (std::nothrow) stacklstm;
+    if (!s) return SL_ERR_OOM;
+    s->T = T; s->B = B; s->I = I; s->H = H; s->dt = dtype; s->device = device;
+    s->stream = (cudaStream_t)stream;
+    if (cudaDeviceGetAttribute(&s->num_sms, cudaDevAttrMultiProcessorCount, device) != cudaSuccess) {
+        delete s;
+        return SL_ERR_UNSUPPORTED;
+    }
+    const size_t TB = (size_t)T * B, T1B = (size_t)(T + 1) * B, K = (size_t)I + H, G = 4 * (size_t)H;
+    const size_t es = elem_size(dtype);
+    bool ok = alloc(s, &s->p_traj, T1B * 4) && alloc(s, &s->top, T1B * 4) && alloc(s, &s->slot_last, T1B * 4) &&
+              alloc(s, &s->err, 16) && alloc(s, &s->hist_h, T1B * H * es) && alloc(s, &s->hist_c, T1B * H * 4) &&
+              alloc(s, &s->gates, TB * G * (dtype == SL_BF16 ? 2 : 4)) && alloc(s, &s->a_rm, TB * K * es) &&
+              alloc(s, &s->dhist_h, T1B * H * 4) && alloc(s, &s->dhist_c, T1B * H * 4) &&
+              alloc(s, &s->dG, TB * G * es);
+    if (ok && dtype == SL_FP32) ok = alloc(s, &s->w_fwd, K * G * 4);
+    if (ok && dtype == SL_BF16) ok = sl::bf16_prepare(s) == cudaSuccess;
+    if (ok) ok = sl::configure_prepass(s) == cudaSuccess;
+    if (ok && !s->prepass_smem) ok = alloc(s, &s->slot_scratch, T1B * 4);
+    if (ok) ok = cudaMemset(s->err, 0, 16) == cudaSuccess;
+    if (!ok) {
+        cudaGetLastError();
+        free_all(s);
+        delete s;
+        return SL_ERR_OOM;
+    }
+    *out = s;
+    return SL_OK;
+}
+
+sl_status stacklstm_set_stream(stacklstm_t s, void *stream)
+{
+    if (!s) return SL_ERR_ARG;
+    s->stream = (cudaStream_t)stream;
+    return SL_OK;
+}
+
+sl_status stacklstm_set_async(stacklstm_t s, int async)
+{
+    if (!s) return SL_ERR_ARG;
+    s->async = async != 0;
+    return SL_OK;
+}
+
+sl_status stacklstm_forward(stacklstm_t s, const void *x, const int8_t *ops, const void *h0, const float *c0,
+                            const void *W, const float *bias, void *h_stack, float *c_stack, int32_t *p_final,
+                            int32_t *p_traj, int32_t *src, void *y)
+{
+    if (!s) return SL_ERR_ARG;
+    s->last_error.clear();
+    if (!x || !ops || !h0 || !c0 || !W || !bias || !p_final)
+        return fail(s, SL_ERR_ARG, "x, ops, h0, c0, W, bias and p_final are required");
+    const void *ptrs[] = {x, h0, c0, W, bias, h_stack, c_stack, p_final, p_traj, src, y};
+    for (const void *p : ptrs)
+        if (p && !aligned16(p)) return fail(s, SL_ERR_ARG, "tensor pointers must be 16-byte aligned");
+    DeviceGuard g(s->device);
+    const int T = s->T, B = s->B, H = s->H;
+    const size_t es = elem_size(s->dt);
+    cudaError_t e;
+    s->fwd_done = 0;
+    if ((e = sl::launch_prepass(s, ops))) return cuda_fail(s, e, "prepass");
+    if (s->dt == SL_FP32)
+        e = sl::fp32_forward(s, (const float *)x, (const float *)h0, c0, (const float *)W, bias);
+    else
+        e = sl::bf16_forward(s, (const __nv_bfloat16 *)x, (const __nv_bfloat16 *)h0, c0,
+                             (const __nv_bfloat16 *)W, bias);
+    if (e) return cuda_fail(s, e, "forward");
+    if ((e = cudaMemcpyAsync(p_final, s->p_traj + (size_t)T * B, sizeof(int32_t) * B, cudaMemcpyDeviceToDevice,
+                             s->stream)))
+        return cuda_fail(s, e, "p_final");
+    if (p_traj && (e = cudaMemcpyAsync(p_traj, s->p_traj, sizeof(int32_t) * (T + 1) * B, cudaMemcpyDeviceToDevice,
+                                       s->stream)))
+        return cuda_fail(s, e, "p_traj");
+    if (src && (e = cudaMemcpyAsync(src, s->top, sizeof(int32_t) * (T + 1) * B, cudaMemcpyDeviceToDevice,
+                                    s->stream)))
+        return cuda_fail(s, e, "src");
+    if (y && (e = sl::launch_gather_rows(s, s->top + B, T * B, es, s->hist_h, y, H))) return cuda_fail(s, e, "y");
+    if (h_stack && (e = sl::launch_gather_rows(s, s->slot_last, (T + 1) * B, es, s->hist_h, h_stack, H)))
+        return cuda_fail(s, e, "h_stack");
+    if (c_stack && (e = sl::launch_gather_rows(s, s->slot_last, (T + 1) * B, 4, s->hist_c, c_stack, H)))
+        return cuda_fail(s, e, "c_stack");
+    s->fwd_done = 1;
+    return s->async ? SL_OK : read_status(s);
+}
+
+sl_status stacklstm_backward(stacklstm_t s, const float *d_top_h, const float *dy, float *dx, float *dh0,
+                             float *dc0, float *dW, float *dbias)
+{
+    if (!s) return SL_ERR_ARG;
+    s->last_error.clear();
+    if (!s->fwd_done) return fail(s, SL_ERR_STATE, "backward needs a completed forward on this handle");
+    const void *ptrs[] = {d_top_h, dy, dx, dh0, dc0, dW, dbias};
+    for (const void *p : ptrs)
+        if (p && !aligned16(p)) return fail(s, SL_ERR_ARG, "tensor pointers must be 16-byte aligned");
+    DeviceGuard g(s->device);
+    const int T = s->T, B = s->B, H = s->H;
+    const size_t hist_bytes = sizeof(float) * (size_t)(T + 1) * B * H;
+    cudaError_t e;
+    if ((e = cudaMemsetAsync(s->dhist_h, 0, hist_bytes, s->stream))) return cuda_fail(s, e, "clear");
+    if ((e = cudaMemsetAsync(s->dhist_c, 0, hist_bytes, s->stream))) return cuda_fail(s, e, "clear");
+    if ((e = sl::launch_seed_grads(s, d_top_h, dy))) return cuda_fail(s, e, "seed");
+    if (s->dt == SL_FP32)
+        e = sl::fp32_backward(s, dx, dW, dbias);
+    else
+        e = sl::bf16_backward(s, dx, dW, dbias);
+    if (e) return cuda_fail(s, e, "backward");
+    // slot 0 always holds the initial state, which is history row 0
+    if (dh0 && (e = cudaMemcpyAsync(dh0, s->dhist_h, sizeof(float) * B * H, cudaMemcpyDeviceToDevice, s->stream)))
+        return cuda_fail(s, e, "dh0");
+    if (dc0 && (e = cudaMemcpyAsync(dc0, s->dhist_c, sizeof(float) * B * H, cudaMemcpyDeviceToDevice, s->stream)))
+        return cuda_fail(s, e, "dc0");
+    return s->async ? SL_OK : read_status(s);
+}
+
+sl_status stacklstm_status(stacklstm_t s)
+{
+    if (!s) return SL_ERR_ARG;
+    DeviceGuard g(s->device);
+    return read_status(s);
+}
+
+sl_status stacklstm_destroy(stacklstm_t s)
+{
+    if (!s) return SL_OK;
+    {
+        DeviceGuard g(s->device);
+        cudaStreamSynchronize(s->stream);
+        free_all(s);
+        cudaGetLastError();
+    }
+    delete s;
+    return SL_OK;
+}
+
+}  // extern "C"

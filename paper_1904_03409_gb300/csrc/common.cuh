@@ -1,0 +1,76 @@
+// common.cuh -- internal declarations shared by the library's translation units.
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include <string>
+#include <vector>
+
+#include "../../include/stacklstm.h"
+
+// The handle: problem sizes, stream, and the device workspace it owns.
+struct stacklstm {
+    int T = 0, B = 0, I = 0, H = 0;
+    sl_dtype dt = SL_FP32;
+    int device = 0;
+    cudaStream_t stream = nullptr;
+    int async = 0;
+    int fwd_done = 0;
+    int num_sms = 0;
+    int prepass_smem = 0;  // dynamic shared memory of the index prepass (0: global scratch)
+
+    // integer bookkeeping, written by the prepass (all [T+1][B] int32)
+    int32_t *p_traj = nullptr;     // pointer before step t (t = T: after the last step)
+    int32_t *top = nullptr;        // history index of the top at time t ("src")
+    int32_t *slot_last = nullptr;  // history index last written to each slot (-1: never)
+    int32_t *slot_scratch = nullptr;  // global slot-tag stack when it does not fit on chip
+    int32_t *err = nullptr;           // device-detected status (first error wins)
+
+    // forward state, write-once history: index 0 = initial state, t+1 = written at step t
+    void *hist_h = nullptr;  // [T+1][B][H] dtype
+    float *hist_c = nullptr;  // [T+1][B][H]
+    void *gates = nullptr;    // [T][B][4H] activated i,f,g,o (fp32 path: float, bf16: half)
+    void *a_rm = nullptr;     // [T][B][I+H] the contraction operand [x_t ; h_read] (dtype)
+
+    // backward state
+    float *dhist_h = nullptr;  // [T+1][B][H] gradient w.r.t. each history state
+    float *dhist_c = nullptr;  // [T+1][B][H]
+    void *dG = nullptr;        // [T][B][4H] gate pre-activation gradients (fp32 / bf16)
+
+    // packed weights (taken at forward)
+    void *w_fwd = nullptr;  // fp32: W^T [4H][I+H] float; bf16: forward operand tiles
+    void *w_bwd = nullptr;  // bf16: backward operand tiles
+    float *dw_part = nullptr;  // split-K partials of the weight-gradient contraction
+    size_t dw_part_elems = 0;
+
+    std::string last_error;
+    std::vector<void *> allocs;
+};
+
+namespace sl {
+
+// ---- index / gather kernels (index_kernels.cu)
+cudaError_t launch_prepass(stacklstm *s, const int8_t *ops);
+cudaError_t launch_gather_rows(stacklstm *s, const int32_t *idx, int rows, size_t elem_bytes,
+                               const void *hist, void *out, int row_elems);
+cudaError_t launch_seed_grads(stacklstm *s, const float *d_top_h, const float *dy);
+
+// ---- fp32 CUDA-core path (fp32_path.cu)
+cudaError_t fp32_forward(stacklstm *s, const float *x, const float *h0, const float *c0,
+                         const float *W, const float *bias);
+cudaError_t fp32_backward(stacklstm *s, float *dx, float *dW, float *dbias);
+
+// ---- bf16 tensor-core path (bf16_path.cu)
+cudaError_t bf16_prepare(stacklstm *s);
+cudaError_t bf16_forward(stacklstm *s, const __nv_bfloat16 *x, const __nv_bfloat16 *h0,
+                         const float *c0, const __nv_bfloat16 *W, const float *bias);
+cudaError_t bf16_backward(stacklstm *s, float *dx, float *dW, float *dbias);
+size_t bf16_workspace_bytes(int T, int B, int I, int H, int num_sms);
+const char *bf16_unsupported(int T, int B, int I, int H);
+
+inline unsigned ceil_div(size_t a, size_t b) { return (unsigned)((a + b - 1) / b); }
+
+}  // namespace sl

@@ -1,0 +1,154 @@
+// index_kernels.cu -- integer bookkeeping of the homogenized step and row gathers.
+//
+// The prepass turns the op stream into every index the state kernels use, so the time
+// loop itself never branches on an op (Algorithm 1 has no op-dependent branch):
+//   p_traj[t]   pointer before step t: p_0 = 0, p_{t+1} = p_t + op_t (Sec. 3);
+//   top[t]      history index of the state at slot p_t at time t: 0 is the initial state,
+//               tau + 1 the state step tau wrote. Step t reads history row top[t];
+//   slot_last   history index last written to each slot after the last step (-1: never).
+// Every step writes slot p_t + 1 (Algorithm 1), which in history terms is row t + 1.
+#include <algorithm>
+
+#include "common.cuh"
+
+namespace sl {
+namespace {
+
+constexpr int kPrepassThreads = 32;
+
+// One thread per instance. The per-instance stack of slot tags lives in a column of
+// shared memory (slot-major, so the 32 threads of a warp hit 32 distinct banks) or, for
+// long sequences, in a global [T+1][B] scratch with the same coalesced layout.
+template <bool kOnChip>
+__global__ void __launch_bounds__(kPrepassThreads)
+prepass_kernel(int T, int B, const int8_t *__restrict__ ops, int32_t *__restrict__ p_traj,
+               int32_t *__restrict__ top, int32_t *__restrict__ slot_last,
+               int32_t *__restrict__ gscratch, int32_t *__restrict__ err)
+{
+    extern __shared__ int32_t s_tag[];
+    const int lane = threadIdx.x;
+    const int b = blockIdx.x * kPrepassThreads + lane;
+    if (b >= B) return;
+    auto tag = [&](int slot) -> int32_t & {
+        return kOnChip ? s_tag[slot * kPrepassThreads + lane] : gscratch[(size_t)slot * B + b];
+    };
+    tag(0) = 0;
+    for (int slot = 1; slot <= T; ++slot) tag(slot) = -1;
+    int p = 0, e = SL_OK;
+    for (int t = 0; t < T; ++t) {
+        int op = ops[(size_t)t * B + b];
+        if (op < -1 || op > 1) {  // recorded, then run as a hold so indices stay in range
+            if (e == SL_OK) e = SL_ERR_OP;
+            op = 0;
+        }
+        if (p + op < 0) {
+            if (e == SL_OK) e = SL_ERR_UNDERFLOW;
+            op = 0;
+        }
+        p_traj[(size_t)t * B + b] = p;
+        top[(size_t)t * B + b] = tag(p);
+        tag(p + 1) = t + 1;  // Algorithm 1: every step writes slot p + 1
+        p += op;
+    }
+    p_traj[(size_t)T * B + b] = p;
+    top[(size_t)T * B + b] = tag(p);
+    for (int slot = 0; slot <= T; ++slot) slot_last[(size_t)slot * B + b] = tag(slot);
+    if (e != SL_OK) atomicCAS(err, 0, e);
+}
+
+// out[r] = hist row (idx[r], r % B), or zeros where idx[r] < 0. E is the raw element
+// bit pattern (uint32_t for float, uint16_t for bf16): a pure copy.
+template <typename E>
+__global__ void gather_rows_kernel(const int32_t *__restrict__ idx, int B, size_t rows, int row_elems,
+                                   const E *__restrict__ hist, E *__restrict__ out)
+{
+    const size_t total = rows * (size_t)row_elems;
+    for (size_t e = blockIdx.x * (size_t)blockDim.x + threadIdx.x; e < total;
+         e += (size_t)gridDim.x * blockDim.x) {
+        const size_t r = e / row_elems;
+        const int k = (int)(e - r * row_elems);
+        const int src = idx[r];
+        const int b = (int)(r % B);
+        out[e] = src >= 0 ? hist[((size_t)src * B + b) * row_elems + k] : (E)0;
+    }
+}
+
+// Seed the gradient history with the loss terms before the reverse loop:
+// d_top_h goes to the final top, dy_t to the top after step t (Algorithm 1's output).
+// One thread per (b, j); its additions run in a fixed order (final top, then t = T-1..0).
+__global__ void seed_grads_kernel(int T, int B, int H, const int32_t *__restrict__ top,
+                                  const float *__restrict__ d_top_h, const float *__restrict__ dy,
+                                  float *__restrict__ dhist_h)
+{
+    const size_t n = (size_t)B * H;
+    for (size_t e = blockIdx.x * (size_t)blockDim.x + threadIdx.x; e < n;
+         e += (size_t)gridDim.x * blockDim.x) {
+        const int b = (int)(e / H), j = (int)(e - (size_t)b * H);
+        if (d_top_h) {
+            const int s = top[(size_t)T * B + b];
+            dhist_h[((size_t)s * B + b) * H + j] += d_top_h[e];
+        }
+        if (dy)
+            for (int t = T - 1; t >= 0; --t) {
+                const int s = top[(size_t)(t + 1) * B + b];
+                dhist_h[((size_t)s * B + b) * H + j] += dy[(size_t)t * n + e];
+            }
+    }
+}
+
+}  // namespace
+
+// The slot-tag stack goes on chip when (T + 1) slots x 32 instances fit in shared memory.
+cudaError_t configure_prepass(stacklstm *s)
+{
+    const size_t bytes = (size_t)(s->T + 1) * kPrepassThreads * sizeof(int32_t);
+    int optin = 0;
+    cudaError_t e = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, s->device);
+    if (e) return e;
+    s->prepass_smem = 0;
+    if (bytes + 1024 <= (size_t)optin) {
+        if (bytes > 48 * 1024 &&
+            (e = cudaFuncSetAttribute(prepass_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes)))
+            return e;
+        s->prepass_smem = (int)bytes;
+    }
+    return cudaSuccess;
+}
+
+cudaError_t launch_prepass(stacklstm *s, const int8_t *ops)
+{
+    const unsigned grid = ceil_div(s->B, kPrepassThreads);
+    if (s->prepass_smem > 0)
+        prepass_kernel<true><<<grid, kPrepassThreads, s->prepass_smem, s->stream>>>(
+            s->T, s->B, ops, s->p_traj, s->top, s->slot_last, nullptr, s->err);
+    else
+        prepass_kernel<false><<<grid, kPrepassThreads, 0, s->stream>>>(
+            s->T, s->B, ops, s->p_traj, s->top, s->slot_last, s->slot_scratch, s->err);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_gather_rows(stacklstm *s, const int32_t *idx, int rows, size_t elem_bytes,
+                               const void *hist, void *out, int row_elems)
+{
+    const size_t total = (size_t)rows * row_elems;
+    const unsigned grid = (unsigned)std::min<size_t>(ceil_div(total, 256), (size_t)s->num_sms * 16);
+    if (total == 0) return cudaSuccess;
+    if (elem_bytes == 4)
+        gather_rows_kernel<uint32_t><<<grid, 256, 0, s->stream>>>(
+            idx, s->B, rows, row_elems, (const uint32_t *)hist, (uint32_t *)out);
+    else
+        gather_rows_kernel<uint16_t><<<grid, 256, 0, s->stream>>>(
+            idx, s->B, rows, row_elems, (const uint16_t *)hist, (uint16_t *)out);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_seed_grads(stacklstm *s, const float *d_top_h, const float *dy)
+{
+    if (!d_top_h && !dy) return cudaSuccess;
+    const size_t n = (size_t)s->B * s->H;
+    const unsigned grid = (unsigned)std::min<size_t>(ceil_div(n, 256), (size_t)s->num_sms * 16);
+    seed_grads_kernel<<<grid, 256, 0, s->stream>>>(s->T, s->B, s->H, s->top, d_top_h, dy, s->dhist_h);
+    return cudaGetLastError();
+}
+
+}  // namespace sl

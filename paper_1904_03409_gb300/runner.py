@@ -1,0 +1,70 @@
+"""Move a synthetic workload onto the device, run it through the C ABI, read results back.
+
+Marshalling only (numpy <-> torch device tensors); the computation is the library's.
+"""
+from __future__ import annotations
+
+from typing import Optional
+
+import numpy as np
+
+from . import binding as bd
+
+
+def upload(w, device: int = 0) -> dict:
+    """Device tensors of a workload: inputs in the workload's dtype, c0/bias/seeds fp32."""
+    import torch
+    dev = torch.device("cuda", device)
+    dt = torch.bfloat16 if w.dtype == "bf16" else torch.float32
+    f = lambda a: torch.from_numpy(np.ascontiguousarray(a, dtype=np.float32)).to(dev)
+    return dict(x=f(w.x).to(dt), ops=torch.from_numpy(np.ascontiguousarray(w.ops, np.int8)).to(dev),
+                h0=f(w.h0).to(dt), c0=f(w.c0), W=f(w.W).to(dt), bias=f(w.bias), d_top_h=f(w.d_top_h),
+                dy=None if w.dy is None else f(w.dy))
+
+
+def alloc_outputs(w, device: int = 0, forward_outputs: bool = True) -> dict:
+    import torch
+    dev = torch.device("cuda", device)
+    dt = torch.bfloat16 if w.dtype == "bf16" else torch.float32
+    T, B, I, H = w.T, w.B, w.I, w.H
+    e = lambda *s, d=torch.float32: torch.empty(*s, dtype=d, device=dev)
+    out = dict(p_final=e(B, d=torch.int32), dx=e(T, B, I), dh0=e(B, H), dc0=e(B, H), dW=e(I + H, 4 * H),
+               dbias=e(4 * H))
+    if forward_outputs:
+        out.update(h_stack=e(T + 1, B, H, d=dt), c_stack=e(T + 1, B, H), p_traj=e(T + 1, B, d=torch.int32),
+                   src=e(T + 1, B, d=torch.int32), y=e(T, B, H, d=dt))
+    return out
+
+
+def forward_backward(hd, ins: dict, out: dict, d_top_h=None, dy=None):
+    bd.stacklstm_forward(hd, ins["x"], ins["ops"], ins["h0"], ins["c0"], ins["W"], ins["bias"],
+                         out.get("h_stack"), out.get("c_stack"), out["p_final"], out.get("p_traj"),
+                         out.get("src"), out.get("y"))
+    bd.stacklstm_backward(hd, ins["d_top_h"] if d_top_h is None else d_top_h, ins.get("dy") if dy is None else dy,
+                          out.get("dx"), out.get("dh0"), out.get("dc0"), out.get("dW"), out.get("dbias"))
+
+
+def to_numpy(out: dict) -> dict:
+    import torch
+    res = {}
+    for k, v in out.items():
+        if v is None:
+            continue
+        res[k] = (v.float() if v.dtype == torch.bfloat16 else v).cpu().numpy()
+    return res
+
+
+def run(w, device: int = 0, d_top_h: Optional[np.ndarray] = None) -> dict:
+    """Forward + backward of workload ``w`` on ``cuda:device``; numpy results."""
+    import torch
+    hd = bd.stacklstm_create(w.T, w.B, w.I, w.H, bd.SL_BF16 if w.dtype == "bf16" else bd.SL_FP32, device)
+    try:
+        ins = upload(w, device)
+        out = alloc_outputs(w, device)
+        seed = None if d_top_h is None else torch.from_numpy(np.ascontiguousarray(d_top_h, np.float32)).to(
+            ins["x"].device)
+        forward_backward(hd, ins, out, d_top_h=seed)
+        torch.cuda.synchronize(device)
+        return to_numpy(out)
+    finally:
+        hd.destroy()
