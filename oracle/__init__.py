@@ -25,7 +25,7 @@ _LIB = os.path.join(_LIB_DIR, "libstacklstm_oracle.so")
 
 MODES = {"homogenized": 0, "definition": 1}
 ERRORS = {1: "bad op", 2: "stack underflow", 3: "out of memory", 4: "bad argument"}
-OUTPUTS = ("p_traj", "src", "y", "stack_h", "stack_c", "dx", "dh0", "dc0", "dW", "dbias")
+OUTPUTS = ("p_traj", "src", "y", "h_stack", "c_stack", "dx", "dh0", "dc0", "dW", "dbias")
 
 _lib = None
 
@@ -79,7 +79,7 @@ def run(x, ops, h0, c0, W, bias, d_top_h=None, dy=None, mode: str = "homogenized
     (gate column blocks i, f, g, o), bias [4H], d_top_h [B, H], dy [T, B, H].
     Returns a dict with the requested ``outputs`` (fp64 / int32 numpy arrays):
     p_traj [T+1, B], src [T+1, B] (history index of the top at each time: 0 is the
-    initial state, t+1 the state written at step t), y [T, B, H], stack_h/stack_c
+    initial state, t+1 the state written at step t), y [T, B, H], h_stack/c_stack
     [T+1, B, H] (final slot-indexed stack, never-written slots 0), dx [T, B, I],
     dh0/dc0 [B, H], dW [I+H, 4H], dbias [4H].
     """
@@ -97,8 +97,8 @@ def run(x, ops, h0, c0, W, bias, d_top_h=None, dy=None, mode: str = "homogenized
                 bias=_in(bias, np.float64, (4 * H,)), d_top_h=_in(d_top_h, np.float64, (B, H)),
                 dy=_in(dy, np.float64, (T, B, H)))
     shapes = {"p_traj": ((T + 1, B), np.int32), "src": ((T + 1, B), np.int32),
-              "y": ((T, B, H), np.float64), "stack_h": ((T + 1, B, H), np.float64),
-              "stack_c": ((T + 1, B, H), np.float64), "dx": ((T, B, I), np.float64),
+              "y": ((T, B, H), np.float64), "h_stack": ((T + 1, B, H), np.float64),
+              "c_stack": ((T + 1, B, H), np.float64), "dx": ((T, B, I), np.float64),
               "dh0": ((B, H), np.float64), "dc0": ((B, H), np.float64),
               "dW": ((I + H, 4 * H), np.float64), "dbias": ((4 * H,), np.float64)}
     outputs = tuple(outputs)

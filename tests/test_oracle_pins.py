@@ -142,12 +142,12 @@ def test_golden_arc_standard_trace():
     assert list(r["src"][:, 0]) == [int(v) for v in g["src"]]
     # final slot-indexed stack: slot s holds the state written at step tag-1 (tag 0 = h0)
     tags = [int(v) for v in g["final_tags"]]
-    assert tags[0] == 0 and np.array_equal(r["stack_h"][0, 0], c["h0"][0])
+    assert tags[0] == 0 and np.array_equal(r["h_stack"][0, 0], c["h0"][0])
     for s, tag in enumerate(tags[1:], start=1):
         t = tag - 1
         # a live state written at step t is the top after step t, hence y_t
         if r["p_traj"][t + 1, 0] == s:
-            assert np.array_equal(r["stack_h"][s, 0], r["y"][t, 0])
+            assert np.array_equal(r["h_stack"][s, 0], r["y"][t, 0])
     live = dict(kv.split(":") for kv in g["live_slots"])
     assert sorted(int(k) for k in live) == list(range(r["p_traj"][-1, 0] + 1))
 
@@ -164,7 +164,7 @@ def test_pop_then_push_rewrites_same_state():
     # b=0: p = 0 1 2 1 1 2 ; step 4 reads slot 1 (state of step 0) as step 1 did
     assert list(r["p_traj"][:, 0]) == [0, 1, 2, 1, 1, 2]
     assert np.array_equal(r["y"][4, 0], r["y"][1, 0])
-    assert np.array_equal(r["stack_h"][2, 0], r["y"][1, 0])
+    assert np.array_equal(r["h_stack"][2, 0], r["y"][1, 0])
     # b=1: p = 0 1 1 0 0 1 ; step 4 reads slot 0 (h0) as step 0 did
     assert list(r["p_traj"][:, 1]) == [0, 1, 1, 0, 0, 1]
     assert np.array_equal(r["y"][4, 1], r["y"][0, 1])
@@ -180,8 +180,8 @@ def test_definition_equals_homogenized_live(seed):
         assert np.array_equal(rh[k], rd[k]), k
     for b in range(B):
         live = rh["p_traj"][-1, b] + 1
-        assert np.array_equal(rh["stack_h"][:live, b], rd["stack_h"][:live, b])
-        assert np.array_equal(rh["stack_c"][:live, b], rd["stack_c"][:live, b])
+        assert np.array_equal(rh["h_stack"][:live, b], rd["h_stack"][:live, b])
+        assert np.array_equal(rh["c_stack"][:live, b], rd["c_stack"][:live, b])
 
 
 def test_dead_writes_get_zero_input_gradient():
@@ -283,7 +283,7 @@ def test_trailing_holds_and_unbatched_equivalence():
         assert r["p_traj"][-1, b] == r1["p_traj"][-1, 0]
         assert np.array_equal(r["y"][n - 1:, b], np.repeat(r1["y"][n - 1:n, 0], T - n + 1, 0))
         live = r1["p_traj"][-1, 0] + 1
-        assert np.array_equal(r["stack_h"][:live, b], r1["stack_h"][:live, 0])
+        assert np.array_equal(r["h_stack"][:live, b], r1["h_stack"][:live, 0])
         assert np.array_equal(r["dx"][:n, b], r1["dx"][:, 0])
         assert np.all(r["dx"][n:, b] == 0.0)
         assert np.array_equal(r["dh0"][b], r1["dh0"][0])
@@ -297,7 +297,7 @@ def test_batch_permutation():
     cp = {k: (v[:, perm] if k in ("x", "ops", "dy") else v[perm] if k in ("h0", "c0", "d_top_h") else v)
           for k, v in c.items()}
     rp = oracle.run(**cp)
-    for k in ("p_traj", "src", "y", "dx", "stack_h"):
+    for k in ("p_traj", "src", "y", "dx", "h_stack"):
         assert np.array_equal(rp[k], r[k][:, perm]), k
     for k in ("dh0", "dc0"):
         assert np.array_equal(rp[k], r[k][perm]), k
@@ -334,8 +334,8 @@ def test_closed_form_with_zero_weights():
         depth_max = int(r["p_traj"][:-1, b].max()) + 1  # highest slot any step wrote
         for j in range(1, min(depth_max, T) + 1):
             cj = i * g * (1 - f ** j) / (1 - f)
-            assert np.allclose(r["stack_c"][j, b], cj, rtol=1e-13, atol=1e-15)
-            assert np.allclose(r["stack_h"][j, b], o * np.tanh(cj), rtol=1e-13, atol=1e-15)
+            assert np.allclose(r["c_stack"][j, b], cj, rtol=1e-13, atol=1e-15)
+            assert np.allclose(r["h_stack"][j, b], o * np.tanh(cj), rtol=1e-13, atol=1e-15)
     for t in range(T):
         for b in range(B):
             j = r["p_traj"][t + 1, b]
