@@ -54,6 +54,8 @@ def _load():
         dp, ip, bp = ctypes.c_void_p, ctypes.c_int, ctypes.c_void_p
         lib.oracle_stacklstm.argtypes = [ip, ip, ip, ip, ip] + [dp] * 8 + [bp] * 10 + [ip]
         lib.oracle_stacklstm.restype = ctypes.c_int
+        lib.oracle_pointers.argtypes = [ip, ip, bp, bp, bp]
+        lib.oracle_pointers.restype = ctypes.c_int
         _lib = lib
     return _lib
 
@@ -110,6 +112,22 @@ def run(x, ops, h0, c0, W, bias, d_top_h=None, dy=None, mode: str = "homogenized
     if rc != 0:
         raise OracleError(rc)
     return {k: v for k, v in out.items() if v is not None}
+
+
+def pointers(ops) -> dict:
+    """Pointer trajectory p_traj [T+1, B] and read provenance src [T+1, B] of every
+    instance, without the cell arithmetic (same explicit stack of slot tags)."""
+    ops = np.ascontiguousarray(ops)
+    T, B = ops.shape
+    if not np.all((ops >= -1) & (ops <= 1)):
+        raise OracleError(1)
+    ops8 = ops.astype(np.int8)
+    p = np.zeros((T + 1, B), np.int32)
+    s = np.zeros((T + 1, B), np.int32)
+    rc = _load().oracle_pointers(T, B, _ptr(ops8), _ptr(p), _ptr(s))
+    if rc != 0:
+        raise OracleError(rc)
+    return {"p_traj": p, "src": s}
 
 
 def run_instances(inst, x, ops, h0, c0, W, bias, d_top_h=None, dy=None, **kw) -> dict:

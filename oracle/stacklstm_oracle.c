@@ -272,3 +272,33 @@ int oracle_stacklstm(int T, int B, int I, int H, int mode,
     free(rcs); free(pdW); free(pdb);
     return rc;
 }
+
+/*
+ * Pointer trajectory and read provenance only (no cell arithmetic): the same explicit
+ * stack of slot tags as above, for every instance. Fast enough for full-size batches.
+ * Returns 0, or the first error code by instance order.
+ */
+int oracle_pointers(int T, int B, const int8_t *ops, int32_t *p_traj, int32_t *src)
+{
+    if (T < 0 || B < 0) return ORACLE_BAD_ARG;
+    int32_t *tag = malloc((size_t)(T + 1) * sizeof(int32_t));
+    if (!tag) return ORACLE_NOMEM;
+    int rc = ORACLE_OK;
+    for (int b = 0; b < B && rc == ORACLE_OK; ++b) {
+        int p = 0;
+        tag[0] = 0;
+        for (int t = 0; t < T; ++t) {
+            const int op = ops[(size_t)t * B + b];
+            if (op != 1 && op != 0 && op != -1) { rc = ORACLE_BAD_OP; break; }
+            if (p + op < 0) { rc = ORACLE_UNDERFLOW; break; }
+            p_traj[(size_t)t * B + b] = p;
+            src[(size_t)t * B + b] = tag[p];
+            tag[p + 1] = t + 1; /* Algorithm 1: every step writes slot p + 1 */
+            p += op;
+        }
+        p_traj[(size_t)T * B + b] = p;
+        src[(size_t)T * B + b] = tag[p];
+    }
+    free(tag);
+    return rc;
+}

@@ -43,8 +43,18 @@ struct stacklstm {
     // packed weights (taken at forward)
     void *w_fwd = nullptr;  // fp32: W^T [4H][I+H] float; bf16: forward operand tiles
     void *w_bwd = nullptr;  // bf16: backward operand tiles
+    void *w_dx = nullptr;   // bf16: input-gradient operand tiles
     float *dw_part = nullptr;  // split-K partials of the weight-gradient contraction
     size_t dw_part_elems = 0;
+    void *ones = nullptr;      // bf16: one 16-byte piece {1, 0, ..., 0} (bias-gradient row)
+    const void *x_saved = nullptr;  // the caller's x, read again by the weight gradient
+
+    // bf16 tensor-core plan (bf16_path.cu)
+    int uf = 0, ub = 0;      // hidden units per CTA tile: forward, backward
+    int kcf = 0, kcb = 0;    // 64-wide contraction chunks: forward (I+H), backward (4H)
+    int nx = 0, nxt = 0;     // input gradient: columns per tile, number of column tiles
+    int dw_mt = 0, dw_nt = 0, dw_split = 0;  // weight gradient: row tiles, column tiles, splits
+    long long wait_limit = 0;  // clock cycles one bounded device-side wait may spin
 
     std::string last_error;
     std::vector<void *> allocs;

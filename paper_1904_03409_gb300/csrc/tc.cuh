@@ -43,17 +43,31 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t *bar, uint32_t parity)
     return ok != 0;
 }
 
-// Waits for the phase of the given parity to complete, for at most `limit` clock cycles.
+__device__ __forceinline__ bool mbar_test_wait(uint64_t *bar, uint32_t parity)
+{
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(smem_u32(bar)), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
+// Waits for the phase of the given parity to complete, for at most `limit` clock cycles
+// (checked before every potentially suspending try_wait, so a zero budget never blocks).
 // Returns false on timeout, or early once *abort is set by another thread of the CTA.
 __device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, long long limit,
                                           volatile int *abort)
 {
-    if (mbar_try_wait(bar, parity)) return true;
+    if (mbar_test_wait(bar, parity)) return true;
     const long long t0 = clock64();
     while (true) {
-        if (mbar_try_wait(bar, parity)) return true;
+        if (clock64() - t0 >= limit) return false;
         if (abort && *abort) return false;
-        if (clock64() - t0 > limit) return false;
+        if (mbar_try_wait(bar, parity)) return true;
     }
 }
 

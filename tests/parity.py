@@ -4,6 +4,9 @@ Integer results (pointer trajectories, read provenance, final pointers) must mat
 bit for bit. Floats: fp32 path max-abs error <= 1e-4; bf16 path max-abs error <=
 3e-2 times the tensor's largest oracle magnitude.
 """
+import json
+import os
+
 import numpy as np
 
 FP32_TOL = 1e-4
@@ -41,4 +44,12 @@ def compare(got, ref, dtype, keys=None, inst=None):
             tol = tol_for(dtype, ref[k])
             assert np.isfinite(err) and err <= tol, "%s: max abs err %.3g > tol %.3g" % (k, err, tol)
             report[k] = (err, tol)
+    log = os.environ.get("PARITY_LOG")
+    if log:
+        import inspect
+        who = os.environ.get("PYTEST_CURRENT_TEST", inspect.stack()[1].function).split(" ")[0]
+        with open(log, "a") as f:
+            f.write(json.dumps({"test": who, "dtype": dtype,
+                                "max_abs_err": {k: v[0] for k, v in report.items() if k not in INT_KEYS},
+                                "tol": {k: v[1] for k, v in report.items() if k not in INT_KEYS}}) + "\n")
     return report

@@ -353,3 +353,13 @@ def test_errors():
     with pytest.raises(oracle.OracleError) as e:
         oracle.run(**c)
     assert e.value.code == 1
+
+
+def test_pointer_only_entry_matches_full_oracle():
+    c = rand_case(60, 9, 3, 2, 12, probs=(0.4, 0.4, 0.2))
+    r = oracle.run(**c, outputs=("p_traj", "src"))
+    q = oracle.pointers(c["ops"])
+    assert np.array_equal(r["p_traj"], q["p_traj"]) and np.array_equal(r["src"], q["src"])
+    for b in range(9):
+        ps, tops = replay(c["ops"][:, b])
+        assert list(q["p_traj"][:, b]) == ps and list(q["src"][:, b]) == tops
