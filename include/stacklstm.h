@@ -102,8 +102,9 @@ sl_status stacklstm_set_async(stacklstm_t s, int async);
  *   src     [T+1, B]    provenance of the top at each time: 0 is the initial state,
  *                       t + 1 is the state written at step t; src[t] is what step t read
  *   y       [T, B, H]   step outputs: h at the top after step t's pointer move (dtype)
- * The handle keeps what backward needs (a packed copy of W, the states read, the gates),
- * so x and W may change after forward returns.
+ * The handle keeps what backward needs (packed copies of W, the state history, the
+ * gates), so W may change after forward returns; x must stay valid and unchanged until
+ * the matching backward returns (the weight gradient reads it again).
  */
 sl_status stacklstm_forward(stacklstm_t s, const void *x, const int8_t *ops, const void *h0,
                             const float *c0, const void *W, const float *bias, void *h_stack,
@@ -121,6 +122,35 @@ sl_status stacklstm_forward(stacklstm_t s, const void *x, const int8_t *ops, con
  */
 sl_status stacklstm_backward(stacklstm_t s, const float *d_top_h, const float *dy, float *dx,
                              float *dh0, float *dc0, float *dW, float *dbias);
+
+/*
+ * Phases of a forward + backward, as stacklstm_get_timing reports them. Each phase is a
+ * contiguous run of kernel launches on the handle's stream.
+ */
+typedef enum {
+    SL_PHASE_PREPASS = 0,  /* op validation and the index prepass                      */
+    SL_PHASE_FORWARD = 1,  /* weight packing and the T forward step launches           */
+    SL_PHASE_OUTPUTS = 2,  /* optional forward outputs (y, h_stack, c_stack, p_traj)   */
+    SL_PHASE_BACKWARD = 3, /* gradient seeding and the T backward step launches        */
+    SL_PHASE_DX = 4,       /* the input-gradient contraction dx = dG W_x^T             */
+    SL_PHASE_DW = 5,       /* the weight- and bias-gradient contraction and reduction  */
+    SL_NUM_PHASES = 6
+} sl_phase;
+
+/*
+ * stacklstm_set_timing -- on != 0: record a CUDA event pair on the handle's stream around
+ * every phase of later calls. Resets the accumulated times and launch counts either way.
+ */
+sl_status stacklstm_set_timing(stacklstm_t s, int on);
+
+/*
+ * stacklstm_get_timing -- synchronize the handle's stream and write, for the first n
+ * phases (n <= SL_NUM_PHASES), the device time in milliseconds accumulated since the last
+ * stacklstm_set_timing (ms, nullable; zeros for phases run while timing was off) and the
+ * number of this library's kernel launches (launches, nullable; always counted).
+ * Host pointers.
+ */
+sl_status stacklstm_get_timing(stacklstm_t s, double *ms, long long *launches, int n);
 
 /* Synchronize the handle's stream and return (then clear) any device-detected error. */
 sl_status stacklstm_status(stacklstm_t s);

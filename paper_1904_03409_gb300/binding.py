@@ -55,10 +55,13 @@ def load(path: Optional[str] = None):
     lib.stacklstm_destroy.argtypes = [vp]
     lib.stacklstm_status_string.argtypes = [i]
     lib.stacklstm_status_string.restype = ctypes.c_char_p
+    lib.stacklstm_set_timing.argtypes = [vp, i]
+    lib.stacklstm_get_timing.argtypes = [vp, vp, vp, i]
     lib.stacklstm_last_error.argtypes = [vp]
     lib.stacklstm_last_error.restype = ctypes.c_char_p
     for fn in ("stacklstm_create", "stacklstm_forward", "stacklstm_backward", "stacklstm_set_stream",
-               "stacklstm_set_async", "stacklstm_status", "stacklstm_destroy"):
+               "stacklstm_set_async", "stacklstm_status", "stacklstm_destroy", "stacklstm_set_timing",
+               "stacklstm_get_timing"):
         getattr(lib, fn).restype = ctypes.c_int
     _lib = lib
     return lib
@@ -164,6 +167,23 @@ def stacklstm_backward(hd: StackLSTMHandle, d_top_h=None, dy=None, dx=None, dh0=
             _ptr(dx, d, f, (T, B, I), "dx"), _ptr(dh0, d, f, (B, H), "dh0"), _ptr(dc0, d, f, (B, H), "dc0"),
             _ptr(dW, d, f, (I + H, 4 * H), "dW"), _ptr(dbias, d, f, (4 * H,), "dbias")]
     _check(hd.h, load().stacklstm_backward(hd.h, *args), "stacklstm_backward")
+
+
+PHASES = ("prepass", "forward", "outputs", "backward", "dx", "dw")
+
+
+def stacklstm_set_timing(hd: StackLSTMHandle, on: bool):
+    """Record CUDA events around each phase of later calls; resets the totals."""
+    _check(hd.h, load().stacklstm_set_timing(hd.h, int(bool(on))), "stacklstm_set_timing")
+
+
+def stacklstm_get_timing(hd: StackLSTMHandle) -> dict:
+    """{phase: (milliseconds, kernel launches)} accumulated since the last set_timing."""
+    n = len(PHASES)
+    ms = (ctypes.c_double * n)()
+    ln = (ctypes.c_longlong * n)()
+    _check(hd.h, load().stacklstm_get_timing(hd.h, ms, ln, n), "stacklstm_get_timing")
+    return {p: (ms[i], ln[i]) for i, p in enumerate(PHASES)}
 
 
 def stacklstm_destroy(hd: StackLSTMHandle):

@@ -64,6 +64,62 @@ bool alloc(stacklstm *s, P **out, size_t bytes)
     return true;
 }
 
+// Records a CUDA event pair around one phase on the handle's stream when timing is on;
+// always adds the phase's kernel launches to its count.
+struct Phase {
+    stacklstm *s;
+    int ph;
+    long long l0;
+    cudaEvent_t a = nullptr;
+    Phase(stacklstm *s_, int ph_) : s(s_), ph(ph_), l0(s_->launches)
+    {
+        if (s->timing) {
+            a = take_event(s);
+            if (a) cudaEventRecord(a, s->stream);
+        }
+    }
+    ~Phase()
+    {
+        s->phase_launches[ph] += s->launches - l0;
+        if (a) {
+            cudaEvent_t b = take_event(s);
+            if (b) {
+                cudaEventRecord(b, s->stream);
+                s->pending.push_back({ph, a, b});
+            } else {
+                s->event_pool.push_back(a);
+            }
+        }
+    }
+    static cudaEvent_t take_event(stacklstm *s)
+    {
+        if (!s->event_pool.empty()) {
+            cudaEvent_t e = s->event_pool.back();
+            s->event_pool.pop_back();
+            return e;
+        }
+        cudaEvent_t e = nullptr;
+        if (cudaEventCreate(&e) != cudaSuccess) {
+            cudaGetLastError();
+            return nullptr;
+        }
+        return e;
+    }
+};
+
+// Folds completed event pairs into the per-phase totals (the stream must be idle).
+void collect_timing(stacklstm *s)
+{
+    for (auto &p : s->pending) {
+        float ms = 0.0f;
+        if (cudaEventElapsedTime(&ms, p.a, p.b) == cudaSuccess) s->phase_ms[p.phase] += ms;
+        s->event_pool.push_back(p.a);
+        s->event_pool.push_back(p.b);
+    }
+    s->pending.clear();
+    cudaGetLastError();
+}
+
 // Reads back the device error flag (synchronizing the stream) and clears it.
 sl_status read_status(stacklstm *s)
 {
@@ -186,27 +242,37 @@ sl_status stacklstm_forward(stacklstm_t s, const void *x, const int8_t *ops, con
     const size_t es = elem_size(s->dt);
     cudaError_t e;
     s->fwd_done = 0;
-    if ((e = sl::launch_prepass(s, ops))) return cuda_fail(s, e, "prepass");
-    if (s->dt == SL_FP32)
-        e = sl::fp32_forward(s, (const float *)x, (const float *)h0, c0, (const float *)W, bias);
-    else
-        e = sl::bf16_forward(s, (const __nv_bfloat16 *)x, (const __nv_bfloat16 *)h0, c0,
-                             (const __nv_bfloat16 *)W, bias);
-    if (e) return cuda_fail(s, e, "forward");
-    if ((e = cudaMemcpyAsync(p_final, s->p_traj + (size_t)T * B, sizeof(int32_t) * B, cudaMemcpyDeviceToDevice,
-                             s->stream)))
-        return cuda_fail(s, e, "p_final");
-    if (p_traj && (e = cudaMemcpyAsync(p_traj, s->p_traj, sizeof(int32_t) * (T + 1) * B, cudaMemcpyDeviceToDevice,
-                                       s->stream)))
-        return cuda_fail(s, e, "p_traj");
-    if (src && (e = cudaMemcpyAsync(src, s->top, sizeof(int32_t) * (T + 1) * B, cudaMemcpyDeviceToDevice,
-                                    s->stream)))
-        return cuda_fail(s, e, "src");
-    if (y && (e = sl::launch_gather_rows(s, s->top + B, T * B, es, s->hist_h, y, H))) return cuda_fail(s, e, "y");
-    if (h_stack && (e = sl::launch_gather_rows(s, s->slot_last, (T + 1) * B, es, s->hist_h, h_stack, H)))
-        return cuda_fail(s, e, "h_stack");
-    if (c_stack && (e = sl::launch_gather_rows(s, s->slot_last, (T + 1) * B, 4, s->hist_c, c_stack, H)))
-        return cuda_fail(s, e, "c_stack");
+    {
+        Phase ph(s, SL_PHASE_PREPASS);
+        if ((e = sl::launch_prepass(s, ops))) return cuda_fail(s, e, "prepass");
+    }
+    {
+        Phase ph(s, SL_PHASE_FORWARD);
+        if (s->dt == SL_FP32)
+            e = sl::fp32_forward(s, (const float *)x, (const float *)h0, c0, (const float *)W, bias);
+        else
+            e = sl::bf16_forward(s, (const __nv_bfloat16 *)x, (const __nv_bfloat16 *)h0, c0,
+                                 (const __nv_bfloat16 *)W, bias);
+        if (e) return cuda_fail(s, e, "forward");
+    }
+    {
+        Phase ph(s, SL_PHASE_OUTPUTS);
+        if ((e = cudaMemcpyAsync(p_final, s->p_traj + (size_t)T * B, sizeof(int32_t) * B,
+                                 cudaMemcpyDeviceToDevice, s->stream)))
+            return cuda_fail(s, e, "p_final");
+        if (p_traj && (e = cudaMemcpyAsync(p_traj, s->p_traj, sizeof(int32_t) * (T + 1) * B,
+                                           cudaMemcpyDeviceToDevice, s->stream)))
+            return cuda_fail(s, e, "p_traj");
+        if (src && (e = cudaMemcpyAsync(src, s->top, sizeof(int32_t) * (T + 1) * B, cudaMemcpyDeviceToDevice,
+                                        s->stream)))
+            return cuda_fail(s, e, "src");
+        if (y && (e = sl::launch_gather_rows(s, s->top + B, T * B, es, s->hist_h, y, H)))
+            return cuda_fail(s, e, "y");
+        if (h_stack && (e = sl::launch_gather_rows(s, s->slot_last, (T + 1) * B, es, s->hist_h, h_stack, H)))
+            return cuda_fail(s, e, "h_stack");
+        if (c_stack && (e = sl::launch_gather_rows(s, s->slot_last, (T + 1) * B, 4, s->hist_c, c_stack, H)))
+            return cuda_fail(s, e, "c_stack");
+    }
     s->fwd_done = 1;
     return s->async ? SL_OK : read_status(s);
 }
@@ -224,20 +290,59 @@ sl_status stacklstm_backward(stacklstm_t s, const float *d_top_h, const float *d
     const int T = s->T, B = s->B, H = s->H;
     const size_t hist_bytes = sizeof(float) * (size_t)(T + 1) * B * H;
     cudaError_t e;
-    if ((e = cudaMemsetAsync(s->dhist_h, 0, hist_bytes, s->stream))) return cuda_fail(s, e, "clear");
-    if ((e = cudaMemsetAsync(s->dhist_c, 0, hist_bytes, s->stream))) return cuda_fail(s, e, "clear");
-    if ((e = sl::launch_seed_grads(s, d_top_h, dy))) return cuda_fail(s, e, "seed");
-    if (s->dt == SL_FP32)
-        e = sl::fp32_backward(s, dx, dW, dbias);
-    else
-        e = sl::bf16_backward(s, dx, dW, dbias);
-    if (e) return cuda_fail(s, e, "backward");
+    {
+        Phase ph(s, SL_PHASE_BACKWARD);
+        if ((e = cudaMemsetAsync(s->dhist_h, 0, hist_bytes, s->stream))) return cuda_fail(s, e, "clear");
+        if ((e = cudaMemsetAsync(s->dhist_c, 0, hist_bytes, s->stream))) return cuda_fail(s, e, "clear");
+        if ((e = sl::launch_seed_grads(s, d_top_h, dy))) return cuda_fail(s, e, "seed");
+        e = s->dt == SL_FP32 ? sl::fp32_backward_steps(s) : sl::bf16_backward_steps(s);
+        if (e) return cuda_fail(s, e, "backward");
+    }
+    {
+        Phase ph(s, SL_PHASE_DX);
+        e = s->dt == SL_FP32 ? sl::fp32_dx(s, dx) : sl::bf16_dx(s, dx);
+        if (e) return cuda_fail(s, e, "dx");
+    }
+    {
+        Phase ph(s, SL_PHASE_DW);
+        e = s->dt == SL_FP32 ? sl::fp32_dw(s, dW, dbias) : sl::bf16_dw(s, dW, dbias);
+        if (e) return cuda_fail(s, e, "dW");
+    }
     // slot 0 always holds the initial state, which is history row 0
     if (dh0 && (e = cudaMemcpyAsync(dh0, s->dhist_h, sizeof(float) * B * H, cudaMemcpyDeviceToDevice, s->stream)))
         return cuda_fail(s, e, "dh0");
     if (dc0 && (e = cudaMemcpyAsync(dc0, s->dhist_c, sizeof(float) * B * H, cudaMemcpyDeviceToDevice, s->stream)))
         return cuda_fail(s, e, "dc0");
     return s->async ? SL_OK : read_status(s);
+}
+
+sl_status stacklstm_set_timing(stacklstm_t s, int on)
+{
+    if (!s) return SL_ERR_ARG;
+    DeviceGuard g(s->device);
+    cudaError_t e = cudaStreamSynchronize(s->stream);
+    if (e != cudaSuccess) return cuda_fail(s, e, "synchronize");
+    collect_timing(s);
+    s->timing = on != 0;
+    for (int i = 0; i < SL_NUM_PHASES; ++i) {
+        s->phase_ms[i] = 0.0;
+        s->phase_launches[i] = 0;
+    }
+    return SL_OK;
+}
+
+sl_status stacklstm_get_timing(stacklstm_t s, double *ms, long long *launches, int n)
+{
+    if (!s || n < 0 || n > SL_NUM_PHASES) return SL_ERR_ARG;
+    DeviceGuard g(s->device);
+    cudaError_t e = cudaStreamSynchronize(s->stream);
+    if (e != cudaSuccess) return cuda_fail(s, e, "synchronize");
+    collect_timing(s);
+    for (int i = 0; i < n; ++i) {
+        if (ms) ms[i] = s->phase_ms[i];
+        if (launches) launches[i] = s->phase_launches[i];
+    }
+    return SL_OK;
 }
 
 sl_status stacklstm_status(stacklstm_t s)
@@ -253,6 +358,9 @@ sl_status stacklstm_destroy(stacklstm_t s)
     {
         DeviceGuard g(s->device);
         cudaStreamSynchronize(s->stream);
+        collect_timing(s);
+        for (cudaEvent_t ev : s->event_pool) cudaEventDestroy(ev);
+        s->event_pool.clear();
         free_all(s);
         cudaGetLastError();
     }

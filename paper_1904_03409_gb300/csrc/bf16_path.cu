@@ -777,6 +777,7 @@ cudaError_t bf16_forward(stacklstm *s, const __nv_bfloat16 *x, const __nv_bfloat
         W, H, I, H, s->ub, s->kcb, nctb, (__nv_bfloat16 *)s->w_bwd);
     pack_rows<<<grid_for(s, (size_t)s->nxt * s->kcb * s->nx * kChunk), 256, 0, s->stream>>>(
         W, H, 0, I, s->nx, s->kcb, s->nxt, (__nv_bfloat16 *)s->w_dx);
+    s->launches += 3;
     if ((e = cudaGetLastError())) return e;
     const StepArgs a = step_args(s, x, bias, s->w_fwd, s->kcf);
     const dim3 grid(nctf, ceil_div(B, kRows));
@@ -789,16 +790,18 @@ cudaError_t bf16_forward(stacklstm *s, const __nv_bfloat16 *x, const __nv_bfloat
         else
             e = launch(fwd_step_tc<8, kSf8>, grid, Layout<kSf8, 32>::kBytes, s->stream, pdl, a, t);
         if (e) return e;
+        s->launches += 1;
     }
     return cudaGetLastError();
 }
 
-cudaError_t bf16_backward(stacklstm *s, float *dx, float *dW, float *dbias)
+cudaError_t bf16_backward_steps(stacklstm *s)
 {
-    const int T = s->T, B = s->B, I = s->I, H = s->H;
+    const int T = s->T, B = s->B, H = s->H;
     cudaError_t e;
     const StepArgs a = step_args(s, (const __nv_bfloat16 *)s->x_saved, nullptr, s->w_bwd, s->kcb);
     pointwise_last<<<grid_for(s, (size_t)B * (H / 8)), 256, 0, s->stream>>>(a);
+    s->launches += 1;
     if ((e = cudaGetLastError())) return e;
     const dim3 grid(ceil_div(H, s->ub), ceil_div(B, kRows));
     for (int t = T - 1; t >= 0; --t) {
@@ -808,8 +811,16 @@ cudaError_t bf16_backward(stacklstm *s, float *dx, float *dW, float *dbias)
         else
             e = launch(bwd_step_tc<16, kSb>, grid, Layout<kSb, 16>::kBytes, s->stream, pdl, a, t);
         if (e) return e;
+        s->launches += 1;
     }
+    return cudaGetLastError();
+}
+
+cudaError_t bf16_dx(stacklstm *s, float *dx)
+{
+    const int T = s->T, B = s->B, I = s->I, H = s->H;
     const size_t R = (size_t)T * B;
+    cudaError_t e;
     if (dx) {
         DxArgs d;
         d.dG = (const __nv_bfloat16 *)s->dG; d.R = R; d.I = I; d.H = H; d.kc = s->kcb;
@@ -822,7 +833,16 @@ cudaError_t bf16_backward(stacklstm *s, float *dx, float *dW, float *dbias)
         default: e = launch(dx_tc<256, kSx>, g, Layout<kSx, 256>::kBytes, s->stream, false, d); break;
         }
         if (e) return e;
+        s->launches += 1;
     }
+    return cudaGetLastError();
+}
+
+cudaError_t bf16_dw(stacklstm *s, float *dW, float *dbias)
+{
+    const int T = s->T, B = s->B, I = s->I, H = s->H;
+    const size_t R = (size_t)T * B;
+    cudaError_t e;
     if (dW || dbias) {
         DwArgs w;
         w.T = T; w.B = B; w.I = I; w.H = H;
@@ -836,6 +856,7 @@ cudaError_t bf16_backward(stacklstm *s, float *dx, float *dW, float *dbias)
             return e;
         dw_reduce<<<grid_for(s, (size_t)(I + H + 1) * 4 * H), 256, 0, s->stream>>>(
             I + H, 4 * H, s->dw_split, s->dw_part, w.rows_part, w.ld_part, dW, dbias);
+        s->launches += 2;
     }
     return cudaGetLastError();
 }

@@ -56,6 +56,19 @@ struct stacklstm {
     int dw_mt = 0, dw_nt = 0, dw_split = 0;  // weight gradient: row tiles, column tiles, splits
     long long wait_limit = 0;  // clock cycles one bounded device-side wait may spin
 
+    // launch accounting and optional per-phase event timing (api.cu)
+    long long launches = 0;  // kernel launches of this library, running total
+    int timing = 0;
+    int cur_phase = -1;
+    double phase_ms[SL_NUM_PHASES] = {};
+    long long phase_launches[SL_NUM_PHASES] = {};
+    struct EventPair {
+        int phase;
+        cudaEvent_t a, b;
+    };
+    std::vector<EventPair> pending;
+    std::vector<cudaEvent_t> event_pool;
+
     std::string last_error;
     std::vector<void *> allocs;
 };
@@ -71,13 +84,17 @@ cudaError_t launch_seed_grads(stacklstm *s, const float *d_top_h, const float *d
 // ---- fp32 CUDA-core path (fp32_path.cu)
 cudaError_t fp32_forward(stacklstm *s, const float *x, const float *h0, const float *c0,
                          const float *W, const float *bias);
-cudaError_t fp32_backward(stacklstm *s, float *dx, float *dW, float *dbias);
+cudaError_t fp32_backward_steps(stacklstm *s);
+cudaError_t fp32_dx(stacklstm *s, float *dx);
+cudaError_t fp32_dw(stacklstm *s, float *dW, float *dbias);
 
 // ---- bf16 tensor-core path (bf16_path.cu)
 cudaError_t bf16_prepare(stacklstm *s);
 cudaError_t bf16_forward(stacklstm *s, const __nv_bfloat16 *x, const __nv_bfloat16 *h0,
                          const float *c0, const __nv_bfloat16 *W, const float *bias);
-cudaError_t bf16_backward(stacklstm *s, float *dx, float *dW, float *dbias);
+cudaError_t bf16_backward_steps(stacklstm *s);
+cudaError_t bf16_dx(stacklstm *s, float *dx);
+cudaError_t bf16_dw(stacklstm *s, float *dW, float *dbias);
 size_t bf16_workspace_bytes(int T, int B, int I, int H, int num_sms);
 const char *bf16_unsupported(int T, int B, int I, int H);
 

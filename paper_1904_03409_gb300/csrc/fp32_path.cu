@@ -131,20 +131,26 @@ __global__ void dx_f32(int I, int H, const float *__restrict__ WT, const float *
     dx[r * I + k] = acc;
 }
 
-// dW[k][n] = sum_r a_rm[r][k] dG[r][n] and dbias[n] = sum_r dG[r][n], r ascending.
+// dW[k][n] = sum_r a_rm[r][k] dG[r][n] and dbias[n] = sum_r dG[r][n], r ascending, with
+// compensated (Kahan) summation so long fp32 sums keep their accuracy.
 __global__ void dw_f32(size_t R, int K, int G, const float *__restrict__ a_rm, const float *__restrict__ dG,
                        float *__restrict__ dW, float *__restrict__ dbias)
 {
     const size_t n_out = (size_t)(K + 1) * G;
     for (size_t e = blockIdx.x * (size_t)blockDim.x + threadIdx.x; e < n_out; e += (size_t)gridDim.x * blockDim.x) {
         const int k = (int)(e / G), n = (int)(e - (size_t)k * G);
-        float acc = 0.0f;
+        float acc = 0.0f, comp = 0.0f;
+        for (size_t r = 0; r < R; ++r) {
+            const float term = (k < K ? a_rm[r * K + k] : 1.0f) * dG[r * G + n];
+            const float y = term - comp;
+            const float t = acc + y;
+            comp = (t - acc) - y;
+            acc = t;
+        }
         if (k < K) {
-            for (size_t r = 0; r < R; ++r) acc = fmaf(a_rm[r * K + k], dG[r * G + n], acc);
             if (dW) dW[(size_t)k * G + n] = acc;
-        } else {
-            for (size_t r = 0; r < R; ++r) acc += dG[r * G + n];
-            if (dbias) dbias[n] = acc;
+        } else if (dbias) {
+            dbias[n] = acc;
         }
     }
 }
@@ -174,12 +180,13 @@ cudaError_t fp32_forward(stacklstm *s, const float *x, const float *h0, const fl
     for (int t = 0; t < T; ++t)
         fwd_step_f32<<<grid, threads, smem, s->stream>>>(t, B, I, H, x, W, bias, s->top, hh, s->hist_c,
                                                           (float *)s->gates, (float *)s->a_rm);
+    s->launches += 1 + T;
     return cudaGetLastError();
 }
 
-cudaError_t fp32_backward(stacklstm *s, float *dx, float *dW, float *dbias)
+cudaError_t fp32_backward_steps(stacklstm *s)
 {
-    const int T = s->T, B = s->B, I = s->I, H = s->H, K = I + H, G = 4 * H;
+    const int T = s->T, B = s->B, I = s->I, H = s->H, G = 4 * H;
     const float *WT = (const float *)s->w_fwd;
     float *dG = (float *)s->dG;
     const int threads = std::min(128, ((H + 31) / 32) * 32);
@@ -190,6 +197,15 @@ cudaError_t fp32_backward(stacklstm *s, float *dx, float *dW, float *dbias)
         bwd_contract_f32<<<dim3(ceil_div(H, threads), B), threads, sizeof(float) * G, s->stream>>>(
             t, B, I, H, s->top, WT, dG, s->dhist_h);
     }
+    s->launches += 2 * T;
+    return cudaGetLastError();
+}
+
+cudaError_t fp32_dx(stacklstm *s, float *dx)
+{
+    const int T = s->T, B = s->B, I = s->I, H = s->H, G = 4 * H;
+    const float *WT = (const float *)s->w_fwd;
+    const float *dG = (const float *)s->dG;
     if (dx && T > 0) {
         const int tx = std::min(128, ((I + 31) / 32) * 32);
         // grid.y is limited to 65535 rows per launch
@@ -197,11 +213,20 @@ cudaError_t fp32_backward(stacklstm *s, float *dx, float *dW, float *dbias)
             const unsigned rows = (unsigned)std::min<size_t>(65535, (size_t)T * B - r0);
             dx_f32<<<dim3(ceil_div(I, tx), rows), tx, sizeof(float) * G, s->stream>>>(I, H, WT, dG + r0 * G,
                                                                                       dx + r0 * I);
+            s->launches += 1;
         }
     }
+    return cudaGetLastError();
+}
+
+cudaError_t fp32_dw(stacklstm *s, float *dW, float *dbias)
+{
+    const int T = s->T, B = s->B, I = s->I, H = s->H, K = I + H, G = 4 * H;
+    const float *dG = (const float *)s->dG;
     if (dW || dbias)
         dw_f32<<<grid_for(s, (size_t)(K + 1) * G, 128), 128, 0, s->stream>>>(
             (size_t)T * B, K, G, (const float *)s->a_rm, dG, dW, dbias);
+    if (dW || dbias) s->launches += 1;
     return cudaGetLastError();
 }
 

@@ -124,6 +124,7 @@ cudaError_t launch_prepass(stacklstm *s, const int8_t *ops)
     else
         prepass_kernel<false><<<grid, kPrepassThreads, 0, s->stream>>>(
             s->T, s->B, ops, s->p_traj, s->top, s->slot_last, s->slot_scratch, s->err);
+    s->launches += 1;
     return cudaGetLastError();
 }
 
@@ -139,6 +140,7 @@ cudaError_t launch_gather_rows(stacklstm *s, const int32_t *idx, int rows, size_
     else
         gather_rows_kernel<uint16_t><<<grid, 256, 0, s->stream>>>(
             idx, s->B, rows, row_elems, (const uint16_t *)hist, (uint16_t *)out);
+    s->launches += 1;
     return cudaGetLastError();
 }
 
@@ -148,6 +150,7 @@ cudaError_t launch_seed_grads(stacklstm *s, const float *d_top_h, const float *d
     const size_t n = (size_t)s->B * s->H;
     const unsigned grid = (unsigned)std::min<size_t>(ceil_div(n, 256), (size_t)s->num_sms * 16);
     seed_grads_kernel<<<grid, 256, 0, s->stream>>>(s->T, s->B, s->H, s->top, d_top_h, dy, s->dhist_h);
+    s->launches += 1;
     return cudaGetLastError();
 }
 
