@@ -3,27 +3,29 @@
 // Forward, one launch per step t (Algorithm 1, no op-dependent branch). A CTA owns 128
 // batch rows and U hidden units with all four of their gates (N = 4U gate columns), so
 // the LSTM cell runs in the epilogue straight out of tensor memory:
-//   1. gather the contraction operand [x_t ; h_read] (h_read = history row top[t], the
-//      state at the stack top) into a 128-byte-swizzled shared-memory ring with 16-byte
-//      cp.async copies; the packed weight tile streams through the same ring by bulk copy;
+//   1. the contraction operand [x_t ; h_read] streams through a ring of 128-byte-swizzled
+//      shared-memory stages: x_t tiles by TMA (rows t*B + b are contiguous), h_read rows
+//      (history row top[t][b], the state at each stack top) by 16-byte cp.async, one
+//      thread per row; the packed weight tile arrives by bulk copy into the same stage;
 //   2. tcgen05.mma (bf16 in, fp32 accumulate) into tensor memory, issued by one thread;
-//   3. epilogue: tcgen05.ld of the 4U pre-activations of each row, bias, sigmoid/tanh,
-//      c' = f c_read + i g, h' = o tanh(c'); write history row t + 1 (stack slot p_t + 1),
-//      and save the activated gates (fp16) for the backward.
-// The x_t part of the contraction does not depend on the previous step: with
-// programmatic dependent launch it is loaded and multiplied before the step waits for
-// its predecessor.
+//   3. epilogue: tcgen05.ld of each row's 4U pre-activations, bias, sigmoid/tanh,
+//      c' = f c_read + i g, h' = o tanh(c'); write history row t + 1 (stack slot p_t + 1)
+//      and the activated gates (fp16) for the backward.
+// The x_t chunks do not depend on the previous step: with programmatic dependent launch
+// they are loaded and multiplied before the step waits for its predecessor.
 //
 // Backward, one launch per step in reverse time (Sec. 5). A CTA owns 128 rows and U
-// hidden units of dh_read = dG_t W_h^T (contraction over the 4H gate columns). Its
-// epilogue adds dh_read to the gradient of the state step t read (history row top[t]),
-// then runs the pointwise backward of step t - 1 for the same rows and units, which now
-// has its complete (dh', dc'): it writes dG_{t-1} (bf16) and adds dc_read. Every
-// (row, unit) of the gradient history has one owner, so there are no atomics.
+// hidden units of dh_read = dG_t W_h^T (contraction over the 4H gate columns, dG_t tiles
+// by TMA). Its epilogue adds dh_read to the gradient of the state step t read (history
+// row top[t]), then runs the pointwise backward of step t - 1 for the same rows and
+// units, which now has its complete (dh', dc'): it writes dG_{t-1} (bf16) and adds
+// dc_read. Every (row, unit) of the gradient history has one owner: no atomics.
 //
 // After the loop: dx = dG W_x^T (one K-major contraction over all T*B rows) and
 // dW = [x ; h_read]^T dG with dbias as one extra all-ones operand row (an MN-major,
 // split-K contraction whose partial sums are reduced in a fixed order).
+#include <cuda.h>
+#include <cudaTypedefs.h>
 #include <stdlib.h>
 
 #include <algorithm>
@@ -41,35 +43,36 @@ constexpr int kThreads = 128;  // four warps: one per 32-lane quadrant of tensor
 constexpr int kRows = 128;     // MMA M: batch rows (or weight rows) per CTA tile
 constexpr int kChunk = 64;     // contraction elements per chunk: one 128-byte swizzled row
 constexpr uint32_t kAStage = kRows * 128;
+constexpr int kMaxStages = 16;
 constexpr long long kDrainLimit = 4000000000LL;  // wait for own copies / MMAs before exit
 
 // --------------------------------------------------------------------------- smem
+// Dynamic shared memory: [S A stages][S B stages][full[16] empty[16] done][tmem][abort],
+// based at the first 1024-byte boundary (128-byte swizzle atoms are 1024 bytes).
 struct Ctl {
-    uint32_t a0, b0;  // shared addresses of stage 0 of the A and B rings
+    uint32_t a0, b0, b_bytes;  // shared addresses of stage 0 of each ring; B stage size
     uint64_t *full, *empty, *done;
     uint32_t *tmem_slot;
     volatile int *abort;
 };
 
-template <int S, int NB>
-struct Layout {
-    static constexpr uint32_t kB = (uint32_t)NB * 128;
-    static constexpr uint32_t kBars = S * (kAStage + kB);
-    static constexpr uint32_t kBytes = kBars + (2 * S + 1) * 8 + 16 + 1024;  // + alignment slack
-};
+__host__ __device__ constexpr uint32_t smem_bytes(int S, int NB)
+{
+    return 1024 + (uint32_t)S * (kAStage + (uint32_t)NB * 128) + (2 * kMaxStages + 1) * 8 + 16;
+}
 
-template <int S, int NB>
-__device__ __forceinline__ Ctl carve(uint8_t *raw)
+__device__ __forceinline__ Ctl carve(uint8_t *raw, int S, int NB)
 {
     const uint32_t off = smem_u32(raw);
     uint8_t *base = raw + ((1024u - (off & 1023u)) & 1023u);
     Ctl c;
+    c.b_bytes = (uint32_t)NB * 128;
     c.a0 = smem_u32(base);
     c.b0 = c.a0 + S * kAStage;
-    uint8_t *bars = base + Layout<S, NB>::kBars;
+    uint8_t *bars = base + S * (kAStage + c.b_bytes);
     c.full = (uint64_t *)bars;
-    c.empty = c.full + S;
-    c.done = c.empty + S;
+    c.empty = c.full + kMaxStages;
+    c.done = c.empty + kMaxStages;
     c.tmem_slot = (uint32_t *)(c.done + 1);
     c.abort = (volatile int *)(c.tmem_slot + 1);
     return c;
@@ -81,8 +84,8 @@ __device__ __forceinline__ void set_abort(const Ctl &c, int32_t *err)
     atomicCAS(err, 0, (int)SL_ERR_TIMEOUT);
 }
 
-template <int S>
-__device__ __forceinline__ void prologue(const Ctl &c, uint32_t ncols)
+// Barrier init and tensor-memory allocation; ends with a CTA barrier.
+__device__ __forceinline__ uint32_t prologue(const Ctl &c, int S, uint32_t ncols)
 {
     if (threadIdx.x == 0) {
         for (int s = 0; s < S; ++s) {
@@ -94,6 +97,10 @@ __device__ __forceinline__ void prologue(const Ctl &c, uint32_t ncols)
         tc::fence_mbar_init();
     }
     if (threadIdx.x < 32) tc::tmem_alloc(c.tmem_slot, ncols);
+    tc::tc_fence_before();
+    __syncthreads();
+    tc::tc_fence_after();
+    return *c.tmem_slot;
 }
 
 __device__ __forceinline__ void finish(const Ctl &c, uint32_t tmem, uint32_t ncols)
@@ -110,67 +117,63 @@ struct TmemCols {
 
 // ---------------------------------------------------------------------- mainloop
 // Streams KC contraction chunks through an S-stage ring and accumulates D = A B^T in
-// tensor memory. Every thread issues its share of the A-chunk copies (load_a); the B
-// chunk either arrives by one bulk copy from a packed tile (kBulkB) or is loaded by the
-// threads too (load_b). Thread 0 issues the MMAs (issue(stage, chunk)) and commits each
-// chunk to the stage's `empty` barrier. Before chunk `dep_chunk` is loaded every thread
-// waits for the preceding grid (programmatic dependent launch). On return the
-// accumulator is complete (or the CTA has aborted; *c.abort is then set and uniform).
-template <int S, int NB, bool kBulkB, class LoadA, class LoadB, class Issue>
-__device__ __forceinline__ void mainloop(const Ctl &c, int KC, const uint8_t *__restrict__ bpack, int dep_chunk,
-                                         long long limit, int32_t *err, LoadA load_a, LoadB load_b, Issue issue)
+// tensor memory. Thread 0 issues, per chunk, the TMA tiles and bulk copies of the stage
+// (tma(chunk, stage, full_barrier), which also sets the expected bytes) and the MMAs
+// (issue(stage, chunk)), committing each chunk to the stage's `empty` barrier. With
+// kGather the other threads also copy their share of the A chunk (gather(chunk, stage))
+// by cp.async. Before chunk `dep_chunk` is loaded the loaders wait for the preceding
+// grid (programmatic dependent launch); every thread has waited on return. On return the
+// accumulator is complete, or the CTA has aborted (*c.abort set, uniform).
+template <bool kGather, class Tma, class Gather, class Issue>
+__device__ __forceinline__ void mainloop(const Ctl &c, int S, int KC, int dep_chunk, long long limit, int32_t *err,
+                                         Tma tma, Gather gather, Issue issue)
 {
-    constexpr uint32_t kB = (uint32_t)NB * 128;
     const int tid = threadIdx.x;
-    int n_issued = 0, n_waited = 0;  // bulk B copies (thread 0)
-    for (int it = 0; it < KC + S - 1; ++it) {
-        if (it < KC) {
-            const int s = it % S, use = it / S;
-            if (use > 0 && !*c.abort)
-                if (!tc::mbar_wait(&c.empty[s], (use - 1) & 1, limit, c.abort)) set_abort(c, err);
-            if (it == dep_chunk) tc::grid_dep_wait();
-            if (!*c.abort) {
-                if (kBulkB) {
+    int n_issued = 0, n_waited = 0;  // thread 0: chunks whose copies were issued / awaited
+    if (kGather || tid == 0) {
+        for (int it = 0; it < KC + S - 1; ++it) {
+            if (it < KC) {
+                const int s = it % S, use = it / S;
+                if (use > 0 && !*c.abort)
+                    if (!tc::mbar_wait(&c.empty[s], (use - 1) & 1, limit, c.abort)) set_abort(c, err);
+                if (it == dep_chunk) tc::grid_dep_wait();
+                if (!*c.abort) {
                     if (tid == 0) {
-                        tc::mbar_arrive_expect_tx(&c.full[s], kB);
-                        tc::bulk_g2s(c.b0 + s * kB, bpack + (size_t)it * kB, kB, &c.full[s]);
+                        tma(it, s, &c.full[s]);
                         ++n_issued;
                     }
-                } else {
-                    load_b(it, c.b0 + s * kB);
+                    if (kGather) gather(it, s);
                 }
-                load_a(it, c.a0 + s * kAStage);
+                if (kGather) tc::cp_async_commit();
             }
-            tc::cp_async_commit();
-        }
-        const int j = it - (S - 1);
-        if (j >= 0) {
-            tc::cp_async_wait_dyn(min(it, KC - 1) - j);
-            tc::fence_proxy_async();
-            __syncthreads();
-            if (tid == 0 && !*c.abort) {
-                const int s = j % S;
-                bool ok = true;
-                if (kBulkB) {
-                    ok = j < n_issued && tc::mbar_wait(&c.full[s], (j / S) & 1, limit, c.abort);
-                    if (ok) ++n_waited;
+            const int j = it - (S - 1);
+            if (j >= 0) {
+                if (kGather) {
+                    tc::cp_async_wait_dyn(min(it, KC - 1) - j);
+                    tc::fence_proxy_async();
+                    __syncthreads();
                 }
-                if (ok) {
-                    tc::tc_fence_after();
-                    issue(s, j);
-                    tc::mma_commit(&c.empty[s]);
-                } else {
-                    set_abort(c, err);
+                if (tid == 0 && !*c.abort) {
+                    const int s = j % S;
+                    if (j < n_issued && tc::mbar_wait(&c.full[s], (j / S) & 1, limit, c.abort)) {
+                        ++n_waited;
+                        tc::tc_fence_after();
+                        issue(s, j);
+                        tc::mma_commit(&c.empty[s]);
+                    } else {
+                        set_abort(c, err);
+                    }
                 }
             }
         }
     }
+    tc::grid_dep_wait();  // every thread: later reads may touch the preceding grid's output
     if (tid == 0) {
         tc::mma_commit(c.done);  // arrives once every MMA issued above has completed
-        for (int jj = n_waited; jj < n_issued; ++jj)  // bulk copies still in flight after an abort
+        for (int jj = n_waited; jj < n_issued; ++jj)  // copies still in flight after an abort
             tc::mbar_wait(&c.full[jj % S], (jj / S) & 1, kDrainLimit, nullptr);
     }
-    tc::cp_async_wait<0>();
+    if (kGather) tc::cp_async_wait<0>();
     if (!tc::mbar_wait(c.done, 0, limit, nullptr)) {
         set_abort(c, err);
         tc::mbar_wait(c.done, 0, kDrainLimit, nullptr);
@@ -194,9 +197,10 @@ __device__ __forceinline__ void issue_kmajor(uint32_t tmem, uint32_t a_stage, ui
 // ----------------------------------------------------------------------- helpers
 __device__ __forceinline__ float sigm(float z) { return 1.0f / (1.0f + __expf(-z)); }
 
-__device__ __forceinline__ void ld8f(const float *p, float (&v)[8])
+// L2-coherent read (bypasses L1) of state another CTA or an earlier launch wrote.
+__device__ __forceinline__ void ld8f_cg(const float *p, float (&v)[8])
 {
-    const float4 a = *(const float4 *)p, b = *(const float4 *)(p + 4);
+    const float4 a = __ldcg((const float4 *)p), b = __ldcg((const float4 *)(p + 4));
     v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w; v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
 }
 __device__ __forceinline__ void st8f(float *p, const float (&v)[8])
@@ -238,7 +242,7 @@ __device__ __forceinline__ void unpack8_f16(uint4 u, float (&v)[8])
 // ------------------------------------------------------------------ arguments
 struct StepArgs {
     int T, B, I, H;
-    const __nv_bfloat16 *x;     // [T][B][I]
+    int kcx, KC, S;             // x-part chunks, all chunks, ring depth
     const int32_t *top;         // [T+1][B]
     __nv_bfloat16 *hist_h;      // [T+1][B][H]
     float *hist_c;              // [T+1][B][H]
@@ -247,75 +251,63 @@ struct StepArgs {
     const uint8_t *wpack;       // packed B-operand tiles of this kernel
     float *dhist_h, *dhist_c;   // [T+1][B][H]
     __nv_bfloat16 *dG;          // [T][B][4H]
-    int kc;                     // contraction chunks
     long long limit;
     int32_t *err;
 };
 
 // ------------------------------------------------------------------ forward step
-template <int U, int S>
-__global__ void __launch_bounds__(kThreads, 1) fwd_step_tc(StepArgs a, int t)
+// The contraction runs over [x_t padded to 64 ; h_read padded to 64]: chunks < kcx
+// come from x_t by TMA, the rest are gathered history rows.
+template <int U>
+__global__ void __launch_bounds__(kThreads, 1)
+fwd_step_tc(const __grid_constant__ CUtensorMap tm_x, StepArgs a, int t)
 {
     constexpr int NB = 4 * U;
     constexpr uint32_t kCols = TmemCols<NB>::value;
     extern __shared__ uint8_t smem_raw[];
-    __shared__ int s_src[kRows];
-    const Ctl c = carve<S, NB>(smem_raw);
+    const Ctl c = carve(smem_raw, a.S, NB);
     const int tid = threadIdx.x, warp = tid >> 5;
     const int ct = blockIdx.x, row0 = blockIdx.y * kRows;
-    const int B = a.B, I = a.I, H = a.H;
+    const int B = a.B, H = a.H, kcx = a.kcx;
+    // this thread's tile row and the history row it reads (the prepass ran before step 0)
+    const int b = row0 + tid;
+    const bool row_ok = b < B;
+    const int src = row_ok ? a.top[(size_t)t * B + b] : 0;
+    const __nv_bfloat16 *hrow = a.hist_h + ((size_t)src * B + b) * H;
+    const uint32_t tmem = prologue(c, a.S, kCols);
 
-    prologue<S>(c, kCols);
-    // history row each tile row reads (the prepass finished before the first step)
-    for (int r = tid; r < kRows; r += kThreads) s_src[r] = row0 + r < B ? a.top[(size_t)t * B + row0 + r] : 0;
-    tc::tc_fence_before();
-    __syncthreads();
-    tc::tc_fence_after();
-    const uint32_t tmem = *c.tmem_slot;
-
-    const __nv_bfloat16 *xt = a.x + (size_t)t * B * I;
-    auto load_a = [&](int kc, uint32_t dst) {
-        // 128 rows x 8 pieces of 16 bytes; 8 consecutive threads cover one 128-byte row
-#pragma unroll 4
-        for (int p = tid; p < kRows * 8; p += kThreads) {
-            const int r = p >> 3, q = p & 7;
-            const int b = row0 + r, k = kc * kChunk + q * 8;
-            const void *src = a.x;
-            uint32_t bytes = 0;
-            if (b < B) {
-                if (k < I) {
-                    src = xt + (size_t)b * I + k;
-                    bytes = 16;
-                } else if (k < I + H) {
-                    src = a.hist_h + ((size_t)s_src[r] * B + b) * H + (k - I);
-                    bytes = 16;
-                }
-            }
-            tc::cp_async16(dst + sw128(r, q), src, bytes);
+    const uint8_t *bpack = a.wpack + (size_t)ct * a.KC * c.b_bytes;
+    auto tma = [&](int it, int s, uint64_t *bar) {
+        tc::mbar_arrive_expect_tx(bar, c.b_bytes + (it < kcx ? kAStage : 0u));
+        if (it < kcx) tc::tma_load_2d(c.a0 + s * kAStage, &tm_x, it * kChunk, t * B + row0, bar);
+        tc::bulk_g2s(c.b0 + s * c.b_bytes, bpack + (size_t)it * c.b_bytes, c.b_bytes, bar);
+    };
+    auto gather = [&](int it, int s) {
+        if (it < kcx || !row_ok) return;  // rows past B stay unread: their results are never stored
+        const int k0 = (it - kcx) * kChunk;
+        const uint32_t dst = c.a0 + s * kAStage;
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+            const int k = k0 + q * 8;
+            tc::cp_async16(dst + sw128(tid, q), k < H ? (const void *)(hrow + k) : (const void *)hrow,
+                           k < H ? 16u : 0u);
         }
     };
-    auto no_b = [](int, uint32_t) {};
-    auto issue = [&](int s, int j) {
-        issue_kmajor<NB>(tmem, c.a0 + s * kAStage, c.b0 + s * Layout<S, NB>::kB, j);
-    };
-    const uint8_t *bpack = a.wpack + (size_t)ct * a.kc * NB * 128;
-    // chunks that touch h_read depend on the previous step
-    mainloop<S, NB, true>(c, a.kc, bpack, I / kChunk, a.limit, a.err, load_a, no_b, issue);
+    auto issue = [&](int s, int j) { issue_kmajor<NB>(tmem, c.a0 + s * kAStage, c.b0 + s * c.b_bytes, j); };
+    mainloop<true>(c, a.S, a.KC, kcx, a.limit, a.err, tma, gather, issue);
     tc::grid_dep_launch();
 
     if (!*c.abort) {
-        const int r = tid, b = row0 + r;
         const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
-        const int src = s_src[r];
 #pragma unroll 1
         for (int cu = 0; cu < U / 8; ++cu) {
             float z[4][8];
 #pragma unroll
             for (int g = 0; g < 4; ++g) tc::tmem_ld8(trow + g * U + cu * 8, z[g]);
             const int u = ct * U + cu * 8;
-            if (b < B && u < H) {
+            if (row_ok && u < H) {
                 float cr[8], cn[8], hn[8], gv[4][8];
-                ld8f(a.hist_c + ((size_t)src * B + b) * H + u, cr);
+                ld8f_cg(a.hist_c + ((size_t)src * B + b) * H + u, cr);
 #pragma unroll
                 for (int e = 0; e < 8; ++e) {
                     const float ig = sigm(z[0][e] + __ldg(a.bias + u + e));
@@ -349,10 +341,10 @@ __device__ __forceinline__ void pointwise8(const StepArgs &a, int tp, int b, int
     const int s1 = a.top[(size_t)tp * B + b];
     const size_t rd = ((size_t)s1 * B + b) * H + u;
     float dh[8], dcn[8], cn[8], cr[8], ig[8], fg[8], gg[8], og[8];
-    ld8f(a.dhist_h + wr, dh);
-    ld8f(a.dhist_c + wr, dcn);
-    ld8f(a.hist_c + wr, cn);
-    ld8f(a.hist_c + rd, cr);
+    ld8f_cg(a.dhist_h + wr, dh);
+    ld8f_cg(a.dhist_c + wr, dcn);
+    ld8f_cg(a.hist_c + wr, cn);
+    ld8f_cg(a.hist_c + rd, cr);
     const __half *gt = a.gates + ((size_t)tp * B + b) * 4 * H + u;
     unpack8_f16(*(const uint4 *)(gt), ig);
     unpack8_f16(*(const uint4 *)(gt + H), fg);
@@ -373,7 +365,7 @@ __device__ __forceinline__ void pointwise8(const StepArgs &a, int tp, int b, int
 #pragma unroll
     for (int g = 0; g < 4; ++g) *(uint4 *)(dg + (size_t)g * H) = pack8_bf16(d[g]);
     float acc[8];
-    ld8f(a.dhist_c + rd, acc);
+    ld8f_cg(a.dhist_c + rd, acc);
 #pragma unroll
     for (int e = 0; e < 8; ++e) acc[e] += dcr[e];
     st8f(a.dhist_c + rd, acc);
@@ -390,57 +382,44 @@ __global__ void pointwise_last(StepArgs a)
     }
 }
 
-template <int U, int S>
-__global__ void __launch_bounds__(kThreads, 1) bwd_step_tc(StepArgs a, int t)
+template <int U>
+__global__ void __launch_bounds__(kThreads, 1)
+bwd_step_tc(const __grid_constant__ CUtensorMap tm_g, StepArgs a, int t)
 {
     constexpr int NB = U;
     constexpr uint32_t kCols = TmemCols<NB>::value;
     extern __shared__ uint8_t smem_raw[];
-    __shared__ int s_src[kRows];
-    const Ctl c = carve<S, NB>(smem_raw);
+    const Ctl c = carve(smem_raw, a.S, NB);
     const int tid = threadIdx.x, warp = tid >> 5;
     const int ct = blockIdx.x, row0 = blockIdx.y * kRows;
-    const int B = a.B, H = a.H, G = 4 * H;
+    const int B = a.B, H = a.H;
+    const int b = row0 + tid;
+    const bool row_ok = b < B;
+    const int src = row_ok ? a.top[(size_t)t * B + b] : 0;
+    const uint32_t tmem = prologue(c, a.S, kCols);
 
-    prologue<S>(c, kCols);
-    for (int r = tid; r < kRows; r += kThreads) s_src[r] = row0 + r < B ? a.top[(size_t)t * B + row0 + r] : 0;
-    tc::tc_fence_before();
-    __syncthreads();
-    tc::tc_fence_after();
-    const uint32_t tmem = *c.tmem_slot;
-
-    const __nv_bfloat16 *dgt = a.dG + (size_t)t * B * G;
-    auto load_a = [&](int kc, uint32_t dst) {
-#pragma unroll 4
-        for (int p = tid; p < kRows * 8; p += kThreads) {
-            const int r = p >> 3, q = p & 7;
-            const int b = row0 + r, n = kc * kChunk + q * 8;
-            const bool ok = b < B && n < G;
-            tc::cp_async16(dst + sw128(r, q), ok ? (const void *)(dgt + (size_t)b * G + n) : (const void *)a.dG,
-                           ok ? 16u : 0u);
-        }
+    const uint8_t *bpack = a.wpack + (size_t)ct * a.KC * c.b_bytes;
+    auto tma = [&](int it, int s, uint64_t *bar) {
+        tc::mbar_arrive_expect_tx(bar, kAStage + c.b_bytes);
+        tc::tma_load_2d(c.a0 + s * kAStage, &tm_g, it * kChunk, t * B + row0, bar);
+        tc::bulk_g2s(c.b0 + s * c.b_bytes, bpack + (size_t)it * c.b_bytes, c.b_bytes, bar);
     };
-    auto no_b = [](int, uint32_t) {};
-    auto issue = [&](int s, int j) {
-        issue_kmajor<NB>(tmem, c.a0 + s * kAStage, c.b0 + s * Layout<S, NB>::kB, j);
-    };
-    const uint8_t *bpack = a.wpack + (size_t)ct * a.kc * NB * 128;
-    mainloop<S, NB, true>(c, a.kc, bpack, 0, a.limit, a.err, load_a, no_b, issue);
+    auto no_gather = [](int, int) {};
+    auto issue = [&](int s, int j) { issue_kmajor<NB>(tmem, c.a0 + s * kAStage, c.b0 + s * c.b_bytes, j); };
+    mainloop<false>(c, a.S, a.KC, 0, a.limit, a.err, tma, no_gather, issue);
     tc::grid_dep_launch();
 
     if (!*c.abort) {
-        const int r = tid, b = row0 + r;
         const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
-        const int src = s_src[r];
 #pragma unroll 1
         for (int cu = 0; cu < U / 8; ++cu) {
             float acc[8];
             tc::tmem_ld8(trow + cu * 8, acc);
             const int u = ct * U + cu * 8;
-            if (b < B && u < H) {
+            if (row_ok && u < H) {
                 float *d = a.dhist_h + ((size_t)src * B + b) * H + u;
                 float v[8];
-                ld8f(d, v);
+                ld8f_cg(d, v);
 #pragma unroll
                 for (int e = 0; e < 8; ++e) v[e] += acc[e];
                 st8f(d, v);
@@ -453,44 +432,33 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_step_tc(StepArgs a, int t)
 
 // ------------------------------------------------------------- input gradient
 struct DxArgs {
-    const __nv_bfloat16 *dG;  // [R][4H]
     size_t R;
-    int I, H, kc;
+    int I, KC, S;
     const uint8_t *wpack;
     float *dx;  // [R][I]
     long long limit;
     int32_t *err;
 };
 
-template <int N, int S>
-__global__ void __launch_bounds__(kThreads, 1) dx_tc(DxArgs a)
+template <int N>
+__global__ void __launch_bounds__(kThreads, 1) dx_tc(const __grid_constant__ CUtensorMap tm_g, DxArgs a)
 {
     constexpr uint32_t kCols = TmemCols<N>::value;
     extern __shared__ uint8_t smem_raw[];
-    const Ctl c = carve<S, N>(smem_raw);
+    const Ctl c = carve(smem_raw, a.S, N);
     const int tid = threadIdx.x, warp = tid >> 5;
     const int ct = blockIdx.x;
     const size_t row0 = (size_t)blockIdx.y * kRows;
-    const int G = 4 * a.H;
-    prologue<S>(c, kCols);
-    tc::tc_fence_before();
-    __syncthreads();
-    tc::tc_fence_after();
-    const uint32_t tmem = *c.tmem_slot;
-    auto load_a = [&](int kc, uint32_t dst) {
-#pragma unroll 4
-        for (int p = tid; p < kRows * 8; p += kThreads) {
-            const int r = p >> 3, q = p & 7;
-            const size_t row = row0 + r;
-            const int n = kc * kChunk + q * 8;
-            const bool ok = row < a.R && n < G;
-            tc::cp_async16(dst + sw128(r, q), ok ? (const void *)(a.dG + row * G + n) : (const void *)a.dG,
-                           ok ? 16u : 0u);
-        }
+    const uint32_t tmem = prologue(c, a.S, kCols);
+    const uint8_t *bpack = a.wpack + (size_t)ct * a.KC * c.b_bytes;
+    auto tma = [&](int it, int s, uint64_t *bar) {
+        tc::mbar_arrive_expect_tx(bar, kAStage + c.b_bytes);
+        tc::tma_load_2d(c.a0 + s * kAStage, &tm_g, it * kChunk, (int)row0, bar);
+        tc::bulk_g2s(c.b0 + s * c.b_bytes, bpack + (size_t)it * c.b_bytes, c.b_bytes, bar);
     };
-    auto no_b = [](int, uint32_t) {};
-    auto issue = [&](int s, int j) { issue_kmajor<N>(tmem, c.a0 + s * kAStage, c.b0 + s * Layout<S, N>::kB, j); };
-    mainloop<S, N, true>(c, a.kc, a.wpack + (size_t)ct * a.kc * N * 128, -1, a.limit, a.err, load_a, no_b, issue);
+    auto no_gather = [](int, int) {};
+    auto issue = [&](int s, int j) { issue_kmajor<N>(tmem, c.a0 + s * kAStage, c.b0 + s * c.b_bytes, j); };
+    mainloop<false>(c, a.S, a.KC, -1, a.limit, a.err, tma, no_gather, issue);
     if (!*c.abort) {
         const size_t row = row0 + tid;
         const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
@@ -508,81 +476,88 @@ __global__ void __launch_bounds__(kThreads, 1) dx_tc(DxArgs a)
 // ------------------------------------------------------------- weight gradient
 // dW_ext[m][n] = sum_r A[r][m] dG[r][n] over r = t * B + b, where A[r] = [x_t ; h_read ; 1]
 // (m = I + H is the all-ones row, which yields dbias). Both operands are read MN-major:
-// 64 consecutive r per chunk, 64-wide MN blocks of 128-byte swizzled rows.
+// 64 consecutive r per chunk; each 64-wide MN block is 64 rows of 128 swizzled bytes.
+// dG blocks and x blocks (fully inside x) arrive by TMA; the other A blocks are gathered.
 struct DwArgs {
-    int T, B, I, H;
-    const __nv_bfloat16 *x, *hist_h, *dG, *ones;
+    int B, I, H;
+    const __nv_bfloat16 *x, *hist_h, *ones;
     const int32_t *top;
-    size_t R;
-    int n_tiles_n, split;
+    int R;
+    int n_tiles_n, split, S;
     float *part;  // [split][mt * 128][nt * 256]
     size_t ld_part, rows_part;
     long long limit;
     int32_t *err;
 };
 
-template <int S>
-__global__ void __launch_bounds__(kThreads, 1) dw_tc(DwArgs a)
+__global__ void __launch_bounds__(kThreads, 1)
+dw_tc(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtensorMap tm_g, DwArgs a)
 {
     constexpr int NB = 256;
     constexpr uint32_t kCols = 256;
+    constexpr uint32_t kBlk = 64 * 128;  // one MN block of a chunk
     extern __shared__ uint8_t smem_raw[];
-    const Ctl c = carve<S, NB>(smem_raw);
+    const Ctl c = carve(smem_raw, a.S, NB);
     const int tid = threadIdx.x, warp = tid >> 5;
     const int mt = blockIdx.x / a.n_tiles_n, nt = blockIdx.x % a.n_tiles_n, sp = blockIdx.y;
-    const int B = a.B, I = a.I, H = a.H, G = 4 * H;
-    const size_t RC = (a.R + kChunk - 1) / kChunk;
-    const size_t c_lo = RC * sp / a.split, c_hi = RC * (sp + 1) / a.split;
-    const int KC = (int)(c_hi - c_lo);
-    prologue<S>(c, kCols);
-    tc::tc_fence_before();
-    __syncthreads();
-    tc::tc_fence_after();
-    const uint32_t tmem = *c.tmem_slot;
+    const int B = a.B, I = a.I, H = a.H;
+    const int RC = (a.R + kChunk - 1) / kChunk;
+    const int c_lo = (int)((long long)RC * sp / a.split), c_hi = (int)((long long)RC * (sp + 1) / a.split);
+    const int KC = c_hi - c_lo;
+    const uint32_t tmem = prologue(c, a.S, kCols);
 
-    auto load_a = [&](int kc, uint32_t dst) {  // 64 r-rows x (2 blocks x 8 pieces)
-#pragma unroll 4
-        for (int p = tid; p < kChunk * 16; p += kThreads) {
-            const int rr = p >> 4, blk = (p >> 3) & 1, q = p & 7;
-            const size_t r = (c_lo + kc) * kChunk + rr;
-            const int m = mt * kRows + blk * 64 + q * 8;
-            const void *src = a.ones;
+    auto tma = [&](int it, int s, uint64_t *bar) {
+        const int r0 = (c_lo + it) * kChunk;
+        uint32_t bytes = 4 * kBlk;
+        for (int blk = 0; blk < 2; ++blk)
+            if (mt * kRows + blk * 64 + 64 <= I) bytes += kBlk;
+        tc::mbar_arrive_expect_tx(bar, bytes);
+        for (int blk = 0; blk < 2; ++blk) {
+            const int m0 = mt * kRows + blk * 64;
+            if (m0 + 64 <= I) tc::tma_load_2d(c.a0 + s * kAStage + blk * kBlk, &tm_x, m0, r0, bar);
+        }
+        for (int nb = 0; nb < 4; ++nb)
+            tc::tma_load_2d(c.b0 + s * c.b_bytes + nb * kBlk, &tm_g, nt * NB + nb * 64, r0, bar);
+    };
+    // thread -> (r-row rr, block blk): one 128-byte row segment of eight 16-byte pieces
+    auto gather = [&](int it, int s) {
+        const int rr = tid & 63, blk = tid >> 6;
+        const int m0 = mt * kRows + blk * 64;
+        if (m0 + 64 <= I) return;  // arrives by TMA
+        const int r = (c_lo + it) * kChunk + rr;
+        const uint32_t dst = c.a0 + s * kAStage + blk * kBlk;
+        const bool r_ok = r < a.R;
+        const int tb = r_ok ? r / B : 0;
+        const int bb = r - tb * B;
+        const __nv_bfloat16 *hrow = a.hist_h + ((size_t)(r_ok ? a.top[r] : 0) * B + bb) * H;
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+            const int m = m0 + q * 8;
+            const void *p = a.ones;
             uint32_t bytes = 0;
-            if (r < a.R) {
+            if (r_ok) {
                 if (m < I) {
-                    src = a.x + r * I + m;
+                    p = a.x + (size_t)r * I + m;
                     bytes = 16;
                 } else if (m < I + H) {
-                    const size_t b = r % B;
-                    src = a.hist_h + ((size_t)a.top[r] * B + b) * H + (m - I);
+                    p = hrow + (m - I);
                     bytes = 16;
                 } else if (m == I + H) {
                     bytes = 16;
                 }
             }
-            tc::cp_async16(dst + blk * 8192 + sw128(rr, q), src, bytes);
-        }
-    };
-    auto load_b = [&](int kc, uint32_t dst) {  // 64 r-rows x (4 blocks x 8 pieces)
-#pragma unroll 4
-        for (int p = tid; p < kChunk * 32; p += kThreads) {
-            const int rr = p >> 5, blk = (p >> 3) & 3, q = p & 7;
-            const size_t r = (c_lo + kc) * kChunk + rr;
-            const int n = nt * NB + blk * 64 + q * 8;
-            const bool ok = r < a.R && n < G;
-            tc::cp_async16(dst + blk * 8192 + sw128(rr, q), ok ? (const void *)(a.dG + r * G + n) : (const void *)a.dG,
-                           ok ? 16u : 0u);
+            tc::cp_async16(dst + sw128(rr, q), p, bytes);
         }
     };
     auto issue = [&](int s, int j) {
         constexpr uint32_t idesc = tc::idesc_bf16(NB, 1, 1);
-        const uint32_t as = c.a0 + s * kAStage, bs = c.b0 + s * Layout<S, NB>::kB;
+        const uint32_t as = c.a0 + s * kAStage, bs = c.b0 + s * c.b_bytes;
 #pragma unroll
         for (int k = 0; k < kChunk / 16; ++k)  // 16 r-rows = two 8-row groups = 2048 bytes
-            tc::mma_bf16(tmem, tc::smem_desc(as + k * 2048, 8192, 1024), tc::smem_desc(bs + k * 2048, 8192, 1024),
+            tc::mma_bf16(tmem, tc::smem_desc(as + k * 2048, kBlk, 1024), tc::smem_desc(bs + k * 2048, kBlk, 1024),
                          idesc, (j | k) != 0);
     };
-    if (KC > 0) mainloop<S, NB, false>(c, KC, nullptr, -1, a.limit, a.err, load_a, load_b, issue);
+    if (KC > 0) mainloop<true>(c, a.S, KC, -1, a.limit, a.err, tma, gather, issue);
     if (!*c.abort) {
         const size_t m = (size_t)mt * kRows + tid;
         float *dst = a.part + ((size_t)sp * a.rows_part + m) * a.ld_part + (size_t)nt * NB;
@@ -621,12 +596,12 @@ __global__ void dw_reduce(int K, int G, int split, const float *__restrict__ par
 
 // ------------------------------------------------------------------ packing
 // Forward operand: for column tile ct, rows n = g * U + j hold gate g of hidden unit
-// ct * U + j; each row is the matching column of W over the contraction [x ; h] (zero
-// padded), in 64-element chunks of 128-byte swizzled rows.
-__global__ void pack_fwd(const __nv_bfloat16 *__restrict__ W, int I, int H, int U, int KC, int n_ct,
+// ct * U + j; each row is the matching column of W over the contraction
+// [x padded to 64 ; h padded to 64], in 64-element chunks of 128-byte swizzled rows.
+__global__ void pack_fwd(const __nv_bfloat16 *__restrict__ W, int I, int H, int U, int kcx, int KC, int n_ct,
                          __nv_bfloat16 *__restrict__ out)
 {
-    const int NB = 4 * U, K = I + H, G = 4 * H;
+    const int NB = 4 * U, G = 4 * H;
     const size_t n = (size_t)n_ct * KC * NB * kChunk;
     for (size_t e = blockIdx.x * (size_t)blockDim.x + threadIdx.x; e < n; e += (size_t)gridDim.x * blockDim.x) {
         const int col = (int)(e % kChunk);
@@ -634,8 +609,17 @@ __global__ void pack_fwd(const __nv_bfloat16 *__restrict__ W, int I, int H, int 
         const int row = (int)(rowi % NB);
         const size_t tile = rowi / NB;
         const int kc = (int)(tile % KC), ct = (int)(tile / KC);
-        const int g = row / U, unit = ct * U + row % U, k = kc * kChunk + col;
-        const __nv_bfloat16 v = (unit < H && k < K) ? W[(size_t)k * G + g * H + unit] : __float2bfloat16(0.0f);
+        const int g = row / U, unit = ct * U + row % U;
+        int wrow = -1;
+        if (kc < kcx) {
+            const int k = kc * kChunk + col;
+            if (k < I) wrow = k;
+        } else {
+            const int k = (kc - kcx) * kChunk + col;
+            if (k < H) wrow = I + k;
+        }
+        const __nv_bfloat16 v =
+            (unit < H && wrow >= 0) ? W[(size_t)wrow * G + g * H + unit] : __float2bfloat16(0.0f);
         const size_t byte = tile * NB * 128 + sw128(row, col >> 3) + (col & 7) * 2;
         out[byte / 2] = v;
     }
@@ -663,8 +647,36 @@ __global__ void pack_rows(const __nv_bfloat16 *__restrict__ W, int H, int row0, 
 }
 
 // ------------------------------------------------------------------ host side
-constexpr int kSf32 = 3, kSf16 = 4, kSf8 = 4;  // forward ring depths by U
-constexpr int kSb = 4, kSx = 4, kSw = 4;
+PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+
+cudaError_t get_encoder()
+{
+    if (g_encode) return cudaSuccess;
+    cudaDriverEntryPointQueryResult q;
+    void *fn = nullptr;
+    cudaError_t e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q);
+    if (e != cudaSuccess) return e;
+    if (q != cudaDriverEntryPointSuccess || !fn) return cudaErrorNotSupported;
+    g_encode = (PFN_cuTensorMapEncodeTiled_v12000)fn;
+    return cudaSuccess;
+}
+
+// Row-major bf16 matrix [rows][cols] read in boxes of 64 columns x box_rows rows with
+// 128-byte swizzling; out-of-range elements read as zero.
+cudaError_t make_map(void *slot, const void *base, uint64_t rows, uint64_t cols, uint32_t box_rows)
+{
+    cuuint64_t dims[2] = {cols, rows};
+    cuuint64_t strides[1] = {cols * 2};
+    cuuint32_t box[2] = {(cuuint32_t)kChunk, box_rows};
+    cuuint32_t es[2] = {1, 1};
+    CUresult r = g_encode((CUtensorMap *)slot, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(base), dims,
+                          strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                          CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
+}
+
+enum { kMapX128 = 0, kMapX64 = 1, kMapG128 = 2, kMapG64 = 3 };
+const CUtensorMap &map(const stacklstm *s, int i) { return *(const CUtensorMap *)s->tmaps[i]; }
 
 template <typename Kern, typename... Args>
 cudaError_t launch(Kern kernel, dim3 grid, size_t smem, cudaStream_t st, bool pdl, Args... args)
@@ -682,25 +694,41 @@ cudaError_t launch(Kern kernel, dim3 grid, size_t smem, cudaStream_t st, bool pd
     return cudaLaunchKernelEx(&cfg, kernel, args...);
 }
 
+constexpr uint32_t kSmemCap = 225 * 1024;
+
 template <typename Kern>
-cudaError_t allow_smem(Kern k, uint32_t bytes)
+cudaError_t allow_smem(Kern k)
 {
-    return cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
+    return cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemCap);
+}
+
+// Ring depth: as many stages as the contraction has chunks, within a shared-memory
+// budget that leaves room for two CTAs per SM when the grid needs more than one wave.
+int pick_stages(int KC, int NB, size_t ctas, int sms)
+{
+    const uint32_t budget = ctas > (size_t)sms ? 100 * 1024 : 200 * 1024;
+    const uint32_t stage = kAStage + (uint32_t)NB * 128;
+    int S = (int)((budget - 1024 - (2 * kMaxStages + 1) * 8 - 16) / stage);
+    return std::max(2, std::min({S, KC, kMaxStages}));
 }
 
 int pick_dx_n(int I) { return I <= 32 ? 32 : I <= 64 ? 64 : I <= 128 ? 128 : 256; }
 
-unsigned grid_for(const stacklstm *s, size_t n) { return (unsigned)std::max<size_t>(1, std::min<size_t>(ceil_div(n, 256), (size_t)s->num_sms * 16)); }
+unsigned grid_for(const stacklstm *s, size_t n)
+{
+    return (unsigned)std::max<size_t>(1, std::min<size_t>(ceil_div(n, 256), (size_t)s->num_sms * 16));
+}
 
-StepArgs step_args(stacklstm *s, const __nv_bfloat16 *x, const float *bias, const void *wpack, int kc)
+StepArgs step_args(stacklstm *s, const float *bias, const void *wpack, int kcx, int KC, int S)
 {
     StepArgs a;
     a.T = s->T; a.B = s->B; a.I = s->I; a.H = s->H;
-    a.x = x; a.top = s->top;
+    a.kcx = kcx; a.KC = KC; a.S = S;
+    a.top = s->top;
     a.hist_h = (__nv_bfloat16 *)s->hist_h; a.hist_c = s->hist_c; a.gates = (__half *)s->gates;
     a.bias = bias; a.wpack = (const uint8_t *)wpack;
     a.dhist_h = s->dhist_h; a.dhist_c = s->dhist_c; a.dG = (__nv_bfloat16 *)s->dG;
-    a.kc = kc; a.limit = s->wait_limit; a.err = s->err;
+    a.limit = s->wait_limit; a.err = s->err;
     return a;
 }
 
@@ -708,24 +736,31 @@ StepArgs step_args(stacklstm *s, const __nv_bfloat16 *x, const float *bias, cons
 
 const char *bf16_unsupported(int T, int B, int I, int H)
 {
-    (void)T; (void)B;
     if (I % 8 || H % 8) return "bf16 path needs I and H to be multiples of 8";
+    if ((long long)T * B >= (1LL << 31) - 256) return "T * B too large for 32-bit tensor coordinates";
     return nullptr;
 }
 
 cudaError_t bf16_prepare(stacklstm *s)
 {
-    const int B = s->B, I = s->I, H = s->H, rt = (int)ceil_div(B, kRows), sms = s->num_sms;
+    cudaError_t e;
+    if ((e = get_encoder())) return e;
+    const int T = s->T, B = s->B, I = s->I, H = s->H, rt = (int)ceil_div(B, kRows), sms = s->num_sms;
     s->uf = (int)ceil_div(H, 32) * rt >= sms ? 32 : (int)ceil_div(H, 16) * rt >= sms / 2 ? 16 : 8;
     s->ub = (int)ceil_div(H, 32) * rt >= sms ? 32 : 16;
-    s->kcf = (int)ceil_div(I + H, kChunk);
+    s->kcx = (int)ceil_div(I, kChunk);
+    s->kcf = s->kcx + (int)ceil_div(H, kChunk);
     s->kcb = (int)ceil_div(4 * H, kChunk);
     s->nx = pick_dx_n(I);
     s->nxt = (int)ceil_div(I, s->nx);
     s->dw_mt = (int)ceil_div(I + H + 1, kRows);
     s->dw_nt = (int)ceil_div(4 * H, 256);
-    const size_t RC = ceil_div((size_t)s->T * B, kChunk);
+    const size_t R = (size_t)T * B, RC = ceil_div(R, kChunk);
     s->dw_split = (int)std::max<size_t>(1, std::min<size_t>(sms / std::max(1, s->dw_mt * s->dw_nt), RC / 2));
+    s->sf = pick_stages(s->kcf, 4 * s->uf, ceil_div(H, s->uf) * (size_t)rt, sms);
+    s->sb = pick_stages(s->kcb, s->ub, ceil_div(H, s->ub) * (size_t)rt, sms);
+    s->sx = pick_stages(s->kcb, s->nx, s->nxt * ceil_div(R, kRows), sms);
+    s->sw = pick_stages((int)ceil_div(RC, s->dw_split), 256, (size_t)s->dw_mt * s->dw_nt * s->dw_split, sms);
     const char *lim = getenv("STACKLSTM_WAIT_LIMIT_CYCLES");
     s->wait_limit = lim ? atoll(lim) : 4000000000LL;
 
@@ -734,7 +769,6 @@ cudaError_t bf16_prepare(stacklstm *s)
     const size_t dx_bytes = (size_t)s->nxt * s->kcb * s->nx * 128;
     s->dw_part_elems = (size_t)s->dw_split * s->dw_mt * kRows * s->dw_nt * 256;
     void *p;
-    cudaError_t e;
     if ((e = cudaMalloc(&p, fwd_bytes))) return e;
     s->allocs.push_back(p); s->w_fwd = p;
     if ((e = cudaMalloc(&p, bwd_bytes))) return e;
@@ -747,17 +781,15 @@ cudaError_t bf16_prepare(stacklstm *s)
     s->allocs.push_back(p); s->ones = p;
     const uint16_t one[8] = {0x3F80, 0, 0, 0, 0, 0, 0, 0};  // bf16 1.0 followed by zeros
     if ((e = cudaMemcpy(s->ones, one, 16, cudaMemcpyHostToDevice))) return e;
+    // dG is workspace: its tensor maps are fixed for the handle's lifetime
+    if ((e = make_map(s->tmaps[kMapG128], s->dG, R, 4 * (uint64_t)H, kRows))) return e;
+    if ((e = make_map(s->tmaps[kMapG64], s->dG, R, 4 * (uint64_t)H, kChunk))) return e;
 
-    if ((e = allow_smem(fwd_step_tc<32, kSf32>, Layout<kSf32, 128>::kBytes))) return e;
-    if ((e = allow_smem(fwd_step_tc<16, kSf16>, Layout<kSf16, 64>::kBytes))) return e;
-    if ((e = allow_smem(fwd_step_tc<8, kSf8>, Layout<kSf8, 32>::kBytes))) return e;
-    if ((e = allow_smem(bwd_step_tc<32, kSb>, Layout<kSb, 32>::kBytes))) return e;
-    if ((e = allow_smem(bwd_step_tc<16, kSb>, Layout<kSb, 16>::kBytes))) return e;
-    if ((e = allow_smem(dx_tc<32, kSx>, Layout<kSx, 32>::kBytes))) return e;
-    if ((e = allow_smem(dx_tc<64, kSx>, Layout<kSx, 64>::kBytes))) return e;
-    if ((e = allow_smem(dx_tc<128, kSx>, Layout<kSx, 128>::kBytes))) return e;
-    if ((e = allow_smem(dx_tc<256, kSx>, Layout<kSx, 256>::kBytes))) return e;
-    if ((e = allow_smem(dw_tc<kSw>, Layout<kSw, 256>::kBytes))) return e;
+    if ((e = allow_smem(fwd_step_tc<32>)) || (e = allow_smem(fwd_step_tc<16>)) || (e = allow_smem(fwd_step_tc<8>)) ||
+        (e = allow_smem(bwd_step_tc<32>)) || (e = allow_smem(bwd_step_tc<16>)) || (e = allow_smem(dx_tc<32>)) ||
+        (e = allow_smem(dx_tc<64>)) || (e = allow_smem(dx_tc<128>)) || (e = allow_smem(dx_tc<256>)) ||
+        (e = allow_smem(dw_tc)))
+        return e;
     return cudaSuccess;
 }
 
@@ -767,28 +799,32 @@ cudaError_t bf16_forward(stacklstm *s, const __nv_bfloat16 *x, const __nv_bfloat
     const int T = s->T, B = s->B, I = s->I, H = s->H;
     cudaError_t e;
     s->x_saved = x;
+    if ((e = make_map(s->tmaps[kMapX128], x, (uint64_t)T * B, I, kRows))) return e;
+    if ((e = make_map(s->tmaps[kMapX64], x, (uint64_t)T * B, I, kChunk))) return e;
     if ((e = cudaMemcpyAsync(s->hist_h, h0, sizeof(__nv_bfloat16) * B * H, cudaMemcpyDeviceToDevice, s->stream)))
         return e;
     if ((e = cudaMemcpyAsync(s->hist_c, c0, sizeof(float) * B * H, cudaMemcpyDeviceToDevice, s->stream))) return e;
     const int nctf = (int)ceil_div(H, s->uf), nctb = (int)ceil_div(H, s->ub);
     pack_fwd<<<grid_for(s, (size_t)nctf * s->kcf * 4 * s->uf * kChunk), 256, 0, s->stream>>>(
-        W, I, H, s->uf, s->kcf, nctf, (__nv_bfloat16 *)s->w_fwd);
+        W, I, H, s->uf, s->kcx, s->kcf, nctf, (__nv_bfloat16 *)s->w_fwd);
     pack_rows<<<grid_for(s, (size_t)nctb * s->kcb * s->ub * kChunk), 256, 0, s->stream>>>(
         W, H, I, H, s->ub, s->kcb, nctb, (__nv_bfloat16 *)s->w_bwd);
     pack_rows<<<grid_for(s, (size_t)s->nxt * s->kcb * s->nx * kChunk), 256, 0, s->stream>>>(
         W, H, 0, I, s->nx, s->kcb, s->nxt, (__nv_bfloat16 *)s->w_dx);
     s->launches += 3;
     if ((e = cudaGetLastError())) return e;
-    const StepArgs a = step_args(s, x, bias, s->w_fwd, s->kcf);
+    const StepArgs a = step_args(s, bias, s->w_fwd, s->kcx, s->kcf, s->sf);
     const dim3 grid(nctf, ceil_div(B, kRows));
+    const size_t smem = smem_bytes(s->sf, 4 * s->uf);
+    const CUtensorMap &tmx = map(s, kMapX128);
     for (int t = 0; t < T; ++t) {
         const bool pdl = t > 0;
         if (s->uf == 32)
-            e = launch(fwd_step_tc<32, kSf32>, grid, Layout<kSf32, 128>::kBytes, s->stream, pdl, a, t);
+            e = launch(fwd_step_tc<32>, grid, smem, s->stream, pdl, tmx, a, t);
         else if (s->uf == 16)
-            e = launch(fwd_step_tc<16, kSf16>, grid, Layout<kSf16, 64>::kBytes, s->stream, pdl, a, t);
+            e = launch(fwd_step_tc<16>, grid, smem, s->stream, pdl, tmx, a, t);
         else
-            e = launch(fwd_step_tc<8, kSf8>, grid, Layout<kSf8, 32>::kBytes, s->stream, pdl, a, t);
+            e = launch(fwd_step_tc<8>, grid, smem, s->stream, pdl, tmx, a, t);
         if (e) return e;
         s->launches += 1;
     }
@@ -799,17 +835,19 @@ cudaError_t bf16_backward_steps(stacklstm *s)
 {
     const int T = s->T, B = s->B, H = s->H;
     cudaError_t e;
-    const StepArgs a = step_args(s, (const __nv_bfloat16 *)s->x_saved, nullptr, s->w_bwd, s->kcb);
+    const StepArgs a = step_args(s, nullptr, s->w_bwd, 0, s->kcb, s->sb);
     pointwise_last<<<grid_for(s, (size_t)B * (H / 8)), 256, 0, s->stream>>>(a);
     s->launches += 1;
     if ((e = cudaGetLastError())) return e;
     const dim3 grid(ceil_div(H, s->ub), ceil_div(B, kRows));
+    const size_t smem = smem_bytes(s->sb, s->ub);
+    const CUtensorMap &tmg = map(s, kMapG128);
     for (int t = T - 1; t >= 0; --t) {
         const bool pdl = t < T - 1;
         if (s->ub == 32)
-            e = launch(bwd_step_tc<32, kSb>, grid, Layout<kSb, 32>::kBytes, s->stream, pdl, a, t);
+            e = launch(bwd_step_tc<32>, grid, smem, s->stream, pdl, tmg, a, t);
         else
-            e = launch(bwd_step_tc<16, kSb>, grid, Layout<kSb, 16>::kBytes, s->stream, pdl, a, t);
+            e = launch(bwd_step_tc<16>, grid, smem, s->stream, pdl, tmg, a, t);
         if (e) return e;
         s->launches += 1;
     }
@@ -818,46 +856,43 @@ cudaError_t bf16_backward_steps(stacklstm *s)
 
 cudaError_t bf16_dx(stacklstm *s, float *dx)
 {
-    const int T = s->T, B = s->B, I = s->I, H = s->H;
-    const size_t R = (size_t)T * B;
+    if (!dx) return cudaSuccess;
+    const size_t R = (size_t)s->T * s->B;
+    DxArgs d;
+    d.R = R; d.I = s->I; d.KC = s->kcb; d.S = s->sx;
+    d.wpack = (const uint8_t *)s->w_dx; d.dx = dx; d.limit = s->wait_limit; d.err = s->err;
+    const dim3 g(s->nxt, ceil_div(R, kRows));
+    const size_t smem = smem_bytes(s->sx, s->nx);
+    const CUtensorMap &tmg = map(s, kMapG128);
     cudaError_t e;
-    if (dx) {
-        DxArgs d;
-        d.dG = (const __nv_bfloat16 *)s->dG; d.R = R; d.I = I; d.H = H; d.kc = s->kcb;
-        d.wpack = (const uint8_t *)s->w_dx; d.dx = dx; d.limit = s->wait_limit; d.err = s->err;
-        const dim3 g(s->nxt, ceil_div(R, kRows));
-        switch (s->nx) {
-        case 32: e = launch(dx_tc<32, kSx>, g, Layout<kSx, 32>::kBytes, s->stream, false, d); break;
-        case 64: e = launch(dx_tc<64, kSx>, g, Layout<kSx, 64>::kBytes, s->stream, false, d); break;
-        case 128: e = launch(dx_tc<128, kSx>, g, Layout<kSx, 128>::kBytes, s->stream, false, d); break;
-        default: e = launch(dx_tc<256, kSx>, g, Layout<kSx, 256>::kBytes, s->stream, false, d); break;
-        }
-        if (e) return e;
-        s->launches += 1;
+    switch (s->nx) {
+    case 32: e = launch(dx_tc<32>, g, smem, s->stream, false, tmg, d); break;
+    case 64: e = launch(dx_tc<64>, g, smem, s->stream, false, tmg, d); break;
+    case 128: e = launch(dx_tc<128>, g, smem, s->stream, false, tmg, d); break;
+    default: e = launch(dx_tc<256>, g, smem, s->stream, false, tmg, d); break;
     }
+    if (e) return e;
+    s->launches += 1;
     return cudaGetLastError();
 }
 
 cudaError_t bf16_dw(stacklstm *s, float *dW, float *dbias)
 {
+    if (!dW && !dbias) return cudaSuccess;
     const int T = s->T, B = s->B, I = s->I, H = s->H;
-    const size_t R = (size_t)T * B;
-    cudaError_t e;
-    if (dW || dbias) {
-        DwArgs w;
-        w.T = T; w.B = B; w.I = I; w.H = H;
-        w.x = (const __nv_bfloat16 *)s->x_saved; w.hist_h = (const __nv_bfloat16 *)s->hist_h;
-        w.dG = (const __nv_bfloat16 *)s->dG; w.ones = (const __nv_bfloat16 *)s->ones; w.top = s->top;
-        w.R = R; w.n_tiles_n = s->dw_nt; w.split = s->dw_split; w.part = s->dw_part;
-        w.ld_part = (size_t)s->dw_nt * 256; w.rows_part = (size_t)s->dw_mt * kRows;
-        w.limit = s->wait_limit; w.err = s->err;
-        if ((e = launch(dw_tc<kSw>, dim3(s->dw_mt * s->dw_nt, s->dw_split), Layout<kSw, 256>::kBytes, s->stream,
-                        false, w)))
-            return e;
-        dw_reduce<<<grid_for(s, (size_t)(I + H + 1) * 4 * H), 256, 0, s->stream>>>(
-            I + H, 4 * H, s->dw_split, s->dw_part, w.rows_part, w.ld_part, dW, dbias);
-        s->launches += 2;
-    }
+    DwArgs w;
+    w.B = B; w.I = I; w.H = H;
+    w.x = (const __nv_bfloat16 *)s->x_saved; w.hist_h = (const __nv_bfloat16 *)s->hist_h;
+    w.ones = (const __nv_bfloat16 *)s->ones; w.top = s->top;
+    w.R = T * B; w.n_tiles_n = s->dw_nt; w.split = s->dw_split; w.S = s->sw; w.part = s->dw_part;
+    w.ld_part = (size_t)s->dw_nt * 256; w.rows_part = (size_t)s->dw_mt * kRows;
+    w.limit = s->wait_limit; w.err = s->err;
+    cudaError_t e = launch(dw_tc, dim3(s->dw_mt * s->dw_nt, s->dw_split), smem_bytes(s->sw, 256), s->stream, false,
+                           map(s, kMapX64), map(s, kMapG64), w);
+    if (e) return e;
+    dw_reduce<<<grid_for(s, (size_t)(I + H + 1) * 4 * H), 256, 0, s->stream>>>(
+        I + H, 4 * H, s->dw_split, s->dw_part, w.rows_part, w.ld_part, dW, dbias);
+    s->launches += 2;
     return cudaGetLastError();
 }
 

@@ -51,7 +51,9 @@ struct stacklstm {
 
     // bf16 tensor-core plan (bf16_path.cu)
     int uf = 0, ub = 0;      // hidden units per CTA tile: forward, backward
-    int kcf = 0, kcb = 0;    // 64-wide contraction chunks: forward (I+H), backward (4H)
+    int kcx = 0, kcf = 0, kcb = 0;  // 64-wide contraction chunks: x part, forward total, backward
+    int sf = 0, sb = 0, sx = 0, sw = 0;  // ring depths: forward, backward, dx, dW
+    alignas(64) unsigned char tmaps[4][128] = {};  // TMA descriptors (bf16_path.cu)
     int nx = 0, nxt = 0;     // input gradient: columns per tile, number of column tiles
     int dw_mt = 0, dw_nt = 0, dw_split = 0;  // weight gradient: row tiles, column tiles, splits
     long long wait_limit = 0;  // clock cycles one bounded device-side wait may spin

@@ -90,7 +90,16 @@ __device__ __forceinline__ void cp_async_wait_dyn(int n)
     case 3: cp_async_wait<3>(); break;
     case 4: cp_async_wait<4>(); break;
     case 5: cp_async_wait<5>(); break;
-    default: cp_async_wait<6>(); break;
+    case 6: cp_async_wait<6>(); break;
+    case 7: cp_async_wait<7>(); break;
+    case 8: cp_async_wait<8>(); break;
+    case 9: cp_async_wait<9>(); break;
+    case 10: cp_async_wait<10>(); break;
+    case 11: cp_async_wait<11>(); break;
+    case 12: cp_async_wait<12>(); break;
+    case 13: cp_async_wait<13>(); break;
+    case 14: cp_async_wait<14>(); break;
+    default: cp_async_wait<15>(); break;
     }
 }
 
@@ -105,6 +114,18 @@ __device__ __forceinline__ void bulk_g2s(uint32_t dst, const void *src, uint32_t
     asm volatile(
         "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
         "l"(src), "r"(bytes), "r"(smem_u32(bar))
+        : "memory");
+}
+
+// 2-D tiled tensor load (TMA): the box at (c0 = innermost column, c1 = row) of the tensor
+// map lands at dst (1024-byte aligned for 128-byte swizzling); completes the box's bytes
+// on the mbarrier. Out-of-range elements read as zero. c0 * element size must be a
+// multiple of 16 bytes.
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const void *tmap, int c0, int c1, uint64_t *bar)
+{
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];"
+        ::"r"(dst), "l"((uint64_t)tmap), "r"(c0), "r"(c1), "r"(smem_u32(bar))
         : "memory");
 }
 
