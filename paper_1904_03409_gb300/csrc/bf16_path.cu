@@ -128,9 +128,11 @@ template <bool kGather, class Tma, class Gather, class Issue>
 __device__ __forceinline__ void mainloop(const Ctl &c, int S, int KC, int dep_chunk, long long limit, int32_t *err,
                                          Tma tma, Gather gather, Issue issue)
 {
-    const int tid = threadIdx.x;
-    int n_issued = 0, n_waited = 0;  // thread 0: chunks whose copies were issued / awaited
-    if (kGather || tid == 0) {
+    // Every blocking wait below runs warp-uniformly: a try_wait suspends its whole warp,
+    // so a lone issuing lane must never share its warp with spinning lanes.
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    int n_issued = 0, n_waited = 0;  // warp 0: chunks whose copies were issued / awaited
+    if (kGather || warp == 0) {
         for (int it = 0; it < KC + S - 1; ++it) {
             if (it < KC) {
                 const int s = it % S, use = it / S;
@@ -138,10 +140,8 @@ __device__ __forceinline__ void mainloop(const Ctl &c, int S, int KC, int dep_ch
                     if (!tc::mbar_wait(&c.empty[s], (use - 1) & 1, limit, c.abort)) set_abort(c, err);
                 if (it == dep_chunk) tc::grid_dep_wait();
                 if (!*c.abort) {
-                    if (tid == 0) {
-                        tma(it, s, &c.full[s]);
-                        ++n_issued;
-                    }
+                    if (tid == 0) tma(it, s, &c.full[s]);
+                    if (warp == 0) ++n_issued;
                     if (kGather) gather(it, s);
                 }
                 if (kGather) tc::cp_async_commit();
@@ -153,13 +153,16 @@ __device__ __forceinline__ void mainloop(const Ctl &c, int S, int KC, int dep_ch
                     tc::fence_proxy_async();
                     __syncthreads();
                 }
-                if (tid == 0 && !*c.abort) {
+                if (warp == 0 && !*c.abort) {
                     const int s = j % S;
                     if (j < n_issued && tc::mbar_wait(&c.full[s], (j / S) & 1, limit, c.abort)) {
                         ++n_waited;
-                        tc::tc_fence_after();
-                        issue(s, j);
-                        tc::mma_commit(&c.empty[s]);
+                        if (lane == 0) {
+                            tc::tc_fence_after();
+                            issue(s, j);
+                            tc::mma_commit(&c.empty[s]);
+                        }
+                        __syncwarp();
                     } else {
                         set_abort(c, err);
                     }
@@ -168,8 +171,8 @@ __device__ __forceinline__ void mainloop(const Ctl &c, int S, int KC, int dep_ch
         }
     }
     tc::grid_dep_wait();  // every thread: later reads may touch the preceding grid's output
-    if (tid == 0) {
-        tc::mma_commit(c.done);  // arrives once every MMA issued above has completed
+    if (warp == 0) {
+        if (lane == 0) tc::mma_commit(c.done);  // arrives once every MMA issued above has completed
         for (int jj = n_waited; jj < n_issued; ++jj)  // copies still in flight after an abort
             tc::mbar_wait(&c.full[jj % S], (jj / S) & 1, kDrainLimit, nullptr);
     }
@@ -195,7 +198,16 @@ __device__ __forceinline__ void issue_kmajor(uint32_t tmem, uint32_t a_stage, ui
 }
 
 // ----------------------------------------------------------------------- helpers
-__device__ __forceinline__ float sigm(float z) { return 1.0f / (1.0f + __expf(-z)); }
+// Cell nonlinearities of the bf16 path: the hardware tanh approximation (PTX
+// tanh.approx.f32, relative error about 2^-11, below the bf16 rounding of h), and the
+// logistic sigmoid through the identity sigmoid(z) = 1/2 + tanh(z / 2) / 2.
+__device__ __forceinline__ float tanh_hw(float x)
+{
+    float y;
+    asm("tanh.approx.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+__device__ __forceinline__ float sigm(float z) { return fmaf(0.5f, tanh_hw(0.5f * z), 0.5f); }
 
 // L2-coherent read (bypasses L1) of state another CTA or an earlier launch wrote.
 __device__ __forceinline__ void ld8f_cg(const float *p, float (&v)[8])
@@ -312,10 +324,10 @@ fwd_step_tc(const __grid_constant__ CUtensorMap tm_x, StepArgs a, int t)
                 for (int e = 0; e < 8; ++e) {
                     const float ig = sigm(z[0][e] + __ldg(a.bias + u + e));
                     const float fg = sigm(z[1][e] + __ldg(a.bias + H + u + e));
-                    const float gg = tanhf(z[2][e] + __ldg(a.bias + 2 * H + u + e));
+                    const float gg = tanh_hw(z[2][e] + __ldg(a.bias + 2 * H + u + e));
                     const float og = sigm(z[3][e] + __ldg(a.bias + 3 * H + u + e));
                     cn[e] = fmaf(fg, cr[e], ig * gg);
-                    hn[e] = og * tanhf(cn[e]);
+                    hn[e] = og * tanh_hw(cn[e]);
                     gv[0][e] = ig; gv[1][e] = fg; gv[2][e] = gg; gv[3][e] = og;
                 }
                 const size_t w = ((size_t)(t + 1) * B + b) * H + u;
@@ -353,7 +365,7 @@ __device__ __forceinline__ void pointwise8(const StepArgs &a, int tp, int b, int
     float d[4][8], dcr[8];
 #pragma unroll
     for (int e = 0; e < 8; ++e) {
-        const float tcn = tanhf(cn[e]);
+        const float tcn = tanh_hw(cn[e]);
         const float dc = dcn[e] + dh[e] * og[e] * (1.0f - tcn * tcn);
         d[0][e] = dc * gg[e] * ig[e] * (1.0f - ig[e]);
         d[1][e] = dc * cr[e] * fg[e] * (1.0f - fg[e]);
@@ -594,6 +606,458 @@ __global__ void dw_reduce(int K, int G, int split, const float *__restrict__ par
     }
 }
 
+
+// ------------------------------------------------------------ persistent steps
+// One cooperative launch runs all T steps. Each CTA keeps one column tile (U hidden
+// units; its weight tile stays in shared memory when it fits) and a fixed set of row
+// tiles (rt = slot, slot + n_slot, ...), so every (instance, unit) has one owner for the
+// whole launch. The only inter-CTA dependency is within a row tile: step t reads the
+// hidden states (forward) or gate gradients (backward) that all column tiles of the row
+// tile wrote at the previous step, so each row tile has a counter of completed steps,
+// raised with release semantics after a tile's stores and waited on with acquire
+// semantics (a bounded spin) before the dependent chunks are loaded.
+struct PersistArgs {
+    StepArgs s;
+    int n_ct, n_rt, n_slot;  // column tiles; row tiles; CTAs per column tile
+    int w_res;               // 1: weight tile resident in shared memory
+    int32_t *cnt;            // [n_rt] completed steps per row tile, zero at launch
+};
+
+__host__ __device__ constexpr uint32_t psmem_bytes(int S, int NB, int KC, int w_res)
+{
+    return 1024 + (w_res ? (uint32_t)KC * NB * 128 : 0u) + (uint32_t)S * kAStage +
+           (w_res ? 0u : (uint32_t)S * NB * 128) + (2 * kMaxStages + 2) * 8 + 16;
+}
+
+struct PCtl {
+    Ctl c;
+    uint32_t w0;     // resident weight tile (w_res)
+    uint64_t *wbar;  // its bulk-copy barrier
+};
+
+__device__ __forceinline__ PCtl pcarve(uint8_t *raw, int S, int NB, int KC, int w_res)
+{
+    const uint32_t off = smem_u32(raw);
+    uint8_t *base = raw + ((1024u - (off & 1023u)) & 1023u);
+    PCtl p;
+    Ctl &c = p.c;
+    c.b_bytes = (uint32_t)NB * 128;
+    const uint32_t wbytes = w_res ? (uint32_t)KC * c.b_bytes : 0u;
+    p.w0 = smem_u32(base);
+    c.a0 = p.w0 + wbytes;
+    c.b0 = c.a0 + S * kAStage;
+    uint8_t *bars = base + wbytes + S * kAStage + (w_res ? 0u : S * c.b_bytes);
+    c.full = (uint64_t *)bars;
+    c.empty = c.full + kMaxStages;
+    c.done = c.empty + kMaxStages;
+    p.wbar = c.done + 1;
+    c.tmem_slot = (uint32_t *)(p.wbar + 1);
+    c.abort = (volatile int *)(c.tmem_slot + 1);
+    return p;
+}
+
+// Like mainloop, but the ring's chunk counter runs on across tiles (gbase = chunks
+// before this tile) and the done barrier completes once per tile (parity tile & 1).
+// dep() runs when chunk dep_chunk is about to be loaded.
+template <bool kGather, class Tma, class Gather, class Issue, class Dep>
+__device__ __forceinline__ void pmainloop(const Ctl &c, int S, int KC, uint32_t gbase, uint32_t tile, int dep_chunk,
+                                          long long limit, int32_t *err, Tma tma, Gather gather, Issue issue, Dep dep)
+{
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    int n_issued = 0, n_waited = 0;
+    if (kGather || warp == 0) {
+        for (int it = 0; it < KC + S - 1; ++it) {
+            if (it < KC) {
+                const uint32_t g = gbase + it;
+                const int s = (int)(g % S);
+                const uint32_t use = g / S;
+                if (use > 0 && !*c.abort)
+                    if (!tc::mbar_wait(&c.empty[s], (use - 1) & 1, limit, c.abort)) set_abort(c, err);
+                if (it == dep_chunk) dep();
+                if (!*c.abort) {
+                    if (tid == 0) tma(it, s, &c.full[s]);
+                    if (warp == 0) ++n_issued;
+                    if (kGather) gather(it, s);
+                }
+                if (kGather) tc::cp_async_commit();
+            }
+            const int j = it - (S - 1);
+            if (j >= 0) {
+                if (kGather) {
+                    tc::cp_async_wait_dyn(min(it, KC - 1) - j);
+                    tc::fence_proxy_async();
+                    __syncthreads();
+                }
+                if (warp == 0 && !*c.abort) {
+                    const uint32_t g = gbase + j;
+                    const int s = (int)(g % S);
+                    if (j < n_issued && tc::mbar_wait(&c.full[s], (g / S) & 1, limit, c.abort)) {
+                        ++n_waited;
+                        if (lane == 0) {
+                            tc::tc_fence_after();
+                            issue(s, j);
+                            tc::mma_commit(&c.empty[s]);
+                        }
+                        __syncwarp();
+                    } else {
+                        set_abort(c, err);
+                    }
+                }
+            }
+        }
+    }
+    if (warp == 0) {
+        if (lane == 0) tc::mma_commit(c.done);
+        for (int jj = n_waited; jj < n_issued; ++jj) {
+            const uint32_t g = gbase + jj;
+            tc::mbar_wait(&c.full[g % S], (g / S) & 1, kDrainLimit, nullptr);
+        }
+    }
+    if (kGather) tc::cp_async_wait<0>();
+    if (!tc::mbar_wait(c.done, tile & 1, limit, nullptr)) {
+        set_abort(c, err);
+        tc::mbar_wait(c.done, tile & 1, kDrainLimit, nullptr);
+    }
+    __syncthreads();
+    tc::tc_fence_after();
+}
+
+// Bounded spin until *cnt >= target (acquire). False on timeout or abort.
+__device__ __forceinline__ bool spin_until(const int32_t *cnt, int target, long long limit, volatile int *abort)
+{
+    if (tc::ld_acquire_gpu(cnt) >= target) return true;
+    const long long t0 = clock64();
+    while (true) {
+        if (clock64() - t0 >= limit) return false;
+        if (*abort) return false;
+        __nanosleep(32);
+        if (tc::ld_acquire_gpu(cnt) >= target) return true;
+    }
+}
+
+// After a tile's stores: make them visible to the async proxy and to other CTAs, then
+// count the step as done for this row tile.
+__device__ __forceinline__ void tile_done(int32_t *cnt)
+{
+    tc::fence_proxy_async_global();
+    tc::tc_fence_before();
+    __syncthreads();
+    if (threadIdx.x == 0) tc::red_release_gpu_add(cnt, 1);
+}
+
+template <int U>
+__global__ void __launch_bounds__(kThreads, 1) fwd_persist(const __grid_constant__ CUtensorMap tm_x, PersistArgs p)
+{
+    constexpr int NB = 4 * U, NC = U / 8;
+    constexpr uint32_t kCols = TmemCols<NB>::value;
+    const StepArgs &a = p.s;
+    extern __shared__ uint8_t smem_raw[];
+    __shared__ float s_bias[4 * U];
+    const PCtl pc = pcarve(smem_raw, a.S, NB, a.KC, p.w_res);
+    const Ctl &c = pc.c;
+    const int tid = threadIdx.x, warp = tid >> 5;
+    const int ct = blockIdx.x % p.n_ct, slot = blockIdx.x / p.n_ct;
+    const int B = a.B, H = a.H, kcx = a.kcx, KC = a.KC, S = a.S, kch = KC - kcx;
+    const long long limit = a.limit;
+    if (tid == 0) tc::mbar_init(pc.wbar, 1);
+    for (int i = tid; i < 4 * U; i += kThreads) {
+        const int g = i / U, u = ct * U + i % U;
+        s_bias[i] = u < H ? a.bias[g * H + u] : 0.0f;
+    }
+    const uint32_t tmem = prologue(c, S, kCols);
+    const uint8_t *wtile = a.wpack + (size_t)ct * KC * c.b_bytes;
+    if (p.w_res && tid == 0) {
+        tc::mbar_arrive_expect_tx(pc.wbar, KC * c.b_bytes);
+        tc::bulk_g2s(pc.w0, wtile, KC * c.b_bytes, pc.wbar);
+    }
+    const int lane = tid & 31;
+    bool w_ready = !p.w_res;  // warp 0
+    int n_issued = 0, n_waited = 0;  // warp 0: chunk copies issued / awaited (abort drain)
+    uint32_t gbase = 0, tiles = 0;
+    bool stop = false;
+
+    // warp 0 (lane 0 issues): load chunk it of the tile (x tile by TMA and/or streamed
+    // weight chunk); the stage's previous MMAs must have drained first
+    auto produce = [&](int t, int row0, int it, uint32_t g) {
+        const int s = (int)(g % S);
+        if (g >= (uint32_t)S && !tc::mbar_wait(&c.empty[s], (g / S - 1) & 1, limit, c.abort)) {
+            set_abort(c, a.err);
+            return;
+        }
+        if (lane == 0) {
+            tc::mbar_arrive_expect_tx(&c.full[s], (it < kcx ? kAStage : 0u) + (p.w_res ? 0u : c.b_bytes));
+            if (it < kcx) tc::tma_load_2d(c.a0 + s * kAStage, &tm_x, it * kChunk, t * B + row0, &c.full[s]);
+            if (!p.w_res) tc::bulk_g2s(c.b0 + s * c.b_bytes, wtile + (size_t)it * c.b_bytes, c.b_bytes, &c.full[s]);
+        }
+        __syncwarp();
+        ++n_issued;
+    };
+    // warp 0 (lane 0 issues): MMAs of chunk it once its copies landed
+    auto consume = [&](int it, uint32_t g) {
+        const int s = (int)(g % S);
+        if (!w_ready) {
+            if (!tc::mbar_wait(pc.wbar, 0, limit, c.abort)) {
+                set_abort(c, a.err);
+                return;
+            }
+            w_ready = true;
+        }
+        if (!tc::mbar_wait(&c.full[s], (g / S) & 1, limit, c.abort)) {
+            set_abort(c, a.err);
+            return;
+        }
+        ++n_waited;
+        if (lane == 0) {
+            tc::tc_fence_after();
+            issue_kmajor<NB>(tmem, c.a0 + s * kAStage, p.w_res ? pc.w0 + it * c.b_bytes : c.b0 + s * c.b_bytes, it);
+            tc::mma_commit(&c.empty[s]);
+        }
+        __syncwarp();
+    };
+
+    for (int t = 0; t < a.T && !stop; ++t) {
+        for (int rt = slot; rt < p.n_rt; rt += p.n_slot) {
+            const int row0 = rt * kRows, b = row0 + tid;
+            const bool row_ok = b < B;
+            const int src = row_ok ? a.top[(size_t)t * B + b] : 0;
+            const __nv_bfloat16 *hrow = a.hist_h + ((size_t)src * B + b) * H;
+            // this CTA wrote c_read itself (same units) at an earlier step, or it is c0
+            float cr[U];
+#pragma unroll
+            for (int cu = 0; cu < NC; ++cu) {
+                const int u = ct * U + cu * 8;
+                float v[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+                if (row_ok && u < H) ld8f_cg(a.hist_c + ((size_t)src * B + b) * H + u, v);
+#pragma unroll
+                for (int e = 0; e < 8; ++e) cr[cu * 8 + e] = v[e];
+            }
+            // x_t chunks: independent of other CTAs, multiplied before the row-tile wait
+            if (warp == 0 && !*c.abort) {
+                const int lag = min(S, kcx) - 1;
+                for (int it = 0; it < kcx + lag && !*c.abort; ++it) {
+                    if (it < kcx) produce(t, row0, it, gbase + it);
+                    if (it - lag >= 0 && !*c.abort) consume(it - lag, gbase + it - lag);
+                }
+                // h_read of step t was written at step t - 1 by every column tile of this row tile
+                if (t > 0 && !*c.abort && !spin_until(p.cnt + rt, p.n_ct * t, limit, c.abort)) set_abort(c, a.err);
+                __syncwarp();
+            }
+            __syncthreads();
+            // h_read chunks: gathered rows, S-deep ring, a CTA barrier per chunk consumed
+            const int lag = min(S, kch) - 1;
+            for (int ih = 0; ih < kch + lag; ++ih) {
+                if (ih < kch && !*c.abort) {
+                    const int it = kcx + ih;
+                    const uint32_t g = gbase + it;
+                    const int s = (int)(g % S);
+                    if (g >= (uint32_t)S && !tc::mbar_wait(&c.empty[s], (g / S - 1) & 1, limit, c.abort))
+                        set_abort(c, a.err);
+                    if (warp == 0 && !*c.abort) produce(t, row0, it, g);
+                    if (row_ok && !*c.abort) {
+                        const int k0 = ih * kChunk;
+                        const uint32_t dst = c.a0 + s * kAStage;
+#pragma unroll
+                        for (int q = 0; q < 8; ++q) {
+                            const int k = k0 + q * 8;
+                            tc::cp_async16(dst + sw128(tid, q), k < H ? (const void *)(hrow + k) : (const void *)hrow,
+                                           k < H ? 16u : 0u);
+                        }
+                    }
+                }
+                tc::cp_async_commit();
+                const int jh = ih - lag;
+                if (jh >= 0) {
+                    tc::cp_async_wait_dyn(min(ih, kch - 1) - jh);
+                    tc::fence_proxy_async();
+                    __syncthreads();
+                    if (warp == 0 && !*c.abort) consume(kcx + jh, gbase + kcx + jh);
+                }
+            }
+            if (tid == 0) tc::mma_commit(c.done);
+            if (!tc::mbar_wait(c.done, tiles & 1, limit, nullptr)) {
+                set_abort(c, a.err);
+                tc::mbar_wait(c.done, tiles & 1, kDrainLimit, nullptr);
+            }
+            gbase += KC;
+            ++tiles;
+            __syncthreads();
+            tc::tc_fence_after();
+            if (*c.abort) {
+                stop = true;
+                break;
+            }
+            const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
+#pragma unroll
+            for (int cu = 0; cu < NC; ++cu) {
+                float z[4][8];
+#pragma unroll
+                for (int g = 0; g < 4; ++g) tc::tmem_ld8(trow + g * U + cu * 8, z[g]);
+                const int u = ct * U + cu * 8;
+                if (row_ok && u < H) {
+                    float cn[8], hn[8], gv[4][8];
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) {
+                        const int j = cu * 8 + e;
+                        const float ig = sigm(z[0][e] + s_bias[j]);
+                        const float fg = sigm(z[1][e] + s_bias[U + j]);
+                        const float gg = tanh_hw(z[2][e] + s_bias[2 * U + j]);
+                        const float og = sigm(z[3][e] + s_bias[3 * U + j]);
+                        cn[e] = fmaf(fg, cr[j], ig * gg);
+                        hn[e] = og * tanh_hw(cn[e]);
+                        gv[0][e] = ig; gv[1][e] = fg; gv[2][e] = gg; gv[3][e] = og;
+                    }
+                    const size_t w = ((size_t)(t + 1) * B + b) * H + u;
+                    *(uint4 *)(a.hist_h + w) = pack8_bf16(hn);
+                    st8f(a.hist_c + w, cn);
+                    __half *gt = a.gates + ((size_t)t * B + b) * 4 * H + u;
+#pragma unroll
+                    for (int g = 0; g < 4; ++g) *(uint4 *)(gt + (size_t)g * H) = pack8_f16(gv[g]);
+                }
+            }
+            // count the step done for this row tile (release orders the stores above)
+            tc::tc_fence_before();
+            __syncthreads();
+            if (tid == 0) tc::red_release_gpu_add(p.cnt + rt, 1);
+        }
+    }
+    if (warp == 0) {
+        for (int jj = n_waited; jj < n_issued; ++jj) {  // copies still in flight after an abort
+            const uint32_t g = (uint32_t)jj;
+            tc::mbar_wait(&c.full[g % S], (g / S) & 1, kDrainLimit, nullptr);
+        }
+        if (!w_ready) tc::mbar_wait(pc.wbar, 0, kDrainLimit, nullptr);
+    }
+    tc::cp_async_wait<0>();
+    finish(c, tmem, kCols);
+}
+
+template <int U>
+__global__ void __launch_bounds__(kThreads, 1) bwd_persist(const __grid_constant__ CUtensorMap tm_g, PersistArgs p)
+{
+    constexpr int NB = U, NC = U / 8;
+    constexpr uint32_t kCols = TmemCols<NB>::value;
+    const StepArgs &a = p.s;
+    extern __shared__ uint8_t smem_raw[];
+    const PCtl pc = pcarve(smem_raw, a.S, NB, a.KC, p.w_res);
+    const Ctl &c = pc.c;
+    const int tid = threadIdx.x, warp = tid >> 5;
+    const int ct = blockIdx.x % p.n_ct, slot = blockIdx.x / p.n_ct;
+    const int B = a.B, H = a.H, KC = a.KC, S = a.S, T = a.T;
+    if (tid == 0) tc::mbar_init(pc.wbar, 1);
+    const uint32_t tmem = prologue(c, S, kCols);
+    const uint8_t *wtile = a.wpack + (size_t)ct * KC * c.b_bytes;
+    if (p.w_res && tid == 0) {
+        tc::mbar_arrive_expect_tx(pc.wbar, KC * c.b_bytes);
+        tc::bulk_g2s(pc.w0, wtile, KC * c.b_bytes, pc.wbar);
+    }
+    // the resident weight tile must land before the first MMA (warp 0, uniformly)
+    if (p.w_res && (tid >> 5) == 0 && !tc::mbar_wait(pc.wbar, 0, a.limit, c.abort)) {
+        set_abort(c, a.err);
+        tc::mbar_wait(pc.wbar, 0, kDrainLimit, nullptr);
+    }
+    uint32_t gbase = 0, tiles = 0;
+    bool stop = false;
+    for (int t = T - 1; t >= 0 && !stop; --t) {
+        const int need = T - 1 - t;  // steps every column tile finished before this one
+        for (int rt = slot; rt < p.n_rt; rt += p.n_slot) {
+            const int row0 = rt * kRows, b = row0 + tid;
+            const bool row_ok = b < B;
+            const int src = row_ok ? a.top[(size_t)t * B + b] : 0;
+            const int s1 = (row_ok && t >= 1) ? a.top[(size_t)(t - 1) * B + b] : 0;
+            // Prefetch every epilogue operand: the gradient history of this CTA's units is
+            // written only by this CTA; gates and cell states come from the forward.
+            float dh_src[U], dh_t[U], dc_t[U], cn[U], cr[U], dc_rd[U];
+            uint4 gq[NC][4];
+#pragma unroll
+            for (int cu = 0; cu < NC; ++cu) {
+                const int u = ct * U + cu * 8;
+                const bool ok = row_ok && u < H;
+                float v[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+                if (ok) ld8f_cg(a.dhist_h + ((size_t)src * B + b) * H + u, v);
+#pragma unroll
+                for (int e = 0; e < 8; ++e) dh_src[cu * 8 + e] = v[e];
+                if (ok && t >= 1) {
+                    const size_t wr = ((size_t)t * B + b) * H + u, rd = ((size_t)s1 * B + b) * H + u;
+                    float w1[8], w2[8], w3[8], w4[8], w5[8];
+                    ld8f_cg(a.dhist_h + wr, w1);
+                    ld8f_cg(a.dhist_c + wr, w2);
+                    ld8f_cg(a.hist_c + wr, w3);
+                    ld8f_cg(a.hist_c + rd, w4);
+                    ld8f_cg(a.dhist_c + rd, w5);
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) {
+                        dh_t[cu * 8 + e] = w1[e]; dc_t[cu * 8 + e] = w2[e]; cn[cu * 8 + e] = w3[e];
+                        cr[cu * 8 + e] = w4[e]; dc_rd[cu * 8 + e] = w5[e];
+                    }
+                    const __half *gt = a.gates + ((size_t)(t - 1) * B + b) * 4 * H + u;
+#pragma unroll
+                    for (int g = 0; g < 4; ++g) gq[cu][g] = *(const uint4 *)(gt + (size_t)g * H);
+                }
+            }
+            auto tma = [&](int it, int s, uint64_t *bar) {
+                tc::mbar_arrive_expect_tx(bar, kAStage + (p.w_res ? 0u : c.b_bytes));
+                tc::tma_load_2d(c.a0 + s * kAStage, &tm_g, it * kChunk, t * B + row0, bar);
+                if (!p.w_res) tc::bulk_g2s(c.b0 + s * c.b_bytes, wtile + (size_t)it * c.b_bytes, c.b_bytes, bar);
+            };
+            auto no_gather = [](int, int) {};
+            auto issue = [&](int s, int j) {
+                issue_kmajor<NB>(tmem, c.a0 + s * kAStage, p.w_res ? pc.w0 + j * c.b_bytes : c.b0 + s * c.b_bytes, j);
+            };
+            // dG_t was written at the previous step by every column tile (thread 0 only)
+            auto dep = [&]() {
+                if (need == 0) return;
+                if (!*c.abort && !spin_until(p.cnt + rt, p.n_ct * need, a.limit, c.abort)) set_abort(c, a.err);
+                tc::fence_proxy_async_global();
+            };
+            pmainloop<false>(c, S, KC, gbase, tiles, 0, a.limit, a.err, tma, no_gather, issue, dep);
+            gbase += KC;
+            ++tiles;
+            if (*c.abort) {
+                stop = true;
+                break;
+            }
+            const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
+#pragma unroll
+            for (int cu = 0; cu < NC; ++cu) {
+                float acc[8];
+                tc::tmem_ld8(trow + cu * 8, acc);
+                const int u = ct * U + cu * 8;
+                if (row_ok && u < H) {
+                    float v[8];
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) v[e] = dh_src[cu * 8 + e] + acc[e];
+                    st8f(a.dhist_h + ((size_t)src * B + b) * H + u, v);
+                    if (t >= 1) {
+                        float ig[8], fg[8], gg[8], og[8], d[4][8], dcr[8];
+                        unpack8_f16(gq[cu][0], ig);
+                        unpack8_f16(gq[cu][1], fg);
+                        unpack8_f16(gq[cu][2], gg);
+                        unpack8_f16(gq[cu][3], og);
+#pragma unroll
+                        for (int e = 0; e < 8; ++e) {
+                            const int j = cu * 8 + e;
+                            const float dh = src == t ? v[e] : dh_t[j];  // the state read at t is row t
+                            const float tcn = tanh_hw(cn[j]);
+                            const float dc = dc_t[j] + dh * og[e] * (1.0f - tcn * tcn);
+                            d[0][e] = dc * gg[e] * ig[e] * (1.0f - ig[e]);
+                            d[1][e] = dc * cr[j] * fg[e] * (1.0f - fg[e]);
+                            d[2][e] = dc * ig[e] * (1.0f - gg[e] * gg[e]);
+                            d[3][e] = dh * tcn * og[e] * (1.0f - og[e]);
+                            dcr[e] = dc_rd[j] + dc * fg[e];
+                        }
+                        __nv_bfloat16 *dg = a.dG + ((size_t)(t - 1) * B + b) * 4 * H + u;
+#pragma unroll
+                        for (int g = 0; g < 4; ++g) *(uint4 *)(dg + (size_t)g * H) = pack8_bf16(d[g]);
+                        st8f(a.dhist_c + ((size_t)s1 * B + b) * H + u, dcr);
+                    }
+                }
+            }
+            tile_done(p.cnt + rt);
+        }
+    }
+    finish(c, tmem, kCols);
+}
+
 // ------------------------------------------------------------------ packing
 // Forward operand: for column tile ct, rows n = g * U + j hold gate g of hidden unit
 // ct * U + j; each row is the matching column of W over the contraction
@@ -714,6 +1178,60 @@ int pick_stages(int KC, int NB, size_t ctas, int sms)
 
 int pick_dx_n(int I) { return I <= 32 ? 32 : I <= 64 ? 64 : I <= 128 ? 128 : 256; }
 
+template <typename Kern, typename... Args>
+cudaError_t launch_coop(Kern kernel, dim3 grid, size_t smem, cudaStream_t st, Args... args)
+{
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeCooperative;
+    at[0].val.cooperative = 1;
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, args...);
+}
+
+// Plans a persistent launch. For each shared-memory budget (one, two or three CTAs per
+// SM) the weight tile stays resident when it leaves room for a ring of at least two
+// stages, and the grid is sized from the occupancy of that footprint so every CTA is
+// co-resident; the budget needing the fewest row tiles per CTA per step wins (ties: the
+// deeper ring). Returns false if not even one CTA per column tile fits.
+template <typename Kern>
+bool plan_persist(Kern kernel, int KC, int NB, int n_ct, int n_rt, int sms, int *slot, int *wres, int *S)
+{
+    const uint32_t fixed = 1024 + (2 * kMaxStages + 2) * 8 + 16 + 1024 /* static */;
+    const uint32_t wbytes = (uint32_t)KC * NB * 128;
+    int best_rounds = 1 << 30;
+    bool found = false;
+    for (uint32_t budget : {200u * 1024, 100u * 1024, 66u * 1024}) {
+        const int wr = wbytes + 2 * kAStage + fixed <= budget;
+        const uint32_t stage = kAStage + (wr ? 0u : (uint32_t)NB * 128);
+        if (budget < fixed + (wr ? wbytes : 0u) + 2 * stage) continue;
+        const int st = std::max(2, std::min({(int)((budget - fixed - (wr ? wbytes : 0u)) / stage), KC, kMaxStages}));
+        int per_sm = 0;
+        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kernel, kThreads, psmem_bytes(st, NB, KC, wr)) !=
+            cudaSuccess) {
+            cudaGetLastError();
+            continue;
+        }
+        const long long resident = (long long)per_sm * sms;
+        if (resident < n_ct) continue;
+        const int sl = (int)std::min<long long>(n_rt, resident / n_ct);
+        const int rounds = (n_rt + sl - 1) / sl;
+        if (rounds < best_rounds) {
+            best_rounds = rounds;
+            *slot = sl;
+            *wres = wr;
+            *S = st;
+            found = true;
+        }
+    }
+    return found;
+}
+
 unsigned grid_for(const stacklstm *s, size_t n)
 {
     return (unsigned)std::max<size_t>(1, std::min<size_t>(ceil_div(n, 256), (size_t)s->num_sms * 16));
@@ -757,12 +1275,35 @@ cudaError_t bf16_prepare(stacklstm *s)
     s->dw_nt = (int)ceil_div(4 * H, 256);
     const size_t R = (size_t)T * B, RC = ceil_div(R, kChunk);
     s->dw_split = (int)std::max<size_t>(1, std::min<size_t>(sms / std::max(1, s->dw_mt * s->dw_nt), RC / 2));
+    const char *lim = getenv("STACKLSTM_WAIT_LIMIT_CYCLES");
+    s->wait_limit = lim ? atoll(lim) : 4000000000LL;
+    if ((e = allow_smem(fwd_persist<32>)) || (e = allow_smem(fwd_persist<16>)) || (e = allow_smem(fwd_persist<8>)) ||
+        (e = allow_smem(bwd_persist<16>)) || (e = allow_smem(fwd_step_tc<32>)) ||
+        (e = allow_smem(fwd_step_tc<16>)) || (e = allow_smem(fwd_step_tc<8>)) || (e = allow_smem(bwd_step_tc<32>)) ||
+        (e = allow_smem(bwd_step_tc<16>)) || (e = allow_smem(dx_tc<32>)) || (e = allow_smem(dx_tc<64>)) ||
+        (e = allow_smem(dx_tc<128>)) || (e = allow_smem(dx_tc<256>)) || (e = allow_smem(dw_tc)))
+        return e;
+
+    // persistent step kernels unless disabled (STACKLSTM_STEP_KERNELS=1 keeps one launch per step)
+    const char *per_step = getenv("STACKLSTM_STEP_KERNELS");
+    if (!(per_step && atoi(per_step) != 0)) {
+        const int nctf = (int)ceil_div(H, s->uf);
+        if (s->uf == 32)
+            s->pf = plan_persist(fwd_persist<32>, s->kcf, 128, nctf, rt, sms, &s->pf_slot, &s->pf_wres, &s->pf_S);
+        else if (s->uf == 16)
+            s->pf = plan_persist(fwd_persist<16>, s->kcf, 64, nctf, rt, sms, &s->pf_slot, &s->pf_wres, &s->pf_S);
+        else
+            s->pf = plan_persist(fwd_persist<8>, s->kcf, 32, nctf, rt, sms, &s->pf_slot, &s->pf_wres, &s->pf_S);
+        // the persistent backward keeps 16-unit tiles (its prefetched epilogue operands
+        // need the registers); the weight packing follows
+        s->pb = plan_persist(bwd_persist<16>, s->kcb, 16, (int)ceil_div(H, 16), rt, sms, &s->pb_slot, &s->pb_wres,
+                             &s->pb_S);
+        if (s->pb) s->ub = 16;
+    }
     s->sf = pick_stages(s->kcf, 4 * s->uf, ceil_div(H, s->uf) * (size_t)rt, sms);
     s->sb = pick_stages(s->kcb, s->ub, ceil_div(H, s->ub) * (size_t)rt, sms);
     s->sx = pick_stages(s->kcb, s->nx, s->nxt * ceil_div(R, kRows), sms);
     s->sw = pick_stages((int)ceil_div(RC, s->dw_split), 256, (size_t)s->dw_mt * s->dw_nt * s->dw_split, sms);
-    const char *lim = getenv("STACKLSTM_WAIT_LIMIT_CYCLES");
-    s->wait_limit = lim ? atoll(lim) : 4000000000LL;
 
     const size_t fwd_bytes = (size_t)ceil_div(H, s->uf) * s->kcf * 4 * s->uf * 128;
     const size_t bwd_bytes = (size_t)ceil_div(H, s->ub) * s->kcb * s->ub * 128;
@@ -781,15 +1322,14 @@ cudaError_t bf16_prepare(stacklstm *s)
     s->allocs.push_back(p); s->ones = p;
     const uint16_t one[8] = {0x3F80, 0, 0, 0, 0, 0, 0, 0};  // bf16 1.0 followed by zeros
     if ((e = cudaMemcpy(s->ones, one, 16, cudaMemcpyHostToDevice))) return e;
+    if (s->pf || s->pb) {
+        if ((e = cudaMalloc(&p, 2 * sizeof(int32_t) * rt))) return e;
+        s->allocs.push_back(p);
+        s->rowcnt = (int32_t *)p;
+    }
     // dG is workspace: its tensor maps are fixed for the handle's lifetime
     if ((e = make_map(s->tmaps[kMapG128], s->dG, R, 4 * (uint64_t)H, kRows))) return e;
     if ((e = make_map(s->tmaps[kMapG64], s->dG, R, 4 * (uint64_t)H, kChunk))) return e;
-
-    if ((e = allow_smem(fwd_step_tc<32>)) || (e = allow_smem(fwd_step_tc<16>)) || (e = allow_smem(fwd_step_tc<8>)) ||
-        (e = allow_smem(bwd_step_tc<32>)) || (e = allow_smem(bwd_step_tc<16>)) || (e = allow_smem(dx_tc<32>)) ||
-        (e = allow_smem(dx_tc<64>)) || (e = allow_smem(dx_tc<128>)) || (e = allow_smem(dx_tc<256>)) ||
-        (e = allow_smem(dw_tc)))
-        return e;
     return cudaSuccess;
 }
 
@@ -813,6 +1353,25 @@ cudaError_t bf16_forward(stacklstm *s, const __nv_bfloat16 *x, const __nv_bfloat
         W, H, 0, I, s->nx, s->kcb, s->nxt, (__nv_bfloat16 *)s->w_dx);
     s->launches += 3;
     if ((e = cudaGetLastError())) return e;
+    if (s->pf) {
+        PersistArgs p;
+        p.s = step_args(s, bias, s->w_fwd, s->kcx, s->kcf, s->pf_S);
+        p.n_ct = nctf; p.n_rt = (int)ceil_div(B, kRows); p.n_slot = s->pf_slot; p.w_res = s->pf_wres;
+        p.cnt = s->rowcnt;
+        if ((e = cudaMemsetAsync(p.cnt, 0, sizeof(int32_t) * p.n_rt, s->stream))) return e;
+        const dim3 g(nctf * p.n_slot);
+        const size_t sm = psmem_bytes(p.s.S, 4 * s->uf, s->kcf, p.w_res);
+        const CUtensorMap &tm = map(s, kMapX128);
+        if (s->uf == 32)
+            e = launch_coop(fwd_persist<32>, g, sm, s->stream, tm, p);
+        else if (s->uf == 16)
+            e = launch_coop(fwd_persist<16>, g, sm, s->stream, tm, p);
+        else
+            e = launch_coop(fwd_persist<8>, g, sm, s->stream, tm, p);
+        if (e) return e;
+        s->launches += 1;
+        return cudaGetLastError();
+    }
     const StepArgs a = step_args(s, bias, s->w_fwd, s->kcx, s->kcf, s->sf);
     const dim3 grid(nctf, ceil_div(B, kRows));
     const size_t smem = smem_bytes(s->sf, 4 * s->uf);
@@ -839,6 +1398,20 @@ cudaError_t bf16_backward_steps(stacklstm *s)
     pointwise_last<<<grid_for(s, (size_t)B * (H / 8)), 256, 0, s->stream>>>(a);
     s->launches += 1;
     if ((e = cudaGetLastError())) return e;
+    if (s->pb) {
+        PersistArgs p;
+        p.s = step_args(s, nullptr, s->w_bwd, 0, s->kcb, s->pb_S);
+        p.n_ct = (int)ceil_div(H, s->ub); p.n_rt = (int)ceil_div(B, kRows); p.n_slot = s->pb_slot;
+        p.w_res = s->pb_wres; p.cnt = s->rowcnt + p.n_rt;
+        if ((e = cudaMemsetAsync(p.cnt, 0, sizeof(int32_t) * p.n_rt, s->stream))) return e;
+        const dim3 g(p.n_ct * p.n_slot);
+        const size_t sm = psmem_bytes(p.s.S, s->ub, s->kcb, p.w_res);
+        const CUtensorMap &tm = map(s, kMapG128);
+        e = launch_coop(bwd_persist<16>, g, sm, s->stream, tm, p);
+        if (e) return e;
+        s->launches += 1;
+        return cudaGetLastError();
+    }
     const dim3 grid(ceil_div(H, s->ub), ceil_div(B, kRows));
     const size_t smem = smem_bytes(s->sb, s->ub);
     const CUtensorMap &tmg = map(s, kMapG128);

@@ -54,6 +54,12 @@ struct stacklstm {
     int kcx = 0, kcf = 0, kcb = 0;  // 64-wide contraction chunks: x part, forward total, backward
     int sf = 0, sb = 0, sx = 0, sw = 0;  // ring depths: forward, backward, dx, dW
     alignas(64) unsigned char tmaps[4][128] = {};  // TMA descriptors (bf16_path.cu)
+    // persistent step kernels (one launch for all T steps); 0 = per-step launches
+    int pf = 0, pb = 0;            // forward / backward run persistent
+    int pf_slot = 0, pb_slot = 0;  // CTAs per column tile (each takes every n_slot-th row tile)
+    int pf_wres = 0, pb_wres = 0;  // weight tile resident in shared memory
+    int pf_S = 0, pb_S = 0;        // ring depths of the persistent kernels
+    int32_t *rowcnt = nullptr;     // [2][row tiles] completed steps per row tile
     int nx = 0, nxt = 0;     // input gradient: columns per tile, number of column tiles
     int dw_mt = 0, dw_nt = 0, dw_split = 0;  // weight gradient: row tiles, column tiles, splits
     long long wait_limit = 0;  // clock cycles one bounded device-side wait may spin

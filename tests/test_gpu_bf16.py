@@ -132,3 +132,16 @@ def test_wait_timeout_is_reported_and_context_survives():
     finally:
         hd.destroy()
     compare(runner.run(w), oracle_all(w), "bf16")
+
+
+@pytest.mark.parametrize("T,B,I,H,seed", [(20, 200, 24, 40, 12), (9, 300, 136, 72, 13)])
+def test_per_step_kernels_match_oracle(T, B, I, H, seed):
+    """The one-launch-per-step kernels (used when a persistent grid cannot be
+    co-resident) stay parity-green too."""
+    w = case(T, B, I, H, seed, bias_scale=0.3, h0_scale=0.5, c0_scale=0.5, dy_scale=0.5)
+    os.environ["STACKLSTM_STEP_KERNELS"] = "1"
+    try:
+        got = runner.run(w)
+    finally:
+        del os.environ["STACKLSTM_STEP_KERNELS"]
+    compare(got, oracle_all(w), "bf16")
