@@ -165,6 +165,32 @@ const char *stacklstm_status_string(sl_status st);
  * next call on the handle. */
 const char *stacklstm_last_error(stacklstm_t s);
 
+/*
+ * stacklstm_pointers_noalloc -- the index prepass alone (pointer trajectory and read
+ * provenance of every instance), for callers that cannot allocate device memory: code
+ * running while a stream is being captured into a CUDA graph (a cudaMalloc there is not
+ * a stream operation and breaks or is refused by the capture), and services whose
+ * memory is fully reserved up front by a pooling allocator, where a library's own
+ * cudaMalloc fails or synchronizes the device mid-pipeline. It needs no handle and
+ * allocates nothing: it calls no cudaMalloc, cudaFree or allocating routine.
+ * The paper has no counterpart; it is a convenience of this library.
+ *   T, B     sizes; (T + 1) * B must not exceed 1,048,576, else SL_ERR_UNSUPPORTED
+ *   ops      [T, B] int8 device pointer, ops in {-1, 0, +1}
+ *   p_traj   [T + 1, B] int32 device output, as stacklstm_forward's p_traj
+ *   src      [T + 1, B] int32 device output, as stacklstm_forward's src
+ *   stream   cudaStream_t (NULL = legacy default stream); the call synchronizes it
+ * Returns SL_OK, SL_ERR_OP / SL_ERR_UNDERFLOW (bad op stream; indices are still written,
+ * bad ops run as holds), SL_ERR_ARG, SL_ERR_UNSUPPORTED or SL_ERR_CUDA.
+ * Scratch: an 8 MiB array in the library's device memory, held on every GPU that loads
+ * the library until the process exits. All calls share it, so calls that overlap on a
+ * GPU (other streams, other host threads) race; it keeps the previous call's contents
+ * and the call itself clears what must start at zero. The first call on a device looks
+ * up the array's device address (a one-time set-up): make that first call before any
+ * stream capture begins.
+ */
+sl_status stacklstm_pointers_noalloc(int T, int B, const int8_t *ops, int32_t *p_traj, int32_t *src,
+                                     void *stream);
+
 #ifdef __cplusplus
 }
 #endif

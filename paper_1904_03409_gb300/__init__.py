@@ -9,10 +9,10 @@ draws them.
 """
 from .binding import (SL_BF16, SL_FP32, StackLSTMError, StackLSTMHandle, load, stacklstm_backward,
                       stacklstm_create, stacklstm_destroy, stacklstm_forward, stacklstm_set_async,
-                      stacklstm_get_timing, stacklstm_set_stream, stacklstm_set_timing, stacklstm_status,
+                      stacklstm_get_timing, stacklstm_pointers_noalloc, stacklstm_set_stream, stacklstm_set_timing, stacklstm_status,
                       stacklstm_status_string)
 
 __all__ = ["SL_BF16", "SL_FP32", "StackLSTMError", "StackLSTMHandle", "load", "stacklstm_backward",
            "stacklstm_create", "stacklstm_destroy", "stacklstm_forward", "stacklstm_set_async",
-           "stacklstm_get_timing", "stacklstm_set_stream", "stacklstm_set_timing", "stacklstm_status",
+           "stacklstm_get_timing", "stacklstm_pointers_noalloc", "stacklstm_set_stream", "stacklstm_set_timing", "stacklstm_status",
            "stacklstm_status_string"]

@@ -57,6 +57,8 @@ def load(path: Optional[str] = None):
     lib.stacklstm_status_string.restype = ctypes.c_char_p
     lib.stacklstm_set_timing.argtypes = [vp, i]
     lib.stacklstm_get_timing.argtypes = [vp, vp, vp, i]
+    lib.stacklstm_pointers_noalloc.argtypes = [i, i, vp, vp, vp, vp]
+    lib.stacklstm_pointers_noalloc.restype = ctypes.c_int
     lib.stacklstm_last_error.argtypes = [vp]
     lib.stacklstm_last_error.restype = ctypes.c_char_p
     for fn in ("stacklstm_create", "stacklstm_forward", "stacklstm_backward", "stacklstm_set_stream",
@@ -167,6 +169,23 @@ def stacklstm_backward(hd: StackLSTMHandle, d_top_h=None, dy=None, dx=None, dh0=
             _ptr(dx, d, f, (T, B, I), "dx"), _ptr(dh0, d, f, (B, H), "dh0"), _ptr(dc0, d, f, (B, H), "dc0"),
             _ptr(dW, d, f, (I + H, 4 * H), "dW"), _ptr(dbias, d, f, (4 * H,), "dbias")]
     _check(hd.h, load().stacklstm_backward(hd.h, *args), "stacklstm_backward")
+
+
+def stacklstm_pointers_noalloc(ops, p_traj, src, stream=None):
+    """Pointer trajectory and read provenance of an op stream without a handle and without
+    any device allocation (see include/stacklstm.h). ops [T, B] int8, p_traj and src
+    [T+1, B] int32, all on the current CUDA device."""
+    import torch
+    T, B = ops.shape
+    d = ops.device.index
+    if stream is None:
+        stream = torch.cuda.current_stream(d)
+    raw = stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream)
+    args = [_ptr(ops, d, torch.int8, (T, B), "ops"), _ptr(p_traj, d, torch.int32, (T + 1, B), "p_traj"),
+            _ptr(src, d, torch.int32, (T + 1, B), "src")]
+    st = load().stacklstm_pointers_noalloc(T, B, *args, ctypes.c_void_p(raw))
+    if st != 0:
+        raise StackLSTMError(st, "stacklstm_pointers_noalloc")
 
 
 PHASES = ("prepass", "forward", "outputs", "backward", "dx", "dw")

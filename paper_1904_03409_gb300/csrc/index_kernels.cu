@@ -8,6 +8,7 @@
 //   slot_last   history index last written to each slot after the last step (-1: never).
 // Every step writes slot p_t + 1 (Algorithm 1), which in history terms is row t + 1.
 #include <algorithm>
+#include <mutex>
 
 #include "common.cuh"
 
@@ -154,4 +155,67 @@ cudaError_t launch_seed_grads(stacklstm *s, const float *d_top_h, const float *d
     return cudaGetLastError();
 }
 
+// ------------------------------------------------------------ allocation-free prepass
+// stacklstm_pointers_noalloc runs the prepass above for callers that cannot allocate
+// device memory. Its scratch (the slot-tag stack, the last-writer table and a status
+// word) is this file-scope array, which every GPU that loads the library holds until
+// the process exits. Every call shares it and it keeps the last call's contents.
+namespace {
+constexpr size_t kNoAllocMaxSlots = (size_t)1 << 20;  // (T + 1) * B at most
+constexpr int kNoAllocMaxDevices = 64;
+__device__ __align__(256) int32_t g_noalloc_scratch[2 * kNoAllocMaxSlots + 64];
+
+std::mutex g_noalloc_mu;
+int32_t *g_noalloc_addr[kNoAllocMaxDevices] = {};
+
+// Device address of the scratch on the current device (the host-side name of the array
+// is only a stand-in). Looked up once per device.
+cudaError_t noalloc_scratch(int32_t **out)
+{
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= kNoAllocMaxDevices) return cudaErrorInvalidDevice;
+    std::lock_guard<std::mutex> lock(g_noalloc_mu);
+    if (!g_noalloc_addr[dev]) {
+        void *p = nullptr;
+        if ((e = cudaGetSymbolAddress(&p, g_noalloc_scratch)) != cudaSuccess) return e;
+        g_noalloc_addr[dev] = (int32_t *)p;
+    }
+    *out = g_noalloc_addr[dev];
+    return cudaSuccess;
+}
+}  // namespace
 }  // namespace sl
+
+extern "C" sl_status stacklstm_pointers_noalloc(int T, int B, const int8_t *ops, int32_t *p_traj, int32_t *src,
+                                                void *stream)
+{
+    using namespace sl;
+    if (T < 1 || B < 1 || !ops || !p_traj || !src) return SL_ERR_ARG;
+    if ((size_t)(T + 1) * (size_t)B > kNoAllocMaxSlots) return SL_ERR_UNSUPPORTED;
+    cudaStream_t st = (cudaStream_t)stream;
+    int32_t *scratch = nullptr;
+    if (noalloc_scratch(&scratch) != cudaSuccess) {
+        cudaGetLastError();
+        return SL_ERR_CUDA;
+    }
+    int32_t *tags = scratch, *last = scratch + kNoAllocMaxSlots, *err = scratch + 2 * kNoAllocMaxSlots;
+    // the status word must start at zero; the kernel initialises every slot tag it reads
+    if (cudaMemsetAsync(err, 0, sizeof(int32_t), st) != cudaSuccess) {
+        cudaGetLastError();
+        return SL_ERR_CUDA;
+    }
+    prepass_kernel<false><<<ceil_div(B, kPrepassThreads), kPrepassThreads, 0, st>>>(T, B, ops, p_traj, src, last,
+                                                                                   tags, err);
+    int32_t h = 0;
+    cudaError_t e = cudaGetLastError();
+    if (e == cudaSuccess) e = cudaMemcpyAsync(&h, err, sizeof h, cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+    if (e != cudaSuccess) {
+        cudaGetLastError();
+        return SL_ERR_CUDA;
+    }
+    return (sl_status)h;
+}
+
