@@ -257,6 +257,7 @@ struct StepArgs {
     int kcx, KC, S;             // x-part chunks, all chunks, ring depth
     const int32_t *top;         // [T+1][B]
     __nv_bfloat16 *hist_h;      // [T+1][B][H]
+    __nv_bfloat16 *hr;          // [T+1][B][H] h operand of each step
     float *hist_c;              // [T+1][B][H]
     __half *gates;              // [T][B][4H]
     const float *bias;          // [4H]
@@ -267,12 +268,43 @@ struct StepArgs {
     int32_t *err;
 };
 
+
+// Forward epilogue for one tile row and 8 hidden units: the cell on pre-activations z
+// (gate blocks i, f, g, o), writes history row t + 1 (h', c'), the gates, and the h
+// operand of step t + 1: h' when step t pushed (the new state is the next top), else the
+// older top, a row this tile already wrote (hcopy).
+__device__ __forceinline__ void fwd_cell8(const StepArgs &a, int t, int b, int u, const float (&z)[4][8],
+                                          const float *bias_i, const float *bias_f, const float *bias_g,
+                                          const float *bias_o, const float *cr, bool next_is_new, uint4 hcopy)
+{
+    const int B = a.B, H = a.H;
+    float cn[8], hn[8], gv[4][8];
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+        const float ig = sigm(z[0][e] + bias_i[e]);
+        const float fg = sigm(z[1][e] + bias_f[e]);
+        const float gg = tanh_hw(z[2][e] + bias_g[e]);
+        const float og = sigm(z[3][e] + bias_o[e]);
+        cn[e] = fmaf(fg, cr[e], ig * gg);
+        hn[e] = og * tanh_hw(cn[e]);
+        gv[0][e] = ig; gv[1][e] = fg; gv[2][e] = gg; gv[3][e] = og;
+    }
+    const size_t w = ((size_t)(t + 1) * B + b) * H + u;
+    const uint4 hb = pack8_bf16(hn);
+    *(uint4 *)(a.hist_h + w) = hb;
+    *(uint4 *)(a.hr + w) = next_is_new ? hb : hcopy;
+    st8f(a.hist_c + w, cn);
+    __half *gt = a.gates + ((size_t)t * B + b) * 4 * H + u;
+#pragma unroll
+    for (int g = 0; g < 4; ++g) *(uint4 *)(gt + (size_t)g * H) = pack8_f16(gv[g]);
+}
+
 // ------------------------------------------------------------------ forward step
-// The contraction runs over [x_t padded to 64 ; h_read padded to 64]: chunks < kcx
-// come from x_t by TMA, the rest are gathered history rows.
+// The contraction runs over [x_t padded to 64 ; h_read padded to 64]: chunks < kcx are
+// TMA tiles of x_t, the rest TMA tiles of hr[t] (the h operand the previous step wrote).
 template <int U>
 __global__ void __launch_bounds__(kThreads, 1)
-fwd_step_tc(const __grid_constant__ CUtensorMap tm_x, StepArgs a, int t)
+fwd_step_tc(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtensorMap tm_h, StepArgs a, int t)
 {
     constexpr int NB = 4 * U;
     constexpr uint32_t kCols = TmemCols<NB>::value;
@@ -281,32 +313,26 @@ fwd_step_tc(const __grid_constant__ CUtensorMap tm_x, StepArgs a, int t)
     const int tid = threadIdx.x, warp = tid >> 5;
     const int ct = blockIdx.x, row0 = blockIdx.y * kRows;
     const int B = a.B, H = a.H, kcx = a.kcx;
-    // this thread's tile row and the history row it reads (the prepass ran before step 0)
     const int b = row0 + tid;
     const bool row_ok = b < B;
+    // the prepass ran before the first step: its indices are safe to read early
     const int src = row_ok ? a.top[(size_t)t * B + b] : 0;
-    const __nv_bfloat16 *hrow = a.hist_h + ((size_t)src * B + b) * H;
+    const int s_next = row_ok ? a.top[(size_t)(t + 1) * B + b] : 0;
     const uint32_t tmem = prologue(c, a.S, kCols);
 
     const uint8_t *bpack = a.wpack + (size_t)ct * a.KC * c.b_bytes;
     auto tma = [&](int it, int s, uint64_t *bar) {
-        tc::mbar_arrive_expect_tx(bar, c.b_bytes + (it < kcx ? kAStage : 0u));
-        if (it < kcx) tc::tma_load_2d(c.a0 + s * kAStage, &tm_x, it * kChunk, t * B + row0, bar);
+        tc::mbar_arrive_expect_tx(bar, c.b_bytes + kAStage);
+        if (it < kcx)
+            tc::tma_load_2d(c.a0 + s * kAStage, &tm_x, it * kChunk, t * B + row0, bar);
+        else
+            tc::tma_load_2d(c.a0 + s * kAStage, &tm_h, (it - kcx) * kChunk, t * B + row0, bar);
         tc::bulk_g2s(c.b0 + s * c.b_bytes, bpack + (size_t)it * c.b_bytes, c.b_bytes, bar);
     };
-    auto gather = [&](int it, int s) {
-        if (it < kcx || !row_ok) return;  // rows past B stay unread: their results are never stored
-        const int k0 = (it - kcx) * kChunk;
-        const uint32_t dst = c.a0 + s * kAStage;
-#pragma unroll
-        for (int q = 0; q < 8; ++q) {
-            const int k = k0 + q * 8;
-            tc::cp_async16(dst + sw128(tid, q), k < H ? (const void *)(hrow + k) : (const void *)hrow,
-                           k < H ? 16u : 0u);
-        }
-    };
+    auto no_gather = [](int, int) {};
     auto issue = [&](int s, int j) { issue_kmajor<NB>(tmem, c.a0 + s * kAStage, c.b0 + s * c.b_bytes, j); };
-    mainloop<true>(c, a.S, a.KC, kcx, a.limit, a.err, tma, gather, issue);
+    // chunks of hr[t] depend on the previous step
+    mainloop<false>(c, a.S, a.KC, kcx, a.limit, a.err, tma, no_gather, issue);
     tc::grid_dep_launch();
 
     if (!*c.abort) {
@@ -318,24 +344,20 @@ fwd_step_tc(const __grid_constant__ CUtensorMap tm_x, StepArgs a, int t)
             for (int g = 0; g < 4; ++g) tc::tmem_ld8(trow + g * U + cu * 8, z[g]);
             const int u = ct * U + cu * 8;
             if (row_ok && u < H) {
-                float cr[8], cn[8], hn[8], gv[4][8];
+                float cr[8];
                 ld8f_cg(a.hist_c + ((size_t)src * B + b) * H + u, cr);
+                const bool is_new = s_next == t + 1;
+                const uint4 hc = is_new ? make_uint4(0, 0, 0, 0)
+                                        : __ldcg((const uint4 *)(a.hr + ((size_t)s_next * B + b) * H + u));
+                float bi[8], bf[8], bg[8], bo[8];
 #pragma unroll
                 for (int e = 0; e < 8; ++e) {
-                    const float ig = sigm(z[0][e] + __ldg(a.bias + u + e));
-                    const float fg = sigm(z[1][e] + __ldg(a.bias + H + u + e));
-                    const float gg = tanh_hw(z[2][e] + __ldg(a.bias + 2 * H + u + e));
-                    const float og = sigm(z[3][e] + __ldg(a.bias + 3 * H + u + e));
-                    cn[e] = fmaf(fg, cr[e], ig * gg);
-                    hn[e] = og * tanh_hw(cn[e]);
-                    gv[0][e] = ig; gv[1][e] = fg; gv[2][e] = gg; gv[3][e] = og;
+                    bi[e] = __ldg(a.bias + u + e);
+                    bf[e] = __ldg(a.bias + H + u + e);
+                    bg[e] = __ldg(a.bias + 2 * H + u + e);
+                    bo[e] = __ldg(a.bias + 3 * H + u + e);
                 }
-                const size_t w = ((size_t)(t + 1) * B + b) * H + u;
-                *(uint4 *)(a.hist_h + w) = pack8_bf16(hn);
-                st8f(a.hist_c + w, cn);
-                __half *gt = a.gates + ((size_t)t * B + b) * 4 * H + u;
-#pragma unroll
-                for (int g = 0; g < 4; ++g) *(uint4 *)(gt + (size_t)g * H) = pack8_f16(gv[g]);
+                fwd_cell8(a, t, b, u, z, bi, bf, bg, bo, cr, is_new, hc);
             }
         }
     }
@@ -489,11 +511,12 @@ __global__ void __launch_bounds__(kThreads, 1) dx_tc(const __grid_constant__ CUt
 // dW_ext[m][n] = sum_r A[r][m] dG[r][n] over r = t * B + b, where A[r] = [x_t ; h_read ; 1]
 // (m = I + H is the all-ones row, which yields dbias). Both operands are read MN-major:
 // 64 consecutive r per chunk; each 64-wide MN block is 64 rows of 128 swizzled bytes.
-// dG blocks and x blocks (fully inside x) arrive by TMA; the other A blocks are gathered.
+// dG blocks, x blocks and h blocks (each fully inside x or inside h; the h operand of
+// step t is hr[t], rows t * B + b) arrive by TMA; a block straddling x and h, or holding
+// the ones row, is copied piece by piece.
 struct DwArgs {
     int B, I, H;
-    const __nv_bfloat16 *x, *hist_h, *ones;
-    const int32_t *top;
+    const __nv_bfloat16 *x, *hr, *ones;
     int R;
     int n_tiles_n, split, S;
     float *part;  // [split][mt * 128][nt * 256]
@@ -503,7 +526,8 @@ struct DwArgs {
 };
 
 __global__ void __launch_bounds__(kThreads, 1)
-dw_tc(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtensorMap tm_g, DwArgs a)
+dw_tc(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtensorMap tm_h,
+      const __grid_constant__ CUtensorMap tm_g, DwArgs a)
 {
     constexpr int NB = 256;
     constexpr uint32_t kCols = 256;
@@ -512,21 +536,26 @@ dw_tc(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtensor
     const Ctl c = carve(smem_raw, a.S, NB);
     const int tid = threadIdx.x, warp = tid >> 5;
     const int mt = blockIdx.x / a.n_tiles_n, nt = blockIdx.x % a.n_tiles_n, sp = blockIdx.y;
-    const int B = a.B, I = a.I, H = a.H;
+    const int I = a.I, H = a.H;
     const int RC = (a.R + kChunk - 1) / kChunk;
     const int c_lo = (int)((long long)RC * sp / a.split), c_hi = (int)((long long)RC * (sp + 1) / a.split);
     const int KC = c_hi - c_lo;
     const uint32_t tmem = prologue(c, a.S, kCols);
 
+    auto in_x = [&](int m0) { return m0 + 64 <= I; };
+    auto in_h = [&](int m0) { return m0 >= I && m0 + 64 <= I + H; };
     auto tma = [&](int it, int s, uint64_t *bar) {
         const int r0 = (c_lo + it) * kChunk;
         uint32_t bytes = 4 * kBlk;
-        for (int blk = 0; blk < 2; ++blk)
-            if (mt * kRows + blk * 64 + 64 <= I) bytes += kBlk;
+        for (int blk = 0; blk < 2; ++blk) {
+            const int m0 = mt * kRows + blk * 64;
+            if (in_x(m0) || in_h(m0)) bytes += kBlk;
+        }
         tc::mbar_arrive_expect_tx(bar, bytes);
         for (int blk = 0; blk < 2; ++blk) {
             const int m0 = mt * kRows + blk * 64;
-            if (m0 + 64 <= I) tc::tma_load_2d(c.a0 + s * kAStage + blk * kBlk, &tm_x, m0, r0, bar);
+            if (in_x(m0)) tc::tma_load_2d(c.a0 + s * kAStage + blk * kBlk, &tm_x, m0, r0, bar);
+            else if (in_h(m0)) tc::tma_load_2d(c.a0 + s * kAStage + blk * kBlk, &tm_h, m0 - I, r0, bar);
         }
         for (int nb = 0; nb < 4; ++nb)
             tc::tma_load_2d(c.b0 + s * c.b_bytes + nb * kBlk, &tm_g, nt * NB + nb * 64, r0, bar);
@@ -535,13 +564,11 @@ dw_tc(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtensor
     auto gather = [&](int it, int s) {
         const int rr = tid & 63, blk = tid >> 6;
         const int m0 = mt * kRows + blk * 64;
-        if (m0 + 64 <= I) return;  // arrives by TMA
+        if (in_x(m0) || in_h(m0)) return;  // arrives by TMA
         const int r = (c_lo + it) * kChunk + rr;
         const uint32_t dst = c.a0 + s * kAStage + blk * kBlk;
         const bool r_ok = r < a.R;
-        const int tb = r_ok ? r / B : 0;
-        const int bb = r - tb * B;
-        const __nv_bfloat16 *hrow = a.hist_h + ((size_t)(r_ok ? a.top[r] : 0) * B + bb) * H;
+        const __nv_bfloat16 *hrow = a.hr + (size_t)(r_ok ? r : 0) * H;
 #pragma unroll
         for (int q = 0; q < 8; ++q) {
             const int m = m0 + q * 8;
@@ -746,7 +773,8 @@ __device__ __forceinline__ void tile_done(int32_t *cnt)
 }
 
 template <int U>
-__global__ void __launch_bounds__(kThreads, 1) fwd_persist(const __grid_constant__ CUtensorMap tm_x, PersistArgs p)
+__global__ void __launch_bounds__(kThreads, 1)
+fwd_persist(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtensorMap tm_h, PersistArgs p)
 {
     constexpr int NB = 4 * U, NC = U / 8;
     constexpr uint32_t kCols = TmemCols<NB>::value;
@@ -755,9 +783,9 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_persist(const __grid_constant
     __shared__ float s_bias[4 * U];
     const PCtl pc = pcarve(smem_raw, a.S, NB, a.KC, p.w_res);
     const Ctl &c = pc.c;
-    const int tid = threadIdx.x, warp = tid >> 5;
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int ct = blockIdx.x % p.n_ct, slot = blockIdx.x / p.n_ct;
-    const int B = a.B, H = a.H, kcx = a.kcx, KC = a.KC, S = a.S, kch = KC - kcx;
+    const int B = a.B, H = a.H, kcx = a.kcx, KC = a.KC, S = a.S, T = a.T;
     const long long limit = a.limit;
     if (tid == 0) tc::mbar_init(pc.wbar, 1);
     for (int i = tid; i < 4 * U; i += kThreads) {
@@ -770,14 +798,10 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_persist(const __grid_constant
         tc::mbar_arrive_expect_tx(pc.wbar, KC * c.b_bytes);
         tc::bulk_g2s(pc.w0, wtile, KC * c.b_bytes, pc.wbar);
     }
-    const int lane = tid & 31;
-    bool w_ready = !p.w_res;  // warp 0
+    bool w_ready = !p.w_res;        // warp 0
     int n_issued = 0, n_waited = 0;  // warp 0: chunk copies issued / awaited (abort drain)
-    uint32_t gbase = 0, tiles = 0;
-    bool stop = false;
 
-    // warp 0 (lane 0 issues): load chunk it of the tile (x tile by TMA and/or streamed
-    // weight chunk); the stage's previous MMAs must have drained first
+    // warp 0, lane 0 issues: load chunk it of tile (t, row0) into ring slot g
     auto produce = [&](int t, int row0, int it, uint32_t g) {
         const int s = (int)(g % S);
         if (g >= (uint32_t)S && !tc::mbar_wait(&c.empty[s], (g / S - 1) & 1, limit, c.abort)) {
@@ -785,14 +809,17 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_persist(const __grid_constant
             return;
         }
         if (lane == 0) {
-            tc::mbar_arrive_expect_tx(&c.full[s], (it < kcx ? kAStage : 0u) + (p.w_res ? 0u : c.b_bytes));
-            if (it < kcx) tc::tma_load_2d(c.a0 + s * kAStage, &tm_x, it * kChunk, t * B + row0, &c.full[s]);
+            tc::mbar_arrive_expect_tx(&c.full[s], kAStage + (p.w_res ? 0u : c.b_bytes));
+            if (it < kcx)
+                tc::tma_load_2d(c.a0 + s * kAStage, &tm_x, it * kChunk, t * B + row0, &c.full[s]);
+            else
+                tc::tma_load_2d(c.a0 + s * kAStage, &tm_h, (it - kcx) * kChunk, t * B + row0, &c.full[s]);
             if (!p.w_res) tc::bulk_g2s(c.b0 + s * c.b_bytes, wtile + (size_t)it * c.b_bytes, c.b_bytes, &c.full[s]);
         }
         __syncwarp();
         ++n_issued;
     };
-    // warp 0 (lane 0 issues): MMAs of chunk it once its copies landed
+    // warp 0, lane 0 issues: MMAs of chunk it once its copies landed
     auto consume = [&](int it, uint32_t g) {
         const int s = (int)(g % S);
         if (!w_ready) {
@@ -815,65 +842,58 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_persist(const __grid_constant
         __syncwarp();
     };
 
-    for (int t = 0; t < a.T && !stop; ++t) {
+    // tiles in order: (t, rt) for t = 0.., rt = slot, slot + n_slot, ...
+    int x_pre = 0;  // warp 0: x chunks of the coming tile already issued
+    uint32_t gbase = 0, tiles = 0;
+    bool stop = false;
+    for (int t = 0; t < T && !stop; ++t) {
         for (int rt = slot; rt < p.n_rt; rt += p.n_slot) {
             const int row0 = rt * kRows, b = row0 + tid;
             const bool row_ok = b < B;
             const int src = row_ok ? a.top[(size_t)t * B + b] : 0;
-            const __nv_bfloat16 *hrow = a.hist_h + ((size_t)src * B + b) * H;
-            // this CTA wrote c_read itself (same units) at an earlier step, or it is c0
+            const int s_next = row_ok ? a.top[(size_t)(t + 1) * B + b] : 0;
+            const bool is_new = s_next == t + 1;
+            // operands this CTA wrote itself (same units): c_read, and the older top the
+            // next step reads when step t does not push
             float cr[U];
+            uint4 hc[NC];
 #pragma unroll
             for (int cu = 0; cu < NC; ++cu) {
                 const int u = ct * U + cu * 8;
                 float v[8] = {0, 0, 0, 0, 0, 0, 0, 0};
-                if (row_ok && u < H) ld8f_cg(a.hist_c + ((size_t)src * B + b) * H + u, v);
+                hc[cu] = make_uint4(0, 0, 0, 0);
+                if (row_ok && u < H) {
+                    ld8f_cg(a.hist_c + ((size_t)src * B + b) * H + u, v);
+                    if (!is_new) hc[cu] = __ldcg((const uint4 *)(a.hr + ((size_t)s_next * B + b) * H + u));
+                }
 #pragma unroll
                 for (int e = 0; e < 8; ++e) cr[cu * 8 + e] = v[e];
             }
-            // x_t chunks: independent of other CTAs, multiplied before the row-tile wait
             if (warp == 0 && !*c.abort) {
-                const int lag = min(S, kcx) - 1;
-                for (int it = 0; it < kcx + lag && !*c.abort; ++it) {
-                    if (it < kcx) produce(t, row0, it, gbase + it);
-                    if (it - lag >= 0 && !*c.abort) consume(it - lag, gbase + it - lag);
-                }
-                // h_read of step t was written at step t - 1 by every column tile of this row tile
-                if (t > 0 && !*c.abort && !spin_until(p.cnt + rt, p.n_ct * t, limit, c.abort)) set_abort(c, a.err);
-                __syncwarp();
-            }
-            __syncthreads();
-            // h_read chunks: gathered rows, S-deep ring, a CTA barrier per chunk consumed
-            const int lag = min(S, kch) - 1;
-            for (int ih = 0; ih < kch + lag; ++ih) {
-                if (ih < kch && !*c.abort) {
-                    const int it = kcx + ih;
-                    const uint32_t g = gbase + it;
-                    const int s = (int)(g % S);
-                    if (g >= (uint32_t)S && !tc::mbar_wait(&c.empty[s], (g / S - 1) & 1, limit, c.abort))
-                        set_abort(c, a.err);
-                    if (warp == 0 && !*c.abort) produce(t, row0, it, g);
-                    if (row_ok && !*c.abort) {
-                        const int k0 = ih * kChunk;
-                        const uint32_t dst = c.a0 + s * kAStage;
-#pragma unroll
-                        for (int q = 0; q < 8; ++q) {
-                            const int k = k0 + q * 8;
-                            tc::cp_async16(dst + sw128(tid, q), k < H ? (const void *)(hrow + k) : (const void *)hrow,
-                                           k < H ? 16u : 0u);
+                // one produce/consume loop: produce while the ring has room (chunk it needs
+                // chunk it - S consumed), else consume. Chunks below x_pre were prefetched.
+                // Before the first h chunk, wait until every column tile of this row tile
+                // finished step t - 1 (they wrote hr[t]).
+                bool dep_done = t == 0;
+                for (int it = x_pre, jc = 0; jc < KC && !*c.abort;) {
+                    if (it < KC && it - jc < S) {
+                        if (it >= kcx && !dep_done) {
+                            if (!spin_until(p.cnt + rt, p.n_ct * t, limit, c.abort)) set_abort(c, a.err);
+                            tc::fence_proxy_async_global();
+                            __syncwarp();
+                            dep_done = true;
+                            if (*c.abort) break;
                         }
+                        produce(t, row0, it, gbase + it);
+                        ++it;
+                    } else {
+                        consume(jc, gbase + jc);
+                        ++jc;
                     }
                 }
-                tc::cp_async_commit();
-                const int jh = ih - lag;
-                if (jh >= 0) {
-                    tc::cp_async_wait_dyn(min(ih, kch - 1) - jh);
-                    tc::fence_proxy_async();
-                    __syncthreads();
-                    if (warp == 0 && !*c.abort) consume(kcx + jh, gbase + kcx + jh);
-                }
+                if (lane == 0) tc::mma_commit(c.done);
+                __syncwarp();
             }
-            if (tid == 0) tc::mma_commit(c.done);
             if (!tc::mbar_wait(c.done, tiles & 1, limit, nullptr)) {
                 set_abort(c, a.err);
                 tc::mbar_wait(c.done, tiles & 1, kDrainLimit, nullptr);
@@ -886,6 +906,17 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_persist(const __grid_constant
                 stop = true;
                 break;
             }
+            // prefetch the next tile's x chunks (the whole ring is free: this tile's MMAs are done)
+            x_pre = 0;
+            {
+                int tn = t, rn = rt + p.n_slot;
+                if (rn >= p.n_rt) {
+                    rn = slot;
+                    ++tn;
+                }
+                if (tn < T && warp == 0)
+                    for (; x_pre < min(kcx, S) && !*c.abort; ++x_pre) produce(tn, rn * kRows, x_pre, gbase + x_pre);
+            }
             const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
 #pragma unroll
             for (int cu = 0; cu < NC; ++cu) {
@@ -893,41 +924,21 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_persist(const __grid_constant
 #pragma unroll
                 for (int g = 0; g < 4; ++g) tc::tmem_ld8(trow + g * U + cu * 8, z[g]);
                 const int u = ct * U + cu * 8;
-                if (row_ok && u < H) {
-                    float cn[8], hn[8], gv[4][8];
-#pragma unroll
-                    for (int e = 0; e < 8; ++e) {
-                        const int j = cu * 8 + e;
-                        const float ig = sigm(z[0][e] + s_bias[j]);
-                        const float fg = sigm(z[1][e] + s_bias[U + j]);
-                        const float gg = tanh_hw(z[2][e] + s_bias[2 * U + j]);
-                        const float og = sigm(z[3][e] + s_bias[3 * U + j]);
-                        cn[e] = fmaf(fg, cr[j], ig * gg);
-                        hn[e] = og * tanh_hw(cn[e]);
-                        gv[0][e] = ig; gv[1][e] = fg; gv[2][e] = gg; gv[3][e] = og;
-                    }
-                    const size_t w = ((size_t)(t + 1) * B + b) * H + u;
-                    *(uint4 *)(a.hist_h + w) = pack8_bf16(hn);
-                    st8f(a.hist_c + w, cn);
-                    __half *gt = a.gates + ((size_t)t * B + b) * 4 * H + u;
-#pragma unroll
-                    for (int g = 0; g < 4; ++g) *(uint4 *)(gt + (size_t)g * H) = pack8_f16(gv[g]);
-                }
+                if (row_ok && u < H)
+                    fwd_cell8(a, t, b, u, z, s_bias + cu * 8, s_bias + U + cu * 8, s_bias + 2 * U + cu * 8,
+                              s_bias + 3 * U + cu * 8, cr + cu * 8, is_new, hc[cu]);
             }
-            // count the step done for this row tile (release orders the stores above)
-            tc::tc_fence_before();
-            __syncthreads();
-            if (tid == 0) tc::red_release_gpu_add(p.cnt + rt, 1);
+            // hr[t + 1] is read by TMA: generic writes -> async proxy, then release the step
+            tile_done(p.cnt + rt);
         }
     }
     if (warp == 0) {
-        for (int jj = n_waited; jj < n_issued; ++jj) {  // copies still in flight after an abort
+        for (int jj = n_waited; jj < n_issued; ++jj) {  // copies still in flight after an abort or prefetch
             const uint32_t g = (uint32_t)jj;
             tc::mbar_wait(&c.full[g % S], (g / S) & 1, kDrainLimit, nullptr);
         }
         if (!w_ready) tc::mbar_wait(pc.wbar, 0, kDrainLimit, nullptr);
     }
-    tc::cp_async_wait<0>();
     finish(c, tmem, kCols);
 }
 
@@ -1139,7 +1150,7 @@ cudaError_t make_map(void *slot, const void *base, uint64_t rows, uint64_t cols,
     return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
 }
 
-enum { kMapX128 = 0, kMapX64 = 1, kMapG128 = 2, kMapG64 = 3 };
+enum { kMapX128 = 0, kMapX64 = 1, kMapG128 = 2, kMapG64 = 3, kMapH128 = 4, kMapH64 = 5 };
 const CUtensorMap &map(const stacklstm *s, int i) { return *(const CUtensorMap *)s->tmaps[i]; }
 
 template <typename Kern, typename... Args>
@@ -1243,7 +1254,8 @@ StepArgs step_args(stacklstm *s, const float *bias, const void *wpack, int kcx, 
     a.T = s->T; a.B = s->B; a.I = s->I; a.H = s->H;
     a.kcx = kcx; a.KC = KC; a.S = S;
     a.top = s->top;
-    a.hist_h = (__nv_bfloat16 *)s->hist_h; a.hist_c = s->hist_c; a.gates = (__half *)s->gates;
+    a.hist_h = (__nv_bfloat16 *)s->hist_h; a.hr = (__nv_bfloat16 *)s->hr;
+    a.hist_c = s->hist_c; a.gates = (__half *)s->gates;
     a.bias = bias; a.wpack = (const uint8_t *)wpack;
     a.dhist_h = s->dhist_h; a.dhist_c = s->dhist_c; a.dG = (__nv_bfloat16 *)s->dG;
     a.limit = s->wait_limit; a.err = s->err;
@@ -1330,6 +1342,9 @@ cudaError_t bf16_prepare(stacklstm *s)
     // dG is workspace: its tensor maps are fixed for the handle's lifetime
     if ((e = make_map(s->tmaps[kMapG128], s->dG, R, 4 * (uint64_t)H, kRows))) return e;
     if ((e = make_map(s->tmaps[kMapG64], s->dG, R, 4 * (uint64_t)H, kChunk))) return e;
+    const uint64_t R1 = (uint64_t)(T + 1) * B;
+    if ((e = make_map(s->tmaps[kMapH128], s->hr, R1, (uint64_t)H, kRows))) return e;
+    if ((e = make_map(s->tmaps[kMapH64], s->hr, R1, (uint64_t)H, kChunk))) return e;
     return cudaSuccess;
 }
 
@@ -1342,6 +1357,8 @@ cudaError_t bf16_forward(stacklstm *s, const __nv_bfloat16 *x, const __nv_bfloat
     if ((e = make_map(s->tmaps[kMapX128], x, (uint64_t)T * B, I, kRows))) return e;
     if ((e = make_map(s->tmaps[kMapX64], x, (uint64_t)T * B, I, kChunk))) return e;
     if ((e = cudaMemcpyAsync(s->hist_h, h0, sizeof(__nv_bfloat16) * B * H, cudaMemcpyDeviceToDevice, s->stream)))
+        return e;
+    if ((e = cudaMemcpyAsync(s->hr, h0, sizeof(__nv_bfloat16) * B * H, cudaMemcpyDeviceToDevice, s->stream)))
         return e;
     if ((e = cudaMemcpyAsync(s->hist_c, c0, sizeof(float) * B * H, cudaMemcpyDeviceToDevice, s->stream))) return e;
     const int nctf = (int)ceil_div(H, s->uf), nctb = (int)ceil_div(H, s->ub);
@@ -1361,13 +1378,13 @@ cudaError_t bf16_forward(stacklstm *s, const __nv_bfloat16 *x, const __nv_bfloat
         if ((e = cudaMemsetAsync(p.cnt, 0, sizeof(int32_t) * p.n_rt, s->stream))) return e;
         const dim3 g(nctf * p.n_slot);
         const size_t sm = psmem_bytes(p.s.S, 4 * s->uf, s->kcf, p.w_res);
-        const CUtensorMap &tm = map(s, kMapX128);
+        const CUtensorMap &tm = map(s, kMapX128), &th = map(s, kMapH128);
         if (s->uf == 32)
-            e = launch_coop(fwd_persist<32>, g, sm, s->stream, tm, p);
+            e = launch_coop(fwd_persist<32>, g, sm, s->stream, tm, th, p);
         else if (s->uf == 16)
-            e = launch_coop(fwd_persist<16>, g, sm, s->stream, tm, p);
+            e = launch_coop(fwd_persist<16>, g, sm, s->stream, tm, th, p);
         else
-            e = launch_coop(fwd_persist<8>, g, sm, s->stream, tm, p);
+            e = launch_coop(fwd_persist<8>, g, sm, s->stream, tm, th, p);
         if (e) return e;
         s->launches += 1;
         return cudaGetLastError();
@@ -1375,15 +1392,15 @@ cudaError_t bf16_forward(stacklstm *s, const __nv_bfloat16 *x, const __nv_bfloat
     const StepArgs a = step_args(s, bias, s->w_fwd, s->kcx, s->kcf, s->sf);
     const dim3 grid(nctf, ceil_div(B, kRows));
     const size_t smem = smem_bytes(s->sf, 4 * s->uf);
-    const CUtensorMap &tmx = map(s, kMapX128);
+    const CUtensorMap &tmx = map(s, kMapX128), &tmh = map(s, kMapH128);
     for (int t = 0; t < T; ++t) {
         const bool pdl = t > 0;
         if (s->uf == 32)
-            e = launch(fwd_step_tc<32>, grid, smem, s->stream, pdl, tmx, a, t);
+            e = launch(fwd_step_tc<32>, grid, smem, s->stream, pdl, tmx, tmh, a, t);
         else if (s->uf == 16)
-            e = launch(fwd_step_tc<16>, grid, smem, s->stream, pdl, tmx, a, t);
+            e = launch(fwd_step_tc<16>, grid, smem, s->stream, pdl, tmx, tmh, a, t);
         else
-            e = launch(fwd_step_tc<8>, grid, smem, s->stream, pdl, tmx, a, t);
+            e = launch(fwd_step_tc<8>, grid, smem, s->stream, pdl, tmx, tmh, a, t);
         if (e) return e;
         s->launches += 1;
     }
@@ -1455,13 +1472,13 @@ cudaError_t bf16_dw(stacklstm *s, float *dW, float *dbias)
     const int T = s->T, B = s->B, I = s->I, H = s->H;
     DwArgs w;
     w.B = B; w.I = I; w.H = H;
-    w.x = (const __nv_bfloat16 *)s->x_saved; w.hist_h = (const __nv_bfloat16 *)s->hist_h;
-    w.ones = (const __nv_bfloat16 *)s->ones; w.top = s->top;
+    w.x = (const __nv_bfloat16 *)s->x_saved; w.hr = (const __nv_bfloat16 *)s->hr;
+    w.ones = (const __nv_bfloat16 *)s->ones;
     w.R = T * B; w.n_tiles_n = s->dw_nt; w.split = s->dw_split; w.S = s->sw; w.part = s->dw_part;
     w.ld_part = (size_t)s->dw_nt * 256; w.rows_part = (size_t)s->dw_mt * kRows;
     w.limit = s->wait_limit; w.err = s->err;
     cudaError_t e = launch(dw_tc, dim3(s->dw_mt * s->dw_nt, s->dw_split), smem_bytes(s->sw, 256), s->stream, false,
-                           map(s, kMapX64), map(s, kMapG64), w);
+                           map(s, kMapX64), map(s, kMapH64), map(s, kMapG64), w);
     if (e) return e;
     dw_reduce<<<grid_for(s, (size_t)(I + H + 1) * 4 * H), 256, 0, s->stream>>>(
         I + H, 4 * H, s->dw_split, s->dw_part, w.rows_part, w.ld_part, dW, dbias);

@@ -31,6 +31,7 @@ struct stacklstm {
 
     // forward state, write-once history: index 0 = initial state, t+1 = written at step t
     void *hist_h = nullptr;  // [T+1][B][H] dtype
+    void *hr = nullptr;      // bf16: [T+1][B][H] h operand of each step, hr[t][b] = hist_h[top[t][b]][b]
     float *hist_c = nullptr;  // [T+1][B][H]
     void *gates = nullptr;    // [T][B][4H] activated i,f,g,o (fp32 path: float, bf16: half)
     void *a_rm = nullptr;     // [T][B][I+H] the contraction operand [x_t ; h_read] (dtype)
@@ -53,7 +54,7 @@ struct stacklstm {
     int uf = 0, ub = 0;      // hidden units per CTA tile: forward, backward
     int kcx = 0, kcf = 0, kcb = 0;  // 64-wide contraction chunks: x part, forward total, backward
     int sf = 0, sb = 0, sx = 0, sw = 0;  // ring depths: forward, backward, dx, dW
-    alignas(64) unsigned char tmaps[4][128] = {};  // TMA descriptors (bf16_path.cu)
+    alignas(64) unsigned char tmaps[6][128] = {};  // TMA descriptors (bf16_path.cu)
     // persistent step kernels (one launch for all T steps); 0 = per-step launches
     int pf = 0, pb = 0;            // forward / backward run persistent
     int pf_slot = 0, pb_slot = 0;  // CTAs per column tile (each takes every n_slot-th row tile)
