@@ -161,6 +161,11 @@ sl_status stacklstm_destroy(stacklstm_t s);
 /* Static, human-readable name of a status code. */
 const char *stacklstm_status_string(sl_status st);
 
+/* One-line description of how the handle runs: dtype path, kernels (persistent or one
+ * launch per step), tile sizes, cluster sizes, ring depths. Valid until the handle is
+ * destroyed. */
+const char *stacklstm_plan(stacklstm_t s);
+
 /* One-line message for the last failure on the handle ("" if none). Valid until the
  * next call on the handle. */
 const char *stacklstm_last_error(stacklstm_t s);

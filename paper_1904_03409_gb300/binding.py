@@ -59,6 +59,8 @@ def load(path: Optional[str] = None):
     lib.stacklstm_get_timing.argtypes = [vp, vp, vp, i]
     lib.stacklstm_pointers_noalloc.argtypes = [i, i, vp, vp, vp, vp]
     lib.stacklstm_pointers_noalloc.restype = ctypes.c_int
+    lib.stacklstm_plan.argtypes = [vp]
+    lib.stacklstm_plan.restype = ctypes.c_char_p
     lib.stacklstm_last_error.argtypes = [vp]
     lib.stacklstm_last_error.restype = ctypes.c_char_p
     for fn in ("stacklstm_create", "stacklstm_forward", "stacklstm_backward", "stacklstm_set_stream",
@@ -203,6 +205,11 @@ def stacklstm_get_timing(hd: StackLSTMHandle) -> dict:
     ln = (ctypes.c_longlong * n)()
     _check(hd.h, load().stacklstm_get_timing(hd.h, ms, ln, n), "stacklstm_get_timing")
     return {p: (ms[i], ln[i]) for i, p in enumerate(PHASES)}
+
+
+def stacklstm_plan(hd: StackLSTMHandle) -> str:
+    """How the handle runs (kernels, tiles, clusters, ring depths)."""
+    return load().stacklstm_plan(hd.h).decode()
 
 
 def stacklstm_destroy(hd: StackLSTMHandle):

@@ -166,6 +166,8 @@ const char *stacklstm_status_string(sl_status st)
 
 const char *stacklstm_last_error(stacklstm_t s) { return s ? s->last_error.c_str() : "null handle"; }
 
+const char *stacklstm_plan(stacklstm_t s) { return s ? s->plan.c_str() : "null handle"; }
+
 sl_status stacklstm_create(stacklstm_t *out, int T, int B, int I, int H, sl_dtype dtype, int device,
                            void *stream)
 {
@@ -208,6 +210,7 @@ sl_status stacklstm_create(stacklstm_t *out, int T, int B, int I, int H, sl_dtyp
         delete s;
         return SL_ERR_OOM;
     }
+    s->plan = dtype == SL_BF16 ? sl::bf16_describe(s) : "fp32 CUDA cores; one launch per step";
     *out = s;
     return SL_OK;
 }

@@ -26,6 +26,7 @@
 // split-K contraction whose partial sums are reduced in a fixed order).
 #include <cuda.h>
 #include <cudaTypedefs.h>
+#include <stdio.h>
 #include <stdlib.h>
 
 #include <algorithm>
@@ -643,10 +644,18 @@ __global__ void dw_reduce(int K, int G, int split, const float *__restrict__ par
 // tile wrote at the previous step, so each row tile has a counter of completed steps,
 // raised with release semantics after a tile's stores and waited on with acquire
 // semantics (a bounded spin) before the dependent chunks are loaded.
+//
+// With cl > 1, the cl CTAs of a thread-block cluster share their row tiles and hold cl
+// consecutive column tiles, so they need the same A operand: chunk it is loaded once, by
+// cluster rank it % cl, and multicast into the same ring stage of every CTA of the
+// cluster. Each CTA arms its own `full` barrier with the chunk's bytes; `empty` counts cl
+// arrivals because every CTA commits its MMA completions to the `empty` barrier of all
+// CTAs of the cluster, so a stage is refilled only after every consumer drained it.
 struct PersistArgs {
     StepArgs s;
-    int n_ct, n_rt, n_slot;  // column tiles; row tiles; CTAs per column tile
+    int n_ct, n_rt, n_slot;  // column tiles (a multiple of cl); row tiles; CTAs per column tile
     int w_res;               // 1: weight tile resident in shared memory
+    int cl;                  // cluster size along the column tiles (1: no multicast)
     int32_t *cnt;            // [n_rt] completed steps per row tile, zero at launch
 };
 
@@ -683,70 +692,49 @@ __device__ __forceinline__ PCtl pcarve(uint8_t *raw, int S, int NB, int KC, int 
     return p;
 }
 
-// Like mainloop, but the ring's chunk counter runs on across tiles (gbase = chunks
-// before this tile) and the done barrier completes once per tile (parity tile & 1).
-// dep() runs when chunk dep_chunk is about to be loaded.
-template <bool kGather, class Tma, class Gather, class Issue, class Dep>
-__device__ __forceinline__ void pmainloop(const Ctl &c, int S, int KC, uint32_t gbase, uint32_t tile, int dep_chunk,
-                                          long long limit, int32_t *err, Tma tma, Gather gather, Issue issue, Dep dep)
+// Barrier init (empty counts one arrival per CTA of the cluster), tensor-memory
+// allocation, then a cluster barrier so no multicast reaches an uninitialised barrier.
+__device__ __forceinline__ uint32_t pprologue(const PCtl &pc, int S, uint32_t ncols, int cl)
 {
-    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    int n_issued = 0, n_waited = 0;
-    if (kGather || warp == 0) {
-        for (int it = 0; it < KC + S - 1; ++it) {
-            if (it < KC) {
-                const uint32_t g = gbase + it;
-                const int s = (int)(g % S);
-                const uint32_t use = g / S;
-                if (use > 0 && !*c.abort)
-                    if (!tc::mbar_wait(&c.empty[s], (use - 1) & 1, limit, c.abort)) set_abort(c, err);
-                if (it == dep_chunk) dep();
-                if (!*c.abort) {
-                    if (tid == 0) tma(it, s, &c.full[s]);
-                    if (warp == 0) ++n_issued;
-                    if (kGather) gather(it, s);
-                }
-                if (kGather) tc::cp_async_commit();
-            }
-            const int j = it - (S - 1);
-            if (j >= 0) {
-                if (kGather) {
-                    tc::cp_async_wait_dyn(min(it, KC - 1) - j);
-                    tc::fence_proxy_async();
-                    __syncthreads();
-                }
-                if (warp == 0 && !*c.abort) {
-                    const uint32_t g = gbase + j;
-                    const int s = (int)(g % S);
-                    if (j < n_issued && tc::mbar_wait(&c.full[s], (g / S) & 1, limit, c.abort)) {
-                        ++n_waited;
-                        if (lane == 0) {
-                            tc::tc_fence_after();
-                            issue(s, j);
-                            tc::mma_commit(&c.empty[s]);
-                        }
-                        __syncwarp();
-                    } else {
-                        set_abort(c, err);
-                    }
-                }
-            }
+    const Ctl &c = pc.c;
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < S; ++s) {
+            tc::mbar_init(&c.full[s], 1);
+            tc::mbar_init(&c.empty[s], (uint32_t)cl);
         }
+        tc::mbar_init(c.done, 1);
+        tc::mbar_init(pc.wbar, 1);
+        *c.abort = 0;
+        tc::fence_mbar_init();
     }
-    if (warp == 0) {
-        if (lane == 0) tc::mma_commit(c.done);
-        for (int jj = n_waited; jj < n_issued; ++jj) {
-            const uint32_t g = gbase + jj;
-            tc::mbar_wait(&c.full[g % S], (g / S) & 1, kDrainLimit, nullptr);
-        }
-    }
-    if (kGather) tc::cp_async_wait<0>();
-    if (!tc::mbar_wait(c.done, tile & 1, limit, nullptr)) {
-        set_abort(c, err);
-        tc::mbar_wait(c.done, tile & 1, kDrainLimit, nullptr);
-    }
+    if (threadIdx.x < 32) tc::tmem_alloc(c.tmem_slot, ncols);
+    tc::tc_fence_before();
     __syncthreads();
+    if (cl > 1) tc::cluster_sync();
     tc::tc_fence_after();
+    return *c.tmem_slot;
+}
+
+// One MMA chunk's completion goes to the stage's empty barrier of every CTA of the cluster.
+__device__ __forceinline__ void commit_empty(uint64_t *bar, int cl)
+{
+    if (cl > 1)
+        tc::mma_commit_mc(bar, (uint16_t)((1u << cl) - 1));
+    else
+        tc::mma_commit(bar);
+}
+
+// Loads chunk `it` of a tile into ring slot g: arms this CTA's full barrier with `bytes`
+// (A chunk plus this CTA's streamed weight chunk), and, if this CTA is the chunk's issuer,
+// loads the A box into every CTA of the cluster. Called by lane 0 of warp 0.
+__device__ __forceinline__ void load_a_chunk(const Ctl &c, int s, uint32_t bytes, const CUtensorMap *tm, int c0,
+                                             int c1, int it, int cl, uint32_t rank)
+{
+    tc::mbar_arrive_expect_tx(&c.full[s], bytes);
+    if (cl == 1)
+        tc::tma_load_2d(c.a0 + s * kAStage, tm, c0, c1, &c.full[s]);
+    else if ((uint32_t)(it % cl) == rank)
+        tc::tma_load_2d_mc(c.a0 + s * kAStage, tm, c0, c1, &c.full[s], (uint16_t)((1u << cl) - 1));
 }
 
 // Bounded spin until *cnt >= target (acquire). False on timeout or abort.
@@ -762,8 +750,8 @@ __device__ __forceinline__ bool spin_until(const int32_t *cnt, int target, long 
     }
 }
 
-// After a tile's stores: make them visible to the async proxy and to other CTAs, then
-// count the step as done for this row tile.
+// After a tile's stores: make them visible to the async proxy (TMA readers) and to other
+// CTAs, then count the step done for this row tile.
 __device__ __forceinline__ void tile_done(int32_t *cnt)
 {
     tc::fence_proxy_async_global();
@@ -784,24 +772,25 @@ fwd_persist(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CU
     const PCtl pc = pcarve(smem_raw, a.S, NB, a.KC, p.w_res);
     const Ctl &c = pc.c;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int ct = blockIdx.x % p.n_ct, slot = blockIdx.x / p.n_ct;
+    const int ct = blockIdx.x % p.n_ct, slot = blockIdx.x / p.n_ct, cl = p.cl;
+    const uint32_t rank = cl > 1 ? tc::cluster_rank() : 0;
     const int B = a.B, H = a.H, kcx = a.kcx, KC = a.KC, S = a.S, T = a.T;
     const long long limit = a.limit;
-    if (tid == 0) tc::mbar_init(pc.wbar, 1);
     for (int i = tid; i < 4 * U; i += kThreads) {
         const int g = i / U, u = ct * U + i % U;
         s_bias[i] = u < H ? a.bias[g * H + u] : 0.0f;
     }
-    const uint32_t tmem = prologue(c, S, kCols);
+    const uint32_t tmem = pprologue(pc, S, kCols, cl);
     const uint8_t *wtile = a.wpack + (size_t)ct * KC * c.b_bytes;
     if (p.w_res && tid == 0) {
         tc::mbar_arrive_expect_tx(pc.wbar, KC * c.b_bytes);
         tc::bulk_g2s(pc.w0, wtile, KC * c.b_bytes, pc.wbar);
     }
     bool w_ready = !p.w_res;        // warp 0
-    int n_issued = 0, n_waited = 0;  // warp 0: chunk copies issued / awaited (abort drain)
+    int n_issued = 0, n_waited = 0;  // warp 0: chunks armed / consumed (abort drain)
 
-    // warp 0, lane 0 issues: load chunk it of tile (t, row0) into ring slot g
+    // warp 0 (lane 0 issues): chunk it of tile (t, row0) into ring slot g, once every
+    // CTA of the cluster drained the chunk that used the stage before
     auto produce = [&](int t, int row0, int it, uint32_t g) {
         const int s = (int)(g % S);
         if (g >= (uint32_t)S && !tc::mbar_wait(&c.empty[s], (g / S - 1) & 1, limit, c.abort)) {
@@ -809,17 +798,17 @@ fwd_persist(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CU
             return;
         }
         if (lane == 0) {
-            tc::mbar_arrive_expect_tx(&c.full[s], kAStage + (p.w_res ? 0u : c.b_bytes));
+            const uint32_t bytes = kAStage + (p.w_res ? 0u : c.b_bytes);
             if (it < kcx)
-                tc::tma_load_2d(c.a0 + s * kAStage, &tm_x, it * kChunk, t * B + row0, &c.full[s]);
+                load_a_chunk(c, s, bytes, &tm_x, it * kChunk, t * B + row0, it, cl, rank);
             else
-                tc::tma_load_2d(c.a0 + s * kAStage, &tm_h, (it - kcx) * kChunk, t * B + row0, &c.full[s]);
+                load_a_chunk(c, s, bytes, &tm_h, (it - kcx) * kChunk, t * B + row0, it, cl, rank);
             if (!p.w_res) tc::bulk_g2s(c.b0 + s * c.b_bytes, wtile + (size_t)it * c.b_bytes, c.b_bytes, &c.full[s]);
         }
         __syncwarp();
         ++n_issued;
     };
-    // warp 0, lane 0 issues: MMAs of chunk it once its copies landed
+    // warp 0 (lane 0 issues): MMAs of chunk it once its bytes landed
     auto consume = [&](int it, uint32_t g) {
         const int s = (int)(g % S);
         if (!w_ready) {
@@ -837,7 +826,7 @@ fwd_persist(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CU
         if (lane == 0) {
             tc::tc_fence_after();
             issue_kmajor<NB>(tmem, c.a0 + s * kAStage, p.w_res ? pc.w0 + it * c.b_bytes : c.b0 + s * c.b_bytes, it);
-            tc::mma_commit(&c.empty[s]);
+            commit_empty(&c.empty[s], cl);
         }
         __syncwarp();
     };
@@ -933,12 +922,13 @@ fwd_persist(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CU
         }
     }
     if (warp == 0) {
-        for (int jj = n_waited; jj < n_issued; ++jj) {  // copies still in flight after an abort or prefetch
+        for (int jj = n_waited; jj < n_issued; ++jj) {  // chunks armed but not consumed (abort)
             const uint32_t g = (uint32_t)jj;
             tc::mbar_wait(&c.full[g % S], (g / S) & 1, kDrainLimit, nullptr);
         }
         if (!w_ready) tc::mbar_wait(pc.wbar, 0, kDrainLimit, nullptr);
     }
+    if (cl > 1) tc::cluster_sync();  // nobody leaves while a peer may still multicast into it
     finish(c, tmem, kCols);
 }
 
@@ -951,21 +941,23 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_persist(const __grid_constant
     extern __shared__ uint8_t smem_raw[];
     const PCtl pc = pcarve(smem_raw, a.S, NB, a.KC, p.w_res);
     const Ctl &c = pc.c;
-    const int tid = threadIdx.x, warp = tid >> 5;
-    const int ct = blockIdx.x % p.n_ct, slot = blockIdx.x / p.n_ct;
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int ct = blockIdx.x % p.n_ct, slot = blockIdx.x / p.n_ct, cl = p.cl;
+    const uint32_t rank = cl > 1 ? tc::cluster_rank() : 0;
     const int B = a.B, H = a.H, KC = a.KC, S = a.S, T = a.T;
-    if (tid == 0) tc::mbar_init(pc.wbar, 1);
-    const uint32_t tmem = prologue(c, S, kCols);
+    const long long limit = a.limit;
+    const uint32_t tmem = pprologue(pc, S, kCols, cl);
     const uint8_t *wtile = a.wpack + (size_t)ct * KC * c.b_bytes;
     if (p.w_res && tid == 0) {
         tc::mbar_arrive_expect_tx(pc.wbar, KC * c.b_bytes);
         tc::bulk_g2s(pc.w0, wtile, KC * c.b_bytes, pc.wbar);
     }
     // the resident weight tile must land before the first MMA (warp 0, uniformly)
-    if (p.w_res && (tid >> 5) == 0 && !tc::mbar_wait(pc.wbar, 0, a.limit, c.abort)) {
+    if (p.w_res && warp == 0 && !tc::mbar_wait(pc.wbar, 0, limit, c.abort)) {
         set_abort(c, a.err);
         tc::mbar_wait(pc.wbar, 0, kDrainLimit, nullptr);
     }
+    int n_issued = 0, n_waited = 0;
     uint32_t gbase = 0, tiles = 0;
     bool stop = false;
     for (int t = T - 1; t >= 0 && !stop; --t) {
@@ -1005,28 +997,65 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_persist(const __grid_constant
                     for (int g = 0; g < 4; ++g) gq[cu][g] = *(const uint4 *)(gt + (size_t)g * H);
                 }
             }
-            auto tma = [&](int it, int s, uint64_t *bar) {
-                tc::mbar_arrive_expect_tx(bar, kAStage + (p.w_res ? 0u : c.b_bytes));
-                tc::tma_load_2d(c.a0 + s * kAStage, &tm_g, it * kChunk, t * B + row0, bar);
-                if (!p.w_res) tc::bulk_g2s(c.b0 + s * c.b_bytes, wtile + (size_t)it * c.b_bytes, c.b_bytes, bar);
-            };
-            auto no_gather = [](int, int) {};
-            auto issue = [&](int s, int j) {
-                issue_kmajor<NB>(tmem, c.a0 + s * kAStage, p.w_res ? pc.w0 + j * c.b_bytes : c.b0 + s * c.b_bytes, j);
-            };
-            // dG_t was written at the previous step by every column tile (thread 0 only)
-            auto dep = [&]() {
-                if (need == 0) return;
-                if (!*c.abort && !spin_until(p.cnt + rt, p.n_ct * need, a.limit, c.abort)) set_abort(c, a.err);
-                tc::fence_proxy_async_global();
-            };
-            pmainloop<false>(c, S, KC, gbase, tiles, 0, a.limit, a.err, tma, no_gather, issue, dep);
+            if (warp == 0 && !*c.abort) {
+                // dG_t was written at the previous step by every column tile of this row tile
+                if (need > 0) {
+                    if (!spin_until(p.cnt + rt, p.n_ct * need, limit, c.abort)) set_abort(c, a.err);
+                    tc::fence_proxy_async_global();
+                    __syncwarp();
+                }
+                for (int it = 0, jc = 0; jc < KC && !*c.abort;) {
+                    if (it < KC && it - jc < S) {
+                        const uint32_t g = gbase + it;
+                        const int s = (int)(g % S);
+                        if (g >= (uint32_t)S && !tc::mbar_wait(&c.empty[s], (g / S - 1) & 1, limit, c.abort)) {
+                            set_abort(c, a.err);
+                            break;
+                        }
+                        if (lane == 0) {
+                            load_a_chunk(c, s, kAStage + (p.w_res ? 0u : c.b_bytes), &tm_g, it * kChunk, t * B + row0,
+                                         it, cl, rank);
+                            if (!p.w_res)
+                                tc::bulk_g2s(c.b0 + s * c.b_bytes, wtile + (size_t)it * c.b_bytes, c.b_bytes,
+                                             &c.full[s]);
+                        }
+                        __syncwarp();
+                        ++n_issued;
+                        ++it;
+                    } else {
+                        const uint32_t g = gbase + jc;
+                        const int s = (int)(g % S);
+                        if (!tc::mbar_wait(&c.full[s], (g / S) & 1, limit, c.abort)) {
+                            set_abort(c, a.err);
+                            break;
+                        }
+                        ++n_waited;
+                        if (lane == 0) {
+                            tc::tc_fence_after();
+                            issue_kmajor<NB>(tmem, c.a0 + s * kAStage,
+                                             p.w_res ? pc.w0 + jc * c.b_bytes : c.b0 + s * c.b_bytes, jc);
+                            commit_empty(&c.empty[s], cl);
+                        }
+                        __syncwarp();
+                        ++jc;
+                    }
+                }
+                if (lane == 0) tc::mma_commit(c.done);
+                __syncwarp();
+            }
+            if (!tc::mbar_wait(c.done, tiles & 1, limit, nullptr)) {
+                set_abort(c, a.err);
+                tc::mbar_wait(c.done, tiles & 1, kDrainLimit, nullptr);
+            }
             gbase += KC;
             ++tiles;
+            __syncthreads();
+            tc::tc_fence_after();
             if (*c.abort) {
                 stop = true;
                 break;
             }
+            if (need > 0) (void)tc::ld_acquire_gpu(p.cnt + rt);  // every thread: acquire before reading
             const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
 #pragma unroll
             for (int cu = 0; cu < NC; ++cu) {
@@ -1066,6 +1095,12 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_persist(const __grid_constant
             tile_done(p.cnt + rt);
         }
     }
+    if (warp == 0)
+        for (int jj = n_waited; jj < n_issued; ++jj) {  // chunks armed but not consumed (abort)
+            const uint32_t g = (uint32_t)jj;
+            tc::mbar_wait(&c.full[g % S], (g / S) & 1, kDrainLimit, nullptr);
+        }
+    if (cl > 1) tc::cluster_sync();  // nobody leaves while a peer may still multicast into it
     finish(c, tmem, kCols);
 }
 
@@ -1189,58 +1224,91 @@ int pick_stages(int KC, int NB, size_t ctas, int sms)
 
 int pick_dx_n(int I) { return I <= 32 ? 32 : I <= 64 ? 64 : I <= 128 ? 128 : 256; }
 
+
+// Plans a persistent launch. Column tiles may form thread-block clusters of cl CTAs that
+// share their A chunks by multicast (the tile count is then padded to a multiple of cl;
+// padding tiles hold zero weights and store nothing). Multicast pays only when the
+// column tiles' re-reads of the A operand are a large L2 stream (want_mc); the cluster
+// sizes tried are then 16, 8, 4, 2 and 1, else 1. For each size and shared-memory budget
+// (one, two or three CTAs per SM) the weight tile stays resident when it leaves room for a
+// ring of at least two stages, and the grid is sized from the number of co-resident
+// clusters of that footprint. The fewest row tiles per CTA per step wins; ties go to the
+// larger cluster, then the deeper ring. Returns false if nothing fits.
+template <typename Kern>
+bool plan_persist(Kern kernel, int KC, int NB, int n_ct, int n_rt, bool want_mc, int *slot, int *wres, int *S,
+                  int *cl, int *nct_pad)
+{
+    const uint32_t fixed = 1024 + (2 * kMaxStages + 2) * 8 + 16 + 1024 /* static */;
+    const uint32_t wbytes = (uint32_t)KC * NB * 128;
+    int best_rounds = 1 << 30, best_c = 0;
+    bool found = false;
+    for (int c : {16, 8, 4, 2, 1}) {
+        if (c > 1 && (!want_mc || c / 2 >= n_ct)) continue;
+        const int pad = (n_ct + c - 1) / c * c;
+        if (c > 8 && cudaFuncSetAttribute(kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess) {
+            cudaGetLastError();
+            continue;
+        }
+        for (uint32_t budget : {200u * 1024, 100u * 1024, 66u * 1024}) {
+            const int wr = wbytes + 2 * kAStage + fixed <= budget;
+            const uint32_t stage = kAStage + (wr ? 0u : (uint32_t)NB * 128);
+            if (budget < fixed + (wr ? wbytes : 0u) + 2 * stage) continue;
+            const int st =
+                std::max(2, std::min({(int)((budget - fixed - (wr ? wbytes : 0u)) / stage), KC, kMaxStages}));
+            cudaLaunchConfig_t cfg = {};
+            cfg.gridDim = dim3(pad);
+            cfg.blockDim = dim3(kThreads);
+            cfg.dynamicSmemBytes = psmem_bytes(st, NB, KC, wr);
+            cudaLaunchAttribute at[1];
+            at[0].id = cudaLaunchAttributeClusterDimension;
+            at[0].val.clusterDim.x = c;
+            at[0].val.clusterDim.y = 1;
+            at[0].val.clusterDim.z = 1;
+            cfg.attrs = at;
+            cfg.numAttrs = 1;
+            int clusters = 0;
+            if (cudaOccupancyMaxActiveClusters(&clusters, kernel, &cfg) != cudaSuccess) {
+                cudaGetLastError();
+                continue;
+            }
+            const int groups = pad / c;  // clusters that cover the column tiles once
+            if (clusters < groups) continue;
+            const int sl = std::min(n_rt, clusters / groups);
+            const int rounds = (n_rt + sl - 1) / sl;
+            if (rounds < best_rounds || (rounds == best_rounds && c > best_c)) {
+                best_rounds = rounds;
+                best_c = c;
+                *slot = sl;
+                *wres = wr;
+                *S = st;
+                *cl = c;
+                *nct_pad = pad;
+                found = true;
+            }
+        }
+    }
+    return found;
+}
+
+// Cooperative (all CTAs co-resident) cluster launch of a persistent kernel.
 template <typename Kern, typename... Args>
-cudaError_t launch_coop(Kern kernel, dim3 grid, size_t smem, cudaStream_t st, Args... args)
+cudaError_t launch_persist(Kern kernel, dim3 grid, size_t smem, cudaStream_t st, int cl, Args... args)
 {
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = grid;
     cfg.blockDim = dim3(kThreads);
     cfg.dynamicSmemBytes = smem;
     cfg.stream = st;
-    cudaLaunchAttribute at[1];
+    cudaLaunchAttribute at[2];
     at[0].id = cudaLaunchAttributeCooperative;
     at[0].val.cooperative = 1;
+    at[1].id = cudaLaunchAttributeClusterDimension;
+    at[1].val.clusterDim.x = cl;
+    at[1].val.clusterDim.y = 1;
+    at[1].val.clusterDim.z = 1;
     cfg.attrs = at;
-    cfg.numAttrs = 1;
+    cfg.numAttrs = 2;
     return cudaLaunchKernelEx(&cfg, kernel, args...);
-}
-
-// Plans a persistent launch. For each shared-memory budget (one, two or three CTAs per
-// SM) the weight tile stays resident when it leaves room for a ring of at least two
-// stages, and the grid is sized from the occupancy of that footprint so every CTA is
-// co-resident; the budget needing the fewest row tiles per CTA per step wins (ties: the
-// deeper ring). Returns false if not even one CTA per column tile fits.
-template <typename Kern>
-bool plan_persist(Kern kernel, int KC, int NB, int n_ct, int n_rt, int sms, int *slot, int *wres, int *S)
-{
-    const uint32_t fixed = 1024 + (2 * kMaxStages + 2) * 8 + 16 + 1024 /* static */;
-    const uint32_t wbytes = (uint32_t)KC * NB * 128;
-    int best_rounds = 1 << 30;
-    bool found = false;
-    for (uint32_t budget : {200u * 1024, 100u * 1024, 66u * 1024}) {
-        const int wr = wbytes + 2 * kAStage + fixed <= budget;
-        const uint32_t stage = kAStage + (wr ? 0u : (uint32_t)NB * 128);
-        if (budget < fixed + (wr ? wbytes : 0u) + 2 * stage) continue;
-        const int st = std::max(2, std::min({(int)((budget - fixed - (wr ? wbytes : 0u)) / stage), KC, kMaxStages}));
-        int per_sm = 0;
-        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kernel, kThreads, psmem_bytes(st, NB, KC, wr)) !=
-            cudaSuccess) {
-            cudaGetLastError();
-            continue;
-        }
-        const long long resident = (long long)per_sm * sms;
-        if (resident < n_ct) continue;
-        const int sl = (int)std::min<long long>(n_rt, resident / n_ct);
-        const int rounds = (n_rt + sl - 1) / sl;
-        if (rounds < best_rounds) {
-            best_rounds = rounds;
-            *slot = sl;
-            *wres = wr;
-            *S = st;
-            found = true;
-        }
-    }
-    return found;
 }
 
 unsigned grid_for(const stacklstm *s, size_t n)
@@ -1263,6 +1331,21 @@ StepArgs step_args(stacklstm *s, const float *bias, const void *wpack, int kcx, 
 }
 
 }  // namespace
+
+std::string bf16_describe(const stacklstm *s)
+{
+    char buf[512];
+    const int rt = (int)ceil_div(s->B, kRows);
+    snprintf(buf, sizeof buf,
+             "bf16 tcgen05; row tiles %d; forward %s U=%d chunks %d (x %d)%s; backward %s U=%d chunks %d; "
+             "persistent fwd: slots %d cluster %d col tiles %d ring %d w_res %d; persistent bwd: slots %d cluster %d "
+             "col tiles %d ring %d w_res %d; step rings fwd %d bwd %d; dx N=%d x%d ring %d; dW %dx%d tiles x%d "
+             "splits ring %d",
+             rt, s->pf ? "persistent" : "per-step", s->uf, s->kcf, s->kcx, "", s->pb ? "persistent" : "per-step",
+             s->ub, s->kcb, s->pf_slot, s->pf_cl, s->pf_nct, s->pf_S, s->pf_wres, s->pb_slot, s->pb_cl, s->pb_nct,
+             s->pb_S, s->pb_wres, s->sf, s->sb, s->nx, s->nxt, s->sx, s->dw_mt, s->dw_nt, s->dw_split, s->sw);
+    return buf;
+}
 
 const char *bf16_unsupported(int T, int B, int I, int H)
 {
@@ -1299,17 +1382,27 @@ cudaError_t bf16_prepare(stacklstm *s)
     // persistent step kernels unless disabled (STACKLSTM_STEP_KERNELS=1 keeps one launch per step)
     const char *per_step = getenv("STACKLSTM_STEP_KERNELS");
     if (!(per_step && atoi(per_step) != 0)) {
-        const int nctf = (int)ceil_div(H, s->uf);
+        // A-operand bytes the column tiles re-read from L2 per step without multicast
+        const int nctf = (int)ceil_div(H, s->uf), nctb16 = (int)ceil_div(H, 16);
+        // multicast clusters measured slower than independent CTAs on every workload tried
+        // so far; STACKLSTM_MULTICAST=1 enables them where the re-read stream is large
+        const char *mc = getenv("STACKLSTM_MULTICAST");
+        const bool mc_on = mc && atoi(mc) != 0;
+        const bool mcf = mc_on && (double)rt * kAStage * s->kcf * nctf >= 8e6;
+        const bool mcb = mc_on && (double)rt * kAStage * s->kcb * nctb16 >= 8e6;
         if (s->uf == 32)
-            s->pf = plan_persist(fwd_persist<32>, s->kcf, 128, nctf, rt, sms, &s->pf_slot, &s->pf_wres, &s->pf_S);
+            s->pf = plan_persist(fwd_persist<32>, s->kcf, 128, nctf, rt, mcf, &s->pf_slot, &s->pf_wres, &s->pf_S,
+                                 &s->pf_cl, &s->pf_nct);
         else if (s->uf == 16)
-            s->pf = plan_persist(fwd_persist<16>, s->kcf, 64, nctf, rt, sms, &s->pf_slot, &s->pf_wres, &s->pf_S);
+            s->pf = plan_persist(fwd_persist<16>, s->kcf, 64, nctf, rt, mcf, &s->pf_slot, &s->pf_wres, &s->pf_S,
+                                 &s->pf_cl, &s->pf_nct);
         else
-            s->pf = plan_persist(fwd_persist<8>, s->kcf, 32, nctf, rt, sms, &s->pf_slot, &s->pf_wres, &s->pf_S);
+            s->pf = plan_persist(fwd_persist<8>, s->kcf, 32, nctf, rt, mcf, &s->pf_slot, &s->pf_wres, &s->pf_S,
+                                 &s->pf_cl, &s->pf_nct);
         // the persistent backward keeps 16-unit tiles (its prefetched epilogue operands
         // need the registers); the weight packing follows
-        s->pb = plan_persist(bwd_persist<16>, s->kcb, 16, (int)ceil_div(H, 16), rt, sms, &s->pb_slot, &s->pb_wres,
-                             &s->pb_S);
+        s->pb = plan_persist(bwd_persist<16>, s->kcb, 16, nctb16, rt, mcb, &s->pb_slot, &s->pb_wres,
+                             &s->pb_S, &s->pb_cl, &s->pb_nct);
         if (s->pb) s->ub = 16;
     }
     s->sf = pick_stages(s->kcf, 4 * s->uf, ceil_div(H, s->uf) * (size_t)rt, sms);
@@ -1317,8 +1410,10 @@ cudaError_t bf16_prepare(stacklstm *s)
     s->sx = pick_stages(s->kcb, s->nx, s->nxt * ceil_div(R, kRows), sms);
     s->sw = pick_stages((int)ceil_div(RC, s->dw_split), 256, (size_t)s->dw_mt * s->dw_nt * s->dw_split, sms);
 
-    const size_t fwd_bytes = (size_t)ceil_div(H, s->uf) * s->kcf * 4 * s->uf * 128;
-    const size_t bwd_bytes = (size_t)ceil_div(H, s->ub) * s->kcb * s->ub * 128;
+    const size_t fwd_bytes = (size_t)std::max<size_t>(ceil_div(H, s->uf), s->pf ? s->pf_nct : 0) * s->kcf * 4 *
+                             s->uf * 128;
+    const size_t bwd_bytes = (size_t)std::max<size_t>(ceil_div(H, s->ub), s->pb ? s->pb_nct : 0) * s->kcb * s->ub *
+                             128;
     const size_t dx_bytes = (size_t)s->nxt * s->kcb * s->nx * 128;
     s->dw_part_elems = (size_t)s->dw_split * s->dw_mt * kRows * s->dw_nt * 256;
     void *p;
@@ -1361,7 +1456,8 @@ cudaError_t bf16_forward(stacklstm *s, const __nv_bfloat16 *x, const __nv_bfloat
     if ((e = cudaMemcpyAsync(s->hr, h0, sizeof(__nv_bfloat16) * B * H, cudaMemcpyDeviceToDevice, s->stream)))
         return e;
     if ((e = cudaMemcpyAsync(s->hist_c, c0, sizeof(float) * B * H, cudaMemcpyDeviceToDevice, s->stream))) return e;
-    const int nctf = (int)ceil_div(H, s->uf), nctb = (int)ceil_div(H, s->ub);
+    const int nctf = std::max((int)ceil_div(H, s->uf), s->pf ? s->pf_nct : 0);
+    const int nctb = std::max((int)ceil_div(H, s->ub), s->pb ? s->pb_nct : 0);
     pack_fwd<<<grid_for(s, (size_t)nctf * s->kcf * 4 * s->uf * kChunk), 256, 0, s->stream>>>(
         W, I, H, s->uf, s->kcx, s->kcf, nctf, (__nv_bfloat16 *)s->w_fwd);
     pack_rows<<<grid_for(s, (size_t)nctb * s->kcb * s->ub * kChunk), 256, 0, s->stream>>>(
@@ -1373,18 +1469,18 @@ cudaError_t bf16_forward(stacklstm *s, const __nv_bfloat16 *x, const __nv_bfloat
     if (s->pf) {
         PersistArgs p;
         p.s = step_args(s, bias, s->w_fwd, s->kcx, s->kcf, s->pf_S);
-        p.n_ct = nctf; p.n_rt = (int)ceil_div(B, kRows); p.n_slot = s->pf_slot; p.w_res = s->pf_wres;
-        p.cnt = s->rowcnt;
+        p.n_ct = s->pf_nct; p.n_rt = (int)ceil_div(B, kRows); p.n_slot = s->pf_slot; p.w_res = s->pf_wres;
+        p.cl = s->pf_cl; p.cnt = s->rowcnt;
         if ((e = cudaMemsetAsync(p.cnt, 0, sizeof(int32_t) * p.n_rt, s->stream))) return e;
-        const dim3 g(nctf * p.n_slot);
+        const dim3 g(p.n_ct * p.n_slot);
         const size_t sm = psmem_bytes(p.s.S, 4 * s->uf, s->kcf, p.w_res);
         const CUtensorMap &tm = map(s, kMapX128), &th = map(s, kMapH128);
         if (s->uf == 32)
-            e = launch_coop(fwd_persist<32>, g, sm, s->stream, tm, th, p);
+            e = launch_persist(fwd_persist<32>, g, sm, s->stream, p.cl, tm, th, p);
         else if (s->uf == 16)
-            e = launch_coop(fwd_persist<16>, g, sm, s->stream, tm, th, p);
+            e = launch_persist(fwd_persist<16>, g, sm, s->stream, p.cl, tm, th, p);
         else
-            e = launch_coop(fwd_persist<8>, g, sm, s->stream, tm, th, p);
+            e = launch_persist(fwd_persist<8>, g, sm, s->stream, p.cl, tm, th, p);
         if (e) return e;
         s->launches += 1;
         return cudaGetLastError();
@@ -1418,13 +1514,13 @@ cudaError_t bf16_backward_steps(stacklstm *s)
     if (s->pb) {
         PersistArgs p;
         p.s = step_args(s, nullptr, s->w_bwd, 0, s->kcb, s->pb_S);
-        p.n_ct = (int)ceil_div(H, s->ub); p.n_rt = (int)ceil_div(B, kRows); p.n_slot = s->pb_slot;
-        p.w_res = s->pb_wres; p.cnt = s->rowcnt + p.n_rt;
+        p.n_ct = s->pb_nct; p.n_rt = (int)ceil_div(B, kRows); p.n_slot = s->pb_slot;
+        p.w_res = s->pb_wres; p.cl = s->pb_cl; p.cnt = s->rowcnt + p.n_rt;
         if ((e = cudaMemsetAsync(p.cnt, 0, sizeof(int32_t) * p.n_rt, s->stream))) return e;
         const dim3 g(p.n_ct * p.n_slot);
         const size_t sm = psmem_bytes(p.s.S, s->ub, s->kcb, p.w_res);
         const CUtensorMap &tm = map(s, kMapG128);
-        e = launch_coop(bwd_persist<16>, g, sm, s->stream, tm, p);
+        e = launch_persist(bwd_persist<16>, g, sm, s->stream, p.cl, tm, p);
         if (e) return e;
         s->launches += 1;
         return cudaGetLastError();

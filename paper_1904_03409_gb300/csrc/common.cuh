@@ -60,6 +60,8 @@ struct stacklstm {
     int pf_slot = 0, pb_slot = 0;  // CTAs per column tile (each takes every n_slot-th row tile)
     int pf_wres = 0, pb_wres = 0;  // weight tile resident in shared memory
     int pf_S = 0, pb_S = 0;        // ring depths of the persistent kernels
+    int pf_cl = 1, pb_cl = 1;      // thread-block cluster sizes (column tiles sharing A by multicast)
+    int pf_nct = 0, pb_nct = 0;    // column tiles, padded to a multiple of the cluster size
     int32_t *rowcnt = nullptr;     // [2][row tiles] completed steps per row tile
     int nx = 0, nxt = 0;     // input gradient: columns per tile, number of column tiles
     int dw_mt = 0, dw_nt = 0, dw_split = 0;  // weight gradient: row tiles, column tiles, splits
@@ -78,6 +80,7 @@ struct stacklstm {
     std::vector<EventPair> pending;
     std::vector<cudaEvent_t> event_pool;
 
+    std::string plan;  // stacklstm_plan
     std::string last_error;
     std::vector<void *> allocs;
 };
@@ -106,6 +109,7 @@ cudaError_t bf16_dx(stacklstm *s, float *dx);
 cudaError_t bf16_dw(stacklstm *s, float *dW, float *dbias);
 size_t bf16_workspace_bytes(int T, int B, int I, int H, int num_sms);
 const char *bf16_unsupported(int T, int B, int I, int H);
+std::string bf16_describe(const stacklstm *s);
 
 inline unsigned ceil_div(size_t a, size_t b) { return (unsigned)((a + b - 1) / b); }
 
