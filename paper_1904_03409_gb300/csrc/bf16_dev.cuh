@@ -1,0 +1,178 @@
+// bf16_dev.cuh -- device helpers shared by the bf16 tensor-core kernels (bf16_path.cu,
+// bf16_persist.cu): tile constants, the K-major MMA issue of one contraction chunk, the cell
+// nonlinearities, vector loads/stores and packing, the step arguments and the forward
+// cell epilogue (Algorithm 1: the LSTM cell on the gathered top state, written to history
+// row t + 1).
+#pragma once
+
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
+#include "common.cuh"
+#include "tc.cuh"
+
+namespace sl {
+using tc::smem_u32;
+using tc::sw128;
+
+constexpr int kThreads = 128;  // four warps: one per 32-lane quadrant of tensor memory
+constexpr int kRows = 128;     // MMA M: batch rows (or weight rows) per CTA tile
+constexpr int kChunk = 64;     // contraction elements per chunk: one 128-byte swizzled row
+constexpr uint32_t kAStage = kRows * 128;
+constexpr int kMaxStages = 16;
+constexpr long long kDrainLimit = 4000000000LL;  // wait for own copies / MMAs before exit
+
+template <int N>
+struct TmemCols {
+    static constexpr uint32_t value = N <= 32 ? 32 : N <= 64 ? 64 : N <= 128 ? 128 : 256;
+};
+
+
+// K-major operands, both 128-byte swizzled rows of 64 bf16: four MMAs of K = 16 per chunk
+// step through the swizzle atom by advancing the start address 32 bytes.
+template <int N>
+__device__ __forceinline__ void issue_kmajor(uint32_t tmem, uint32_t a_stage, uint32_t b_stage, int chunk)
+{
+    constexpr uint32_t idesc = tc::idesc_bf16(N);
+#pragma unroll
+    for (int k = 0; k < kChunk / 16; ++k)
+        tc::mma_bf16(tmem, tc::smem_desc(a_stage + k * 32, 16, 1024), tc::smem_desc(b_stage + k * 32, 16, 1024),
+                     idesc, (chunk | k) != 0);
+}
+
+// ----------------------------------------------------------------------- helpers
+// Cell nonlinearities of the bf16 path: the hardware tanh approximation (PTX
+// tanh.approx.f32, relative error about 2^-11, below the bf16 rounding of h), and the
+// logistic sigmoid through the identity sigmoid(z) = 1/2 + tanh(z / 2) / 2.
+__device__ __forceinline__ float tanh_hw(float x)
+{
+    float y;
+    asm("tanh.approx.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+__device__ __forceinline__ float sigm(float z) { return fmaf(0.5f, tanh_hw(0.5f * z), 0.5f); }
+
+// L2-coherent read (bypasses L1) of state another CTA or an earlier launch wrote.
+__device__ __forceinline__ void ld8f_cg(const float *p, float (&v)[8])
+{
+    const float4 a = __ldcg((const float4 *)p), b = __ldcg((const float4 *)(p + 4));
+    v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w; v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+}
+__device__ __forceinline__ void st8f(float *p, const float (&v)[8])
+{
+    *(float4 *)p = make_float4(v[0], v[1], v[2], v[3]);
+    *(float4 *)(p + 4) = make_float4(v[4], v[5], v[6], v[7]);
+}
+__device__ __forceinline__ uint4 pack8_bf16(const float (&v)[8])
+{
+    uint4 o;
+    __nv_bfloat162 t;
+    t = __floats2bfloat162_rn(v[0], v[1]); o.x = *(uint32_t *)&t;
+    t = __floats2bfloat162_rn(v[2], v[3]); o.y = *(uint32_t *)&t;
+    t = __floats2bfloat162_rn(v[4], v[5]); o.z = *(uint32_t *)&t;
+    t = __floats2bfloat162_rn(v[6], v[7]); o.w = *(uint32_t *)&t;
+    return o;
+}
+__device__ __forceinline__ uint4 pack8_f16(const float (&v)[8])
+{
+    uint4 o;
+    __half2 t;
+    t = __floats2half2_rn(v[0], v[1]); o.x = *(uint32_t *)&t;
+    t = __floats2half2_rn(v[2], v[3]); o.y = *(uint32_t *)&t;
+    t = __floats2half2_rn(v[4], v[5]); o.z = *(uint32_t *)&t;
+    t = __floats2half2_rn(v[6], v[7]); o.w = *(uint32_t *)&t;
+    return o;
+}
+__device__ __forceinline__ void unpack8_f16(uint4 u, float (&v)[8])
+{
+    const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const float2 f = __half22float2(*(const __half2 *)&w[i]);
+        v[2 * i] = f.x;
+        v[2 * i + 1] = f.y;
+    }
+}
+
+// ------------------------------------------------------------------ arguments
+struct StepArgs {
+    int T, B, I, H;
+    int kcx, KC, S;             // x-part chunks, all chunks, ring depth
+    const int32_t *top;         // [T+1][B]
+    __nv_bfloat16 *hist_h;      // [T+1][B][H]
+    __nv_bfloat16 *hr;          // [T+1][B][H] h operand of each step
+    float *hist_c;              // [T+1][B][H]
+    __half *gates;              // [T][B][4H]
+    const float *bias;          // [4H]
+    const uint8_t *wpack;       // packed B-operand tiles of this kernel
+    float *dhist_h, *dhist_c;   // [T+1][B][H]
+    __nv_bfloat16 *dG;          // [T][B][4H]
+    long long limit;
+    int32_t *err;
+};
+
+
+// Forward epilogue for one tile row and 8 hidden units: the cell on pre-activations z
+// (gate blocks i, f, g, o), writes history row t + 1 (h', c'), the gates, and the h
+// operand of step t + 1: h' when step t pushed (the new state is the next top), else the
+// older top, a row this tile already wrote (hcopy).
+__device__ __forceinline__ void fwd_cell8(const StepArgs &a, int t, int b, int u, const float (&z)[4][8],
+                                          const float *bias_i, const float *bias_f, const float *bias_g,
+                                          const float *bias_o, const float *cr, bool next_is_new, uint4 hcopy)
+{
+    const int B = a.B, H = a.H;
+    float cn[8], hn[8], gv[4][8];
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+        const float ig = sigm(z[0][e] + bias_i[e]);
+        const float fg = sigm(z[1][e] + bias_f[e]);
+        const float gg = tanh_hw(z[2][e] + bias_g[e]);
+        const float og = sigm(z[3][e] + bias_o[e]);
+        cn[e] = fmaf(fg, cr[e], ig * gg);
+        hn[e] = og * tanh_hw(cn[e]);
+        gv[0][e] = ig; gv[1][e] = fg; gv[2][e] = gg; gv[3][e] = og;
+    }
+    const size_t w = ((size_t)(t + 1) * B + b) * H + u;
+    const uint4 hb = pack8_bf16(hn);
+    *(uint4 *)(a.hist_h + w) = hb;
+    *(uint4 *)(a.hr + w) = next_is_new ? hb : hcopy;
+    st8f(a.hist_c + w, cn);
+    __half *gt = a.gates + ((size_t)t * B + b) * 4 * H + u;
+#pragma unroll
+    for (int g = 0; g < 4; ++g) *(uint4 *)(gt + (size_t)g * H) = pack8_f16(gv[g]);
+}
+
+// ------------------------------------------------------------------ host helpers
+template <typename Kern, typename... Args>
+cudaError_t launch(Kern kernel, dim3 grid, size_t smem, cudaStream_t st, bool pdl, Args... args)
+{
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    at[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = pdl ? at : nullptr;
+    cfg.numAttrs = pdl ? 1 : 0;
+    return cudaLaunchKernelEx(&cfg, kernel, args...);
+}
+
+constexpr uint32_t kSmemCap = 225 * 1024;
+
+template <typename Kern>
+cudaError_t allow_smem(Kern k)
+{
+    return cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemCap);
+}
+
+// Ring depth: as many stages as the contraction has chunks, within a shared-memory
+
+// ---- persistent step kernels (bf16_persist.cu)
+bool bf16_plan_fwd_persist(stacklstm *s, PersistPlan *pl);
+bool bf16_plan_bwd_persist(stacklstm *s, PersistPlan *pl);
+cudaError_t bf16_launch_fwd_persist(stacklstm *s, const StepArgs &a, const CUtensorMap &tm_x, const CUtensorMap &tm_h);
+cudaError_t bf16_launch_bwd_persist(stacklstm *s, const StepArgs &a, const CUtensorMap &tm_g);
+
+}  // namespace sl

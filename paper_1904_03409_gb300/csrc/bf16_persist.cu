@@ -1,0 +1,704 @@
+// bf16_persist.cu -- persistent, warp-specialised step kernels of the bf16 path: one
+// cooperative launch runs all T steps of the forward (Algorithm 1) or of the reverse-time
+// backward (Sec. 5).
+//
+// Each CTA keeps one column tile ct (U hidden units: forward, the 4U gate columns of those
+// units; backward, U columns of dh_read = dG_t W_h^T) and a fixed set of row tiles
+// (rt = slot, slot + n_slot, ...), so every (instance, unit) has one owner for the whole
+// launch. Its tiles run in the order (step, rt). The warps have fixed roles:
+//   producer (warp 4 EP): loads each tile's A operand by TMA into a ring of S stages of G
+//     64-wide contraction chunks (one full / empty mbarrier pair per stage), and the
+//     weight tile: once, resident in shared memory, or per stage by bulk copy;
+//   MMA (warp 4 EP + 1): waits for a stage, issues its 4G tcgen05.mma (bf16 in, fp32
+//     accumulate) in one straight run and commits the stage back. Tiles alternate between
+//     two tensor-memory accumulators, so tile k + 1 is multiplied while tile k's epilogue
+//     runs. An mbarrier wait between MMAs stalls MMA issue for a few hundred cycles, so a
+//     wait covers a whole stage;
+//   epilogue (warps 0 .. 4 EP - 1): warp w reads accumulator lanes 32 (w mod 4) .. + 31
+//     (rows) for unit part w / 4. Forward: the LSTM cell, history row t + 1 and the h
+//     operand of step t + 1. Backward: adds dh_read to the gradient of the state step t
+//     read, then runs the pointwise backward of step t - 1, whose gradient is now complete.
+//
+// The only inter-CTA dependency is within a row tile: step t reads what every column tile
+// of the row tile wrote at the step before (forward: hr[t]; backward: dG_t). Each row tile
+// has a counter of completed steps, raised with release semantics after the epilogue's
+// stores and polled with acquire semantics (a bounded spin) by the producer before it
+// loads the dependent chunks. All CTAs are co-resident (cooperative launch), so the spins
+// end; every wait is bounded and a timeout aborts the whole grid through the error word.
+//
+// With cl > 1 the cl CTAs of a thread-block cluster hold cl consecutive column tiles of
+// the same row tiles and share the A operand: chunk c is loaded by cluster rank c mod cl
+// and multicast into the same stage of every CTA; `empty` counts cl arrivals because each
+// CTA commits its MMA completion to the `empty` barrier of every CTA of the cluster.
+#include <stdio.h>
+
+#include <algorithm>
+
+#include "bf16_dev.cuh"
+
+namespace sl {
+namespace {
+
+using tc::smem_u32;
+
+struct WsArgs {
+    StepArgs s;              // s.kcx: chunks before the dependent ones; s.S: ring stages
+    int n_ct, n_rt, n_slot;  // column tiles (a multiple of cl); row tiles; CTAs per column tile
+    int w_res;               // 1: weight tile resident in shared memory
+    int cl;                  // cluster size along the column tiles (1: no multicast)
+    int32_t *cnt;            // [n_rt] completed steps per row tile, zero at launch
+};
+
+// Dynamic shared memory: [weight tile (w_res)][S stages: G A chunks, then G weight
+// chunks unless resident][barriers], based at the first 1024-byte boundary.
+constexpr uint32_t kBarBytes = (2 * kMaxStages + 6) * 8 + 16;
+
+__host__ __device__ constexpr uint32_t ws_stage_bytes(int G, int NB, int w_res)
+{
+    return (uint32_t)G * (kAStage + (w_res ? 0u : (uint32_t)NB * 128));
+}
+__host__ __device__ constexpr uint32_t ws_smem_bytes(int S, int G, int NB, int KC, int w_res)
+{
+    return 1024 + (w_res ? (uint32_t)KC * NB * 128 : 0u) + (uint32_t)S * ws_stage_bytes(G, NB, w_res) + kBarBytes;
+}
+
+struct WCtl {
+    uint32_t w0, ring0, stage;  // resident weight tile, stage 0, bytes per stage
+    uint64_t *full, *empty, *tfull, *tempty, *wbar, *done;
+    uint32_t *tmem_slot;
+    int *n_issued, *n_consumed;  // groups armed by the producer / consumed by the MMA warp
+    volatile int *abort;
+};
+
+__device__ __forceinline__ WCtl wcarve(uint8_t *raw, int S, int G, int NB, int KC, int w_res)
+{
+    const uint32_t off = smem_u32(raw);
+    uint8_t *base = raw + ((1024u - (off & 1023u)) & 1023u);
+    WCtl c;
+    const uint32_t wbytes = w_res ? (uint32_t)KC * NB * 128 : 0u;
+    c.stage = ws_stage_bytes(G, NB, w_res);
+    c.w0 = smem_u32(base);
+    c.ring0 = c.w0 + wbytes;
+    uint64_t *bars = (uint64_t *)(base + wbytes + (size_t)S * c.stage);
+    c.full = bars;
+    c.empty = bars + kMaxStages;
+    c.tfull = bars + 2 * kMaxStages;
+    c.tempty = c.tfull + 2;
+    c.wbar = c.tempty + 2;
+    c.done = c.wbar + 1;
+    c.tmem_slot = (uint32_t *)(c.done + 1);
+    c.n_issued = (int *)(c.tmem_slot + 1);
+    c.n_consumed = c.n_issued + 1;
+    c.abort = (volatile int *)(c.n_consumed + 1);
+    return c;
+}
+
+__device__ __forceinline__ void ws_abort(const WCtl &c, int32_t *err)
+{
+    *c.abort = 1;
+    atomicCAS(err, 0, (int)SL_ERR_TIMEOUT);
+}
+
+// Bounded spin until *cnt >= target (acquire). False on timeout, on a local abort, or
+// once another CTA recorded an error.
+__device__ __forceinline__ bool spin_until(const int32_t *cnt, int target, long long limit, volatile int *abort,
+                                           const int32_t *err)
+{
+    if (tc::ld_acquire_gpu(cnt) >= target) return true;
+    const long long t0 = clock64();
+    while (true) {
+        if (clock64() - t0 >= limit) return false;
+        if (*abort || *(const volatile int32_t *)err) return false;
+        __nanosleep(32);
+        if (tc::ld_acquire_gpu(cnt) >= target) return true;
+    }
+}
+
+// One stage's MMAs: n (<= G) chunks of four K = 16 steps, K-major operands in 128-byte
+// swizzled rows (A chunks kAStage apart, weight chunks NB * 128 bytes apart).
+template <int NB, int G>
+__device__ __forceinline__ void issue_group(uint32_t d, uint32_t a, uint32_t b, int n, bool first)
+{
+    constexpr uint32_t idesc = tc::idesc_bf16(NB);
+#pragma unroll
+    for (int j = 0; j < G; ++j)
+        if (j < n) {
+#pragma unroll
+            for (int k = 0; k < kChunk / 16; ++k)
+                tc::mma_bf16(d, tc::smem_desc(a + j * kAStage + k * 32, 16, 1024),
+                             tc::smem_desc(b + j * (NB * 128) + k * 32, 16, 1024), idesc,
+                             !(first && j == 0 && k == 0));
+        }
+}
+
+// Loads UE consecutive accumulator columns of this thread's lane (no completion wait).
+template <int UE>
+__device__ __forceinline__ void tmem_cols(uint32_t taddr, uint32_t (&r)[UE])
+{
+    if constexpr (UE % 16 == 0) {
+#pragma unroll
+        for (int i = 0; i < UE / 16; ++i) tc::tmem_ld16_async(taddr + i * 16, *(uint32_t(*)[16])(r + i * 16));
+    } else {
+#pragma unroll
+        for (int i = 0; i < UE / 8; ++i) tc::tmem_ld8_async(taddr + i * 8, *(uint32_t(*)[8])(r + i * 8));
+    }
+}
+
+// chunk range of the stage that starts at chunk c0: never mixes the independent chunks
+// (< split) with the dependent ones
+__device__ __forceinline__ int group_end(int c0, int G, int split, int KC)
+{
+    return min(c0 + G, c0 < split ? split : KC);
+}
+
+// ------------------------------------------------------------------ the kernel
+// kFwd: forward (tm_a = x_t tiles for chunks < kcx, tm_b = hr[t] tiles after them);
+// else backward (tm_b = dG_t tiles, kcx = 0: every chunk depends on the step before).
+template <int U, int EP, int G, bool kFwd>
+__global__ void __launch_bounds__(32 * (4 * EP + 2), 1)
+step_ws(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtensorMap tm_b, WsArgs p)
+{
+    constexpr int NB = kFwd ? 4 * U : U;  // accumulator columns
+    constexpr int E = 4 * EP;             // epilogue warps
+    constexpr int UE = U / EP;            // units per epilogue thread
+    constexpr uint32_t kCols = TmemCols<NB>::value;
+    constexpr uint32_t bchunk = NB * 128;
+    static_assert(UE % 8 == 0, "epilogue works on groups of 8 units");
+    const StepArgs &a = p.s;
+    extern __shared__ uint8_t smem_raw[];
+    __shared__ float s_bias[kFwd ? 4 * U : 4];
+    const int S = a.S, KC = a.KC, split = a.kcx, T = a.T, B = a.B, H = a.H;
+    const WCtl c = wcarve(smem_raw, S, G, NB, KC, p.w_res);
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int ct = blockIdx.x % p.n_ct, slot = blockIdx.x / p.n_ct, cl = p.cl;
+    const uint32_t rank = cl > 1 ? tc::cluster_rank() : 0;
+    const int n_mine = slot < p.n_rt ? (p.n_rt - slot + p.n_slot - 1) / p.n_slot : 0;
+    const int n_tiles = T * n_mine;
+    const long long limit = a.limit;
+    if (kFwd)
+        for (int i = tid; i < 4 * U; i += blockDim.x) {
+            const int g = i / U, u = ct * U + i % U;
+            s_bias[i] = u < H ? a.bias[g * H + u] : 0.0f;
+        }
+    if (tid == 0) {
+        for (int s = 0; s < S; ++s) {
+            tc::mbar_init(&c.full[s], 1);
+            tc::mbar_init(&c.empty[s], (uint32_t)cl);
+        }
+        for (int i = 0; i < 2; ++i) {
+            tc::mbar_init(&c.tfull[i], 1);
+            tc::mbar_init(&c.tempty[i], E);
+        }
+        tc::mbar_init(c.wbar, 1);
+        tc::mbar_init(c.done, 1);
+        *c.n_issued = 0;
+        *c.n_consumed = 0;
+        *c.abort = 0;
+        tc::fence_mbar_init();
+    }
+    if (warp == E) tc::tmem_alloc(c.tmem_slot, 2 * kCols);
+    tc::tc_fence_before();
+    __syncthreads();
+    if (cl > 1) tc::cluster_sync();
+    tc::tc_fence_after();
+    const uint32_t tmem = *c.tmem_slot;
+    const uint8_t *wtile = a.wpack + (size_t)ct * KC * bchunk;
+
+    if (warp == E) {
+        // ------------------------------------------------------------ producer
+        if (lane == 0) {
+            if (p.w_res) {
+                tc::mbar_arrive_expect_tx(c.wbar, KC * bchunk);
+                tc::bulk_g2s(c.w0, wtile, KC * bchunk, c.wbar);
+            }
+            uint32_t g = 0;
+            for (int k = 0; k < n_tiles && !*c.abort; ++k) {
+                const int ks = k / n_mine, rt = slot + (k % n_mine) * p.n_slot;
+                const int t = kFwd ? ks : T - 1 - ks;
+                const int row = t * B + rt * kRows;
+                for (int c0 = 0; c0 < KC;) {
+                    const int c1 = group_end(c0, G, split, KC);
+                    if (c0 == split && ks > 0) {
+                        // every column tile of this row tile finished the step before
+                        if (!spin_until(p.cnt + rt, p.n_ct * ks, limit, c.abort, a.err)) {
+                            ws_abort(c, a.err);
+                            break;
+                        }
+                        tc::fence_proxy_async_global();
+                    }
+                    const int s = (int)(g % S);
+                    if (g >= (uint32_t)S && !tc::mbar_wait(&c.empty[s], (g / S - 1) & 1, limit, c.abort)) {
+                        ws_abort(c, a.err);
+                        break;
+                    }
+                    const uint32_t st = c.ring0 + s * c.stage;
+                    tc::mbar_arrive_expect_tx(&c.full[s], (c1 - c0) * (kAStage + (p.w_res ? 0u : bchunk)));
+                    for (int cc = c0; cc < c1; ++cc) {
+                        const bool first = cc < split;
+                        const CUtensorMap *tm = first ? &tm_a : &tm_b;
+                        const int col = (first ? cc : cc - split) * kChunk;
+                        const uint32_t dst = st + (cc - c0) * kAStage;
+                        if (cl == 1)
+                            tc::tma_load_2d(dst, tm, col, row, &c.full[s]);
+                        else if ((uint32_t)(cc % cl) == rank)
+                            tc::tma_load_2d_mc(dst, tm, col, row, &c.full[s], (uint16_t)((1u << cl) - 1));
+                    }
+                    if (!p.w_res)
+                        tc::bulk_g2s(st + G * kAStage, wtile + (size_t)c0 * bchunk, (c1 - c0) * bchunk, &c.full[s]);
+                    ++g;
+                    c0 = c1;
+                }
+            }
+            *c.n_issued = (int)g;
+        }
+        __syncwarp();
+    } else if (warp == E + 1) {
+        // ------------------------------------------------------------ MMA issue
+        if (lane == 0) {
+            uint32_t g = 0;
+            bool w_ready = !p.w_res;
+            for (int k = 0; k < n_tiles && !*c.abort; ++k) {
+                const int acc = k & 1;
+                if (k >= 2 && !tc::mbar_wait(&c.tempty[acc], ((k >> 1) - 1) & 1, limit, c.abort)) {
+                    ws_abort(c, a.err);
+                    break;
+                }
+                if (!w_ready) {
+                    if (!tc::mbar_wait(c.wbar, 0, limit, c.abort)) {
+                        ws_abort(c, a.err);
+                        break;
+                    }
+                    w_ready = true;
+                }
+                tc::tc_fence_after();
+                const uint32_t d = tmem + acc * kCols;
+                bool bad = false;
+                for (int c0 = 0; c0 < KC;) {
+                    const int c1 = group_end(c0, G, split, KC);
+                    const int s = (int)(g % S);
+                    if (!tc::mbar_wait(&c.full[s], (g / S) & 1, limit, c.abort)) {
+                        ws_abort(c, a.err);
+                        bad = true;
+                        break;
+                    }
+                    tc::tc_fence_after();
+                    const uint32_t st = c.ring0 + s * c.stage;
+                    issue_group<NB, G>(d, st, p.w_res ? c.w0 + c0 * bchunk : st + G * kAStage, c1 - c0, c0 == 0);
+                    if (cl > 1)
+                        tc::mma_commit_mc(&c.empty[s], (uint16_t)((1u << cl) - 1));
+                    else
+                        tc::mma_commit(&c.empty[s]);
+                    ++g;
+                    c0 = c1;
+                }
+                if (bad) break;
+                tc::mma_commit(&c.tfull[acc]);
+            }
+            *c.n_consumed = (int)g;
+            tc::mma_commit(c.done);  // arrives once every MMA issued above has completed
+        }
+        __syncwarp();
+    } else {
+        // ------------------------------------------------------------ epilogue
+        const int q = warp & 3, part = warp >> 2;
+        const uint32_t lane_off = (uint32_t)(q * 32) << 16;
+        for (int k = 0; k < n_tiles; ++k) {
+            const int ks = k / n_mine, rt = slot + (k % n_mine) * p.n_slot;
+            const int t = kFwd ? ks : T - 1 - ks;
+            const int b = rt * kRows + q * 32 + lane;
+            const bool row_ok = b < B;
+            const int u0 = ct * U + part * UE;  // first unit of this thread
+            const int acc = k & 1;
+            const uint32_t taddr = tmem + acc * kCols + lane_off;
+            if constexpr (kFwd) {
+                // operands this thread wrote itself at earlier steps (same rows and units):
+                // c_read, and the older top the next step reads when step t does not push
+                const int src = row_ok ? a.top[(size_t)t * B + b] : 0;
+                const int s_next = row_ok ? a.top[(size_t)(t + 1) * B + b] : 0;
+                const bool is_new = s_next == t + 1;
+                float cr[UE];
+                uint4 hc[UE / 8];
+#pragma unroll
+                for (int cu = 0; cu < UE / 8; ++cu) {
+                    const int u = u0 + cu * 8;
+                    float v[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+                    hc[cu] = make_uint4(0, 0, 0, 0);
+                    if (row_ok && u < H) {
+                        ld8f_cg(a.hist_c + ((size_t)src * B + b) * H + u, v);
+                        if (!is_new) hc[cu] = __ldcg((const uint4 *)(a.hr + ((size_t)s_next * B + b) * H + u));
+                    }
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) cr[cu * 8 + e] = v[e];
+                }
+                const bool ok = tc::mbar_wait(&c.tfull[acc], (k >> 1) & 1, limit, c.abort);
+                if (!ok) ws_abort(c, a.err);
+                __syncwarp();
+                if (tc::bar_any(1, E * 32, !ok || *c.abort)) break;
+                tc::tc_fence_after();
+                uint32_t zr[4][UE];
+#pragma unroll
+                for (int g = 0; g < 4; ++g) tmem_cols<UE>(taddr + g * U + part * UE, zr[g]);
+                tc::tmem_wait_ld();
+                tc::tc_fence_before();
+                __syncwarp();
+                if (lane == 0) tc::mbar_arrive(&c.tempty[acc]);
+#pragma unroll
+                for (int cu = 0; cu < UE / 8; ++cu) {
+                    const int u = u0 + cu * 8;
+                    if (row_ok && u < H) {
+                        float z[4][8];
+#pragma unroll
+                        for (int g = 0; g < 4; ++g)
+#pragma unroll
+                            for (int e = 0; e < 8; ++e) z[g][e] = __uint_as_float(zr[g][cu * 8 + e]);
+                        const int j = part * UE + cu * 8;
+                        fwd_cell8(a, t, b, u, z, s_bias + j, s_bias + U + j, s_bias + 2 * U + j, s_bias + 3 * U + j,
+                                  cr + cu * 8, is_new, hc[cu]);
+                    }
+                }
+            } else {
+                // Every epilogue operand: the gradient history of this thread's units is
+                // written only by this thread (or zeroed before the launch); gates and cell
+                // states come from the forward.
+                const int src = row_ok ? a.top[(size_t)t * B + b] : 0;
+                const int s1 = (row_ok && t >= 1) ? a.top[(size_t)(t - 1) * B + b] : 0;
+                float dh_src[UE], dh_t[UE], dc_t[UE], cn[UE], cr[UE], dc_rd[UE];
+                uint4 gq[UE / 8][4];
+#pragma unroll
+                for (int cu = 0; cu < UE / 8; ++cu) {
+                    const int u = u0 + cu * 8;
+                    const bool uok = row_ok && u < H;
+                    float v[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+                    if (uok) ld8f_cg(a.dhist_h + ((size_t)src * B + b) * H + u, v);
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) dh_src[cu * 8 + e] = v[e];
+                    if (uok && t >= 1) {
+                        const size_t wr = ((size_t)t * B + b) * H + u, rd = ((size_t)s1 * B + b) * H + u;
+                        float w1[8], w2[8], w3[8], w4[8], w5[8];
+                        ld8f_cg(a.dhist_h + wr, w1);
+                        ld8f_cg(a.dhist_c + wr, w2);
+                        ld8f_cg(a.hist_c + wr, w3);
+                        ld8f_cg(a.hist_c + rd, w4);
+                        ld8f_cg(a.dhist_c + rd, w5);
+#pragma unroll
+                        for (int e = 0; e < 8; ++e) {
+                            dh_t[cu * 8 + e] = w1[e];
+                            dc_t[cu * 8 + e] = w2[e];
+                            cn[cu * 8 + e] = w3[e];
+                            cr[cu * 8 + e] = w4[e];
+                            dc_rd[cu * 8 + e] = w5[e];
+                        }
+                        const __half *gt = a.gates + ((size_t)(t - 1) * B + b) * 4 * H + u;
+#pragma unroll
+                        for (int g = 0; g < 4; ++g) gq[cu][g] = *(const uint4 *)(gt + (size_t)g * H);
+                    }
+                }
+                const bool ok = tc::mbar_wait(&c.tfull[acc], (k >> 1) & 1, limit, c.abort);
+                if (!ok) ws_abort(c, a.err);
+                __syncwarp();
+                if (tc::bar_any(1, E * 32, !ok || *c.abort)) break;
+                tc::tc_fence_after();
+                uint32_t dr[UE];
+                tmem_cols<UE>(taddr + part * UE, dr);
+                tc::tmem_wait_ld();
+                tc::tc_fence_before();
+                __syncwarp();
+                if (lane == 0) tc::mbar_arrive(&c.tempty[acc]);
+#pragma unroll
+                for (int cu = 0; cu < UE / 8; ++cu) {
+                    const int u = u0 + cu * 8;
+                    if (!(row_ok && u < H)) continue;
+                    float v[8];
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) v[e] = dh_src[cu * 8 + e] + __uint_as_float(dr[cu * 8 + e]);
+                    st8f(a.dhist_h + ((size_t)src * B + b) * H + u, v);
+                    if (t >= 1) {
+                        float ig[8], fg[8], gg[8], og[8], d[4][8], dcr[8];
+                        unpack8_f16(gq[cu][0], ig);
+                        unpack8_f16(gq[cu][1], fg);
+                        unpack8_f16(gq[cu][2], gg);
+                        unpack8_f16(gq[cu][3], og);
+#pragma unroll
+                        for (int e = 0; e < 8; ++e) {
+                            const int j = cu * 8 + e;
+                            const float dh = src == t ? v[e] : dh_t[j];  // the state read at t is row t
+                            const float tcn = tanh_hw(cn[j]);
+                            const float dc = dc_t[j] + dh * og[e] * (1.0f - tcn * tcn);
+                            d[0][e] = dc * gg[e] * ig[e] * (1.0f - ig[e]);
+                            d[1][e] = dc * cr[j] * fg[e] * (1.0f - fg[e]);
+                            d[2][e] = dc * ig[e] * (1.0f - gg[e] * gg[e]);
+                            d[3][e] = dh * tcn * og[e] * (1.0f - og[e]);
+                            dcr[e] = dc_rd[j] + dc * fg[e];
+                        }
+                        __nv_bfloat16 *dg = a.dG + ((size_t)(t - 1) * B + b) * 4 * H + u;
+#pragma unroll
+                        for (int g = 0; g < 4; ++g) *(uint4 *)(dg + (size_t)g * H) = pack8_bf16(d[g]);
+                        st8f(a.dhist_c + ((size_t)s1 * B + b) * H + u, dcr);
+                    }
+                }
+            }
+            // the next step reads these rows by TMA: generic writes -> async proxy, then
+            // release the step for this row tile
+            tc::fence_proxy_async_global();
+            __syncwarp();
+            tc::bar_sync(2, E * 32);
+            if (tid == 0) tc::red_release_gpu_add(p.cnt + rt, 1);
+        }
+    }
+
+    // ---------------------------------------------------------------- teardown
+    __syncthreads();
+    if (warp == E && lane == 0) {
+        // copies still in flight after an abort: stages armed but never consumed
+        for (int g = *c.n_consumed; g < *c.n_issued; ++g)
+            tc::mbar_wait(&c.full[g % S], (uint32_t)(g / S) & 1, kDrainLimit, nullptr);
+        if (p.w_res) tc::mbar_wait(c.wbar, 0, kDrainLimit, nullptr);
+    }
+    if (warp == E + 1 && lane == 0) tc::mbar_wait(c.done, 0, kDrainLimit, nullptr);
+    if (cl > 1) tc::cluster_sync();  // nobody leaves while a peer may still multicast into it
+    tc::tc_fence_before();
+    __syncthreads();
+    if (warp == E) tc::tmem_dealloc(tmem, 2 * kCols);
+}
+
+// ------------------------------------------------------------------ planning
+// Measured back-to-back issue cost (cycles) of one M = 128, K = 16 MMA by N, and the
+// extra issue stall of one mbarrier wait between MMA runs.
+double mma_cycles(int N) { return N <= 16 ? 45 : N <= 32 ? 51 : N <= 64 ? 47 : N <= 128 ? 65 : 128; }
+constexpr double kWaitCycles = 300;
+
+struct Variant {
+    int U, EP, G;
+    const void *fn;
+};
+
+template <int U, int EP, int G, bool kFwd>
+Variant variant()
+{
+    return Variant{U, EP, G, (const void *)step_ws<U, EP, G, kFwd>};
+}
+
+const Variant *fwd_variants(int *n)
+{
+    static const Variant v[] = {variant<8, 1, 4, true>(), variant<16, 2, 4, true>(), variant<32, 2, 2, true>()};
+    *n = 3;
+    return v;
+}
+const Variant *bwd_variants(int *n)
+{
+    static const Variant v[] = {variant<16, 2, 4, false>(), variant<32, 2, 4, false>()};
+    *n = 2;
+    return v;
+}
+
+// Largest residency (CTAs per SM) that leaves every CTA its two accumulators in tensor
+// memory (512 columns per SM); shared memory is padded to enforce it.
+uint32_t pad_for_tmem(const void *fn, int threads, uint32_t smem, uint32_t kcols2)
+{
+    const int max_res = std::max(1, (int)(512 / kcols2));
+    for (; smem <= kSmemCap; smem += 4096) {
+        int r = 0;
+        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&r, fn, threads, smem) != cudaSuccess) {
+            cudaGetLastError();
+            return 0;
+        }
+        if (r <= max_res) return smem;
+    }
+    return kSmemCap;
+}
+
+// Plans one variant: cluster sizes 8, 4, 2 (only when multicast is wanted) and 1; the
+// weight tile resident or streamed; the deepest ring (up to two tiles of stages) that
+// fits. The grid is sized from the number of co-resident CTAs (clusters) of that
+// footprint. Cost = row-tile rounds per step x per-tile MMA issue time; ties go to the
+// resident weight tile, then the larger cluster, then the deeper ring.
+bool plan_variant(const Variant &v, bool fwd, int KC, int split, int n_rt, int H, int sms, bool want_mc,
+                  PersistPlan *pl, double *cost)
+{
+    const int NB = fwd ? 4 * v.U : v.U, n_ct = (H + v.U - 1) / v.U;
+    const int threads = 32 * (4 * v.EP + 2);
+    const uint32_t kcols2 = 2u * (NB <= 32 ? 32 : NB <= 64 ? 64 : NB <= 128 ? 128 : 256);
+    const int groups = (split + v.G - 1) / v.G + (KC - split + v.G - 1) / v.G;
+    const uint32_t fixed = 1024 + kBarBytes + 1024 /* static */;
+    bool found = false;
+    double best = 1e30;
+    int best_key = -1;
+    if (cudaFuncSetAttribute(v.fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemCap) != cudaSuccess) {
+        cudaGetLastError();
+        return false;
+    }
+    for (int cl : {8, 4, 2, 1}) {
+        if (cl > 1 && (!want_mc || cl / 2 >= n_ct)) continue;
+        const int pad = (n_ct + cl - 1) / cl * cl;
+        for (int wr : {1, 0}) {
+            const uint32_t wbytes = wr ? (uint32_t)KC * NB * 128 : 0u;
+            const uint32_t stage = ws_stage_bytes(v.G, NB, wr);
+            if (fixed + wbytes + 2 * stage > kSmemCap) continue;
+            const int S = std::min({(int)((kSmemCap - fixed - wbytes) / stage), kMaxStages, std::max(2, 2 * groups)});
+            uint32_t smem = ws_smem_bytes(S, v.G, NB, KC, wr);
+            smem = pad_for_tmem(v.fn, threads, smem, kcols2);
+            if (!smem) continue;
+            int resident = 0;
+            if (cl == 1) {
+                int r = 0;
+                if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&r, v.fn, threads, smem) != cudaSuccess) {
+                    cudaGetLastError();
+                    continue;
+                }
+                resident = r * sms;
+            } else {
+                cudaLaunchConfig_t cfg = {};
+                cfg.gridDim = dim3(pad);
+                cfg.blockDim = dim3(threads);
+                cfg.dynamicSmemBytes = smem;
+                cudaLaunchAttribute at[1];
+                at[0].id = cudaLaunchAttributeClusterDimension;
+                at[0].val.clusterDim.x = cl;
+                at[0].val.clusterDim.y = 1;
+                at[0].val.clusterDim.z = 1;
+                cfg.attrs = at;
+                cfg.numAttrs = 1;
+                int clusters = 0;
+                if (cudaOccupancyMaxActiveClusters(&clusters, v.fn, &cfg) != cudaSuccess) {
+                    cudaGetLastError();
+                    continue;
+                }
+                resident = clusters * cl;
+            }
+            if (resident < pad) continue;
+            const int sl = std::min(n_rt, resident / pad);
+            const int rounds = (n_rt + sl - 1) / sl;
+            const double c = rounds * (KC * 4 * mma_cycles(NB) + groups * kWaitCycles);
+            const int key = wr * 1000 + cl * 20 + S;
+            if (c < best * 0.999 || (c <= best * 1.001 && key > best_key)) {
+                best = c;
+                best_key = key;
+                pl->on = 1;
+                pl->U = v.U;
+                pl->EP = v.EP;
+                pl->G = v.G;
+                pl->S = S;
+                pl->slot = sl;
+                pl->w_res = wr;
+                pl->cl = cl;
+                pl->n_ct = pad;
+                pl->smem = smem;
+                pl->threads = threads;
+                found = true;
+            }
+        }
+    }
+    *cost = best;
+    return found;
+}
+
+bool plan(stacklstm *s, bool fwd, PersistPlan *pl)
+{
+    int n;
+    const Variant *vs = fwd ? fwd_variants(&n) : bwd_variants(&n);
+    const int n_rt = (int)ceil_div(s->B, kRows);
+    const int KC = fwd ? s->kcf : s->kcb, split = fwd ? s->kcx : 0;
+    const char *mc = getenv("STACKLSTM_MULTICAST");
+    const bool mc_on = mc && atoi(mc) != 0;
+    const char *force = getenv(fwd ? "STACKLSTM_FWD_UNITS" : "STACKLSTM_BWD_UNITS");
+    const int force_u = force ? atoi(force) : 0;
+    double best = 1e30;
+    bool found = false;
+    for (int i = 0; i < n; ++i) {
+        if (force_u && vs[i].U != force_u) continue;
+        PersistPlan cand;
+        double cost;
+        const int n_ct = (s->H + vs[i].U - 1) / vs[i].U;
+        // multicast pays only when the column tiles' re-reads of A are a large L2 stream
+        const bool want_mc = mc_on && (double)n_rt * kAStage * KC * n_ct >= 8e6;
+        if (plan_variant(vs[i], fwd, KC, split, n_rt, s->H, s->num_sms, want_mc, &cand, &cost) && cost < best) {
+            best = cost;
+            *pl = cand;
+            found = true;
+        }
+    }
+    if (!found) pl->on = 0;
+    return found;
+}
+
+template <typename... Args>
+cudaError_t launch_coop(const void *fn, const PersistPlan &pl, cudaStream_t st, Args... args)
+{
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(pl.n_ct * pl.slot);
+    cfg.blockDim = dim3(pl.threads);
+    cfg.dynamicSmemBytes = pl.smem;
+    cfg.stream = st;
+    cudaLaunchAttribute at[2];
+    at[0].id = cudaLaunchAttributeCooperative;
+    at[0].val.cooperative = 1;
+    at[1].id = cudaLaunchAttributeClusterDimension;
+    at[1].val.clusterDim.x = pl.cl;
+    at[1].val.clusterDim.y = 1;
+    at[1].val.clusterDim.z = 1;
+    cfg.attrs = at;
+    cfg.numAttrs = 2;
+    void *argv[] = {(void *)&args...};
+    return cudaLaunchKernelExC(&cfg, fn, argv);
+}
+
+const void *find_fn(bool fwd, const PersistPlan &pl)
+{
+    int n;
+    const Variant *vs = fwd ? fwd_variants(&n) : bwd_variants(&n);
+    for (int i = 0; i < n; ++i)
+        if (vs[i].U == pl.U && vs[i].EP == pl.EP && vs[i].G == pl.G) return vs[i].fn;
+    return nullptr;
+}
+
+}  // namespace
+
+bool bf16_plan_fwd_persist(stacklstm *s, PersistPlan *pl) { return plan(s, true, pl); }
+bool bf16_plan_bwd_persist(stacklstm *s, PersistPlan *pl) { return plan(s, false, pl); }
+
+cudaError_t bf16_launch_fwd_persist(stacklstm *s, const StepArgs &a, const CUtensorMap &tm_x, const CUtensorMap &tm_h)
+{
+    const PersistPlan &pl = s->pf;
+    WsArgs p;
+    p.s = a;
+    p.s.S = pl.S;
+    p.n_ct = pl.n_ct;
+    p.n_rt = (int)ceil_div(s->B, kRows);
+    p.n_slot = pl.slot;
+    p.w_res = pl.w_res;
+    p.cl = pl.cl;
+    p.cnt = s->rowcnt;
+    cudaError_t e = cudaMemsetAsync(p.cnt, 0, sizeof(int32_t) * p.n_rt, s->stream);
+    if (e) return e;
+    const void *fn = find_fn(true, pl);
+    if (!fn) return cudaErrorInvalidDeviceFunction;
+    e = launch_coop(fn, pl, s->stream, tm_x, tm_h, p);
+    if (e) return e;
+    s->launches += 1;
+    return cudaGetLastError();
+}
+
+cudaError_t bf16_launch_bwd_persist(stacklstm *s, const StepArgs &a, const CUtensorMap &tm_g)
+{
+    const PersistPlan &pl = s->pb;
+    WsArgs p;
+    p.s = a;
+    p.s.S = pl.S;
+    p.s.kcx = 0;
+    p.n_ct = pl.n_ct;
+    p.n_rt = (int)ceil_div(s->B, kRows);
+    p.n_slot = pl.slot;
+    p.w_res = pl.w_res;
+    p.cl = pl.cl;
+    p.cnt = s->rowcnt + p.n_rt;
+    cudaError_t e = cudaMemsetAsync(p.cnt, 0, sizeof(int32_t) * p.n_rt, s->stream);
+    if (e) return e;
+    const void *fn = find_fn(false, pl);
+    if (!fn) return cudaErrorInvalidDeviceFunction;
+    e = launch_coop(fn, pl, s->stream, tm_g, tm_g, p);
+    if (e) return e;
+    s->launches += 1;
+    return cudaGetLastError();
+}
+
+}  // namespace sl

@@ -11,6 +11,21 @@
 
 #include "../../include/stacklstm.h"
 
+// A planned persistent step kernel: one cooperative launch runs all T steps.
+struct PersistPlan {
+    int on = 0;         // 1: persistent; 0: one launch per step
+    int U = 0;          // hidden units per column tile
+    int EP = 1;         // epilogue warps per tensor-memory lane quadrant (4 * EP epilogue warps)
+    int G = 1;          // contraction chunks per ring stage
+    int S = 0;          // ring stages
+    int slot = 0;       // CTAs per column tile (each takes every slot-th row tile)
+    int w_res = 0;      // weight tile resident in shared memory
+    int cl = 1;         // thread-block cluster size along the column tiles (A multicast)
+    int n_ct = 0;       // column tiles, padded to a multiple of cl
+    unsigned smem = 0;  // dynamic shared memory per CTA
+    int threads = 0;    // threads per CTA
+};
+
 // The handle: problem sizes, stream, and the device workspace it owns.
 struct stacklstm {
     int T = 0, B = 0, I = 0, H = 0;
@@ -55,13 +70,8 @@ struct stacklstm {
     int kcx = 0, kcf = 0, kcb = 0;  // 64-wide contraction chunks: x part, forward total, backward
     int sf = 0, sb = 0, sx = 0, sw = 0;  // ring depths: forward, backward, dx, dW
     alignas(64) unsigned char tmaps[6][128] = {};  // TMA descriptors (bf16_path.cu)
-    // persistent step kernels (one launch for all T steps); 0 = per-step launches
-    int pf = 0, pb = 0;            // forward / backward run persistent
-    int pf_slot = 0, pb_slot = 0;  // CTAs per column tile (each takes every n_slot-th row tile)
-    int pf_wres = 0, pb_wres = 0;  // weight tile resident in shared memory
-    int pf_S = 0, pb_S = 0;        // ring depths of the persistent kernels
-    int pf_cl = 1, pb_cl = 1;      // thread-block cluster sizes (column tiles sharing A by multicast)
-    int pf_nct = 0, pb_nct = 0;    // column tiles, padded to a multiple of the cluster size
+    // persistent step kernels (one launch for all T steps; bf16_persist.cu)
+    PersistPlan pf, pb;            // forward, backward (on = 0: one launch per step)
     int32_t *rowcnt = nullptr;     // [2][row tiles] completed steps per row tile
     int nx = 0, nxt = 0;     // input gradient: columns per tile, number of column tiles
     int dw_mt = 0, dw_nt = 0, dw_split = 0;  // weight gradient: row tiles, column tiles, splits
