@@ -47,6 +47,7 @@ struct WsArgs {
     int w_res;               // 1: weight tile resident in shared memory
     int cl;                  // cluster size along the column tiles (1: no multicast)
     int32_t *cnt;            // [n_rt] completed steps per row tile, zero at launch
+    int vec32;               // H % 16 == 0: 16-unit groups of 16-bit rows are 32-byte aligned
 };
 
 // Dynamic shared memory: [weight tile (w_res)][S stages: G A chunks, then G weight
@@ -149,6 +150,283 @@ __device__ __forceinline__ void tmem_cols(uint32_t taddr, uint32_t (&r)[UE])
 __device__ __forceinline__ int group_end(int c0, int G, int split, int KC)
 {
     return min(c0 + G, c0 < split ? split : KC);
+}
+
+// ------------------------------------------------------------- vector access
+// NG (8 or 16) consecutive values of one row per thread: 16- or 32-byte accesses, so a
+// lane fills whole 32-byte L2 sectors where the row layout allows (fp32: always; 16-bit
+// rows: when H is a multiple of 16). Addresses are NG * element size aligned.
+__device__ __forceinline__ void st_v8(void *p, const uint32_t *w)
+{
+    asm volatile("st.global.v8.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8};" ::"l"(p), "r"(w[0]), "r"(w[1]), "r"(w[2]),
+                 "r"(w[3]), "r"(w[4]), "r"(w[5]), "r"(w[6]), "r"(w[7])
+                 : "memory");
+}
+__device__ __forceinline__ void ld_v8(const void *p, uint32_t *w)
+{
+    asm volatile("ld.global.cg.v8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
+                 : "=r"(w[0]), "=r"(w[1]), "=r"(w[2]), "=r"(w[3]), "=r"(w[4]), "=r"(w[5]), "=r"(w[6]), "=r"(w[7])
+                 : "l"(p)
+                 : "memory");
+}
+__device__ __forceinline__ void st_v4(void *p, const uint32_t *w)
+{
+    *(uint4 *)p = make_uint4(w[0], w[1], w[2], w[3]);
+}
+__device__ __forceinline__ void ld_v4(const void *p, uint32_t *w)
+{
+    const uint4 v = __ldcg((const uint4 *)p);
+    w[0] = v.x; w[1] = v.y; w[2] = v.z; w[3] = v.w;
+}
+// NG 16-bit values (raw words, NG / 2 of them)
+template <int NG>
+__device__ __forceinline__ void st_h(void *p, const uint32_t *w)
+{
+    if constexpr (NG == 16) st_v8(p, w); else st_v4(p, w);
+}
+template <int NG>
+__device__ __forceinline__ void ld_h(const void *p, uint32_t *w)
+{
+    if constexpr (NG == 16) ld_v8(p, w); else ld_v4(p, w);
+}
+// NG fp32 values (32-byte pieces)
+template <int NG>
+__device__ __forceinline__ void st_f(float *p, const float *v)
+{
+#pragma unroll
+    for (int i = 0; i < NG / 8; ++i) st_v8(p + 8 * i, (const uint32_t *)(v + 8 * i));
+}
+template <int NG>
+__device__ __forceinline__ void ld_f(const float *p, float *v)
+{
+#pragma unroll
+    for (int i = 0; i < NG / 8; ++i) ld_v8(p + 8 * i, (uint32_t *)(v + 8 * i));
+}
+template <int NG>
+__device__ __forceinline__ void pack_bf16(const float *v, uint32_t *w)
+{
+#pragma unroll
+    for (int i = 0; i < NG / 2; ++i) {
+        __nv_bfloat162 t = __floats2bfloat162_rn(v[2 * i], v[2 * i + 1]);
+        w[i] = *(uint32_t *)&t;
+    }
+}
+template <int NG>
+__device__ __forceinline__ void pack_f16(const float *v, uint32_t *w)
+{
+#pragma unroll
+    for (int i = 0; i < NG / 2; ++i) {
+        __half2 t = __floats2half2_rn(v[2 * i], v[2 * i + 1]);
+        w[i] = *(uint32_t *)&t;
+    }
+}
+template <int NG>
+__device__ __forceinline__ void unpack_f16(const uint32_t *w, float *v)
+{
+#pragma unroll
+    for (int i = 0; i < NG / 2; ++i) {
+        const float2 f = __half22float2(*(const __half2 *)&w[i]);
+        v[2 * i] = f.x;
+        v[2 * i + 1] = f.y;
+    }
+}
+
+// ------------------------------------------------------------------ epilogue
+struct EpiCtx {
+    WCtl c;
+    uint32_t tmem;
+    int q, part, lane, tid;  // TMEM lane quadrant, unit part, lane, thread
+    int ct, slot, n_mine, n_tiles;
+    long long limit;
+};
+
+// All tiles of one epilogue thread: row 32 q + lane of each tile, units
+// ct * U + part * UE .. + UE, in access groups of NG units.
+template <int U, int EP, int NG, bool kFwd>
+__device__ __forceinline__ void epilogue_loop(const StepArgs &a, const WsArgs &p, const EpiCtx &e,
+                                              const float *s_bias)
+{
+    constexpr int E = 4 * EP, UE = U / EP;
+    constexpr int NB = kFwd ? 4 * U : U;
+    constexpr uint32_t kCols = TmemCols<NB>::value;
+    const int T = a.T, B = a.B, H = a.H;
+    const uint32_t lane_off = (uint32_t)(e.q * 32) << 16;
+    const int u0 = e.ct * U + e.part * UE;  // first unit of this thread
+    for (int k = 0; k < e.n_tiles; ++k) {
+        const int ks = k / e.n_mine, rt = e.slot + (k % e.n_mine) * p.n_slot;
+        const int t = kFwd ? ks : T - 1 - ks;
+        const int b = rt * kRows + e.q * 32 + e.lane;
+        const bool row_ok = b < B;
+        const int acc = k & 1;
+        const uint32_t taddr = e.tmem + acc * kCols + lane_off;
+        if (k + 1 < e.n_tiles) {
+            // the next tile's epilogue operands into L2 now (their loads then wait on L2,
+            // not HBM); a row the current tile is about to write is harmless to prefetch
+            const int ks1 = (k + 1) / e.n_mine, rt1 = e.slot + ((k + 1) % e.n_mine) * p.n_slot;
+            const int t1 = kFwd ? ks1 : T - 1 - ks1;
+            const int b1 = rt1 * kRows + e.q * 32 + e.lane;
+            if (b1 < B && u0 < H) {
+                const int src1 = a.top[(size_t)t1 * B + b1];
+                if constexpr (kFwd) {
+                    tc::prefetch_l2(a.hist_c + ((size_t)src1 * B + b1) * H + u0);
+                    tc::prefetch_l2(a.hr + ((size_t)a.top[(size_t)(t1 + 1) * B + b1] * B + b1) * H + u0);
+                } else {
+                    tc::prefetch_l2(a.dhist_h + ((size_t)src1 * B + b1) * H + u0);
+                    if (t1 >= 1) {
+                        const int s11 = a.top[(size_t)(t1 - 1) * B + b1];
+                        const size_t wr = ((size_t)t1 * B + b1) * H + u0, rd = ((size_t)s11 * B + b1) * H + u0;
+                        tc::prefetch_l2(a.dhist_h + wr);
+                        tc::prefetch_l2(a.dhist_c + wr);
+                        tc::prefetch_l2(a.hist_c + wr);
+                        tc::prefetch_l2(a.hist_c + rd);
+                        tc::prefetch_l2(a.dhist_c + rd);
+                        const __half *gt = a.gates + ((size_t)(t1 - 1) * B + b1) * 4 * H + u0;
+#pragma unroll
+                        for (int g = 0; g < 4; ++g) tc::prefetch_l2(gt + (size_t)g * H);
+                    }
+                }
+            }
+        }
+        if constexpr (kFwd) {
+            // operands this thread wrote itself at earlier steps (same rows and units):
+            // c_read, and the older top the next step reads when step t does not push
+            const int src = row_ok ? a.top[(size_t)t * B + b] : 0;
+            const int s_next = row_ok ? a.top[(size_t)(t + 1) * B + b] : 0;
+            const bool is_new = s_next == t + 1;
+            float cr[UE];
+            uint32_t hc[UE / 2];
+#pragma unroll
+            for (int cg = 0; cg < UE / NG; ++cg) {
+                const int u = u0 + cg * NG;
+                if (row_ok && u < H) {
+                    ld_f<NG>(a.hist_c + ((size_t)src * B + b) * H + u, cr + cg * NG);
+                    if (!is_new) ld_h<NG>(a.hr + ((size_t)s_next * B + b) * H + u, hc + cg * NG / 2);
+                }
+            }
+            const bool ok = tc::mbar_wait(&e.c.tfull[acc], (k >> 1) & 1, e.limit, e.c.abort);
+            if (!ok) ws_abort(e.c, a.err);
+            __syncwarp();
+            if (tc::bar_any(1, E * 32, !ok || *e.c.abort)) break;
+            tc::tc_fence_after();
+            uint32_t zr[4][UE];
+#pragma unroll
+            for (int g = 0; g < 4; ++g) tmem_cols<UE>(taddr + g * U + e.part * UE, zr[g]);
+            tc::tmem_wait_ld();
+            tc::tc_fence_before();
+            __syncwarp();
+            if (e.lane == 0) tc::mbar_arrive(&e.c.tempty[acc]);
+#pragma unroll
+            for (int cg = 0; cg < UE / NG; ++cg) {
+                const int u = u0 + cg * NG;
+                if (!(row_ok && u < H)) continue;
+                float cn[NG], hn[NG], gv[4][NG];
+#pragma unroll
+                for (int i = 0; i < NG; ++i) {
+                    const int j = cg * NG + i, jb = e.part * UE + j;
+                    const float ig = sigm(__uint_as_float(zr[0][j]) + s_bias[jb]);
+                    const float fg = sigm(__uint_as_float(zr[1][j]) + s_bias[U + jb]);
+                    const float gg = tanh_hw(__uint_as_float(zr[2][j]) + s_bias[2 * U + jb]);
+                    const float og = sigm(__uint_as_float(zr[3][j]) + s_bias[3 * U + jb]);
+                    cn[i] = fmaf(fg, cr[j], ig * gg);
+                    hn[i] = og * tanh_hw(cn[i]);
+                    gv[0][i] = ig; gv[1][i] = fg; gv[2][i] = gg; gv[3][i] = og;
+                }
+                // history row t + 1, the h operand of step t + 1 (h' when step t pushed,
+                // else the older top), the activated gates (fp16) for the backward
+                const size_t w = ((size_t)(t + 1) * B + b) * H + u;
+                uint32_t hb[NG / 2];
+                pack_bf16<NG>(hn, hb);
+                st_h<NG>(a.hist_h + w, hb);
+                st_h<NG>(a.hr + w, is_new ? hb : hc + cg * NG / 2);
+                st_f<NG>(a.hist_c + w, cn);
+                __half *gt = a.gates + ((size_t)t * B + b) * 4 * H + u;
+#pragma unroll
+                for (int g = 0; g < 4; ++g) {
+                    uint32_t gw[NG / 2];
+                    pack_f16<NG>(gv[g], gw);
+                    st_h<NG>(gt + (size_t)g * H, gw);
+                }
+            }
+        } else {
+            // Every epilogue operand: the gradient history of this thread's units is written
+            // only by this thread (or zeroed before the launch); gates and cell states come
+            // from the forward.
+            const int src = row_ok ? a.top[(size_t)t * B + b] : 0;
+            const int s1 = (row_ok && t >= 1) ? a.top[(size_t)(t - 1) * B + b] : 0;
+            float dh_src[UE], dh_t[UE], dc_t[UE], cn[UE], cr[UE], dc_rd[UE];
+            uint32_t gq[4][UE / 2];
+#pragma unroll
+            for (int cg = 0; cg < UE / NG; ++cg) {
+                const int u = u0 + cg * NG;
+                if (!(row_ok && u < H)) continue;
+                ld_f<NG>(a.dhist_h + ((size_t)src * B + b) * H + u, dh_src + cg * NG);
+                if (t >= 1) {
+                    const size_t wr = ((size_t)t * B + b) * H + u, rd = ((size_t)s1 * B + b) * H + u;
+                    ld_f<NG>(a.dhist_h + wr, dh_t + cg * NG);
+                    ld_f<NG>(a.dhist_c + wr, dc_t + cg * NG);
+                    ld_f<NG>(a.hist_c + wr, cn + cg * NG);
+                    ld_f<NG>(a.hist_c + rd, cr + cg * NG);
+                    ld_f<NG>(a.dhist_c + rd, dc_rd + cg * NG);
+                    const __half *gt = a.gates + ((size_t)(t - 1) * B + b) * 4 * H + u;
+#pragma unroll
+                    for (int g = 0; g < 4; ++g) ld_h<NG>(gt + (size_t)g * H, gq[g] + cg * NG / 2);
+                }
+            }
+            const bool ok = tc::mbar_wait(&e.c.tfull[acc], (k >> 1) & 1, e.limit, e.c.abort);
+            if (!ok) ws_abort(e.c, a.err);
+            __syncwarp();
+            if (tc::bar_any(1, E * 32, !ok || *e.c.abort)) break;
+            tc::tc_fence_after();
+            uint32_t dr[UE];
+            tmem_cols<UE>(taddr + e.part * UE, dr);
+            tc::tmem_wait_ld();
+            tc::tc_fence_before();
+            __syncwarp();
+            if (e.lane == 0) tc::mbar_arrive(&e.c.tempty[acc]);
+#pragma unroll
+            for (int cg = 0; cg < UE / NG; ++cg) {
+                const int u = u0 + cg * NG;
+                if (!(row_ok && u < H)) continue;
+                float v[NG];
+#pragma unroll
+                for (int i = 0; i < NG; ++i) v[i] = dh_src[cg * NG + i] + __uint_as_float(dr[cg * NG + i]);
+                st_f<NG>(a.dhist_h + ((size_t)src * B + b) * H + u, v);
+                if (t >= 1) {
+                    float ig[NG], fg[NG], gg[NG], og[NG], d[4][NG], dcr[NG];
+                    unpack_f16<NG>(gq[0] + cg * NG / 2, ig);
+                    unpack_f16<NG>(gq[1] + cg * NG / 2, fg);
+                    unpack_f16<NG>(gq[2] + cg * NG / 2, gg);
+                    unpack_f16<NG>(gq[3] + cg * NG / 2, og);
+#pragma unroll
+                    for (int i = 0; i < NG; ++i) {
+                        const int j = cg * NG + i;
+                        const float dh = src == t ? v[i] : dh_t[j];  // the state read at t is row t
+                        const float tcn = tanh_hw(cn[j]);
+                        const float dc = dc_t[j] + dh * og[i] * (1.0f - tcn * tcn);
+                        d[0][i] = dc * gg[i] * ig[i] * (1.0f - ig[i]);
+                        d[1][i] = dc * cr[j] * fg[i] * (1.0f - fg[i]);
+                        d[2][i] = dc * ig[i] * (1.0f - gg[i] * gg[i]);
+                        d[3][i] = dh * tcn * og[i] * (1.0f - og[i]);
+                        dcr[i] = dc_rd[j] + dc * fg[i];
+                    }
+                    __nv_bfloat16 *dg = a.dG + ((size_t)(t - 1) * B + b) * 4 * H + u;
+#pragma unroll
+                    for (int g = 0; g < 4; ++g) {
+                        uint32_t w[NG / 2];
+                        pack_bf16<NG>(d[g], w);
+                        st_h<NG>(dg + (size_t)g * H, w);
+                    }
+                    st_f<NG>(a.dhist_c + ((size_t)s1 * B + b) * H + u, dcr);
+                }
+            }
+        }
+        // the next step reads these rows by TMA: generic writes -> async proxy, then
+        // release the step for this row tile
+        tc::fence_proxy_async_global();
+        __syncwarp();
+        tc::bar_sync(2, E * 32);
+        if (e.tid == 0) tc::red_release_gpu_add(p.cnt + rt, 1);
+    }
 }
 
 // ------------------------------------------------------------------ the kernel
@@ -300,150 +578,12 @@ step_ws(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtens
         __syncwarp();
     } else {
         // ------------------------------------------------------------ epilogue
-        const int q = warp & 3, part = warp >> 2;
-        const uint32_t lane_off = (uint32_t)(q * 32) << 16;
-        for (int k = 0; k < n_tiles; ++k) {
-            const int ks = k / n_mine, rt = slot + (k % n_mine) * p.n_slot;
-            const int t = kFwd ? ks : T - 1 - ks;
-            const int b = rt * kRows + q * 32 + lane;
-            const bool row_ok = b < B;
-            const int u0 = ct * U + part * UE;  // first unit of this thread
-            const int acc = k & 1;
-            const uint32_t taddr = tmem + acc * kCols + lane_off;
-            if constexpr (kFwd) {
-                // operands this thread wrote itself at earlier steps (same rows and units):
-                // c_read, and the older top the next step reads when step t does not push
-                const int src = row_ok ? a.top[(size_t)t * B + b] : 0;
-                const int s_next = row_ok ? a.top[(size_t)(t + 1) * B + b] : 0;
-                const bool is_new = s_next == t + 1;
-                float cr[UE];
-                uint4 hc[UE / 8];
-#pragma unroll
-                for (int cu = 0; cu < UE / 8; ++cu) {
-                    const int u = u0 + cu * 8;
-                    float v[8] = {0, 0, 0, 0, 0, 0, 0, 0};
-                    hc[cu] = make_uint4(0, 0, 0, 0);
-                    if (row_ok && u < H) {
-                        ld8f_cg(a.hist_c + ((size_t)src * B + b) * H + u, v);
-                        if (!is_new) hc[cu] = __ldcg((const uint4 *)(a.hr + ((size_t)s_next * B + b) * H + u));
-                    }
-#pragma unroll
-                    for (int e = 0; e < 8; ++e) cr[cu * 8 + e] = v[e];
-                }
-                const bool ok = tc::mbar_wait(&c.tfull[acc], (k >> 1) & 1, limit, c.abort);
-                if (!ok) ws_abort(c, a.err);
-                __syncwarp();
-                if (tc::bar_any(1, E * 32, !ok || *c.abort)) break;
-                tc::tc_fence_after();
-                uint32_t zr[4][UE];
-#pragma unroll
-                for (int g = 0; g < 4; ++g) tmem_cols<UE>(taddr + g * U + part * UE, zr[g]);
-                tc::tmem_wait_ld();
-                tc::tc_fence_before();
-                __syncwarp();
-                if (lane == 0) tc::mbar_arrive(&c.tempty[acc]);
-#pragma unroll
-                for (int cu = 0; cu < UE / 8; ++cu) {
-                    const int u = u0 + cu * 8;
-                    if (row_ok && u < H) {
-                        float z[4][8];
-#pragma unroll
-                        for (int g = 0; g < 4; ++g)
-#pragma unroll
-                            for (int e = 0; e < 8; ++e) z[g][e] = __uint_as_float(zr[g][cu * 8 + e]);
-                        const int j = part * UE + cu * 8;
-                        fwd_cell8(a, t, b, u, z, s_bias + j, s_bias + U + j, s_bias + 2 * U + j, s_bias + 3 * U + j,
-                                  cr + cu * 8, is_new, hc[cu]);
-                    }
-                }
-            } else {
-                // Every epilogue operand: the gradient history of this thread's units is
-                // written only by this thread (or zeroed before the launch); gates and cell
-                // states come from the forward.
-                const int src = row_ok ? a.top[(size_t)t * B + b] : 0;
-                const int s1 = (row_ok && t >= 1) ? a.top[(size_t)(t - 1) * B + b] : 0;
-                float dh_src[UE], dh_t[UE], dc_t[UE], cn[UE], cr[UE], dc_rd[UE];
-                uint4 gq[UE / 8][4];
-#pragma unroll
-                for (int cu = 0; cu < UE / 8; ++cu) {
-                    const int u = u0 + cu * 8;
-                    const bool uok = row_ok && u < H;
-                    float v[8] = {0, 0, 0, 0, 0, 0, 0, 0};
-                    if (uok) ld8f_cg(a.dhist_h + ((size_t)src * B + b) * H + u, v);
-#pragma unroll
-                    for (int e = 0; e < 8; ++e) dh_src[cu * 8 + e] = v[e];
-                    if (uok && t >= 1) {
-                        const size_t wr = ((size_t)t * B + b) * H + u, rd = ((size_t)s1 * B + b) * H + u;
-                        float w1[8], w2[8], w3[8], w4[8], w5[8];
-                        ld8f_cg(a.dhist_h + wr, w1);
-                        ld8f_cg(a.dhist_c + wr, w2);
-                        ld8f_cg(a.hist_c + wr, w3);
-                        ld8f_cg(a.hist_c + rd, w4);
-                        ld8f_cg(a.dhist_c + rd, w5);
-#pragma unroll
-                        for (int e = 0; e < 8; ++e) {
-                            dh_t[cu * 8 + e] = w1[e];
-                            dc_t[cu * 8 + e] = w2[e];
-                            cn[cu * 8 + e] = w3[e];
-                            cr[cu * 8 + e] = w4[e];
-                            dc_rd[cu * 8 + e] = w5[e];
-                        }
-                        const __half *gt = a.gates + ((size_t)(t - 1) * B + b) * 4 * H + u;
-#pragma unroll
-                        for (int g = 0; g < 4; ++g) gq[cu][g] = *(const uint4 *)(gt + (size_t)g * H);
-                    }
-                }
-                const bool ok = tc::mbar_wait(&c.tfull[acc], (k >> 1) & 1, limit, c.abort);
-                if (!ok) ws_abort(c, a.err);
-                __syncwarp();
-                if (tc::bar_any(1, E * 32, !ok || *c.abort)) break;
-                tc::tc_fence_after();
-                uint32_t dr[UE];
-                tmem_cols<UE>(taddr + part * UE, dr);
-                tc::tmem_wait_ld();
-                tc::tc_fence_before();
-                __syncwarp();
-                if (lane == 0) tc::mbar_arrive(&c.tempty[acc]);
-#pragma unroll
-                for (int cu = 0; cu < UE / 8; ++cu) {
-                    const int u = u0 + cu * 8;
-                    if (!(row_ok && u < H)) continue;
-                    float v[8];
-#pragma unroll
-                    for (int e = 0; e < 8; ++e) v[e] = dh_src[cu * 8 + e] + __uint_as_float(dr[cu * 8 + e]);
-                    st8f(a.dhist_h + ((size_t)src * B + b) * H + u, v);
-                    if (t >= 1) {
-                        float ig[8], fg[8], gg[8], og[8], d[4][8], dcr[8];
-                        unpack8_f16(gq[cu][0], ig);
-                        unpack8_f16(gq[cu][1], fg);
-                        unpack8_f16(gq[cu][2], gg);
-                        unpack8_f16(gq[cu][3], og);
-#pragma unroll
-                        for (int e = 0; e < 8; ++e) {
-                            const int j = cu * 8 + e;
-                            const float dh = src == t ? v[e] : dh_t[j];  // the state read at t is row t
-                            const float tcn = tanh_hw(cn[j]);
-                            const float dc = dc_t[j] + dh * og[e] * (1.0f - tcn * tcn);
-                            d[0][e] = dc * gg[e] * ig[e] * (1.0f - ig[e]);
-                            d[1][e] = dc * cr[j] * fg[e] * (1.0f - fg[e]);
-                            d[2][e] = dc * ig[e] * (1.0f - gg[e] * gg[e]);
-                            d[3][e] = dh * tcn * og[e] * (1.0f - og[e]);
-                            dcr[e] = dc_rd[j] + dc * fg[e];
-                        }
-                        __nv_bfloat16 *dg = a.dG + ((size_t)(t - 1) * B + b) * 4 * H + u;
-#pragma unroll
-                        for (int g = 0; g < 4; ++g) *(uint4 *)(dg + (size_t)g * H) = pack8_bf16(d[g]);
-                        st8f(a.dhist_c + ((size_t)s1 * B + b) * H + u, dcr);
-                    }
-                }
-            }
-            // the next step reads these rows by TMA: generic writes -> async proxy, then
-            // release the step for this row tile
-            tc::fence_proxy_async_global();
-            __syncwarp();
-            tc::bar_sync(2, E * 32);
-            if (tid == 0) tc::red_release_gpu_add(p.cnt + rt, 1);
-        }
+        constexpr int NG = UE % 16 == 0 ? 16 : 8;
+        const EpiCtx e{c, tmem, warp & 3, warp >> 2, lane, tid, ct, slot, n_mine, n_tiles, limit};
+        if (NG == 16 && p.vec32)
+            epilogue_loop<U, EP, NG, kFwd>(a, p, e, s_bias);
+        else
+            epilogue_loop<U, EP, 8, kFwd>(a, p, e, s_bias);
     }
 
     // ---------------------------------------------------------------- teardown
@@ -480,14 +620,16 @@ Variant variant()
 
 const Variant *fwd_variants(int *n)
 {
-    static const Variant v[] = {variant<8, 1, 4, true>(), variant<16, 2, 4, true>(), variant<32, 2, 2, true>()};
-    *n = 3;
+    static const Variant v[] = {variant<8, 1, 4, true>(),  variant<16, 1, 4, true>(), variant<16, 2, 4, true>(),
+                                variant<32, 2, 2, true>(), variant<32, 4, 2, true>()};
+    *n = 5;
     return v;
 }
 const Variant *bwd_variants(int *n)
 {
-    static const Variant v[] = {variant<16, 2, 4, false>(), variant<32, 2, 4, false>()};
-    *n = 2;
+    static const Variant v[] = {variant<16, 1, 4, false>(), variant<16, 2, 4, false>(), variant<32, 2, 4, false>(),
+                                variant<32, 4, 4, false>()};
+    *n = 4;
     return v;
 }
 
@@ -602,10 +744,15 @@ bool plan(stacklstm *s, bool fwd, PersistPlan *pl)
     const bool mc_on = mc && atoi(mc) != 0;
     const char *force = getenv(fwd ? "STACKLSTM_FWD_UNITS" : "STACKLSTM_BWD_UNITS");
     const int force_u = force ? atoi(force) : 0;
+    // epilogue warp groups: one for 16-unit tiles (a thread then holds 16 units, whole
+    // 32-byte sectors), two for 32-unit tiles (measured best); STACKLSTM_*_EP overrides
+    const char *force_ep = getenv(fwd ? "STACKLSTM_FWD_EP" : "STACKLSTM_BWD_EP");
     double best = 1e30;
     bool found = false;
     for (int i = 0; i < n; ++i) {
         if (force_u && vs[i].U != force_u) continue;
+        const int want_ep = force_ep ? atoi(force_ep) : vs[i].U == 16 ? 1 : 2;
+        if (vs[i].U >= 16 && vs[i].EP != want_ep) continue;
         PersistPlan cand;
         double cost;
         const int n_ct = (s->H + vs[i].U - 1) / vs[i].U;
@@ -668,6 +815,7 @@ cudaError_t bf16_launch_fwd_persist(stacklstm *s, const StepArgs &a, const CUten
     p.w_res = pl.w_res;
     p.cl = pl.cl;
     p.cnt = s->rowcnt;
+    p.vec32 = s->H % 16 == 0;
     cudaError_t e = cudaMemsetAsync(p.cnt, 0, sizeof(int32_t) * p.n_rt, s->stream);
     if (e) return e;
     const void *fn = find_fn(true, pl);
@@ -691,6 +839,7 @@ cudaError_t bf16_launch_bwd_persist(stacklstm *s, const StepArgs &a, const CUten
     p.w_res = pl.w_res;
     p.cl = pl.cl;
     p.cnt = s->rowcnt + p.n_rt;
+    p.vec32 = s->H % 16 == 0;
     cudaError_t e = cudaMemsetAsync(p.cnt, 0, sizeof(int32_t) * p.n_rt, s->stream);
     if (e) return e;
     const void *fn = find_fn(false, pl);

@@ -98,6 +98,12 @@ __device__ __forceinline__ bool bar_any(int id, int nthreads, bool v)
     return r != 0;
 }
 
+// Brings the line holding p into L2 (no register result, no completion to wait for).
+__device__ __forceinline__ void prefetch_l2(const void *p)
+{
+    asm volatile("prefetch.global.L2 [%0];" ::"l"(p));
+}
+
 // ------------------------------------------------------------------ cp.async (16 B)
 // src_bytes = 0 writes 16 zero bytes without reading global memory.
 __device__ __forceinline__ void cp_async16(uint32_t dst, const void *src, uint32_t src_bytes)
