@@ -175,4 +175,9 @@ bool bf16_plan_bwd_persist(stacklstm *s, PersistPlan *pl);
 cudaError_t bf16_launch_fwd_persist(stacklstm *s, const StepArgs &a, const CUtensorMap &tm_x, const CUtensorMap &tm_h);
 cudaError_t bf16_launch_bwd_persist(stacklstm *s, const StepArgs &a, const CUtensorMap &tm_g);
 
+// ---- weight / bias gradients (bf16_dw.cu)
+cudaError_t bf16_plan_dw(stacklstm *s);
+cudaError_t bf16_launch_dw(stacklstm *s, const CUtensorMap &tm_x, const CUtensorMap &tm_h, const CUtensorMap &tm_g,
+                           float *dW, float *dbias);
+
 }  // namespace sl

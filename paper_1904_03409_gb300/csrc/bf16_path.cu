@@ -21,9 +21,9 @@
 // units, which now has its complete (dh', dc'): it writes dG_{t-1} (bf16) and adds
 // dc_read. Every (row, unit) of the gradient history has one owner: no atomics.
 //
-// After the loop: dx = dG W_x^T (one K-major contraction over all T*B rows) and
-// dW = [x ; h_read]^T dG with dbias as one extra all-ones operand row (an MN-major,
-// split-K contraction whose partial sums are reduced in a fixed order).
+// After the loop: dx = dG W_x^T (one K-major contraction over all T*B rows); dW and dbias
+// are in bf16_dw.cu. The persistent (one launch for all steps) versions of the step
+// kernels are in bf16_persist.cu.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 #include <stdio.h>
@@ -380,133 +380,6 @@ __global__ void __launch_bounds__(kThreads, 1) dx_tc(const __grid_constant__ CUt
     finish(c, tmem, kCols);
 }
 
-// ------------------------------------------------------------- weight gradient
-// dW_ext[m][n] = sum_r A[r][m] dG[r][n] over r = t * B + b, where A[r] = [x_t ; h_read ; 1]
-// (m = I + H is the all-ones row, which yields dbias). Both operands are read MN-major:
-// 64 consecutive r per chunk; each 64-wide MN block is 64 rows of 128 swizzled bytes.
-// dG blocks, x blocks and h blocks (each fully inside x or inside h; the h operand of
-// step t is hr[t], rows t * B + b) arrive by TMA; a block straddling x and h, or holding
-// the ones row, is copied piece by piece.
-struct DwArgs {
-    int B, I, H;
-    const __nv_bfloat16 *x, *hr, *ones;
-    int R;
-    int n_tiles_n, split, S;
-    float *part;  // [split][mt * 128][nt * 256]
-    size_t ld_part, rows_part;
-    long long limit;
-    int32_t *err;
-};
-
-__global__ void __launch_bounds__(kThreads, 1)
-dw_tc(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtensorMap tm_h,
-      const __grid_constant__ CUtensorMap tm_g, DwArgs a)
-{
-    constexpr int NB = 256;
-    constexpr uint32_t kCols = 256;
-    constexpr uint32_t kBlk = 64 * 128;  // one MN block of a chunk
-    extern __shared__ uint8_t smem_raw[];
-    const Ctl c = carve(smem_raw, a.S, NB);
-    const int tid = threadIdx.x, warp = tid >> 5;
-    const int mt = blockIdx.x / a.n_tiles_n, nt = blockIdx.x % a.n_tiles_n, sp = blockIdx.y;
-    const int I = a.I, H = a.H;
-    const int RC = (a.R + kChunk - 1) / kChunk;
-    const int c_lo = (int)((long long)RC * sp / a.split), c_hi = (int)((long long)RC * (sp + 1) / a.split);
-    const int KC = c_hi - c_lo;
-    const uint32_t tmem = prologue(c, a.S, kCols);
-
-    auto in_x = [&](int m0) { return m0 + 64 <= I; };
-    auto in_h = [&](int m0) { return m0 >= I && m0 + 64 <= I + H; };
-    auto tma = [&](int it, int s, uint64_t *bar) {
-        const int r0 = (c_lo + it) * kChunk;
-        uint32_t bytes = 4 * kBlk;
-        for (int blk = 0; blk < 2; ++blk) {
-            const int m0 = mt * kRows + blk * 64;
-            if (in_x(m0) || in_h(m0)) bytes += kBlk;
-        }
-        tc::mbar_arrive_expect_tx(bar, bytes);
-        for (int blk = 0; blk < 2; ++blk) {
-            const int m0 = mt * kRows + blk * 64;
-            if (in_x(m0)) tc::tma_load_2d(c.a0 + s * kAStage + blk * kBlk, &tm_x, m0, r0, bar);
-            else if (in_h(m0)) tc::tma_load_2d(c.a0 + s * kAStage + blk * kBlk, &tm_h, m0 - I, r0, bar);
-        }
-        for (int nb = 0; nb < 4; ++nb)
-            tc::tma_load_2d(c.b0 + s * c.b_bytes + nb * kBlk, &tm_g, nt * NB + nb * 64, r0, bar);
-    };
-    // thread -> (r-row rr, block blk): one 128-byte row segment of eight 16-byte pieces
-    auto gather = [&](int it, int s) {
-        const int rr = tid & 63, blk = tid >> 6;
-        const int m0 = mt * kRows + blk * 64;
-        if (in_x(m0) || in_h(m0)) return;  // arrives by TMA
-        const int r = (c_lo + it) * kChunk + rr;
-        const uint32_t dst = c.a0 + s * kAStage + blk * kBlk;
-        const bool r_ok = r < a.R;
-        const __nv_bfloat16 *hrow = a.hr + (size_t)(r_ok ? r : 0) * H;
-#pragma unroll
-        for (int q = 0; q < 8; ++q) {
-            const int m = m0 + q * 8;
-            const void *p = a.ones;
-            uint32_t bytes = 0;
-            if (r_ok) {
-                if (m < I) {
-                    p = a.x + (size_t)r * I + m;
-                    bytes = 16;
-                } else if (m < I + H) {
-                    p = hrow + (m - I);
-                    bytes = 16;
-                } else if (m == I + H) {
-                    bytes = 16;
-                }
-            }
-            tc::cp_async16(dst + sw128(rr, q), p, bytes);
-        }
-    };
-    auto issue = [&](int s, int j) {
-        constexpr uint32_t idesc = tc::idesc_bf16(NB, 1, 1);
-        const uint32_t as = c.a0 + s * kAStage, bs = c.b0 + s * c.b_bytes;
-#pragma unroll
-        for (int k = 0; k < kChunk / 16; ++k)  // 16 r-rows = two 8-row groups = 2048 bytes
-            tc::mma_bf16(tmem, tc::smem_desc(as + k * 2048, kBlk, 1024), tc::smem_desc(bs + k * 2048, kBlk, 1024),
-                         idesc, (j | k) != 0);
-    };
-    if (KC > 0) mainloop<true>(c, a.S, KC, -1, a.limit, a.err, tma, gather, issue);
-    if (!*c.abort) {
-        const size_t m = (size_t)mt * kRows + tid;
-        float *dst = a.part + ((size_t)sp * a.rows_part + m) * a.ld_part + (size_t)nt * NB;
-        const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
-#pragma unroll 1
-        for (int cu = 0; cu < NB / 16; ++cu) {
-            float v[16];
-            tc::tmem_ld16(trow + cu * 16, v);
-            if (KC == 0)
-                for (int e = 0; e < 16; ++e) v[e] = 0.0f;
-            *(float4 *)(dst + cu * 16) = make_float4(v[0], v[1], v[2], v[3]);
-            *(float4 *)(dst + cu * 16 + 4) = make_float4(v[4], v[5], v[6], v[7]);
-            *(float4 *)(dst + cu * 16 + 8) = make_float4(v[8], v[9], v[10], v[11]);
-            *(float4 *)(dst + cu * 16 + 12) = make_float4(v[12], v[13], v[14], v[15]);
-        }
-    }
-    finish(c, tmem, kCols);
-}
-
-// Fixed-order reduction of the split-K partials into dW and dbias.
-__global__ void dw_reduce(int K, int G, int split, const float *__restrict__ part, size_t rows_part, size_t ld,
-                          float *__restrict__ dW, float *__restrict__ dbias)
-{
-    const size_t n = (size_t)(K + 1) * G;
-    for (size_t e = blockIdx.x * (size_t)blockDim.x + threadIdx.x; e < n; e += (size_t)gridDim.x * blockDim.x) {
-        const size_t m = e / G, col = e - m * G;
-        float acc = 0.0f;
-        for (int s = 0; s < split; ++s) acc += part[((size_t)s * rows_part + m) * ld + col];
-        if (m < (size_t)K) {
-            if (dW) dW[m * G + col] = acc;
-        } else if (dbias) {
-            dbias[col] = acc;
-        }
-    }
-}
-
-
 // ------------------------------------------------------------------ packing
 // Forward operand: for column tile ct, rows n = g * U + j hold gate g of hidden unit
 // ct * U + j; each row is the matching column of W over the contraction
@@ -633,10 +506,10 @@ std::string bf16_describe(const stacklstm *s)
              "bf16 tcgen05; row tiles %d; chunks fwd %d (x %d) bwd %d; "
              "forward %s U=%d [EP %d G %d ring %d slots %d cluster %d col tiles %d w_res %d smem %u threads %d]; "
              "backward %s U=%d [EP %d G %d ring %d slots %d cluster %d col tiles %d w_res %d smem %u threads %d]; "
-             "step rings fwd %d bwd %d; dx N=%d x%d ring %d; dW %dx%d tiles x%d splits ring %d",
+             "step rings fwd %d bwd %d; dx N=%d x%d ring %d; dW %dx%d tiles of 128x%d x%d splits ring %d",
              rt, s->kcf, s->kcx, s->kcb, f.on ? "persistent" : "per-step", s->uf, f.EP, f.G, f.S, f.slot, f.cl, f.n_ct,
              f.w_res, f.smem, f.threads, b.on ? "persistent" : "per-step", s->ub, b.EP, b.G, b.S, b.slot, b.cl, b.n_ct,
-             b.w_res, b.smem, b.threads, s->sf, s->sb, s->nx, s->nxt, s->sx, s->dw_mt, s->dw_nt, s->dw_split, s->sw);
+             b.w_res, b.smem, b.threads, s->sf, s->sb, s->nx, s->nxt, s->sx, s->dw_mt, s->dw_nt, s->dw_ntile, s->dw_split, s->sw);
     return buf;
 }
 
@@ -659,17 +532,14 @@ cudaError_t bf16_prepare(stacklstm *s)
     s->kcb = (int)ceil_div(4 * H, kChunk);
     s->nx = pick_dx_n(I);
     s->nxt = (int)ceil_div(I, s->nx);
-    s->dw_mt = (int)ceil_div(I + H + 1, kRows);
-    s->dw_nt = (int)ceil_div(4 * H, 256);
-    const size_t R = (size_t)T * B, RC = ceil_div(R, kChunk);
-    s->dw_split = (int)std::max<size_t>(1, std::min<size_t>(sms / std::max(1, s->dw_mt * s->dw_nt), RC / 2));
+    const size_t R = (size_t)T * B;
     const char *lim = getenv("STACKLSTM_WAIT_LIMIT_CYCLES");
     s->wait_limit = lim ? atoll(lim) : 4000000000LL;
     if ((e = allow_smem(fwd_step_tc<32>)) || (e = allow_smem(fwd_step_tc<16>)) || (e = allow_smem(fwd_step_tc<8>)) ||
         (e = allow_smem(bwd_step_tc<32>)) || (e = allow_smem(bwd_step_tc<16>)) || (e = allow_smem(dx_tc<32>)) ||
-        (e = allow_smem(dx_tc<64>)) || (e = allow_smem(dx_tc<128>)) || (e = allow_smem(dx_tc<256>)) ||
-        (e = allow_smem(dw_tc)))
+        (e = allow_smem(dx_tc<64>)) || (e = allow_smem(dx_tc<128>)) || (e = allow_smem(dx_tc<256>)))
         return e;
+    if ((e = bf16_plan_dw(s))) return e;
 
     // persistent step kernels unless disabled (STACKLSTM_STEP_KERNELS=1 keeps one launch per step)
     const char *per_step = getenv("STACKLSTM_STEP_KERNELS");
@@ -680,14 +550,12 @@ cudaError_t bf16_prepare(stacklstm *s)
     s->sf = pick_stages(s->kcf, 4 * s->uf, ceil_div(H, s->uf) * (size_t)rt, sms);
     s->sb = pick_stages(s->kcb, s->ub, ceil_div(H, s->ub) * (size_t)rt, sms);
     s->sx = pick_stages(s->kcb, s->nx, s->nxt * ceil_div(R, kRows), sms);
-    s->sw = pick_stages((int)ceil_div(RC, s->dw_split), 256, (size_t)s->dw_mt * s->dw_nt * s->dw_split, sms);
 
     const size_t fwd_bytes = (size_t)std::max<size_t>(ceil_div(H, s->uf), s->pf.on ? s->pf.n_ct : 0) * s->kcf * 4 *
                              s->uf * 128;
     const size_t bwd_bytes = (size_t)std::max<size_t>(ceil_div(H, s->ub), s->pb.on ? s->pb.n_ct : 0) * s->kcb * s->ub *
                              128;
     const size_t dx_bytes = (size_t)s->nxt * s->kcb * s->nx * 128;
-    s->dw_part_elems = (size_t)s->dw_split * s->dw_mt * kRows * s->dw_nt * 256;
     void *p;
     if ((e = cudaMalloc(&p, fwd_bytes))) return e;
     s->allocs.push_back(p); s->w_fwd = p;
@@ -697,10 +565,6 @@ cudaError_t bf16_prepare(stacklstm *s)
     s->allocs.push_back(p); s->w_dx = p;
     if ((e = cudaMalloc(&p, s->dw_part_elems * sizeof(float)))) return e;
     s->allocs.push_back(p); s->dw_part = (float *)p;
-    if ((e = cudaMalloc(&p, 16))) return e;
-    s->allocs.push_back(p); s->ones = p;
-    const uint16_t one[8] = {0x3F80, 0, 0, 0, 0, 0, 0, 0};  // bf16 1.0 followed by zeros
-    if ((e = cudaMemcpy(s->ones, one, 16, cudaMemcpyHostToDevice))) return e;
     if (s->pf.on || s->pb.on) {
         if ((e = cudaMalloc(&p, 2 * sizeof(int32_t) * rt))) return e;
         s->allocs.push_back(p);
@@ -808,21 +672,7 @@ cudaError_t bf16_dx(stacklstm *s, float *dx)
 cudaError_t bf16_dw(stacklstm *s, float *dW, float *dbias)
 {
     if (!dW && !dbias) return cudaSuccess;
-    const int T = s->T, B = s->B, I = s->I, H = s->H;
-    DwArgs w;
-    w.B = B; w.I = I; w.H = H;
-    w.x = (const __nv_bfloat16 *)s->x_saved; w.hr = (const __nv_bfloat16 *)s->hr;
-    w.ones = (const __nv_bfloat16 *)s->ones;
-    w.R = T * B; w.n_tiles_n = s->dw_nt; w.split = s->dw_split; w.S = s->sw; w.part = s->dw_part;
-    w.ld_part = (size_t)s->dw_nt * 256; w.rows_part = (size_t)s->dw_mt * kRows;
-    w.limit = s->wait_limit; w.err = s->err;
-    cudaError_t e = launch(dw_tc, dim3(s->dw_mt * s->dw_nt, s->dw_split), smem_bytes(s->sw, 256), s->stream, false,
-                           map(s, kMapX64), map(s, kMapH64), map(s, kMapG64), w);
-    if (e) return e;
-    dw_reduce<<<grid_for(s, (size_t)(I + H + 1) * 4 * H), 256, 0, s->stream>>>(
-        I + H, 4 * H, s->dw_split, s->dw_part, w.rows_part, w.ld_part, dW, dbias);
-    s->launches += 2;
-    return cudaGetLastError();
+    return bf16_launch_dw(s, map(s, kMapX64), map(s, kMapH64), map(s, kMapG64), dW, dbias);
 }
 
 }  // namespace sl

@@ -62,7 +62,6 @@ struct stacklstm {
     void *w_dx = nullptr;   // bf16: input-gradient operand tiles
     float *dw_part = nullptr;  // split-K partials of the weight-gradient contraction
     size_t dw_part_elems = 0;
-    void *ones = nullptr;      // bf16: one 16-byte piece {1, 0, ..., 0} (bias-gradient row)
     const void *x_saved = nullptr;  // the caller's x, read again by the weight gradient
 
     // bf16 tensor-core plan (bf16_path.cu)
@@ -74,7 +73,8 @@ struct stacklstm {
     PersistPlan pf, pb;            // forward, backward (on = 0: one launch per step)
     int32_t *rowcnt = nullptr;     // [2][row tiles] completed steps per row tile
     int nx = 0, nxt = 0;     // input gradient: columns per tile, number of column tiles
-    int dw_mt = 0, dw_nt = 0, dw_split = 0;  // weight gradient: row tiles, column tiles, splits
+    int dw_mt = 0, dw_nt = 0, dw_split = 0;  // weight gradient: m tiles, column tiles, splits
+    int dw_ntile = 0;                        // weight gradient: gate columns per tile
     long long wait_limit = 0;  // clock cycles one bounded device-side wait may spin
 
     // launch accounting and optional per-phase event timing (api.cu)
