@@ -18,6 +18,7 @@ from __future__ import annotations
 import argparse
 import hashlib
 import json
+import re
 import math
 import os
 import statistics
@@ -42,11 +43,11 @@ def dist_env():
     return int(os.environ.get("RANK", 0)), int(os.environ.get("WORLD_SIZE", 1)), int(os.environ.get("LOCAL_RANK", 0))
 
 
-def get_workload(name):
+def get_workload(name, T=None):
     from paper_1904_03409_gb300 import workloads as wl
     if name.startswith("sweep:"):
         return wl.config_workload("sweep", B=int(name.split(":")[1]))
-    return wl.config_workload(name)
+    return wl.config_workload(name, T=T)
 
 
 def describe(w):
@@ -70,10 +71,10 @@ def work_per_inst_step(I, H):
     """Flops and bytes per instance-step, per kernel phase and for the whole step (bf16
     path). Whole step: F = 24 H (I + H), Q = 8 I + 46 H."""
     return {
-        "forward": {"flops": 8 * H * (I + H), "bytes": 2 * I + 12 * H, "kernel": "fwd_step_tc"},
-        "backward": {"flops": 8 * H * H, "bytes": 34 * H, "kernel": "bwd_step_tc"},
-        "dx": {"flops": 8 * H * I, "bytes": 4 * I, "kernel": "dx_tc"},
-        "dw": {"flops": 8 * H * (I + H + 1), "bytes": 2 * I, "kernel": "dw_tc"},
+        "forward": {"flops": 8 * H * (I + H), "bytes": 2 * I + 12 * H},
+        "backward": {"flops": 8 * H * H, "bytes": 34 * H},
+        "dx": {"flops": 8 * H * I, "bytes": 4 * I},
+        "dw": {"flops": 8 * H * (I + H + 1), "bytes": 2 * I},
         "step": {"flops": 24 * H * (I + H), "bytes": 8 * I + 46 * H},
     }
 
@@ -91,7 +92,24 @@ def roofline_of(work_flops, work_bytes, seconds, peaks, src, sustained):
             "frac": ach / peaks["hbm_gbs"], "peak_source": "%s HBM copy" % src}
 
 
-def kernel_traffic(kernel, workload):
+def phase_kernel(plan, phase):
+    """(kernel name, source file) of the kernel that does a phase's work, from the plan."""
+    if phase in ("forward", "backward"):
+        m = re.search(phase + r" (persistent|per-step) U=(\d+)", plan)
+        if m and m.group(1) == "persistent":
+            return "step_ws<U=%s,%s>" % (m.group(2), phase), "bf16_persist.cu"
+        return ("fwd_step_tc" if phase == "forward" else "bwd_step_tc"), "bf16_path.cu"
+    if phase == "dx":
+        return "dx_tc", "bf16_path.cu"
+    return "dw_ws", "bf16_dw.cu"
+
+
+def source_sha(fname):
+    src = os.path.join(ROOT, "paper_1904_03409_gb300", "csrc", fname)
+    return hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+
+
+def kernel_traffic(kernel, fname, workload):
     """DRAM bytes per launch of `kernel` from the committed ncu summary, if it was taken
     on this workload with the kernel source as it is now; else None."""
     p = os.path.join(ROOT, "profiles", "dram_traffic.json")
@@ -99,8 +117,7 @@ def kernel_traffic(kernel, workload):
         return None
     with open(p) as f:
         d = json.load(f)
-    src = os.path.join(ROOT, "paper_1904_03409_gb300", "csrc", "bf16_path.cu")
-    sha = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+    sha = source_sha(fname)
     for e in d.get("entries", []):
         if e.get("kernel") == kernel and e.get("workload") == workload and e.get("source_sha") == sha:
             return e.get("dram_bytes_per_launch")
@@ -179,7 +196,7 @@ def run_ours(args, rank, world, local):
         build.build()
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
-    w = get_workload(args.workload)
+    w = get_workload(args.workload, args.T)
     res = measure_workload(w, args.steps, args.warmup, local, world, sample_clocks=True, e2e=True)
 
     line = {"metric": METRIC, "value": res["value"], "unit": UNIT, "n_gpus": world, "steps": res["steps"],
@@ -191,7 +208,8 @@ def run_ours(args, rank, world, local):
                        "l2": "flushed between timed steps (256 MiB write outside the timed events)",
                        "parallelism": "replicas" if world > 1 else "single GPU"},
             "roofline": res["roofline"], "step_roofline": res["step_roofline"], "phases_ms_per_step":
-            res["phases"], "e2e": res["e2e"], "gpu_launches": res["gpu_launches"], "clocks": res["clocks"]}
+            res["phases"], "e2e": res["e2e"], "gpu_launches": res["gpu_launches"], "clocks": res["clocks"],
+            "plan": res["plan"]}
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(w, args.cpu_seconds)
     if rank == 0 and world == 1 and not args.no_extra and args.workload == "parser64":
@@ -221,6 +239,7 @@ def measure_workload(w, steps, warmup, local, world, sample_clocks, e2e):
     dev = torch.device("cuda", local)
     stream = torch.cuda.current_stream(dev)
     hd = bd.stacklstm_create(w.T, w.B, w.I, w.H, bd.SL_BF16 if w.dtype == "bf16" else bd.SL_FP32, local, stream)
+    plan = bd.stacklstm_plan(hd)
     bd.stacklstm_set_async(hd, True)
     ins = runner.upload(w, local)
     out = runner.alloc_outputs(w, local, forward_outputs=False)
@@ -268,21 +287,26 @@ def measure_workload(w, steps, warmup, local, world, sample_clocks, e2e):
     wk = work_per_inst_step(w.I, w.H)
     phase_ms = {p: timing[p][0] / steps for p in timing}
     dom = max(("forward", "backward", "dx", "dw"), key=lambda p: phase_ms[p])
-    # the step phases run T launches of one kernel; dx and dw one launch each
-    per_launch_units = w.B if dom in ("forward", "backward") else w.B * w.T
-    launches_per_step = w.T if dom in ("forward", "backward") else 1
+    kname, kfile = phase_kernel(plan, dom)
+    # a persistent step kernel is one launch over all T steps; the per-step kernels are T
+    # launches of B instance-steps each; dx and dW are one contraction over all T * B rows
+    # (dW: plus its fixed-order reduction of the split partials)
+    per_step_kernels = dom in ("forward", "backward") and "persistent" not in kname and "step_ws" not in kname
+    per_launch_units = w.B if per_step_kernels else w.B * w.T
+    launches_per_step = w.T if per_step_kernels else 1
     launch_s = phase_ms[dom] / 1e3 / launches_per_step
     rf = roofline_of(wk[dom]["flops"] * per_launch_units, wk[dom]["bytes"] * per_launch_units, launch_s, peaks, src,
                      sustained=True)
-    rf.update({"kernel": wk[dom]["kernel"], "phase": dom, "launch_us": launch_s * 1e6,
+    rf.update({"kernel": kname, "phase": dom, "launch_us": launch_s * 1e6,
                "units_per_launch": per_launch_units, "unit_of_work": "instance-step",
                "algorithmic_flops_per_unit": wk[dom]["flops"], "algorithmic_bytes_per_unit": wk[dom]["bytes"],
-               "traffic": kernel_traffic(wk[dom]["kernel"], w.name)})
+               "traffic": kernel_traffic(kname, kfile, w.name)})
     sec = total_ms / 1e3 / steps
     srf = roofline_of(wk["step"]["flops"] * w.B * w.T, wk["step"]["bytes"] * w.B * w.T, sec, peaks, src,
                       sustained=True)
     res = {"value": world * w.B * w.T * steps / (total_ms / 1e3), "ms_per_step": total_ms / steps, "steps": steps,
            "roofline": rf, "step_roofline": srf, "phases": {p: round(v, 4) for p, v in phase_ms.items()},
+           "plan": plan,
            "gpu_launches": int(n_launch), "clocks": clocks.summary() if clocks else None}
     if e2e:
         res["e2e"] = measure_e2e(w, hd, ins, out, steps, world, local, flush)
@@ -382,7 +406,7 @@ def cpu_baseline(w, seconds):
 def run_reference(args, rank, world):
     if rank != 0:
         return
-    w = get_workload(args.workload)
+    w = get_workload(args.workload, args.T)
     inst, cores = oracle_sample(w, args.ref_step_seconds)
     for _ in range(args.warmup):
         run_oracle(w, inst, cores)
@@ -412,6 +436,8 @@ def main():
     ap.add_argument("--ref-step-seconds", type=float, default=3.0, help="oracle work per reference step")
     ap.add_argument("--no-extra", action="store_true", help="skip the large/stress side measurements")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--T", type=int, default=None,
+                    help="fewer steps for tiny/large/stress (a smaller case of the same shape, for profiling)")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")

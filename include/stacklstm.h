@@ -128,13 +128,15 @@ sl_status stacklstm_backward(stacklstm_t s, const float *d_top_h, const float *d
  * contiguous run of kernel launches on the handle's stream.
  */
 typedef enum {
-    SL_PHASE_PREPASS = 0,  /* op validation and the index prepass                      */
-    SL_PHASE_FORWARD = 1,  /* weight packing and the T forward step launches           */
-    SL_PHASE_OUTPUTS = 2,  /* optional forward outputs (y, h_stack, c_stack, p_traj)   */
-    SL_PHASE_BACKWARD = 3, /* gradient seeding and the T backward step launches        */
-    SL_PHASE_DX = 4,       /* the input-gradient contraction dx = dG W_x^T             */
-    SL_PHASE_DW = 5,       /* the weight- and bias-gradient contraction and reduction  */
-    SL_NUM_PHASES = 6
+    SL_PHASE_PREPASS = 0,    /* op validation and the index prepass                              */
+    SL_PHASE_FORWARD = 1,    /* the forward steps (one persistent launch, or T launches)         */
+    SL_PHASE_OUTPUTS = 2,    /* optional forward outputs (y, h_stack, c_stack, p_traj)           */
+    SL_PHASE_BACKWARD = 3,   /* the reverse-time backward steps (one launch, or T / 2T launches) */
+    SL_PHASE_DX = 4,         /* the input-gradient contraction dx = dG W_x^T                     */
+    SL_PHASE_DW = 5,         /* the weight- and bias-gradient contraction and its reduction      */
+    SL_PHASE_FWD_SETUP = 6,  /* weight packing and the initial state, before the forward steps   */
+    SL_PHASE_BWD_SETUP = 7,  /* clearing and seeding the gradient history, last-step pointwise   */
+    SL_NUM_PHASES = 8
 } sl_phase;
 
 /*

@@ -190,7 +190,7 @@ def stacklstm_pointers_noalloc(ops, p_traj, src, stream=None):
         raise StackLSTMError(st, "stacklstm_pointers_noalloc")
 
 
-PHASES = ("prepass", "forward", "outputs", "backward", "dx", "dw")
+PHASES = ("prepass", "forward", "outputs", "backward", "dx", "dw", "fwd_setup", "bwd_setup")
 
 
 def stacklstm_set_timing(hd: StackLSTMHandle, on: bool):

@@ -250,12 +250,20 @@ sl_status stacklstm_forward(stacklstm_t s, const void *x, const int8_t *ops, con
         if ((e = sl::launch_prepass(s, ops))) return cuda_fail(s, e, "prepass");
     }
     {
+        Phase ph(s, SL_PHASE_FWD_SETUP);
+        if (s->dt == SL_FP32)
+            e = sl::fp32_forward_setup(s, (const float *)h0, c0, (const float *)W);
+        else
+            e = sl::bf16_forward_setup(s, (const __nv_bfloat16 *)x, (const __nv_bfloat16 *)h0, c0,
+                                       (const __nv_bfloat16 *)W);
+        if (e) return cuda_fail(s, e, "forward setup");
+    }
+    {
         Phase ph(s, SL_PHASE_FORWARD);
         if (s->dt == SL_FP32)
-            e = sl::fp32_forward(s, (const float *)x, (const float *)h0, c0, (const float *)W, bias);
+            e = sl::fp32_forward_steps(s, (const float *)x, (const float *)W, bias);
         else
-            e = sl::bf16_forward(s, (const __nv_bfloat16 *)x, (const __nv_bfloat16 *)h0, c0,
-                                 (const __nv_bfloat16 *)W, bias);
+            e = sl::bf16_forward_steps(s, bias);
         if (e) return cuda_fail(s, e, "forward");
     }
     {
@@ -294,10 +302,14 @@ sl_status stacklstm_backward(stacklstm_t s, const float *d_top_h, const float *d
     const size_t hist_bytes = sizeof(float) * (size_t)(T + 1) * B * H;
     cudaError_t e;
     {
-        Phase ph(s, SL_PHASE_BACKWARD);
+        Phase ph(s, SL_PHASE_BWD_SETUP);
         if ((e = cudaMemsetAsync(s->dhist_h, 0, hist_bytes, s->stream))) return cuda_fail(s, e, "clear");
         if ((e = cudaMemsetAsync(s->dhist_c, 0, hist_bytes, s->stream))) return cuda_fail(s, e, "clear");
         if ((e = sl::launch_seed_grads(s, d_top_h, dy))) return cuda_fail(s, e, "seed");
+        if (s->dt == SL_BF16 && (e = sl::bf16_backward_setup(s))) return cuda_fail(s, e, "backward setup");
+    }
+    {
+        Phase ph(s, SL_PHASE_BACKWARD);
         e = s->dt == SL_FP32 ? sl::fp32_backward_steps(s) : sl::bf16_backward_steps(s);
         if (e) return cuda_fail(s, e, "backward");
     }

@@ -579,8 +579,8 @@ cudaError_t bf16_prepare(stacklstm *s)
     return cudaSuccess;
 }
 
-cudaError_t bf16_forward(stacklstm *s, const __nv_bfloat16 *x, const __nv_bfloat16 *h0, const float *c0,
-                         const __nv_bfloat16 *W, const float *bias)
+cudaError_t bf16_forward_setup(stacklstm *s, const __nv_bfloat16 *x, const __nv_bfloat16 *h0, const float *c0,
+                               const __nv_bfloat16 *W)
 {
     const int T = s->T, B = s->B, I = s->I, H = s->H;
     cudaError_t e;
@@ -601,7 +601,14 @@ cudaError_t bf16_forward(stacklstm *s, const __nv_bfloat16 *x, const __nv_bfloat
     pack_rows<<<grid_for(s, (size_t)s->nxt * s->kcb * s->nx * kChunk), 256, 0, s->stream>>>(
         W, H, 0, I, s->nx, s->kcb, s->nxt, (__nv_bfloat16 *)s->w_dx);
     s->launches += 3;
-    if ((e = cudaGetLastError())) return e;
+    return cudaGetLastError();
+}
+
+cudaError_t bf16_forward_steps(stacklstm *s, const float *bias)
+{
+    const int T = s->T, B = s->B, H = s->H;
+    const int nctf = std::max((int)ceil_div(H, s->uf), s->pf.on ? s->pf.n_ct : 0);
+    cudaError_t e;
     if (s->pf.on)
         return bf16_launch_fwd_persist(s, step_args(s, bias, s->w_fwd, s->kcx, s->kcf, s->pf.S), map(s, kMapX128),
                                        map(s, kMapH128));
@@ -623,14 +630,20 @@ cudaError_t bf16_forward(stacklstm *s, const __nv_bfloat16 *x, const __nv_bfloat
     return cudaGetLastError();
 }
 
+// Pointwise backward of the last step, before the reverse loop.
+cudaError_t bf16_backward_setup(stacklstm *s)
+{
+    const StepArgs a = step_args(s, nullptr, s->w_bwd, 0, s->kcb, s->sb);
+    pointwise_last<<<grid_for(s, (size_t)s->B * (s->H / 8)), 256, 0, s->stream>>>(a);
+    s->launches += 1;
+    return cudaGetLastError();
+}
+
 cudaError_t bf16_backward_steps(stacklstm *s)
 {
     const int T = s->T, B = s->B, H = s->H;
     cudaError_t e;
     const StepArgs a = step_args(s, nullptr, s->w_bwd, 0, s->kcb, s->sb);
-    pointwise_last<<<grid_for(s, (size_t)B * (H / 8)), 256, 0, s->stream>>>(a);
-    s->launches += 1;
-    if ((e = cudaGetLastError())) return e;
     if (s->pb.on) return bf16_launch_bwd_persist(s, step_args(s, nullptr, s->w_bwd, 0, s->kcb, s->pb.S), map(s, kMapG128));
     const dim3 grid(ceil_div(H, s->ub), ceil_div(B, kRows));
     const size_t smem = smem_bytes(s->sb, s->ub);

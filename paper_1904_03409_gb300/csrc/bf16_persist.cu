@@ -153,6 +153,9 @@ __device__ __forceinline__ int group_end(int c0, int G, int split, int KC)
 }
 
 // ------------------------------------------------------------- vector access
+#ifndef LD_V8_OP
+#define LD_V8_OP "ld.global.cg.v8.b32"
+#endif
 // NG (8 or 16) consecutive values of one row per thread: 16- or 32-byte accesses, so a
 // lane fills whole 32-byte L2 sectors where the row layout allows (fp32: always; 16-bit
 // rows: when H is a multiple of 16). Addresses are NG * element size aligned.
@@ -164,7 +167,7 @@ __device__ __forceinline__ void st_v8(void *p, const uint32_t *w)
 }
 __device__ __forceinline__ void ld_v8(const void *p, uint32_t *w)
 {
-    asm volatile("ld.global.cg.v8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
+    asm volatile(LD_V8_OP " {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
                  : "=r"(w[0]), "=r"(w[1]), "=r"(w[2]), "=r"(w[3]), "=r"(w[4]), "=r"(w[5]), "=r"(w[6]), "=r"(w[7])
                  : "l"(p)
                  : "memory");
@@ -348,66 +351,77 @@ __device__ __forceinline__ void epilogue_loop(const StepArgs &a, const WsArgs &p
                 }
             }
         } else {
-            // Every epilogue operand: the gradient history of this thread's units is written
-            // only by this thread (or zeroed before the launch); gates and cell states come
-            // from the forward.
+            // Epilogue operands: the gradient history of this thread's units is written only
+            // by this thread (or zeroed before the launch); gates and cell states come from
+            // the forward. With one access group per thread they are loaded before the
+            // accumulator wait; with several, group by group (their lines are already on
+            // their way to L2), which bounds the registers they hold.
+            constexpr int NGRP = UE / NG;
+            constexpr bool kEarly = UE <= 16;
+            constexpr int NO = kEarly ? UE : NG;  // units whose operands are held at once
             const int src = row_ok ? a.top[(size_t)t * B + b] : 0;
             const int s1 = (row_ok && t >= 1) ? a.top[(size_t)(t - 1) * B + b] : 0;
-            float dh_src[UE], dh_t[UE], dc_t[UE], cn[UE], cr[UE], dc_rd[UE];
-            uint32_t gq[4][UE / 2];
-#pragma unroll
-            for (int cg = 0; cg < UE / NG; ++cg) {
-                const int u = u0 + cg * NG;
-                if (!(row_ok && u < H)) continue;
-                ld_f<NG>(a.dhist_h + ((size_t)src * B + b) * H + u, dh_src + cg * NG);
+            float dh_src[NO], dh_t[NO], dc_t[NO], cn[NO], cr[NO], dc_rd[NO];
+            uint32_t gq[4][NO / 2];
+            // operands of units u .. u + NG - 1 into slot j (units j * NG ..) of the arrays
+            auto load_ops = [&](int u, int j) {
+                ld_f<NG>(a.dhist_h + ((size_t)src * B + b) * H + u, dh_src + j * NG);
                 if (t >= 1) {
                     const size_t wr = ((size_t)t * B + b) * H + u, rd = ((size_t)s1 * B + b) * H + u;
-                    ld_f<NG>(a.dhist_h + wr, dh_t + cg * NG);
-                    ld_f<NG>(a.dhist_c + wr, dc_t + cg * NG);
-                    ld_f<NG>(a.hist_c + wr, cn + cg * NG);
-                    ld_f<NG>(a.hist_c + rd, cr + cg * NG);
-                    ld_f<NG>(a.dhist_c + rd, dc_rd + cg * NG);
+                    ld_f<NG>(a.dhist_h + wr, dh_t + j * NG);
+                    ld_f<NG>(a.dhist_c + wr, dc_t + j * NG);
+                    ld_f<NG>(a.hist_c + wr, cn + j * NG);
+                    ld_f<NG>(a.hist_c + rd, cr + j * NG);
+                    ld_f<NG>(a.dhist_c + rd, dc_rd + j * NG);
                     const __half *gt = a.gates + ((size_t)(t - 1) * B + b) * 4 * H + u;
 #pragma unroll
-                    for (int g = 0; g < 4; ++g) ld_h<NG>(gt + (size_t)g * H, gq[g] + cg * NG / 2);
+                    for (int g = 0; g < 4; ++g) ld_h<NG>(gt + (size_t)g * H, gq[g] + j * NG / 2);
                 }
-            }
+            };
+            if (kEarly)
+#pragma unroll
+                for (int cg = 0; cg < NGRP; ++cg)
+                    if (row_ok && u0 + cg * NG < H) load_ops(u0 + cg * NG, cg);
             const bool ok = tc::mbar_wait(&e.c.tfull[acc], (k >> 1) & 1, e.limit, e.c.abort);
             if (!ok) ws_abort(e.c, a.err);
             __syncwarp();
             if (tc::bar_any(1, E * 32, !ok || *e.c.abort)) break;
             tc::tc_fence_after();
-            uint32_t dr[UE];
-            tmem_cols<UE>(taddr + e.part * UE, dr);
-            tc::tmem_wait_ld();
-            tc::tc_fence_before();
-            __syncwarp();
-            if (e.lane == 0) tc::mbar_arrive(&e.c.tempty[acc]);
 #pragma unroll
-            for (int cg = 0; cg < UE / NG; ++cg) {
+            for (int cg = 0; cg < NGRP; ++cg) {
                 const int u = u0 + cg * NG;
+                const int j = kEarly ? cg : 0;  // operand slot of this group
+                uint32_t dr[NG];
+                tmem_cols<NG>(taddr + e.part * UE + cg * NG, dr);
+                tc::tmem_wait_ld();
+                if (cg == NGRP - 1) {
+                    tc::tc_fence_before();
+                    __syncwarp();
+                    if (e.lane == 0) tc::mbar_arrive(&e.c.tempty[acc]);
+                }
                 if (!(row_ok && u < H)) continue;
+                if (!kEarly) load_ops(u, 0);
                 float v[NG];
 #pragma unroll
-                for (int i = 0; i < NG; ++i) v[i] = dh_src[cg * NG + i] + __uint_as_float(dr[cg * NG + i]);
+                for (int i = 0; i < NG; ++i) v[i] = dh_src[j * NG + i] + __uint_as_float(dr[i]);
                 st_f<NG>(a.dhist_h + ((size_t)src * B + b) * H + u, v);
                 if (t >= 1) {
                     float ig[NG], fg[NG], gg[NG], og[NG], d[4][NG], dcr[NG];
-                    unpack_f16<NG>(gq[0] + cg * NG / 2, ig);
-                    unpack_f16<NG>(gq[1] + cg * NG / 2, fg);
-                    unpack_f16<NG>(gq[2] + cg * NG / 2, gg);
-                    unpack_f16<NG>(gq[3] + cg * NG / 2, og);
+                    unpack_f16<NG>(gq[0] + j * NG / 2, ig);
+                    unpack_f16<NG>(gq[1] + j * NG / 2, fg);
+                    unpack_f16<NG>(gq[2] + j * NG / 2, gg);
+                    unpack_f16<NG>(gq[3] + j * NG / 2, og);
 #pragma unroll
                     for (int i = 0; i < NG; ++i) {
-                        const int j = cg * NG + i;
-                        const float dh = src == t ? v[i] : dh_t[j];  // the state read at t is row t
-                        const float tcn = tanh_hw(cn[j]);
-                        const float dc = dc_t[j] + dh * og[i] * (1.0f - tcn * tcn);
+                        const int q = j * NG + i;
+                        const float dh = src == t ? v[i] : dh_t[q];  // the state read at t is row t
+                        const float tcn = tanh_hw(cn[q]);
+                        const float dc = dc_t[q] + dh * og[i] * (1.0f - tcn * tcn);
                         d[0][i] = dc * gg[i] * ig[i] * (1.0f - ig[i]);
-                        d[1][i] = dc * cr[j] * fg[i] * (1.0f - fg[i]);
+                        d[1][i] = dc * cr[q] * fg[i] * (1.0f - fg[i]);
                         d[2][i] = dc * ig[i] * (1.0f - gg[i] * gg[i]);
                         d[3][i] = dh * tcn * og[i] * (1.0f - og[i]);
-                        dcr[i] = dc_rd[j] + dc * fg[i];
+                        dcr[i] = dc_rd[q] + dc * fg[i];
                     }
                     __nv_bfloat16 *dg = a.dG + ((size_t)(t - 1) * B + b) * 4 * H + u;
 #pragma unroll
@@ -628,8 +642,8 @@ const Variant *fwd_variants(int *n)
 const Variant *bwd_variants(int *n)
 {
     static const Variant v[] = {variant<16, 1, 4, false>(), variant<16, 2, 4, false>(), variant<32, 2, 4, false>(),
-                                variant<32, 4, 4, false>()};
-    *n = 4;
+                                variant<32, 4, 4, false>(), variant<64, 2, 2, false>()};
+    *n = 5;
     return v;
 }
 

@@ -104,16 +104,18 @@ cudaError_t launch_gather_rows(stacklstm *s, const int32_t *idx, int rows, size_
 cudaError_t launch_seed_grads(stacklstm *s, const float *d_top_h, const float *dy);
 
 // ---- fp32 CUDA-core path (fp32_path.cu)
-cudaError_t fp32_forward(stacklstm *s, const float *x, const float *h0, const float *c0,
-                         const float *W, const float *bias);
+cudaError_t fp32_forward_setup(stacklstm *s, const float *h0, const float *c0, const float *W);
+cudaError_t fp32_forward_steps(stacklstm *s, const float *x, const float *W, const float *bias);
 cudaError_t fp32_backward_steps(stacklstm *s);
 cudaError_t fp32_dx(stacklstm *s, float *dx);
 cudaError_t fp32_dw(stacklstm *s, float *dW, float *dbias);
 
 // ---- bf16 tensor-core path (bf16_path.cu)
 cudaError_t bf16_prepare(stacklstm *s);
-cudaError_t bf16_forward(stacklstm *s, const __nv_bfloat16 *x, const __nv_bfloat16 *h0,
-                         const float *c0, const __nv_bfloat16 *W, const float *bias);
+cudaError_t bf16_forward_setup(stacklstm *s, const __nv_bfloat16 *x, const __nv_bfloat16 *h0,
+                               const float *c0, const __nv_bfloat16 *W);
+cudaError_t bf16_forward_steps(stacklstm *s, const float *bias);
+cudaError_t bf16_backward_setup(stacklstm *s);
 cudaError_t bf16_backward_steps(stacklstm *s);
 cudaError_t bf16_dx(stacklstm *s, float *dx);
 cudaError_t bf16_dw(stacklstm *s, float *dW, float *dbias);

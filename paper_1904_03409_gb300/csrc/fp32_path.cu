@@ -162,25 +162,30 @@ unsigned grid_for(const stacklstm *s, size_t n, int threads)
 
 }  // namespace
 
-cudaError_t fp32_forward(stacklstm *s, const float *x, const float *h0, const float *c0, const float *W,
-                         const float *bias)
+cudaError_t fp32_forward_setup(stacklstm *s, const float *h0, const float *c0, const float *W)
 {
-    const int T = s->T, B = s->B, I = s->I, H = s->H, K = I + H, G = 4 * H;
-    float *hh = (float *)s->hist_h;
+    const int B = s->B, I = s->I, H = s->H, K = I + H, G = 4 * H;
     cudaError_t e;
     // history row 0 = the initial state (stack slot 0)
-    if ((e = cudaMemcpyAsync(hh, h0, sizeof(float) * B * H, cudaMemcpyDeviceToDevice, s->stream))) return e;
+    if ((e = cudaMemcpyAsync(s->hist_h, h0, sizeof(float) * B * H, cudaMemcpyDeviceToDevice, s->stream))) return e;
     if ((e = cudaMemcpyAsync(s->hist_c, c0, sizeof(float) * B * H, cudaMemcpyDeviceToDevice, s->stream)))
         return e;
     // W^T for the backward contractions (so backward needs nothing the caller owns)
     transpose_f32<<<grid_for(s, (size_t)K * G, 256), 256, 0, s->stream>>>(K, G, W, (float *)s->w_fwd);
+    s->launches += 1;
+    return cudaGetLastError();
+}
+
+cudaError_t fp32_forward_steps(stacklstm *s, const float *x, const float *W, const float *bias)
+{
+    const int T = s->T, B = s->B, I = s->I, H = s->H, K = I + H;
     const int threads = std::min(128, ((H + 31) / 32) * 32);
     const dim3 grid(ceil_div(H, threads), B);
     const size_t smem = sizeof(float) * K;
     for (int t = 0; t < T; ++t)
-        fwd_step_f32<<<grid, threads, smem, s->stream>>>(t, B, I, H, x, W, bias, s->top, hh, s->hist_c,
-                                                          (float *)s->gates, (float *)s->a_rm);
-    s->launches += 1 + T;
+        fwd_step_f32<<<grid, threads, smem, s->stream>>>(t, B, I, H, x, W, bias, s->top, (float *)s->hist_h,
+                                                          s->hist_c, (float *)s->gates, (float *)s->a_rm);
+    s->launches += T;
     return cudaGetLastError();
 }
 

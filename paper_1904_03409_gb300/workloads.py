@@ -204,9 +204,15 @@ CONFIGS = {
 }
 
 
-def config_workload(name: str, B: Optional[int] = None) -> Workload:
-    """The named workload. ``sweep`` needs B (one of its batch sizes)."""
+def config_workload(name: str, B: Optional[int] = None, T: Optional[int] = None) -> Workload:
+    """The named workload. ``sweep`` needs B (one of its batch sizes). T, for the workloads
+    with a fixed step count (tiny, large, stress), generates the same recipe with fewer
+    steps (a smaller case of the same shape, e.g. for profiling)."""
     cfg = dict(CONFIGS[name])
+    if T is not None:
+        if "T" not in cfg:
+            raise ValueError("%s has no fixed step count to change" % name)
+        cfg["T"] = T
     if name == "sweep":
         if B is None or B not in cfg["B"]:
             raise ValueError("sweep needs B in %s" % (cfg["B"],))
