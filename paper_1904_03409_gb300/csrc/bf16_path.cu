@@ -505,11 +505,12 @@ std::string bf16_describe(const stacklstm *s)
     snprintf(buf, sizeof buf,
              "bf16 tcgen05; row tiles %d; chunks fwd %d (x %d) bwd %d; "
              "forward %s U=%d [EP %d G %d ring %d slots %d cluster %d col tiles %d w_res %d smem %u threads %d]; "
-             "backward %s U=%d [EP %d G %d ring %d slots %d cluster %d col tiles %d w_res %d smem %u threads %d]; "
+             "backward %s U=%d [EP %d G %d ring %d slots %d cluster %d col tiles %d w_res %d smem %u threads %d "
+             "contraction parts %d]; "
              "step rings fwd %d bwd %d; dx N=%d x%d ring %d; dW %dx%d tiles of 128x%d x%d splits ring %d",
              rt, s->kcf, s->kcx, s->kcb, f.on ? "persistent" : "per-step", s->uf, f.EP, f.G, f.S, f.slot, f.cl, f.n_ct,
              f.w_res, f.smem, f.threads, b.on ? "persistent" : "per-step", s->ub, b.EP, b.G, b.S, b.slot, b.cl, b.n_ct,
-             b.w_res, b.smem, b.threads, s->sf, s->sb, s->nx, s->nxt, s->sx, s->dw_mt, s->dw_nt, s->dw_ntile, s->dw_split, s->sw);
+             b.w_res, b.smem, b.threads, b.KS, s->sf, s->sb, s->nx, s->nxt, s->sx, s->dw_mt, s->dw_nt, s->dw_ntile, s->dw_split, s->sw);
     return buf;
 }
 
@@ -565,6 +566,15 @@ cudaError_t bf16_prepare(stacklstm *s)
     s->allocs.push_back(p); s->w_dx = p;
     if ((e = cudaMalloc(&p, s->dw_part_elems * sizeof(float)))) return e;
     s->allocs.push_back(p); s->dw_part = (float *)p;
+    if (s->pb.on && s->pb.KS > 1) {
+        const size_t n_rt = ceil_div(B, kRows), pairs = n_rt * s->pb.n_ct;
+        if ((e = cudaMalloc(&p, sizeof(float) * pairs * s->pb.KS * kRows * s->pb.U))) return e;
+        s->allocs.push_back(p);
+        s->split_part = (float *)p;
+        if ((e = cudaMalloc(&p, sizeof(int32_t) * pairs))) return e;
+        s->allocs.push_back(p);
+        s->split_cnt = (int32_t *)p;
+    }
     if (s->pf.on || s->pb.on) {
         if ((e = cudaMalloc(&p, 2 * sizeof(int32_t) * rt))) return e;
         s->allocs.push_back(p);

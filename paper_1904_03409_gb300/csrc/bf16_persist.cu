@@ -48,6 +48,8 @@ struct WsArgs {
     int cl;                  // cluster size along the column tiles (1: no multicast)
     int32_t *cnt;            // [n_rt] completed steps per row tile, zero at launch
     int vec32;               // H % 16 == 0: 16-unit groups of 16-bit rows are 32-byte aligned
+    float *part;             // split contraction: [n_rt][n_ct][KS][128][U] partial dh_read rows
+    int32_t *pcnt;           // split contraction: [n_rt][n_ct] partials written, zero at launch
 };
 
 // Dynamic shared memory: [weight tile (w_res)][S stages: G A chunks, then G weight
@@ -239,22 +241,28 @@ struct EpiCtx {
     WCtl c;
     uint32_t tmem;
     int q, part, lane, tid;  // TMEM lane quadrant, unit part, lane, thread
-    int ct, slot, n_mine, n_tiles;
+    int ct, kp, slot, n_mine, n_tiles;  // column tile, contraction part, slot
     long long limit;
 };
 
-// All tiles of one epilogue thread: row 32 q + lane of each tile, units
-// ct * U + part * UE .. + UE, in access groups of NG units.
-template <int U, int EP, int NG, bool kFwd>
+// All tiles of one epilogue thread: row 32 q + lane of each tile, in access groups of NG
+// units. Without a split contraction (KS = 1) the thread finishes units
+// ct * U + part * UE .. + UE straight from its accumulator lane. With KS > 1 (backward
+// only) the KS CTAs of a column tile each hold a partial dh_read over a quarter (half ...)
+// of the 4H contraction: every CTA writes its whole partial row to an L2 scratch, counts
+// it, waits for the other parts, then sums the parts in part order (deterministic) for the
+// U / KS units it finishes: ct * U + kp * U / KS .. + U / KS.
+template <int U, int EP, int NG, bool kFwd, int KS>
 __device__ __forceinline__ void epilogue_loop(const StepArgs &a, const WsArgs &p, const EpiCtx &e,
                                               const float *s_bias)
 {
-    constexpr int E = 4 * EP, UE = U / EP;
+    static_assert(KS == 1 || (!kFwd && EP == 1), "split contraction: backward, one epilogue warp group");
+    constexpr int E = 4 * EP, UE = U / KS / EP;  // units this thread finishes
     constexpr int NB = kFwd ? 4 * U : U;
     constexpr uint32_t kCols = TmemCols<NB>::value;
     const int T = a.T, B = a.B, H = a.H;
     const uint32_t lane_off = (uint32_t)(e.q * 32) << 16;
-    const int u0 = e.ct * U + e.part * UE;  // first unit of this thread
+    const int u0 = e.ct * U + e.kp * (U / KS) + e.part * UE;  // first unit of this thread
     for (int k = 0; k < e.n_tiles; ++k) {
         const int ks = k / e.n_mine, rt = e.slot + (k % e.n_mine) * p.n_slot;
         const int t = kFwd ? ks : T - 1 - ks;
@@ -387,17 +395,55 @@ __device__ __forceinline__ void epilogue_loop(const StepArgs &a, const WsArgs &p
             __syncwarp();
             if (tc::bar_any(1, E * 32, !ok || *e.c.abort)) break;
             tc::tc_fence_after();
+            float dsum[KS > 1 ? UE : 1];
+            if constexpr (KS > 1) {
+                // the whole partial row of this lane to the scratch, then the sum of the parts
+                uint32_t pr[U];
+                tmem_cols<U>(taddr, pr);
+                tc::tmem_wait_ld();
+                tc::tc_fence_before();
+                __syncwarp();
+                if (e.lane == 0) tc::mbar_arrive(&e.c.tempty[acc]);
+                const size_t grp = (size_t)rt * p.n_ct + e.ct;
+                float *prow = p.part + ((grp * KS + e.kp) * kRows + e.q * 32 + e.lane) * U;
+#pragma unroll
+                for (int i = 0; i < U / 8; ++i) st_v8(prow + 8 * i, pr + 8 * i);
+                __syncwarp();
+                tc::bar_sync(2, E * 32);
+                bool ok2 = true;
+                if (e.tid == 0) {
+                    tc::red_release_gpu_add(p.pcnt + grp, 1);
+                    ok2 = spin_until(p.pcnt + grp, KS * (ks + 1), e.limit, e.c.abort, a.err);
+                    if (!ok2) ws_abort(e.c, a.err);
+                }
+                __syncwarp();
+                if (tc::bar_any(1, E * 32, !ok2 || *e.c.abort)) break;
+#pragma unroll
+                for (int i = 0; i < UE; ++i) dsum[i] = 0.0f;
+#pragma unroll
+                for (int j = 0; j < KS; ++j) {
+                    float v[UE];
+                    ld_f<UE>(p.part + ((grp * KS + j) * kRows + e.q * 32 + e.lane) * U + e.kp * (U / KS), v);
+#pragma unroll
+                    for (int i = 0; i < UE; ++i) dsum[i] += v[i];
+                }
+            }
 #pragma unroll
             for (int cg = 0; cg < NGRP; ++cg) {
                 const int u = u0 + cg * NG;
                 const int j = kEarly ? cg : 0;  // operand slot of this group
                 uint32_t dr[NG];
-                tmem_cols<NG>(taddr + e.part * UE + cg * NG, dr);
-                tc::tmem_wait_ld();
-                if (cg == NGRP - 1) {
-                    tc::tc_fence_before();
-                    __syncwarp();
-                    if (e.lane == 0) tc::mbar_arrive(&e.c.tempty[acc]);
+                if constexpr (KS > 1) {
+#pragma unroll
+                    for (int i = 0; i < NG; ++i) dr[i] = __float_as_uint(dsum[cg * NG + i]);
+                } else {
+                    tmem_cols<NG>(taddr + e.part * UE + cg * NG, dr);
+                    tc::tmem_wait_ld();
+                    if (cg == NGRP - 1) {
+                        tc::tc_fence_before();
+                        __syncwarp();
+                        if (e.lane == 0) tc::mbar_arrive(&e.c.tempty[acc]);
+                    }
                 }
                 if (!(row_ok && u < H)) continue;
                 if (!kEarly) load_ops(u, 0);
@@ -446,13 +492,15 @@ __device__ __forceinline__ void epilogue_loop(const StepArgs &a, const WsArgs &p
 // ------------------------------------------------------------------ the kernel
 // kFwd: forward (tm_a = x_t tiles for chunks < kcx, tm_b = hr[t] tiles after them);
 // else backward (tm_b = dG_t tiles, kcx = 0: every chunk depends on the step before).
-template <int U, int EP, int G, bool kFwd>
+// KS > 1 (backward): the KS CTAs blockIdx = (slot, ct, kp) split the contraction; part kp
+// takes chunks [KC kp / KS, KC (kp + 1) / KS) and keeps only that slice of the weight tile.
+template <int U, int EP, int G, bool kFwd, int KS>
 __global__ void __launch_bounds__(32 * (4 * EP + 2), 1)
 step_ws(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtensorMap tm_b, WsArgs p)
 {
     constexpr int NB = kFwd ? 4 * U : U;  // accumulator columns
     constexpr int E = 4 * EP;             // epilogue warps
-    constexpr int UE = U / EP;            // units per epilogue thread
+    constexpr int UE = U / KS / EP;       // units each epilogue thread finishes
     constexpr uint32_t kCols = TmemCols<NB>::value;
     constexpr uint32_t bchunk = NB * 128;
     static_assert(UE % 8 == 0, "epilogue works on groups of 8 units");
@@ -460,9 +508,12 @@ step_ws(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtens
     extern __shared__ uint8_t smem_raw[];
     __shared__ float s_bias[kFwd ? 4 * U : 4];
     const int S = a.S, KC = a.KC, split = a.kcx, T = a.T, B = a.B, H = a.H;
-    const WCtl c = wcarve(smem_raw, S, G, NB, KC, p.w_res);
+    const int kp = (int)(blockIdx.x % KS), cidx = (int)(blockIdx.x / KS);
+    const int k0 = KC * kp / KS, k1 = KC * (kp + 1) / KS;  // this CTA's contraction chunks
+    const int dep_c = split > k0 ? split : k0;            // first chunk that needs step t - 1
+    const WCtl c = wcarve(smem_raw, S, G, NB, (KC + KS - 1) / KS, p.w_res);
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int ct = blockIdx.x % p.n_ct, slot = blockIdx.x / p.n_ct, cl = p.cl;
+    const int ct = cidx % p.n_ct, slot = cidx / p.n_ct, cl = p.cl;
     const uint32_t rank = cl > 1 ? tc::cluster_rank() : 0;
     const int n_mine = slot < p.n_rt ? (p.n_rt - slot + p.n_slot - 1) / p.n_slot : 0;
     const int n_tiles = T * n_mine;
@@ -500,19 +551,20 @@ step_ws(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtens
         // ------------------------------------------------------------ producer
         if (lane == 0) {
             if (p.w_res) {
-                tc::mbar_arrive_expect_tx(c.wbar, KC * bchunk);
-                tc::bulk_g2s(c.w0, wtile, KC * bchunk, c.wbar);
+                tc::mbar_arrive_expect_tx(c.wbar, (k1 - k0) * bchunk);
+                tc::bulk_g2s(c.w0, wtile + (size_t)k0 * bchunk, (k1 - k0) * bchunk, c.wbar);
             }
             uint32_t g = 0;
             for (int k = 0; k < n_tiles && !*c.abort; ++k) {
                 const int ks = k / n_mine, rt = slot + (k % n_mine) * p.n_slot;
                 const int t = kFwd ? ks : T - 1 - ks;
                 const int row = t * B + rt * kRows;
-                for (int c0 = 0; c0 < KC;) {
-                    const int c1 = group_end(c0, G, split, KC);
-                    if (c0 == split && ks > 0) {
-                        // every column tile of this row tile finished the step before
-                        if (!spin_until(p.cnt + rt, p.n_ct * ks, limit, c.abort, a.err)) {
+                for (int c0 = k0; c0 < k1;) {
+                    const int c1 = group_end(c0, G, split, k1);
+                    if (c0 == dep_c && ks > 0) {
+                        // every column tile (and contraction part) of this row tile
+                        // finished the step before
+                        if (!spin_until(p.cnt + rt, p.n_ct * KS * ks, limit, c.abort, a.err)) {
                             ws_abort(c, a.err);
                             break;
                         }
@@ -565,8 +617,8 @@ step_ws(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtens
                 tc::tc_fence_after();
                 const uint32_t d = tmem + acc * kCols;
                 bool bad = false;
-                for (int c0 = 0; c0 < KC;) {
-                    const int c1 = group_end(c0, G, split, KC);
+                for (int c0 = k0; c0 < k1;) {
+                    const int c1 = group_end(c0, G, split, k1);
                     const int s = (int)(g % S);
                     if (!tc::mbar_wait(&c.full[s], (g / S) & 1, limit, c.abort)) {
                         ws_abort(c, a.err);
@@ -575,7 +627,8 @@ step_ws(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtens
                     }
                     tc::tc_fence_after();
                     const uint32_t st = c.ring0 + s * c.stage;
-                    issue_group<NB, G>(d, st, p.w_res ? c.w0 + c0 * bchunk : st + G * kAStage, c1 - c0, c0 == 0);
+                    issue_group<NB, G>(d, st, p.w_res ? c.w0 + (c0 - k0) * bchunk : st + G * kAStage, c1 - c0,
+                                       c0 == k0);
                     if (cl > 1)
                         tc::mma_commit_mc(&c.empty[s], (uint16_t)((1u << cl) - 1));
                     else
@@ -593,11 +646,11 @@ step_ws(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtens
     } else {
         // ------------------------------------------------------------ epilogue
         constexpr int NG = UE % 16 == 0 ? 16 : 8;
-        const EpiCtx e{c, tmem, warp & 3, warp >> 2, lane, tid, ct, slot, n_mine, n_tiles, limit};
+        const EpiCtx e{c, tmem, warp & 3, warp >> 2, lane, tid, ct, kp, slot, n_mine, n_tiles, limit};
         if (NG == 16 && p.vec32)
-            epilogue_loop<U, EP, NG, kFwd>(a, p, e, s_bias);
+            epilogue_loop<U, EP, NG, kFwd, KS>(a, p, e, s_bias);
         else
-            epilogue_loop<U, EP, 8, kFwd>(a, p, e, s_bias);
+            epilogue_loop<U, EP, 8, kFwd, KS>(a, p, e, s_bias);
     }
 
     // ---------------------------------------------------------------- teardown
@@ -622,14 +675,14 @@ double mma_cycles(int N) { return N <= 16 ? 45 : N <= 32 ? 51 : N <= 64 ? 47 : N
 constexpr double kWaitCycles = 300;
 
 struct Variant {
-    int U, EP, G;
+    int U, EP, G, KS;
     const void *fn;
 };
 
-template <int U, int EP, int G, bool kFwd>
+template <int U, int EP, int G, bool kFwd, int KS = 1>
 Variant variant()
 {
-    return Variant{U, EP, G, (const void *)step_ws<U, EP, G, kFwd>};
+    return Variant{U, EP, G, KS, (const void *)step_ws<U, EP, G, kFwd, KS>};
 }
 
 const Variant *fwd_variants(int *n)
@@ -642,8 +695,8 @@ const Variant *fwd_variants(int *n)
 const Variant *bwd_variants(int *n)
 {
     static const Variant v[] = {variant<16, 1, 4, false>(), variant<16, 2, 4, false>(), variant<32, 2, 4, false>(),
-                                variant<32, 4, 4, false>(), variant<64, 2, 2, false>()};
-    *n = 5;
+                                variant<32, 4, 4, false>(), variant<64, 2, 2, false>(), variant<64, 1, 2, false, 4>()};
+    *n = 6;
     return v;
 }
 
@@ -674,7 +727,8 @@ bool plan_variant(const Variant &v, bool fwd, int KC, int split, int n_rt, int H
     const int NB = fwd ? 4 * v.U : v.U, n_ct = (H + v.U - 1) / v.U;
     const int threads = 32 * (4 * v.EP + 2);
     const uint32_t kcols2 = 2u * (NB <= 32 ? 32 : NB <= 64 ? 64 : NB <= 128 ? 128 : 256);
-    const int groups = (split + v.G - 1) / v.G + (KC - split + v.G - 1) / v.G;
+    const int KCl = (KC + v.KS - 1) / v.KS;  // chunks of one contraction part
+    const int groups = (split + v.G - 1) / v.G + (KCl - split + v.G - 1) / v.G;
     const uint32_t fixed = 1024 + kBarBytes + 1024 /* static */;
     bool found = false;
     double best = 1e30;
@@ -684,14 +738,14 @@ bool plan_variant(const Variant &v, bool fwd, int KC, int split, int n_rt, int H
         return false;
     }
     for (int cl : {8, 4, 2, 1}) {
-        if (cl > 1 && (!want_mc || cl / 2 >= n_ct)) continue;
-        const int pad = (n_ct + cl - 1) / cl * cl;
+        if (cl > 1 && (!want_mc || cl / 2 >= n_ct || v.KS > 1)) continue;
+        const int pad = (n_ct + cl - 1) / cl * cl * v.KS;  // CTAs per row-tile slot
         for (int wr : {1, 0}) {
-            const uint32_t wbytes = wr ? (uint32_t)KC * NB * 128 : 0u;
+            const uint32_t wbytes = wr ? (uint32_t)KCl * NB * 128 : 0u;
             const uint32_t stage = ws_stage_bytes(v.G, NB, wr);
             if (fixed + wbytes + 2 * stage > kSmemCap) continue;
             const int S = std::min({(int)((kSmemCap - fixed - wbytes) / stage), kMaxStages, std::max(2, 2 * groups)});
-            uint32_t smem = ws_smem_bytes(S, v.G, NB, KC, wr);
+            uint32_t smem = ws_smem_bytes(S, v.G, NB, KCl, wr);
             smem = pad_for_tmem(v.fn, threads, smem, kcols2);
             if (!smem) continue;
             int resident = 0;
@@ -724,7 +778,18 @@ bool plan_variant(const Variant &v, bool fwd, int KC, int split, int n_rt, int H
             if (resident < pad) continue;
             const int sl = std::min(n_rt, resident / pad);
             const int rounds = (n_rt + sl - 1) / sl;
-            const double c = rounds * (KC * 4 * mma_cycles(NB) + groups * kWaitCycles);
+            double c = rounds * (KC * 4 * mma_cycles(NB) + groups * kWaitCycles);
+            if (!fwd) {
+                // backward, per CTA and step: the dG operand (and a streamed weight slice)
+                // at about 50 B/cycle of TMA ingest against the MMA issue time, then the
+                // epilogue's ~48 B per (instance, unit) at about 30 B/cycle of load/store,
+                // plus the partial exchange of a split contraction
+                const double ingest = (128.0 * KCl * 128 + (wr ? 0.0 : (double)NB * KCl * 128)) / 50;
+                const double mma = KCl * 4 * mma_cycles(NB) + groups * kWaitCycles;
+                const double epi = 128.0 * (v.U / v.KS) * 48 / 30 +
+                                   (v.KS > 1 ? 2.0 * 128 * v.U * 4 / 30 + 3000 : 0.0);
+                c = rounds * (std::max(ingest, mma) + epi);
+            }
             const int key = wr * 1000 + cl * 20 + S;
             if (c < best * 0.999 || (c <= best * 1.001 && key > best_key)) {
                 best = c;
@@ -737,7 +802,8 @@ bool plan_variant(const Variant &v, bool fwd, int KC, int split, int n_rt, int H
                 pl->slot = sl;
                 pl->w_res = wr;
                 pl->cl = cl;
-                pl->n_ct = pad;
+                pl->KS = v.KS;
+                pl->n_ct = pad / v.KS;
                 pl->smem = smem;
                 pl->threads = threads;
                 found = true;
@@ -765,8 +831,10 @@ bool plan(stacklstm *s, bool fwd, PersistPlan *pl)
     bool found = false;
     for (int i = 0; i < n; ++i) {
         if (force_u && vs[i].U != force_u) continue;
-        const int want_ep = force_ep ? atoi(force_ep) : vs[i].U == 16 ? 1 : 2;
+        const int want_ep = force_ep ? atoi(force_ep) : vs[i].U == 16 || vs[i].KS > 1 ? 1 : 2;
         if (vs[i].U >= 16 && vs[i].EP != want_ep) continue;
+        const char *force_ks = fwd ? nullptr : getenv("STACKLSTM_BWD_KS");
+        if (force_ks && vs[i].KS != atoi(force_ks)) continue;
         PersistPlan cand;
         double cost;
         const int n_ct = (s->H + vs[i].U - 1) / vs[i].U;
@@ -786,7 +854,7 @@ template <typename... Args>
 cudaError_t launch_coop(const void *fn, const PersistPlan &pl, cudaStream_t st, Args... args)
 {
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(pl.n_ct * pl.slot);
+    cfg.gridDim = dim3(pl.n_ct * pl.KS * pl.slot);
     cfg.blockDim = dim3(pl.threads);
     cfg.dynamicSmemBytes = pl.smem;
     cfg.stream = st;
@@ -808,7 +876,7 @@ const void *find_fn(bool fwd, const PersistPlan &pl)
     int n;
     const Variant *vs = fwd ? fwd_variants(&n) : bwd_variants(&n);
     for (int i = 0; i < n; ++i)
-        if (vs[i].U == pl.U && vs[i].EP == pl.EP && vs[i].G == pl.G) return vs[i].fn;
+        if (vs[i].U == pl.U && vs[i].EP == pl.EP && vs[i].G == pl.G && vs[i].KS == pl.KS) return vs[i].fn;
     return nullptr;
 }
 
@@ -830,6 +898,8 @@ cudaError_t bf16_launch_fwd_persist(stacklstm *s, const StepArgs &a, const CUten
     p.cl = pl.cl;
     p.cnt = s->rowcnt;
     p.vec32 = s->H % 16 == 0;
+    p.part = nullptr;
+    p.pcnt = nullptr;
     cudaError_t e = cudaMemsetAsync(p.cnt, 0, sizeof(int32_t) * p.n_rt, s->stream);
     if (e) return e;
     const void *fn = find_fn(true, pl);
@@ -854,8 +924,11 @@ cudaError_t bf16_launch_bwd_persist(stacklstm *s, const StepArgs &a, const CUten
     p.cl = pl.cl;
     p.cnt = s->rowcnt + p.n_rt;
     p.vec32 = s->H % 16 == 0;
+    p.part = s->split_part;
+    p.pcnt = s->split_cnt;
     cudaError_t e = cudaMemsetAsync(p.cnt, 0, sizeof(int32_t) * p.n_rt, s->stream);
     if (e) return e;
+    if (pl.KS > 1 && (e = cudaMemsetAsync(p.pcnt, 0, sizeof(int32_t) * p.n_rt * p.n_ct, s->stream))) return e;
     const void *fn = find_fn(false, pl);
     if (!fn) return cudaErrorInvalidDeviceFunction;
     e = launch_coop(fn, pl, s->stream, tm_g, tm_g, p);

@@ -21,6 +21,7 @@ struct PersistPlan {
     int slot = 0;       // CTAs per column tile (each takes every slot-th row tile)
     int w_res = 0;      // weight tile resident in shared memory
     int cl = 1;         // thread-block cluster size along the column tiles (A multicast)
+    int KS = 1;         // contraction parts per column tile (backward split contraction)
     int n_ct = 0;       // column tiles, padded to a multiple of cl
     unsigned smem = 0;  // dynamic shared memory per CTA
     int threads = 0;    // threads per CTA
@@ -72,6 +73,8 @@ struct stacklstm {
     // persistent step kernels (one launch for all T steps; bf16_persist.cu)
     PersistPlan pf, pb;            // forward, backward (on = 0: one launch per step)
     int32_t *rowcnt = nullptr;     // [2][row tiles] completed steps per row tile
+    float *split_part = nullptr;   // backward split contraction: partial dh_read rows
+    int32_t *split_cnt = nullptr;  // backward split contraction: partials written per tile pair
     int nx = 0, nxt = 0;     // input gradient: columns per tile, number of column tiles
     int dw_mt = 0, dw_nt = 0, dw_split = 0;  // weight gradient: m tiles, column tiles, splits
     int dw_ntile = 0;                        // weight gradient: gate columns per tile

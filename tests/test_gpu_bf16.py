@@ -145,3 +145,26 @@ def test_per_step_kernels_match_oracle(T, B, I, H, seed):
     finally:
         del os.environ["STACKLSTM_STEP_KERNELS"]
     compare(got, oracle_all(w), "bf16")
+
+
+@pytest.mark.parametrize("T,B,I,H,seed", [(12, 200, 64, 256, 14), (10, 130, 40, 200, 15)])
+def test_split_contraction_backward_matches_oracle(T, B, I, H, seed):
+    """The backward with its 4H contraction split over four CTAs per column tile (partial
+    sums exchanged through L2, summed in part order) stays parity-green, including parts
+    of unequal length (H = 200: 13 chunks over 4 parts)."""
+    w = case(T, B, I, H, seed, bias_scale=0.3, h0_scale=0.5, c0_scale=0.5, dy_scale=0.5)
+    os.environ["STACKLSTM_BWD_UNITS"] = "64"
+    os.environ["STACKLSTM_BWD_KS"] = "4"
+    try:
+        hd = bd.stacklstm_create(w.T, w.B, w.I, w.H, bd.SL_BF16, 0)
+        plan = bd.stacklstm_plan(hd)
+        hd.destroy()
+        got = runner.run(w)
+        again = runner.run(w)
+    finally:
+        del os.environ["STACKLSTM_BWD_UNITS"]
+        del os.environ["STACKLSTM_BWD_KS"]
+    assert "backward persistent U=64" in plan and "contraction parts 4" in plan, plan
+    compare(got, oracle_all(w), "bf16")
+    for k in ("dx", "dW", "dbias", "dh0", "dc0"):
+        assert np.array_equal(got[k], again[k]), k
