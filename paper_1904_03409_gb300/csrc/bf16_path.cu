@@ -620,8 +620,8 @@ cudaError_t bf16_forward_steps(stacklstm *s, const float *bias)
     const int nctf = std::max((int)ceil_div(H, s->uf), s->pf.on ? s->pf.n_ct : 0);
     cudaError_t e;
     if (s->pf.on)
-        return bf16_launch_fwd_persist(s, step_args(s, bias, s->w_fwd, s->kcx, s->kcf, s->pf.S), map(s, kMapX128),
-                                       map(s, kMapH128));
+        return bf16_launch_fwd_persist(s, step_args(s, bias, s->w_fwd, s->kcx, s->kcf, s->pf.S),
+                                       map(s, B <= 64 ? kMapX64 : kMapX128), map(s, B <= 64 ? kMapH64 : kMapH128));
     const StepArgs a = step_args(s, bias, s->w_fwd, s->kcx, s->kcf, s->sf);
     const dim3 grid(nctf, ceil_div(B, kRows));
     const size_t smem = smem_bytes(s->sf, 4 * s->uf);
@@ -654,7 +654,11 @@ cudaError_t bf16_backward_steps(stacklstm *s)
     const int T = s->T, B = s->B, H = s->H;
     cudaError_t e;
     const StepArgs a = step_args(s, nullptr, s->w_bwd, 0, s->kcb, s->sb);
-    if (s->pb.on) return bf16_launch_bwd_persist(s, step_args(s, nullptr, s->w_bwd, 0, s->kcb, s->pb.S), map(s, kMapG128));
+    // one row tile of at most 64 instances: 64-row boxes (the rest of each stage is never
+    // loaded and only feeds accumulator rows that are not stored)
+    if (s->pb.on)
+        return bf16_launch_bwd_persist(s, step_args(s, nullptr, s->w_bwd, 0, s->kcb, s->pb.S),
+                                       map(s, B <= 64 ? kMapG64 : kMapG128));
     const dim3 grid(ceil_div(H, s->ub), ceil_div(B, kRows));
     const size_t smem = smem_bytes(s->sb, s->ub);
     const CUtensorMap &tmg = map(s, kMapG128);

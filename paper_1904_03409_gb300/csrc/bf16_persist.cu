@@ -48,6 +48,7 @@ struct WsArgs {
     int cl;                  // cluster size along the column tiles (1: no multicast)
     int32_t *cnt;            // [n_rt] completed steps per row tile, zero at launch
     int vec32;               // H % 16 == 0: 16-unit groups of 16-bit rows are 32-byte aligned
+    int a_rows;              // rows per A box: 128, or 64 when B <= 64 (one half-filled row tile)
     float *part;             // split contraction: [n_rt][n_ct][KS][128][U] partial dh_read rows
     int32_t *pcnt;           // split contraction: [n_rt][n_ct] partials written, zero at launch
 };
@@ -576,7 +577,7 @@ step_ws(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtens
                         break;
                     }
                     const uint32_t st = c.ring0 + s * c.stage;
-                    tc::mbar_arrive_expect_tx(&c.full[s], (c1 - c0) * (kAStage + (p.w_res ? 0u : bchunk)));
+                    tc::mbar_arrive_expect_tx(&c.full[s], (c1 - c0) * ((uint32_t)p.a_rows * 128 + (p.w_res ? 0u : bchunk)));
                     for (int cc = c0; cc < c1; ++cc) {
                         const bool first = cc < split;
                         const CUtensorMap *tm = first ? &tm_a : &tm_b;
@@ -900,6 +901,7 @@ cudaError_t bf16_launch_fwd_persist(stacklstm *s, const StepArgs &a, const CUten
     p.vec32 = s->H % 16 == 0;
     p.part = nullptr;
     p.pcnt = nullptr;
+    p.a_rows = s->B <= 64 ? 64 : kRows;
     cudaError_t e = cudaMemsetAsync(p.cnt, 0, sizeof(int32_t) * p.n_rt, s->stream);
     if (e) return e;
     const void *fn = find_fn(true, pl);
@@ -926,6 +928,7 @@ cudaError_t bf16_launch_bwd_persist(stacklstm *s, const StepArgs &a, const CUten
     p.vec32 = s->H % 16 == 0;
     p.part = s->split_part;
     p.pcnt = s->split_cnt;
+    p.a_rows = s->B <= 64 ? 64 : kRows;
     cudaError_t e = cudaMemsetAsync(p.cnt, 0, sizeof(int32_t) * p.n_rt, s->stream);
     if (e) return e;
     if (pl.KS > 1 && (e = cudaMemsetAsync(p.pcnt, 0, sizeof(int32_t) * p.n_rt * p.n_ct, s->stream))) return e;
