@@ -261,9 +261,10 @@ __global__ void dw_reduce_pad(int I, int H, int kbx, int split, const float *__r
 
 }  // namespace
 
-// Tile width (512 or 256 gate columns), splits and ring depth: the fewest MMA cycles on
-// the busiest SM (waves x chunks per CTA x width), one CTA per SM; ties go to the wider
-// tile (fewer operand bytes per flop), then to fewer splits.
+// Tile width (512 or 256 gate columns), splits and ring depth: the fewest cycles of MMA on
+// the busiest SM (waves x chunks per CTA x 2 cycles per gate column; one CTA per SM) plus
+// writing and reducing the split partials at the HBM rate (about 3.5 KB per cycle for the
+// whole GPU); ties go to the wider tile (fewer operand bytes per flop), then to fewer splits.
 cudaError_t bf16_plan_dw(stacklstm *s)
 {
     const int I = s->I, H = s->H, sms = s->num_sms;
@@ -273,9 +274,10 @@ cudaError_t bf16_plan_dw(stacklstm *s)
     double best = 1e300;
     for (int NT : {512, 256}) {
         const int n_nt = (int)ceil_div(4 * H, NT), tiles = n_mt * n_nt;
+        const double part_bytes = ((double)n_mt * 128 + 1) * n_nt * NT * 4;  // one split's partials
         for (int split = 1; split <= (int)std::min<size_t>(RC, 256); ++split) {
             const double waves = std::ceil((double)tiles * split / sms);
-            const double cost = waves * (double)ceil_div(RC, split) * NT;
+            const double cost = waves * (double)ceil_div(RC, split) * 2 * NT + 2 * split * part_bytes / 3540;
             if (cost < best * 0.999) {
                 best = cost;
                 s->dw_ntile = NT;
