@@ -696,8 +696,9 @@ const Variant *fwd_variants(int *n)
 const Variant *bwd_variants(int *n)
 {
     static const Variant v[] = {variant<16, 1, 4, false>(), variant<16, 2, 4, false>(), variant<32, 2, 4, false>(),
-                                variant<32, 4, 4, false>(), variant<64, 2, 2, false>(), variant<64, 1, 2, false, 4>()};
-    *n = 6;
+                                variant<32, 4, 4, false>(), variant<64, 2, 2, false>(), variant<64, 1, 2, false, 4>(),
+                                variant<64, 1, 4, false, 4>()};
+    *n = 7;
     return v;
 }
 
@@ -742,6 +743,8 @@ bool plan_variant(const Variant &v, bool fwd, int KC, int split, int n_rt, int H
         if (cl > 1 && (!want_mc || cl / 2 >= n_ct || v.KS > 1)) continue;
         const int pad = (n_ct + cl - 1) / cl * cl * v.KS;  // CTAs per row-tile slot
         for (int wr : {1, 0}) {
+            const char *fw = getenv(fwd ? "STACKLSTM_FWD_WRES" : "STACKLSTM_BWD_WRES");
+            if (fw && atoi(fw) != wr) continue;
             const uint32_t wbytes = wr ? (uint32_t)KCl * NB * 128 : 0u;
             const uint32_t stage = ws_stage_bytes(v.G, NB, wr);
             if (fixed + wbytes + 2 * stage > kSmemCap) continue;
@@ -782,11 +785,12 @@ bool plan_variant(const Variant &v, bool fwd, int KC, int split, int n_rt, int H
             double c = rounds * (KC * 4 * mma_cycles(NB) + groups * kWaitCycles);
             if (!fwd) {
                 // backward, per CTA and step: the dG operand (and a streamed weight slice)
-                // at about 50 B/cycle of TMA ingest against the MMA issue time, then the
-                // epilogue's ~48 B per (instance, unit) at about 30 B/cycle of load/store,
-                // plus the partial exchange of a split contraction
-                const double ingest = (128.0 * KCl * 128 + (wr ? 0.0 : (double)NB * KCl * 128)) / 50;
-                const double mma = KCl * 4 * mma_cycles(NB) + groups * kWaitCycles;
+                // at about 70 B/cycle of TMA ingest against the MMA issue time (about 400
+                // cycles per stage wait inside this kernel), then the epilogue's ~48 B per
+                // (instance, unit) at about 30 B/cycle of load/store, plus the partial
+                // exchange of a split contraction (constants fitted to GB300 measurements)
+                const double ingest = (128.0 * KCl * 128 + (wr ? 0.0 : (double)NB * KCl * 128)) / 70;
+                const double mma = KCl * 4 * mma_cycles(NB) + groups * 400.0;
                 const double epi = 128.0 * (v.U / v.KS) * 48 / 30 +
                                    (v.KS > 1 ? 2.0 * 128 * v.U * 4 / 30 + 3000 : 0.0);
                 c = rounds * (std::max(ingest, mma) + epi);
@@ -836,6 +840,8 @@ bool plan(stacklstm *s, bool fwd, PersistPlan *pl)
         if (vs[i].U >= 16 && vs[i].EP != want_ep) continue;
         const char *force_ks = fwd ? nullptr : getenv("STACKLSTM_BWD_KS");
         if (force_ks && vs[i].KS != atoi(force_ks)) continue;
+        const char *force_g = getenv(fwd ? "STACKLSTM_FWD_G" : "STACKLSTM_BWD_G");
+        if (force_g && vs[i].G != atoi(force_g)) continue;
         PersistPlan cand;
         double cost;
         const int n_ct = (s->H + vs[i].U - 1) / vs[i].U;
