@@ -159,7 +159,7 @@ cudaError_t launch(Kern kernel, dim3 grid, size_t smem, cudaStream_t st, bool pd
     return cudaLaunchKernelEx(&cfg, kernel, args...);
 }
 
-constexpr uint32_t kSmemCap = 225 * 1024;
+constexpr uint32_t kSmemCap = 226 * 1024;  // dynamic shared memory; leaves 1 KB for static
 
 template <typename Kern>
 cudaError_t allow_smem(Kern k)
@@ -172,7 +172,8 @@ cudaError_t allow_smem(Kern k)
 // ---- persistent step kernels (bf16_persist.cu)
 bool bf16_plan_fwd_persist(stacklstm *s, PersistPlan *pl);
 bool bf16_plan_bwd_persist(stacklstm *s, PersistPlan *pl);
-cudaError_t bf16_launch_fwd_persist(stacklstm *s, const StepArgs &a, const CUtensorMap &tm_x, const CUtensorMap &tm_h);
+cudaError_t bf16_launch_fwd_persist(stacklstm *s, const StepArgs &a, const CUtensorMap &tm_x, const CUtensorMap &tm_h,
+                                    const CUtensorMap &tm_gates);
 cudaError_t bf16_launch_bwd_persist(stacklstm *s, const StepArgs &a, const CUtensorMap &tm_g);
 
 // ---- weight / bias gradients (bf16_dw.cu)

@@ -461,7 +461,22 @@ cudaError_t make_map(void *slot, const void *base, uint64_t rows, uint64_t cols,
     return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
 }
 
-enum { kMapX128 = 0, kMapX64 = 1, kMapG128 = 2, kMapG64 = 3, kMapH128 = 4, kMapH64 = 5 };
+// The saved gates [T][B][4][H] (fp16) as a 4-D tensor for the forward's tensor stores:
+// boxes of `units` hidden units x 1 gate x rows instances x 1 step, so a store never
+// writes past H (into the next gate) or past B (into the next step).
+cudaError_t make_gates_map(void *slot, const void *base, int T, int B, int H, uint32_t units)
+{
+    cuuint64_t dims[4] = {(cuuint64_t)H, 4, (cuuint64_t)B, (cuuint64_t)T};
+    cuuint64_t strides[3] = {(cuuint64_t)H * 2, (cuuint64_t)H * 8, (cuuint64_t)H * 8 * B};
+    cuuint32_t box[4] = {units, 1, (cuuint32_t)std::min(B, kRows), 1};
+    cuuint32_t es[4] = {1, 1, 1, 1};
+    CUresult r = g_encode((CUtensorMap *)slot, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 4, const_cast<void *>(base), dims,
+                          strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+                          CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
+}
+
+enum { kMapX128 = 0, kMapX64 = 1, kMapG128 = 2, kMapG64 = 3, kMapH128 = 4, kMapH64 = 5, kMapGates = 6 };
 const CUtensorMap &map(const stacklstm *s, int i) { return *(const CUtensorMap *)s->tmaps[i]; }
 
 // budget that leaves room for two CTAs per SM when the grid needs more than one wave.
@@ -586,6 +601,7 @@ cudaError_t bf16_prepare(stacklstm *s)
     const uint64_t R1 = (uint64_t)(T + 1) * B;
     if ((e = make_map(s->tmaps[kMapH128], s->hr, R1, (uint64_t)H, kRows))) return e;
     if ((e = make_map(s->tmaps[kMapH64], s->hr, R1, (uint64_t)H, kChunk))) return e;
+    if (s->pf.on && (e = make_gates_map(s->tmaps[kMapGates], s->gates, T, B, H, s->pf.U / s->pf.EP))) return e;
     return cudaSuccess;
 }
 
@@ -621,7 +637,8 @@ cudaError_t bf16_forward_steps(stacklstm *s, const float *bias)
     cudaError_t e;
     if (s->pf.on)
         return bf16_launch_fwd_persist(s, step_args(s, bias, s->w_fwd, s->kcx, s->kcf, s->pf.S),
-                                       map(s, B <= 64 ? kMapX64 : kMapX128), map(s, B <= 64 ? kMapH64 : kMapH128));
+                                       map(s, B <= 64 ? kMapX64 : kMapX128), map(s, B <= 64 ? kMapH64 : kMapH128),
+                                       map(s, kMapGates));
     const StepArgs a = step_args(s, bias, s->w_fwd, s->kcx, s->kcf, s->sf);
     const dim3 grid(nctf, ceil_div(B, kRows));
     const size_t smem = smem_bytes(s->sf, 4 * s->uf);

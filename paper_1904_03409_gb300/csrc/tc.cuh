@@ -71,6 +71,13 @@ __device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, long l
     }
 }
 
+// 16-byte shared-memory store to a shared-window address.
+__device__ __forceinline__ void st_shared_v4(uint32_t addr, const uint32_t *w)
+{
+    asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(w[0]), "r"(w[1]), "r"(w[2]), "r"(w[3])
+                 : "memory");
+}
+
 // Plain arrival (count one) on a CTA-local mbarrier.
 __device__ __forceinline__ void mbar_arrive(uint64_t *bar)
 {
@@ -199,6 +206,22 @@ __device__ __forceinline__ void red_release_gpu_add(int *p, int v)
 }
 // generic-proxy global writes <-> async-proxy (TMA) global reads
 __device__ __forceinline__ void fence_proxy_async_global() { asm volatile("fence.proxy.async.global;" ::: "memory"); }
+
+// 4-D tiled tensor store (TMA), shared -> global, bulk-group completion: the box at
+// coordinates (c0 innermost .. c3) of the tensor map is written from src (16-byte
+// aligned, box layout). Parts of the box outside the tensor are not written.
+__device__ __forceinline__ void tma_store_4d(const void *tmap, uint32_t src, int c0, int c1, int c2, int c3)
+{
+    asm volatile("cp.async.bulk.tensor.4d.global.shared::cta.bulk_group [%0, {%2, %3, %4, %5}], [%1];" ::"l"(
+                     (uint64_t)tmap),
+                 "r"(src), "r"(c0), "r"(c1), "r"(c2), "r"(c3)
+                 : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+// every bulk store this thread committed has finished reading shared memory
+__device__ __forceinline__ void bulk_wait_read() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
+// every bulk store this thread committed has completed
+__device__ __forceinline__ void bulk_wait() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
 
 // ------------------------------------------------------------------ PDL
 __device__ __forceinline__ void grid_dep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
