@@ -204,7 +204,13 @@ sl_status stacklstm_create(stacklstm_t *out, int T, int B, int I, int H, sl_dtyp
     if (ok) ok = sl::configure_prepass(s) == cudaSuccess;
     if (ok && !s->prepass_smem) ok = alloc(s, &s->slot_scratch, T1B * 4);
     if (ok) ok = cudaMemset(s->err, 0, 16) == cudaSuccess;
+    if (ok) ok = cudaStreamCreateWithFlags(&s->side, cudaStreamNonBlocking) == cudaSuccess &&
+                 cudaEventCreateWithFlags(&s->side_go, cudaEventDisableTiming) == cudaSuccess &&
+                 cudaEventCreateWithFlags(&s->cleared, cudaEventDisableTiming) == cudaSuccess;
     if (!ok) {
+        if (s->side) cudaStreamDestroy(s->side);
+        if (s->side_go) cudaEventDestroy(s->side_go);
+        if (s->cleared) cudaEventDestroy(s->cleared);
         cudaGetLastError();
         free_all(s);
         delete s;
@@ -260,11 +266,21 @@ sl_status stacklstm_forward(stacklstm_t s, const void *x, const int8_t *ops, con
     }
     {
         Phase ph(s, SL_PHASE_FORWARD);
+        // the gradient history is cleared on the side stream while the forward runs (the
+        // forward leaves most of the memory bandwidth unused); the side stream first waits
+        // for everything queued on the caller's stream so far (a previous backward reads it)
+        if ((e = cudaEventRecord(s->side_go, s->stream))) return cuda_fail(s, e, "forward");
         if (s->dt == SL_FP32)
             e = sl::fp32_forward_steps(s, (const float *)x, (const float *)W, bias);
         else
             e = sl::bf16_forward_steps(s, bias);
         if (e) return cuda_fail(s, e, "forward");
+        const size_t hist_bytes = sizeof(float) * (size_t)(T + 1) * B * H;
+        if ((e = cudaStreamWaitEvent(s->side, s->side_go, 0)) ||
+            (e = cudaMemsetAsync(s->dhist_h, 0, hist_bytes, s->side)) ||
+            (e = cudaMemsetAsync(s->dhist_c, 0, hist_bytes, s->side)) || (e = cudaEventRecord(s->cleared, s->side)))
+            return cuda_fail(s, e, "clear");
+        s->clear_queued = 1;
     }
     {
         Phase ph(s, SL_PHASE_OUTPUTS);
@@ -303,8 +319,14 @@ sl_status stacklstm_backward(stacklstm_t s, const float *d_top_h, const float *d
     cudaError_t e;
     {
         Phase ph(s, SL_PHASE_BWD_SETUP);
-        if ((e = cudaMemsetAsync(s->dhist_h, 0, hist_bytes, s->stream))) return cuda_fail(s, e, "clear");
-        if ((e = cudaMemsetAsync(s->dhist_c, 0, hist_bytes, s->stream))) return cuda_fail(s, e, "clear");
+        if (s->clear_queued) {
+            // cleared on the side stream during the forward
+            if ((e = cudaStreamWaitEvent(s->stream, s->cleared, 0))) return cuda_fail(s, e, "clear");
+            s->clear_queued = 0;
+        } else {
+            if ((e = cudaMemsetAsync(s->dhist_h, 0, hist_bytes, s->stream))) return cuda_fail(s, e, "clear");
+            if ((e = cudaMemsetAsync(s->dhist_c, 0, hist_bytes, s->stream))) return cuda_fail(s, e, "clear");
+        }
         if ((e = sl::launch_seed_grads(s, d_top_h, dy))) return cuda_fail(s, e, "seed");
         if (s->dt == SL_BF16 && (e = sl::bf16_backward_setup(s))) return cuda_fail(s, e, "backward setup");
     }
@@ -373,6 +395,12 @@ sl_status stacklstm_destroy(stacklstm_t s)
     {
         DeviceGuard g(s->device);
         cudaStreamSynchronize(s->stream);
+        if (s->side) {
+            cudaStreamSynchronize(s->side);
+            cudaStreamDestroy(s->side);
+        }
+        if (s->side_go) cudaEventDestroy(s->side_go);
+        if (s->cleared) cudaEventDestroy(s->cleared);
         collect_timing(s);
         for (cudaEvent_t ev : s->event_pool) cudaEventDestroy(ev);
         s->event_pool.clear();

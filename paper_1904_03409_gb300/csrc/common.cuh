@@ -33,6 +33,11 @@ struct stacklstm {
     sl_dtype dt = SL_FP32;
     int device = 0;
     cudaStream_t stream = nullptr;
+    // the gradient history is cleared on a side stream during the forward: `side_go` marks
+    // the caller's stream before the forward steps, `cleared` the end of the clearing
+    cudaStream_t side = nullptr;
+    cudaEvent_t side_go = nullptr, cleared = nullptr;
+    int clear_queued = 0;
     int async = 0;
     int fwd_done = 0;
     int num_sms = 0;
