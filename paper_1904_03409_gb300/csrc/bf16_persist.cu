@@ -725,8 +725,8 @@ const Variant *bwd_variants(int *n)
 {
     static const Variant v[] = {variant<16, 1, 4, false>(), variant<16, 2, 4, false>(), variant<32, 2, 4, false>(),
                                 variant<32, 4, 4, false>(), variant<64, 2, 2, false>(), variant<64, 1, 2, false, 4>(),
-                                variant<64, 1, 4, false, 4>()};
-    *n = 7;
+                                variant<64, 1, 4, false, 4>(), variant<64, 2, 4, false>()};
+    *n = 8;
     return v;
 }
 
