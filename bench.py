@@ -295,11 +295,16 @@ def measure_workload(w, steps, warmup, local, world, sample_clocks, e2e):
     per_launch_units = w.B if per_step_kernels else w.B * w.T
     launches_per_step = w.T if per_step_kernels else 1
     launch_s = phase_ms[dom] / 1e3 / launches_per_step
-    rf = roofline_of(wk[dom]["flops"] * per_launch_units, wk[dom]["bytes"] * per_launch_units, launch_s, peaks, src,
-                     sustained=True)
+    fl, by = wk[dom]["flops"], wk[dom]["bytes"]
+    m = re.search(r"dx CTAs (\d+)", plan)
+    if dom == "backward" and m and int(m.group(1)) > 0:
+        # the backward launch also computed dx on the SMs its step chain leaves idle
+        fl, by = fl + wk["dx"]["flops"], by + wk["dx"]["bytes"]
+        kname += "+dx"
+    rf = roofline_of(fl * per_launch_units, by * per_launch_units, launch_s, peaks, src, sustained=True)
     rf.update({"kernel": kname, "phase": dom, "launch_us": launch_s * 1e6,
                "units_per_launch": per_launch_units, "unit_of_work": "instance-step",
-               "algorithmic_flops_per_unit": wk[dom]["flops"], "algorithmic_bytes_per_unit": wk[dom]["bytes"],
+               "algorithmic_flops_per_unit": fl, "algorithmic_bytes_per_unit": by,
                "traffic": kernel_traffic(kname, kfile, w.name)})
     sec = total_ms / 1e3 / steps
     srf = roofline_of(wk["step"]["flops"] * w.B * w.T, wk["step"]["bytes"] * w.B * w.T, sec, peaks, src,

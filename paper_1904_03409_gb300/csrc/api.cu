@@ -330,12 +330,13 @@ sl_status stacklstm_backward(stacklstm_t s, const float *d_top_h, const float *d
         if ((e = sl::launch_seed_grads(s, d_top_h, dy))) return cuda_fail(s, e, "seed");
         if (s->dt == SL_BF16 && (e = sl::bf16_backward_setup(s))) return cuda_fail(s, e, "backward setup");
     }
+    bool dx_done = false;  // computed by the step launch on otherwise idle SMs
     {
         Phase ph(s, SL_PHASE_BACKWARD);
-        e = s->dt == SL_FP32 ? sl::fp32_backward_steps(s) : sl::bf16_backward_steps(s);
+        e = s->dt == SL_FP32 ? sl::fp32_backward_steps(s) : sl::bf16_backward_steps(s, dx, &dx_done);
         if (e) return cuda_fail(s, e, "backward");
     }
-    {
+    if (!dx_done) {
         Phase ph(s, SL_PHASE_DX);
         e = s->dt == SL_FP32 ? sl::fp32_dx(s, dx) : sl::bf16_dx(s, dx);
         if (e) return cuda_fail(s, e, "dx");

@@ -174,7 +174,8 @@ bool bf16_plan_fwd_persist(stacklstm *s, PersistPlan *pl);
 bool bf16_plan_bwd_persist(stacklstm *s, PersistPlan *pl);
 cudaError_t bf16_launch_fwd_persist(stacklstm *s, const StepArgs &a, const CUtensorMap &tm_x, const CUtensorMap &tm_h,
                                     const CUtensorMap &tm_gates);
-cudaError_t bf16_launch_bwd_persist(stacklstm *s, const StepArgs &a, const CUtensorMap &tm_g);
+cudaError_t bf16_launch_bwd_persist(stacklstm *s, const StepArgs &a, const CUtensorMap &tm_g, float *dx,
+                                    bool *dx_done);
 
 // ---- weight / bias gradients (bf16_dw.cu)
 cudaError_t bf16_plan_dw(stacklstm *s);

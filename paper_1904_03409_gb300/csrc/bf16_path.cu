@@ -521,11 +521,11 @@ std::string bf16_describe(const stacklstm *s)
              "bf16 tcgen05; row tiles %d; chunks fwd %d (x %d) bwd %d; "
              "forward %s U=%d [EP %d G %d ring %d slots %d cluster %d col tiles %d w_res %d smem %u threads %d]; "
              "backward %s U=%d [EP %d G %d ring %d slots %d cluster %d col tiles %d w_res %d smem %u threads %d "
-             "contraction parts %d]; "
+             "contraction parts %d dx CTAs %d ring %d]; "
              "step rings fwd %d bwd %d; dx N=%d x%d ring %d; dW %dx%d tiles of 128x%d x%d splits ring %d",
              rt, s->kcf, s->kcx, s->kcb, f.on ? "persistent" : "per-step", s->uf, f.EP, f.G, f.S, f.slot, f.cl, f.n_ct,
              f.w_res, f.smem, f.threads, b.on ? "persistent" : "per-step", s->ub, b.EP, b.G, b.S, b.slot, b.cl, b.n_ct,
-             b.w_res, b.smem, b.threads, b.KS, s->sf, s->sb, s->nx, s->nxt, s->sx, s->dw_mt, s->dw_nt, s->dw_ntile, s->dw_split, s->sw);
+             b.w_res, b.smem, b.threads, b.KS, b.n_dx, b.dx_S, s->sf, s->sb, s->nx, s->nxt, s->sx, s->dw_mt, s->dw_nt, s->dw_ntile, s->dw_split, s->sw);
     return buf;
 }
 
@@ -666,8 +666,10 @@ cudaError_t bf16_backward_setup(stacklstm *s)
     return cudaGetLastError();
 }
 
-cudaError_t bf16_backward_steps(stacklstm *s)
+// With dx and a plan that has spare SMs, the persistent launch also computes dx (*dx_done).
+cudaError_t bf16_backward_steps(stacklstm *s, float *dx, bool *dx_done)
 {
+    *dx_done = false;
     const int T = s->T, B = s->B, H = s->H;
     cudaError_t e;
     const StepArgs a = step_args(s, nullptr, s->w_bwd, 0, s->kcb, s->sb);
@@ -675,7 +677,7 @@ cudaError_t bf16_backward_steps(stacklstm *s)
     // loaded and only feeds accumulator rows that are not stored)
     if (s->pb.on)
         return bf16_launch_bwd_persist(s, step_args(s, nullptr, s->w_bwd, 0, s->kcb, s->pb.S),
-                                       map(s, B <= 64 ? kMapG64 : kMapG128));
+                                       map(s, B <= 64 ? kMapG64 : kMapG128), dx, dx_done);
     const dim3 grid(ceil_div(H, s->ub), ceil_div(B, kRows));
     const size_t smem = smem_bytes(s->sb, s->ub);
     const CUtensorMap &tmg = map(s, kMapG128);

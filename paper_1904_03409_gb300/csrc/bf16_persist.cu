@@ -51,6 +51,13 @@ struct WsArgs {
     int a_rows;              // rows per A box: 128, or 64 when B <= 64 (one half-filled row tile)
     float *part;             // split contraction: [n_rt][n_ct][KS][128][U] partial dh_read rows
     int32_t *pcnt;           // split contraction: [n_rt][n_ct] partials written, zero at launch
+    // backward: CTAs n_chain .. n_chain + n_dx - 1 compute the input gradient alongside the steps
+    int n_chain, n_dx;
+    int dx_S;                // their ring stages
+    int dx_v8;               // dx is 32-byte aligned (whole-sector row stores)
+    int nxt;                 // 256-column tiles of dx
+    float *dx;               // [T B][I]
+    const uint8_t *wdx;      // W_x packed as [nxt][KC][256 rows][64], 128-byte swizzled rows
 };
 
 // Dynamic shared memory: [weight tile (w_res)][S stages: G A chunks, then G weight
@@ -114,14 +121,14 @@ __device__ __forceinline__ void ws_abort(const WCtl &c, int32_t *err)
 // Bounded spin until *cnt >= target (acquire). False on timeout, on a local abort, or
 // once another CTA recorded an error.
 __device__ __forceinline__ bool spin_until(const int32_t *cnt, int target, long long limit, volatile int *abort,
-                                           const int32_t *err)
+                                           const int32_t *err, unsigned sleep_ns = 32)
 {
     if (tc::ld_acquire_gpu(cnt) >= target) return true;
     const long long t0 = clock64();
     while (true) {
         if (clock64() - t0 >= limit) return false;
         if (*abort || *(const volatile int32_t *)err) return false;
-        __nanosleep(32);
+        __nanosleep(sleep_ns);
         if (tc::ld_acquire_gpu(cnt) >= target) return true;
     }
 }
@@ -517,6 +524,189 @@ __device__ __forceinline__ void epilogue_loop(const StepArgs &a, const WsArgs &p
         if (e.tid == 0) tc::bulk_wait();  // the gate stores completed before the CTA exits
 }
 
+// ------------------------------------------------------------------ input gradient
+// Backward only. The CTAs past the step chain compute dx = dG W_x^T (the input part of the
+// gate-gradient contraction, Sec. 5) on SMs the chain leaves idle. The [T B][4H] gate
+// gradient is cut into 128-row tiles, taken from the last row down so that each tile
+// trails the chain step that completed it; this CTA takes every n_dx-th (tile, 256-column
+// slice of dx) pair. Before loading a tile whose earliest row belongs to step t_lo, the
+// producer waits until every row tile of the chain has completed T - 1 - t_lo steps
+// (chain step t writes the gate gradient of step t - 1, so the rows of t_lo and later are
+// then final), then streams the 4H / 64 contraction chunks with the matching 256-row
+// slices of W_x through an S-stage ring. Accumulators alternate between the two 256-column halves of tensor memory; the
+// epilogue warps store their rows of the finished one while the next tile is multiplied.
+// The role is inlined into the kernel: compiled as a called function, its 32-byte row
+// stores wrote only their first word (found with a NaN-filled output).
+constexpr int kDxN = 256;
+
+template <int EP>
+__device__ __forceinline__ void dx_role(const CUtensorMap *tm_g, const WsArgs &p, uint8_t *smem_raw, int per_step)
+{
+    constexpr int E = 4 * EP;
+    constexpr int CPT = kDxN / EP;  // dx columns per epilogue thread
+    constexpr uint32_t kWChunk = kDxN * 128;
+    const StepArgs &a = p.s;
+    const int T = a.T, B = a.B, I = a.I, KC = a.KC, S = p.dx_S;
+    const size_t R = (size_t)T * B;
+    const int n_rows = (int)((R + kRows - 1) / kRows);
+    const int n_items = n_rows * p.nxt;
+    const int did = (int)blockIdx.x - p.n_chain;
+    const int n_mine = did < n_items ? (n_items - did + p.n_dx - 1) / p.n_dx : 0;
+    const long long limit = a.limit;
+    const WCtl c = wcarve(smem_raw, S, 1, kDxN, KC, 0, 0u);
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    if (tid == 0) {
+        for (int s = 0; s < S; ++s) {
+            tc::mbar_init(&c.full[s], 1);
+            tc::mbar_init(&c.empty[s], 1);
+        }
+        for (int i = 0; i < 2; ++i) {
+            tc::mbar_init(&c.tfull[i], 1);
+            tc::mbar_init(&c.tempty[i], E);
+        }
+        tc::mbar_init(c.done, 1);
+        *c.n_issued = 0;
+        *c.n_consumed = 0;
+        *c.abort = 0;
+        tc::fence_mbar_init();
+    }
+    if (warp == E) tc::tmem_alloc(c.tmem_slot, 2 * kDxN);
+    tc::tc_fence_before();
+    __syncthreads();
+    tc::tc_fence_after();
+    const uint32_t tmem = *c.tmem_slot;
+    auto item = [&](int j, int &row0, int &xt) {
+        const int i = did + j * p.n_dx;
+        row0 = (n_rows - 1 - i / p.nxt) * kRows;
+        xt = i % p.nxt;
+    };
+
+    if (warp == E) {
+        // ------------------------------------------------------------ producer
+        if (lane == 0) {
+            uint32_t g = 0;
+            for (int j = 0; j < n_mine && !*c.abort; ++j) {
+                int row0, xt;
+                item(j, row0, xt);
+                // the row tiles holding the tile's rows: instances b0 .. of step t_lo, and
+                // (B >= 128) at most instances 0 .. 127 of step t_lo + 1; polled slowly, as
+                // the chain's own hand-offs use the same counters
+                const int t_lo = row0 / B, b0 = row0 - t_lo * B, b1 = min(B - 1, b0 + kRows - 1);
+                bool ok = true;
+                for (int rt = b0 / kRows; rt <= b1 / kRows && ok; ++rt)
+                    ok = spin_until(p.cnt + rt, per_step * (T - 1 - t_lo), limit, c.abort, a.err, 1000);
+                if (ok && b0 + kRows > B && t_lo + 1 < T)
+                    ok = spin_until(p.cnt, per_step * (T - 2 - t_lo), limit, c.abort, a.err, 1000);
+                if (!ok) {
+                    ws_abort(c, a.err);
+                    break;
+                }
+                tc::fence_proxy_async_global();
+                const uint8_t *wt = p.wdx + (size_t)xt * KC * kWChunk;
+                bool bad = false;
+                for (int kc = 0; kc < KC; ++kc) {
+                    const int s = (int)(g % S);
+                    if (g >= (uint32_t)S && !tc::mbar_wait(&c.empty[s], (g / S - 1) & 1, limit, c.abort)) {
+                        ws_abort(c, a.err);
+                        bad = true;
+                        break;
+                    }
+                    const uint32_t st = c.ring0 + s * c.stage;
+                    tc::mbar_arrive_expect_tx(&c.full[s], kAStage + kWChunk);
+                    tc::tma_load_2d(st, tm_g, kc * kChunk, row0, &c.full[s]);
+                    tc::bulk_g2s(st + kAStage, wt + (size_t)kc * kWChunk, kWChunk, &c.full[s]);
+                    ++g;
+                }
+                if (bad) break;
+            }
+            *c.n_issued = (int)g;
+        }
+        __syncwarp();
+    } else if (warp == E + 1) {
+        // ------------------------------------------------------------ MMA issue
+        if (lane == 0) {
+            uint32_t g = 0;
+            for (int j = 0; j < n_mine && !*c.abort; ++j) {
+                const int acc = j & 1;
+                if (j >= 2 && !tc::mbar_wait(&c.tempty[acc], ((j >> 1) - 1) & 1, limit, c.abort)) {
+                    ws_abort(c, a.err);
+                    break;
+                }
+                tc::tc_fence_after();
+                const uint32_t d = tmem + acc * kDxN;
+                bool bad = false;
+                for (int kc = 0; kc < KC; ++kc) {
+                    const int s = (int)(g % S);
+                    if (!tc::mbar_wait(&c.full[s], (g / S) & 1, limit, c.abort)) {
+                        ws_abort(c, a.err);
+                        bad = true;
+                        break;
+                    }
+                    tc::tc_fence_after();
+                    const uint32_t st = c.ring0 + s * c.stage;
+                    issue_group<kDxN, 1>(d, st, st + kAStage, 1, kc == 0);
+                    tc::mma_commit(&c.empty[s]);
+                    ++g;
+                }
+                if (bad) break;
+                tc::mma_commit(&c.tfull[acc]);
+            }
+            *c.n_consumed = (int)g;
+            tc::mma_commit(c.done);
+        }
+        __syncwarp();
+    } else {
+        // ------------------------------------------------------------ epilogue
+        const int q = warp & 3, part = warp >> 2;
+        for (int j = 0; j < n_mine; ++j) {
+            int row0, xt;
+            item(j, row0, xt);
+            const int acc = j & 1;
+            const bool ok = tc::mbar_wait(&c.tfull[acc], (j >> 1) & 1, limit, c.abort);
+            if (!ok) {
+                ws_abort(c, a.err);
+                break;
+            }
+            tc::tc_fence_after();
+            const size_t row = (size_t)row0 + q * 32 + lane;
+            const uint32_t taddr = tmem + acc * kDxN + ((uint32_t)(q * 32) << 16) + part * CPT;
+            float *drow = p.dx + row * I;
+#pragma unroll 1
+            for (int cg = 0; cg < CPT / 16; ++cg) {
+                uint32_t v[16];
+                tmem_cols<16>(taddr + cg * 16, v);
+                tc::tmem_wait_ld();
+                const int col = xt * kDxN + part * CPT + cg * 16;
+                if (row < R) {
+#pragma unroll
+                    for (int h = 0; h < 2; ++h)
+                        if (col + 8 * h < I) {  // I is a multiple of 8
+                            if (p.dx_v8)
+                                st_v8(drow + col + 8 * h, v + 8 * h);
+                            else {
+                                st_v4(drow + col + 8 * h, v + 8 * h);
+                                st_v4(drow + col + 8 * h + 4, v + 8 * h + 4);
+                            }
+                        }
+                }
+            }
+            tc::tc_fence_before();
+            __syncwarp();
+            if (lane == 0) tc::mbar_arrive(&c.tempty[acc]);
+        }
+    }
+
+    // ---------------------------------------------------------------- teardown
+    __syncthreads();
+    if (warp == E && lane == 0)
+        for (int g = *c.n_consumed; g < *c.n_issued; ++g)
+            tc::mbar_wait(&c.full[g % S], (uint32_t)(g / S) & 1, kDrainLimit, nullptr);
+    if (warp == E + 1 && lane == 0) tc::mbar_wait(c.done, 0, kDrainLimit, nullptr);
+    tc::tc_fence_before();
+    __syncthreads();
+    if (warp == E) tc::tmem_dealloc(tmem, 2 * kDxN);
+}
+
 // ------------------------------------------------------------------ the kernel
 // kFwd: forward (tm_a = x_t tiles for chunks < kcx, tm_b = hr[t] tiles after them);
 // else backward (tm_b = dG_t tiles, kcx = 0: every chunk depends on the step before).
@@ -536,6 +726,11 @@ step_ws(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtens
     const StepArgs &a = p.s;
     extern __shared__ uint8_t smem_raw[];
     __shared__ float s_bias[kFwd ? 4 * U : 4];
+    if constexpr (!kFwd)
+        if ((int)blockIdx.x >= p.n_chain) {
+            dx_role<EP>(&tm_b, p, smem_raw, p.n_ct * KS);
+            return;
+        }
     const int S = a.S, KC = a.KC, split = a.kcx, T = a.T, B = a.B, H = a.H;
     const int kp = (int)(blockIdx.x % KS), cidx = (int)(blockIdx.x / KS);
     const int k0 = KC * kp / KS, k1 = KC * (kp + 1) / KS;  // this CTA's contraction chunks
@@ -858,6 +1053,15 @@ bool plan_variant(const Variant &v, bool fwd, int KC, int split, int n_rt, int H
     return found;
 }
 
+const void *find_fn(bool fwd, const PersistPlan &pl)
+{
+    int n;
+    const Variant *vs = fwd ? fwd_variants(&n) : bwd_variants(&n);
+    for (int i = 0; i < n; ++i)
+        if (vs[i].U == pl.U && vs[i].EP == pl.EP && vs[i].G == pl.G && vs[i].KS == pl.KS) return vs[i].fn;
+    return nullptr;
+}
+
 bool plan(stacklstm *s, bool fwd, PersistPlan *pl)
 {
     int n;
@@ -893,15 +1097,37 @@ bool plan(stacklstm *s, bool fwd, PersistPlan *pl)
             found = true;
         }
     }
-    if (!found) pl->on = 0;
-    return found;
+    if (!found) {
+        pl->on = 0;
+        return false;
+    }
+    pl->n_dx = 0;
+    pl->dx_S = 0;
+    if (!fwd) {
+        // the input gradient on the SMs the chain leaves idle: one CTA per SM (the role
+        // takes all 512 tensor-memory columns), 256-column dx tiles, full 128-row A boxes
+        const char *fx = getenv("STACKLSTM_DX_SPARE");
+        int r = 0;
+        const int n_chain = pl->n_ct * pl->KS * pl->slot;
+        const int spare = s->num_sms - n_chain;
+        const int S = (int)std::min<uint32_t>(kMaxStages, (pl->smem - 1024 - kBarBytes) / (kAStage + 256u * 128));
+        if ((!fx || atoi(fx) != 0) && s->nx == 256 && s->B >= kRows && pl->cl == 1 && spare >= 4 && S >= 2 &&
+            cudaOccupancyMaxActiveBlocksPerMultiprocessor(&r, find_fn(false, *pl), pl->threads, pl->smem) ==
+                cudaSuccess &&
+            r == 1) {
+            pl->n_dx = fx && atoi(fx) > 0 ? std::min(spare, atoi(fx)) : spare;
+            pl->dx_S = S;
+        }
+        cudaGetLastError();
+    }
+    return true;
 }
 
 template <typename... Args>
-cudaError_t launch_coop(const void *fn, const PersistPlan &pl, cudaStream_t st, Args... args)
+cudaError_t launch_coop(const void *fn, const PersistPlan &pl, int grid, cudaStream_t st, Args... args)
 {
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(pl.n_ct * pl.KS * pl.slot);
+    cfg.gridDim = dim3(grid);
     cfg.blockDim = dim3(pl.threads);
     cfg.dynamicSmemBytes = pl.smem;
     cfg.stream = st;
@@ -918,15 +1144,6 @@ cudaError_t launch_coop(const void *fn, const PersistPlan &pl, cudaStream_t st, 
     return cudaLaunchKernelExC(&cfg, fn, argv);
 }
 
-const void *find_fn(bool fwd, const PersistPlan &pl)
-{
-    int n;
-    const Variant *vs = fwd ? fwd_variants(&n) : bwd_variants(&n);
-    for (int i = 0; i < n; ++i)
-        if (vs[i].U == pl.U && vs[i].EP == pl.EP && vs[i].G == pl.G && vs[i].KS == pl.KS) return vs[i].fn;
-    return nullptr;
-}
-
 }  // namespace
 
 bool bf16_plan_fwd_persist(stacklstm *s, PersistPlan *pl) { return plan(s, true, pl); }
@@ -936,7 +1153,7 @@ cudaError_t bf16_launch_fwd_persist(stacklstm *s, const StepArgs &a, const CUten
                                     const CUtensorMap &tm_gates)
 {
     const PersistPlan &pl = s->pf;
-    WsArgs p;
+    WsArgs p{};
     p.s = a;
     p.s.S = pl.S;
     p.n_ct = pl.n_ct;
@@ -953,16 +1170,17 @@ cudaError_t bf16_launch_fwd_persist(stacklstm *s, const StepArgs &a, const CUten
     if (e) return e;
     const void *fn = find_fn(true, pl);
     if (!fn) return cudaErrorInvalidDeviceFunction;
-    e = launch_coop(fn, pl, s->stream, tm_x, tm_h, tm_gates, p);
+    e = launch_coop(fn, pl, pl.n_ct * pl.slot, s->stream, tm_x, tm_h, tm_gates, p);
     if (e) return e;
     s->launches += 1;
     return cudaGetLastError();
 }
 
-cudaError_t bf16_launch_bwd_persist(stacklstm *s, const StepArgs &a, const CUtensorMap &tm_g)
+cudaError_t bf16_launch_bwd_persist(stacklstm *s, const StepArgs &a, const CUtensorMap &tm_g, float *dx,
+                                    bool *dx_done)
 {
     const PersistPlan &pl = s->pb;
-    WsArgs p;
+    WsArgs p{};
     p.s = a;
     p.s.S = pl.S;
     p.s.kcx = 0;
@@ -976,14 +1194,22 @@ cudaError_t bf16_launch_bwd_persist(stacklstm *s, const StepArgs &a, const CUten
     p.part = s->split_part;
     p.pcnt = s->split_cnt;
     p.a_rows = s->B <= 64 ? 64 : kRows;
+    p.n_chain = pl.n_ct * pl.KS * pl.slot;
+    p.n_dx = dx ? pl.n_dx : 0;
+    p.dx_S = pl.dx_S;
+    p.dx_v8 = ((uintptr_t)dx & 31) == 0;
+    p.nxt = s->nxt;
+    p.dx = dx;
+    p.wdx = (const uint8_t *)s->w_dx;
     cudaError_t e = cudaMemsetAsync(p.cnt, 0, sizeof(int32_t) * p.n_rt, s->stream);
     if (e) return e;
     if (pl.KS > 1 && (e = cudaMemsetAsync(p.pcnt, 0, sizeof(int32_t) * p.n_rt * p.n_ct, s->stream))) return e;
     const void *fn = find_fn(false, pl);
     if (!fn) return cudaErrorInvalidDeviceFunction;
-    e = launch_coop(fn, pl, s->stream, tm_g, tm_g, tm_g, p);
+    e = launch_coop(fn, pl, p.n_chain + p.n_dx, s->stream, tm_g, tm_g, tm_g, p);
     if (e) return e;
     s->launches += 1;
+    *dx_done = p.n_dx > 0;
     return cudaGetLastError();
 }
 

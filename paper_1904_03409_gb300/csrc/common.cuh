@@ -25,6 +25,8 @@ struct PersistPlan {
     int n_ct = 0;       // column tiles, padded to a multiple of cl
     unsigned smem = 0;  // dynamic shared memory per CTA
     int threads = 0;    // threads per CTA
+    int n_dx = 0;       // backward: extra CTAs computing dx on the SMs the steps leave idle
+    int dx_S = 0;       // their ring stages
 };
 
 // The handle: problem sizes, stream, and the device workspace it owns.
@@ -124,7 +126,7 @@ cudaError_t bf16_forward_setup(stacklstm *s, const __nv_bfloat16 *x, const __nv_
                                const float *c0, const __nv_bfloat16 *W);
 cudaError_t bf16_forward_steps(stacklstm *s, const float *bias);
 cudaError_t bf16_backward_setup(stacklstm *s);
-cudaError_t bf16_backward_steps(stacklstm *s);
+cudaError_t bf16_backward_steps(stacklstm *s, float *dx, bool *dx_done);
 cudaError_t bf16_dx(stacklstm *s, float *dx);
 cudaError_t bf16_dw(stacklstm *s, float *dW, float *dbias);
 size_t bf16_workspace_bytes(int T, int B, int I, int H, int num_sms);

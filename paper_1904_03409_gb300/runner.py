@@ -61,6 +61,9 @@ def run(w, device: int = 0, d_top_h: Optional[np.ndarray] = None) -> dict:
     try:
         ins = upload(w, device)
         out = alloc_outputs(w, device)
+        for v in out.values():  # an element the path does not write cannot match the oracle
+            if v.is_floating_point():
+                v.fill_(float("nan"))
         seed = None if d_top_h is None else torch.from_numpy(np.ascontiguousarray(d_top_h, np.float32)).to(
             ins["x"].device)
         forward_backward(hd, ins, out, d_top_h=seed)

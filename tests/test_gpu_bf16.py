@@ -9,6 +9,7 @@ restricted to them, so dW and dbias are the sums over exactly those instances.
 Pointer trajectories and read provenance are compared bit for bit for all instances.
 """
 import os
+import re
 
 import numpy as np
 import pytest
@@ -168,3 +169,51 @@ def test_split_contraction_backward_matches_oracle(T, B, I, H, seed):
     compare(got, oracle_all(w), "bf16")
     for k in ("dx", "dW", "dbias", "dh0", "dc0"):
         assert np.array_equal(got[k], again[k]), k
+
+
+def run_nan_filled(w, env):
+    """Forward + backward with every output buffer filled with NaN first (an element the
+    path fails to write cannot pass), under extra environment settings; (plan, dx)."""
+    old = {k: os.environ.get(k) for k in env}
+    os.environ.update(env)
+    try:
+        hd = bd.stacklstm_create(w.T, w.B, w.I, w.H, bd.SL_BF16, 0)
+    finally:
+        for k, v in old.items():
+            if v is None:
+                os.environ.pop(k, None)
+            else:
+                os.environ[k] = v
+    try:
+        plan = bd.stacklstm_plan(hd)
+        ins = runner.upload(w)
+        out = runner.alloc_outputs(w)
+        for v in out.values():
+            if v.is_floating_point():
+                v.fill_(float("nan"))
+        runner.forward_backward(hd, ins, out)
+        torch.cuda.synchronize()
+        bd.stacklstm_status(hd)
+        return plan, runner.to_numpy(out)
+    finally:
+        hd.destroy()
+
+
+@pytest.mark.parametrize("T,B,I,H,seed", [(11, 200, 264, 64, 16), (9, 129, 256, 256, 17), (40, 512, 256, 256, 18)])
+def test_input_gradient_on_spare_sms_matches_oracle(T, B, I, H, seed):
+    """dx computed by the extra CTAs of the backward launch, on the SMs the step chain
+    leaves idle (128-row tiles that straddle two steps; I = 264: a second, partial
+    256-column tile; B = 512: several tiles per extra CTA), into NaN-filled outputs,
+    matches the oracle and equals bit for bit the separate dx launch (same contraction
+    chunk order). A single extra CTA, trailing the whole chain, too."""
+    w = case(T, B, I, H, seed, bias_scale=0.3, h0_scale=0.5, c0_scale=0.5, dy_scale=0.5)
+    plan, got = run_nan_filled(w, {})
+    m = re.search(r"dx CTAs (\d+)", plan)
+    assert m and int(m.group(1)) >= 4, plan
+    compare(got, oracle_all(w), "bf16")
+    plan0, sep = run_nan_filled(w, {"STACKLSTM_DX_SPARE": "0"})
+    assert "dx CTAs 0" in plan0, plan0
+    assert np.array_equal(got["dx"], sep["dx"])
+    plan1, one = run_nan_filled(w, {"STACKLSTM_DX_SPARE": "1"})
+    assert "dx CTAs 1" in plan1, plan1
+    assert np.array_equal(one["dx"], sep["dx"])
