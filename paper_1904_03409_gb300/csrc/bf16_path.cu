@@ -591,7 +591,8 @@ cudaError_t bf16_prepare(stacklstm *s)
         s->split_cnt = (int32_t *)p;
     }
     if (s->pf.on || s->pb.on) {
-        if ((e = cudaMalloc(&p, 2 * sizeof(int32_t) * rt))) return e;
+        if (const char *cs = getenv("STACKLSTM_CNT_STRIDE")) s->cnt_stride = std::max(1, atoi(cs));
+        if ((e = cudaMalloc(&p, 2 * sizeof(int32_t) * rt * s->cnt_stride))) return e;
         s->allocs.push_back(p);
         s->rowcnt = (int32_t *)p;
     }

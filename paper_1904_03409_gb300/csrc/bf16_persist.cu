@@ -46,7 +46,8 @@ struct WsArgs {
     int n_ct, n_rt, n_slot;  // column tiles (a multiple of cl); row tiles; CTAs per column tile
     int w_res;               // 1: weight tile resident in shared memory
     int cl;                  // cluster size along the column tiles (1: no multicast)
-    int32_t *cnt;            // [n_rt] completed steps per row tile, zero at launch
+    int32_t *cnt;            // [n_rt] completed steps per row tile (cs ints apart), zero at launch
+    int cs;                  // counter stride in ints
     int vec32;               // H % 16 == 0: 16-unit groups of 16-bit rows are 32-byte aligned
     int a_rows;              // rows per A box: 128, or 64 when B <= 64 (one half-filled row tile)
     float *part;             // split contraction: [n_rt][n_ct][KS][128][U] partial dh_read rows
@@ -507,7 +508,7 @@ __device__ __forceinline__ void epilogue_loop(const StepArgs &a, const WsArgs &p
         if constexpr (kFwd) tc::fence_proxy_async();  // staging-tile writes -> the tensor store
         __syncwarp();
         tc::bar_sync(2, E * 32);
-        if (e.tid == 0) tc::red_release_gpu_add(p.cnt + rt, 1);
+        if (e.tid == 0) tc::red_release_gpu_add(p.cnt + rt * p.cs, 1);
         if constexpr (kFwd) {
             if (e.tid == 0) {
 #pragma unroll
@@ -594,7 +595,7 @@ __device__ __forceinline__ void dx_role(const CUtensorMap *tm_g, const WsArgs &p
                 const int t_lo = row0 / B, b0 = row0 - t_lo * B, b1 = min(B - 1, b0 + kRows - 1);
                 bool ok = true;
                 for (int rt = b0 / kRows; rt <= b1 / kRows && ok; ++rt)
-                    ok = spin_until(p.cnt + rt, per_step * (T - 1 - t_lo), limit, c.abort, a.err, 1000);
+                    ok = spin_until(p.cnt + rt * p.cs, per_step * (T - 1 - t_lo), limit, c.abort, a.err, 1000);
                 if (ok && b0 + kRows > B && t_lo + 1 < T)
                     ok = spin_until(p.cnt, per_step * (T - 2 - t_lo), limit, c.abort, a.err, 1000);
                 if (!ok) {
@@ -788,7 +789,7 @@ step_ws(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtens
                     if (c0 == dep_c && ks > 0) {
                         // every column tile (and contraction part) of this row tile
                         // finished the step before
-                        if (!spin_until(p.cnt + rt, p.n_ct * KS * ks, limit, c.abort, a.err)) {
+                        if (!spin_until(p.cnt + rt * p.cs, p.n_ct * KS * ks, limit, c.abort, a.err)) {
                             ws_abort(c, a.err);
                             break;
                         }
@@ -1162,11 +1163,12 @@ cudaError_t bf16_launch_fwd_persist(stacklstm *s, const StepArgs &a, const CUten
     p.w_res = pl.w_res;
     p.cl = pl.cl;
     p.cnt = s->rowcnt;
+    p.cs = s->cnt_stride;
     p.vec32 = s->H % 16 == 0;
     p.part = nullptr;
     p.pcnt = nullptr;
     p.a_rows = s->B <= 64 ? 64 : kRows;
-    cudaError_t e = cudaMemsetAsync(p.cnt, 0, sizeof(int32_t) * p.n_rt, s->stream);
+    cudaError_t e = cudaMemsetAsync(p.cnt, 0, sizeof(int32_t) * p.n_rt * p.cs, s->stream);
     if (e) return e;
     const void *fn = find_fn(true, pl);
     if (!fn) return cudaErrorInvalidDeviceFunction;
@@ -1189,7 +1191,8 @@ cudaError_t bf16_launch_bwd_persist(stacklstm *s, const StepArgs &a, const CUten
     p.n_slot = pl.slot;
     p.w_res = pl.w_res;
     p.cl = pl.cl;
-    p.cnt = s->rowcnt + p.n_rt;
+    p.cs = s->cnt_stride;
+    p.cnt = s->rowcnt + p.n_rt * p.cs;
     p.vec32 = s->H % 16 == 0;
     p.part = s->split_part;
     p.pcnt = s->split_cnt;
@@ -1201,7 +1204,7 @@ cudaError_t bf16_launch_bwd_persist(stacklstm *s, const StepArgs &a, const CUten
     p.nxt = s->nxt;
     p.dx = dx;
     p.wdx = (const uint8_t *)s->w_dx;
-    cudaError_t e = cudaMemsetAsync(p.cnt, 0, sizeof(int32_t) * p.n_rt, s->stream);
+    cudaError_t e = cudaMemsetAsync(p.cnt, 0, sizeof(int32_t) * p.n_rt * p.cs, s->stream);
     if (e) return e;
     if (pl.KS > 1 && (e = cudaMemsetAsync(p.pcnt, 0, sizeof(int32_t) * p.n_rt * p.n_ct, s->stream))) return e;
     const void *fn = find_fn(false, pl);

@@ -79,7 +79,8 @@ struct stacklstm {
     alignas(64) unsigned char tmaps[8][128] = {};  // TMA descriptors (bf16_path.cu)
     // persistent step kernels (one launch for all T steps; bf16_persist.cu)
     PersistPlan pf, pb;            // forward, backward (on = 0: one launch per step)
-    int32_t *rowcnt = nullptr;     // [2][row tiles] completed steps per row tile
+    int32_t *rowcnt = nullptr;     // [2][row tiles][cnt_stride] completed steps per row tile
+    int cnt_stride = 32;           // ints between two row tiles' counters (one 128-byte line each)
     float *split_part = nullptr;   // backward split contraction: partial dh_read rows
     int32_t *split_cnt = nullptr;  // backward split contraction: partials written per tile pair
     int nx = 0, nxt = 0;     // input gradient: columns per tile, number of column tiles
