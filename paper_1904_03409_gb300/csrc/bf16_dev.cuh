@@ -173,7 +173,8 @@ cudaError_t allow_smem(Kern k)
 bool bf16_plan_fwd_persist(stacklstm *s, PersistPlan *pl);
 bool bf16_plan_bwd_persist(stacklstm *s, PersistPlan *pl);
 cudaError_t bf16_launch_fwd_persist(stacklstm *s, const StepArgs &a, const CUtensorMap &tm_x, const CUtensorMap &tm_h,
-                                    const CUtensorMap &tm_gates);
+                                    const CUtensorMap &tm_gates, const CUtensorMap &tm_hh,
+                                    const CUtensorMap &tm_hc);
 cudaError_t bf16_launch_bwd_persist(stacklstm *s, const StepArgs &a, const CUtensorMap &tm_g, float *dx,
                                     bool *dx_done);
 

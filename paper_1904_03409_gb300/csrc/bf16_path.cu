@@ -461,6 +461,15 @@ cudaError_t make_map(void *slot, const void *base, uint64_t rows, uint64_t cols,
     return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
 }
 
+// Swizzle mode of a staging tile whose rows are `bytes` long (16 to 128): the forward's
+// epilogue writes its staging tiles in this layout.
+CUtensorMapSwizzle stage_swizzle(uint32_t bytes)
+{
+    return bytes >= 128 ? CU_TENSOR_MAP_SWIZZLE_128B
+                        : bytes == 64 ? CU_TENSOR_MAP_SWIZZLE_64B
+                                      : bytes == 32 ? CU_TENSOR_MAP_SWIZZLE_32B : CU_TENSOR_MAP_SWIZZLE_NONE;
+}
+
 // The saved gates [T][B][4][H] (fp16) as a 4-D tensor for the forward's tensor stores:
 // boxes of `units` hidden units x 1 gate x rows instances x 1 step, so a store never
 // writes past H (into the next gate) or past B (into the next step).
@@ -471,12 +480,29 @@ cudaError_t make_gates_map(void *slot, const void *base, int T, int B, int H, ui
     cuuint32_t box[4] = {units, 1, (cuuint32_t)std::min(B, kRows), 1};
     cuuint32_t es[4] = {1, 1, 1, 1};
     CUresult r = g_encode((CUtensorMap *)slot, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 4, const_cast<void *>(base), dims,
-                          strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+                          strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, stage_swizzle(units * 2),
                           CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
 }
 
-enum { kMapX128 = 0, kMapX64 = 1, kMapG128 = 2, kMapG64 = 3, kMapH128 = 4, kMapH64 = 5, kMapGates = 6 };
+// The history rows h' [T+1][B][H] (bf16) or c' (fp32) as a 3-D tensor for the forward's
+// tensor stores: boxes of `units` hidden units x rows instances x 1 step.
+cudaError_t make_hist_map(void *slot, const void *base, bool fp32, int T, int B, int H, uint32_t units)
+{
+    const cuuint64_t es = fp32 ? 4 : 2;
+    cuuint64_t dims[3] = {(cuuint64_t)H, (cuuint64_t)B, (cuuint64_t)T + 1};
+    cuuint64_t strides[2] = {(cuuint64_t)H * es, (cuuint64_t)H * es * B};
+    cuuint32_t box[3] = {units, (cuuint32_t)std::min(B, kRows), 1};
+    cuuint32_t el[3] = {1, 1, 1};
+    CUresult r = g_encode((CUtensorMap *)slot, fp32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16,
+                          3, const_cast<void *>(base), dims, strides, box, el, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                          stage_swizzle(units * (uint32_t)es), CU_TENSOR_MAP_L2_PROMOTION_NONE,
+                          CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
+}
+
+enum { kMapX128 = 0, kMapX64 = 1, kMapG128 = 2, kMapG64 = 3, kMapH128 = 4, kMapH64 = 5, kMapGates = 6, kMapHistH = 7,
+       kMapHistC = 8 };
 const CUtensorMap &map(const stacklstm *s, int i) { return *(const CUtensorMap *)s->tmaps[i]; }
 
 // budget that leaves room for two CTAs per SM when the grid needs more than one wave.
@@ -602,7 +628,12 @@ cudaError_t bf16_prepare(stacklstm *s)
     const uint64_t R1 = (uint64_t)(T + 1) * B;
     if ((e = make_map(s->tmaps[kMapH128], s->hr, R1, (uint64_t)H, kRows))) return e;
     if ((e = make_map(s->tmaps[kMapH64], s->hr, R1, (uint64_t)H, kChunk))) return e;
-    if (s->pf.on && (e = make_gates_map(s->tmaps[kMapGates], s->gates, T, B, H, s->pf.U / s->pf.EP))) return e;
+    if (s->pf.on) {
+        const uint32_t ue = (uint32_t)(s->pf.U / s->pf.EP);
+        if ((e = make_gates_map(s->tmaps[kMapGates], s->gates, T, B, H, ue))) return e;
+        if ((e = make_hist_map(s->tmaps[kMapHistH], s->hist_h, false, T, B, H, ue))) return e;
+        if ((e = make_hist_map(s->tmaps[kMapHistC], s->hist_c, true, T, B, H, ue))) return e;
+    }
     return cudaSuccess;
 }
 
@@ -639,7 +670,7 @@ cudaError_t bf16_forward_steps(stacklstm *s, const float *bias)
     if (s->pf.on)
         return bf16_launch_fwd_persist(s, step_args(s, bias, s->w_fwd, s->kcx, s->kcf, s->pf.S),
                                        map(s, B <= 64 ? kMapX64 : kMapX128), map(s, B <= 64 ? kMapH64 : kMapH128),
-                                       map(s, kMapGates));
+                                       map(s, kMapGates), map(s, kMapHistH), map(s, kMapHistC));
     const StepArgs a = step_args(s, bias, s->w_fwd, s->kcx, s->kcf, s->sf);
     const dim3 grid(nctf, ceil_div(B, kRows));
     const size_t smem = smem_bytes(s->sf, 4 * s->uf);

@@ -66,9 +66,11 @@ struct WsArgs {
 // 1024-byte boundary.
 constexpr uint32_t kBarBytes = (2 * kMaxStages + 6) * 8 + 16;
 
-// forward: the activated gates of one tile (4 gates x 128 rows x U units, fp16), staged
-// for the tensor store that writes them out
-__host__ __device__ constexpr uint32_t ws_stg_bytes(bool fwd, int U) { return fwd ? 4u * 128 * U * 2 : 0u; }
+// forward: what one tile writes to the history apart from the h operand of the next step,
+// staged for the tensor stores that write it out: the activated gates (4 gates x 128 rows
+// x U units, fp16), then h' (128 x U, bf16), then c' (128 x U, fp32); each block is laid
+// out [unit part][row][units of the part]
+__host__ __device__ constexpr uint32_t ws_stg_bytes(bool fwd, int U) { return fwd ? 128u * U * (8 + 2 + 4) : 0u; }
 
 __host__ __device__ constexpr uint32_t ws_stage_bytes(int G, int NB, int w_res)
 {
@@ -258,6 +260,29 @@ __device__ __forceinline__ void unpack_f16(const uint32_t *w, float *v)
 // the ring's tensor copies.)
 __device__ __forceinline__ void pf_l2(const void *p, uint32_t) { tc::prefetch_l2(p); }
 
+// Backward: store the gradient-history updates after the step's release, so that the
+// release (and the proxy fence before it) does not wait for them. Their values stay in
+// registers meanwhile: done with one epilogue warp group (6 warps, up to 255 registers a
+// thread), not with two (10 warps share the register file: 168 a thread, and the held
+// values spill; measured slower).
+#ifndef STACKLSTM_DEFER_DHIST
+#define STACKLSTM_DEFER_DHIST 1
+#endif
+template <int EP>
+__host__ __device__ constexpr bool defer_dhist() { return STACKLSTM_DEFER_DHIST != 0 && EP == 1; }
+
+// Byte offset of 16-byte piece q of row r in a staging tile of RB-byte rows, in the layout
+// the tensor map's swizzle mode (32, 64 or 128 bytes for rows of that size; none for
+// 16-byte rows) gives the tile: the offset's 16-byte-piece bits XOR its 128-byte-line bits,
+// over log2(RB / 16) bits. Lanes that write one row each then hit distinct banks.
+template <int RB>
+__device__ __forceinline__ uint32_t stg_swz(uint32_t r, uint32_t q)
+{
+    static_assert(RB == 16 || RB == 32 || RB == 64 || RB == 128, "staging rows of 16 to 128 bytes");
+    const uint32_t o = r * RB + q * 16;
+    return o ^ (((o >> 7) & (RB / 16 - 1)) << 4);
+}
+
 // ------------------------------------------------------------------ epilogue
 struct EpiCtx {
     WCtl c;
@@ -276,7 +301,8 @@ struct EpiCtx {
 // U / KS units it finishes: ct * U + kp * U / KS .. + U / KS.
 template <int U, int EP, int NG, bool kFwd, int KS>
 __device__ __forceinline__ void epilogue_loop(const StepArgs &a, const WsArgs &p, const EpiCtx &e,
-                                              const float *s_bias, const CUtensorMap *tm_gates)
+                                              const float *s_bias, const CUtensorMap *tm_gates,
+                                              const CUtensorMap *tm_hh, const CUtensorMap *tm_hc)
 {
     static_assert(KS == 1 || (!kFwd && EP == 1), "split contraction: backward, one epilogue warp group");
     constexpr int E = 4 * EP, UE = U / KS / EP;  // units this thread finishes
@@ -323,6 +349,11 @@ __device__ __forceinline__ void epilogue_loop(const StepArgs &a, const WsArgs &p
                 }
             }
         }
+        // backward: the gradient-history rows this thread updates, stored after the step's
+        // release (only this thread reads them again, at later steps)
+        constexpr bool kDeferDhist = !kFwd && defer_dhist<EP>();
+        float dfh[kDeferDhist ? UE : 1], dfc[kDeferDhist ? UE : 1];
+        int d_src = 0, d_s1 = 0;
         if constexpr (kFwd) {
             // operands this thread wrote itself at earlier steps (same rows and units):
             // c_read, and the older top the next step reads when step t does not push
@@ -331,6 +362,19 @@ __device__ __forceinline__ void epilogue_loop(const StepArgs &a, const WsArgs &p
             const bool is_new = s_next == t + 1;
             float cr[UE];
             uint32_t hc[UE / 2];
+            if (k >= e.n_mine) {
+                // c' leaves by tensor store: the stores of this row tile's previous step
+                // (n_mine tiles back, so every group but possibly the latest) have completed
+                // before its rows are read back
+                if (e.tid == 0) {
+                    if (e.n_mine == 1)
+                        tc::bulk_wait();
+                    else
+                        tc::bulk_wait_all_but_last();
+                }
+                __syncwarp();
+                tc::bar_sync(3, E * 32);
+            }
 #pragma unroll
             for (int cg = 0; cg < UE / NG; ++cg) {
                 const int u = u0 + cg * NG;
@@ -371,21 +415,30 @@ __device__ __forceinline__ void epilogue_loop(const StepArgs &a, const WsArgs &p
                 // history row t + 1, the h operand of step t + 1 (h' when step t pushed,
                 // else the older top), the activated gates (fp16) for the backward
                 const size_t w = ((size_t)(t + 1) * B + b) * H + u;
+                const uint32_t srow = (uint32_t)(e.q * 32 + e.lane);  // staging row
                 uint32_t hb[NG / 2];
                 pack_bf16<NG>(hn, hb);
-                st_h<NG>(a.hist_h + w, hb);
                 st_h<NG>(a.hr + w, is_new ? hb : hc + cg * NG / 2);
-                st_f<NG>(a.hist_c + w, cn);
+                // h' and c' into their staging tiles
+                const uint32_t htile = e.c.stg + 8u * U * kRows + (uint32_t)(e.part * kRows * UE * 2);
+                const uint32_t ctile = e.c.stg + 10u * U * kRows + (uint32_t)(e.part * kRows * UE * 4);
+#pragma unroll
+                for (int i = 0; i < NG / 8; ++i)
+                    tc::st_shared_v4(htile + stg_swz<UE * 2>(srow, cg * NG / 8 + i), hb + 4 * i);
+#pragma unroll
+                for (int i = 0; i < NG / 4; ++i)
+                    tc::st_shared_v4(ctile + stg_swz<UE * 4>(srow, cg * NG / 4 + i),
+                                     reinterpret_cast<const uint32_t *>(cn) + 4 * i);
                 // gates into the staging tile [gate][part][row][UE units]; a tensor store
                 // writes them out after the tile (nothing reads them before the backward)
 #pragma unroll
                 for (int g = 0; g < 4; ++g) {
                     uint32_t gw[NG / 2];
                     pack_f16<NG>(gv[g], gw);
-                    const uint32_t dst =
-                        e.c.stg + (((g * EP + e.part) * kRows + e.q * 32 + e.lane) * UE + cg * NG) * 2;
+                    const uint32_t tile = e.c.stg + (uint32_t)((g * EP + e.part) * kRows * UE * 2);
 #pragma unroll
-                    for (int i = 0; i < NG / 8; ++i) tc::st_shared_v4(dst + 16 * i, gw + 4 * i);
+                    for (int i = 0; i < NG / 8; ++i)
+                        tc::st_shared_v4(tile + stg_swz<UE * 2>(srow, cg * NG / 8 + i), gw + 4 * i);
                 }
             }
         } else {
@@ -480,7 +533,12 @@ __device__ __forceinline__ void epilogue_loop(const StepArgs &a, const WsArgs &p
                 float v[NG];
 #pragma unroll
                 for (int i = 0; i < NG; ++i) v[i] = dh_src[j * NG + i] + __uint_as_float(dr[i]);
-                st_f<NG>(a.dhist_h + ((size_t)src * B + b) * H + u, v);
+                if constexpr (kDeferDhist) {
+#pragma unroll
+                    for (int i = 0; i < NG; ++i) dfh[cg * NG + i] = v[i];
+                } else {
+                    st_f<NG>(a.dhist_h + ((size_t)src * B + b) * H + u, v);
+                }
                 if (t >= 1) {
                     float ig[NG], fg[NG], gg[NG], og[NG], d[4][NG], dcr[NG];
                     unpack_f16<NG>(gq[0] + j * NG / 2, ig);
@@ -506,9 +564,16 @@ __device__ __forceinline__ void epilogue_loop(const StepArgs &a, const WsArgs &p
                         pack_bf16<NG>(d[g], w);
                         st_h<NG>(dg + (size_t)g * H, w);
                     }
-                    st_f<NG>(a.dhist_c + ((size_t)s1 * B + b) * H + u, dcr);
+                    if constexpr (kDeferDhist) {
+#pragma unroll
+                        for (int i = 0; i < NG; ++i) dfc[cg * NG + i] = dcr[i];
+                    } else {
+                        st_f<NG>(a.dhist_c + ((size_t)s1 * B + b) * H + u, dcr);
+                    }
                 }
             }
+            d_src = src;
+            d_s1 = s1;
         }
         // the next step reads these rows by TMA: generic writes -> async proxy, then
         // release the step for this row tile
@@ -517,6 +582,17 @@ __device__ __forceinline__ void epilogue_loop(const StepArgs &a, const WsArgs &p
         __syncwarp();
         tc::bar_sync(2, E * 32);
         if (e.tid == 0) tc::red_release_gpu_add(p.cnt + rt * p.cs, 1);
+        if constexpr (kDeferDhist) {
+            if (row_ok) {
+#pragma unroll
+                for (int cg = 0; cg < UE / NG; ++cg) {
+                    const int u = u0 + cg * NG;
+                    if (u >= H) continue;
+                    st_f<NG>(a.dhist_h + ((size_t)d_src * B + b) * H + u, dfh + cg * NG);
+                    if (t >= 1) st_f<NG>(a.dhist_c + ((size_t)d_s1 * B + b) * H + u, dfc + cg * NG);
+                }
+            }
+        }
         if constexpr (kFwd) {
             if (e.tid == 0) {
 #pragma unroll
@@ -525,12 +601,19 @@ __device__ __forceinline__ void epilogue_loop(const StepArgs &a, const WsArgs &p
                     for (int q = 0; q < EP; ++q)
                         tc::tma_store_4d(tm_gates, e.c.stg + (uint32_t)((g * EP + q) * kRows * UE * 2),
                                          e.ct * U + q * UE, g, rt * kRows, t);
+#pragma unroll
+                for (int q = 0; q < EP; ++q) {
+                    tc::tma_store_3d(tm_hh, e.c.stg + 8u * U * kRows + (uint32_t)(q * kRows * UE * 2), e.ct * U + q * UE,
+                                     rt * kRows, t + 1);
+                    tc::tma_store_3d(tm_hc, e.c.stg + 10u * U * kRows + (uint32_t)(q * kRows * UE * 4),
+                                     e.ct * U + q * UE, rt * kRows, t + 1);
+                }
                 tc::bulk_commit();
             }
         }
     }
     if constexpr (kFwd)
-        if (e.tid == 0) tc::bulk_wait();  // the gate stores completed before the CTA exits
+        if (e.tid == 0) tc::bulk_wait();  // the history stores completed before the CTA exits
 }
 
 // ------------------------------------------------------------------ input gradient
@@ -724,7 +807,8 @@ __device__ __forceinline__ void dx_role(const CUtensorMap *tm_g, const WsArgs &p
 template <int U, int EP, int G, bool kFwd, int KS>
 __global__ void __launch_bounds__(32 * (4 * EP + 2), 1)
 step_ws(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtensorMap tm_b,
-        const __grid_constant__ CUtensorMap tm_gates, WsArgs p)
+        const __grid_constant__ CUtensorMap tm_gates, const __grid_constant__ CUtensorMap tm_hh,
+        const __grid_constant__ CUtensorMap tm_hc, WsArgs p)
 {
     constexpr int NB = kFwd ? 4 * U : U;  // accumulator columns
     constexpr int E = 4 * EP;             // epilogue warps
@@ -881,9 +965,9 @@ step_ws(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtens
         constexpr int NG = UE % 16 == 0 ? 16 : 8;
         const EpiCtx e{c, tmem, warp & 3, warp >> 2, lane, tid, ct, kp, slot, n_mine, n_tiles, limit};
         if (NG == 16 && p.vec32)
-            epilogue_loop<U, EP, NG, kFwd, KS>(a, p, e, s_bias, &tm_gates);
+            epilogue_loop<U, EP, NG, kFwd, KS>(a, p, e, s_bias, &tm_gates, &tm_hh, &tm_hc);
         else
-            epilogue_loop<U, EP, 8, kFwd, KS>(a, p, e, s_bias, &tm_gates);
+            epilogue_loop<U, EP, 8, kFwd, KS>(a, p, e, s_bias, &tm_gates, &tm_hh, &tm_hc);
     }
 
     // ---------------------------------------------------------------- teardown
@@ -1159,7 +1243,8 @@ bool bf16_plan_fwd_persist(stacklstm *s, PersistPlan *pl) { return plan(s, true,
 bool bf16_plan_bwd_persist(stacklstm *s, PersistPlan *pl) { return plan(s, false, pl); }
 
 cudaError_t bf16_launch_fwd_persist(stacklstm *s, const StepArgs &a, const CUtensorMap &tm_x, const CUtensorMap &tm_h,
-                                    const CUtensorMap &tm_gates)
+                                    const CUtensorMap &tm_gates, const CUtensorMap &tm_hh,
+                                    const CUtensorMap &tm_hc)
 {
     const PersistPlan &pl = s->pf;
     WsArgs p{};
@@ -1180,7 +1265,7 @@ cudaError_t bf16_launch_fwd_persist(stacklstm *s, const StepArgs &a, const CUten
     if (e) return e;
     const void *fn = find_fn(true, pl);
     if (!fn) return cudaErrorInvalidDeviceFunction;
-    e = launch_coop(fn, pl, pl.n_ct * pl.slot, s->stream, tm_x, tm_h, tm_gates, p);
+    e = launch_coop(fn, pl, pl.n_ct * pl.slot, s->stream, tm_x, tm_h, tm_gates, tm_hh, tm_hc, p);
     if (e) return e;
     s->launches += 1;
     return cudaGetLastError();
@@ -1217,7 +1302,7 @@ cudaError_t bf16_launch_bwd_persist(stacklstm *s, const StepArgs &a, const CUten
     if (pl.KS > 1 && (e = cudaMemsetAsync(p.pcnt, 0, sizeof(int32_t) * p.n_rt * p.n_ct, s->stream))) return e;
     const void *fn = find_fn(false, pl);
     if (!fn) return cudaErrorInvalidDeviceFunction;
-    e = launch_coop(fn, pl, p.n_chain + p.n_dx, s->stream, tm_g, tm_g, tm_g, p);
+    e = launch_coop(fn, pl, p.n_chain + p.n_dx, s->stream, tm_g, tm_g, tm_g, tm_g, tm_g, p);
     if (e) return e;
     s->launches += 1;
     *dx_done = p.n_dx > 0;

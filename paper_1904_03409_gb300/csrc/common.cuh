@@ -76,7 +76,7 @@ struct stacklstm {
     int uf = 0, ub = 0;      // hidden units per CTA tile: forward, backward
     int kcx = 0, kcf = 0, kcb = 0;  // 64-wide contraction chunks: x part, forward total, backward
     int sf = 0, sb = 0, sx = 0, sw = 0;  // ring depths: forward, backward, dx, dW
-    alignas(64) unsigned char tmaps[8][128] = {};  // TMA descriptors (bf16_path.cu)
+    alignas(64) unsigned char tmaps[10][128] = {};  // TMA descriptors (bf16_path.cu)
     // persistent step kernels (one launch for all T steps; bf16_persist.cu)
     PersistPlan pf, pb;            // forward, backward (on = 0: one launch per step)
     int32_t *rowcnt = nullptr;     // [2][row tiles][cnt_stride] completed steps per row tile
