@@ -1013,8 +1013,8 @@ const Variant *bwd_variants(int *n)
 {
     static const Variant v[] = {variant<16, 1, 4, false>(), variant<16, 2, 4, false>(), variant<32, 2, 4, false>(),
                                 variant<32, 4, 4, false>(), variant<64, 2, 2, false>(), variant<64, 1, 2, false, 4>(),
-                                variant<64, 1, 4, false, 4>(), variant<64, 2, 4, false>()};
-    *n = 8;
+                                variant<64, 1, 4, false, 4>(), variant<64, 2, 4, false>(), variant<32, 1, 4, false>()};
+    *n = 9;
     return v;
 }
 
@@ -1101,8 +1101,10 @@ bool plan_variant(const Variant &v, bool fwd, int KC, int split, int n_rt, int H
                 resident = clusters * cl;
             }
             if (resident < pad) continue;
-            const int sl = std::min(n_rt, resident / pad);
-            const int rounds = (n_rt + sl - 1) / sl;
+            // the fewest slots that give the same number of row-tile rounds per step: every
+            // slot then has (about) the same work, and the SMs left over take other work
+            const int rounds = (n_rt + std::min(n_rt, resident / pad) - 1) / std::min(n_rt, resident / pad);
+            const int sl = (n_rt + rounds - 1) / rounds;
             // forward, per CTA and step: MMA issue plus the epilogue's ~16 B of stores per
             // (instance, unit) at about 30 B/cycle
             double c = rounds * (KC * 4 * mma_cycles(NB) + groups * kWaitCycles + 128.0 * v.U * 16 / 30);
@@ -1116,7 +1118,10 @@ bool plan_variant(const Variant &v, bool fwd, int KC, int split, int n_rt, int H
                 const double mma = KCl * 4 * mma_cycles(NB) + groups * 400.0;
                 const double epi = 128.0 * (v.U / v.KS) * 48 / 30 +
                                    (v.KS > 1 ? 2.0 * 128 * v.U * 4 / 30 + 3000 : 0.0);
-                c = rounds * (std::max(ingest, mma) + epi);
+                // with two or more row tiles a CTA multiplies one while the epilogue
+                // finishes the other (their chains are independent)
+                const double mm = std::max(ingest, mma);
+                c = rounds > 1 ? rounds * std::max(mm, epi) + std::min(mm, epi) : mm + epi;
             }
             // ties: a plan within 208 KB of shared memory first (beyond it L1 is too small
             // for the epilogue's traffic: the stress forward ran 5% slower with its weight
@@ -1165,14 +1170,18 @@ bool plan(stacklstm *s, bool fwd, PersistPlan *pl)
     const bool mc_on = mc && atoi(mc) != 0;
     const char *force = getenv(fwd ? "STACKLSTM_FWD_UNITS" : "STACKLSTM_BWD_UNITS");
     const int force_u = force ? atoi(force) : 0;
-    // epilogue warp groups: one for 16-unit tiles (a thread then holds 16 units, whole
-    // 32-byte sectors), two for 32-unit tiles (measured best); STACKLSTM_*_EP overrides
+    // epilogue warp groups: forward, one for 16-unit tiles (a thread then holds 16 units,
+    // whole 32-byte sectors), two for 32-unit tiles; backward, one up to 32 units (its
+    // threads then have the registers to hold their gradient-history updates until after
+    // the step's release), two for 64 (all measured best); STACKLSTM_*_EP overrides
     const char *force_ep = getenv(fwd ? "STACKLSTM_FWD_EP" : "STACKLSTM_BWD_EP");
     double best = 1e30;
     bool found = false;
     for (int i = 0; i < n; ++i) {
         if (force_u && vs[i].U != force_u) continue;
-        const int want_ep = force_ep ? atoi(force_ep) : vs[i].U == 16 || vs[i].KS > 1 ? 1 : 2;
+        const int want_ep = force_ep               ? atoi(force_ep)
+                            : vs[i].U == 16 || vs[i].KS > 1 || (!fwd && vs[i].U <= 32) ? 1
+                                                                                          : 2;
         if (vs[i].U >= 16 && vs[i].EP != want_ep) continue;
         const char *force_ks = fwd ? nullptr : getenv("STACKLSTM_BWD_KS");
         if (force_ks && vs[i].KS != atoi(force_ks)) continue;
