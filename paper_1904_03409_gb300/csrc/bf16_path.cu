@@ -540,18 +540,20 @@ StepArgs step_args(stacklstm *s, const float *bias, const void *wpack, int kcx, 
 
 std::string bf16_describe(const stacklstm *s)
 {
-    char buf[768];
+    char buf[1024];
     const int rt = (int)ceil_div(s->B, kRows);
     const PersistPlan &f = s->pf, &b = s->pb;
     snprintf(buf, sizeof buf,
              "bf16 tcgen05; row tiles %d; chunks fwd %d (x %d) bwd %d; "
-             "forward %s U=%d [EP %d G %d ring %d slots %d cluster %d col tiles %d w_res %d smem %u threads %d]; "
+             "forward %s U=%d [EP %d G %d ring %d slots %d cluster %d col tiles %d w_res %d smem %u threads %d "
+             "per SM %d]; "
              "backward %s U=%d [EP %d G %d ring %d slots %d cluster %d col tiles %d w_res %d smem %u threads %d "
+             "per SM %d "
              "contraction parts %d dx CTAs %d ring %d]; "
              "step rings fwd %d bwd %d; dx N=%d x%d ring %d; dW %dx%d tiles of 128x%d x%d splits ring %d",
              rt, s->kcf, s->kcx, s->kcb, f.on ? "persistent" : "per-step", s->uf, f.EP, f.G, f.S, f.slot, f.cl, f.n_ct,
-             f.w_res, f.smem, f.threads, b.on ? "persistent" : "per-step", s->ub, b.EP, b.G, b.S, b.slot, b.cl, b.n_ct,
-             b.w_res, b.smem, b.threads, b.KS, b.n_dx, b.dx_S, s->sf, s->sb, s->nx, s->nxt, s->sx, s->dw_mt, s->dw_nt, s->dw_ntile, s->dw_split, s->sw);
+             f.w_res, f.smem, f.threads, f.per_sm, b.on ? "persistent" : "per-step", s->ub, b.EP, b.G, b.S, b.slot, b.cl, b.n_ct,
+             b.w_res, b.smem, b.threads, b.per_sm, b.KS, b.n_dx, b.dx_S, s->sf, s->sb, s->nx, s->nxt, s->sx, s->dw_mt, s->dw_nt, s->dw_ntile, s->dw_split, s->sw);
     return buf;
 }
 

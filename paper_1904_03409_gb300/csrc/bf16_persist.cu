@@ -311,6 +311,25 @@ __device__ __forceinline__ void epilogue_loop(const StepArgs &a, const WsArgs &p
     const int T = a.T, B = a.B, H = a.H;
     const uint32_t lane_off = (uint32_t)(e.q * 32) << 16;
     const int u0 = e.ct * U + e.kp * (U / KS) + e.part * UE;  // first unit of this thread
+    // The row indices of a tile for this thread: the state it reads (src) and, forward, the
+    // top after the step (s_next) / backward, the state step t - 1 read (s1). They are
+    // loaded a tile ahead, so that no load waits on another at the start of a tile.
+    auto tile_rows = [&](int kk, int &i0, int &i1) {
+        const int ksk = kk / e.n_mine, rtk = e.slot + (kk % e.n_mine) * p.n_slot;
+        const int tk = kFwd ? ksk : T - 1 - ksk;
+        const int bk = rtk * kRows + e.q * 32 + e.lane;
+        i0 = 0;
+        i1 = 0;
+        if (bk < B) {
+            i0 = a.top[(size_t)tk * B + bk];
+            if (kFwd)
+                i1 = a.top[(size_t)(tk + 1) * B + bk];
+            else if (tk >= 1)
+                i1 = a.top[(size_t)(tk - 1) * B + bk];
+        }
+    };
+    int cur0 = 0, cur1 = 0;
+    if (e.n_tiles > 0) tile_rows(0, cur0, cur1);
     for (int k = 0; k < e.n_tiles; ++k) {
         const int ks = k / e.n_mine, rt = e.slot + (k % e.n_mine) * p.n_slot;
         const int t = kFwd ? ks : T - 1 - ks;
@@ -318,37 +337,38 @@ __device__ __forceinline__ void epilogue_loop(const StepArgs &a, const WsArgs &p
         const bool row_ok = b < B;
         const int acc = k & 1;
         const uint32_t taddr = e.tmem + acc * kCols + lane_off;
-        if (k + 1 < e.n_tiles) {
-            // the next tile's epilogue operands into L2 now (their loads then wait on L2,
-            // not HBM); a row the current tile is about to write is harmless to prefetch
+        int nx0 = 0, nx1 = 0;
+        if (k + 1 < e.n_tiles) tile_rows(k + 1, nx0, nx1);
+        // the next tile's epilogue operands into L2 (their loads then wait on L2, not HBM);
+        // called once this tile's own loads are issued. A row the current tile is about to
+        // write is harmless to prefetch.
+        auto prefetch_next = [&]() {
+            if (k + 1 >= e.n_tiles) return;
             const int ks1 = (k + 1) / e.n_mine, rt1 = e.slot + ((k + 1) % e.n_mine) * p.n_slot;
             const int t1 = kFwd ? ks1 : T - 1 - ks1;
             const int b1 = rt1 * kRows + e.q * 32 + e.lane;
-            if (b1 < B && u0 < H) {
-                // this thread's whole row pieces (H and u0 are multiples of 8: 16-byte
-                // aligned, whole 16-byte multiples)
-                const uint32_t n4 = 4u * (uint32_t)min(UE, H - u0), n2 = n4 / 2;
-                const int src1 = a.top[(size_t)t1 * B + b1];
-                if constexpr (kFwd) {
-                    pf_l2(a.hist_c + ((size_t)src1 * B + b1) * H + u0, n4);
-                    pf_l2(a.hr + ((size_t)a.top[(size_t)(t1 + 1) * B + b1] * B + b1) * H + u0, n2);
-                } else {
-                    pf_l2(a.dhist_h + ((size_t)src1 * B + b1) * H + u0, n4);
-                    if (t1 >= 1) {
-                        const int s11 = a.top[(size_t)(t1 - 1) * B + b1];
-                        const size_t wr = ((size_t)t1 * B + b1) * H + u0, rd = ((size_t)s11 * B + b1) * H + u0;
-                        pf_l2(a.dhist_h + wr, n4);
-                        pf_l2(a.dhist_c + wr, n4);
-                        pf_l2(a.hist_c + wr, n4);
-                        pf_l2(a.hist_c + rd, n4);
-                        pf_l2(a.dhist_c + rd, n4);
-                        const __half *gt = a.gates + ((size_t)(t1 - 1) * B + b1) * 4 * H + u0;
+            if (b1 >= B || u0 >= H) return;
+            // this thread's whole row pieces (H and u0 are multiples of 8: 16-byte aligned,
+            // whole 16-byte multiples)
+            const uint32_t n4 = 4u * (uint32_t)min(UE, H - u0), n2 = n4 / 2;
+            if constexpr (kFwd) {
+                pf_l2(a.hist_c + ((size_t)nx0 * B + b1) * H + u0, n4);
+                pf_l2(a.hr + ((size_t)nx1 * B + b1) * H + u0, n2);
+            } else {
+                pf_l2(a.dhist_h + ((size_t)nx0 * B + b1) * H + u0, n4);
+                if (t1 >= 1) {
+                    const size_t wr = ((size_t)t1 * B + b1) * H + u0, rd = ((size_t)nx1 * B + b1) * H + u0;
+                    pf_l2(a.dhist_h + wr, n4);
+                    pf_l2(a.dhist_c + wr, n4);
+                    pf_l2(a.hist_c + wr, n4);
+                    pf_l2(a.hist_c + rd, n4);
+                    pf_l2(a.dhist_c + rd, n4);
+                    const __half *gt = a.gates + ((size_t)(t1 - 1) * B + b1) * 4 * H + u0;
 #pragma unroll
-                        for (int g = 0; g < 4; ++g) pf_l2(gt + (size_t)g * H, n2);
-                    }
+                    for (int g = 0; g < 4; ++g) pf_l2(gt + (size_t)g * H, n2);
                 }
             }
-        }
+        };
         // backward: the gradient-history rows this thread updates, stored after the step's
         // release (only this thread reads them again, at later steps)
         constexpr bool kDeferDhist = !kFwd && defer_dhist<EP>();
@@ -357,8 +377,7 @@ __device__ __forceinline__ void epilogue_loop(const StepArgs &a, const WsArgs &p
         if constexpr (kFwd) {
             // operands this thread wrote itself at earlier steps (same rows and units):
             // c_read, and the older top the next step reads when step t does not push
-            const int src = row_ok ? a.top[(size_t)t * B + b] : 0;
-            const int s_next = row_ok ? a.top[(size_t)(t + 1) * B + b] : 0;
+            const int src = cur0, s_next = cur1;
             const bool is_new = s_next == t + 1;
             float cr[UE];
             uint32_t hc[UE / 2];
@@ -383,6 +402,7 @@ __device__ __forceinline__ void epilogue_loop(const StepArgs &a, const WsArgs &p
                     if (!is_new) ld_h<NG>(a.hr + ((size_t)s_next * B + b) * H + u, hc + cg * NG / 2);
                 }
             }
+            prefetch_next();
             if (e.tid == 0) tc::bulk_wait_read();  // the previous tile's gate stores read the staging tile
             const bool ok = tc::mbar_wait(&e.c.tfull[acc], (k >> 1) & 1, e.limit, e.c.abort);
             if (!ok) ws_abort(e.c, a.err);
@@ -450,8 +470,7 @@ __device__ __forceinline__ void epilogue_loop(const StepArgs &a, const WsArgs &p
             constexpr int NGRP = UE / NG;
             constexpr bool kEarly = UE <= 16;
             constexpr int NO = kEarly ? UE : NG;  // units whose operands are held at once
-            const int src = row_ok ? a.top[(size_t)t * B + b] : 0;
-            const int s1 = (row_ok && t >= 1) ? a.top[(size_t)(t - 1) * B + b] : 0;
+            const int src = cur0, s1 = cur1;
             float dh_src[NO], dh_t[NO], dc_t[NO], cn[NO], cr[NO], dc_rd[NO];
             uint32_t gq[4][NO / 2];
             // operands of units u .. u + NG - 1 into slot j (units j * NG ..) of the arrays
@@ -469,10 +488,13 @@ __device__ __forceinline__ void epilogue_loop(const StepArgs &a, const WsArgs &p
                     for (int g = 0; g < 4; ++g) ld_h<NG>(gt + (size_t)g * H, gq[g] + j * NG / 2);
                 }
             };
-            if (kEarly)
+            if (kEarly) {
+                // (measured: prefetching before this tile's loads suits the one-group tiles)
+                prefetch_next();
 #pragma unroll
                 for (int cg = 0; cg < NGRP; ++cg)
                     if (row_ok && u0 + cg * NG < H) load_ops(u0 + cg * NG, cg);
+            }
             const bool ok = tc::mbar_wait(&e.c.tfull[acc], (k >> 1) & 1, e.limit, e.c.abort);
             if (!ok) ws_abort(e.c, a.err);
             __syncwarp();
@@ -528,8 +550,10 @@ __device__ __forceinline__ void epilogue_loop(const StepArgs &a, const WsArgs &p
                         if (e.lane == 0) tc::mbar_arrive(&e.c.tempty[acc]);
                     }
                 }
-                if (!(row_ok && u < H)) continue;
-                if (!kEarly) load_ops(u, 0);
+                const bool mine = row_ok && u < H;
+                if (!kEarly && mine) load_ops(u, 0);
+                if (!kEarly && cg == 0) prefetch_next();
+                if (!mine) continue;
                 float v[NG];
 #pragma unroll
                 for (int i = 0; i < NG; ++i) v[i] = dh_src[j * NG + i] + __uint_as_float(dr[i]);
@@ -611,6 +635,8 @@ __device__ __forceinline__ void epilogue_loop(const StepArgs &a, const WsArgs &p
                 tc::bulk_commit();
             }
         }
+        cur0 = nx0;
+        cur1 = nx1;
     }
     if constexpr (kFwd)
         if (e.tid == 0) tc::bulk_wait();  // the history stores completed before the CTA exits
@@ -1005,8 +1031,8 @@ Variant variant()
 const Variant *fwd_variants(int *n)
 {
     static const Variant v[] = {variant<8, 1, 4, true>(),  variant<16, 1, 4, true>(), variant<16, 2, 4, true>(),
-                                variant<32, 2, 2, true>(), variant<32, 4, 2, true>()};
-    *n = 5;
+                                variant<32, 2, 2, true>(), variant<32, 4, 2, true>(), variant<16, 1, 1, true>()};
+    *n = 6;
     return v;
 }
 const Variant *bwd_variants(int *n)
@@ -1143,6 +1169,7 @@ bool plan_variant(const Variant &v, bool fwd, int KC, int split, int n_rt, int H
                 pl->n_ct = pad / v.KS;
                 pl->smem = smem;
                 pl->threads = threads;
+                pl->per_sm = resident / sms;
                 found = true;
             }
         }

@@ -25,6 +25,7 @@ struct PersistPlan {
     int n_ct = 0;       // column tiles, padded to a multiple of cl
     unsigned smem = 0;  // dynamic shared memory per CTA
     int threads = 0;    // threads per CTA
+    int per_sm = 1;     // co-resident CTAs per SM at this footprint
     int n_dx = 0;       // backward: extra CTAs computing dx on the SMs the steps leave idle
     int dx_S = 0;       // their ring stages
 };
