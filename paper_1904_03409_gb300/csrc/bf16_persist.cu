@@ -409,25 +409,41 @@ __device__ __forceinline__ void epilogue_loop(const StepArgs &a, const WsArgs &p
             __syncwarp();
             if (tc::bar_any(1, E * 32, !ok || *e.c.abort)) break;
             tc::tc_fence_after();
-            uint32_t zr[4][UE];
+            // the four gates' pre-activations: all UE units at once, or (more than 16
+            // units a thread) group by group, which bounds the registers they take
+            constexpr bool kByGroup = UE > 16;
+            constexpr int ZW = kByGroup ? NG : UE;
+            uint32_t zr[4][ZW];
+            if constexpr (!kByGroup) {
 #pragma unroll
-            for (int g = 0; g < 4; ++g) tmem_cols<UE>(taddr + g * U + e.part * UE, zr[g]);
-            tc::tmem_wait_ld();
-            tc::tc_fence_before();
-            __syncwarp();
-            if (e.lane == 0) tc::mbar_arrive(&e.c.tempty[acc]);
+                for (int g = 0; g < 4; ++g) tmem_cols<UE>(taddr + g * U + e.part * UE, zr[g]);
+                tc::tmem_wait_ld();
+                tc::tc_fence_before();
+                __syncwarp();
+                if (e.lane == 0) tc::mbar_arrive(&e.c.tempty[acc]);
+            }
 #pragma unroll
             for (int cg = 0; cg < UE / NG; ++cg) {
                 const int u = u0 + cg * NG;
+                if constexpr (kByGroup) {
+#pragma unroll
+                    for (int g = 0; g < 4; ++g) tmem_cols<NG>(taddr + g * U + e.part * UE + cg * NG, zr[g]);
+                    tc::tmem_wait_ld();
+                    if (cg == UE / NG - 1) {
+                        tc::tc_fence_before();
+                        __syncwarp();
+                        if (e.lane == 0) tc::mbar_arrive(&e.c.tempty[acc]);
+                    }
+                }
                 if (!(row_ok && u < H)) continue;
                 float cn[NG], hn[NG], gv[4][NG];
 #pragma unroll
                 for (int i = 0; i < NG; ++i) {
-                    const int j = cg * NG + i, jb = e.part * UE + j;
-                    const float ig = sigm(__uint_as_float(zr[0][j]) + s_bias[jb]);
-                    const float fg = sigm(__uint_as_float(zr[1][j]) + s_bias[U + jb]);
-                    const float gg = tanh_hw(__uint_as_float(zr[2][j]) + s_bias[2 * U + jb]);
-                    const float og = sigm(__uint_as_float(zr[3][j]) + s_bias[3 * U + jb]);
+                    const int j = cg * NG + i, jb = e.part * UE + j, jz = kByGroup ? i : j;
+                    const float ig = sigm(__uint_as_float(zr[0][jz]) + s_bias[jb]);
+                    const float fg = sigm(__uint_as_float(zr[1][jz]) + s_bias[U + jb]);
+                    const float gg = tanh_hw(__uint_as_float(zr[2][jz]) + s_bias[2 * U + jb]);
+                    const float og = sigm(__uint_as_float(zr[3][jz]) + s_bias[3 * U + jb]);
                     cn[i] = fmaf(fg, cr[j], ig * gg);
                     hn[i] = og * tanh_hw(cn[i]);
                     gv[0][i] = ig; gv[1][i] = fg; gv[2][i] = gg; gv[3][i] = og;
@@ -1031,8 +1047,8 @@ Variant variant()
 const Variant *fwd_variants(int *n)
 {
     static const Variant v[] = {variant<8, 1, 4, true>(),  variant<16, 1, 4, true>(), variant<16, 2, 4, true>(),
-                                variant<32, 2, 2, true>(), variant<32, 4, 2, true>(), variant<16, 1, 1, true>()};
-    *n = 6;
+                                variant<32, 2, 2, true>(), variant<32, 4, 2, true>()};
+    *n = 5;
     return v;
 }
 const Variant *bwd_variants(int *n)
