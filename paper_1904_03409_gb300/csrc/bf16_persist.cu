@@ -330,6 +330,7 @@ __device__ __forceinline__ void epilogue_loop(const StepArgs &a, const WsArgs &p
     };
     int cur0 = 0, cur1 = 0;
     if (e.n_tiles > 0) tile_rows(0, cur0, cur1);
+    constexpr bool kLatePfBwd = UE > 16;  // backward: operands taken group by group (below)
     for (int k = 0; k < e.n_tiles; ++k) {
         const int ks = k / e.n_mine, rt = e.slot + (k % e.n_mine) * p.n_slot;
         const int t = kFwd ? ks : T - 1 - ks;
@@ -339,9 +340,13 @@ __device__ __forceinline__ void epilogue_loop(const StepArgs &a, const WsArgs &p
         const uint32_t taddr = e.tmem + acc * kCols + lane_off;
         int nx0 = 0, nx1 = 0;
         if (k + 1 < e.n_tiles) tile_rows(k + 1, nx0, nx1);
-        // the next tile's epilogue operands into L2 (their loads then wait on L2, not HBM);
-        // called once this tile's own loads are issued. A row the current tile is about to
-        // write is harmless to prefetch.
+        const bool pf_early = e.n_mine == 1;  // forward; the backward decides by its tile shape
+        // the next tile's epilogue operands into L2 (their loads then wait on L2, not HBM).
+        // Forward with one row tile per CTA, and backward with one access group a thread:
+        // prefetched as soon as this tile's own loads are issued (waiting for the indices);
+        // else once this tile's work is done (the indices have arrived; the forward's next
+        // tile is another row tile's). Measured per shape. A row the current tile is about
+        // to write is harmless to prefetch.
         auto prefetch_next = [&]() {
             if (k + 1 >= e.n_tiles) return;
             const int ks1 = (k + 1) / e.n_mine, rt1 = e.slot + ((k + 1) % e.n_mine) * p.n_slot;
@@ -402,7 +407,7 @@ __device__ __forceinline__ void epilogue_loop(const StepArgs &a, const WsArgs &p
                     if (!is_new) ld_h<NG>(a.hr + ((size_t)s_next * B + b) * H + u, hc + cg * NG / 2);
                 }
             }
-            prefetch_next();
+            if (pf_early) prefetch_next();
             if (e.tid == 0) tc::bulk_wait_read();  // the previous tile's gate stores read the staging tile
             const bool ok = tc::mbar_wait(&e.c.tfull[acc], (k >> 1) & 1, e.limit, e.c.abort);
             if (!ok) ws_abort(e.c, a.err);
@@ -505,7 +510,6 @@ __device__ __forceinline__ void epilogue_loop(const StepArgs &a, const WsArgs &p
                 }
             };
             if (kEarly) {
-                // (measured: prefetching before this tile's loads suits the one-group tiles)
                 prefetch_next();
 #pragma unroll
                 for (int cg = 0; cg < NGRP; ++cg)
@@ -568,7 +572,6 @@ __device__ __forceinline__ void epilogue_loop(const StepArgs &a, const WsArgs &p
                 }
                 const bool mine = row_ok && u < H;
                 if (!kEarly && mine) load_ops(u, 0);
-                if (!kEarly && cg == 0) prefetch_next();
                 if (!mine) continue;
                 float v[NG];
 #pragma unroll
@@ -615,6 +618,7 @@ __device__ __forceinline__ void epilogue_loop(const StepArgs &a, const WsArgs &p
             d_src = src;
             d_s1 = s1;
         }
+        if (kFwd ? !pf_early : kLatePfBwd) prefetch_next();
         // the next step reads these rows by TMA: generic writes -> async proxy, then
         // release the step for this row tile
         tc::fence_proxy_async_global();
