@@ -95,7 +95,9 @@ def roofline_of(work_flops, work_bytes, seconds, peaks, src, sustained):
 def phase_kernel(plan, phase):
     """(kernel name, source file) of the kernel that does a phase's work, from the plan."""
     if phase in ("forward", "backward"):
-        m = re.search(phase + r" (persistent|per-step) U=(\d+)", plan)
+        m = re.search(phase + r" (persistent|per-step|cluster) U=(\d+)", plan)
+        if m and m.group(1) == "cluster":
+            return "step_cl<U=%s,%s>" % (m.group(2), phase), "bf16_cluster.cu"
         if m and m.group(1) == "persistent":
             return "step_ws<U=%s,%s>" % (m.group(2), phase), "bf16_persist.cu"
         return ("fwd_step_tc" if phase == "forward" else "bwd_step_tc"), "bf16_path.cu"
@@ -291,7 +293,7 @@ def measure_workload(w, steps, warmup, local, world, sample_clocks, e2e):
     # a persistent step kernel is one launch over all T steps; the per-step kernels are T
     # launches of B instance-steps each; dx and dW are one contraction over all T * B rows
     # (dW: plus its fixed-order reduction of the split partials)
-    per_step_kernels = dom in ("forward", "backward") and "persistent" not in kname and "step_ws" not in kname
+    per_step_kernels = dom in ("forward", "backward") and "step_ws" not in kname and "step_cl" not in kname
     per_launch_units = w.B if per_step_kernels else w.B * w.T
     launches_per_step = w.T if per_step_kernels else 1
     launch_s = phase_ms[dom] / 1e3 / launches_per_step

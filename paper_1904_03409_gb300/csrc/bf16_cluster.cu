@@ -1,0 +1,464 @@
+// bf16_cluster.cu -- the forward recurrence (Algorithm 1) for one row tile of at most 64
+// instances as a single thread-block cluster. The n_ct column-tile CTAs (16 hidden units
+// each, n_ct <= 16) hand each step's h operand to one another through distributed shared
+// memory: the epilogue of step t stages its 16 units of h_read(t + 1) (h' where step t
+// pushed, else the older top) as one 2 KB slice, and one thread copies the slice into every
+// CTA's operand buffer for step t + 1 with bulk copies that complete on that CTA's
+// mbarrier by byte count. Nothing on the step's critical path goes through global memory
+// or a step counter; the history rows, the h operand rows (for the weight gradient) and
+// the gates are still written to global memory for the backward.
+//
+// Warp roles (192 threads): warps 0..3 epilogue (TMEM lane quadrant w, one instance row
+// per thread; rows >= B idle), warp 4 producer (weight tile once; x_t chunks by TMA into a
+// two-step buffer), warp 5 MMA (x part of step t as soon as x_t lands, then the h part once
+// every slice of h_read(t) has landed; two TMEM accumulators by step parity).
+//
+// x_t chunks are 64-row, 128-byte-swizzled 8 KB tiles; an h slice is 16 units x 64 rows in
+// the unswizzled K-major core-matrix layout ([row / 8][unit / 8][row mod 8][unit mod 8],
+// 2 KB), one K = 16 MMA step. The M = 128 MMAs read 128 rows, so rows 64..127 come from
+// whatever follows (the next tile or slice, or a pad after the last one) and only feed
+// accumulator rows that are never stored.
+#include <stdio.h>
+
+#include <algorithm>
+
+#include "bf16_dev.cuh"
+
+namespace sl {
+namespace {
+
+using tc::smem_u32;
+
+constexpr uint32_t kC64 = 64 * 128;  // one 64-row chunk
+
+struct ClArgs {
+    StepArgs s;  // s.kcx: x chunks; s.KC: all chunks
+    int n_ct;    // column tiles = CTAs of the cluster
+};
+
+// [weight tile KC x NB x 128][h buffers 2 x n_ct x 2 KB][2 KB pad][x buffers 2 x kcx x 8 KB]
+// [8 KB pad][staging 2 x 2 KB][barriers], based at the first 1024-byte boundary
+constexpr uint32_t kSlice = 2048;
+constexpr uint32_t kClBars = 16 * 8 + 16;
+__host__ __device__ constexpr uint32_t cl_smem_bytes(int KC, int kcx, int NB, int n_ct)
+{
+    return 1024 + (uint32_t)KC * NB * 128 + (2u * n_ct + 1) * kSlice + 2u * kcx * kC64 + kC64 + 2 * kSlice + kClBars;
+}
+
+struct ClCtl {
+    uint32_t w0, h0, x0, stg;  // weight tile, h buffers, x buffers, h slice staging
+    uint64_t *wbar, *xfull, *xempty, *hready, *tfull, *tempty, *done;
+    uint32_t *tmem_slot;
+    volatile int *abort;
+};
+
+__device__ __forceinline__ ClCtl cl_carve(uint8_t *raw, int KC, int kcx, int NB, int n_ct)
+{
+    const uint32_t off = smem_u32(raw);
+    uint8_t *base = raw + ((1024u - (off & 1023u)) & 1023u);
+    ClCtl c;
+    const uint32_t wb = (uint32_t)KC * NB * 128, hb = (2u * n_ct + 1) * kSlice, xb = 2u * kcx * kC64 + kC64;
+    c.w0 = smem_u32(base);
+    c.h0 = c.w0 + wb;
+    c.x0 = c.h0 + hb;
+    c.stg = c.x0 + xb;
+    uint64_t *bars = (uint64_t *)(base + wb + hb + xb + 2 * kSlice);
+    c.wbar = bars;
+    c.xfull = bars + 2;
+    c.xempty = bars + 4;
+    c.hready = bars + 6;
+    c.tfull = bars + 8;
+    c.tempty = bars + 10;
+    c.done = bars + 12;
+    c.tmem_slot = (uint32_t *)(bars + 13);
+    c.abort = (volatile int *)(c.tmem_slot + 1);
+    return c;
+}
+
+__device__ __forceinline__ void cl_abort(const ClCtl &c, int32_t *err)
+{
+    *c.abort = 1;
+    atomicCAS(err, 0, (int)SL_ERR_TIMEOUT);
+}
+
+// The address of a shared-memory location of this CTA in the window of cluster CTA `rank`.
+__device__ __forceinline__ uint32_t peer_addr(uint32_t local, uint32_t rank)
+{
+    uint32_t r;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(local), "r"(rank));
+    return r;
+}
+// Bulk copy of `bytes` from this CTA's shared memory into another CTA's (cluster address),
+// completing on the destination CTA's mbarrier (cluster address) by byte count.
+__device__ __forceinline__ void bulk_s2c(uint32_t dst, uint32_t src, uint32_t bytes, uint32_t bar)
+{
+    asm volatile("cp.async.bulk.shared::cluster.shared::cta.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                     dst),
+                 "r"(src), "r"(bytes), "r"(bar)
+                 : "memory");
+}
+// Bounded wait (as tc::mbar_wait) with cluster-scope acquire: the phase was completed by
+// release arrivals of other CTAs of the cluster, after their distributed-shared-memory stores.
+__device__ __forceinline__ bool mbar_wait_cluster(uint64_t *bar, uint32_t parity, long long limit, volatile int *abort)
+{
+    const long long t0 = clock64();
+    while (true) {
+        uint32_t ok;
+        asm volatile(
+            "{\n\t.reg .pred p;\n\t"
+            "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
+            "selp.u32 %0, 1, 0, p;\n\t}"
+            : "=r"(ok)
+            : "r"(smem_u32(bar)), "r"(parity)
+            : "memory");
+        if (ok) return true;
+        if (clock64() - t0 >= limit) return false;
+        if (abort && *abort) return false;
+    }
+}
+// One chunk's four K = 16 MMAs: A (64-row chunk) and the weight chunk (NB rows), K-major,
+// 128-byte swizzled.
+template <int NB>
+__device__ __forceinline__ void cl_mma_chunk(uint32_t d, uint32_t a, uint32_t b, bool first)
+{
+    constexpr uint32_t idesc = tc::idesc_bf16(NB);
+#pragma unroll
+    for (int k = 0; k < kChunk / 16; ++k)
+        tc::mma_bf16(d, tc::smem_desc(a + k * 32, 16, 1024), tc::smem_desc(b + k * 32, 16, 1024), idesc,
+                     !(first && k == 0));
+}
+
+// Unswizzled K-major descriptor of an h slice: core matrices (8 rows x 16 bytes) 128 bytes
+// apart along K, 256 bytes apart along M.
+__device__ __forceinline__ uint64_t slice_desc(uint32_t addr)
+{
+    return (uint64_t)((addr & 0x3FFFFu) >> 4) | ((uint64_t)(128 >> 4) << 16) | ((uint64_t)(256 >> 4) << 32) |
+           ((uint64_t)1 << 46);
+}
+// byte offset of 16-byte piece k (units 8k .. 8k + 7) of row r in an h slice
+__host__ __device__ constexpr uint32_t slice_off(uint32_t r, uint32_t k) { return (r >> 3) * 256 + k * 128 + (r & 7) * 16; }
+
+// Stages this thread's row of h_read(t + 1) (16 units, zero past H or B) as slice buffer
+// `buf`, then (once every epilogue warp has) one thread copies the slice into every CTA's
+// h buffer `buf` at this CTA's slice position, completing on that CTA's hready[buf].
+__device__ __forceinline__ void deliver_slice(const ClCtl &c, int buf, int row, const uint4 (&v)[2], bool valid0,
+                                              bool valid1, uint32_t ct, uint32_t n_ct, int tid)
+{
+    if (row < 64) {
+        const uint4 z = make_uint4(0u, 0u, 0u, 0u);
+        const uint4 a0 = valid0 ? v[0] : z, a1 = valid1 ? v[1] : z;
+        tc::st_shared_v4(c.stg + buf * kSlice + slice_off((uint32_t)row, 0), (const uint32_t *)&a0);
+        tc::st_shared_v4(c.stg + buf * kSlice + slice_off((uint32_t)row, 1), (const uint32_t *)&a1);
+    }
+    tc::fence_proxy_async();  // generic writes -> the bulk copies
+    __syncwarp();
+    tc::bar_sync(2, 4 * 32);
+    if (tid == 0) {
+        const uint32_t dst = c.h0 + (uint32_t)(buf * n_ct + ct) * kSlice, bar = smem_u32(&c.hready[buf]);
+        for (uint32_t r = 0; r < n_ct; ++r) bulk_s2c(peer_addr(dst, r), c.stg + buf * kSlice, kSlice, peer_addr(bar, r));
+    }
+}
+
+template <int U>
+__global__ void __launch_bounds__(192, 1) step_cl(const __grid_constant__ CUtensorMap tm_x, ClArgs p)
+{
+    static_assert(U == 16, "one h slice (two 8-unit core matrices) per CTA");
+    constexpr int NB = 4 * U;
+    constexpr uint32_t kCols = TmemCols<NB>::value;
+    constexpr int E = 4;  // epilogue warps
+    const StepArgs &a = p.s;
+    extern __shared__ uint8_t smem_raw[];
+    __shared__ float s_bias[4 * U];
+    const int T = a.T, B = a.B, H = a.H, KC = a.KC, kcx = a.kcx;
+    const uint32_t ct = tc::cluster_rank(), n_ct = (uint32_t)p.n_ct;
+    const ClCtl c = cl_carve(smem_raw, KC, kcx, NB, (int)n_ct);
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const long long limit = a.limit;
+    for (int i = tid; i < 4 * U; i += blockDim.x) {
+        const int g = i / U, u = (int)ct * U + i % U;
+        s_bias[i] = u < H ? a.bias[g * H + u] : 0.0f;
+    }
+    if (tid == 0) {
+        tc::mbar_init(c.wbar, 1);
+        for (int i = 0; i < 2; ++i) {
+            tc::mbar_init(&c.xfull[i], 1);
+            tc::mbar_init(&c.xempty[i], 1);
+            tc::mbar_init(&c.hready[i], 1);
+            tc::mbar_init(&c.tfull[i], 1);
+            tc::mbar_init(&c.tempty[i], E);
+        }
+        tc::mbar_init(c.done, 1);
+        *c.abort = 0;
+        tc::fence_mbar_init();
+        // the slices of h_read(0) and h_read(1): every CTA's, by byte count
+        for (int t = 0; t < 2 && t < T; ++t) tc::mbar_arrive_expect_tx(&c.hready[t], n_ct * kSlice);
+    }
+    if (warp == E) tc::tmem_alloc(c.tmem_slot, 2 * kCols);
+    tc::tc_fence_before();
+    __syncthreads();
+    tc::cluster_sync();  // every CTA's barriers exist before any copy completes on them
+    tc::tc_fence_after();
+    const uint32_t tmem = *c.tmem_slot;
+
+    if (warp == E) {
+        // ------------------------------------------------------------ producer
+        if (lane == 0) {
+            const uint32_t wbytes = (uint32_t)KC * NB * 128;
+            tc::mbar_arrive_expect_tx(c.wbar, wbytes);
+            tc::bulk_g2s(c.w0, a.wpack + (size_t)ct * wbytes, wbytes, c.wbar);
+            int last = -1;  // last step whose x chunks were issued
+            for (int t = 0; t < T && !*c.abort; ++t) {
+                const int b = t & 1;
+                if (t >= 2 && !tc::mbar_wait(&c.xempty[b], ((t >> 1) - 1) & 1, limit, c.abort)) {
+                    cl_abort(c, a.err);
+                    break;
+                }
+                tc::mbar_arrive_expect_tx(&c.xfull[b], (uint32_t)kcx * kC64);
+                for (int j = 0; j < kcx; ++j)
+                    tc::tma_load_2d(c.x0 + (b * kcx + j) * kC64, &tm_x, j * kChunk, t * B, &c.xfull[b]);
+                last = t;
+            }
+            // copies still in flight after an abort land before the CTA exits (each buffer's
+            // latest phase; phases the MMA warp consumed have completed already)
+            for (int t = max(0, last - 1); t <= last; ++t)
+                tc::mbar_wait(&c.xfull[t & 1], (t >> 1) & 1, kDrainLimit, nullptr);
+        }
+        __syncwarp();
+    } else if (warp == E + 1) {
+        // ------------------------------------------------------------ MMA issue
+        if (lane == 0) {
+            constexpr uint32_t idesc = tc::idesc_bf16(NB);
+            bool ok = tc::mbar_wait(c.wbar, 0, limit, c.abort);
+            int t_h = -1;  // last step whose h slices all landed
+            for (int t = 0; t < T && ok && !*c.abort; ++t) {
+                const int b = t & 1;
+                if (t >= 2 && !(ok = tc::mbar_wait(&c.tempty[b], ((t >> 1) - 1) & 1, limit, c.abort))) break;
+                if (!(ok = tc::mbar_wait(&c.xfull[b], (t >> 1) & 1, limit, c.abort))) break;
+                tc::tc_fence_after();
+                const uint32_t d = tmem + b * kCols;
+                for (int j = 0; j < kcx; ++j)
+                    cl_mma_chunk<NB>(d, c.x0 + (b * kcx + j) * kC64, c.w0 + j * NB * 128, j == 0);
+                tc::mma_commit(&c.xempty[b]);
+                // the h part once every CTA's slice of h_read(t) has landed
+                if (!(ok = mbar_wait_cluster(&c.hready[b], (t >> 1) & 1, limit, c.abort))) break;
+                t_h = t;
+                if (t + 2 < T) tc::mbar_arrive_expect_tx(&c.hready[b], n_ct * kSlice);  // this buffer's next use
+                tc::tc_fence_after();
+                const uint32_t hb = c.h0 + (uint32_t)(b * n_ct) * kSlice;
+                for (uint32_t j = 0; j < n_ct; ++j) {
+                    const uint32_t k = j * U;  // first h unit of slice j
+                    tc::mma_bf16(d, slice_desc(hb + j * kSlice),
+                                 tc::smem_desc(c.w0 + (uint32_t)(kcx + k / kChunk) * NB * 128 + (k % kChunk) * 2, 16, 1024),
+                                 idesc, 1);
+                }
+                tc::mma_commit(&c.tfull[b]);
+            }
+            if (!ok) {
+                cl_abort(c, a.err);
+                // slices other CTAs may still be copying in land before the CTA exits
+                for (int t = t_h + 1; t <= t_h + 2 && t < T; ++t)
+                    tc::mbar_wait(&c.hready[t & 1], (t >> 1) & 1, kDrainLimit, nullptr);
+            }
+            tc::mma_commit(c.done);
+        }
+        __syncwarp();
+    } else {
+        // ------------------------------------------------------------ epilogue
+        const int row = warp * 32 + lane;
+        const bool row_ok = row < B;
+        const bool warp_rows = warp * 32 < B;
+        const int u0 = (int)ct * U;
+        const bool v0 = row_ok && u0 < H, v1 = row_ok && u0 + 8 < H;  // the two 8-unit groups (H % 8 == 0)
+        const uint32_t taddr0 = tmem + ((uint32_t)(warp * 32) << 16);
+        // c of the state step t reads, and (when step t does not push) the h of the older
+        // state that becomes the next step's h operand
+        float crv[U];
+        uint4 hold[2];
+        // top[t + 1][row] and top[t + 2][row] at step t (indices loaded two steps ahead)
+        int s_nxt = 0, s_2 = 0;
+        uint4 h0v[2];
+        if (v0) {
+            const int s_cur = a.top[row];
+            s_nxt = T >= 1 ? a.top[(size_t)B + row] : 0;
+            s_2 = T >= 2 ? a.top[(size_t)2 * B + row] : 0;
+#pragma unroll
+            for (int i = 0; i < 2; ++i) {
+                if (i == 1 && !v1) break;
+                float v[8];
+                ld8f_cg(a.hist_c + ((size_t)s_cur * B + row) * H + u0 + 8 * i, v);
+#pragma unroll
+                for (int k = 0; k < 8; ++k) crv[8 * i + k] = v[k];
+                hold[i] = __ldcg((const uint4 *)(a.hr + ((size_t)s_nxt * B + row) * H + u0 + 8 * i));
+                h0v[i] = __ldcg((const uint4 *)(a.hr + (size_t)row * H + u0 + 8 * i));  // h_read(0)
+            }
+        }
+        deliver_slice(c, 0, row, h0v, v0, v1, ct, n_ct, tid);
+        for (int t = 0; t < T; ++t) {
+            const int b = t & 1;
+            // the next step's operands that rows written before this step hold: issued now,
+            // used after this step's cell (c_read of step t + 1 unless step t pushes; the
+            // older top that is step t + 2's h operand unless it is this step's new state)
+            float cr_n[U];
+            uint4 hold_n[2];
+            int s_3 = 0;
+            if (v0 && t + 1 < T) {
+                if (t + 3 <= T) s_3 = a.top[(size_t)(t + 3) * B + row];
+#pragma unroll
+                for (int i = 0; i < 2; ++i) {
+                    if (i == 1 && !v1) break;
+                    if (s_nxt != t + 1) {
+                        float v[8];
+                        ld8f_cg(a.hist_c + ((size_t)s_nxt * B + row) * H + u0 + 8 * i, v);
+#pragma unroll
+                        for (int k = 0; k < 8; ++k) cr_n[8 * i + k] = v[k];
+                    }
+                    if (s_2 <= t) hold_n[i] = __ldcg((const uint4 *)(a.hr + ((size_t)s_2 * B + row) * H + u0 + 8 * i));
+                }
+            }
+            const bool ok = tc::mbar_wait(&c.tfull[b], (t >> 1) & 1, limit, c.abort);
+            if (!ok) cl_abort(c, a.err);
+            __syncwarp();
+            if (tc::bar_any(1, E * 32, !ok || *c.abort)) break;
+            tc::tc_fence_after();
+            uint32_t zr[4][U];
+            if (warp_rows) {
+#pragma unroll
+                for (int g = 0; g < 4; ++g) tc::tmem_ld16_async(taddr0 + b * kCols + g * U, zr[g]);
+                tc::tmem_wait_ld();
+            }
+            tc::tc_fence_before();
+            __syncwarp();
+            if (lane == 0) tc::mbar_arrive(&c.tempty[b]);
+            // the cell (lanes without a row compute and discard)
+            float cn[U], hn[U], gv[4][U];
+#pragma unroll
+            for (int j = 0; j < U; ++j) {
+                const float ig = sigm(__uint_as_float(zr[0][j]) + s_bias[j]);
+                const float fg = sigm(__uint_as_float(zr[1][j]) + s_bias[U + j]);
+                const float gg = tanh_hw(__uint_as_float(zr[2][j]) + s_bias[2 * U + j]);
+                const float og = sigm(__uint_as_float(zr[3][j]) + s_bias[3 * U + j]);
+                cn[j] = fmaf(fg, crv[j], ig * gg);
+                hn[j] = og * tanh_hw(cn[j]);
+                gv[0][j] = ig; gv[1][j] = fg; gv[2][j] = gg; gv[3][j] = og;
+            }
+            const bool is_new = s_nxt == t + 1;  // step t pushed: h' is the next step's operand
+            uint4 hb[2], hop[2];
+#pragma unroll
+            for (int i = 0; i < 2; ++i) {
+                hb[i] = pack8_bf16(*(const float(*)[8])(hn + 8 * i));
+                hop[i] = is_new ? hb[i] : hold[i];
+            }
+            if (t + 1 < T) deliver_slice(c, (t + 1) & 1, row, hop, v0, v1, ct, n_ct, tid);
+            if (v0) {
+                // history row t + 1, the h operand row t + 1 (for the weight gradient), the gates
+                const size_t w = ((size_t)(t + 1) * B + row) * H + u0;
+                __half *gt = a.gates + ((size_t)t * B + row) * 4 * H + u0;
+#pragma unroll
+                for (int i = 0; i < 2; ++i) {
+                    if (i == 1 && !v1) break;
+                    *(uint4 *)(a.hist_h + w + 8 * i) = hb[i];
+                    *(uint4 *)(a.hr + w + 8 * i) = hop[i];
+                    st8f(a.hist_c + w + 8 * i, *(const float(*)[8])(cn + 8 * i));
+#pragma unroll
+                    for (int g = 0; g < 4; ++g)
+                        *(uint4 *)(gt + (size_t)g * H + 8 * i) = pack8_f16(*(const float(*)[8])(gv[g] + 8 * i));
+                }
+            }
+            if (t + 1 < T) {
+#pragma unroll
+                for (int i = 0; i < 2; ++i) {
+#pragma unroll
+                    for (int k = 0; k < 8; ++k) crv[8 * i + k] = s_nxt == t + 1 ? cn[8 * i + k] : cr_n[8 * i + k];
+                    hold[i] = s_2 == t + 1 ? hb[i] : hold_n[i];
+                }
+                s_nxt = s_2;
+                s_2 = s_3;
+            }
+        }
+    }
+
+    // ---------------------------------------------------------------- teardown
+    __syncthreads();
+    if (warp == E && lane == 0) tc::mbar_wait(c.wbar, 0, kDrainLimit, nullptr);  // after an abort
+    if (warp == E + 1 && lane == 0) tc::mbar_wait(c.done, 0, kDrainLimit, nullptr);
+    tc::cluster_sync();  // no CTA leaves while another may still copy into its shared memory
+    tc::tc_fence_before();
+    __syncthreads();
+    if (warp == E) tc::tmem_dealloc(tmem, 2 * kCols);
+}
+
+constexpr int kClU = 16;  // hidden units per CTA
+
+}  // namespace
+
+// One row tile (B <= 64), at most 16 column tiles of 16 units, the footprint within the
+// shared-memory cap, and a cluster of that size co-resident on this GPU;
+// STACKLSTM_FWD_CLUSTER=0 turns it off.
+bool bf16_plan_fwd_cluster(stacklstm *s, PersistPlan *pl)
+{
+    pl->on = 0;
+    const char *env = getenv("STACKLSTM_FWD_CLUSTER");
+    if (env && atoi(env) == 0) return false;
+    const int n_ct = (int)ceil_div(s->H, kClU);
+    if (s->B > 64 || n_ct > 16) return false;
+    const int NB = 4 * kClU;
+    const uint32_t smem = cl_smem_bytes(s->kcf, s->kcx, NB, n_ct);
+    if (smem > kSmemCap) return false;
+    const void *fn = (const void *)step_cl<kClU>;
+    if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess ||
+        (n_ct > 8 && cudaFuncSetAttribute(fn, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess)) {
+        cudaGetLastError();
+        return false;
+    }
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(n_ct);
+    cfg.blockDim = dim3(192);
+    cfg.dynamicSmemBytes = smem;
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeClusterDimension;
+    at[0].val.clusterDim.x = n_ct;
+    at[0].val.clusterDim.y = 1;
+    at[0].val.clusterDim.z = 1;
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
+    int clusters = 0;
+    if (cudaOccupancyMaxActiveClusters(&clusters, fn, &cfg) != cudaSuccess || clusters < 1) {
+        cudaGetLastError();
+        return false;
+    }
+    pl->on = 1;
+    pl->U = kClU;
+    pl->EP = 1;
+    pl->n_ct = n_ct;
+    pl->cl = n_ct;
+    pl->slot = 1;
+    pl->smem = smem;
+    pl->threads = 192;
+    return true;
+}
+
+cudaError_t bf16_launch_fwd_cluster(stacklstm *s, const StepArgs &a, const CUtensorMap &tm_x)
+{
+    const PersistPlan &pl = s->fc;
+    ClArgs p{};
+    p.s = a;
+    p.n_ct = pl.n_ct;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(pl.n_ct);
+    cfg.blockDim = dim3(pl.threads);
+    cfg.dynamicSmemBytes = pl.smem;
+    cfg.stream = s->stream;
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeClusterDimension;
+    at[0].val.clusterDim.x = pl.n_ct;
+    at[0].val.clusterDim.y = 1;
+    at[0].val.clusterDim.z = 1;
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
+    cudaError_t e = cudaLaunchKernelEx(&cfg, step_cl<kClU>, tm_x, p);
+    if (e) return e;
+    s->launches += 1;
+    return cudaGetLastError();
+}
+
+}  // namespace sl

@@ -172,6 +172,8 @@ cudaError_t allow_smem(Kern k)
 // ---- persistent step kernels (bf16_persist.cu)
 bool bf16_plan_fwd_persist(stacklstm *s, PersistPlan *pl);
 bool bf16_plan_bwd_persist(stacklstm *s, PersistPlan *pl);
+bool bf16_plan_fwd_cluster(stacklstm *s, PersistPlan *pl);
+cudaError_t bf16_launch_fwd_cluster(stacklstm *s, const StepArgs &a, const CUtensorMap &tm_x);
 cudaError_t bf16_launch_fwd_persist(stacklstm *s, const StepArgs &a, const CUtensorMap &tm_x, const CUtensorMap &tm_h,
                                     const CUtensorMap &tm_gates, const CUtensorMap &tm_hh,
                                     const CUtensorMap &tm_hc);

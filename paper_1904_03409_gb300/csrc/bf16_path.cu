@@ -542,7 +542,7 @@ std::string bf16_describe(const stacklstm *s)
 {
     char buf[1024];
     const int rt = (int)ceil_div(s->B, kRows);
-    const PersistPlan &f = s->pf, &b = s->pb;
+    const PersistPlan &f = s->fc.on ? s->fc : s->pf, &b = s->pb;
     snprintf(buf, sizeof buf,
              "bf16 tcgen05; row tiles %d; chunks fwd %d (x %d) bwd %d; "
              "forward %s U=%d [EP %d G %d ring %d slots %d cluster %d col tiles %d w_res %d smem %u threads %d "
@@ -551,7 +551,7 @@ std::string bf16_describe(const stacklstm *s)
              "per SM %d "
              "contraction parts %d dx CTAs %d ring %d]; "
              "step rings fwd %d bwd %d; dx N=%d x%d ring %d; dW %dx%d tiles of 128x%d x%d splits ring %d",
-             rt, s->kcf, s->kcx, s->kcb, f.on ? "persistent" : "per-step", s->uf, f.EP, f.G, f.S, f.slot, f.cl, f.n_ct,
+             rt, s->kcf, s->kcx, s->kcb, s->fc.on ? "cluster" : f.on ? "persistent" : "per-step", s->uf, f.EP, f.G, f.S, f.slot, f.cl, f.n_ct,
              f.w_res, f.smem, f.threads, f.per_sm, b.on ? "persistent" : "per-step", s->ub, b.EP, b.G, b.S, b.slot, b.cl, b.n_ct,
              b.w_res, b.smem, b.threads, b.per_sm, b.KS, b.n_dx, b.dx_S, s->sf, s->sb, s->nx, s->nxt, s->sx, s->dw_mt, s->dw_nt, s->dw_ntile, s->dw_split, s->sw);
     return buf;
@@ -590,6 +590,10 @@ cudaError_t bf16_prepare(stacklstm *s)
     if (!(per_step && atoi(per_step) != 0)) {
         if (bf16_plan_fwd_persist(s, &s->pf)) s->uf = s->pf.U;
         if (bf16_plan_bwd_persist(s, &s->pb)) s->ub = s->pb.U;
+        if (bf16_plan_fwd_cluster(s, &s->fc)) {
+            s->uf = s->fc.U;
+            s->pf.on = 0;
+        }
     }
     s->sf = pick_stages(s->kcf, 4 * s->uf, ceil_div(H, s->uf) * (size_t)rt, sms);
     s->sb = pick_stages(s->kcb, s->ub, ceil_div(H, s->ub) * (size_t)rt, sms);
@@ -669,6 +673,8 @@ cudaError_t bf16_forward_steps(stacklstm *s, const float *bias)
     const int T = s->T, B = s->B, H = s->H;
     const int nctf = std::max((int)ceil_div(H, s->uf), s->pf.on ? s->pf.n_ct : 0);
     cudaError_t e;
+    if (s->fc.on)
+        return bf16_launch_fwd_cluster(s, step_args(s, bias, s->w_fwd, s->kcx, s->kcf, 0), map(s, kMapX64));
     if (s->pf.on)
         return bf16_launch_fwd_persist(s, step_args(s, bias, s->w_fwd, s->kcx, s->kcf, s->pf.S),
                                        map(s, B <= 64 ? kMapX64 : kMapX128), map(s, B <= 64 ? kMapH64 : kMapH128),

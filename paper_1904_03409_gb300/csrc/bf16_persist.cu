@@ -121,10 +121,13 @@ __device__ __forceinline__ void ws_abort(const WCtl &c, int32_t *err)
     atomicCAS(err, 0, (int)SL_ERR_TIMEOUT);
 }
 
+#ifndef STACKLSTM_SPIN_NS
+#define STACKLSTM_SPIN_NS 32
+#endif
 // Bounded spin until *cnt >= target (acquire). False on timeout, on a local abort, or
 // once another CTA recorded an error.
 __device__ __forceinline__ bool spin_until(const int32_t *cnt, int target, long long limit, volatile int *abort,
-                                           const int32_t *err, unsigned sleep_ns = 32)
+                                           const int32_t *err, unsigned sleep_ns = STACKLSTM_SPIN_NS)
 {
     if (tc::ld_acquire_gpu(cnt) >= target) return true;
     const long long t0 = clock64();

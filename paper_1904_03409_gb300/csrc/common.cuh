@@ -80,6 +80,7 @@ struct stacklstm {
     alignas(64) unsigned char tmaps[10][128] = {};  // TMA descriptors (bf16_path.cu)
     // persistent step kernels (one launch for all T steps; bf16_persist.cu)
     PersistPlan pf, pb;            // forward, backward (on = 0: one launch per step)
+    PersistPlan fc;                // forward as one thread-block cluster (one row tile; bf16_cluster.cu)
     int32_t *rowcnt = nullptr;     // [2][row tiles][cnt_stride] completed steps per row tile
     int cnt_stride = 32;           // ints between two row tiles' counters (one 128-byte line each)
     float *split_part = nullptr;   // backward split contraction: partial dh_read rows
