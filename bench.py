@@ -97,7 +97,7 @@ def phase_kernel(plan, phase):
     if phase in ("forward", "backward"):
         m = re.search(phase + r" (persistent|per-step|cluster) U=(\d+)", plan)
         if m and m.group(1) == "cluster":
-            return "step_cl<U=%s,%s>" % (m.group(2), phase), "bf16_cluster.cu"
+            return "%s<U=%s,%s>" % ("step_cl" if phase == "forward" else "step_clb", m.group(2), phase), "bf16_cluster.cu"
         if m and m.group(1) == "persistent":
             return "step_ws<U=%s,%s>" % (m.group(2), phase), "bf16_persist.cu"
         return ("fwd_step_tc" if phase == "forward" else "bwd_step_tc"), "bf16_path.cu"

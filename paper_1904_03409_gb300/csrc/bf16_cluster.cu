@@ -389,6 +389,324 @@ __global__ void __launch_bounds__(192, 1) step_cl(const __grid_constant__ CUtens
 
 constexpr int kClU = 16;  // hidden units per CTA
 
+// ====================================================================== backward
+// The reverse-time backward (Sec. 5) for one row tile (B <= 64) as one thread-block
+// cluster. Step t multiplies dG_t (all 4H gate columns of the row tile) by this CTA's
+// slice of W_h to get dh_read for its 16 units; the epilogue then adds it to the gradient
+// of the state step t read and runs the pointwise backward of step t - 1 for its units,
+// whose gate gradients dG_{t-1} (4 gates x 16 units x 64 rows) it stages as four 2 KB
+// slices and copies into every CTA's dG buffer with one 8 KB bulk copy each. The K order
+// of the contraction is slice order: K step (j, g) covers gate g of units 16 j .. 16 j + 15,
+// so the weights are packed per K step too (16 x 16, 512 bytes, same core-matrix layout).
+// The dG buffer is single: before a CTA copies dG_{t-1} in, every CTA's step-t MMAs have
+// completed (their commits arrive on the `dfree` barrier of every CTA of the cluster).
+//
+// [weight slices 4 n_ct x 512][dG buffer n_ct x 8 KB][2 KB pad][staging 2 x 8 KB][barriers]
+constexpr uint32_t kWSlice = 512;
+constexpr uint32_t kGBlock = 4 * kSlice;  // one CTA's four gate slices
+__host__ __device__ constexpr uint32_t clb_smem_bytes(int n_ct)
+{
+    return 1024 + 4u * n_ct * kWSlice + (uint32_t)n_ct * kGBlock + kSlice + 2 * kGBlock + kClBars;
+}
+
+struct ClbCtl {
+    uint32_t w0, g0, stg;  // weight slices, dG buffer, staging
+    uint64_t *wbar, *gready, *dfree, *tfull, *tempty, *done;
+    uint32_t *tmem_slot;
+    volatile int *abort;
+};
+
+__device__ __forceinline__ ClbCtl clb_carve(uint8_t *raw, int n_ct)
+{
+    const uint32_t off = smem_u32(raw);
+    uint8_t *base = raw + ((1024u - (off & 1023u)) & 1023u);
+    ClbCtl c;
+    const uint32_t wb = 4u * n_ct * kWSlice, gb = (uint32_t)n_ct * kGBlock + kSlice;
+    c.w0 = smem_u32(base);
+    c.g0 = c.w0 + wb;
+    c.stg = c.g0 + gb;
+    uint64_t *bars = (uint64_t *)(base + wb + gb + 2 * kGBlock);
+    c.wbar = bars;
+    c.gready = bars + 1;
+    c.dfree = bars + 2;
+    c.tfull = bars + 3;
+    c.tempty = bars + 5;
+    c.done = bars + 7;
+    c.tmem_slot = (uint32_t *)(bars + 8);
+    c.abort = (volatile int *)(c.tmem_slot + 1);
+    return c;
+}
+
+}  // namespace
+
+// Weight slices of the cluster backward: for CTA ct, K step (j, g), the 16 x 16 block
+// B[n][k] = W[I + 16 ct + n][g H + 16 j + k] (zero past H), in the unswizzled K-major
+// core-matrix layout; out is [n_ct][4 gates][n_ct][512 bytes].
+__global__ void pack_bwd_slices(const __nv_bfloat16 *__restrict__ W, int I, int H, int n_ct,
+                                __nv_bfloat16 *__restrict__ out)
+{
+    const size_t n = (size_t)n_ct * 4 * n_ct * 256;
+    for (size_t e = blockIdx.x * (size_t)blockDim.x + threadIdx.x; e < n; e += (size_t)gridDim.x * blockDim.x) {
+        const int nk = (int)(e % 256), blk = (int)(e / 256);  // element within the block, block index
+        const int nn = nk / 16, kk = nk % 16;
+        const int j = blk % n_ct, g = (blk / n_ct) % 4, ct = blk / (4 * n_ct);
+        const int unit = 16 * ct + nn, ku = 16 * j + kk;
+        const __nv_bfloat16 v = (unit < H && ku < H) ? W[(size_t)(I + unit) * 4 * H + g * H + ku] : __float2bfloat16(0.0f);
+        const uint32_t byte = (uint32_t)(nn >> 3) * 256 + (uint32_t)(kk >> 3) * 128 + (uint32_t)(nn & 7) * 16 + (uint32_t)(kk & 7) * 2;
+        out[((size_t)blk * kWSlice + byte) / 2] = v;
+    }
+}
+
+namespace {
+// this thread's dG_{t-1} (4 gates x 16 units, bf16) as staging block `buf`; zero past H or B
+__device__ __forceinline__ void stage_dg(uint32_t stg, int row, const uint4 (&v)[4][2], bool v0, bool v1)
+{
+    if (row >= 64) return;
+    const uint4 z = make_uint4(0u, 0u, 0u, 0u);
+#pragma unroll
+    for (int g = 0; g < 4; ++g) {
+        const uint4 a0 = v0 ? v[g][0] : z, a1 = v1 ? v[g][1] : z;
+        tc::st_shared_v4(stg + g * kSlice + slice_off((uint32_t)row, 0), (const uint32_t *)&a0);
+        tc::st_shared_v4(stg + g * kSlice + slice_off((uint32_t)row, 1), (const uint32_t *)&a1);
+    }
+}
+
+// After every epilogue warp has staged: thread 0 waits until every CTA's MMAs of the step
+// that read the dG buffer completed (dfree phase `fpar`, skipped for the first delivery),
+// then copies the four slices into every CTA's dG buffer at this CTA's block.
+__device__ __forceinline__ bool deliver_dg(const ClbCtl &c, int buf, int fpar, uint32_t ct, uint32_t n_ct, int tid,
+                                           long long limit, int32_t *err)
+{
+    tc::fence_proxy_async();
+    __syncwarp();
+    tc::bar_sync(2, 4 * 32);
+    bool ok = true;
+    if (tid == 0) {
+        if (fpar >= 0 && !(ok = mbar_wait_cluster(c.dfree, (uint32_t)fpar, limit, c.abort))) {
+            *c.abort = 1;
+            atomicCAS(err, 0, (int)SL_ERR_TIMEOUT);
+        }
+        if (ok) {
+            const uint32_t dst = c.g0 + ct * kGBlock, bar = smem_u32(c.gready);
+            for (uint32_t r = 0; r < n_ct; ++r)
+                bulk_s2c(peer_addr(dst, r), c.stg + buf * kGBlock, kGBlock, peer_addr(bar, r));
+        }
+    }
+    return ok;
+}
+
+template <int U>
+__global__ void __launch_bounds__(192, 1) step_clb(ClArgs p)
+{
+    static_assert(U == 16, "four 16-unit gate slices per CTA");
+    constexpr uint32_t kCols = TmemCols<U>::value;
+    constexpr int E = 4;
+    const StepArgs &a = p.s;
+    extern __shared__ uint8_t smem_raw[];
+    const int T = a.T, B = a.B, H = a.H;
+    const uint32_t ct = tc::cluster_rank(), n_ct = (uint32_t)p.n_ct;
+    const ClbCtl c = clb_carve(smem_raw, (int)n_ct);
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const long long limit = a.limit;
+    if (tid == 0) {
+        tc::mbar_init(c.wbar, 1);
+        tc::mbar_init(c.gready, 1);
+        tc::mbar_init(c.dfree, n_ct);
+        for (int i = 0; i < 2; ++i) {
+            tc::mbar_init(&c.tfull[i], 1);
+            tc::mbar_init(&c.tempty[i], E);
+        }
+        tc::mbar_init(c.done, 1);
+        *c.abort = 0;
+        tc::fence_mbar_init();
+        tc::mbar_arrive_expect_tx(c.gready, n_ct * kGBlock);  // dG of step T - 1
+    }
+    if (warp == E) tc::tmem_alloc(c.tmem_slot, 2 * kCols);
+    tc::tc_fence_before();
+    __syncthreads();
+    tc::cluster_sync();  // every CTA's barriers exist before any copy or commit lands on them
+    tc::tc_fence_after();
+    const uint32_t tmem = *c.tmem_slot;
+
+    if (warp == E) {
+        // ------------------------------------------------------------ weight slices, once
+        if (lane == 0) {
+            const uint32_t wbytes = 4u * n_ct * kWSlice;
+            tc::mbar_arrive_expect_tx(c.wbar, wbytes);
+            tc::bulk_g2s(c.w0, a.wpack + (size_t)ct * wbytes, wbytes, c.wbar);
+        }
+        __syncwarp();
+    } else if (warp == E + 1) {
+        // ------------------------------------------------------------ MMA issue
+        if (lane == 0) {
+            constexpr uint32_t idesc = tc::idesc_bf16(U);
+            bool ok = tc::mbar_wait(c.wbar, 0, limit, c.abort);
+            int k_g = -1;  // last step index whose dG had landed
+            for (int k = 0; k < T && ok && !*c.abort; ++k) {  // step t = T - 1 - k
+                const int acc = k & 1;
+                if (k >= 2 && !(ok = tc::mbar_wait(&c.tempty[acc], ((k >> 1) - 1) & 1, limit, c.abort))) break;
+                if (!(ok = mbar_wait_cluster(c.gready, (uint32_t)(k & 1), limit, c.abort))) break;
+                k_g = k;
+                if (k + 1 < T) tc::mbar_arrive_expect_tx(c.gready, n_ct * kGBlock);  // dG of the next step
+                tc::tc_fence_after();
+                const uint32_t d = tmem + acc * kCols;
+                for (uint32_t j = 0; j < n_ct; ++j)
+#pragma unroll
+                    for (int g = 0; g < 4; ++g)
+                        tc::mma_bf16(d, slice_desc(c.g0 + j * kGBlock + g * kSlice),
+                                     slice_desc(c.w0 + ((uint32_t)g * n_ct + j) * kWSlice), idesc, (j | g) != 0);
+                tc::mma_commit(&c.tfull[acc]);
+                // the dG buffer may be refilled once every CTA's MMAs of this step are done
+                tc::mma_commit_mc(c.dfree, (uint16_t)((1u << n_ct) - 1));
+            }
+            if (!ok) {
+                *c.abort = 1;
+                atomicCAS(a.err, 0, (int)SL_ERR_TIMEOUT);
+                // dG other CTAs may still be copying in lands before the CTA exits
+                if (k_g + 1 < T) tc::mbar_wait(c.gready, (uint32_t)((k_g + 1) & 1), kDrainLimit, nullptr);
+            }
+            tc::mma_commit(c.done);
+            // every CTA's commit of the last step has arrived here before the CTA exits
+            if (ok) mbar_wait_cluster(c.dfree, (uint32_t)((T - 1) & 1), kDrainLimit, nullptr);
+        }
+        __syncwarp();
+    } else {
+        // ------------------------------------------------------------ epilogue
+        const int row = warp * 32 + lane;
+        const bool row_ok = row < B;
+        const bool warp_rows = warp * 32 < B;
+        const int u0 = (int)ct * U;
+        const bool v0 = row_ok && u0 < H, v1 = row_ok && u0 + 8 < H;  // the two 8-unit groups (H % 8 == 0)
+        const uint32_t taddr0 = tmem + ((uint32_t)(warp * 32) << 16);
+        // dG of step T - 1 (written before the launch) into every CTA's dG buffer
+        {
+            uint4 g0[4][2];
+            if (v0)
+#pragma unroll
+                for (int g = 0; g < 4; ++g)
+#pragma unroll
+                    for (int i = 0; i < 2; ++i)
+                        if (i == 0 || v1)
+                            g0[g][i] = __ldcg((const uint4 *)(a.dG + ((size_t)(T - 1) * B + row) * 4 * H + g * H + u0 + 8 * i));
+            stage_dg(c.stg, row, g0, v0, v1);
+            deliver_dg(c, 0, -1, ct, n_ct, tid, limit, a.err);
+        }
+        // the state step t reads (src) and the one step t - 1 read (s1): a step ahead
+        int src = 0, s1 = 0;
+        if (row_ok) {
+            src = a.top[(size_t)(T - 1) * B + row];
+            s1 = T >= 2 ? a.top[(size_t)(T - 2) * B + row] : 0;
+        }
+        for (int k = 0; k < T; ++k) {
+            const int t = T - 1 - k, acc = k & 1;
+            // this step's operands (rows this thread wrote at later steps, or the forward's)
+            float dh_src[U], dh_t[U], dc_t[U], cn[U], cr[U], dc_rd[U];
+            uint4 gq[4][2];
+            int src_n = 0, s1_n = 0;
+            if (row_ok && t >= 1) {
+                src_n = a.top[(size_t)(t - 1) * B + row];
+                s1_n = t >= 2 ? a.top[(size_t)(t - 2) * B + row] : 0;
+            }
+            if (v0)
+#pragma unroll
+                for (int i = 0; i < 2; ++i) {
+                    if (i == 1 && !v1) break;
+                    const size_t us = ((size_t)src * B + row) * H + u0 + 8 * i;
+                    ld8f_cg(a.dhist_h + us, *(float(*)[8])(dh_src + 8 * i));
+                    if (t >= 1) {
+                        const size_t wr = ((size_t)t * B + row) * H + u0 + 8 * i, rd = ((size_t)s1 * B + row) * H + u0 + 8 * i;
+                        ld8f_cg(a.dhist_h + wr, *(float(*)[8])(dh_t + 8 * i));
+                        ld8f_cg(a.dhist_c + wr, *(float(*)[8])(dc_t + 8 * i));
+                        ld8f_cg(a.hist_c + wr, *(float(*)[8])(cn + 8 * i));
+                        ld8f_cg(a.hist_c + rd, *(float(*)[8])(cr + 8 * i));
+                        ld8f_cg(a.dhist_c + rd, *(float(*)[8])(dc_rd + 8 * i));
+                        const __half *gt = a.gates + ((size_t)(t - 1) * B + row) * 4 * H + u0 + 8 * i;
+#pragma unroll
+                        for (int g = 0; g < 4; ++g) gq[g][i] = __ldcg((const uint4 *)(gt + (size_t)g * H));
+                    }
+                }
+            const bool ok = tc::mbar_wait(&c.tfull[acc], (k >> 1) & 1, limit, c.abort);
+            if (!ok) {
+                *c.abort = 1;
+                atomicCAS(a.err, 0, (int)SL_ERR_TIMEOUT);
+            }
+            __syncwarp();
+            if (tc::bar_any(1, E * 32, !ok || *c.abort)) break;
+            tc::tc_fence_after();
+            uint32_t dr[U];
+            if (warp_rows) {
+                tc::tmem_ld16_async(taddr0 + acc * kCols, dr);
+                tc::tmem_wait_ld();
+            }
+            tc::tc_fence_before();
+            __syncwarp();
+            if (lane == 0) tc::mbar_arrive(&c.tempty[acc]);
+            float v[U];
+#pragma unroll
+            for (int j = 0; j < U; ++j) v[j] = dh_src[j] + __uint_as_float(dr[j]);
+            float dcr[U];
+            if (t >= 1) {
+                // the pointwise backward of step t - 1 (lanes without a row compute and discard)
+                float d[4][U];
+#pragma unroll
+                for (int i = 0; i < 2; ++i) {
+                    float ig[8], fg[8], gg[8], og[8];
+                    unpack8_f16(gq[0][i], ig);
+                    unpack8_f16(gq[1][i], fg);
+                    unpack8_f16(gq[2][i], gg);
+                    unpack8_f16(gq[3][i], og);
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) {
+                        const int q = 8 * i + e;
+                        const float dh = src == t ? v[q] : dh_t[q];  // the state read at t is row t
+                        const float tcn = tanh_hw(cn[q]);
+                        const float dc = dc_t[q] + dh * og[e] * (1.0f - tcn * tcn);
+                        d[0][q] = dc * gg[e] * ig[e] * (1.0f - ig[e]);
+                        d[1][q] = dc * cr[q] * fg[e] * (1.0f - fg[e]);
+                        d[2][q] = dc * ig[e] * (1.0f - gg[e] * gg[e]);
+                        d[3][q] = dh * tcn * og[e] * (1.0f - og[e]);
+                        dcr[q] = dc_rd[q] + dc * fg[e];
+                    }
+                }
+                uint4 dg[4][2];
+#pragma unroll
+                for (int g = 0; g < 4; ++g)
+#pragma unroll
+                    for (int i = 0; i < 2; ++i) dg[g][i] = pack8_bf16(*(const float(*)[8])(d[g] + 8 * i));
+                // dG_{t-1} to every CTA first (the next step waits for it), then the stores
+                stage_dg(c.stg + ((k + 1) & 1) * kGBlock, row, dg, v0, v1);
+                deliver_dg(c, (k + 1) & 1, k & 1, ct, n_ct, tid, limit, a.err);
+                if (v0)
+#pragma unroll
+                    for (int i = 0; i < 2; ++i) {
+                        if (i == 1 && !v1) break;
+                        __nv_bfloat16 *gp = a.dG + ((size_t)(t - 1) * B + row) * 4 * H + u0 + 8 * i;
+#pragma unroll
+                        for (int g = 0; g < 4; ++g) *(uint4 *)(gp + (size_t)g * H) = dg[g][i];
+                    }
+            }
+            if (v0)
+#pragma unroll
+                for (int i = 0; i < 2; ++i) {
+                    if (i == 1 && !v1) break;
+                    st8f(a.dhist_h + ((size_t)src * B + row) * H + u0 + 8 * i, *(const float(*)[8])(v + 8 * i));
+                    if (t >= 1) st8f(a.dhist_c + ((size_t)s1 * B + row) * H + u0 + 8 * i, *(const float(*)[8])(dcr + 8 * i));
+                }
+            src = src_n;
+            s1 = s1_n;
+        }
+    }
+
+    // ---------------------------------------------------------------- teardown
+    __syncthreads();
+    if (warp == E && lane == 0) tc::mbar_wait(c.wbar, 0, kDrainLimit, nullptr);  // after an abort
+    if (warp == E + 1 && lane == 0) tc::mbar_wait(c.done, 0, kDrainLimit, nullptr);
+    tc::cluster_sync();  // no CTA leaves while another may still copy into its shared memory
+    tc::tc_fence_before();
+    __syncthreads();
+    if (warp == E) tc::tmem_dealloc(tmem, 2 * kCols);
+}
+
 }  // namespace
 
 // One row tile (B <= 64), at most 16 column tiles of 16 units, the footprint within the
@@ -456,6 +774,93 @@ cudaError_t bf16_launch_fwd_cluster(stacklstm *s, const StepArgs &a, const CUten
     cfg.attrs = at;
     cfg.numAttrs = 1;
     cudaError_t e = cudaLaunchKernelEx(&cfg, step_cl<kClU>, tm_x, p);
+    if (e) return e;
+    s->launches += 1;
+    return cudaGetLastError();
+}
+
+// The backward of one row tile as a cluster: B <= 64, at most 16 column tiles of 16
+// units, a co-resident cluster of that size. Only on request (STACKLSTM_BWD_CLUSTER=1):
+// measured slower than the persistent backward at B = 64, H = 200 (1.40 against 1.07 ms
+// for 185 steps). Each step moves n_ct x n_ct 8 KB copies between the CTAs, issued one
+// after another by one thread of each, and the contraction waits for all of them, where
+// the persistent kernel writes each slice once to L2 and pipelines its loads with the MMAs.
+bool bf16_plan_bwd_cluster(stacklstm *s, PersistPlan *pl)
+{
+    pl->on = 0;
+    const char *env = getenv("STACKLSTM_BWD_CLUSTER");
+    if (!env || atoi(env) == 0) return false;
+    const int n_ct = (int)ceil_div(s->H, kClU);
+    if (s->B > 64 || n_ct > 16) return false;
+    const uint32_t smem = clb_smem_bytes(n_ct);
+    if (smem > kSmemCap) return false;
+    const void *fn = (const void *)step_clb<kClU>;
+    if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess ||
+        (n_ct > 8 && cudaFuncSetAttribute(fn, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess)) {
+        cudaGetLastError();
+        return false;
+    }
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(n_ct);
+    cfg.blockDim = dim3(192);
+    cfg.dynamicSmemBytes = smem;
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeClusterDimension;
+    at[0].val.clusterDim.x = n_ct;
+    at[0].val.clusterDim.y = 1;
+    at[0].val.clusterDim.z = 1;
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
+    int clusters = 0;
+    if (cudaOccupancyMaxActiveClusters(&clusters, fn, &cfg) != cudaSuccess || clusters < 1) {
+        cudaGetLastError();
+        return false;
+    }
+    pl->on = 1;
+    pl->U = kClU;
+    pl->EP = 1;
+    pl->n_ct = n_ct;
+    pl->cl = n_ct;
+    pl->slot = 1;
+    pl->smem = smem;
+    pl->threads = 192;
+    return true;
+}
+
+size_t bf16_bwd_cluster_weight_bytes(int H)
+{
+    const size_t n_ct = ceil_div(H, kClU);
+    return n_ct * 4 * n_ct * kWSlice;
+}
+
+cudaError_t bf16_pack_bwd_cluster(stacklstm *s, const __nv_bfloat16 *W, __nv_bfloat16 *out)
+{
+    const int n_ct = s->bc.n_ct;
+    const size_t n = (size_t)n_ct * 4 * n_ct * 256;
+    pack_bwd_slices<<<(unsigned)std::min<size_t>((n + 255) / 256, 4096), 256, 0, s->stream>>>(W, s->I, s->H, n_ct, out);
+    s->launches += 1;
+    return cudaGetLastError();
+}
+
+cudaError_t bf16_launch_bwd_cluster(stacklstm *s, const StepArgs &a)
+{
+    const PersistPlan &pl = s->bc;
+    ClArgs p{};
+    p.s = a;
+    p.n_ct = pl.n_ct;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(pl.n_ct);
+    cfg.blockDim = dim3(pl.threads);
+    cfg.dynamicSmemBytes = pl.smem;
+    cfg.stream = s->stream;
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeClusterDimension;
+    at[0].val.clusterDim.x = pl.n_ct;
+    at[0].val.clusterDim.y = 1;
+    at[0].val.clusterDim.z = 1;
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
+    cudaError_t e = cudaLaunchKernelEx(&cfg, step_clb<kClU>, p);
     if (e) return e;
     s->launches += 1;
     return cudaGetLastError();

@@ -542,7 +542,7 @@ std::string bf16_describe(const stacklstm *s)
 {
     char buf[1024];
     const int rt = (int)ceil_div(s->B, kRows);
-    const PersistPlan &f = s->fc.on ? s->fc : s->pf, &b = s->pb;
+    const PersistPlan &f = s->fc.on ? s->fc : s->pf, &b = s->bc.on ? s->bc : s->pb;
     snprintf(buf, sizeof buf,
              "bf16 tcgen05; row tiles %d; chunks fwd %d (x %d) bwd %d; "
              "forward %s U=%d [EP %d G %d ring %d slots %d cluster %d col tiles %d w_res %d smem %u threads %d "
@@ -552,7 +552,7 @@ std::string bf16_describe(const stacklstm *s)
              "contraction parts %d dx CTAs %d ring %d]; "
              "step rings fwd %d bwd %d; dx N=%d x%d ring %d; dW %dx%d tiles of 128x%d x%d splits ring %d",
              rt, s->kcf, s->kcx, s->kcb, s->fc.on ? "cluster" : f.on ? "persistent" : "per-step", s->uf, f.EP, f.G, f.S, f.slot, f.cl, f.n_ct,
-             f.w_res, f.smem, f.threads, f.per_sm, b.on ? "persistent" : "per-step", s->ub, b.EP, b.G, b.S, b.slot, b.cl, b.n_ct,
+             f.w_res, f.smem, f.threads, f.per_sm, s->bc.on ? "cluster" : b.on ? "persistent" : "per-step", s->bc.on ? s->bc.U : s->ub, b.EP, b.G, b.S, b.slot, b.cl, b.n_ct,
              b.w_res, b.smem, b.threads, b.per_sm, b.KS, b.n_dx, b.dx_S, s->sf, s->sb, s->nx, s->nxt, s->sx, s->dw_mt, s->dw_nt, s->dw_ntile, s->dw_split, s->sw);
     return buf;
 }
@@ -594,6 +594,7 @@ cudaError_t bf16_prepare(stacklstm *s)
             s->uf = s->fc.U;
             s->pf.on = 0;
         }
+        if (bf16_plan_bwd_cluster(s, &s->bc)) s->pb.on = 0;
     }
     s->sf = pick_stages(s->kcf, 4 * s->uf, ceil_div(H, s->uf) * (size_t)rt, sms);
     s->sb = pick_stages(s->kcb, s->ub, ceil_div(H, s->ub) * (size_t)rt, sms);
@@ -611,6 +612,10 @@ cudaError_t bf16_prepare(stacklstm *s)
     s->allocs.push_back(p); s->w_bwd = p;
     if ((e = cudaMalloc(&p, dx_bytes))) return e;
     s->allocs.push_back(p); s->w_dx = p;
+    if (s->bc.on) {
+        if ((e = cudaMalloc(&p, bf16_bwd_cluster_weight_bytes(H)))) return e;
+        s->allocs.push_back(p); s->w_bcl = p;
+    }
     if ((e = cudaMalloc(&p, s->dw_part_elems * sizeof(float)))) return e;
     s->allocs.push_back(p); s->dw_part = (float *)p;
     if (s->pb.on && s->pb.KS > 1) {
@@ -665,6 +670,7 @@ cudaError_t bf16_forward_setup(stacklstm *s, const __nv_bfloat16 *x, const __nv_
     pack_rows<<<grid_for(s, (size_t)s->nxt * s->kcb * s->nx * kChunk), 256, 0, s->stream>>>(
         W, H, 0, I, s->nx, s->kcb, s->nxt, (__nv_bfloat16 *)s->w_dx);
     s->launches += 3;
+    if (s->bc.on && (e = bf16_pack_bwd_cluster(s, W, (__nv_bfloat16 *)s->w_bcl))) return e;
     return cudaGetLastError();
 }
 
@@ -713,6 +719,7 @@ cudaError_t bf16_backward_steps(stacklstm *s, float *dx, bool *dx_done)
     const int T = s->T, B = s->B, H = s->H;
     cudaError_t e;
     const StepArgs a = step_args(s, nullptr, s->w_bwd, 0, s->kcb, s->sb);
+    if (s->bc.on) return bf16_launch_bwd_cluster(s, step_args(s, nullptr, s->w_bcl, 0, s->kcb, 0));
     // one row tile of at most 64 instances: 64-row boxes (the rest of each stage is never
     // loaded and only feeds accumulator rows that are not stored)
     if (s->pb.on)

@@ -217,3 +217,18 @@ def test_input_gradient_on_spare_sms_matches_oracle(T, B, I, H, seed):
     plan1, one = run_nan_filled(w, {"STACKLSTM_DX_SPARE": "1"})
     assert "dx CTAs 1" in plan1, plan1
     assert np.array_equal(one["dx"], sep["dx"])
+
+
+@pytest.mark.parametrize("T,B,I,H,seed", [(17, 37, 8, 16, 19), (24, 64, 200, 200, 20), (9, 5, 64, 136, 21)])
+def test_cluster_kernels_for_one_row_tile_match_oracle(T, B, I, H, seed):
+    """One row tile (B <= 64): the forward as one thread-block cluster (its default) and the
+    backward as one (on request), into NaN-filled outputs, match the oracle; the cluster
+    backward gives the same gradients as the persistent one up to accumulation order."""
+    w = case(T, B, I, H, seed, bias_scale=0.3, h0_scale=0.5, c0_scale=0.5, dy_scale=0.5)
+    plan, got = run_nan_filled(w, {"STACKLSTM_BWD_CLUSTER": "1"})
+    assert "forward cluster U=16" in plan and "backward cluster U=16" in plan, plan
+    ref = oracle_all(w)
+    compare(got, ref, "bf16")
+    plan_p, per = run_nan_filled(w, {})
+    assert "backward persistent" in plan_p, plan_p
+    compare(per, ref, "bf16")
