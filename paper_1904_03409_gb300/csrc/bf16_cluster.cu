@@ -394,14 +394,15 @@ constexpr int kClU = 16;  // hidden units per CTA
 // cluster. Step t multiplies dG_t (all 4H gate columns of the row tile) by this CTA's
 // slice of W_h to get dh_read for its 16 units; the epilogue then adds it to the gradient
 // of the state step t read and runs the pointwise backward of step t - 1 for its units,
-// whose gate gradients dG_{t-1} (4 gates x 16 units x 64 rows) it stages as four 2 KB
-// slices and copies into every CTA's dG buffer with one 8 KB bulk copy each. The K order
+// whose gate gradients dG_{t-1} (4 gates x 16 units x 64 rows) it writes to global memory
+// and then loads, as four 2 KB slices, into every CTA's dG buffer with multicast tensor
+// loads (one L2 read, delivered to all CTAs of the cluster). The K order
 // of the contraction is slice order: K step (j, g) covers gate g of units 16 j .. 16 j + 15,
 // so the weights are packed per K step too (16 x 16, 512 bytes, same core-matrix layout).
 // The dG buffer is single: before a CTA copies dG_{t-1} in, every CTA's step-t MMAs have
 // completed (their commits arrive on the `dfree` barrier of every CTA of the cluster).
 //
-// [weight slices 4 n_ct x 512][dG buffer n_ct x 8 KB][2 KB pad][staging 2 x 8 KB][barriers]
+// [weight slices 4 n_ct x 512][dG buffer n_ct x 8 KB][2 KB pad][(unused) 2 x 8 KB][barriers]
 constexpr uint32_t kWSlice = 512;
 constexpr uint32_t kGBlock = 4 * kSlice;  // one CTA's four gate slices
 __host__ __device__ constexpr uint32_t clb_smem_bytes(int n_ct)
@@ -458,45 +459,33 @@ __global__ void pack_bwd_slices(const __nv_bfloat16 *__restrict__ W, int I, int 
 }
 
 namespace {
-// this thread's dG_{t-1} (4 gates x 16 units, bf16) as staging block `buf`; zero past H or B
-__device__ __forceinline__ void stage_dg(uint32_t stg, int row, const uint4 (&v)[4][2], bool v0, bool v1)
+// After every epilogue warp has stored its rows of dG for step s to global memory: thread 0
+// waits until every CTA's MMAs of the step that read the dG buffer completed (dfree phase
+// `fpar`, skipped for the first delivery), then loads this CTA's four gate slices of step s
+// from global memory into every CTA's dG buffer with multicast tensor loads (a 4-D view of
+// dG that yields the slice layout: [row / 8][unit / 8][row mod 8][unit mod 8]).
+__device__ __forceinline__ void deliver_dg(const ClbCtl &c, const CUtensorMap *tm_g, int step, int fpar, uint32_t ct,
+                                           uint32_t n_ct, int tid, int B, int H, long long limit, int32_t *err)
 {
-    if (row >= 64) return;
-    const uint4 z = make_uint4(0u, 0u, 0u, 0u);
-#pragma unroll
-    for (int g = 0; g < 4; ++g) {
-        const uint4 a0 = v0 ? v[g][0] : z, a1 = v1 ? v[g][1] : z;
-        tc::st_shared_v4(stg + g * kSlice + slice_off((uint32_t)row, 0), (const uint32_t *)&a0);
-        tc::st_shared_v4(stg + g * kSlice + slice_off((uint32_t)row, 1), (const uint32_t *)&a1);
-    }
-}
-
-// After every epilogue warp has staged: thread 0 waits until every CTA's MMAs of the step
-// that read the dG buffer completed (dfree phase `fpar`, skipped for the first delivery),
-// then copies the four slices into every CTA's dG buffer at this CTA's block.
-__device__ __forceinline__ bool deliver_dg(const ClbCtl &c, int buf, int fpar, uint32_t ct, uint32_t n_ct, int tid,
-                                           long long limit, int32_t *err)
-{
-    tc::fence_proxy_async();
+    tc::fence_proxy_async_global();  // this thread's dG stores -> the tensor loads
     __syncwarp();
     tc::bar_sync(2, 4 * 32);
-    bool ok = true;
     if (tid == 0) {
+        bool ok = true;
         if (fpar >= 0 && !(ok = mbar_wait_cluster(c.dfree, (uint32_t)fpar, limit, c.abort))) {
             *c.abort = 1;
             atomicCAS(err, 0, (int)SL_ERR_TIMEOUT);
         }
-        if (ok) {
-            const uint32_t dst = c.g0 + ct * kGBlock, bar = smem_u32(c.gready);
-            for (uint32_t r = 0; r < n_ct; ++r)
-                bulk_s2c(peer_addr(dst, r), c.stg + buf * kGBlock, kGBlock, peer_addr(bar, r));
-        }
+        if (ok)
+#pragma unroll
+            for (int g = 0; g < 4; ++g)
+                tc::tma_load_4d_mc(c.g0 + ct * kGBlock + g * kSlice, tm_g, 0, 0, (g * H + (int)ct * 16) / 8,
+                                   step * B / 8, c.gready, (uint16_t)((1u << n_ct) - 1));
     }
-    return ok;
 }
 
 template <int U>
-__global__ void __launch_bounds__(192, 1) step_clb(ClArgs p)
+__global__ void __launch_bounds__(192, 1) step_clb(const __grid_constant__ CUtensorMap tm_g, ClArgs p)
 {
     static_assert(U == 16, "four 16-unit gate slices per CTA");
     constexpr uint32_t kCols = TmemCols<U>::value;
@@ -579,18 +568,7 @@ __global__ void __launch_bounds__(192, 1) step_clb(ClArgs p)
         const bool v0 = row_ok && u0 < H, v1 = row_ok && u0 + 8 < H;  // the two 8-unit groups (H % 8 == 0)
         const uint32_t taddr0 = tmem + ((uint32_t)(warp * 32) << 16);
         // dG of step T - 1 (written before the launch) into every CTA's dG buffer
-        {
-            uint4 g0[4][2];
-            if (v0)
-#pragma unroll
-                for (int g = 0; g < 4; ++g)
-#pragma unroll
-                    for (int i = 0; i < 2; ++i)
-                        if (i == 0 || v1)
-                            g0[g][i] = __ldcg((const uint4 *)(a.dG + ((size_t)(T - 1) * B + row) * 4 * H + g * H + u0 + 8 * i));
-            stage_dg(c.stg, row, g0, v0, v1);
-            deliver_dg(c, 0, -1, ct, n_ct, tid, limit, a.err);
-        }
+        deliver_dg(c, &tm_g, T - 1, -1, ct, n_ct, tid, B, H, limit, a.err);
         // the state step t reads (src) and the one step t - 1 read (s1): a step ahead
         int src = 0, s1 = 0;
         if (row_ok) {
@@ -673,9 +651,7 @@ __global__ void __launch_bounds__(192, 1) step_clb(ClArgs p)
                 for (int g = 0; g < 4; ++g)
 #pragma unroll
                     for (int i = 0; i < 2; ++i) dg[g][i] = pack8_bf16(*(const float(*)[8])(d[g] + 8 * i));
-                // dG_{t-1} to every CTA first (the next step waits for it), then the stores
-                stage_dg(c.stg + ((k + 1) & 1) * kGBlock, row, dg, v0, v1);
-                deliver_dg(c, (k + 1) & 1, k & 1, ct, n_ct, tid, limit, a.err);
+                // dG_{t-1} to global memory, then (multicast tensor loads) to every CTA
                 if (v0)
 #pragma unroll
                     for (int i = 0; i < 2; ++i) {
@@ -684,6 +660,7 @@ __global__ void __launch_bounds__(192, 1) step_clb(ClArgs p)
 #pragma unroll
                         for (int g = 0; g < 4; ++g) *(uint4 *)(gp + (size_t)g * H) = dg[g][i];
                     }
+                deliver_dg(c, &tm_g, t - 1, k & 1, ct, n_ct, tid, B, H, limit, a.err);
             }
             if (v0)
 #pragma unroll
@@ -779,19 +756,18 @@ cudaError_t bf16_launch_fwd_cluster(stacklstm *s, const StepArgs &a, const CUten
     return cudaGetLastError();
 }
 
-// The backward of one row tile as a cluster: B <= 64, at most 16 column tiles of 16
-// units, a co-resident cluster of that size. Only on request (STACKLSTM_BWD_CLUSTER=1):
-// measured slower than the persistent backward at B = 64, H = 200 (1.40 against 1.07 ms
-// for 185 steps). Each step moves n_ct x n_ct 8 KB copies between the CTAs, issued one
-// after another by one thread of each, and the contraction waits for all of them, where
-// the persistent kernel writes each slice once to L2 and pipelines its loads with the MMAs.
+// The backward of one row tile as a cluster: B <= 64 and a multiple of 8, at most 16
+// column tiles of 16 units, a co-resident cluster of that size; STACKLSTM_BWD_CLUSTER=0
+// turns it off. (Copying each CTA's 8 KB of dG into every CTA with bulk copies instead of
+// the multicast tensor loads ran 30 % slower than the persistent backward at B = 64,
+// H = 200: n_ct^2 copies a step, issued one after another by one thread of each CTA.)
 bool bf16_plan_bwd_cluster(stacklstm *s, PersistPlan *pl)
 {
     pl->on = 0;
     const char *env = getenv("STACKLSTM_BWD_CLUSTER");
-    if (!env || atoi(env) == 0) return false;
+    if (env && atoi(env) == 0) return false;
     const int n_ct = (int)ceil_div(s->H, kClU);
-    if (s->B > 64 || n_ct > 16) return false;
+    if (s->B > 64 || s->B % 8 || n_ct > 16) return false;  // (whole 8-row groups for the 4-D view)
     const uint32_t smem = clb_smem_bytes(n_ct);
     if (smem > kSmemCap) return false;
     const void *fn = (const void *)step_clb<kClU>;
@@ -842,7 +818,7 @@ cudaError_t bf16_pack_bwd_cluster(stacklstm *s, const __nv_bfloat16 *W, __nv_bfl
     return cudaGetLastError();
 }
 
-cudaError_t bf16_launch_bwd_cluster(stacklstm *s, const StepArgs &a)
+cudaError_t bf16_launch_bwd_cluster(stacklstm *s, const StepArgs &a, const CUtensorMap &tm_g)
 {
     const PersistPlan &pl = s->bc;
     ClArgs p{};
@@ -860,7 +836,7 @@ cudaError_t bf16_launch_bwd_cluster(stacklstm *s, const StepArgs &a)
     at[0].val.clusterDim.z = 1;
     cfg.attrs = at;
     cfg.numAttrs = 1;
-    cudaError_t e = cudaLaunchKernelEx(&cfg, step_clb<kClU>, p);
+    cudaError_t e = cudaLaunchKernelEx(&cfg, step_clb<kClU>, tm_g, p);
     if (e) return e;
     s->launches += 1;
     return cudaGetLastError();

@@ -114,10 +114,12 @@ def test_stress_config_sampled():
     sampled_check(w, [0, 1, 127, 128, 2047, 3000, 4094, 4095])
 
 
-def test_wait_timeout_is_reported_and_context_survives():
-    """With a zero wait budget the bounded device-side waits run out: forward reports
-    SL_ERR_TIMEOUT instead of hanging, and the device stays usable."""
-    w = case(4, 130, 16, 32, 9)
+@pytest.mark.parametrize("B", [130, 40])
+def test_wait_timeout_is_reported_and_context_survives(B):
+    """With a zero wait budget the bounded device-side waits run out: forward (persistent
+    kernel at B = 130, thread-block cluster at B = 40) reports SL_ERR_TIMEOUT instead of
+    hanging, and the device stays usable."""
+    w = case(4, B, 16, 32, 9)
     os.environ["STACKLSTM_WAIT_LIMIT_CYCLES"] = "0"
     try:
         hd = bd.stacklstm_create(w.T, w.B, w.I, w.H, bd.SL_BF16, 0)
@@ -219,16 +221,18 @@ def test_input_gradient_on_spare_sms_matches_oracle(T, B, I, H, seed):
     assert np.array_equal(one["dx"], sep["dx"])
 
 
-@pytest.mark.parametrize("T,B,I,H,seed", [(17, 37, 8, 16, 19), (24, 64, 200, 200, 20), (9, 5, 64, 136, 21)])
+@pytest.mark.parametrize("T,B,I,H,seed", [(17, 40, 8, 16, 19), (24, 64, 200, 200, 20), (9, 8, 64, 136, 21),
+                                         (12, 37, 24, 40, 22)])
 def test_cluster_kernels_for_one_row_tile_match_oracle(T, B, I, H, seed):
-    """One row tile (B <= 64): the forward as one thread-block cluster (its default) and the
-    backward as one (on request), into NaN-filled outputs, match the oracle; the cluster
-    backward gives the same gradients as the persistent one up to accumulation order."""
+    """One row tile (B <= 64): the forward and (B a multiple of 8) the backward as one
+    thread-block cluster each, their defaults, into NaN-filled outputs, match the oracle,
+    as do the persistent kernels they replace."""
     w = case(T, B, I, H, seed, bias_scale=0.3, h0_scale=0.5, c0_scale=0.5, dy_scale=0.5)
-    plan, got = run_nan_filled(w, {"STACKLSTM_BWD_CLUSTER": "1"})
-    assert "forward cluster U=16" in plan and "backward cluster U=16" in plan, plan
+    plan, got = run_nan_filled(w, {})
+    assert "forward cluster U=16" in plan, plan
+    assert ("backward cluster U=16" in plan) == (B % 8 == 0), plan
     ref = oracle_all(w)
     compare(got, ref, "bf16")
-    plan_p, per = run_nan_filled(w, {})
-    assert "backward persistent" in plan_p, plan_p
+    plan_p, per = run_nan_filled(w, {"STACKLSTM_BWD_CLUSTER": "0", "STACKLSTM_FWD_CLUSTER": "0"})
+    assert "forward persistent" in plan_p and "backward persistent" in plan_p, plan_p
     compare(per, ref, "bf16")
