@@ -139,7 +139,7 @@ __device__ __forceinline__ uint64_t slice_desc(uint32_t addr)
 __host__ __device__ constexpr uint32_t slice_off(uint32_t r, uint32_t k) { return (r >> 3) * 256 + k * 128 + (r & 7) * 16; }
 
 // Stages this thread's row of h_read(t + 1) (16 units, zero past H or B) as slice buffer
-// `buf`, then (once every epilogue warp has) one thread copies the slice into every CTA's
+// `buf`, then (once every epilogue warp has) lane r of warp 0 copies the slice into CTA r's
 // h buffer `buf` at this CTA's slice position, completing on that CTA's hready[buf].
 __device__ __forceinline__ void deliver_slice(const ClCtl &c, int buf, int row, const uint4 (&v)[2], bool valid0,
                                               bool valid1, uint32_t ct, uint32_t n_ct, int tid)
@@ -153,9 +153,9 @@ __device__ __forceinline__ void deliver_slice(const ClCtl &c, int buf, int row, 
     tc::fence_proxy_async();  // generic writes -> the bulk copies
     __syncwarp();
     tc::bar_sync(2, 4 * 32);
-    if (tid == 0) {
+    if (tid < (int)n_ct) {  // lane r of warp 0 copies to CTA r (all at once)
         const uint32_t dst = c.h0 + (uint32_t)(buf * n_ct + ct) * kSlice, bar = smem_u32(&c.hready[buf]);
-        for (uint32_t r = 0; r < n_ct; ++r) bulk_s2c(peer_addr(dst, r), c.stg + buf * kSlice, kSlice, peer_addr(bar, r));
+        bulk_s2c(peer_addr(dst, (uint32_t)tid), c.stg + buf * kSlice, kSlice, peer_addr(bar, (uint32_t)tid));
     }
 }
 
