@@ -32,8 +32,9 @@ using tc::smem_u32;
 constexpr uint32_t kC64 = 64 * 128;  // one 64-row chunk
 
 struct ClArgs {
-    StepArgs s;  // s.kcx: x chunks; s.KC: all chunks
-    int n_ct;    // column tiles = CTAs of the cluster
+    StepArgs s;     // s.kcx: x chunks; s.KC: all chunks
+    int n_ct;       // column tiles = CTAs of the cluster
+    uint8_t *gscr;  // backward: [T][n_ct] swizzled 8 KB dG blocks
 };
 
 // [weight tile KC x NB x 128][h buffers 2 x n_ct x 2 KB][2 KB pad][x buffers 2 x kcx x 8 KB]
@@ -395,23 +396,26 @@ constexpr int kClU = 16;  // hidden units per CTA
 // slice of W_h to get dh_read for its 16 units; the epilogue then adds it to the gradient
 // of the state step t read and runs the pointwise backward of step t - 1 for its units,
 // whose gate gradients dG_{t-1} (4 gates x 16 units x 64 rows) it writes to global memory
-// and then loads, as four 2 KB slices, into every CTA's dG buffer with multicast tensor
-// loads (one L2 read, delivered to all CTAs of the cluster). The K order
-// of the contraction is slice order: K step (j, g) covers gate g of units 16 j .. 16 j + 15,
-// so the weights are packed per K step too (16 x 16, 512 bytes, same core-matrix layout).
-// The dG buffer is single: before a CTA copies dG_{t-1} in, every CTA's step-t MMAs have
-// completed (their commits arrive on the `dfree` barrier of every CTA of the cluster).
+// twice: in the [T B][4H] layout (for the input and weight gradients) and as one block of
+// 64 rows x 128 bytes (gate-major, 16 units a gate) already in the 128-byte-swizzled
+// operand layout, which one multicast bulk copy then loads into every CTA's dG buffer (one
+// L2 read of 8 KB, delivered to all CTAs of the cluster, completing on their mbarrier by
+// byte count). The K order of the contraction is block order: chunk j is CTA j's block,
+// K = 16 g + e for unit 16 j + e of gate g; the weights are packed to match (16 rows x 64,
+// 128-byte swizzled, per chunk). The dG buffer is single: before a CTA loads dG_{t-1} in,
+// every CTA's step-t MMAs have completed (their commits arrive on the `dfree` barrier of
+// every CTA of the cluster).
 //
-// [weight slices 4 n_ct x 512][dG buffer n_ct x 8 KB][2 KB pad][(unused) 2 x 8 KB][barriers]
-constexpr uint32_t kWSlice = 512;
-constexpr uint32_t kGBlock = 4 * kSlice;  // one CTA's four gate slices
+// [weight chunks n_ct x 2 KB][dG buffer n_ct x 8 KB][8 KB pad][barriers]
+constexpr uint32_t kWChunkB = 16 * 128;  // one weight chunk: 16 rows x 64 K
+constexpr uint32_t kGBlock = 64 * 128;   // one CTA's dG block: 64 rows x 64 K
 __host__ __device__ constexpr uint32_t clb_smem_bytes(int n_ct)
 {
-    return 1024 + 4u * n_ct * kWSlice + (uint32_t)n_ct * kGBlock + kSlice + 2 * kGBlock + kClBars;
+    return 1024 + (uint32_t)n_ct * kWChunkB + (uint32_t)n_ct * kGBlock + kGBlock + kClBars;
 }
 
 struct ClbCtl {
-    uint32_t w0, g0, stg;  // weight slices, dG buffer, staging
+    uint32_t w0, g0;  // weight chunks, dG buffer
     uint64_t *wbar, *gready, *dfree, *tfull, *tempty, *done;
     uint32_t *tmem_slot;
     volatile int *abort;
@@ -422,11 +426,10 @@ __device__ __forceinline__ ClbCtl clb_carve(uint8_t *raw, int n_ct)
     const uint32_t off = smem_u32(raw);
     uint8_t *base = raw + ((1024u - (off & 1023u)) & 1023u);
     ClbCtl c;
-    const uint32_t wb = 4u * n_ct * kWSlice, gb = (uint32_t)n_ct * kGBlock + kSlice;
+    const uint32_t wb = (uint32_t)n_ct * kWChunkB, gb = (uint32_t)n_ct * kGBlock + kGBlock;
     c.w0 = smem_u32(base);
     c.g0 = c.w0 + wb;
-    c.stg = c.g0 + gb;
-    uint64_t *bars = (uint64_t *)(base + wb + gb + 2 * kGBlock);
+    uint64_t *bars = (uint64_t *)(base + wb + gb);
     c.wbar = bars;
     c.gready = bars + 1;
     c.dfree = bars + 2;
@@ -440,34 +443,56 @@ __device__ __forceinline__ ClbCtl clb_carve(uint8_t *raw, int n_ct)
 
 }  // namespace
 
-// Weight slices of the cluster backward: for CTA ct, K step (j, g), the 16 x 16 block
-// B[n][k] = W[I + 16 ct + n][g H + 16 j + k] (zero past H), in the unswizzled K-major
-// core-matrix layout; out is [n_ct][4 gates][n_ct][512 bytes].
+// Weight chunks of the cluster backward: for CTA ct, chunk j, the 16 x 64 block
+// B[n][16 g + e] = W[I + 16 ct + n][g H + 16 j + e] (zero past H), 128-byte swizzled rows;
+// out is [n_ct][n_ct chunks][16 rows][64].
 __global__ void pack_bwd_slices(const __nv_bfloat16 *__restrict__ W, int I, int H, int n_ct,
                                 __nv_bfloat16 *__restrict__ out)
 {
-    const size_t n = (size_t)n_ct * 4 * n_ct * 256;
+    const size_t n = (size_t)n_ct * n_ct * 16 * 64;
     for (size_t e = blockIdx.x * (size_t)blockDim.x + threadIdx.x; e < n; e += (size_t)gridDim.x * blockDim.x) {
-        const int nk = (int)(e % 256), blk = (int)(e / 256);  // element within the block, block index
-        const int nn = nk / 16, kk = nk % 16;
-        const int j = blk % n_ct, g = (blk / n_ct) % 4, ct = blk / (4 * n_ct);
-        const int unit = 16 * ct + nn, ku = 16 * j + kk;
+        const int kk = (int)(e % 64), nn = (int)((e / 64) % 16);
+        const int blk = (int)(e / (64 * 16)), j = blk % n_ct, ct = blk / n_ct;
+        const int g = kk / 16, unit = 16 * ct + nn, ku = 16 * j + kk % 16;
         const __nv_bfloat16 v = (unit < H && ku < H) ? W[(size_t)(I + unit) * 4 * H + g * H + ku] : __float2bfloat16(0.0f);
-        const uint32_t byte = (uint32_t)(nn >> 3) * 256 + (uint32_t)(kk >> 3) * 128 + (uint32_t)(nn & 7) * 16 + (uint32_t)(kk & 7) * 2;
-        out[((size_t)blk * kWSlice + byte) / 2] = v;
+        const uint32_t byte = sw128((uint32_t)nn, (uint32_t)kk >> 3) + (uint32_t)(kk & 7) * 2;
+        out[((size_t)blk * kWChunkB + byte) / 2] = v;
     }
 }
 
 namespace {
-// After every epilogue warp has stored its rows of dG for step s to global memory: thread 0
-// waits until every CTA's MMAs of the step that read the dG buffer completed (dfree phase
-// `fpar`, skipped for the first delivery), then loads this CTA's four gate slices of step s
-// from global memory into every CTA's dG buffer with multicast tensor loads (a 4-D view of
-// dG that yields the slice layout: [row / 8][unit / 8][row mod 8][unit mod 8]).
-__device__ __forceinline__ void deliver_dg(const ClbCtl &c, const CUtensorMap *tm_g, int step, int fpar, uint32_t ct,
-                                           uint32_t n_ct, int tid, int B, int H, long long limit, int32_t *err)
+// Bulk copy of `bytes` from global memory into the same shared-memory offset of every CTA
+// of cta_mask, completing on the mbarrier at the same offset in each.
+__device__ __forceinline__ void bulk_g2s_mc(uint32_t dst, const void *src, uint32_t bytes, uint64_t *bar,
+                                            uint16_t cta_mask)
 {
-    tc::fence_proxy_async_global();  // this thread's dG stores -> the tensor loads
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.multicast::cluster [%0], [%1], %2, [%3], "
+        "%4;" ::"r"(dst),
+        "l"(src), "r"(bytes), "r"(smem_u32(bar)), "h"(cta_mask)
+        : "memory");
+}
+
+// This thread's row of a dG block (4 gates x 16 units, zero past H or B) into the swizzled
+// global block `blk` (64 rows x 128 bytes).
+__device__ __forceinline__ void store_dg_block(uint8_t *blk, int row, const uint4 (&v)[4][2], bool v0, bool v1)
+{
+    if (row >= 64) return;
+    const uint4 z = make_uint4(0u, 0u, 0u, 0u);
+#pragma unroll
+    for (int g = 0; g < 4; ++g)
+#pragma unroll
+        for (int i = 0; i < 2; ++i)
+            *(uint4 *)(blk + sw128((uint32_t)row, (uint32_t)(2 * g + i))) = (i == 0 ? v0 : v1) ? v[g][i] : z;
+}
+
+// After every epilogue warp has stored its rows of the block: thread 0 waits until every
+// CTA's MMAs of the step that read the dG buffer completed (dfree phase `fpar`, skipped for
+// the first delivery), then loads the block into every CTA's dG buffer at this CTA's chunk.
+__device__ __forceinline__ void deliver_dg(const ClbCtl &c, const uint8_t *blk, int fpar, uint32_t ct, uint32_t n_ct,
+                                           int tid, long long limit, int32_t *err)
+{
+    tc::fence_proxy_async_global();  // this thread's block stores -> the bulk copy
     __syncwarp();
     tc::bar_sync(2, 4 * 32);
     if (tid == 0) {
@@ -476,16 +501,12 @@ __device__ __forceinline__ void deliver_dg(const ClbCtl &c, const CUtensorMap *t
             *c.abort = 1;
             atomicCAS(err, 0, (int)SL_ERR_TIMEOUT);
         }
-        if (ok)
-#pragma unroll
-            for (int g = 0; g < 4; ++g)
-                tc::tma_load_4d_mc(c.g0 + ct * kGBlock + g * kSlice, tm_g, 0, 0, (g * H + (int)ct * 16) / 8,
-                                   step * B / 8, c.gready, (uint16_t)((1u << n_ct) - 1));
+        if (ok) bulk_g2s_mc(c.g0 + ct * kGBlock, blk, kGBlock, c.gready, (uint16_t)((1u << n_ct) - 1));
     }
 }
 
 template <int U>
-__global__ void __launch_bounds__(192, 1) step_clb(const __grid_constant__ CUtensorMap tm_g, ClArgs p)
+__global__ void __launch_bounds__(192, 1) step_clb(ClArgs p)
 {
     static_assert(U == 16, "four 16-unit gate slices per CTA");
     constexpr uint32_t kCols = TmemCols<U>::value;
@@ -520,7 +541,7 @@ __global__ void __launch_bounds__(192, 1) step_clb(const __grid_constant__ CUten
     if (warp == E) {
         // ------------------------------------------------------------ weight slices, once
         if (lane == 0) {
-            const uint32_t wbytes = 4u * n_ct * kWSlice;
+            const uint32_t wbytes = n_ct * kWChunkB;
             tc::mbar_arrive_expect_tx(c.wbar, wbytes);
             tc::bulk_g2s(c.w0, a.wpack + (size_t)ct * wbytes, wbytes, c.wbar);
         }
@@ -541,9 +562,9 @@ __global__ void __launch_bounds__(192, 1) step_clb(const __grid_constant__ CUten
                 const uint32_t d = tmem + acc * kCols;
                 for (uint32_t j = 0; j < n_ct; ++j)
 #pragma unroll
-                    for (int g = 0; g < 4; ++g)
-                        tc::mma_bf16(d, slice_desc(c.g0 + j * kGBlock + g * kSlice),
-                                     slice_desc(c.w0 + ((uint32_t)g * n_ct + j) * kWSlice), idesc, (j | g) != 0);
+                    for (int kq = 0; kq < kChunk / 16; ++kq)
+                        tc::mma_bf16(d, tc::smem_desc(c.g0 + j * kGBlock + kq * 32, 16, 1024),
+                                     tc::smem_desc(c.w0 + j * kWChunkB + kq * 32, 16, 1024), idesc, (j | kq) != 0);
                 tc::mma_commit(&c.tfull[acc]);
                 // the dG buffer may be refilled once every CTA's MMAs of this step are done
                 tc::mma_commit_mc(c.dfree, (uint16_t)((1u << n_ct) - 1));
@@ -568,7 +589,19 @@ __global__ void __launch_bounds__(192, 1) step_clb(const __grid_constant__ CUten
         const bool v0 = row_ok && u0 < H, v1 = row_ok && u0 + 8 < H;  // the two 8-unit groups (H % 8 == 0)
         const uint32_t taddr0 = tmem + ((uint32_t)(warp * 32) << 16);
         // dG of step T - 1 (written before the launch) into every CTA's dG buffer
-        deliver_dg(c, &tm_g, T - 1, -1, ct, n_ct, tid, B, H, limit, a.err);
+        {
+            uint4 g0v[4][2];
+            if (v0)
+#pragma unroll
+                for (int g = 0; g < 4; ++g)
+#pragma unroll
+                    for (int i = 0; i < 2; ++i)
+                        if (i == 0 || v1)
+                            g0v[g][i] = __ldcg((const uint4 *)(a.dG + ((size_t)(T - 1) * B + row) * 4 * H + g * H + u0 + 8 * i));
+            uint8_t *blk = p.gscr + ((size_t)(T - 1) * n_ct + ct) * kGBlock;
+            store_dg_block(blk, row, g0v, v0, v1);
+            deliver_dg(c, blk, -1, ct, n_ct, tid, limit, a.err);
+        }
         // the state step t reads (src) and the one step t - 1 read (s1): a step ahead
         int src = 0, s1 = 0;
         if (row_ok) {
@@ -651,7 +684,7 @@ __global__ void __launch_bounds__(192, 1) step_clb(const __grid_constant__ CUten
                 for (int g = 0; g < 4; ++g)
 #pragma unroll
                     for (int i = 0; i < 2; ++i) dg[g][i] = pack8_bf16(*(const float(*)[8])(d[g] + 8 * i));
-                // dG_{t-1} to global memory, then (multicast tensor loads) to every CTA
+                // dG_{t-1} to global memory, then (multicast bulk copy of its block) to every CTA
                 if (v0)
 #pragma unroll
                     for (int i = 0; i < 2; ++i) {
@@ -660,7 +693,9 @@ __global__ void __launch_bounds__(192, 1) step_clb(const __grid_constant__ CUten
 #pragma unroll
                         for (int g = 0; g < 4; ++g) *(uint4 *)(gp + (size_t)g * H) = dg[g][i];
                     }
-                deliver_dg(c, &tm_g, t - 1, k & 1, ct, n_ct, tid, B, H, limit, a.err);
+                uint8_t *blk = p.gscr + ((size_t)(t - 1) * n_ct + ct) * kGBlock;
+                store_dg_block(blk, row, dg, v0, v1);
+                deliver_dg(c, blk, k & 1, ct, n_ct, tid, limit, a.err);
             }
             if (v0)
 #pragma unroll
@@ -756,9 +791,8 @@ cudaError_t bf16_launch_fwd_cluster(stacklstm *s, const StepArgs &a, const CUten
     return cudaGetLastError();
 }
 
-// The backward of one row tile as a cluster: B <= 64 and a multiple of 8, at most 16
-// column tiles of 16 units, a co-resident cluster of that size; STACKLSTM_BWD_CLUSTER=0
-// turns it off. (Copying each CTA's 8 KB of dG into every CTA with bulk copies instead of
+// The backward of one row tile as a cluster: B <= 64, at most 16 column tiles of 16 units,
+// a co-resident cluster of that size; STACKLSTM_BWD_CLUSTER=0 turns it off. (Copying each CTA's 8 KB of dG into every CTA with bulk copies instead of
 // the multicast tensor loads ran 30 % slower than the persistent backward at B = 64,
 // H = 200: n_ct^2 copies a step, issued one after another by one thread of each CTA.)
 bool bf16_plan_bwd_cluster(stacklstm *s, PersistPlan *pl)
@@ -767,7 +801,7 @@ bool bf16_plan_bwd_cluster(stacklstm *s, PersistPlan *pl)
     const char *env = getenv("STACKLSTM_BWD_CLUSTER");
     if (env && atoi(env) == 0) return false;
     const int n_ct = (int)ceil_div(s->H, kClU);
-    if (s->B > 64 || s->B % 8 || n_ct > 16) return false;  // (whole 8-row groups for the 4-D view)
+    if (s->B > 64 || n_ct > 16) return false;
     const uint32_t smem = clb_smem_bytes(n_ct);
     if (smem > kSmemCap) return false;
     const void *fn = (const void *)step_clb<kClU>;
@@ -803,27 +837,30 @@ bool bf16_plan_bwd_cluster(stacklstm *s, PersistPlan *pl)
     return true;
 }
 
+size_t bf16_bwd_cluster_block_bytes(int T, int H) { return (size_t)T * ceil_div(H, kClU) * kGBlock; }
+
 size_t bf16_bwd_cluster_weight_bytes(int H)
 {
     const size_t n_ct = ceil_div(H, kClU);
-    return n_ct * 4 * n_ct * kWSlice;
+    return n_ct * n_ct * kWChunkB;
 }
 
 cudaError_t bf16_pack_bwd_cluster(stacklstm *s, const __nv_bfloat16 *W, __nv_bfloat16 *out)
 {
     const int n_ct = s->bc.n_ct;
-    const size_t n = (size_t)n_ct * 4 * n_ct * 256;
+    const size_t n = (size_t)n_ct * n_ct * 16 * 64;
     pack_bwd_slices<<<(unsigned)std::min<size_t>((n + 255) / 256, 4096), 256, 0, s->stream>>>(W, s->I, s->H, n_ct, out);
     s->launches += 1;
     return cudaGetLastError();
 }
 
-cudaError_t bf16_launch_bwd_cluster(stacklstm *s, const StepArgs &a, const CUtensorMap &tm_g)
+cudaError_t bf16_launch_bwd_cluster(stacklstm *s, const StepArgs &a)
 {
     const PersistPlan &pl = s->bc;
     ClArgs p{};
     p.s = a;
     p.n_ct = pl.n_ct;
+    p.gscr = (uint8_t *)s->g_bcl;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(pl.n_ct);
     cfg.blockDim = dim3(pl.threads);
@@ -836,7 +873,7 @@ cudaError_t bf16_launch_bwd_cluster(stacklstm *s, const StepArgs &a, const CUten
     at[0].val.clusterDim.z = 1;
     cfg.attrs = at;
     cfg.numAttrs = 1;
-    cudaError_t e = cudaLaunchKernelEx(&cfg, step_clb<kClU>, tm_g, p);
+    cudaError_t e = cudaLaunchKernelEx(&cfg, step_clb<kClU>, p);
     if (e) return e;
     s->launches += 1;
     return cudaGetLastError();

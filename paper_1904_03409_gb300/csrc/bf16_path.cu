@@ -501,24 +501,8 @@ cudaError_t make_hist_map(void *slot, const void *base, bool fp32, int T, int B,
     return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
 }
 
-// The gate gradients dG [T B][4H] (bf16) as the 4-D view [row / 8][unit / 8][row mod 8][unit mod 8]
-// (fastest last) whose 8 x 8 x 2 x 8 boxes are the cluster backward's 16-unit, 64-row slices
-// in the unswizzled K-major core-matrix layout (T B a multiple of 8).
-cudaError_t make_cl_dg_map(void *slot, const void *base, int T, int B, int H)
-{
-    const cuuint64_t G = 4 * (cuuint64_t)H;
-    cuuint64_t dims[4] = {8, 8, G / 8, (cuuint64_t)T * B / 8};
-    cuuint64_t strides[3] = {G * 2, 16, 8 * G * 2};
-    cuuint32_t box[4] = {8, 8, 2, 8};
-    cuuint32_t el[4] = {1, 1, 1, 1};
-    CUresult r = g_encode((CUtensorMap *)slot, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void *>(base), dims,
-                          strides, box, el, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
-                          CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-    return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
-}
-
 enum { kMapX128 = 0, kMapX64 = 1, kMapG128 = 2, kMapG64 = 3, kMapH128 = 4, kMapH64 = 5, kMapGates = 6, kMapHistH = 7,
-       kMapHistC = 8, kMapGcl = 9 };
+       kMapHistC = 8 };
 const CUtensorMap &map(const stacklstm *s, int i) { return *(const CUtensorMap *)s->tmaps[i]; }
 
 // budget that leaves room for two CTAs per SM when the grid needs more than one wave.
@@ -631,6 +615,8 @@ cudaError_t bf16_prepare(stacklstm *s)
     if (s->bc.on) {
         if ((e = cudaMalloc(&p, bf16_bwd_cluster_weight_bytes(H)))) return e;
         s->allocs.push_back(p); s->w_bcl = p;
+        if ((e = cudaMalloc(&p, bf16_bwd_cluster_block_bytes(T, H)))) return e;
+        s->allocs.push_back(p); s->g_bcl = p;
     }
     if ((e = cudaMalloc(&p, s->dw_part_elems * sizeof(float)))) return e;
     s->allocs.push_back(p); s->dw_part = (float *)p;
@@ -652,7 +638,6 @@ cudaError_t bf16_prepare(stacklstm *s)
     // dG is workspace: its tensor maps are fixed for the handle's lifetime
     if ((e = make_map(s->tmaps[kMapG128], s->dG, R, 4 * (uint64_t)H, kRows))) return e;
     if ((e = make_map(s->tmaps[kMapG64], s->dG, R, 4 * (uint64_t)H, kChunk))) return e;
-    if (s->bc.on && make_cl_dg_map(s->tmaps[kMapGcl], s->dG, T, B, H) != cudaSuccess) s->bc.on = 0;
     const uint64_t R1 = (uint64_t)(T + 1) * B;
     if ((e = make_map(s->tmaps[kMapH128], s->hr, R1, (uint64_t)H, kRows))) return e;
     if ((e = make_map(s->tmaps[kMapH64], s->hr, R1, (uint64_t)H, kChunk))) return e;
@@ -736,7 +721,7 @@ cudaError_t bf16_backward_steps(stacklstm *s, float *dx, bool *dx_done)
     const int T = s->T, B = s->B, H = s->H;
     cudaError_t e;
     const StepArgs a = step_args(s, nullptr, s->w_bwd, 0, s->kcb, s->sb);
-    if (s->bc.on) return bf16_launch_bwd_cluster(s, step_args(s, nullptr, s->w_bcl, 0, s->kcb, 0), map(s, kMapGcl));
+    if (s->bc.on) return bf16_launch_bwd_cluster(s, step_args(s, nullptr, s->w_bcl, 0, s->kcb, 0));
     // one row tile of at most 64 instances: 64-row boxes (the rest of each stage is never
     // loaded and only feeds accumulator rows that are not stored)
     if (s->pb.on)

@@ -82,7 +82,8 @@ struct stacklstm {
     PersistPlan pf, pb;            // forward, backward (on = 0: one launch per step)
     PersistPlan fc;                // forward as one thread-block cluster (one row tile; bf16_cluster.cu)
     PersistPlan bc;                // backward as one thread-block cluster (one row tile; bf16_cluster.cu)
-    void *w_bcl = nullptr;         // its weight slices
+    void *w_bcl = nullptr;         // its weight chunks
+    void *g_bcl = nullptr;         // its swizzled dG blocks [T][column tiles][8 KB]
     int32_t *rowcnt = nullptr;     // [2][row tiles][cnt_stride] completed steps per row tile
     int cnt_stride = 32;           // ints between two row tiles' counters (one 128-byte line each)
     float *split_part = nullptr;   // backward split contraction: partial dh_read rows

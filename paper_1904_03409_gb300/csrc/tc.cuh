@@ -183,17 +183,6 @@ __device__ __forceinline__ void cluster_sync()
 }
 // TMA tile load delivered to the same shared-memory offset of every CTA in cta_mask; each
 // destination CTA's mbarrier at the same offset receives the box's bytes.
-// 4-D tile load multicast to the CTAs of cta_mask (same shared-memory offset and mbarrier
-// in each).
-__device__ __forceinline__ void tma_load_4d_mc(uint32_t dst, const void *tmap, int c0, int c1, int c2, int c3,
-                                               uint64_t *bar, uint16_t cta_mask)
-{
-    asm volatile(
-        "cp.async.bulk.tensor.4d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.multicast::cluster"
-        " [%0], [%1, {%2, %3, %4, %5}], [%6], %7;" ::"r"(dst),
-        "l"((uint64_t)tmap), "r"(c0), "r"(c1), "r"(c2), "r"(c3), "r"(smem_u32(bar)), "h"(cta_mask)
-        : "memory");
-}
 __device__ __forceinline__ void tma_load_2d_mc(uint32_t dst, const void *tmap, int c0, int c1, uint64_t *bar,
                                                uint16_t cta_mask)
 {
