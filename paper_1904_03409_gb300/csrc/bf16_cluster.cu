@@ -1,10 +1,10 @@
 // bf16_cluster.cu -- the forward recurrence (Algorithm 1) for one row tile of at most 64
 // instances as a single thread-block cluster. The n_ct column-tile CTAs (16 hidden units
 // each, n_ct <= 16) hand each step's h operand to one another through distributed shared
-// memory: the epilogue of step t stages its 16 units of h_read(t + 1) (h' where step t
-// pushed, else the older top) as one 2 KB slice, and one thread copies the slice into every
-// CTA's operand buffer for step t + 1 with bulk copies that complete on that CTA's
-// mbarrier by byte count. Nothing on the step's critical path goes through global memory
+// memory: the epilogue of step t writes its 16 units of h_read(t + 1) (h' where step t
+// pushed, else the older top) as one 2 KB slice block to global memory, and one multicast
+// bulk copy loads it into every CTA's operand buffer for step t + 1, completing on that
+// CTA's mbarrier by byte count. Nothing on the step's critical path goes through global memory
 // or a step counter; the history rows, the h operand rows (for the weight gradient) and
 // the gates are still written to global memory for the backward.
 //
@@ -38,16 +38,16 @@ struct ClArgs {
 };
 
 // [weight tile KC x NB x 128][h buffers 2 x n_ct x 2 KB][2 KB pad][x buffers 2 x kcx x 8 KB]
-// [8 KB pad][staging 2 x 2 KB][barriers], based at the first 1024-byte boundary
+// [8 KB pad][barriers], based at the first 1024-byte boundary
 constexpr uint32_t kSlice = 2048;
 constexpr uint32_t kClBars = 16 * 8 + 16;
 __host__ __device__ constexpr uint32_t cl_smem_bytes(int KC, int kcx, int NB, int n_ct)
 {
-    return 1024 + (uint32_t)KC * NB * 128 + (2u * n_ct + 1) * kSlice + 2u * kcx * kC64 + kC64 + 2 * kSlice + kClBars;
+    return 1024 + (uint32_t)KC * NB * 128 + (2u * n_ct + 1) * kSlice + 2u * kcx * kC64 + kC64 + kClBars;
 }
 
 struct ClCtl {
-    uint32_t w0, h0, x0, stg;  // weight tile, h buffers, x buffers, h slice staging
+    uint32_t w0, h0, x0;  // weight tile, h buffers, x buffers
     uint64_t *wbar, *xfull, *xempty, *hready, *tfull, *tempty, *done;
     uint32_t *tmem_slot;
     volatile int *abort;
@@ -62,8 +62,7 @@ __device__ __forceinline__ ClCtl cl_carve(uint8_t *raw, int KC, int kcx, int NB,
     c.w0 = smem_u32(base);
     c.h0 = c.w0 + wb;
     c.x0 = c.h0 + hb;
-    c.stg = c.x0 + xb;
-    uint64_t *bars = (uint64_t *)(base + wb + hb + xb + 2 * kSlice);
+    uint64_t *bars = (uint64_t *)(base + wb + hb + xb);
     c.wbar = bars;
     c.xfull = bars + 2;
     c.xempty = bars + 4;
@@ -98,6 +97,18 @@ __device__ __forceinline__ void bulk_s2c(uint32_t dst, uint32_t src, uint32_t by
                  "r"(src), "r"(bytes), "r"(bar)
                  : "memory");
 }
+// Bulk copy of `bytes` from global memory into the same shared-memory offset of every CTA
+// of cta_mask, completing on the mbarrier at the same offset in each.
+__device__ __forceinline__ void bulk_g2s_mc(uint32_t dst, const void *src, uint32_t bytes, uint64_t *bar,
+                                            uint16_t cta_mask)
+{
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.multicast::cluster [%0], [%1], %2, [%3], "
+        "%4;" ::"r"(dst),
+        "l"(src), "r"(bytes), "r"(smem_u32(bar)), "h"(cta_mask)
+        : "memory");
+}
+
 // Bounded wait (as tc::mbar_wait) with cluster-scope acquire: the phase was completed by
 // release arrivals of other CTAs of the cluster, after their distributed-shared-memory stores.
 __device__ __forceinline__ bool mbar_wait_cluster(uint64_t *bar, uint32_t parity, long long limit, volatile int *abort)
@@ -139,25 +150,24 @@ __device__ __forceinline__ uint64_t slice_desc(uint32_t addr)
 // byte offset of 16-byte piece k (units 8k .. 8k + 7) of row r in an h slice
 __host__ __device__ constexpr uint32_t slice_off(uint32_t r, uint32_t k) { return (r >> 3) * 256 + k * 128 + (r & 7) * 16; }
 
-// Stages this thread's row of h_read(t + 1) (16 units, zero past H or B) as slice buffer
-// `buf`, then (once every epilogue warp has) lane r of warp 0 copies the slice into CTA r's
-// h buffer `buf` at this CTA's slice position, completing on that CTA's hready[buf].
-__device__ __forceinline__ void deliver_slice(const ClCtl &c, int buf, int row, const uint4 (&v)[2], bool valid0,
-                                              bool valid1, uint32_t ct, uint32_t n_ct, int tid)
+// Writes this thread's row of h_read(s) (16 units, zero past H or B) into its global slice
+// block `blk` (2 KB, the slice layout), then (once every epilogue warp has) one multicast
+// bulk copy loads the block into every CTA's h buffer `buf` at this CTA's slice position,
+// completing on that CTA's hready[buf]: one L2 read delivered to all CTAs.
+__device__ __forceinline__ void deliver_slice(const ClCtl &c, uint8_t *blk, int buf, int row, const uint4 (&v)[2],
+                                              bool valid0, bool valid1, uint32_t ct, uint32_t n_ct, int tid)
 {
     if (row < 64) {
         const uint4 z = make_uint4(0u, 0u, 0u, 0u);
-        const uint4 a0 = valid0 ? v[0] : z, a1 = valid1 ? v[1] : z;
-        tc::st_shared_v4(c.stg + buf * kSlice + slice_off((uint32_t)row, 0), (const uint32_t *)&a0);
-        tc::st_shared_v4(c.stg + buf * kSlice + slice_off((uint32_t)row, 1), (const uint32_t *)&a1);
+        *(uint4 *)(blk + slice_off((uint32_t)row, 0)) = valid0 ? v[0] : z;
+        *(uint4 *)(blk + slice_off((uint32_t)row, 1)) = valid1 ? v[1] : z;
     }
-    tc::fence_proxy_async();  // generic writes -> the bulk copies
+    tc::fence_proxy_async_global();  // this thread's block stores -> the bulk copy
     __syncwarp();
     tc::bar_sync(2, 4 * 32);
-    if (tid < (int)n_ct) {  // lane r of warp 0 copies to CTA r (all at once)
-        const uint32_t dst = c.h0 + (uint32_t)(buf * n_ct + ct) * kSlice, bar = smem_u32(&c.hready[buf]);
-        bulk_s2c(peer_addr(dst, (uint32_t)tid), c.stg + buf * kSlice, kSlice, peer_addr(bar, (uint32_t)tid));
-    }
+    if (tid == 0)
+        bulk_g2s_mc(c.h0 + (uint32_t)(buf * n_ct + ct) * kSlice, blk, kSlice, &c.hready[buf],
+                    (uint16_t)((1u << n_ct) - 1));
 }
 
 template <int U>
@@ -293,7 +303,7 @@ __global__ void __launch_bounds__(192, 1) step_cl(const __grid_constant__ CUtens
                 h0v[i] = __ldcg((const uint4 *)(a.hr + (size_t)row * H + u0 + 8 * i));  // h_read(0)
             }
         }
-        deliver_slice(c, 0, row, h0v, v0, v1, ct, n_ct, tid);
+        deliver_slice(c, p.gscr + (size_t)ct * kSlice, 0, row, h0v, v0, v1, ct, n_ct, tid);
         for (int t = 0; t < T; ++t) {
             const int b = t & 1;
             // the next step's operands that rows written before this step hold: issued now,
@@ -349,7 +359,9 @@ __global__ void __launch_bounds__(192, 1) step_cl(const __grid_constant__ CUtens
                 hb[i] = pack8_bf16(*(const float(*)[8])(hn + 8 * i));
                 hop[i] = is_new ? hb[i] : hold[i];
             }
-            if (t + 1 < T) deliver_slice(c, (t + 1) & 1, row, hop, v0, v1, ct, n_ct, tid);
+            if (t + 1 < T)
+                deliver_slice(c, p.gscr + ((size_t)(t + 1) * n_ct + ct) * kSlice, (t + 1) & 1, row, hop, v0, v1, ct, n_ct,
+                              tid);
             if (v0) {
                 // history row t + 1, the h operand row t + 1 (for the weight gradient), the gates
                 const size_t w = ((size_t)(t + 1) * B + row) * H + u0;
@@ -461,18 +473,6 @@ __global__ void pack_bwd_slices(const __nv_bfloat16 *__restrict__ W, int I, int 
 }
 
 namespace {
-// Bulk copy of `bytes` from global memory into the same shared-memory offset of every CTA
-// of cta_mask, completing on the mbarrier at the same offset in each.
-__device__ __forceinline__ void bulk_g2s_mc(uint32_t dst, const void *src, uint32_t bytes, uint64_t *bar,
-                                            uint16_t cta_mask)
-{
-    asm volatile(
-        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.multicast::cluster [%0], [%1], %2, [%3], "
-        "%4;" ::"r"(dst),
-        "l"(src), "r"(bytes), "r"(smem_u32(bar)), "h"(cta_mask)
-        : "memory");
-}
-
 // This thread's row of a dG block (4 gates x 16 units, zero past H or B) into the swizzled
 // global block `blk` (64 rows x 128 bytes).
 __device__ __forceinline__ void store_dg_block(uint8_t *blk, int row, const uint4 (&v)[4][2], bool v0, bool v1)
@@ -773,6 +773,7 @@ cudaError_t bf16_launch_fwd_cluster(stacklstm *s, const StepArgs &a, const CUten
     ClArgs p{};
     p.s = a;
     p.n_ct = pl.n_ct;
+    p.gscr = (uint8_t *)s->g_fcl;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(pl.n_ct);
     cfg.blockDim = dim3(pl.threads);
@@ -837,6 +838,7 @@ bool bf16_plan_bwd_cluster(stacklstm *s, PersistPlan *pl)
     return true;
 }
 
+size_t bf16_fwd_cluster_block_bytes(int T, int H) { return (size_t)T * ceil_div(H, kClU) * kSlice; }
 size_t bf16_bwd_cluster_block_bytes(int T, int H) { return (size_t)T * ceil_div(H, kClU) * kGBlock; }
 
 size_t bf16_bwd_cluster_weight_bytes(int H)

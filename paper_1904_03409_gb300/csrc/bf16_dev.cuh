@@ -179,6 +179,7 @@ size_t bf16_bwd_cluster_weight_bytes(int H);
 cudaError_t bf16_pack_bwd_cluster(stacklstm *s, const __nv_bfloat16 *W, __nv_bfloat16 *out);
 cudaError_t bf16_launch_bwd_cluster(stacklstm *s, const StepArgs &a);
 size_t bf16_bwd_cluster_block_bytes(int T, int H);
+size_t bf16_fwd_cluster_block_bytes(int T, int H);
 cudaError_t bf16_launch_fwd_persist(stacklstm *s, const StepArgs &a, const CUtensorMap &tm_x, const CUtensorMap &tm_h,
                                     const CUtensorMap &tm_gates, const CUtensorMap &tm_hh,
                                     const CUtensorMap &tm_hc);

@@ -612,6 +612,10 @@ cudaError_t bf16_prepare(stacklstm *s)
     s->allocs.push_back(p); s->w_bwd = p;
     if ((e = cudaMalloc(&p, dx_bytes))) return e;
     s->allocs.push_back(p); s->w_dx = p;
+    if (s->fc.on) {
+        if ((e = cudaMalloc(&p, bf16_fwd_cluster_block_bytes(T, H)))) return e;
+        s->allocs.push_back(p); s->g_fcl = p;
+    }
     if (s->bc.on) {
         if ((e = cudaMalloc(&p, bf16_bwd_cluster_weight_bytes(H)))) return e;
         s->allocs.push_back(p); s->w_bcl = p;

@@ -81,6 +81,7 @@ struct stacklstm {
     // persistent step kernels (one launch for all T steps; bf16_persist.cu)
     PersistPlan pf, pb;            // forward, backward (on = 0: one launch per step)
     PersistPlan fc;                // forward as one thread-block cluster (one row tile; bf16_cluster.cu)
+    void *g_fcl = nullptr;         // its h slice blocks [T][column tiles][2 KB]
     PersistPlan bc;                // backward as one thread-block cluster (one row tile; bf16_cluster.cu)
     void *w_bcl = nullptr;         // its weight chunks
     void *g_bcl = nullptr;         // its swizzled dG blocks [T][column tiles][8 KB]
