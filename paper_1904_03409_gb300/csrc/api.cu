@@ -196,7 +196,7 @@ sl_status stacklstm_create(stacklstm_t *out, int T, int B, int I, int H, sl_dtyp
     const size_t es = elem_size(dtype);
     bool ok = alloc(s, &s->p_traj, T1B * 4) && alloc(s, &s->top, T1B * 4) && alloc(s, &s->slot_last, T1B * 4) &&
               alloc(s, &s->err, 16) && alloc(s, &s->hist_h, T1B * H * es) && alloc(s, &s->hr, dtype == SL_BF16 ? T1B * H * 2 : 16) && alloc(s, &s->hist_c, T1B * H * 4) &&
-              alloc(s, &s->gates, TB * G * (dtype == SL_BF16 ? 2 : 4)) && alloc(s, &s->a_rm, dtype == SL_FP32 ? TB * K * es : 16) &&
+              alloc(s, &s->gates, dtype == SL_BF16 ? TB * 4 * (((size_t)H + 15) / 16 * 16) * 2 : TB * G * 4) && alloc(s, &s->a_rm, dtype == SL_FP32 ? TB * K * es : 16) &&
               alloc(s, &s->dhist_h, T1B * H * 4) && alloc(s, &s->dhist_c, T1B * H * 4) &&
               alloc(s, &s->dG, TB * G * es);
     if (ok && dtype == SL_FP32) ok = alloc(s, &s->w_fwd, K * G * 4);

@@ -81,22 +81,6 @@ __device__ __forceinline__ void cl_abort(const ClCtl &c, int32_t *err)
     atomicCAS(err, 0, (int)SL_ERR_TIMEOUT);
 }
 
-// The address of a shared-memory location of this CTA in the window of cluster CTA `rank`.
-__device__ __forceinline__ uint32_t peer_addr(uint32_t local, uint32_t rank)
-{
-    uint32_t r;
-    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(local), "r"(rank));
-    return r;
-}
-// Bulk copy of `bytes` from this CTA's shared memory into another CTA's (cluster address),
-// completing on the destination CTA's mbarrier (cluster address) by byte count.
-__device__ __forceinline__ void bulk_s2c(uint32_t dst, uint32_t src, uint32_t bytes, uint32_t bar)
-{
-    asm volatile("cp.async.bulk.shared::cluster.shared::cta.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
-                     dst),
-                 "r"(src), "r"(bytes), "r"(bar)
-                 : "memory");
-}
 // Bulk copy of `bytes` from global memory into the same shared-memory offset of every CTA
 // of cta_mask, completing on the mbarrier at the same offset in each.
 __device__ __forceinline__ void bulk_g2s_mc(uint32_t dst, const void *src, uint32_t bytes, uint64_t *bar,
@@ -296,7 +280,7 @@ __global__ void __launch_bounds__(192, 1) step_cl(const __grid_constant__ CUtens
             for (int i = 0; i < 2; ++i) {
                 if (i == 1 && !v1) break;
                 float v[8];
-                ld8f_cg(a.hist_c + ((size_t)s_cur * B + row) * H + u0 + 8 * i, v);
+                ld8f_a32(a.hist_c + ((size_t)s_cur * B + row) * H + u0 + 8 * i, v);
 #pragma unroll
                 for (int k = 0; k < 8; ++k) crv[8 * i + k] = v[k];
                 hold[i] = __ldcg((const uint4 *)(a.hr + ((size_t)s_nxt * B + row) * H + u0 + 8 * i));
@@ -319,7 +303,7 @@ __global__ void __launch_bounds__(192, 1) step_cl(const __grid_constant__ CUtens
                     if (i == 1 && !v1) break;
                     if (s_nxt != t + 1) {
                         float v[8];
-                        ld8f_cg(a.hist_c + ((size_t)s_nxt * B + row) * H + u0 + 8 * i, v);
+                        ld8f_a32(a.hist_c + ((size_t)s_nxt * B + row) * H + u0 + 8 * i, v);
 #pragma unroll
                         for (int k = 0; k < 8; ++k) cr_n[8 * i + k] = v[k];
                     }
@@ -365,16 +349,31 @@ __global__ void __launch_bounds__(192, 1) step_cl(const __grid_constant__ CUtens
             if (v0) {
                 // history row t + 1, the h operand row t + 1 (for the weight gradient), the gates
                 const size_t w = ((size_t)(t + 1) * B + row) * H + u0;
-                __half *gt = a.gates + ((size_t)t * B + row) * 4 * H + u0;
 #pragma unroll
                 for (int i = 0; i < 2; ++i) {
                     if (i == 1 && !v1) break;
                     *(uint4 *)(a.hist_h + w + 8 * i) = hb[i];
                     *(uint4 *)(a.hr + w + 8 * i) = hop[i];
-                    st8f(a.hist_c + w + 8 * i, *(const float(*)[8])(cn + 8 * i));
+                    st8f_a32(a.hist_c + w + 8 * i, *(const float(*)[8])(cn + 8 * i));
+                }
+                if (a.gates_blk) {
+                    // this CTA's 4 x 16 gates of the row: one 128-byte block, a 32-byte store a gate
+                    __half *gt = a.gates + (((size_t)t * B + row) * n_ct + ct) * 4 * U;
 #pragma unroll
-                    for (int g = 0; g < 4; ++g)
-                        *(uint4 *)(gt + (size_t)g * H + 8 * i) = pack8_f16(*(const float(*)[8])(gv[g] + 8 * i));
+                    for (int g = 0; g < 4; ++g) {
+                        const uint4 lo = pack8_f16(*(const float(*)[8])(gv[g])), hi = pack8_f16(*(const float(*)[8])(gv[g] + 8));
+                        const uint32_t q[8] = {lo.x, lo.y, lo.z, lo.w, hi.x, hi.y, hi.z, hi.w};
+                        st8u_a32(gt + g * U, q);
+                    }
+                } else {
+                    __half *gt = a.gates + ((size_t)t * B + row) * 4 * H + u0;
+#pragma unroll
+                    for (int i = 0; i < 2; ++i) {
+                        if (i == 1 && !v1) break;
+#pragma unroll
+                        for (int g = 0; g < 4; ++g)
+                            *(uint4 *)(gt + (size_t)g * H + 8 * i) = pack8_f16(*(const float(*)[8])(gv[g] + 8 * i));
+                    }
                 }
             }
             if (t + 1 < T) {
@@ -416,14 +415,16 @@ constexpr int kClU = 16;  // hidden units per CTA
 // K = 16 g + e for unit 16 j + e of gate g; the weights are packed to match (16 rows x 64,
 // 128-byte swizzled, per chunk). The dG buffer is single: before a CTA loads dG_{t-1} in,
 // every CTA's step-t MMAs have completed (their commits arrive on the `dfree` barrier of
-// every CTA of the cluster).
+// every CTA of the cluster). The MMAs are M = 64 (the row tile exactly): each reads 2 KB of
+// dG where an M = 128 one would read 4 KB, half of it padding, and the 52 or so MMAs of
+// N = 16 a step are bound by those operand reads.
 //
-// [weight chunks n_ct x 2 KB][dG buffer n_ct x 8 KB][8 KB pad][barriers]
+// [weight chunks n_ct x 2 KB][dG buffer n_ct x 8 KB][barriers]
 constexpr uint32_t kWChunkB = 16 * 128;  // one weight chunk: 16 rows x 64 K
 constexpr uint32_t kGBlock = 64 * 128;   // one CTA's dG block: 64 rows x 64 K
 __host__ __device__ constexpr uint32_t clb_smem_bytes(int n_ct)
 {
-    return 1024 + (uint32_t)n_ct * kWChunkB + (uint32_t)n_ct * kGBlock + kGBlock + kClBars;
+    return 1024 + (uint32_t)n_ct * kWChunkB + (uint32_t)n_ct * kGBlock + kClBars;
 }
 
 struct ClbCtl {
@@ -438,7 +439,7 @@ __device__ __forceinline__ ClbCtl clb_carve(uint8_t *raw, int n_ct)
     const uint32_t off = smem_u32(raw);
     uint8_t *base = raw + ((1024u - (off & 1023u)) & 1023u);
     ClbCtl c;
-    const uint32_t wb = (uint32_t)n_ct * kWChunkB, gb = (uint32_t)n_ct * kGBlock + kGBlock;
+    const uint32_t wb = (uint32_t)n_ct * kWChunkB, gb = (uint32_t)n_ct * kGBlock;
     c.w0 = smem_u32(base);
     c.g0 = c.w0 + wb;
     uint64_t *bars = (uint64_t *)(base + wb + gb);
@@ -475,15 +476,20 @@ __global__ void pack_bwd_slices(const __nv_bfloat16 *__restrict__ W, int I, int 
 namespace {
 // This thread's row of a dG block (4 gates x 16 units, zero past H or B) into the swizzled
 // global block `blk` (64 rows x 128 bytes).
+// The 16-byte pieces 2g and 2g + 1 of a row (gate g) land in one aligned 32-byte pair under
+// the 128-byte swizzle, in swapped order on odd rows: one 32-byte store a gate.
 __device__ __forceinline__ void store_dg_block(uint8_t *blk, int row, const uint4 (&v)[4][2], bool v0, bool v1)
 {
     if (row >= 64) return;
     const uint4 z = make_uint4(0u, 0u, 0u, 0u);
+    const bool odd = row & 1;
 #pragma unroll
-    for (int g = 0; g < 4; ++g)
-#pragma unroll
-        for (int i = 0; i < 2; ++i)
-            *(uint4 *)(blk + sw128((uint32_t)row, (uint32_t)(2 * g + i))) = (i == 0 ? v0 : v1) ? v[g][i] : z;
+    for (int g = 0; g < 4; ++g) {
+        const uint4 lo = v0 ? v[g][0] : z, hi = v1 ? v[g][1] : z;
+        const uint4 a = odd ? hi : lo, b = odd ? lo : hi;
+        const uint32_t w[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
+        st8u_a32(blk + (sw128((uint32_t)row, (uint32_t)(2 * g)) & ~31u), w);
+    }
 }
 
 // After every epilogue warp has stored its rows of the block: thread 0 waits until every
@@ -549,7 +555,7 @@ __global__ void __launch_bounds__(192, 1) step_clb(ClArgs p)
     } else if (warp == E + 1) {
         // ------------------------------------------------------------ MMA issue
         if (lane == 0) {
-            constexpr uint32_t idesc = tc::idesc_bf16(U);
+            constexpr uint32_t idesc = tc::idesc_bf16(U, 0, 0, 64);
             bool ok = tc::mbar_wait(c.wbar, 0, limit, c.abort);
             int k_g = -1;  // last step index whose dG had landed
             for (int k = 0; k < T && ok && !*c.abort; ++k) {  // step t = T - 1 - k
@@ -582,9 +588,10 @@ __global__ void __launch_bounds__(192, 1) step_clb(ClArgs p)
         __syncwarp();
     } else {
         // ------------------------------------------------------------ epilogue
-        const int row = warp * 32 + lane;
+        // M = 64 accumulator: rows 16 w .. 16 w + 15 in lanes 0..15 of TMEM lane quadrant w
+        const int row = lane < 16 ? warp * 16 + lane : 64;  // lanes 16..31 hold no row
         const bool row_ok = row < B;
-        const bool warp_rows = warp * 32 < B;
+        const bool warp_rows = warp * 16 < B;
         const int u0 = (int)ct * U;
         const bool v0 = row_ok && u0 < H, v1 = row_ok && u0 + 8 < H;  // the two 8-unit groups (H % 8 == 0)
         const uint32_t taddr0 = tmem + ((uint32_t)(warp * 32) << 16);
@@ -623,19 +630,31 @@ __global__ void __launch_bounds__(192, 1) step_clb(ClArgs p)
                 for (int i = 0; i < 2; ++i) {
                     if (i == 1 && !v1) break;
                     const size_t us = ((size_t)src * B + row) * H + u0 + 8 * i;
-                    ld8f_cg(a.dhist_h + us, *(float(*)[8])(dh_src + 8 * i));
+                    ld8f_a32(a.dhist_h + us, *(float(*)[8])(dh_src + 8 * i));
                     if (t >= 1) {
                         const size_t wr = ((size_t)t * B + row) * H + u0 + 8 * i, rd = ((size_t)s1 * B + row) * H + u0 + 8 * i;
-                        ld8f_cg(a.dhist_h + wr, *(float(*)[8])(dh_t + 8 * i));
-                        ld8f_cg(a.dhist_c + wr, *(float(*)[8])(dc_t + 8 * i));
-                        ld8f_cg(a.hist_c + wr, *(float(*)[8])(cn + 8 * i));
-                        ld8f_cg(a.hist_c + rd, *(float(*)[8])(cr + 8 * i));
-                        ld8f_cg(a.dhist_c + rd, *(float(*)[8])(dc_rd + 8 * i));
-                        const __half *gt = a.gates + ((size_t)(t - 1) * B + row) * 4 * H + u0 + 8 * i;
+                        ld8f_a32(a.dhist_h + wr, *(float(*)[8])(dh_t + 8 * i));
+                        ld8f_a32(a.dhist_c + wr, *(float(*)[8])(dc_t + 8 * i));
+                        ld8f_a32(a.hist_c + wr, *(float(*)[8])(cn + 8 * i));
+                        ld8f_a32(a.hist_c + rd, *(float(*)[8])(cr + 8 * i));
+                        ld8f_a32(a.dhist_c + rd, *(float(*)[8])(dc_rd + 8 * i));
+                        if (!a.gates_blk) {
+                            const __half *gt = a.gates + ((size_t)(t - 1) * B + row) * 4 * H + u0 + 8 * i;
 #pragma unroll
-                        for (int g = 0; g < 4; ++g) gq[g][i] = __ldcg((const uint4 *)(gt + (size_t)g * H));
+                            for (int g = 0; g < 4; ++g) gq[g][i] = __ldcg((const uint4 *)(gt + (size_t)g * H));
+                        }
                     }
                 }
+            if (v0 && t >= 1 && a.gates_blk) {
+                const __half *gt = a.gates + (((size_t)(t - 1) * B + row) * n_ct + ct) * 4 * U;
+#pragma unroll
+                for (int g = 0; g < 4; ++g) {
+                    uint32_t q[8];
+                    ld8u_a32(gt + g * U, q);
+                    gq[g][0] = make_uint4(q[0], q[1], q[2], q[3]);
+                    gq[g][1] = make_uint4(q[4], q[5], q[6], q[7]);
+                }
+            }
             const bool ok = tc::mbar_wait(&c.tfull[acc], (k >> 1) & 1, limit, c.abort);
             if (!ok) {
                 *c.abort = 1;
@@ -684,7 +703,11 @@ __global__ void __launch_bounds__(192, 1) step_clb(ClArgs p)
                 for (int g = 0; g < 4; ++g)
 #pragma unroll
                     for (int i = 0; i < 2; ++i) dg[g][i] = pack8_bf16(*(const float(*)[8])(d[g] + 8 * i));
-                // dG_{t-1} to global memory, then (multicast bulk copy of its block) to every CTA
+                // dG_{t-1}: its block to global memory, then (multicast bulk copy) to every CTA
+                uint8_t *blk = p.gscr + ((size_t)(t - 1) * n_ct + ct) * kGBlock;
+                store_dg_block(blk, row, dg, v0, v1);
+                deliver_dg(c, blk, k & 1, ct, n_ct, tid, limit, a.err);
+                // and in the [T B][4H] layout (for the input and weight gradients), after the delivery
                 if (v0)
 #pragma unroll
                     for (int i = 0; i < 2; ++i) {
@@ -693,16 +716,13 @@ __global__ void __launch_bounds__(192, 1) step_clb(ClArgs p)
 #pragma unroll
                         for (int g = 0; g < 4; ++g) *(uint4 *)(gp + (size_t)g * H) = dg[g][i];
                     }
-                uint8_t *blk = p.gscr + ((size_t)(t - 1) * n_ct + ct) * kGBlock;
-                store_dg_block(blk, row, dg, v0, v1);
-                deliver_dg(c, blk, k & 1, ct, n_ct, tid, limit, a.err);
             }
             if (v0)
 #pragma unroll
                 for (int i = 0; i < 2; ++i) {
                     if (i == 1 && !v1) break;
-                    st8f(a.dhist_h + ((size_t)src * B + row) * H + u0 + 8 * i, *(const float(*)[8])(v + 8 * i));
-                    if (t >= 1) st8f(a.dhist_c + ((size_t)s1 * B + row) * H + u0 + 8 * i, *(const float(*)[8])(dcr + 8 * i));
+                    st8f_a32(a.dhist_h + ((size_t)src * B + row) * H + u0 + 8 * i, *(const float(*)[8])(v + 8 * i));
+                    if (t >= 1) st8f_a32(a.dhist_c + ((size_t)s1 * B + row) * H + u0 + 8 * i, *(const float(*)[8])(dcr + 8 * i));
                 }
             src = src_n;
             s1 = s1_n;
@@ -772,6 +792,7 @@ cudaError_t bf16_launch_fwd_cluster(stacklstm *s, const StepArgs &a, const CUten
     const PersistPlan &pl = s->fc;
     ClArgs p{};
     p.s = a;
+    p.s.gates_blk = s->bc.on;  // the cluster backward (and its last-step pointwise) reads the blocked layout
     p.n_ct = pl.n_ct;
     p.gscr = (uint8_t *)s->g_fcl;
     cudaLaunchConfig_t cfg = {};
@@ -861,6 +882,7 @@ cudaError_t bf16_launch_bwd_cluster(stacklstm *s, const StepArgs &a)
     const PersistPlan &pl = s->bc;
     ClArgs p{};
     p.s = a;
+    p.s.gates_blk = s->fc.on;  // the cluster forward wrote the blocked layout
     p.n_ct = pl.n_ct;
     p.gscr = (uint8_t *)s->g_bcl;
     cudaLaunchConfig_t cfg = {};

@@ -63,6 +63,34 @@ __device__ __forceinline__ void st8f(float *p, const float (&v)[8])
     *(float4 *)p = make_float4(v[0], v[1], v[2], v[3]);
     *(float4 *)(p + 4) = make_float4(v[4], v[5], v[6], v[7]);
 }
+// The same as one 32-byte access: p must be 32-byte aligned (the fp32 history rows, whose
+// length H is a multiple of 8, at a multiple of 8 units).
+__device__ __forceinline__ void ld8f_a32(const float *p, float (&v)[8])
+{
+    asm volatile("ld.global.cg.v8.f32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
+                 : "=f"(v[0]), "=f"(v[1]), "=f"(v[2]), "=f"(v[3]), "=f"(v[4]), "=f"(v[5]), "=f"(v[6]), "=f"(v[7])
+                 : "l"(p)
+                 : "memory");
+}
+__device__ __forceinline__ void ld8u_a32(const void *p, uint32_t (&w)[8])
+{
+    asm volatile("ld.global.cg.v8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
+                 : "=r"(w[0]), "=r"(w[1]), "=r"(w[2]), "=r"(w[3]), "=r"(w[4]), "=r"(w[5]), "=r"(w[6]), "=r"(w[7])
+                 : "l"(p)
+                 : "memory");
+}
+__device__ __forceinline__ void st8u_a32(void *p, const uint32_t (&w)[8])
+{
+    asm volatile("st.global.v8.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8};" ::"l"(p), "r"(w[0]), "r"(w[1]), "r"(w[2]),
+                 "r"(w[3]), "r"(w[4]), "r"(w[5]), "r"(w[6]), "r"(w[7])
+                 : "memory");
+}
+__device__ __forceinline__ void st8f_a32(float *p, const float (&v)[8])
+{
+    asm volatile("st.global.v8.f32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8};" ::"l"(p), "f"(v[0]), "f"(v[1]), "f"(v[2]),
+                 "f"(v[3]), "f"(v[4]), "f"(v[5]), "f"(v[6]), "f"(v[7])
+                 : "memory");
+}
 __device__ __forceinline__ uint4 pack8_bf16(const float (&v)[8])
 {
     uint4 o;
@@ -102,7 +130,8 @@ struct StepArgs {
     __nv_bfloat16 *hist_h;      // [T+1][B][H]
     __nv_bfloat16 *hr;          // [T+1][B][H] h operand of each step
     float *hist_c;              // [T+1][B][H]
-    __half *gates;              // [T][B][4H]
+    __half *gates;              // [T][B][4H], or (gates_blk) [T][B][H / 16][4][16]
+    int gates_blk;              // the blocked gate layout (the cluster forward and backward pair)
     const float *bias;          // [4H]
     const uint8_t *wpack;       // packed B-operand tiles of this kernel
     float *dhist_h, *dhist_c;   // [T+1][B][H]

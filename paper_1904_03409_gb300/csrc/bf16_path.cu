@@ -252,11 +252,14 @@ __device__ __forceinline__ void pointwise8(const StepArgs &a, int tp, int b, int
     ld8f_cg(a.dhist_c + wr, dcn);
     ld8f_cg(a.hist_c + wr, cn);
     ld8f_cg(a.hist_c + rd, cr);
-    const __half *gt = a.gates + ((size_t)tp * B + b) * 4 * H + u;
+    // gate g of unit u: row-major [T][B][4H], or blocked [T][B][H / 16][4][16]
+    const size_t gs = a.gates_blk ? 16 : (size_t)H;
+    const __half *gt = a.gates_blk ? a.gates + (((size_t)tp * B + b) * ((H + 15) / 16) + u / 16) * 64 + u % 16
+                                   : a.gates + ((size_t)tp * B + b) * 4 * H + u;
     unpack8_f16(*(const uint4 *)(gt), ig);
-    unpack8_f16(*(const uint4 *)(gt + H), fg);
-    unpack8_f16(*(const uint4 *)(gt + 2 * (size_t)H), gg);
-    unpack8_f16(*(const uint4 *)(gt + 3 * (size_t)H), og);
+    unpack8_f16(*(const uint4 *)(gt + gs), fg);
+    unpack8_f16(*(const uint4 *)(gt + 2 * gs), gg);
+    unpack8_f16(*(const uint4 *)(gt + 3 * gs), og);
     float d[4][8], dcr[8];
 #pragma unroll
     for (int e = 0; e < 8; ++e) {
@@ -529,7 +532,7 @@ StepArgs step_args(stacklstm *s, const float *bias, const void *wpack, int kcx, 
     a.kcx = kcx; a.KC = KC; a.S = S;
     a.top = s->top;
     a.hist_h = (__nv_bfloat16 *)s->hist_h; a.hr = (__nv_bfloat16 *)s->hr;
-    a.hist_c = s->hist_c; a.gates = (__half *)s->gates;
+    a.hist_c = s->hist_c; a.gates = (__half *)s->gates; a.gates_blk = 0;
     a.bias = bias; a.wpack = (const uint8_t *)wpack;
     a.dhist_h = s->dhist_h; a.dhist_c = s->dhist_c; a.dG = (__nv_bfloat16 *)s->dG;
     a.limit = s->wait_limit; a.err = s->err;
@@ -712,7 +715,8 @@ cudaError_t bf16_forward_steps(stacklstm *s, const float *bias)
 // Pointwise backward of the last step, before the reverse loop.
 cudaError_t bf16_backward_setup(stacklstm *s)
 {
-    const StepArgs a = step_args(s, nullptr, s->w_bwd, 0, s->kcb, s->sb);
+    StepArgs a = step_args(s, nullptr, s->w_bwd, 0, s->kcb, s->sb);
+    a.gates_blk = s->fc.on && s->bc.on;  // the layout the cluster forward wrote for the cluster backward
     pointwise_last<<<grid_for(s, (size_t)s->B * (s->H / 8)), 256, 0, s->stream>>>(a);
     s->launches += 1;
     return cudaGetLastError();

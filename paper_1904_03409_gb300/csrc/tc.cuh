@@ -261,12 +261,11 @@ __device__ __forceinline__ uint64_t smem_desc(uint32_t addr, uint32_t lbo_bytes,
            ((uint64_t)((sbo_bytes >> 4) & 0x3FFFu) << 32) | ((uint64_t)1 << 46) | (kSwizzle128B << 61);
 }
 
-// Instruction descriptor, kind::f16: D fp32, A and B bf16, M = 128, N given;
+// Instruction descriptor, kind::f16: D fp32, A and B bf16, M (64 or 128) and N given;
 // a_mn / b_mn select MN-major (1) instead of K-major (0) operands.
-__host__ __device__ constexpr uint32_t idesc_bf16(uint32_t N, uint32_t a_mn = 0, uint32_t b_mn = 0)
+__host__ __device__ constexpr uint32_t idesc_bf16(uint32_t N, uint32_t a_mn = 0, uint32_t b_mn = 0, uint32_t M = 128)
 {
-    return (1u << 4) | (1u << 7) | (1u << 10) | (a_mn << 15) | (b_mn << 16) | ((N >> 3) << 17) |
-           ((128u >> 4) << 24);
+    return (1u << 4) | (1u << 7) | (1u << 10) | (a_mn << 15) | (b_mn << 16) | ((N >> 3) << 17) | ((M >> 4) << 24);
 }
 
 // D[tmem] (+)= A[smem] * B[smem]^T, issued by one thread.

@@ -235,3 +235,9 @@ def test_cluster_kernels_for_one_row_tile_match_oracle(T, B, I, H, seed):
     plan_p, per = run_nan_filled(w, {"STACKLSTM_BWD_CLUSTER": "0", "STACKLSTM_FWD_CLUSTER": "0"})
     assert "forward persistent" in plan_p and "backward persistent" in plan_p, plan_p
     compare(per, ref, "bf16")
+    # one cluster kernel beside a persistent one: the saved gates keep the row-major layout
+    for env, want in (({"STACKLSTM_BWD_CLUSTER": "0"}, ("forward cluster", "backward persistent")),
+                      ({"STACKLSTM_FWD_CLUSTER": "0"}, ("forward persistent", "backward cluster"))):
+        plan_m, mixed = run_nan_filled(w, env)
+        assert all(x in plan_m for x in want), plan_m
+        compare(mixed, ref, "bf16")
