@@ -9,15 +9,15 @@
 // the gates are still written to global memory for the backward.
 //
 // Warp roles (192 threads): warps 0..3 epilogue (TMEM lane quadrant w, one instance row
-// per thread; rows >= B idle), warp 4 producer (weight tile once; x_t chunks by TMA into a
+// per thread of lanes 0..15; rows >= B idle), warp 4 producer (weight tile once; x_t chunks by TMA into a
 // two-step buffer), warp 5 MMA (x part of step t as soon as x_t lands, then the h part once
 // every slice of h_read(t) has landed; two TMEM accumulators by step parity).
 //
 // x_t chunks are 64-row, 128-byte-swizzled 8 KB tiles; an h slice is 16 units x 64 rows in
 // the unswizzled K-major core-matrix layout ([row / 8][unit / 8][row mod 8][unit mod 8],
-// 2 KB), one K = 16 MMA step. The M = 128 MMAs read 128 rows, so rows 64..127 come from
-// whatever follows (the next tile or slice, or a pad after the last one) and only feed
-// accumulator rows that are never stored.
+// 2 KB), one K = 16 MMA step. The MMAs are M = 64, the row tile exactly: accumulator rows
+// 16 w .. 16 w + 15 sit in lanes 0..15 of TMEM lane quadrant w, so each epilogue warp
+// takes 16 rows.
 #include <stdio.h>
 
 #include <algorithm>
@@ -37,13 +37,13 @@ struct ClArgs {
     uint8_t *gscr;  // backward: [T][n_ct] swizzled 8 KB dG blocks
 };
 
-// [weight tile KC x NB x 128][h buffers 2 x n_ct x 2 KB][2 KB pad][x buffers 2 x kcx x 8 KB]
-// [8 KB pad][barriers], based at the first 1024-byte boundary
+// [weight tile KC x NB x 128][h buffers 2 x n_ct x 2 KB][x buffers 2 x kcx x 8 KB][barriers],
+// based at the first 1024-byte boundary
 constexpr uint32_t kSlice = 2048;
 constexpr uint32_t kClBars = 16 * 8 + 16;
 __host__ __device__ constexpr uint32_t cl_smem_bytes(int KC, int kcx, int NB, int n_ct)
 {
-    return 1024 + (uint32_t)KC * NB * 128 + (2u * n_ct + 1) * kSlice + 2u * kcx * kC64 + kC64 + kClBars;
+    return 1024 + (uint32_t)KC * NB * 128 + 2u * n_ct * kSlice + 2u * kcx * kC64 + kClBars;
 }
 
 struct ClCtl {
@@ -58,7 +58,7 @@ __device__ __forceinline__ ClCtl cl_carve(uint8_t *raw, int KC, int kcx, int NB,
     const uint32_t off = smem_u32(raw);
     uint8_t *base = raw + ((1024u - (off & 1023u)) & 1023u);
     ClCtl c;
-    const uint32_t wb = (uint32_t)KC * NB * 128, hb = (2u * n_ct + 1) * kSlice, xb = 2u * kcx * kC64 + kC64;
+    const uint32_t wb = (uint32_t)KC * NB * 128, hb = 2u * n_ct * kSlice, xb = 2u * kcx * kC64;
     c.w0 = smem_u32(base);
     c.h0 = c.w0 + wb;
     c.x0 = c.h0 + hb;
@@ -117,7 +117,7 @@ __device__ __forceinline__ bool mbar_wait_cluster(uint64_t *bar, uint32_t parity
 template <int NB>
 __device__ __forceinline__ void cl_mma_chunk(uint32_t d, uint32_t a, uint32_t b, bool first)
 {
-    constexpr uint32_t idesc = tc::idesc_bf16(NB);
+    constexpr uint32_t idesc = tc::idesc_bf16(NB, 0, 0, 64);
 #pragma unroll
     for (int k = 0; k < kChunk / 16; ++k)
         tc::mma_bf16(d, tc::smem_desc(a + k * 32, 16, 1024), tc::smem_desc(b + k * 32, 16, 1024), idesc,
@@ -222,7 +222,7 @@ __global__ void __launch_bounds__(192, 1) step_cl(const __grid_constant__ CUtens
     } else if (warp == E + 1) {
         // ------------------------------------------------------------ MMA issue
         if (lane == 0) {
-            constexpr uint32_t idesc = tc::idesc_bf16(NB);
+            constexpr uint32_t idesc = tc::idesc_bf16(NB, 0, 0, 64);
             bool ok = tc::mbar_wait(c.wbar, 0, limit, c.abort);
             int t_h = -1;  // last step whose h slices all landed
             for (int t = 0; t < T && ok && !*c.abort; ++t) {
@@ -259,9 +259,10 @@ __global__ void __launch_bounds__(192, 1) step_cl(const __grid_constant__ CUtens
         __syncwarp();
     } else {
         // ------------------------------------------------------------ epilogue
-        const int row = warp * 32 + lane;
+        // M = 64 accumulator: rows 16 w .. 16 w + 15 in lanes 0..15 of TMEM lane quadrant w
+        const int row = lane < 16 ? warp * 16 + lane : 64;  // lanes 16..31 hold no row
         const bool row_ok = row < B;
-        const bool warp_rows = warp * 32 < B;
+        const bool warp_rows = warp * 16 < B;
         const int u0 = (int)ct * U;
         const bool v0 = row_ok && u0 < H, v1 = row_ok && u0 + 8 < H;  // the two 8-unit groups (H % 8 == 0)
         const uint32_t taddr0 = tmem + ((uint32_t)(warp * 32) << 16);
