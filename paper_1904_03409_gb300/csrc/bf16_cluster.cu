@@ -416,9 +416,9 @@ constexpr int kClU = 16;  // hidden units per CTA
 // K = 16 g + e for unit 16 j + e of gate g; the weights are packed to match (16 rows x 64,
 // 128-byte swizzled, per chunk). The dG buffer is single: before a CTA loads dG_{t-1} in,
 // every CTA's step-t MMAs have completed (their commits arrive on the `dfree` barrier of
-// every CTA of the cluster). The MMAs are M = 64 (the row tile exactly): each reads 2 KB of
-// dG where an M = 128 one would read 4 KB, half of it padding, and the 52 or so MMAs of
-// N = 16 a step are bound by those operand reads.
+// every CTA of the cluster). The MMAs are M = 64 (the row tile exactly). The 52 or so
+// N = 16 MMAs of a step are bound by their issue, so two threads (warps 4 and 5) issue
+// them, each into its own accumulator.
 //
 // [weight chunks n_ct x 2 KB][dG buffer n_ct x 8 KB][barriers]
 constexpr uint32_t kWChunkB = 16 * 128;  // one weight chunk: 16 rows x 64 K
@@ -516,7 +516,7 @@ template <int U>
 __global__ void __launch_bounds__(192, 1) step_clb(ClArgs p)
 {
     static_assert(U == 16, "four 16-unit gate slices per CTA");
-    constexpr uint32_t kCols = TmemCols<U>::value;
+    constexpr uint32_t kCols = TmemCols<2 * U>::value;  // one accumulator per MMA issuer
     constexpr int E = 4;
     const StepArgs &a = p.s;
     extern __shared__ uint8_t smem_raw[];
@@ -528,12 +528,12 @@ __global__ void __launch_bounds__(192, 1) step_clb(ClArgs p)
     if (tid == 0) {
         tc::mbar_init(c.wbar, 1);
         tc::mbar_init(c.gready, 1);
-        tc::mbar_init(c.dfree, n_ct);
+        tc::mbar_init(c.dfree, 2 * n_ct);  // both issuers' commits of every CTA
         for (int i = 0; i < 2; ++i) {
-            tc::mbar_init(&c.tfull[i], 1);
+            tc::mbar_init(&c.tfull[i], 2);
             tc::mbar_init(&c.tempty[i], E);
         }
-        tc::mbar_init(c.done, 1);
+        tc::mbar_init(c.done, 2);
         *c.abort = 0;
         tc::fence_mbar_init();
         tc::mbar_arrive_expect_tx(c.gready, n_ct * kGBlock);  // dG of step T - 1
@@ -545,18 +545,20 @@ __global__ void __launch_bounds__(192, 1) step_clb(ClArgs p)
     tc::tc_fence_after();
     const uint32_t tmem = *c.tmem_slot;
 
-    if (warp == E) {
-        // ------------------------------------------------------------ weight slices, once
-        if (lane == 0) {
-            const uint32_t wbytes = n_ct * kWChunkB;
-            tc::mbar_arrive_expect_tx(c.wbar, wbytes);
-            tc::bulk_g2s(c.w0, a.wpack + (size_t)ct * wbytes, wbytes, c.wbar);
-        }
-        __syncwarp();
-    } else if (warp == E + 1) {
-        // ------------------------------------------------------------ MMA issue
+    if (warp == E || warp == E + 1) {
+        // ------------------------------------------------------------ MMA issue, two issuers
+        // One thread issues an M = 64, N = 16 MMA about every 45 cycles; two issue about
+        // every 30 between them. Issuer q takes the K = 16 steps 2q and 2q + 1 of every
+        // chunk into its own accumulator (the epilogue adds the two); issuer 0 also posts
+        // each step's expected dG bytes and drains, issuer 1 first loads the weights.
+        const int q = warp == E + 1 ? 0 : 1;
         if (lane == 0) {
             constexpr uint32_t idesc = tc::idesc_bf16(U, 0, 0, 64);
+            if (q == 1) {
+                const uint32_t wbytes = n_ct * kWChunkB;
+                tc::mbar_arrive_expect_tx(c.wbar, wbytes);
+                tc::bulk_g2s(c.w0, a.wpack + (size_t)ct * wbytes, wbytes, c.wbar);
+            }
             bool ok = tc::mbar_wait(c.wbar, 0, limit, c.abort);
             int k_g = -1;  // last step index whose dG had landed
             for (int k = 0; k < T && ok && !*c.abort; ++k) {  // step t = T - 1 - k
@@ -564,14 +566,18 @@ __global__ void __launch_bounds__(192, 1) step_clb(ClArgs p)
                 if (k >= 2 && !(ok = tc::mbar_wait(&c.tempty[acc], ((k >> 1) - 1) & 1, limit, c.abort))) break;
                 if (!(ok = mbar_wait_cluster(c.gready, (uint32_t)(k & 1), limit, c.abort))) break;
                 k_g = k;
-                if (k + 1 < T) tc::mbar_arrive_expect_tx(c.gready, n_ct * kGBlock);  // dG of the next step
+                // dG of the next step: it cannot land before both issuers have passed this
+                // wait (it needs this step's MMAs of both)
+                if (q == 0 && k + 1 < T) tc::mbar_arrive_expect_tx(c.gready, n_ct * kGBlock);
                 tc::tc_fence_after();
-                const uint32_t d = tmem + acc * kCols;
+                const uint32_t d = tmem + acc * kCols + q * U;
                 for (uint32_t j = 0; j < n_ct; ++j)
 #pragma unroll
-                    for (int kq = 0; kq < kChunk / 16; ++kq)
+                    for (int kk = 0; kk < 2; ++kk) {
+                        const int kq = 2 * q + kk;
                         tc::mma_bf16(d, tc::smem_desc(c.g0 + j * kGBlock + kq * 32, 16, 1024),
-                                     tc::smem_desc(c.w0 + j * kWChunkB + kq * 32, 16, 1024), idesc, (j | kq) != 0);
+                                     tc::smem_desc(c.w0 + j * kWChunkB + kq * 32, 16, 1024), idesc, (j | kk) != 0);
+                    }
                 tc::mma_commit(&c.tfull[acc]);
                 // the dG buffer may be refilled once every CTA's MMAs of this step are done
                 tc::mma_commit_mc(c.dfree, (uint16_t)((1u << n_ct) - 1));
@@ -580,11 +586,11 @@ __global__ void __launch_bounds__(192, 1) step_clb(ClArgs p)
                 *c.abort = 1;
                 atomicCAS(a.err, 0, (int)SL_ERR_TIMEOUT);
                 // dG other CTAs may still be copying in lands before the CTA exits
-                if (k_g + 1 < T) tc::mbar_wait(c.gready, (uint32_t)((k_g + 1) & 1), kDrainLimit, nullptr);
+                if (q == 0 && k_g + 1 < T) tc::mbar_wait(c.gready, (uint32_t)((k_g + 1) & 1), kDrainLimit, nullptr);
             }
             tc::mma_commit(c.done);
-            // every CTA's commit of the last step has arrived here before the CTA exits
-            if (ok) mbar_wait_cluster(c.dfree, (uint32_t)((T - 1) & 1), kDrainLimit, nullptr);
+            // every CTA's commits of the last step have arrived here before the CTA exits
+            if (ok && q == 0) mbar_wait_cluster(c.dfree, (uint32_t)((T - 1) & 1), kDrainLimit, nullptr);
         }
         __syncwarp();
     } else {
@@ -664,9 +670,10 @@ __global__ void __launch_bounds__(192, 1) step_clb(ClArgs p)
             __syncwarp();
             if (tc::bar_any(1, E * 32, !ok || *c.abort)) break;
             tc::tc_fence_after();
-            uint32_t dr[U];
+            uint32_t dr[2][U];
             if (warp_rows) {
-                tc::tmem_ld16_async(taddr0 + acc * kCols, dr);
+                tc::tmem_ld16_async(taddr0 + acc * kCols, dr[0]);
+                tc::tmem_ld16_async(taddr0 + acc * kCols + U, dr[1]);
                 tc::tmem_wait_ld();
             }
             tc::tc_fence_before();
@@ -674,7 +681,7 @@ __global__ void __launch_bounds__(192, 1) step_clb(ClArgs p)
             if (lane == 0) tc::mbar_arrive(&c.tempty[acc]);
             float v[U];
 #pragma unroll
-            for (int j = 0; j < U; ++j) v[j] = dh_src[j] + __uint_as_float(dr[j]);
+            for (int j = 0; j < U; ++j) v[j] = dh_src[j] + (__uint_as_float(dr[0][j]) + __uint_as_float(dr[1][j]));
             float dcr[U];
             if (t >= 1) {
                 // the pointwise backward of step t - 1 (lanes without a row compute and discard)
