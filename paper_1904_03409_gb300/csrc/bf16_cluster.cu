@@ -8,10 +8,12 @@
 // or a step counter; the history rows, the h operand rows (for the weight gradient) and
 // the gates are still written to global memory for the backward.
 //
-// Warp roles (192 threads): warps 0..3 epilogue (TMEM lane quadrant w, one instance row
-// per thread of lanes 0..15; rows >= B idle), warp 4 producer (weight tile once; x_t chunks by TMA into a
-// two-step buffer), warp 5 MMA (x part of step t as soon as x_t lands, then the h part once
-// every slice of h_read(t) has landed; two TMEM accumulators by step parity).
+// Warp roles (224 threads): warps 0..3 epilogue (TMEM lane quadrant w, one instance row
+// per thread of lanes 0..15; rows >= B idle), warp 4 producer (weight tile once; x_t chunks
+// by TMA into a two-step buffer), warps 5 and 6 MMA issue (warp 6: the x part of step t as
+// soon as x_t lands; once every slice of h_read(t) has landed, warp 5 the even slices and
+// warp 6 the odd ones, each into its own accumulator; accumulators double-buffered by step
+// parity).
 //
 // x_t chunks are 64-row, 128-byte-swizzled 8 KB tiles; an h slice is 16 units x 64 rows in
 // the unswizzled K-major core-matrix layout ([row / 8][unit / 8][row mod 8][unit mod 8],
@@ -154,12 +156,14 @@ __device__ __forceinline__ void deliver_slice(const ClCtl &c, uint8_t *blk, int 
                     (uint16_t)((1u << n_ct) - 1));
 }
 
+constexpr int kClFwdThreads = 224;  // 4 epilogue warps, producer, two MMA issuers
+
 template <int U>
-__global__ void __launch_bounds__(192, 1) step_cl(const __grid_constant__ CUtensorMap tm_x, ClArgs p)
+__global__ void __launch_bounds__(kClFwdThreads, 1) step_cl(const __grid_constant__ CUtensorMap tm_x, ClArgs p)
 {
     static_assert(U == 16, "one h slice (two 8-unit core matrices) per CTA");
     constexpr int NB = 4 * U;
-    constexpr uint32_t kCols = TmemCols<NB>::value;
+    constexpr uint32_t kCols = TmemCols<2 * NB>::value;  // one accumulator per MMA issuer
     constexpr int E = 4;  // epilogue warps
     const StepArgs &a = p.s;
     extern __shared__ uint8_t smem_raw[];
@@ -179,10 +183,10 @@ __global__ void __launch_bounds__(192, 1) step_cl(const __grid_constant__ CUtens
             tc::mbar_init(&c.xfull[i], 1);
             tc::mbar_init(&c.xempty[i], 1);
             tc::mbar_init(&c.hready[i], 1);
-            tc::mbar_init(&c.tfull[i], 1);
+            tc::mbar_init(&c.tfull[i], 2);
             tc::mbar_init(&c.tempty[i], E);
         }
-        tc::mbar_init(c.done, 1);
+        tc::mbar_init(c.done, 2);
         *c.abort = 0;
         tc::fence_mbar_init();
         // the slices of h_read(0) and h_read(1): every CTA's, by byte count
@@ -219,8 +223,13 @@ __global__ void __launch_bounds__(192, 1) step_cl(const __grid_constant__ CUtens
                 tc::mbar_wait(&c.xfull[t & 1], (t >> 1) & 1, kDrainLimit, nullptr);
         }
         __syncwarp();
-    } else if (warp == E + 1) {
-        // ------------------------------------------------------------ MMA issue
+    } else if (warp == E + 1 || warp == E + 2) {
+        // ------------------------------------------------------------ MMA issue, two issuers
+        // The h part (one MMA per slice) is the step's critical path and its MMAs are bound
+        // by their issue, so two threads split it, each into its own accumulator (the
+        // epilogue adds the two). Issuer 1 also runs the x part, ahead of the h slices,
+        // into its accumulator; issuer 0 takes the even slices, issuer 1 the odd ones.
+        const int q = warp - (E + 1);
         if (lane == 0) {
             constexpr uint32_t idesc = tc::idesc_bf16(NB, 0, 0, 64);
             bool ok = tc::mbar_wait(c.wbar, 0, limit, c.abort);
@@ -228,31 +237,36 @@ __global__ void __launch_bounds__(192, 1) step_cl(const __grid_constant__ CUtens
             for (int t = 0; t < T && ok && !*c.abort; ++t) {
                 const int b = t & 1;
                 if (t >= 2 && !(ok = tc::mbar_wait(&c.tempty[b], ((t >> 1) - 1) & 1, limit, c.abort))) break;
-                if (!(ok = tc::mbar_wait(&c.xfull[b], (t >> 1) & 1, limit, c.abort))) break;
-                tc::tc_fence_after();
-                const uint32_t d = tmem + b * kCols;
-                for (int j = 0; j < kcx; ++j)
-                    cl_mma_chunk<NB>(d, c.x0 + (b * kcx + j) * kC64, c.w0 + j * NB * 128, j == 0);
-                tc::mma_commit(&c.xempty[b]);
+                const uint32_t d = tmem + b * kCols + q * NB;
+                if (q == 1) {
+                    if (!(ok = tc::mbar_wait(&c.xfull[b], (t >> 1) & 1, limit, c.abort))) break;
+                    tc::tc_fence_after();
+                    for (int j = 0; j < kcx; ++j)
+                        cl_mma_chunk<NB>(d, c.x0 + (b * kcx + j) * kC64, c.w0 + j * NB * 128, j == 0);
+                    tc::mma_commit(&c.xempty[b]);
+                }
                 // the h part once every CTA's slice of h_read(t) has landed
                 if (!(ok = mbar_wait_cluster(&c.hready[b], (t >> 1) & 1, limit, c.abort))) break;
                 t_h = t;
-                if (t + 2 < T) tc::mbar_arrive_expect_tx(&c.hready[b], n_ct * kSlice);  // this buffer's next use
+                // this buffer's next use: its slices cannot land before both issuers have
+                // passed this wait (they need this step's MMAs of both)
+                if (q == 0 && t + 2 < T) tc::mbar_arrive_expect_tx(&c.hready[b], n_ct * kSlice);
                 tc::tc_fence_after();
                 const uint32_t hb = c.h0 + (uint32_t)(b * n_ct) * kSlice;
-                for (uint32_t j = 0; j < n_ct; ++j) {
+                for (uint32_t j = (uint32_t)q; j < n_ct; j += 2) {
                     const uint32_t k = j * U;  // first h unit of slice j
                     tc::mma_bf16(d, slice_desc(hb + j * kSlice),
                                  tc::smem_desc(c.w0 + (uint32_t)(kcx + k / kChunk) * NB * 128 + (k % kChunk) * 2, 16, 1024),
-                                 idesc, 1);
+                                 idesc, q == 1 || j != 0);
                 }
                 tc::mma_commit(&c.tfull[b]);
             }
             if (!ok) {
                 cl_abort(c, a.err);
                 // slices other CTAs may still be copying in land before the CTA exits
-                for (int t = t_h + 1; t <= t_h + 2 && t < T; ++t)
-                    tc::mbar_wait(&c.hready[t & 1], (t >> 1) & 1, kDrainLimit, nullptr);
+                if (q == 0)
+                    for (int t = t_h + 1; t <= t_h + 2 && t < T; ++t)
+                        tc::mbar_wait(&c.hready[t & 1], (t >> 1) & 1, kDrainLimit, nullptr);
             }
             tc::mma_commit(c.done);
         }
@@ -321,6 +335,18 @@ __global__ void __launch_bounds__(192, 1) step_cl(const __grid_constant__ CUtens
 #pragma unroll
                 for (int g = 0; g < 4; ++g) tc::tmem_ld16_async(taddr0 + b * kCols + g * U, zr[g]);
                 tc::tmem_wait_ld();
+#pragma unroll
+                for (int h2 = 0; h2 < 2; ++h2) {  // the second issuer's accumulator, two gates at a time
+                    uint32_t z1[2][U];
+#pragma unroll
+                    for (int g = 0; g < 2; ++g) tc::tmem_ld16_async(taddr0 + b * kCols + NB + (2 * h2 + g) * U, z1[g]);
+                    tc::tmem_wait_ld();
+#pragma unroll
+                    for (int g = 0; g < 2; ++g)
+#pragma unroll
+                        for (int j = 0; j < U; ++j)
+                            zr[2 * h2 + g][j] = __float_as_uint(__uint_as_float(zr[2 * h2 + g][j]) + __uint_as_float(z1[g][j]));
+                }
             }
             tc::tc_fence_before();
             __syncwarp();
@@ -770,7 +796,7 @@ bool bf16_plan_fwd_cluster(stacklstm *s, PersistPlan *pl)
     }
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(n_ct);
-    cfg.blockDim = dim3(192);
+    cfg.blockDim = dim3(kClFwdThreads);
     cfg.dynamicSmemBytes = smem;
     cudaLaunchAttribute at[1];
     at[0].id = cudaLaunchAttributeClusterDimension;
@@ -791,7 +817,7 @@ bool bf16_plan_fwd_cluster(stacklstm *s, PersistPlan *pl)
     pl->cl = n_ct;
     pl->slot = 1;
     pl->smem = smem;
-    pl->threads = 192;
+    pl->threads = kClFwdThreads;
     return true;
 }
 
