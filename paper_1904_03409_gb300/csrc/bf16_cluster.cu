@@ -538,11 +538,16 @@ __device__ __forceinline__ void deliver_dg(const ClbCtl &c, const uint8_t *blk, 
     }
 }
 
+constexpr int kClbIssuers = 4;                          // MMA issue warps
+constexpr int kClBwdThreads = (4 + kClbIssuers) * 32;  // and 4 epilogue warps
+
 template <int U>
-__global__ void __launch_bounds__(192, 1) step_clb(ClArgs p)
+__global__ void __launch_bounds__(kClBwdThreads, 1) step_clb(ClArgs p)
 {
     static_assert(U == 16, "four 16-unit gate slices per CTA");
-    constexpr uint32_t kCols = TmemCols<2 * U>::value;  // one accumulator per MMA issuer
+    constexpr int NI = kClbIssuers;
+    static_assert(NI == 2 || NI == 4, "each issuer takes 4 / NI of a chunk's K = 16 steps");
+    constexpr uint32_t kCols = TmemCols<NI * U>::value;  // one accumulator per MMA issuer
     constexpr int E = 4;
     const StepArgs &a = p.s;
     extern __shared__ uint8_t smem_raw[];
@@ -554,12 +559,12 @@ __global__ void __launch_bounds__(192, 1) step_clb(ClArgs p)
     if (tid == 0) {
         tc::mbar_init(c.wbar, 1);
         tc::mbar_init(c.gready, 1);
-        tc::mbar_init(c.dfree, 2 * n_ct);  // both issuers' commits of every CTA
+        tc::mbar_init(c.dfree, NI * n_ct);  // every issuer's commits of every CTA
         for (int i = 0; i < 2; ++i) {
-            tc::mbar_init(&c.tfull[i], 2);
+            tc::mbar_init(&c.tfull[i], NI);
             tc::mbar_init(&c.tempty[i], E);
         }
-        tc::mbar_init(c.done, 2);
+        tc::mbar_init(c.done, NI);
         *c.abort = 0;
         tc::fence_mbar_init();
         tc::mbar_arrive_expect_tx(c.gready, n_ct * kGBlock);  // dG of step T - 1
@@ -571,13 +576,13 @@ __global__ void __launch_bounds__(192, 1) step_clb(ClArgs p)
     tc::tc_fence_after();
     const uint32_t tmem = *c.tmem_slot;
 
-    if (warp == E || warp == E + 1) {
-        // ------------------------------------------------------------ MMA issue, two issuers
+    if (warp >= E) {
+        // ------------------------------------------------------------ MMA issue, NI issuers
         // One thread issues an M = 64, N = 16 MMA about every 45 cycles; two issue about
-        // every 30 between them. Issuer q takes the K = 16 steps 2q and 2q + 1 of every
-        // chunk into its own accumulator (the epilogue adds the two); issuer 0 also posts
-        // each step's expected dG bytes and drains, issuer 1 first loads the weights.
-        const int q = warp == E + 1 ? 0 : 1;
+        // every 30 between them. Issuer q takes the K = 16 steps 4q / NI .. of every chunk
+        // into its own accumulator (the epilogue adds them); issuer 0 also posts each
+        // step's expected dG bytes and drains, issuer 1 first loads the weights.
+        const int q = warp - E;
         if (lane == 0) {
             constexpr uint32_t idesc = tc::idesc_bf16(U, 0, 0, 64);
             if (q == 1) {
@@ -599,8 +604,8 @@ __global__ void __launch_bounds__(192, 1) step_clb(ClArgs p)
                 const uint32_t d = tmem + acc * kCols + q * U;
                 for (uint32_t j = 0; j < n_ct; ++j)
 #pragma unroll
-                    for (int kk = 0; kk < 2; ++kk) {
-                        const int kq = 2 * q + kk;
+                    for (int kk = 0; kk < 4 / NI; ++kk) {
+                        const int kq = (4 / NI) * q + kk;
                         tc::mma_bf16(d, tc::smem_desc(c.g0 + j * kGBlock + kq * 32, 16, 1024),
                                      tc::smem_desc(c.w0 + j * kWChunkB + kq * 32, 16, 1024), idesc, (j | kk) != 0);
                     }
@@ -696,18 +701,24 @@ __global__ void __launch_bounds__(192, 1) step_clb(ClArgs p)
             __syncwarp();
             if (tc::bar_any(1, E * 32, !ok || *c.abort)) break;
             tc::tc_fence_after();
-            uint32_t dr[2][U];
-            if (warp_rows) {
-                tc::tmem_ld16_async(taddr0 + acc * kCols, dr[0]);
-                tc::tmem_ld16_async(taddr0 + acc * kCols + U, dr[1]);
-                tc::tmem_wait_ld();
-            }
+            float v[U];  // dh_src + the issuers' partial sums, added in issuer order
+#pragma unroll
+            for (int j = 0; j < U; ++j) v[j] = 0.0f;
+            if (warp_rows)
+#pragma unroll
+                for (int q2 = 0; q2 < NI; q2 += 2) {
+                    uint32_t dr[2][U];
+                    tc::tmem_ld16_async(taddr0 + acc * kCols + q2 * U, dr[0]);
+                    tc::tmem_ld16_async(taddr0 + acc * kCols + (q2 + 1) * U, dr[1]);
+                    tc::tmem_wait_ld();
+#pragma unroll
+                    for (int j = 0; j < U; ++j) v[j] += __uint_as_float(dr[0][j]) + __uint_as_float(dr[1][j]);
+                }
             tc::tc_fence_before();
             __syncwarp();
             if (lane == 0) tc::mbar_arrive(&c.tempty[acc]);
-            float v[U];
 #pragma unroll
-            for (int j = 0; j < U; ++j) v[j] = dh_src[j] + (__uint_as_float(dr[0][j]) + __uint_as_float(dr[1][j]));
+            for (int j = 0; j < U; ++j) v[j] += dh_src[j];
             float dcr[U];
             if (t >= 1) {
                 // the pointwise backward of step t - 1 (lanes without a row compute and discard)
@@ -868,7 +879,7 @@ bool bf16_plan_bwd_cluster(stacklstm *s, PersistPlan *pl)
     }
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(n_ct);
-    cfg.blockDim = dim3(192);
+    cfg.blockDim = dim3(kClBwdThreads);
     cfg.dynamicSmemBytes = smem;
     cudaLaunchAttribute at[1];
     at[0].id = cudaLaunchAttributeClusterDimension;
@@ -889,7 +900,7 @@ bool bf16_plan_bwd_cluster(stacklstm *s, PersistPlan *pl)
     pl->cl = n_ct;
     pl->slot = 1;
     pl->smem = smem;
-    pl->threads = 192;
+    pl->threads = kClBwdThreads;
     return true;
 }
 
