@@ -225,6 +225,8 @@ def run_ours(args, rank, world, local):
                                              "roofline": r["roofline"], "step_roofline": r["step_roofline"],
                                              "phases_ms_per_step": r["phases"]}
             del wx
+        torch.cuda.empty_cache()
+        line["other_workloads"]["arc_hybrid64"] = measure_group("arc_hybrid64", 20, 3, local)
     if rank == 0:
         print(json.dumps(line), flush=True)
     if world > 1:
@@ -319,6 +321,66 @@ def measure_workload(w, steps, warmup, local, world, sample_clocks, e2e):
         res["e2e"] = measure_e2e(w, hd, ins, out, steps, world, local, flush)
     hd.destroy()
     del ins, out, flush
+    torch.cuda.empty_cache()
+    return res
+
+
+def measure_group(name, steps, warmup, local):
+    """The three StackLSTMs of an arc-hybrid parser batch (stack, buffer, action history),
+    forward + backward at the same time, one stream each; against the same three timed one
+    at a time. value = instance-steps of all three / second."""
+    import torch
+    from paper_1904_03409_gb300 import runner, workloads as wl
+
+    g = wl.make_arc_hybrid(**wl.GROUPS[name])
+    dev = torch.device("cuda", local)
+    cur = torch.cuda.current_stream(dev)
+    hds = runner.create_group(g, local)
+    ins = {k: runner.upload(g[k], local) for k in runner.GROUP_MEMBERS}
+    outs = {k: runner.alloc_outputs(g[k], local, forward_outputs=False) for k in runner.GROUP_MEMBERS}
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    for _ in range(max(1, warmup)):
+        runner.group_forward_backward(hds, ins, outs)
+    torch.cuda.synchronize(dev)
+    runner.group_status(hds)
+
+    def timed(members):
+        evs = []
+        for _ in range(steps):
+            flush.zero_()
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(cur)
+            if members is None:
+                runner.group_forward_backward(hds, ins, outs)
+            else:
+                hd, st = hds[members]
+                st.wait_stream(cur)
+                runner.forward_backward(hd, ins[members], outs[members])
+                cur.wait_stream(st)
+            b.record(cur)
+            evs.append((a, b))
+        torch.cuda.synchronize(dev)
+        runner.group_status(hds)
+        return sum(x.elapsed_time(y) for x, y in evs) / steps
+
+    ms = timed(None)
+    alone = {k: timed(k) for k in runner.GROUP_MEMBERS}
+    units = sum(g[k].B * g[k].T for k in runner.GROUP_MEMBERS)
+    peaks, src = load_peaks()
+    fl = sum(work_per_inst_step(g[k].I, g[k].H)["step"]["flops"] * g[k].B * g[k].T for k in runner.GROUP_MEMBERS)
+    by = sum(work_per_inst_step(g[k].I, g[k].H)["step"]["bytes"] * g[k].B * g[k].T for k in runner.GROUP_MEMBERS)
+    res = {"workload": "%s: arc-hybrid parser batch, B=%d, n~U[10,60]; stack LSTM T=%d I=%d, buffer LSTM T=%d I=%d "
+                       "(n pushes, then a pop per Shift), action LSTM T=%d I=%d; H=%d; seed %d" % (
+                           name, g["stack"].B, g["stack"].T, g["stack"].I, g["buffer"].T, g["buffer"].I,
+                           g["action"].T, g["action"].I, g["stack"].H, g["stack"].seed),
+           "value": units / (ms / 1e3), "unit": "instance-steps/s (three StackLSTMs)",
+           "transitions_per_s": g["stack"].B * g["stack"].T / (ms / 1e3),
+           "ms_per_step": ms, "ms_one_at_a_time": {k: round(v, 4) for k, v in alone.items()},
+           "overlap_speedup": round(sum(alone.values()) / ms, 3), "steps": steps, "warmup": warmup,
+           "step_roofline": roofline_of(fl, by, ms / 1e3, peaks, src, sustained=True)}
+    for hd, _ in hds.values():
+        hd.destroy()
+    del ins, outs, flush
     torch.cuda.empty_cache()
     return res
 

@@ -71,3 +71,59 @@ def run(w, device: int = 0, d_top_h: Optional[np.ndarray] = None) -> dict:
         return to_numpy(out)
     finally:
         hd.destroy()
+
+
+GROUP_MEMBERS = ("stack", "buffer", "action")
+
+
+def create_group(group: dict, device: int = 0) -> dict:
+    """One handle per StackLSTM of a parser workload group, each on its own CUDA stream and
+    in asynchronous mode, so that their launches can run at the same time."""
+    import torch
+    hds = {}
+    for k in GROUP_MEMBERS:
+        w = group[k]
+        st = torch.cuda.Stream(device)
+        hd = bd.stacklstm_create(w.T, w.B, w.I, w.H, bd.SL_BF16 if w.dtype == "bf16" else bd.SL_FP32, device, st)
+        bd.stacklstm_set_async(hd, True)
+        hds[k] = (hd, st)
+    return hds
+
+
+def group_forward_backward(hds: dict, ins: dict, outs: dict):
+    """Enqueue forward + backward of every member on its own stream, after the current
+    stream's work; the current stream then waits for all of them."""
+    import torch
+    cur = torch.cuda.current_stream()
+    for k in GROUP_MEMBERS:
+        hd, st = hds[k]
+        st.wait_stream(cur)
+        forward_backward(hd, ins[k], outs[k])
+    for k in GROUP_MEMBERS:
+        cur.wait_stream(hds[k][1])
+
+
+def group_status(hds: dict):
+    for hd, _ in hds.values():
+        bd.stacklstm_status(hd)
+
+
+def run_group(group: dict, device: int = 0) -> dict:
+    """Forward + backward of the three StackLSTMs of a parser workload group at the same
+    time (one stream each), into NaN-filled outputs; numpy results per member."""
+    import torch
+    hds = create_group(group, device)
+    try:
+        ins = {k: upload(group[k], device) for k in GROUP_MEMBERS}
+        outs = {k: alloc_outputs(group[k], device) for k in GROUP_MEMBERS}
+        for o in outs.values():
+            for v in o.values():
+                if v.is_floating_point():
+                    v.fill_(float("nan"))
+        group_forward_backward(hds, ins, outs)
+        torch.cuda.synchronize(device)
+        group_status(hds)
+        return {k: to_numpy(outs[k]) for k in GROUP_MEMBERS}
+    finally:
+        for hd, _ in hds.values():
+            hd.destroy()

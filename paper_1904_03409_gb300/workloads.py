@@ -121,6 +121,42 @@ def ops_arc_standard(rng: np.random.Generator, B: int, n_range=(10, 60)):
     return ops, np.array([len(s) for s in streams], dtype=np.int32)
 
 
+def arc_hybrid_transitions(rng: np.random.Generator, n: int) -> list:
+    """One uniformly random valid arc-hybrid transition sequence over n tokens.
+
+    Parser state: a token stack and a buffer holding the tokens not yet shifted. Shift
+    (move the buffer front onto the stack) is valid while the buffer is non-empty,
+    Left-Arc (the stack top becomes a dependent of the buffer front; pop the stack) while
+    both are non-empty, Right-Arc (the stack top becomes a dependent of the token below it;
+    pop the stack) while the stack holds at least two tokens. The next transition is chosen
+    uniformly among the valid ones; the sequence ends with an empty buffer and one token
+    on the stack (the root), after n shifts and n - 1 arcs: 2n - 1 transitions.
+    """
+    buf, stack, seq = n, 0, []
+    while buf > 0 or stack > 1:
+        valid = []
+        if buf > 0:
+            valid.append("S")
+        if stack >= 1 and buf > 0:
+            valid.append("LA")
+        if stack >= 2:
+            valid.append("RA")
+        tr = valid[int(rng.integers(len(valid)))]
+        seq.append(tr)
+        if tr == "S":
+            buf -= 1
+            stack += 1
+        else:
+            stack -= 1
+    return seq
+
+
+# Table 1, arc-hybrid rows: (stack op, buffer op) of each transition; the action history
+# pushes every transition.
+ARC_HYBRID_OPS = {"S": (PUSH, POP), "LA": (POP, HOLD), "RA": (POP, HOLD)}
+ARC_HYBRID_ACTIONS = ("S", "LA", "RA")
+
+
 # ------------------------------------------------------------------------- workload
 @dataclasses.dataclass
 class Workload:
@@ -202,6 +238,83 @@ CONFIGS = {
     "stress": dict(T=512, B=4096, I=256, H=256, dtype="bf16", seed=4, ops_kind="random_walk",
                    probs=(0.6, 0.3, 0.1)),
 }
+
+
+def make_arc_hybrid(B: int, seed: int, H: int = 200, I_tok: int = 200, I_act: int = 48, dtype: str = "bf16",
+                    n_range=(10, 60)) -> dict:
+    """The three StackLSTMs of an arc-hybrid parser over one batch (Table 1), as three
+    workloads driven by one transition sequence per instance.
+
+    - ``stack``: per transition, Shift pushes, Left-Arc and Right-Arc pop; its input at
+      every step is the representation of the token at the buffer front (zeros once the
+      buffer is empty), which is the token a Shift moves onto the stack.
+    - ``buffer``: filled first by n pushes of the sentence's token representations, last
+      token first, so the first token is on top; then per transition, Shift pops and the
+      arcs hold (input zeros).
+    - ``action``: the transition history, pushed every transition, input the embedding of
+      the transition taken.
+
+    Each is hold-padded to its batch maximum (stack and action 2n - 1 steps, buffer
+    3n - 1). Draws, in order: (1) per instance n ~ U{n_lo..n_hi} and its transitions,
+    instance-major; (2) token representations [n_hi, B, I_tok]; (3) action embeddings
+    [3, I_act]; (4) W of the stack, buffer and action LSTMs, each U(-1/sqrt(H), 1/sqrt(H)).
+    Biases, h0 and c0 are zero; the loss seed is d(final top h) = 1 for each. Returns a
+    dict with the three workloads and ``transitions`` ([T_s, B] int8 action ids, -1 past
+    the end) and ``n`` ([B] sentence lengths).
+    """
+    rng = np.random.default_rng(seed)
+    seqs, ns = [], []
+    for _ in range(B):
+        n = int(rng.integers(n_range[0], n_range[1] + 1))
+        ns.append(n)
+        seqs.append(arc_hybrid_transitions(rng, n))
+    rep = rng.standard_normal((n_range[1], B, I_tok), dtype=np.float32)
+    emb = rng.standard_normal((len(ARC_HYBRID_ACTIONS), I_act), dtype=np.float32)
+    r = 1.0 / math.sqrt(H)
+    Ws = [rng.uniform(-r, r, size=(I + H, 4 * H)).astype(np.float32) for I in (I_tok, I_tok, I_act)]
+    Ts = max(len(q) for q in seqs)
+    Tb = max(n + len(q) for n, q in zip(ns, seqs))
+    ops_s, ops_a = np.zeros((Ts, B), np.int8), np.zeros((Ts, B), np.int8)
+    ops_b = np.zeros((Tb, B), np.int8)
+    x_s, x_a = np.zeros((Ts, B, I_tok), np.float32), np.zeros((Ts, B, I_act), np.float32)
+    x_b = np.zeros((Tb, B, I_tok), np.float32)
+    trans = np.full((Ts, B), -1, np.int8)
+    for b, (n, q) in enumerate(zip(ns, seqs)):
+        for i in range(n):  # the buffer: token n - 1 first, token 0 on top
+            ops_b[i, b] = PUSH
+            x_b[i, b] = rep[n - 1 - i, b]
+        front = 0  # index of the token at the buffer front
+        for k, tr in enumerate(q):
+            so, bo = ARC_HYBRID_OPS[tr]
+            ops_s[k, b], ops_b[n + k, b], ops_a[k, b] = so, bo, PUSH
+            if front < n:
+                x_s[k, b] = rep[front, b]
+            x_a[k, b] = emb[ARC_HYBRID_ACTIONS.index(tr)]
+            trans[k, b] = ARC_HYBRID_ACTIONS.index(tr)
+            if tr == "S":
+                front += 1
+    lens_s = np.array([len(q) for q in seqs], np.int32)
+    lens_b = np.array([n + len(q) for n, q in zip(ns, seqs)], np.int32)
+    if dtype == "bf16":
+        x_s, x_b, x_a = round_to_bf16(x_s), round_to_bf16(x_b), round_to_bf16(x_a)
+        Ws = [round_to_bf16(W) for W in Ws]
+    elif dtype != "fp32":
+        raise ValueError(dtype)
+    out = {}
+    for name, ops, x, W, lens in (("stack", ops_s, x_s, Ws[0], lens_s), ("buffer", ops_b, x_b, Ws[1], lens_b),
+                                  ("action", ops_a, x_a, Ws[2], lens_s)):
+        T, I = ops.shape[0], x.shape[2]
+        out[name] = Workload(name="arc_hybrid_" + name, T=int(T), B=B, I=I, H=H, dtype=dtype, seed=seed, ops=ops,
+                             lengths=lens, x=x, W=W, bias=np.zeros(4 * H, np.float32),
+                             h0=np.zeros((B, H), np.float32), c0=np.zeros((B, H), np.float32),
+                             d_top_h=np.ones((B, H), dtype=np.float32))
+    out["transitions"] = trans
+    out["n"] = np.array(ns, np.int32)
+    return out
+
+
+# Parser workloads of three StackLSTMs (stack, buffer, action history) per batch.
+GROUPS = {"arc_hybrid64": dict(B=64, seed=5, H=200, I_tok=200, I_act=48, dtype="bf16")}
 
 
 def config_workload(name: str, B: Optional[int] = None, T: Optional[int] = None) -> Workload:
