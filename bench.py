@@ -227,6 +227,8 @@ def run_ours(args, rank, world, local):
             del wx
         torch.cuda.empty_cache()
         line["other_workloads"]["arc_hybrid64"] = measure_group("arc_hybrid64", 20, 3, local)
+        torch.cuda.empty_cache()
+        line["other_workloads"]["parser_step64"] = measure_parser("arc_hybrid64", 20, 3, local)
     if rank == 0:
         print(json.dumps(line), flush=True)
     if world > 1:
@@ -381,6 +383,48 @@ def measure_group(name, steps, warmup, local):
     for hd, _ in hds.values():
         hd.destroy()
     del ins, outs, flush
+    torch.cuda.empty_cache()
+    return res
+
+
+def measure_parser(name, steps, warmup, local):
+    """A whole parser training step of the recurrent part on an arc-hybrid batch: the three
+    StackLSTM forwards at the same time, the parser head (200-wide ReLU state, softmax over
+    the transitions, cross-entropy), the three backwards seeded by the head's gradients.
+    value = instance-transitions / second."""
+    import torch
+    from paper_1904_03409_gb300 import runner, workloads as wl
+
+    g = wl.make_arc_hybrid(**wl.GROUPS[name])
+    dev = torch.device("cuda", local)
+    cur = torch.cuda.current_stream(dev)
+    ps = runner.create_parser(g, local)
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    for _ in range(max(1, warmup)):
+        runner.parser_step(ps)
+    torch.cuda.synchronize(dev)
+    runner.group_status(ps["hds"])
+    evs = []
+    for _ in range(steps):
+        flush.zero_()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(cur)
+        runner.parser_step(ps)
+        b.record(cur)
+        evs.append((a, b))
+    torch.cuda.synchronize(dev)
+    runner.group_status(ps["hds"])
+    ms = sum(x.elapsed_time(y) for x, y in evs) / steps
+    st = g["stack"]
+    hp = g["head"]
+    res = {"workload": "%s: arc-hybrid parser batch B=%d (as arc_hybrid64) plus the parser head: P=%d ReLU state "
+                       "over [stack; buffer; action] tops, softmax over %d transitions, cross-entropy; the "
+                       "StackLSTMs' backward seeded only by the head" % (name, st.B, hp["P"], hp["A"]),
+           "value": st.B * st.T / (ms / 1e3), "unit": "instance-transitions/s (padded, T=%d)" % st.T,
+           "real_transitions_per_s": float(g["L"].sum()) / (ms / 1e3), "ms_per_step": ms, "steps": steps,
+           "warmup": warmup}
+    runner.destroy_parser(ps)
+    del ps, flush
     torch.cuda.empty_cache()
     return res
 

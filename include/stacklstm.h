@@ -198,6 +198,67 @@ const char *stacklstm_last_error(stacklstm_t s);
 sl_status stacklstm_pointers_noalloc(int T, int B, const int8_t *ops, int32_t *p_traj, int32_t *src,
                                      void *stream);
 
+/*
+ * The parser head after the three StackLSTMs of a transition-based parser: the stack,
+ * the buffer and the action history (Sec. 4.1, which uses arc-hybrid; Table 1 gives each
+ * transition's stack and buffer ops). Before transition k of instance b the head reads
+ * the three tops (the output of Algorithm 1 of each StackLSTM):
+ *   s  = y_stack[k - 1, b]          (h0_stack[b] when k = 0)
+ *   bu = y_buffer[n[b] - 1 + k, b]  (the buffer StackLSTM is filled by n[b] pushes first)
+ *   a  = y_action[k - 1, b]         (h0_action[b] when k = 0)
+ * and computes p = ReLU(Wp [s; bu; a] + dp), the parser state (P wide; 200 in Sec. 4.1),
+ * z = Wz p + q over the A transitions, and the row loss logsumexp(z) - z[gold[k, b]].
+ * Transitions k >= L[b] are padding: no loss, no gradient. The paper fixes only the
+ * state width; the ReLU layer and the softmax follow the parser architecture its
+ * experiments reuse. bf16 inputs, fp32 arithmetic (CUDA cores); deterministic.
+ *
+ * stacklstm_head_create -- a head for T transitions (the stack and action StackLSTMs'
+ *   step count), a buffer StackLSTM of Tb steps, B instances, hidden width H (a multiple
+ *   of 8), state width P (<= 256) and A transitions (2..8). Owns its workspace (about
+ *   T B (6H + 8P + 4A) bytes). Calls are ordered on `stream`; SL_ERR_ARG,
+ *   SL_ERR_UNSUPPORTED or SL_ERR_OOM on failure, leaving *out NULL.
+ */
+typedef struct stacklstm_head *stacklstm_head_t;
+sl_status stacklstm_head_create(stacklstm_head_t *out, int T, int Tb, int B, int H, int P, int A, int device,
+                                void *stream);
+
+/*
+ * stacklstm_head_run -- loss and gradients of the head, enqueued on the head's stream.
+ * Inputs (device pointers; StackLSTM outputs 16-byte aligned):
+ *   y_stack, y_action [T, B, H] bf16; y_buffer [Tb, B, H] bf16; h0_stack, h0_action
+ *   [B, H] bf16; n, L [B] int32 (sentence lengths, transitions per instance);
+ *   gold [T, B] int8 transition ids in [0, A) for k < L[b]; Wp [P, 3H] bf16; dp [P];
+ *   Wz [A, P]; q [A] (float).
+ * Outputs (float, device):
+ *   loss_rows [T, B] (0 on padding; the loss is their sum);
+ *   dy_stack, dy_action [T, B, H] and dy_buffer [Tb, B, H]: the gradient of the loss
+ *     w.r.t. each StackLSTM output, to pass as stacklstm_backward's dy (rows the head
+ *     does not read are 0);
+ *   dWp [P, 3H], ddp [P], dWz [A, P], dq [A].
+ * The gradients w.r.t. h0_stack and h0_action (the k = 0 reads) stay in the workspace
+ * for stacklstm_head_add_h0_grads. A transition whose length or label is out of range is
+ * skipped and reported by stacklstm_head_status (SL_ERR_ARG).
+ */
+sl_status stacklstm_head_run(stacklstm_head_t h, const void *y_stack, const void *h0_stack, const void *y_buffer,
+                             const void *y_action, const void *h0_action, const int32_t *n, const int32_t *L,
+                             const int8_t *gold, const void *Wp, const float *dp, const float *Wz, const float *q,
+                             float *loss_rows, float *dy_stack, float *dy_buffer, float *dy_action, float *dWp,
+                             float *ddp, float *dWz, float *dq);
+
+/* Add the last run's gradients w.r.t. h0_stack and h0_action into dh0_stack and
+ * dh0_action ([B, H] float, device; either may be NULL): call it after the StackLSTMs'
+ * stacklstm_backward wrote their dh0, to get the whole gradient of the initial states. */
+sl_status stacklstm_head_add_h0_grads(stacklstm_head_t h, float *dh0_stack, float *dh0_action);
+
+/* Synchronize the head's stream; return (then clear) a device-detected error. */
+sl_status stacklstm_head_status(stacklstm_head_t h);
+
+/* Free the head and its workspace (synchronizes its stream first). NULL is a no-op. */
+sl_status stacklstm_head_destroy(stacklstm_head_t h);
+
+/* One-line message for the last failure on the head ("" if none). */
+const char *stacklstm_head_last_error(stacklstm_head_t h);
+
 #ifdef __cplusplus
 }
 #endif

@@ -63,9 +63,17 @@ def load(path: Optional[str] = None):
     lib.stacklstm_plan.restype = ctypes.c_char_p
     lib.stacklstm_last_error.argtypes = [vp]
     lib.stacklstm_last_error.restype = ctypes.c_char_p
+    lib.stacklstm_head_create.argtypes = [ctypes.POINTER(vp), i, i, i, i, i, i, i, vp]
+    lib.stacklstm_head_run.argtypes = [vp] * 21
+    lib.stacklstm_head_add_h0_grads.argtypes = [vp, vp, vp]
+    lib.stacklstm_head_status.argtypes = [vp]
+    lib.stacklstm_head_destroy.argtypes = [vp]
+    lib.stacklstm_head_last_error.argtypes = [vp]
+    lib.stacklstm_head_last_error.restype = ctypes.c_char_p
     for fn in ("stacklstm_create", "stacklstm_forward", "stacklstm_backward", "stacklstm_set_stream",
                "stacklstm_set_async", "stacklstm_status", "stacklstm_destroy", "stacklstm_set_timing",
-               "stacklstm_get_timing"):
+               "stacklstm_get_timing", "stacklstm_head_create", "stacklstm_head_run", "stacklstm_head_add_h0_grads",
+               "stacklstm_head_status", "stacklstm_head_destroy"):
         getattr(lib, fn).restype = ctypes.c_int
     _lib = lib
     return lib
@@ -214,3 +222,75 @@ def stacklstm_plan(hd: StackLSTMHandle) -> str:
 
 def stacklstm_destroy(hd: StackLSTMHandle):
     hd.destroy()
+
+
+# ------------------------------------------------------------------ parser head
+class StackLSTMHeadHandle:
+    """Owns one parser-head handle (stacklstm_head_*); ``destroy`` frees it."""
+
+    def __init__(self, h, T, Tb, B, H, P, A, device):
+        self.h, self.T, self.Tb, self.B, self.H, self.P, self.A, self.device = h, T, Tb, B, H, P, A, device
+
+    def destroy(self):
+        if self.h is not None and _lib is not None:
+            _lib.stacklstm_head_destroy(self.h)
+        self.h = None
+
+    def __del__(self):
+        try:
+            self.destroy()
+        except Exception:
+            pass
+
+
+def _check_head(handle, st: int, where: str):
+    if st != 0:
+        msg = load().stacklstm_head_last_error(handle).decode() if handle else ""
+        raise StackLSTMError(st, where, msg)
+
+
+def stacklstm_head_create(T: int, Tb: int, B: int, H: int, P: int, A: int, device: int = 0, stream=None):
+    """A parser head for T transitions, a Tb-step buffer StackLSTM, B instances, hidden H,
+    state P, A transitions; ``stream`` as for stacklstm_create."""
+    import torch
+    if stream is None:
+        stream = torch.cuda.current_stream(device)
+    raw = stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream)
+    h = ctypes.c_void_p()
+    _check_head(None, load().stacklstm_head_create(ctypes.byref(h), T, Tb, B, H, P, A, device, ctypes.c_void_p(raw)),
+                "stacklstm_head_create")
+    return StackLSTMHeadHandle(h, T, Tb, B, H, P, A, device)
+
+
+def stacklstm_head_run(hh: StackLSTMHeadHandle, y_stack, h0_stack, y_buffer, y_action, h0_action, n, L, gold, Wp,
+                       dp, Wz, q, loss_rows, dy_stack, dy_buffer, dy_action, dWp, ddp, dWz, dq):
+    """Loss rows and gradients of the parser head; see include/stacklstm.h for layouts."""
+    import torch
+    T, Tb, B, H, P, A, d = hh.T, hh.Tb, hh.B, hh.H, hh.P, hh.A, hh.device
+    bf, f = torch.bfloat16, torch.float32
+    args = [_ptr(y_stack, d, bf, (T, B, H), "y_stack"), _ptr(h0_stack, d, bf, (B, H), "h0_stack"),
+            _ptr(y_buffer, d, bf, (Tb, B, H), "y_buffer"), _ptr(y_action, d, bf, (T, B, H), "y_action"),
+            _ptr(h0_action, d, bf, (B, H), "h0_action"), _ptr(n, d, torch.int32, (B,), "n"),
+            _ptr(L, d, torch.int32, (B,), "L"), _ptr(gold, d, torch.int8, (T, B), "gold"),
+            _ptr(Wp, d, bf, (P, 3 * H), "Wp"), _ptr(dp, d, f, (P,), "dp"), _ptr(Wz, d, f, (A, P), "Wz"),
+            _ptr(q, d, f, (A,), "q"), _ptr(loss_rows, d, f, (T, B), "loss_rows"),
+            _ptr(dy_stack, d, f, (T, B, H), "dy_stack"), _ptr(dy_buffer, d, f, (Tb, B, H), "dy_buffer"),
+            _ptr(dy_action, d, f, (T, B, H), "dy_action"), _ptr(dWp, d, f, (P, 3 * H), "dWp"),
+            _ptr(ddp, d, f, (P,), "ddp"), _ptr(dWz, d, f, (A, P), "dWz"), _ptr(dq, d, f, (A,), "dq")]
+    _check_head(hh.h, load().stacklstm_head_run(hh.h, *args), "stacklstm_head_run")
+
+
+def stacklstm_head_add_h0_grads(hh: StackLSTMHeadHandle, dh0_stack=None, dh0_action=None):
+    import torch
+    B, H, d, f = hh.B, hh.H, hh.device, torch.float32
+    _check_head(hh.h, load().stacklstm_head_add_h0_grads(hh.h, _ptr(dh0_stack, d, f, (B, H), "dh0_stack"),
+                                                         _ptr(dh0_action, d, f, (B, H), "dh0_action")),
+                "stacklstm_head_add_h0_grads")
+
+
+def stacklstm_head_status(hh: StackLSTMHeadHandle):
+    _check_head(hh.h, load().stacklstm_head_status(hh.h), "stacklstm_head_status")
+
+
+def stacklstm_head_destroy(hh: StackLSTMHeadHandle):
+    hh.destroy()

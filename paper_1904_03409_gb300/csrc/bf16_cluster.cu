@@ -800,7 +800,7 @@ bool bf16_plan_fwd_cluster(stacklstm *s, PersistPlan *pl)
     const uint32_t smem = cl_smem_bytes(s->kcf, s->kcx, NB, n_ct);
     if (smem > kSmemCap) return false;
     const void *fn = (const void *)step_cl<kClU>;
-    if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess ||
+    if (smem_at_least(fn, smem) != cudaSuccess ||
         (n_ct > 8 && cudaFuncSetAttribute(fn, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess)) {
         cudaGetLastError();
         return false;
@@ -872,7 +872,7 @@ bool bf16_plan_bwd_cluster(stacklstm *s, PersistPlan *pl)
     const uint32_t smem = clb_smem_bytes(n_ct);
     if (smem > kSmemCap) return false;
     const void *fn = (const void *)step_clb<kClU>;
-    if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess ||
+    if (smem_at_least(fn, smem) != cudaSuccess ||
         (n_ct > 8 && cudaFuncSetAttribute(fn, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess)) {
         cudaGetLastError();
         return false;

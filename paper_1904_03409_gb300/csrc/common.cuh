@@ -116,6 +116,10 @@ namespace sl {
 
 // ---- index / gather kernels (index_kernels.cu)
 cudaError_t launch_prepass(stacklstm *s, const int8_t *ops);
+// Raise kernel `fn`'s dynamic shared-memory limit on the current device to at least
+// `bytes`. The limit belongs to the function, not to a handle, so handles of different
+// sizes (created in any order, used from any stream) only ever raise it.
+cudaError_t smem_at_least(const void *fn, size_t bytes);
 cudaError_t launch_gather_rows(stacklstm *s, const int32_t *idx, int rows, size_t elem_bytes,
                                const void *hist, void *out, int row_elems);
 cudaError_t launch_seed_grads(stacklstm *s, const float *d_top_h, const float *dy);

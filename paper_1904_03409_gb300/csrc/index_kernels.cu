@@ -8,6 +8,7 @@
 //   slot_last   history index last written to each slot after the last step (-1: never).
 // Every step writes slot p_t + 1 (Algorithm 1), which in history terms is row t + 1.
 #include <algorithm>
+#include <map>
 #include <mutex>
 
 #include "common.cuh"
@@ -99,6 +100,21 @@ __global__ void seed_grads_kernel(int T, int B, int H, const int32_t *__restrict
 
 }  // namespace
 
+cudaError_t smem_at_least(const void *fn, size_t bytes)
+{
+    static std::mutex m;
+    static std::map<std::pair<int, const void *>, size_t> set;
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e) return e;
+    std::lock_guard<std::mutex> lk(m);
+    size_t &cur = set[{dev, fn}];
+    if (bytes <= cur) return cudaSuccess;
+    if ((e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes))) return e;
+    cur = bytes;
+    return cudaSuccess;
+}
+
 // The slot-tag stack goes on chip when (T + 1) slots x 32 instances fit in shared memory.
 cudaError_t configure_prepass(stacklstm *s)
 {
@@ -108,9 +124,7 @@ cudaError_t configure_prepass(stacklstm *s)
     if (e) return e;
     s->prepass_smem = 0;
     if (bytes + 1024 <= (size_t)optin) {
-        if (bytes > 48 * 1024 &&
-            (e = cudaFuncSetAttribute(prepass_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes)))
-            return e;
+        if (bytes > 48 * 1024 && (e = smem_at_least((const void *)prepass_kernel<true>, bytes))) return e;
         s->prepass_smem = (int)bytes;
     }
     return cudaSuccess;

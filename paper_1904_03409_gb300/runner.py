@@ -127,3 +127,80 @@ def run_group(group: dict, device: int = 0) -> dict:
     finally:
         for hd, _ in hds.values():
             hd.destroy()
+
+
+def create_parser(group: dict, device: int = 0) -> dict:
+    """The three StackLSTM handles of ``create_group`` plus a parser head on the current
+    stream, and the device tensors of a whole parser step."""
+    import torch
+    dev = torch.device("cuda", device)
+    hds = create_group(group, device)
+    hp, st, bu = group["head"], group["stack"], group["buffer"]
+    head = bd.stacklstm_head_create(st.T, bu.T, st.B, st.H, hp["P"], hp["A"], device)
+    f = lambda a, dt=torch.float32: torch.from_numpy(np.ascontiguousarray(a, dtype=np.float32)).to(dev).to(dt)
+    hin = dict(n=torch.from_numpy(group["n"].astype(np.int32)).to(dev), L=torch.from_numpy(group["L"].astype(np.int32)).to(dev),
+               gold=torch.from_numpy(group["transitions"].astype(np.int8)).to(dev), Wp=f(hp["Wp"], torch.bfloat16),
+               dp=f(hp["dp"]), Wz=f(hp["Wz"]), q=f(hp["q"]))
+    e = lambda *s: torch.empty(*s, dtype=torch.float32, device=dev)
+    T, Tb, B, H, P, A = st.T, bu.T, st.B, st.H, hp["P"], hp["A"]
+    hout = dict(loss_rows=e(T, B), dy_stack=e(T, B, H), dy_buffer=e(Tb, B, H), dy_action=e(T, B, H),
+                dWp=e(P, 3 * H), ddp=e(P), dWz=e(A, P), dq=e(A))
+    ins = {k: upload(group[k], device) for k in GROUP_MEMBERS}
+    outs = {k: alloc_outputs(group[k], device) for k in GROUP_MEMBERS}
+    return dict(hds=hds, head=head, hin=hin, hout=hout, ins=ins, outs=outs)
+
+
+def parser_step(ps: dict):
+    """One training step of the parser's recurrent part: the three StackLSTM forwards at
+    the same time, the head on the current stream, the three backwards (seeded only by
+    the head's gradients) at the same time, then the head's initial-state gradients."""
+    import torch
+    cur = torch.cuda.current_stream()
+    hds, ins, outs, hin, hout = ps["hds"], ps["ins"], ps["outs"], ps["hin"], ps["hout"]
+    for k in GROUP_MEMBERS:
+        hd, st = hds[k]
+        st.wait_stream(cur)
+        o, i = outs[k], ins[k]
+        bd.stacklstm_forward(hd, i["x"], i["ops"], i["h0"], i["c0"], i["W"], i["bias"], o.get("h_stack"),
+                             o.get("c_stack"), o["p_final"], o.get("p_traj"), o.get("src"), o["y"])
+    for k in GROUP_MEMBERS:
+        cur.wait_stream(hds[k][1])
+    bd.stacklstm_head_run(ps["head"], outs["stack"]["y"], ins["stack"]["h0"], outs["buffer"]["y"],
+                          outs["action"]["y"], ins["action"]["h0"], hin["n"], hin["L"], hin["gold"], hin["Wp"],
+                          hin["dp"], hin["Wz"], hin["q"], hout["loss_rows"], hout["dy_stack"], hout["dy_buffer"],
+                          hout["dy_action"], hout["dWp"], hout["ddp"], hout["dWz"], hout["dq"])
+    for k in GROUP_MEMBERS:
+        hd, st = hds[k]
+        st.wait_stream(cur)
+        o = outs[k]
+        bd.stacklstm_backward(hd, None, hout["dy_" + k], o["dx"], o["dh0"], o["dc0"], o["dW"], o["dbias"])
+    for k in GROUP_MEMBERS:
+        cur.wait_stream(hds[k][1])
+    bd.stacklstm_head_add_h0_grads(ps["head"], outs["stack"]["dh0"], outs["action"]["dh0"])
+
+
+def destroy_parser(ps: dict):
+    for hd, _ in ps["hds"].values():
+        hd.destroy()
+    ps["head"].destroy()
+
+
+def run_parser(group: dict, device: int = 0) -> dict:
+    """One parser step into NaN-filled outputs; numpy results: {member: outputs} and
+    ``head`` (loss rows and the head's gradients)."""
+    import torch
+    ps = create_parser(group, device)
+    try:
+        for d in list(ps["outs"].values()) + [ps["hout"]]:
+            for v in d.values():
+                if v.is_floating_point():
+                    v.fill_(float("nan"))
+        parser_step(ps)
+        torch.cuda.synchronize(device)
+        group_status(ps["hds"])
+        bd.stacklstm_head_status(ps["head"])
+        res = {k: to_numpy(ps["outs"][k]) for k in GROUP_MEMBERS}
+        res["head"] = to_numpy(ps["hout"])
+        return res
+    finally:
+        destroy_parser(ps)

@@ -241,7 +241,7 @@ CONFIGS = {
 
 
 def make_arc_hybrid(B: int, seed: int, H: int = 200, I_tok: int = 200, I_act: int = 48, dtype: str = "bf16",
-                    n_range=(10, 60)) -> dict:
+                    n_range=(10, 60), P: int = 200) -> dict:
     """The three StackLSTMs of an arc-hybrid parser over one batch (Table 1), as three
     workloads driven by one transition sequence per instance.
 
@@ -257,10 +257,12 @@ def make_arc_hybrid(B: int, seed: int, H: int = 200, I_tok: int = 200, I_act: in
     Each is hold-padded to its batch maximum (stack and action 2n - 1 steps, buffer
     3n - 1). Draws, in order: (1) per instance n ~ U{n_lo..n_hi} and its transitions,
     instance-major; (2) token representations [n_hi, B, I_tok]; (3) action embeddings
-    [3, I_act]; (4) W of the stack, buffer and action LSTMs, each U(-1/sqrt(H), 1/sqrt(H)).
-    Biases, h0 and c0 are zero; the loss seed is d(final top h) = 1 for each. Returns a
-    dict with the three workloads and ``transitions`` ([T_s, B] int8 action ids, -1 past
-    the end) and ``n`` ([B] sentence lengths).
+    [3, I_act]; (4) W of the stack, buffer and action LSTMs, each U(-1/sqrt(H), 1/sqrt(H));
+    (5) the parser head's Wp [P, 3H] ~ U(-1/sqrt(3H), 1/sqrt(3H)) and Wz [3, P] ~
+    U(-1/sqrt(P), 1/sqrt(P)) (its biases dp, q zero). Biases, h0 and c0 of the StackLSTMs
+    are zero; each workload's own loss seed is d(final top h) = 1. Returns a dict with the
+    three workloads, ``transitions`` ([T_s, B] int8 action ids, -1 past the end), ``n``
+    ([B] sentence lengths), ``L`` ([B] transitions) and ``head`` (Wp, dp, Wz, q).
     """
     rng = np.random.default_rng(seed)
     seqs, ns = [], []
@@ -272,6 +274,9 @@ def make_arc_hybrid(B: int, seed: int, H: int = 200, I_tok: int = 200, I_act: in
     emb = rng.standard_normal((len(ARC_HYBRID_ACTIONS), I_act), dtype=np.float32)
     r = 1.0 / math.sqrt(H)
     Ws = [rng.uniform(-r, r, size=(I + H, 4 * H)).astype(np.float32) for I in (I_tok, I_tok, I_act)]
+    A = len(ARC_HYBRID_ACTIONS)
+    Wp = rng.uniform(-1.0 / math.sqrt(3 * H), 1.0 / math.sqrt(3 * H), size=(P, 3 * H)).astype(np.float32)
+    Wz = rng.uniform(-1.0 / math.sqrt(P), 1.0 / math.sqrt(P), size=(A, P)).astype(np.float32)
     Ts = max(len(q) for q in seqs)
     Tb = max(n + len(q) for n, q in zip(ns, seqs))
     ops_s, ops_a = np.zeros((Ts, B), np.int8), np.zeros((Ts, B), np.int8)
@@ -298,6 +303,7 @@ def make_arc_hybrid(B: int, seed: int, H: int = 200, I_tok: int = 200, I_act: in
     if dtype == "bf16":
         x_s, x_b, x_a = round_to_bf16(x_s), round_to_bf16(x_b), round_to_bf16(x_a)
         Ws = [round_to_bf16(W) for W in Ws]
+        Wp = round_to_bf16(Wp)
     elif dtype != "fp32":
         raise ValueError(dtype)
     out = {}
@@ -310,6 +316,8 @@ def make_arc_hybrid(B: int, seed: int, H: int = 200, I_tok: int = 200, I_act: in
                              d_top_h=np.ones((B, H), dtype=np.float32))
     out["transitions"] = trans
     out["n"] = np.array(ns, np.int32)
+    out["L"] = lens_s
+    out["head"] = dict(Wp=Wp, dp=np.zeros(P, np.float32), Wz=Wz, q=np.zeros(A, np.float32), P=P, A=A)
     return out
 
 

@@ -123,3 +123,108 @@ def test_arc_hybrid_three_stacklstms_at_once_match_oracle():
         for name in ("dx", "dW", "dbias", "dh0", "y", "h_stack", "p_traj"):
             assert np.array_equal(got[k][name], alone[name], equal_nan=True), (k, name)
     torch.cuda.empty_cache()
+
+
+def parser_oracle(g, got):
+    """The oracle of one parser step, stage by stage on the inputs the GPU stage saw:
+    each StackLSTM's forward; the head on the GPU's StackLSTM outputs; each StackLSTM's
+    backward seeded by the GPU head's output gradients. Also the head on the oracle's own
+    (fp64) outputs, for the end-to-end loss."""
+    from oracle import parser_head as ph
+    import os
+    nt = max(1, len(os.sched_getaffinity(0)))
+    hp = g["head"]
+    fw = {}
+    for k in ("stack", "buffer", "action"):
+        w = g[k]
+        fw[k] = oracle.run(w.x, w.ops, w.h0, w.c0, w.W, w.bias, d_top_h=np.zeros_like(w.h0), nthreads=nt,
+                           outputs=("p_traj", "src", "y", "h_stack", "c_stack"))
+    args = (g["action"].h0, g["n"], g["L"], g["transitions"], hp["Wp"], hp["dp"], hp["Wz"], hp["q"])
+    head = ph.forward_backward(got["stack"]["y"], g["stack"].h0, got["buffer"]["y"], got["action"]["y"], *args)
+    head64 = ph.forward_backward(fw["stack"]["y"], g["stack"].h0, fw["buffer"]["y"], fw["action"]["y"], *args)
+    bw = {}
+    for k in ("stack", "buffer", "action"):
+        w = g[k]
+        bw[k] = oracle.run(w.x, w.ops, w.h0, w.c0, w.W, w.bias, d_top_h=np.zeros_like(w.h0),
+                           dy=got["head"]["dy_" + k], nthreads=nt, outputs=("dx", "dh0", "dc0", "dW", "dbias"))
+    bw["stack"]["dh0"] = bw["stack"]["dh0"] + head["dh0_stack"]
+    bw["action"]["dh0"] = bw["action"]["dh0"] + head["dh0_action"]
+    return fw, head, bw, head64
+
+
+@pytest.mark.gpu
+def test_parser_step_three_stacklstms_and_head_match_oracle():
+    """A whole parser step through the C ABI (the three StackLSTMs at the same time, the
+    head, the three backwards seeded by the head), each stage against the oracle on the
+    inputs that stage received; the total loss against the all-fp64 chain."""
+    import torch
+    from paper_1904_03409_gb300 import runner
+    from parity import BF16_REL
+    g = wl.make_arc_hybrid(**wl.GROUPS["arc_hybrid64"])
+    got = runner.run_parser(g)
+    fw, head, bw, head64 = parser_oracle(g, got)
+    for k in runner.GROUP_MEMBERS:
+        compare(got[k], fw[k], "bf16", keys=("p_traj", "src", "p_final", "y", "h_stack", "c_stack"))
+        compare(got[k], bw[k], "bf16", keys=("dx", "dh0", "dc0", "dW", "dbias"))
+    gh = got["head"]
+    for name in ("loss_rows", "dy_stack", "dy_buffer", "dy_action", "dWp", "ddp", "dWz", "dq"):
+        err = float(np.abs(gh[name].astype(np.float64) - head[name]).max())
+        tol = BF16_REL * float(np.abs(head[name]).max())
+        assert np.isfinite(err) and err <= tol, (name, err, tol)
+    # padding transitions carry no loss; the total loss is close to the all-fp64 chain's
+    assert np.all(gh["loss_rows"][g["transitions"] < 0] == 0.0)
+    assert abs(gh["loss_rows"].sum() - head64["loss"]) <= 1e-2 * abs(head64["loss"])
+    # reproducible bit for bit
+    again = runner.run_parser(g)
+    for name in ("dWp", "ddp", "dWz", "dq", "dy_buffer"):
+        assert np.array_equal(gh[name], again["head"][name]), name
+    assert np.array_equal(got["stack"]["dW"], again["stack"]["dW"])
+    torch.cuda.empty_cache()
+
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("B,H,P,A,n_hi,seed", [(5, 16, 24, 3, 6, 1), (3, 200, 200, 3, 30, 2), (37, 8, 8, 5, 9, 3)])
+def test_parser_head_alone_matches_oracle(B, H, P, A, n_hi, seed):
+    """The head on random bf16 StackLSTM outputs (ragged lengths, row tiles with a
+    ragged tail, several widths) against the head oracle."""
+    import torch
+    from oracle import parser_head as ph
+    from paper_1904_03409_gb300 import binding as bd
+    from parity import BF16_REL
+    rng = np.random.default_rng(seed)
+    n = rng.integers(1, n_hi + 1, size=B).astype(np.int32)
+    L = (2 * n - 1).astype(np.int32)
+    T, Tb = int(L.max()), int((n + L).max())
+    r = lambda *s: wl.round_to_bf16(rng.standard_normal(s).astype(np.float32))
+    ys, yb, ya, h0s, h0a = r(T, B, H), r(Tb, B, H), r(T, B, H), r(B, H), r(B, H)
+    gold = np.where(np.arange(T)[:, None] < L[None, :], rng.integers(0, A, (T, B)), -1).astype(np.int8)
+    Wp = wl.round_to_bf16((rng.standard_normal((P, 3 * H)) / np.sqrt(3 * H)).astype(np.float32))
+    dp = (0.1 * rng.standard_normal(P)).astype(np.float32)
+    Wz = (rng.standard_normal((A, P)) / np.sqrt(P)).astype(np.float32)
+    q = (0.1 * rng.standard_normal(A)).astype(np.float32)
+    want = ph.forward_backward(ys, h0s, yb, ya, h0a, n, L, gold, Wp, dp, Wz, q)
+    dev = torch.device("cuda", 0)
+    bf = lambda a: torch.from_numpy(a).to(dev).to(torch.bfloat16)
+    f = lambda a: torch.from_numpy(np.ascontiguousarray(a, np.float32)).to(dev)
+    e = lambda *s: torch.full(s, float("nan"), dtype=torch.float32, device=dev)
+    out = dict(loss_rows=e(T, B), dy_stack=e(T, B, H), dy_buffer=e(Tb, B, H), dy_action=e(T, B, H),
+               dWp=e(P, 3 * H), ddp=e(P), dWz=e(A, P), dq=e(A))
+    hh = bd.stacklstm_head_create(T, Tb, B, H, P, A, 0)
+    try:
+        bd.stacklstm_head_run(hh, bf(ys), bf(h0s), bf(yb), bf(ya), bf(h0a), torch.from_numpy(n).to(dev),
+                              torch.from_numpy(L).to(dev), torch.from_numpy(gold).to(dev), bf(Wp), f(dp), f(Wz), f(q),
+                              *out.values())
+        dh0s, dh0a = torch.zeros(B, H, device=dev), torch.zeros(B, H, device=dev)
+        bd.stacklstm_head_add_h0_grads(hh, dh0s, dh0a)
+        bd.stacklstm_head_status(hh)
+    finally:
+        hh.destroy()
+    got = {k: v.cpu().numpy() for k, v in out.items()}
+    got["dh0_stack"], got["dh0_action"] = dh0s.cpu().numpy(), dh0a.cpu().numpy()
+    for name in got:
+        err = float(np.abs(got[name].astype(np.float64) - want[name]).max())
+        tol = BF16_REL * max(float(np.abs(want[name]).max()), 1e-30)
+        assert np.isfinite(err) and err <= tol, (name, err, tol)
+    # rows the head does not read get exactly zero gradient
+    assert np.all(got["dy_buffer"][want["dy_buffer"] == 0] == 0)
+    assert np.all(got["dy_stack"][want["dy_stack"] == 0] == 0)
