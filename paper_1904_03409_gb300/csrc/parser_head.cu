@@ -378,7 +378,11 @@ sl_status stacklstm_head_create(stacklstm_head_t *out, int T, int Tb, int B, int
     h->smem = head_smem_bytes(R, H, P, A);
     int prev = -1;
     cudaGetDevice(&prev);
-    cudaSetDevice(device);
+    if (cudaSetDevice(device) != cudaSuccess) {
+        cudaGetLastError();
+        delete h;
+        return SL_ERR_ARG;  // no such device
+    }
     const size_t NR = (size_t)T * B, K = 3 * (size_t)H;
     const size_t part = std::max((size_t)h->S * P * K, (size_t)kSmallChunks * ((size_t)A * P + P + A));
     bool ok = cudaMalloc(&h->wpt, K * P * 2) == cudaSuccess && cudaMalloc(&h->u, NR * K * 2) == cudaSuccess &&

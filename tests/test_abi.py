@@ -59,3 +59,23 @@ def test_binding_refuses_without_library(tmp_path):
             binding.load(str(tmp_path / "missing.so"))
     finally:
         binding._lib = saved
+
+
+@pytest.mark.parametrize("T,Tb,B,H,P,A,want", [(0, 4, 2, 8, 8, 3, 1), (4, 0, 2, 8, 8, 3, 1), (4, 4, 0, 8, 8, 3, 1),
+                                               (4, 4, 2, 0, 8, 3, 1), (4, 4, 2, 8, 0, 3, 1), (4, 4, 2, 8, 8, 1, 1),
+                                               (4, 4, 2, 12, 8, 3, 7), (4, 4, 2, 8, 300, 3, 7),
+                                               (4, 4, 2, 8, 8, 9, 7)])
+def test_head_create_rejects_bad_sizes(lib, T, Tb, B, H, P, A, want):
+    # the parser head: H a multiple of 8, state width <= 256, 2..8 transitions
+    h = ctypes.c_void_p()
+    assert lib.stacklstm_head_create(ctypes.byref(h), T, Tb, B, H, P, A, 0, None) == want
+    assert h.value is None
+
+
+def test_head_null_handle(lib):
+    assert lib.stacklstm_head_create(None, 4, 4, 2, 8, 8, 3, 0, None) == 1
+    assert lib.stacklstm_head_run(*([None] * 21)) == 1
+    assert lib.stacklstm_head_add_h0_grads(None, None, None) == 1
+    assert lib.stacklstm_head_status(None) == 1
+    assert lib.stacklstm_head_destroy(None) == 0
+    assert lib.stacklstm_head_last_error(None).decode() == "null handle"
