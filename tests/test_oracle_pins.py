@@ -184,6 +184,31 @@ def test_definition_equals_homogenized_live(seed):
         assert np.array_equal(rh["c_stack"][:live, b], rd["c_stack"][:live, b])
 
 
+@pytest.mark.parametrize("seed", range(4))
+def test_only_push_writes_are_ever_read(seed):
+    """Observation 2: a state written by a pop or a hold step (to slot p + 1, above the
+    top) is overwritten by the next push before the pointer reaches it, so the history
+    rows that are ever a top are exactly the initial state and the push steps' writes;
+    a brute-force list-stack replay of the slot contents agrees."""
+    rng = np.random.default_rng(100 + seed)
+    T, B = 60, 7
+    ops = wl.ops_random_walk(rng, B, T, (0.4, 0.35, 0.25))
+    src = oracle.pointers(ops)["src"]
+    for b in range(B):
+        read = set(src[:, b].tolist())
+        want = {0} | {t + 1 for t in range(T) if ops[t, b] == 1}
+        assert read == want
+        # replay: slots hold history rows; every step writes slot p + 1, then moves p
+        slots, p, tops = [0], 0, [0]
+        for t in range(T):
+            if len(slots) <= p + 1:
+                slots.append(None)
+            slots[p + 1] = t + 1
+            p += int(ops[t, b])
+            tops.append(slots[p])
+        assert tops == src[:, b].tolist()
+
+
 def test_dead_writes_get_zero_input_gradient():
     T, B, I, H = 40, 4, 5, 3
     c = rand_case(T, B, I, H, 11, probs=(0.4, 0.4, 0.2))
