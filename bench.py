@@ -113,7 +113,8 @@ def source_sha(fname):
 
 def kernel_traffic(kernel, fname, workload):
     """DRAM bytes per launch of `kernel` from the committed ncu summary, if it was taken
-    on this workload with the kernel source as it is now; else None."""
+    on this workload with the kernel source as it is now (or a later revision listed as
+    changing host code only); else None."""
     p = os.path.join(ROOT, "profiles", "dram_traffic.json")
     if not os.path.exists(p):
         return None
@@ -121,7 +122,8 @@ def kernel_traffic(kernel, fname, workload):
         d = json.load(f)
     sha = source_sha(fname)
     for e in d.get("entries", []):
-        if e.get("kernel") == kernel and e.get("workload") == workload and e.get("source_sha") == sha:
+        same = e.get("source_sha") == sha or sha in e.get("host_only_revisions", [])
+        if e.get("kernel") == kernel and e.get("workload") == workload and same:
             return e.get("dram_bytes_per_launch")
     return None
 
