@@ -214,9 +214,11 @@ sl_status stacklstm_pointers_noalloc(int T, int B, const int8_t *ops, int32_t *p
  *
  * stacklstm_head_create -- a head for T transitions (the stack and action StackLSTMs'
  *   step count), a buffer StackLSTM of Tb steps, B instances, hidden width H (a multiple
- *   of 8), state width P (<= 256) and A transitions (2..8). Owns its workspace (about
- *   T B (6H + 8P + 4A) bytes). Calls are ordered on `stream`; SL_ERR_ARG,
- *   SL_ERR_UNSUPPORTED or SL_ERR_OOM on failure, leaving *out NULL.
+ *   of 8), state width P (<= 256) and A transitions (2..8). Owns its workspace: about
+ *   T B (6H + 8P + 4A) bytes for the gathered tops, states and gradients, plus up to
+ *   16 x P x 3H floats of weight-gradient partial sums. Calls are ordered on `stream`;
+ *   SL_ERR_ARG (bad size or device), SL_ERR_UNSUPPORTED or SL_ERR_OOM on failure,
+ *   leaving *out NULL.
  */
 typedef struct stacklstm_head *stacklstm_head_t;
 sl_status stacklstm_head_create(stacklstm_head_t *out, int T, int Tb, int B, int H, int P, int A, int device,
