@@ -157,6 +157,28 @@ ARC_HYBRID_OPS = {"S": (PUSH, POP), "LA": (POP, HOLD), "RA": (POP, HOLD)}
 ARC_HYBRID_ACTIONS = ("S", "LA", "RA")
 
 
+def arc_hybrid_op_streams(seq, n: int) -> dict:
+    """The op streams of one sentence's transitions for the three StackLSTMs, and which
+    token each step's input is (-1: a zero input).
+
+    buffer: n pushes of tokens n - 1 .. 0 (token 0 ends on top), then per transition its
+    buffer op (input zero); stack: per transition its stack op, input the buffer-front
+    token (-1 once the buffer is empty); action: a push per transition."""
+    out = dict(stack_ops=[], stack_tok=[], buffer_ops=[PUSH] * n, buffer_tok=list(range(n - 1, -1, -1)),
+               action_ops=[])
+    front = 0
+    for tr in seq:
+        so, bo = ARC_HYBRID_OPS[tr]
+        out["stack_ops"].append(so)
+        out["stack_tok"].append(front if front < n else -1)
+        out["buffer_ops"].append(bo)
+        out["buffer_tok"].append(-1)
+        out["action_ops"].append(PUSH)
+        if tr == "S":
+            front += 1
+    return out
+
+
 # ------------------------------------------------------------------------- workload
 @dataclasses.dataclass
 class Workload:
@@ -285,19 +307,18 @@ def make_arc_hybrid(B: int, seed: int, H: int = 200, I_tok: int = 200, I_act: in
     x_b = np.zeros((Tb, B, I_tok), np.float32)
     trans = np.full((Ts, B), -1, np.int8)
     for b, (n, q) in enumerate(zip(ns, seqs)):
-        for i in range(n):  # the buffer: token n - 1 first, token 0 on top
-            ops_b[i, b] = PUSH
-            x_b[i, b] = rep[n - 1 - i, b]
-        front = 0  # index of the token at the buffer front
+        st = arc_hybrid_op_streams(q, n)
+        ops_b[: len(st["buffer_ops"]), b] = st["buffer_ops"]
+        ops_s[: len(q), b] = st["stack_ops"]
+        ops_a[: len(q), b] = st["action_ops"]
+        for t, tok in enumerate(st["buffer_tok"]):
+            if tok >= 0:
+                x_b[t, b] = rep[tok, b]
         for k, tr in enumerate(q):
-            so, bo = ARC_HYBRID_OPS[tr]
-            ops_s[k, b], ops_b[n + k, b], ops_a[k, b] = so, bo, PUSH
-            if front < n:
-                x_s[k, b] = rep[front, b]
+            if st["stack_tok"][k] >= 0:
+                x_s[k, b] = rep[st["stack_tok"][k], b]
             x_a[k, b] = emb[ARC_HYBRID_ACTIONS.index(tr)]
             trans[k, b] = ARC_HYBRID_ACTIONS.index(tr)
-            if tr == "S":
-                front += 1
     lens_s = np.array([len(q) for q in seqs], np.int32)
     lens_b = np.array([n + len(q) for n, q in zip(ns, seqs)], np.int32)
     if dtype == "bf16":

@@ -33,6 +33,43 @@ def replay(seq, n):
     return shifted, arcs
 
 
+def read_golden(name):
+    import os
+    out = {}
+    with open(os.path.join(os.path.dirname(__file__), "golden", name)) as f:
+        for line in f:
+            if line.strip() and not line.startswith("#"):
+                k, v = line.split(":", 1)
+                out[k.strip()] = v.split()
+    return out
+
+
+def test_golden_arc_hybrid_trace():
+    """A hand-derived arc-hybrid trace (tests/golden/arc_hybrid_trace.txt, from Table 1,
+    Sec. 3 and Algorithm 1): op streams, input tokens, pointer provenance, the arcs, and
+    the buffer top the head reads before each transition."""
+    g = read_golden("arc_hybrid_trace.txt")
+    seq, n = g["transitions"], 3
+    ints = lambda v: [int(x) for x in v]
+    tok = lambda v: [-1 if x == "-" else int(x) for x in v]
+    st = wl.arc_hybrid_op_streams(seq, n)
+    for k in ("stack_ops", "buffer_ops", "action_ops"):
+        assert st[k] == ints(g[k]), k
+    assert st["stack_tok"] == tok(g["stack_tok"]) and st["buffer_tok"] == tok(g["buffer_tok"])
+    src = {}
+    for name in ("stack", "buffer"):
+        ops = np.array(st[name + "_ops"], np.int8)[:, None]
+        src[name] = oracle.pointers(ops)["src"][:, 0]
+        assert list(src[name]) == ints(g[name + "_src"]), name
+    _, arcs = replay(seq, n)
+    assert ["%d>%d" % a for a in arcs] == g["arcs"]
+    for k in range(len(seq)):
+        row = n - 1 + k
+        assert row == int(g["head_buffer_row"][k])
+        h = int(src["buffer"][row + 1])  # the top after buffer step `row`
+        assert (st["buffer_tok"][h - 1] if h > 0 else -1) == tok(g["head_buffer_token"])[k]
+
+
 @pytest.mark.parametrize("seed", range(5))
 def test_arc_hybrid_transitions_are_valid_trees(seed):
     rng = np.random.default_rng(seed)
