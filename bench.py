@@ -6,11 +6,16 @@ steps (Algorithm 1) and the reverse-time backward with dx, dW and dbias. The met
 instance-steps per second, B * T per step (hold padding included: the homogenized
 method computes padded steps too).
 
-  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME] [--impl ours|reference]
+  python bench.py [--gpus 1] [--steps K] [--warmup W] [--workload NAME] [--impl ours|reference]
 
-Prints ONE JSON line (rank 0). Under torchrun each rank runs its own replica of the
-workload on its own GPU (instances are independent; no collective on the data path);
-the job value is all ranks' instance-steps over the slowest rank's time.
+Prints ONE JSON line. The headline is the parser-scale workload (B=64, I=H=200); unless
+--workload names one workload or --no-extra is given, the line also carries a full record
+(throughput, roofline, clocks, end-to-end rate, CPU baseline, step latency) for every
+other workload: tiny, each batch size of the sweep, large, stress, and the arc-hybrid
+parser batch. The library runs on one GPU: its one-row-tile kernels deliver operands
+between the CTAs of a thread-block cluster with multicast copies, which are for a
+process on one GPU; --gpus N > 1 (or a torchrun world larger than one) is refused
+before any library call.
 --impl reference times the fp64 CPU oracle on the host cores on the same workload.
 """
 from __future__ import annotations
@@ -18,9 +23,9 @@ from __future__ import annotations
 import argparse
 import hashlib
 import json
-import re
 import math
 import os
+import re
 import statistics
 import subprocess
 import sys
@@ -36,6 +41,12 @@ METRIC = "fwd+bwd StackLSTM instance-steps/s"
 UNIT = "instance-steps/s"
 L2_FLUSH_BYTES = 256 << 20  # > the 129 MB L2
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+# fp32 FFMA peak (the fp32 path runs on CUDA cores, TF32 off): 128 fp32 lanes per SM,
+# 2 flops per FFMA, at the maximum SM clock
+FP32_LANES_PER_SM = 128
+SIDE_WORKLOADS = ("tiny", "sweep:1", "sweep:8", "sweep:32", "sweep:128", "sweep:512", "sweep:1024", "large",
+                  "stress")
+DATA = "synthetic (seeded; shapes and op statistics of the parsing workloads, no treebank)"
 
 
 # ----------------------------------------------------------------------------- setup
@@ -50,11 +61,16 @@ def get_workload(name, T=None):
     return wl.config_workload(name, T=T)
 
 
+def wkey(w):
+    """Workload key: the config name, with the batch size for the sweep."""
+    return "sweep:%d" % w.B if w.name == "sweep" else w.name
+
+
 def describe(w):
     ops = {"tiny": "uniform valid push/pop/hold", "parser64": "random valid arc-standard sequences flattened to "
            "push/pop (n~U[10,60]), hold-padded", "large": "push/pop/hold .5/.3/.2, ragged lengths U[64,256], "
            "hold-padded", "stress": "push/pop/hold .6/.3/.1, all real steps", "sweep": "as parser64"}
-    return ("%s: B=%d T=%d I=%d H=%d, %s, seed %d" % (w.name, w.B, w.T, w.I, w.H, ops.get(w.name, ""), w.seed))
+    return ("%s: B=%d T=%d I=%d H=%d, %s, seed %d" % (wkey(w), w.B, w.T, w.I, w.H, ops.get(w.name, ""), w.seed))
 
 
 def load_peaks():
@@ -62,14 +78,25 @@ def load_peaks():
     if os.path.exists(p):
         with open(p) as f:
             d = json.load(f)
-        return {k: float(d[k]) for k in FALLBACK_PEAKS}, "measured"
-    return dict(FALLBACK_PEAKS), "fallback"
+        peaks = {k: float(d[k]) for k in FALLBACK_PEAKS}
+        peaks["sm_max_mhz"] = float(d.get("sm_max_mhz", 2070.0))
+        return peaks, "measured"
+    peaks = dict(FALLBACK_PEAKS)
+    peaks["sm_max_mhz"] = 2070.0
+    return peaks, "fallback"
 
 
 # ---------------------------------------------------------------- algorithmic work
-def work_per_inst_step(I, H):
-    """Flops and bytes per instance-step, per kernel phase and for the whole step (bf16
-    path). Whole step: F = 24 H (I + H), Q = 8 I + 46 H."""
+def work_per_inst_step(I, H, dtype="bf16"):
+    """Flops and bytes per instance-step, per kernel phase and for the whole step.
+    bf16 path: whole step F = 24 H (I + H), Q = 8 I + 46 H. fp32 path: the same flops,
+    Q = 12 I + 52 H (4-byte x, h and gates)."""
+    if dtype == "fp32":
+        return {"forward": {"flops": 8 * H * (I + H), "bytes": 4 * I + 16 * H},
+                "backward": {"flops": 8 * H * H, "bytes": 36 * H},
+                "dx": {"flops": 8 * H * I, "bytes": 4 * I},
+                "dw": {"flops": 8 * H * (I + H + 1), "bytes": 4 * I},
+                "step": {"flops": 24 * H * (I + H), "bytes": 12 * I + 52 * H}}
     return {
         "forward": {"flops": 8 * H * (I + H), "bytes": 2 * I + 12 * H},
         "backward": {"flops": 8 * H * H, "bytes": 34 * H},
@@ -79,31 +106,47 @@ def work_per_inst_step(I, H):
     }
 
 
-def roofline_of(work_flops, work_bytes, seconds, peaks, src, sustained):
-    tf_peak = peaks["bf16_tflops_sustained" if sustained else "bf16_tflops"]
-    t_tensor = work_flops / (tf_peak * 1e12)
+def roofline_of(work_flops, work_bytes, seconds, peaks, src, dtype="bf16", sms=152):
+    """The tighter of the contraction's compute roofline and the HBM byte roofline.
+    bf16: tensor cores at the measured burst bf16 rate (every timed region here is
+    milliseconds long). fp32: CUDA-core FFMA at the peak derived from the SM count, the
+    fp32 lanes per SM and the maximum SM clock."""
+    if dtype == "fp32":
+        peak_t = sms * FP32_LANES_PER_SM * 2 * peaks["sm_max_mhz"] * 1e6 / 1e12
+        bound_c, psrc = "alu", "derived fp32 FFMA: %d SMs x %d lanes x 2 flops x %.0f MHz" % (
+            sms, FP32_LANES_PER_SM, peaks["sm_max_mhz"])
+    else:
+        peak_t = peaks["bf16_tflops"]
+        bound_c, psrc = "tensor", "%s bf16 burst" % src
+    t_c = work_flops / (peak_t * 1e12)
     t_hbm = work_bytes / (peaks["hbm_gbs"] * 1e9)
-    if t_tensor >= t_hbm:
+    if t_c >= t_hbm:
         ach = work_flops / seconds / 1e12
-        return {"bound": "tensor", "achieved": ach, "peak": tf_peak, "unit": "TFLOP/s", "frac": ach / tf_peak,
-                "peak_source": "%s bf16 %s" % (src, "sustained" if sustained else "burst")}
+        return {"bound": bound_c, "achieved": ach, "peak": peak_t, "unit": "TFLOP/s", "frac": ach / peak_t,
+                "peak_source": psrc}
     ach = work_bytes / seconds / 1e9
     return {"bound": "hbm", "achieved": ach, "peak": peaks["hbm_gbs"], "unit": "GB/s",
             "frac": ach / peaks["hbm_gbs"], "peak_source": "%s HBM copy" % src}
 
 
-def phase_kernel(plan, phase):
-    """(kernel name, source file) of the kernel that does a phase's work, from the plan."""
+def phase_kernel(plan, phase, dtype):
+    """(kernel name, source file, launches per pass) of the kernel that does a phase's
+    work, from the plan."""
+    if dtype == "fp32":
+        return {"forward": ("fwd_step_f32", "fp32_path.cu", "T"),
+                "backward": ("bwd_pointwise_f32+bwd_contract_f32", "fp32_path.cu", "2T"),
+                "dx": ("dx_f32", "fp32_path.cu", 1), "dw": ("dw_f32", "fp32_path.cu", 1)}[phase]
     if phase in ("forward", "backward"):
         m = re.search(phase + r" (persistent|per-step|cluster) U=(\d+)", plan)
         if m and m.group(1) == "cluster":
-            return "%s<U=%s,%s>" % ("step_cl" if phase == "forward" else "step_clb", m.group(2), phase), "bf16_cluster.cu"
+            return ("%s<U=%s,%s>" % ("step_cl" if phase == "forward" else "step_clb", m.group(2), phase),
+                    "bf16_cluster.cu", 1)
         if m and m.group(1) == "persistent":
-            return "step_ws<U=%s,%s>" % (m.group(2), phase), "bf16_persist.cu"
-        return ("fwd_step_tc" if phase == "forward" else "bwd_step_tc"), "bf16_path.cu"
+            return "step_ws<U=%s,%s>" % (m.group(2), phase), "bf16_persist.cu", 1
+        return ("fwd_step_tc" if phase == "forward" else "bwd_step_tc"), "bf16_path.cu", "T"
     if phase == "dx":
-        return "dx_tc", "bf16_path.cu"
-    return "dw_ws", "bf16_dw.cu"
+        return "dx_tc", "bf16_path.cu", 1
+    return "dw_ws", "bf16_dw.cu", 1
 
 
 def source_sha(fname):
@@ -170,6 +213,7 @@ class ClockSampler:
             win = [r for _, r in self.rows][-3:]
         if not win:
             return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no nvidia-smi samples"], "samples": 0}
+
         def num(v):
             try:
                 return float(v)
@@ -185,72 +229,61 @@ class ClockSampler:
 
 
 # ------------------------------------------------------------------------- our arm
-def run_ours(args, rank, world, local):
+def run_ours(args):
     import torch
-    from paper_1904_03409_gb300 import binding as bd
-    from paper_1904_03409_gb300 import build, runner
+    from paper_1904_03409_gb300 import build
 
-    if world > 1:
-        import torch.distributed as dist
-        dist.init_process_group("gloo")
-        if rank == 0:
-            build.build()
-        dist.barrier()
-    else:
-        build.build()
-    torch.cuda.set_device(local)
-    dev = torch.device("cuda", local)
+    build.build()
+    torch.cuda.set_device(0)
     w = get_workload(args.workload, args.T)
-    res = measure_workload(w, args.steps, args.warmup, local, world, sample_clocks=True, e2e=True)
-
-    line = {"metric": METRIC, "value": res["value"], "unit": UNIT, "n_gpus": world, "steps": res["steps"],
-            "warmup": args.warmup, "ms_per_step": res["ms_per_step"], "higher_is_better": True,
-            "scaling": "weak", "vs_baseline": None, "dtype": "bf16" if w.dtype == "bf16" else "fp32",
-            "data": "synthetic (seeded; shapes and op statistics of the parsing workloads, no treebank)",
-            "config": {"workload": describe(w), "B": w.B, "T": w.T, "I": w.I, "H": w.H,
-                       "real_step_share": round(w.real_step_share, 4),
-                       "l2": "flushed between timed steps (256 MiB write outside the timed events)",
-                       "parallelism": "replicas" if world > 1 else "single GPU"},
-            "roofline": res["roofline"], "step_roofline": res["step_roofline"], "phases_ms_per_step":
-            res["phases"], "e2e": res["e2e"], "gpu_launches": res["gpu_launches"], "clocks": res["clocks"],
-            "plan": res["plan"]}
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        line["cpu_baseline"] = cpu_baseline(w, args.cpu_seconds)
-    if rank == 0 and world == 1 and not args.no_extra and args.workload == "parser64":
-        line["other_workloads"] = {}
-        for name in ("large", "stress"):
+    rec = measure_record(w, args.steps, args.warmup, args.cpu_seconds, not args.no_cpu_baseline, min_seconds=0.0)
+    line = {"metric": METRIC, "value": rec.pop("value"), "unit": UNIT, "n_gpus": 1, "steps": rec.pop("steps"),
+            "warmup": args.warmup, "ms_per_step": rec.pop("ms_per_step"), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16" if w.dtype == "bf16" else "f32",
+            "data": DATA, "config": rec.pop("config")}
+    line.update(rec)
+    if not args.no_extra and args.workload == "parser64" and args.T is None:
+        line["workloads"] = {}
+        for name in SIDE_WORKLOADS:
             torch.cuda.empty_cache()
             wx = get_workload(name)
-            r = measure_workload(wx, 5, 3, local, 1, sample_clocks=False, e2e=False)
-            line["other_workloads"][name] = {"workload": describe(wx), "value": r["value"],
-                                             "ms_per_step": r["ms_per_step"], "steps": 5, "warmup": 3,
-                                             "roofline": r["roofline"], "step_roofline": r["step_roofline"],
-                                             "phases_ms_per_step": r["phases"]}
+            line["workloads"][name] = measure_record(wx, max(20, args.steps), args.warmup, args.side_cpu_seconds,
+                                                     not args.no_cpu_baseline, min_seconds=0.3)
             del wx
         torch.cuda.empty_cache()
-        line["other_workloads"]["arc_hybrid64"] = measure_group("arc_hybrid64", 20, 3, local)
+        line["workloads"]["arc_hybrid64"] = measure_group("arc_hybrid64", max(20, args.steps), args.warmup)
         torch.cuda.empty_cache()
-        line["other_workloads"]["parser_step64"] = measure_parser("arc_hybrid64", 20, 3, local)
-    if rank == 0:
-        print(json.dumps(line), flush=True)
-    if world > 1:
-        import torch.distributed as dist
-        dist.barrier()
-        dist.destroy_process_group()
+        line["workloads"]["parser_step64"] = measure_parser("arc_hybrid64", max(20, args.steps), args.warmup)
+    print(json.dumps(line), flush=True)
 
 
-def measure_workload(w, steps, warmup, local, world, sample_clocks, e2e):
+def measure_record(w, steps, warmup, cpu_seconds, with_cpu, min_seconds):
+    """One workload's full record: device-timed throughput with the clocks seen during
+    the timed region, the roofline of its dominant kernel and of the whole step, the
+    end-to-end rate through host buffers, per-step latency, and the oracle on the host
+    cores as a baseline."""
+    res = measure_workload(w, steps, warmup, min_seconds)
+    res["config"] = {"workload": describe(w), "B": w.B, "T": w.T, "I": w.I, "H": w.H,
+                     "real_step_share": round(w.real_step_share, 4),
+                     "l2": "flushed between timed steps (256 MiB write outside the timed events)",
+                     "parallelism": "single GPU"}
+    if with_cpu:
+        res["cpu_baseline"] = cpu_baseline(w, cpu_seconds)
+    return res
+
+
+def measure_workload(w, steps, warmup, min_seconds=0.0):
     import torch
     from paper_1904_03409_gb300 import binding as bd
     from paper_1904_03409_gb300 import runner
 
-    dev = torch.device("cuda", local)
+    dev = torch.device("cuda", 0)
     stream = torch.cuda.current_stream(dev)
-    hd = bd.stacklstm_create(w.T, w.B, w.I, w.H, bd.SL_BF16 if w.dtype == "bf16" else bd.SL_FP32, local, stream)
+    hd = bd.stacklstm_create(w.T, w.B, w.I, w.H, bd.SL_BF16 if w.dtype == "bf16" else bd.SL_FP32, 0, stream)
     plan = bd.stacklstm_plan(hd)
     bd.stacklstm_set_async(hd, True)
-    ins = runner.upload(w, local)
-    out = runner.alloc_outputs(w, local, forward_outputs=False)
+    ins = runner.upload(w, 0)
+    out = runner.alloc_outputs(w, 0, forward_outputs=False)
     flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
 
     def step():
@@ -259,77 +292,72 @@ def measure_workload(w, steps, warmup, local, world, sample_clocks, e2e):
     for _ in range(max(1, warmup)):
         step()
     bd.stacklstm_status(hd)
-    if steps <= 0:  # auto: about 2 s of timed work
+    if steps <= 0 or min_seconds > 0:  # auto (or a floor): time enough steps for the clock samples
         t0 = time.time()
         step()
         bd.stacklstm_status(hd)
-        steps = int(min(2000, max(10, math.ceil(2.0 / max(time.time() - t0, 1e-4)))))
+        one = max(time.time() - t0, 1e-5)
+        want = 2.0 if steps <= 0 else min_seconds
+        steps = int(min(2000, max(steps, 10, math.ceil(want / one))))
 
     bd.stacklstm_set_timing(hd, True)
     launches0 = hd_launches(hd)
     evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
-    clocks = ClockSampler(local) if sample_clocks else None
-    if clocks:
-        time.sleep(0.3)
-    barrier(world)
+    clocks = ClockSampler(0)
+    time.sleep(0.3)
     torch.cuda.synchronize(dev)
-    if clocks:
-        clocks.start()
+    clocks.start()
     for i in range(steps):
         flush.zero_()
         evs[i][0].record(stream)
         step()
         evs[i][1].record(stream)
     torch.cuda.synchronize(dev)
-    if clocks:
-        clocks.stop()
-    barrier(world)
+    clocks.stop()
     bd.stacklstm_status(hd)
     total_ms = sum(a.elapsed_time(b) for a, b in evs)
-    total_ms = max_over_ranks(total_ms, world)
     timing = bd.stacklstm_get_timing(hd)
     n_launch = hd_launches(hd) - launches0
     bd.stacklstm_set_timing(hd, False)
 
     peaks, src = load_peaks()
-    wk = work_per_inst_step(w.I, w.H)
+    sms = torch.cuda.get_device_properties(dev).multi_processor_count
+    wk = work_per_inst_step(w.I, w.H, w.dtype)
     phase_ms = {p: timing[p][0] / steps for p in timing}
     dom = max(("forward", "backward", "dx", "dw"), key=lambda p: phase_ms[p])
-    kname, kfile = phase_kernel(plan, dom)
-    # a persistent step kernel is one launch over all T steps; the per-step kernels are T
-    # launches of B instance-steps each; dx and dW are one contraction over all T * B rows
-    # (dW: plus its fixed-order reduction of the split partials)
-    per_step_kernels = dom in ("forward", "backward") and "step_ws" not in kname and "step_cl" not in kname
-    per_launch_units = w.B if per_step_kernels else w.B * w.T
-    launches_per_step = w.T if per_step_kernels else 1
-    launch_s = phase_ms[dom] / 1e3 / launches_per_step
+    kname, kfile, lpp = phase_kernel(plan, dom, w.dtype)
+    # a persistent or cluster step kernel is one launch over all T steps; the per-step
+    # kernels are T (or 2T) launches of B instance-steps each; dx and dW are one
+    # contraction over all T * B rows (dW: plus its fixed-order reduction of the partials)
+    launches_per_pass = {"T": w.T, "2T": 2 * w.T}.get(lpp, lpp)
+    per_launch_units = w.B * w.T / launches_per_pass
+    launch_s = phase_ms[dom] / 1e3 / launches_per_pass
     fl, by = wk[dom]["flops"], wk[dom]["bytes"]
     m = re.search(r"dx CTAs (\d+)", plan)
     if dom == "backward" and m and int(m.group(1)) > 0:
         # the backward launch also computed dx on the SMs its step chain leaves idle
         fl, by = fl + wk["dx"]["flops"], by + wk["dx"]["bytes"]
         kname += "+dx"
-    rf = roofline_of(fl * per_launch_units, by * per_launch_units, launch_s, peaks, src, sustained=True)
+    rf = roofline_of(fl * per_launch_units, by * per_launch_units, launch_s, peaks, src, w.dtype, sms)
     rf.update({"kernel": kname, "phase": dom, "launch_us": launch_s * 1e6,
-               "units_per_launch": per_launch_units, "unit_of_work": "instance-step",
-               "algorithmic_flops_per_unit": fl, "algorithmic_bytes_per_unit": by,
-               "traffic": kernel_traffic(kname, kfile, w.name)})
+               "launches_per_pass": launches_per_pass, "units_per_launch": per_launch_units,
+               "unit_of_work": "instance-step", "algorithmic_flops_per_unit": fl,
+               "algorithmic_bytes_per_unit": by, "traffic": kernel_traffic(kname, kfile, wkey(w))})
     sec = total_ms / 1e3 / steps
-    srf = roofline_of(wk["step"]["flops"] * w.B * w.T, wk["step"]["bytes"] * w.B * w.T, sec, peaks, src,
-                      sustained=True)
-    res = {"value": world * w.B * w.T * steps / (total_ms / 1e3), "ms_per_step": total_ms / steps, "steps": steps,
-           "roofline": rf, "step_roofline": srf, "phases": {p: round(v, 4) for p, v in phase_ms.items()},
-           "plan": plan,
-           "gpu_launches": int(n_launch), "clocks": clocks.summary() if clocks else None}
-    if e2e:
-        res["e2e"] = measure_e2e(w, hd, ins, out, steps, world, local, flush)
+    srf = roofline_of(wk["step"]["flops"] * w.B * w.T, wk["step"]["bytes"] * w.B * w.T, sec, peaks, src, w.dtype, sms)
+    res = {"value": w.B * w.T * steps / (total_ms / 1e3), "ms_per_step": total_ms / steps, "steps": steps,
+           "roofline": rf, "step_roofline": srf, "phases_ms_per_step": {p: round(v, 4) for p, v in phase_ms.items()},
+           "step_latency_us": {"forward": 1e3 * phase_ms["forward"] / w.T,
+                               "backward": 1e3 * (phase_ms["backward"] + phase_ms["dx"]) / w.T},
+           "plan": plan, "gpu_launches": int(n_launch), "clocks": clocks.summary()}
+    res["e2e"] = measure_e2e(w, hd, ins, out, steps, flush)
     hd.destroy()
     del ins, out, flush
     torch.cuda.empty_cache()
     return res
 
 
-def measure_group(name, steps, warmup, local):
+def measure_group(name, steps, warmup):
     """The three StackLSTMs of an arc-hybrid parser batch (stack, buffer, action history),
     forward + backward at the same time, one stream each; against the same three timed one
     at a time. value = instance-steps of all three / second."""
@@ -337,11 +365,11 @@ def measure_group(name, steps, warmup, local):
     from paper_1904_03409_gb300 import runner, workloads as wl
 
     g = wl.make_arc_hybrid(**wl.GROUPS[name])
-    dev = torch.device("cuda", local)
+    dev = torch.device("cuda", 0)
     cur = torch.cuda.current_stream(dev)
-    hds = runner.create_group(g, local)
-    ins = {k: runner.upload(g[k], local) for k in runner.GROUP_MEMBERS}
-    outs = {k: runner.alloc_outputs(g[k], local, forward_outputs=False) for k in runner.GROUP_MEMBERS}
+    hds = runner.create_group(g, 0)
+    ins = {k: runner.upload(g[k], 0) for k in runner.GROUP_MEMBERS}
+    outs = {k: runner.alloc_outputs(g[k], 0, forward_outputs=False) for k in runner.GROUP_MEMBERS}
     flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
     for _ in range(max(1, warmup)):
         runner.group_forward_backward(hds, ins, outs)
@@ -367,7 +395,11 @@ def measure_group(name, steps, warmup, local):
         runner.group_status(hds)
         return sum(x.elapsed_time(y) for x, y in evs) / steps
 
+    clocks = ClockSampler(0)
+    time.sleep(0.3)
+    clocks.start()
     ms = timed(None)
+    clocks.stop()
     alone = {k: timed(k) for k in runner.GROUP_MEMBERS}
     units = sum(g[k].B * g[k].T for k in runner.GROUP_MEMBERS)
     peaks, src = load_peaks()
@@ -381,7 +413,7 @@ def measure_group(name, steps, warmup, local):
            "transitions_per_s": g["stack"].B * g["stack"].T / (ms / 1e3),
            "ms_per_step": ms, "ms_one_at_a_time": {k: round(v, 4) for k, v in alone.items()},
            "overlap_speedup": round(sum(alone.values()) / ms, 3), "steps": steps, "warmup": warmup,
-           "step_roofline": roofline_of(fl, by, ms / 1e3, peaks, src, sustained=True)}
+           "step_roofline": roofline_of(fl, by, ms / 1e3, peaks, src), "clocks": clocks.summary()}
     for hd, _ in hds.values():
         hd.destroy()
     del ins, outs, flush
@@ -389,7 +421,7 @@ def measure_group(name, steps, warmup, local):
     return res
 
 
-def measure_parser(name, steps, warmup, local):
+def measure_parser(name, steps, warmup):
     """A whole parser training step of the recurrent part on an arc-hybrid batch: the three
     StackLSTM forwards at the same time, the parser head (200-wide ReLU state, softmax over
     the transitions, cross-entropy), the three backwards seeded by the head's gradients.
@@ -398,15 +430,18 @@ def measure_parser(name, steps, warmup, local):
     from paper_1904_03409_gb300 import runner, workloads as wl
 
     g = wl.make_arc_hybrid(**wl.GROUPS[name])
-    dev = torch.device("cuda", local)
+    dev = torch.device("cuda", 0)
     cur = torch.cuda.current_stream(dev)
-    ps = runner.create_parser(g, local)
+    ps = runner.create_parser(g, 0)
     flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
     for _ in range(max(1, warmup)):
         runner.parser_step(ps)
     torch.cuda.synchronize(dev)
     runner.group_status(ps["hds"])
     evs = []
+    clocks = ClockSampler(0)
+    time.sleep(0.3)
+    clocks.start()
     for _ in range(steps):
         flush.zero_()
         a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -415,6 +450,7 @@ def measure_parser(name, steps, warmup, local):
         b.record(cur)
         evs.append((a, b))
     torch.cuda.synchronize(dev)
+    clocks.stop()
     runner.group_status(ps["hds"])
     ms = sum(x.elapsed_time(y) for x, y in evs) / steps
     st = g["stack"]
@@ -424,7 +460,7 @@ def measure_parser(name, steps, warmup, local):
                        "StackLSTMs' backward seeded only by the head" % (name, st.B, hp["P"], hp["A"]),
            "value": st.B * st.T / (ms / 1e3), "unit": "instance-transitions/s (padded, T=%d)" % st.T,
            "real_transitions_per_s": float(g["L"].sum()) / (ms / 1e3), "ms_per_step": ms, "steps": steps,
-           "warmup": warmup}
+           "warmup": warmup, "clocks": clocks.summary()}
     runner.destroy_parser(ps)
     del ps, flush
     torch.cuda.empty_cache()
@@ -436,13 +472,13 @@ def hd_launches(hd):
     return sum(v[1] for v in bd.stacklstm_get_timing(hd).values())
 
 
-def measure_e2e(w, hd, ins, out, steps, world, local, flush):
+def measure_e2e(w, hd, ins, out, steps, flush):
     """Same metric through the ABI with the step's inputs copied from pinned host memory
     and its results (all gradients, final pointers) read back, inside the timed events."""
     import torch
     from paper_1904_03409_gb300 import runner
 
-    dev = torch.device("cuda", local)
+    dev = torch.device("cuda", 0)
     stream = torch.cuda.current_stream(dev)
     keys_in = ["x", "ops", "h0", "c0", "W", "bias", "d_top_h"]
     keys_out = ["p_final", "dx", "dh0", "dc0", "dW", "dbias"]
@@ -452,7 +488,6 @@ def measure_e2e(w, hd, ins, out, steps, world, local, flush):
     d2h = sum(t.numel() * t.element_size() for t in host_out.values())
     n = max(3, min(steps, 50))
     evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n)]
-    barrier(world)
     torch.cuda.synchronize(dev)
     for i in range(n):
         flush.zero_()
@@ -464,26 +499,9 @@ def measure_e2e(w, hd, ins, out, steps, world, local, flush):
             host_out[k].copy_(out[k], non_blocking=True)
         evs[i][1].record(stream)
     torch.cuda.synchronize(dev)
-    barrier(world)
-    total = max_over_ranks(sum(a.elapsed_time(b) for a, b in evs), world)
-    return {"value": world * w.B * w.T * n / (total / 1e3), "unit": UNIT, "h2d_bytes_per_step": int(h2d),
+    total = sum(a.elapsed_time(b) for a, b in evs)
+    return {"value": w.B * w.T * n / (total / 1e3), "unit": UNIT, "h2d_bytes_per_step": int(h2d),
             "d2h_bytes_per_step": int(d2h), "steps": n}
-
-
-def barrier(world):
-    if world > 1:
-        import torch.distributed as dist
-        dist.barrier()
-
-
-def max_over_ranks(v, world):
-    if world == 1:
-        return v
-    import torch
-    import torch.distributed as dist
-    t = torch.tensor([v], dtype=torch.float64)
-    dist.all_reduce(t, op=dist.ReduceOp.MAX)
-    return float(t.item())
 
 
 # ------------------------------------------------------------------ CPU (oracle)
@@ -497,7 +515,7 @@ def oracle_sample(w, seconds):
     oracle.run_instances(one, w.x, w.ops, w.h0, w.c0, w.W, w.bias, d_top_h=w.d_top_h, nthreads=1)
     t1 = max(time.time() - t0, 1e-6)
     n = int(max(1, min(w.B, math.floor(seconds * cores / t1))))
-    return list(range(n)), cores
+    return list(range(n)), min(cores, n)
 
 
 def run_oracle(w, inst, cores):
@@ -518,9 +536,7 @@ def cpu_baseline(w, seconds):
                       % (len(inst), w.B, reps, w.T, el)}
 
 
-def run_reference(args, rank, world):
-    if rank != 0:
-        return
+def run_reference(args, world):
     w = get_workload(args.workload, args.T)
     inst, cores = oracle_sample(w, args.ref_step_seconds)
     for _ in range(args.warmup):
@@ -531,8 +547,7 @@ def run_reference(args, rank, world):
     sample = "%d of %d instances per step (all T=%d steps, forward + backward, fp64)" % (len(inst), w.B, w.T)
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
             "steps": len(times), "warmup": args.warmup, "ms_per_step": 1e3 * el / len(times),
-            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-            "data": "synthetic (seeded; shapes and op statistics of the parsing workloads, no treebank)",
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": DATA,
             "config": {"workload": describe(w), "B": w.B, "T": w.T, "I": w.I, "H": w.H,
                        "reference": "fp64 CPU oracle (plain C, one instance at a time), host cores"},
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": sample},
@@ -542,27 +557,33 @@ def run_reference(args, rank, world):
 
 def main():
     ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
-    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--gpus", type=int, default=1, help="must be 1: the library runs on one GPU")
     ap.add_argument("--steps", type=int, default=0, help="timed steps (0: about 2 s of work)")
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
     ap.add_argument("--workload", default="parser64", help="tiny | parser64 | large | stress | sweep:B")
-    ap.add_argument("--cpu-seconds", type=float, default=10.0, help="oracle CPU-baseline budget")
+    ap.add_argument("--cpu-seconds", type=float, default=10.0, help="oracle CPU-baseline budget (headline)")
+    ap.add_argument("--side-cpu-seconds", type=float, default=3.0, help="oracle CPU-baseline budget (others)")
     ap.add_argument("--ref-step-seconds", type=float, default=3.0, help="oracle work per reference step")
-    ap.add_argument("--no-extra", action="store_true", help="skip the large/stress side measurements")
+    ap.add_argument("--no-extra", action="store_true", help="the named workload only")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--T", type=int, default=None,
                     help="fewer steps for tiny/large/stress (a smaller case of the same shape, for profiling)")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
-    rank, world, local = dist_env()
-    if world != args.gpus and world > 1:
-        print("warning: WORLD_SIZE=%d but --gpus %d" % (world, args.gpus), file=sys.stderr)
+    rank, world, _ = dist_env()
     if args.impl == "reference":
-        run_reference(args, rank, world)
-    else:
-        run_ours(args, rank, world, local)
+        # the oracle runs on the host cores: rank 0 alone under torchrun
+        if rank == 0:
+            run_reference(args, world)
+        return
+    if args.gpus != 1 or world > 1:
+        print("bench.py: this library runs on one GPU (its one-row-tile kernels use cluster multicast "
+              "copies, which are for a process on one GPU); run it with --gpus 1 and no torchrun world",
+              file=sys.stderr)
+        sys.exit(2)
+    run_ours(args)
 
 
 if __name__ == "__main__":

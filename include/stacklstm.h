@@ -37,6 +37,23 @@
  *            and all accumulations are fp32. Requires I % 8 == 0 and H % 8 == 0.
  *   c0, c_stack, bias and every gradient are float in both modes.
  */
+/*
+ * Test hooks. stacklstm_create reads these environment variables; they exist so that the
+ * tests can reach every kernel plan the library has on shapes where the planner would pick
+ * another one. Results are the same under every setting (within the stated tolerances);
+ * only speed changes. Unset, the planner decides.
+ *   STACKLSTM_WAIT_LIMIT_CYCLES=n  clock budget of one bounded device-side wait
+ *                                  (default 4e9); 0 makes every wait run out at once, so
+ *                                  calls report SL_ERR_TIMEOUT
+ *   STACKLSTM_STEP_KERNELS=1       one launch per time step instead of the persistent and
+ *                                  cluster kernels
+ *   STACKLSTM_FWD_CLUSTER=0        no thread-block-cluster forward for one row tile
+ *   STACKLSTM_BWD_CLUSTER=0        no thread-block-cluster backward for one row tile
+ *   STACKLSTM_BWD_SPLIT=k          the persistent backward with its 4H contraction split
+ *                                  over k CTAs per 64-unit column tile (k = 4)
+ *   STACKLSTM_DX_SPARE=0 | k       dx in its own launch (0), or by at most k extra CTAs of
+ *                                  the persistent backward launch
+ */
 #ifndef STACKLSTM_H
 #define STACKLSTM_H
 
@@ -174,26 +191,28 @@ const char *stacklstm_last_error(stacklstm_t s);
 
 /*
  * stacklstm_pointers_noalloc -- the index prepass alone (pointer trajectory and read
- * provenance of every instance), for callers that cannot allocate device memory: code
- * running while a stream is being captured into a CUDA graph (a cudaMalloc there is not
- * a stream operation and breaks or is refused by the capture), and services whose
- * memory is fully reserved up front by a pooling allocator, where a library's own
- * cudaMalloc fails or synchronizes the device mid-pipeline. It needs no handle and
- * allocates nothing: it calls no cudaMalloc, cudaFree or allocating routine.
+ * provenance of every instance), for callers that cannot allocate device memory when
+ * they need it: services whose device memory is all reserved up front by a pooling
+ * allocator (a library's own cudaMalloc then fails, or takes memory the pool counted
+ * on), and callers that must not let a cudaMalloc or cudaFree synchronize the device
+ * while other streams are busy. It needs no handle and allocates nothing: it calls no
+ * cudaMalloc, cudaFree or allocating routine.
  * The paper has no counterpart; it is a convenience of this library.
  *   T, B     sizes; (T + 1) * B must not exceed 1,048,576, else SL_ERR_UNSUPPORTED
  *   ops      [T, B] int8 device pointer, ops in {-1, 0, +1}
  *   p_traj   [T + 1, B] int32 device output, as stacklstm_forward's p_traj
  *   src      [T + 1, B] int32 device output, as stacklstm_forward's src
- *   stream   cudaStream_t (NULL = legacy default stream); the call synchronizes it
+ *   stream   cudaStream_t (NULL = legacy default stream)
+ * The three pointers must belong to the current device, which runs the kernel. The call
+ * enqueues the prepass on `stream`, then reads its status word back to the host and
+ * synchronizes `stream` before it returns.
  * Returns SL_OK, SL_ERR_OP / SL_ERR_UNDERFLOW (bad op stream; indices are still written,
  * bad ops run as holds), SL_ERR_ARG, SL_ERR_UNSUPPORTED or SL_ERR_CUDA.
  * Scratch: an 8 MiB array in the library's device memory, held on every GPU that loads
  * the library until the process exits. All calls share it, so calls that overlap on a
  * GPU (other streams, other host threads) race; it keeps the previous call's contents
  * and the call itself clears what must start at zero. The first call on a device looks
- * up the array's device address (a one-time set-up): make that first call before any
- * stream capture begins.
+ * up the array's device address (a one-time set-up on that device).
  */
 sl_status stacklstm_pointers_noalloc(int T, int B, const int8_t *ops, int32_t *p_traj, int32_t *src,
                                      void *stream);

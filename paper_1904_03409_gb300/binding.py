@@ -184,16 +184,19 @@ def stacklstm_backward(hd: StackLSTMHandle, d_top_h=None, dy=None, dx=None, dh0=
 def stacklstm_pointers_noalloc(ops, p_traj, src, stream=None):
     """Pointer trajectory and read provenance of an op stream without a handle and without
     any device allocation (see include/stacklstm.h). ops [T, B] int8, p_traj and src
-    [T+1, B] int32, all on the current CUDA device."""
+    [T+1, B] int32, all on one CUDA device, which is made current for the call."""
     import torch
     T, B = ops.shape
     d = ops.device.index
     if stream is None:
         stream = torch.cuda.current_stream(d)
     raw = stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream)
+    if hasattr(stream, "device") and stream.device.index != d:
+        raise ValueError("stream must belong to cuda:%d, the device of ops" % d)
     args = [_ptr(ops, d, torch.int8, (T, B), "ops"), _ptr(p_traj, d, torch.int32, (T + 1, B), "p_traj"),
             _ptr(src, d, torch.int32, (T + 1, B), "src")]
-    st = load().stacklstm_pointers_noalloc(T, B, *args, ctypes.c_void_p(raw))
+    with torch.cuda.device(d):  # the library launches on the current device
+        st = load().stacklstm_pointers_noalloc(T, B, *args, ctypes.c_void_p(raw))
     if st != 0:
         raise StackLSTMError(st, "stacklstm_pointers_noalloc")
 

@@ -788,7 +788,7 @@ __global__ void __launch_bounds__(kClBwdThreads, 1) step_clb(ClArgs p)
 
 // One row tile (B <= 64), at most 16 column tiles of 16 units, the footprint within the
 // shared-memory cap, and a cluster of that size co-resident on this GPU;
-// STACKLSTM_FWD_CLUSTER=0 turns it off.
+// STACKLSTM_FWD_CLUSTER=0 turns it off (test hook, include/stacklstm.h).
 bool bf16_plan_fwd_cluster(stacklstm *s, PersistPlan *pl)
 {
     pl->on = 0;
@@ -859,7 +859,8 @@ cudaError_t bf16_launch_fwd_cluster(stacklstm *s, const StepArgs &a, const CUten
 }
 
 // The backward of one row tile as a cluster: B <= 64, at most 16 column tiles of 16 units,
-// a co-resident cluster of that size; STACKLSTM_BWD_CLUSTER=0 turns it off. (Copying each CTA's 8 KB of dG into every CTA with bulk copies instead of
+// a co-resident cluster of that size; STACKLSTM_BWD_CLUSTER=0 turns it off (test hook,
+// include/stacklstm.h). (Copying each CTA's 8 KB of dG into every CTA with bulk copies instead of
 // the multicast tensor loads ran 30 % slower than the persistent backward at B = 64,
 // H = 200: n_ct^2 copies a step, issued one after another by one thread of each CTA.)
 bool bf16_plan_bwd_cluster(stacklstm *s, PersistPlan *pl)

@@ -279,17 +279,8 @@ cudaError_t bf16_plan_dw(stacklstm *s)
     const size_t tiles = (size_t)n_mt * s->dw_nt, want = 4 * (size_t)sms;  // two waves of two CTAs per SM
     const size_t max_split = std::max<size_t>(1, RC / 16);
     s->dw_split = (int)std::min(max_split, std::max<size_t>(1, ceil_div(want, tiles)));
-    // STACKLSTM_DW_NT / STACKLSTM_DW_SPLIT / STACKLSTM_DW_S pin the tile width, splits, stages
-    if (const char *v = getenv("STACKLSTM_DW_NT")) {
-        s->dw_ntile = atoi(v) == 256 ? 256 : 512;
-        s->dw_nt = (int)ceil_div(4 * H, s->dw_ntile);
-    }
-    if (const char *v = getenv("STACKLSTM_DW_SPLIT")) s->dw_split = std::max(1, std::min(atoi(v), (int)RC));
     s->dw_mt = n_mt;
     s->sw = 2;
-    if (const char *v = getenv("STACKLSTM_DW_S"))
-        s->sw = std::max(2, std::min<int>(atoi(v), (int)((kSmemCap - dw_smem_bytes(0, s->dw_ntile)) /
-                                                         dw_stage_bytes(s->dw_ntile))));
     s->dw_part_elems = (size_t)s->dw_split * ((size_t)n_mt * 128 + 1) * ((size_t)s->dw_nt * s->dw_ntile);
     cudaError_t e;
     if ((e = allow_smem(dw_ws<512>)) || (e = allow_smem(dw_ws<256>))) return e;

@@ -580,6 +580,7 @@ cudaError_t bf16_prepare(stacklstm *s)
     s->nx = pick_dx_n(I);
     s->nxt = (int)ceil_div(I, s->nx);
     const size_t R = (size_t)T * B;
+    // test hook (include/stacklstm.h): the clock budget of one device-side wait
     const char *lim = getenv("STACKLSTM_WAIT_LIMIT_CYCLES");
     s->wait_limit = lim ? atoll(lim) : 4000000000LL;
     if ((e = allow_smem(fwd_step_tc<32>)) || (e = allow_smem(fwd_step_tc<16>)) || (e = allow_smem(fwd_step_tc<8>)) ||
@@ -588,7 +589,8 @@ cudaError_t bf16_prepare(stacklstm *s)
         return e;
     if ((e = bf16_plan_dw(s))) return e;
 
-    // persistent step kernels unless disabled (STACKLSTM_STEP_KERNELS=1 keeps one launch per step)
+    // persistent step kernels unless disabled (test hook, include/stacklstm.h:
+    // STACKLSTM_STEP_KERNELS=1 keeps one launch per step)
     const char *per_step = getenv("STACKLSTM_STEP_KERNELS");
     if (!(per_step && atoi(per_step) != 0)) {
         if (bf16_plan_fwd_persist(s, &s->pf)) s->uf = s->pf.U;
@@ -637,7 +639,6 @@ cudaError_t bf16_prepare(stacklstm *s)
         s->split_cnt = (int32_t *)p;
     }
     if (s->pf.on || s->pb.on) {
-        if (const char *cs = getenv("STACKLSTM_CNT_STRIDE")) s->cnt_stride = std::max(1, atoi(cs));
         if ((e = cudaMalloc(&p, 2 * sizeof(int32_t) * rt * s->cnt_stride))) return e;
         s->allocs.push_back(p);
         s->rowcnt = (int32_t *)p;

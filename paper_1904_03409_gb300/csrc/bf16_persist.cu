@@ -25,11 +25,6 @@
 // stores and polled with acquire semantics (a bounded spin) by the producer before it
 // loads the dependent chunks. All CTAs are co-resident (cooperative launch), so the spins
 // end; every wait is bounded and a timeout aborts the whole grid through the error word.
-//
-// With cl > 1 the cl CTAs of a thread-block cluster hold cl consecutive column tiles of
-// the same row tiles and share the A operand: chunk c is loaded by cluster rank c mod cl
-// and multicast into the same stage of every CTA; `empty` counts cl arrivals because each
-// CTA commits its MMA completion to the `empty` barrier of every CTA of the cluster.
 #include <stdio.h>
 
 #include <algorithm>
@@ -45,7 +40,6 @@ struct WsArgs {
     StepArgs s;              // s.kcx: chunks before the dependent ones; s.S: ring stages
     int n_ct, n_rt, n_slot;  // column tiles (a multiple of cl); row tiles; CTAs per column tile
     int w_res;               // 1: weight tile resident in shared memory
-    int cl;                  // cluster size along the column tiles (1: no multicast)
     int32_t *cnt;            // [n_rt] completed steps per row tile (cs ints apart), zero at launch
     int cs;                  // counter stride in ints
     int vec32;               // H % 16 == 0: 16-unit groups of 16-bit rows are 32-byte aligned
@@ -879,8 +873,7 @@ step_ws(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtens
     const int dep_c = split > k0 ? split : k0;            // first chunk that needs step t - 1
     const WCtl c = wcarve(smem_raw, S, G, NB, (KC + KS - 1) / KS, p.w_res, ws_stg_bytes(kFwd, U));
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int ct = cidx % p.n_ct, slot = cidx / p.n_ct, cl = p.cl;
-    const uint32_t rank = cl > 1 ? tc::cluster_rank() : 0;
+    const int ct = cidx % p.n_ct, slot = cidx / p.n_ct;
     const int n_mine = slot < p.n_rt ? (p.n_rt - slot + p.n_slot - 1) / p.n_slot : 0;
     const int n_tiles = T * n_mine;
     const long long limit = a.limit;
@@ -892,7 +885,7 @@ step_ws(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtens
     if (tid == 0) {
         for (int s = 0; s < S; ++s) {
             tc::mbar_init(&c.full[s], 1);
-            tc::mbar_init(&c.empty[s], (uint32_t)cl);
+            tc::mbar_init(&c.empty[s], 1);
         }
         for (int i = 0; i < 2; ++i) {
             tc::mbar_init(&c.tfull[i], 1);
@@ -908,7 +901,6 @@ step_ws(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtens
     if (warp == E) tc::tmem_alloc(c.tmem_slot, 2 * kCols);
     tc::tc_fence_before();
     __syncthreads();
-    if (cl > 1) tc::cluster_sync();
     tc::tc_fence_after();
     const uint32_t tmem = *c.tmem_slot;
     const uint8_t *wtile = a.wpack + (size_t)ct * KC * bchunk;
@@ -948,10 +940,7 @@ step_ws(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtens
                         const CUtensorMap *tm = first ? &tm_a : &tm_b;
                         const int col = (first ? cc : cc - split) * kChunk;
                         const uint32_t dst = st + (cc - c0) * kAStage;
-                        if (cl == 1)
-                            tc::tma_load_2d(dst, tm, col, row, &c.full[s]);
-                        else if ((uint32_t)(cc % cl) == rank)
-                            tc::tma_load_2d_mc(dst, tm, col, row, &c.full[s], (uint16_t)((1u << cl) - 1));
+                        tc::tma_load_2d(dst, tm, col, row, &c.full[s]);
                     }
                     if (!p.w_res)
                         tc::bulk_g2s(st + G * kAStage, wtile + (size_t)c0 * bchunk, (c1 - c0) * bchunk, &c.full[s]);
@@ -995,10 +984,7 @@ step_ws(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtens
                     const uint32_t st = c.ring0 + s * c.stage;
                     issue_group<NB, G>(d, st, p.w_res ? c.w0 + (c0 - k0) * bchunk : st + G * kAStage, c1 - c0,
                                        c0 == k0);
-                    if (cl > 1)
-                        tc::mma_commit_mc(&c.empty[s], (uint16_t)((1u << cl) - 1));
-                    else
-                        tc::mma_commit(&c.empty[s]);
+                    tc::mma_commit(&c.empty[s]);
                     ++g;
                     c0 = c1;
                 }
@@ -1028,7 +1014,6 @@ step_ws(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtens
         if (p.w_res) tc::mbar_wait(c.wbar, 0, kDrainLimit, nullptr);
     }
     if (warp == E + 1 && lane == 0) tc::mbar_wait(c.done, 0, kDrainLimit, nullptr);
-    if (cl > 1) tc::cluster_sync();  // nobody leaves while a peer may still multicast into it
     tc::tc_fence_before();
     __syncthreads();
     if (warp == E) tc::tmem_dealloc(tmem, 2 * kCols);
@@ -1083,13 +1068,12 @@ uint32_t pad_for_tmem(const void *fn, int threads, uint32_t smem, uint32_t kcols
     return kSmemCap;
 }
 
-// Plans one variant: cluster sizes 8, 4, 2 (only when multicast is wanted) and 1; the
-// weight tile resident or streamed; the deepest ring (up to two tiles of stages) that
-// fits. The grid is sized from the number of co-resident CTAs (clusters) of that
-// footprint. Cost = row-tile rounds per step x per-tile MMA issue time; ties go to the
-// resident weight tile, then the larger cluster, then the deeper ring.
-bool plan_variant(const Variant &v, bool fwd, int KC, int split, int n_rt, int H, int sms, bool want_mc,
-                  uint32_t cap, PersistPlan *pl, double *cost)
+// Plans one variant: the weight tile resident or streamed, a two-stage ring. The grid is
+// sized from the number of co-resident CTAs of that footprint. Cost = row-tile rounds per
+// step x per-tile time (constants fitted to GB300 measurements); ties go to plans within
+// 208 KB of shared memory, then to the resident weight tile.
+bool plan_variant(const Variant &v, bool fwd, int KC, int split, int n_rt, int H, int sms, uint32_t cap,
+                  PersistPlan *pl, double *cost)
 {
     const int NB = fwd ? 4 * v.U : v.U, n_ct = (H + v.U - 1) / v.U;
     const int threads = 32 * (4 * v.EP + 2);
@@ -1097,6 +1081,7 @@ bool plan_variant(const Variant &v, bool fwd, int KC, int split, int n_rt, int H
     const int KCl = (KC + v.KS - 1) / v.KS;  // chunks of one contraction part
     const int groups = (split + v.G - 1) / v.G + (KCl - split + v.G - 1) / v.G;
     const uint32_t fixed = 1024 + kBarBytes;  // alignment pad and barriers (kSmemCap already leaves static room)
+    const int pad = n_ct * v.KS;              // CTAs per row-tile slot
     bool found = false;
     double best = 1e30;
     int best_key = -1;
@@ -1104,97 +1089,67 @@ bool plan_variant(const Variant &v, bool fwd, int KC, int split, int n_rt, int H
         cudaGetLastError();
         return false;
     }
-    for (int cl : {8, 4, 2, 1}) {
-        if (cl > 1 && (!want_mc || cl / 2 >= n_ct || v.KS > 1)) continue;
-        const int pad = (n_ct + cl - 1) / cl * cl * v.KS;  // CTAs per row-tile slot
-        for (int wr : {1, 0}) {
-            const char *fw = getenv(fwd ? "STACKLSTM_FWD_WRES" : "STACKLSTM_BWD_WRES");
-            if (fw && atoi(fw) != wr) continue;
-            const uint32_t wbytes = wr ? (uint32_t)KCl * NB * 128 : 0u;
-            const uint32_t stage = ws_stage_bytes(v.G, NB, wr);
-            const uint32_t stg = ws_stg_bytes(fwd, v.U);
-            if (fixed + wbytes + stg + 2 * stage > cap) continue;
-            // two stages: deeper rings measured slower (their copies compete with the
-            // epilogue's loads and stores); STACKLSTM_*_S asks for more
-            const char *fs = getenv(fwd ? "STACKLSTM_FWD_S" : "STACKLSTM_BWD_S");
-            const int S = std::min({(int)((cap - fixed - wbytes - stg) / stage), kMaxStages, std::max(2, 2 * groups),
-                                    fs ? std::max(2, atoi(fs)) : 2});
-            uint32_t smem = ws_smem_bytes(S, v.G, NB, KCl, wr, stg);
-            smem = pad_for_tmem(v.fn, threads, smem, kcols2);
-            if (!smem) continue;
-            int resident = 0;
-            if (cl == 1) {
-                int r = 0;
-                if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&r, v.fn, threads, smem) != cudaSuccess) {
-                    cudaGetLastError();
-                    continue;
-                }
-                resident = r * sms;
-            } else {
-                cudaLaunchConfig_t cfg = {};
-                cfg.gridDim = dim3(pad);
-                cfg.blockDim = dim3(threads);
-                cfg.dynamicSmemBytes = smem;
-                cudaLaunchAttribute at[1];
-                at[0].id = cudaLaunchAttributeClusterDimension;
-                at[0].val.clusterDim.x = cl;
-                at[0].val.clusterDim.y = 1;
-                at[0].val.clusterDim.z = 1;
-                cfg.attrs = at;
-                cfg.numAttrs = 1;
-                int clusters = 0;
-                if (cudaOccupancyMaxActiveClusters(&clusters, v.fn, &cfg) != cudaSuccess) {
-                    cudaGetLastError();
-                    continue;
-                }
-                resident = clusters * cl;
-            }
-            if (resident < pad) continue;
-            // the fewest slots that give the same number of row-tile rounds per step: every
-            // slot then has (about) the same work, and the SMs left over take other work
-            const int rounds = (n_rt + std::min(n_rt, resident / pad) - 1) / std::min(n_rt, resident / pad);
-            const int sl = (n_rt + rounds - 1) / rounds;
-            // forward, per CTA and step: MMA issue plus the epilogue's ~16 B of stores per
-            // (instance, unit) at about 30 B/cycle
-            double c = rounds * (KC * 4 * mma_cycles(NB) + groups * kWaitCycles + 128.0 * v.U * 16 / 30);
-            if (!fwd) {
-                // backward, per CTA and step: the dG operand (and a streamed weight slice)
-                // at about 70 B/cycle of TMA ingest against the MMA issue time (about 400
-                // cycles per stage wait inside this kernel), then the epilogue's ~48 B per
-                // (instance, unit) at about 30 B/cycle of load/store, plus the partial
-                // exchange of a split contraction (constants fitted to GB300 measurements)
-                const double ingest = (128.0 * KCl * 128 + (wr ? 0.0 : (double)NB * KCl * 128)) / 70;
-                const double mma = KCl * 4 * mma_cycles(NB) + groups * 400.0;
-                const double epi = 128.0 * (v.U / v.KS) * 48 / 30 +
-                                   (v.KS > 1 ? 2.0 * 128 * v.U * 4 / 30 + 3000 : 0.0);
-                // with two or more row tiles a CTA multiplies one while the epilogue
-                // finishes the other (their chains are independent)
-                const double mm = std::max(ingest, mma);
-                c = rounds > 1 ? rounds * std::max(mm, epi) + std::min(mm, epi) : mm + epi;
-            }
-            // ties: a plan within 208 KB of shared memory first (beyond it L1 is too small
-            // for the epilogue's traffic: the stress forward ran 5% slower with its weight
-            // tile resident at 230 KB than streamed at 165 KB), then the resident weight
-            // tile, the larger cluster, the deeper ring
-            const int key = (smem <= 208u * 1024) * 10000 + wr * 1000 + cl * 20 + S;
-            if (c < best * 0.999 || (c <= best * 1.001 && key > best_key)) {
-                best = c;
-                best_key = key;
-                pl->on = 1;
-                pl->U = v.U;
-                pl->EP = v.EP;
-                pl->G = v.G;
-                pl->S = S;
-                pl->slot = sl;
-                pl->w_res = wr;
-                pl->cl = cl;
-                pl->KS = v.KS;
-                pl->n_ct = pad / v.KS;
-                pl->smem = smem;
-                pl->threads = threads;
-                pl->per_sm = resident / sms;
-                found = true;
-            }
+    for (int wr : {1, 0}) {
+        const uint32_t wbytes = wr ? (uint32_t)KCl * NB * 128 : 0u;
+        const uint32_t stage = ws_stage_bytes(v.G, NB, wr);
+        const uint32_t stg = ws_stg_bytes(fwd, v.U);
+        if (fixed + wbytes + stg + 2 * stage > cap) continue;
+        // two stages: deeper rings measured slower (their copies compete with the
+        // epilogue's loads and stores)
+        const int S = 2;
+        uint32_t smem = ws_smem_bytes(S, v.G, NB, KCl, wr, stg);
+        smem = pad_for_tmem(v.fn, threads, smem, kcols2);
+        if (!smem) continue;
+        int r = 0;
+        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&r, v.fn, threads, smem) != cudaSuccess) {
+            cudaGetLastError();
+            continue;
+        }
+        const int resident = r * sms;
+        if (resident < pad) continue;
+        // the fewest slots that give the same number of row-tile rounds per step: every
+        // slot then has (about) the same work, and the SMs left over take other work
+        const int rounds = (n_rt + std::min(n_rt, resident / pad) - 1) / std::min(n_rt, resident / pad);
+        const int sl = (n_rt + rounds - 1) / rounds;
+        // forward, per CTA and step: MMA issue plus the epilogue's ~16 B of stores per
+        // (instance, unit) at about 30 B/cycle
+        double c = rounds * (KC * 4 * mma_cycles(NB) + groups * kWaitCycles + 128.0 * v.U * 16 / 30);
+        if (!fwd) {
+            // backward, per CTA and step: the dG operand (and a streamed weight slice)
+            // at about 70 B/cycle of TMA ingest against the MMA issue time (about 400
+            // cycles per stage wait inside this kernel), then the epilogue's ~48 B per
+            // (instance, unit) at about 30 B/cycle of load/store, plus the partial
+            // exchange of a split contraction
+            const double ingest = (128.0 * KCl * 128 + (wr ? 0.0 : (double)NB * KCl * 128)) / 70;
+            const double mma = KCl * 4 * mma_cycles(NB) + groups * 400.0;
+            const double epi = 128.0 * (v.U / v.KS) * 48 / 30 +
+                               (v.KS > 1 ? 2.0 * 128 * v.U * 4 / 30 + 3000 : 0.0);
+            // with two or more row tiles a CTA multiplies one while the epilogue
+            // finishes the other (their chains are independent)
+            const double mm = std::max(ingest, mma);
+            c = rounds > 1 ? rounds * std::max(mm, epi) + std::min(mm, epi) : mm + epi;
+        }
+        // ties: a plan within 208 KB of shared memory first (beyond it L1 is too small
+        // for the epilogue's traffic: the stress forward ran 5% slower with its weight
+        // tile resident at 230 KB than streamed at 165 KB), then the resident weight tile
+        const int key = (smem <= 208u * 1024) * 10000 + wr * 1000;
+        if (c < best * 0.999 || (c <= best * 1.001 && key > best_key)) {
+            best = c;
+            best_key = key;
+            pl->on = 1;
+            pl->U = v.U;
+            pl->EP = v.EP;
+            pl->G = v.G;
+            pl->S = S;
+            pl->slot = sl;
+            pl->w_res = wr;
+            pl->cl = 1;
+            pl->KS = v.KS;
+            pl->n_ct = n_ct;
+            pl->smem = smem;
+            pl->threads = threads;
+            pl->per_sm = r;
+            found = true;
         }
     }
     *cost = best;
@@ -1216,34 +1171,23 @@ bool plan(stacklstm *s, bool fwd, PersistPlan *pl)
     const Variant *vs = fwd ? fwd_variants(&n) : bwd_variants(&n);
     const int n_rt = (int)ceil_div(s->B, kRows);
     const int KC = fwd ? s->kcf : s->kcb, split = fwd ? s->kcx : 0;
-    const char *mc = getenv("STACKLSTM_MULTICAST");
-    const bool mc_on = mc && atoi(mc) != 0;
-    const char *force = getenv(fwd ? "STACKLSTM_FWD_UNITS" : "STACKLSTM_BWD_UNITS");
-    const int force_u = force ? atoi(force) : 0;
-    // epilogue warp groups: forward, one for 16-unit tiles (a thread then holds 16 units,
-    // whole 32-byte sectors), two for 32-unit tiles; backward, one up to 32 units (its
-    // threads then have the registers to hold their gradient-history updates until after
-    // the step's release), two for 64 (all measured best); STACKLSTM_*_EP overrides
-    const char *force_ep = getenv(fwd ? "STACKLSTM_FWD_EP" : "STACKLSTM_BWD_EP");
+    // test hook (include/stacklstm.h): STACKLSTM_BWD_SPLIT = k asks for the backward whose
+    // 4H contraction is split over k CTAs per 64-unit column tile
+    const char *force_split = fwd ? nullptr : getenv("STACKLSTM_BWD_SPLIT");
+    const int want_ks = force_split ? atoi(force_split) : 0;
     double best = 1e30;
     bool found = false;
     for (int i = 0; i < n; ++i) {
-        if (force_u && vs[i].U != force_u) continue;
-        const int want_ep = force_ep               ? atoi(force_ep)
-                            : vs[i].U == 16 || vs[i].KS > 1 || (!fwd && vs[i].U <= 32) ? 1
-                                                                                          : 2;
+        // epilogue warp groups: forward, one for 16-unit tiles (a thread then holds 16
+        // units, whole 32-byte sectors), two for 32-unit tiles; backward, one up to 32
+        // units (its threads then have the registers to hold their gradient-history
+        // updates until after the step's release), two for 64 (all measured best)
+        const int want_ep = vs[i].U == 16 || vs[i].KS > 1 || (!fwd && vs[i].U <= 32) ? 1 : 2;
         if (vs[i].U >= 16 && vs[i].EP != want_ep) continue;
-        const char *force_ks = fwd ? nullptr : getenv("STACKLSTM_BWD_KS");
-        if (force_ks && vs[i].KS != atoi(force_ks)) continue;
-        const char *force_g = getenv(fwd ? "STACKLSTM_FWD_G" : "STACKLSTM_BWD_G");
-        if (force_g && vs[i].G != atoi(force_g)) continue;
+        if (want_ks > 0 && (vs[i].KS != want_ks || vs[i].U != 64)) continue;
         PersistPlan cand;
         double cost;
-        const int n_ct = (s->H + vs[i].U - 1) / vs[i].U;
-        // multicast pays only when the column tiles' re-reads of A are a large L2 stream
-        const bool want_mc = mc_on && (double)n_rt * kAStage * KC * n_ct >= 8e6;
-        if (plan_variant(vs[i], fwd, KC, split, n_rt, s->H, s->num_sms, want_mc, kSmemCap, &cand, &cost) &&
-            cost < best) {
+        if (plan_variant(vs[i], fwd, KC, split, n_rt, s->H, s->num_sms, kSmemCap, &cand, &cost) && cost < best) {
             best = cost;
             *pl = cand;
             found = true;
@@ -1257,13 +1201,15 @@ bool plan(stacklstm *s, bool fwd, PersistPlan *pl)
     pl->dx_S = 0;
     if (!fwd) {
         // the input gradient on the SMs the chain leaves idle: one CTA per SM (the role
-        // takes all 512 tensor-memory columns), 256-column dx tiles, full 128-row A boxes
+        // takes all 512 tensor-memory columns), 256-column dx tiles, full 128-row A boxes.
+        // Test hook (include/stacklstm.h): STACKLSTM_DX_SPARE = 0 keeps dx out of the
+        // launch, = k > 0 gives it at most k CTAs
         const char *fx = getenv("STACKLSTM_DX_SPARE");
         int r = 0;
         const int n_chain = pl->n_ct * pl->KS * pl->slot;
         const int spare = s->num_sms - n_chain;
         const int S = (int)std::min<uint32_t>(kMaxStages, (pl->smem - 1024 - kBarBytes) / (kAStage + 256u * 128));
-        if ((!fx || atoi(fx) != 0) && s->nx == 256 && s->B >= kRows && pl->cl == 1 && spare >= 4 && S >= 2 &&
+        if ((!fx || atoi(fx) != 0) && s->nx == 256 && s->B >= kRows && spare >= 4 && S >= 2 &&
             cudaOccupancyMaxActiveBlocksPerMultiprocessor(&r, find_fn(false, *pl), pl->threads, pl->smem) ==
                 cudaSuccess &&
             r == 1) {
@@ -1313,7 +1259,6 @@ cudaError_t bf16_launch_fwd_persist(stacklstm *s, const StepArgs &a, const CUten
     p.n_rt = (int)ceil_div(s->B, kRows);
     p.n_slot = pl.slot;
     p.w_res = pl.w_res;
-    p.cl = pl.cl;
     p.cnt = s->rowcnt;
     p.cs = s->cnt_stride;
     p.vec32 = s->H % 16 == 0;
@@ -1342,7 +1287,6 @@ cudaError_t bf16_launch_bwd_persist(stacklstm *s, const StepArgs &a, const CUten
     p.n_rt = (int)ceil_div(s->B, kRows);
     p.n_slot = pl.slot;
     p.w_res = pl.w_res;
-    p.cl = pl.cl;
     p.cs = s->cnt_stride;
     p.cnt = s->rowcnt + p.n_rt * p.cs;
     p.vec32 = s->H % 16 == 0;

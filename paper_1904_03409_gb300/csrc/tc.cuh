@@ -181,17 +181,6 @@ __device__ __forceinline__ void cluster_sync()
 {
     asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
-// TMA tile load delivered to the same shared-memory offset of every CTA in cta_mask; each
-// destination CTA's mbarrier at the same offset receives the box's bytes.
-__device__ __forceinline__ void tma_load_2d_mc(uint32_t dst, const void *tmap, int c0, int c1, uint64_t *bar,
-                                               uint16_t cta_mask)
-{
-    asm volatile(
-        "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.multicast::cluster"
-        " [%0], [%1, {%2, %3}], [%4], %5;" ::"r"(dst),
-        "l"((uint64_t)tmap), "r"(c0), "r"(c1), "r"(smem_u32(bar)), "h"(cta_mask)
-        : "memory");
-}
 
 // ------------------------------------------------------------------ inter-CTA counters
 __device__ __forceinline__ int ld_acquire_gpu(const int *p)

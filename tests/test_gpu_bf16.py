@@ -156,8 +156,7 @@ def test_split_contraction_backward_matches_oracle(T, B, I, H, seed):
     sums exchanged through L2, summed in part order) stays parity-green, including parts
     of unequal length (H = 200: 13 chunks over 4 parts)."""
     w = case(T, B, I, H, seed, bias_scale=0.3, h0_scale=0.5, c0_scale=0.5, dy_scale=0.5)
-    os.environ["STACKLSTM_BWD_UNITS"] = "64"
-    os.environ["STACKLSTM_BWD_KS"] = "4"
+    os.environ["STACKLSTM_BWD_SPLIT"] = "4"
     try:
         hd = bd.stacklstm_create(w.T, w.B, w.I, w.H, bd.SL_BF16, 0)
         plan = bd.stacklstm_plan(hd)
@@ -165,8 +164,7 @@ def test_split_contraction_backward_matches_oracle(T, B, I, H, seed):
         got = runner.run(w)
         again = runner.run(w)
     finally:
-        del os.environ["STACKLSTM_BWD_UNITS"]
-        del os.environ["STACKLSTM_BWD_KS"]
+        del os.environ["STACKLSTM_BWD_SPLIT"]
     assert "backward persistent U=64" in plan and "contraction parts 4" in plan, plan
     compare(got, oracle_all(w), "bf16")
     for k in ("dx", "dW", "dbias", "dh0", "dc0"):

@@ -1,12 +1,14 @@
 """The allocation-free index prepass (stacklstm_pointers_noalloc).
 
 Some callers of this library cannot allocate device memory at the moment they need the
-pointer bookkeeping: code inside CUDA-graph stream capture, and services whose memory is
-reserved up front by a pooling allocator. For them the prepass runs on a fixed scratch
-array built into the library. These tests check, through the C ABI on cuda:0, that its
-pointer trajectories and read provenance equal those of stacklstm_forward bit for bit on
-two calls in a row (the second call runs on the scratch the first one left behind), and
-that sizes beyond its limit are refused. The file is named to be collected last.
+pointer bookkeeping: services whose device memory is all reserved up front by a pooling
+allocator, and callers that must not let a cudaMalloc or cudaFree synchronize the device
+while other streams run. For them the prepass runs on a fixed scratch array built into
+the library. These tests check, through the C ABI on cuda:0, that its pointer
+trajectories and read provenance equal those of stacklstm_forward bit for bit on two
+calls in a row (the second call runs on the scratch the first one left behind), that a
+call changes neither torch's allocated memory nor the device's free memory, and that
+sizes beyond its limit are refused. The file is named to be collected last.
 """
 import numpy as np
 import pytest
@@ -43,6 +45,22 @@ def test_matches_forward_on_two_calls_in_a_row():
             p, s = via_noalloc(w)
             assert np.array_equal(p, ref_p)
             assert np.array_equal(s, ref_s)
+
+
+def test_a_call_allocates_no_device_memory():
+    w = wl.config_workload("parser64")
+    dev = torch.device("cuda", 0)
+    ops = torch.from_numpy(np.ascontiguousarray(w.ops, np.int8)).to(dev)
+    p = torch.empty(w.T + 1, w.B, dtype=torch.int32, device=dev)
+    s = torch.empty(w.T + 1, w.B, dtype=torch.int32, device=dev)
+    bd.stacklstm_pointers_noalloc(ops, p, s)  # the device's one-time set-up happens here
+    torch.cuda.synchronize(dev)
+    for _ in range(2):
+        alloc0, free0 = torch.cuda.memory_allocated(dev), torch.cuda.mem_get_info(dev)[0]
+        bd.stacklstm_pointers_noalloc(ops, p, s)
+        torch.cuda.synchronize(dev)
+        assert torch.cuda.memory_allocated(dev) == alloc0
+        assert torch.cuda.mem_get_info(dev)[0] == free0
 
 
 def test_refuses_sizes_beyond_its_scratch():
