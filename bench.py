@@ -263,6 +263,11 @@ def measure_record(w, steps, warmup, cpu_seconds, with_cpu, min_seconds):
     end-to-end rate through host buffers, per-step latency, and the oracle on the host
     cores as a baseline."""
     res = measure_workload(w, steps, warmup, min_seconds)
+    if w.dtype == "bf16":
+        # the push-only mode (dead writes skipped, Observation 2 of Sec. 3) on the same
+        # workload: same metric (real B * T instance-steps per second), its own roofline
+        # over the B * steps_run virtual steps it computes
+        res["push_only"] = measure_workload(w, steps, warmup, min_seconds, push_only=True, with_e2e=False)
     res["config"] = {"workload": describe(w), "B": w.B, "T": w.T, "I": w.I, "H": w.H,
                      "real_step_share": round(w.real_step_share, 4),
                      "l2": "flushed between timed steps (256 MiB write outside the timed events)",
@@ -272,7 +277,7 @@ def measure_record(w, steps, warmup, cpu_seconds, with_cpu, min_seconds):
     return res
 
 
-def measure_workload(w, steps, warmup, min_seconds=0.0):
+def measure_workload(w, steps, warmup, min_seconds=0.0, push_only=False, with_e2e=True):
     import torch
     from paper_1904_03409_gb300 import binding as bd
     from paper_1904_03409_gb300 import runner
@@ -280,6 +285,8 @@ def measure_workload(w, steps, warmup, min_seconds=0.0):
     dev = torch.device("cuda", 0)
     stream = torch.cuda.current_stream(dev)
     hd = bd.stacklstm_create(w.T, w.B, w.I, w.H, bd.SL_BF16 if w.dtype == "bf16" else bd.SL_FP32, 0, stream)
+    if push_only:
+        bd.stacklstm_set_mode(hd, bd.SL_MODE_PUSH_ONLY)
     plan = bd.stacklstm_plan(hd)
     bd.stacklstm_set_async(hd, True)
     ins = runner.upload(w, 0)
@@ -319,6 +326,7 @@ def measure_workload(w, steps, warmup, min_seconds=0.0):
     timing = bd.stacklstm_get_timing(hd)
     n_launch = hd_launches(hd) - launches0
     bd.stacklstm_set_timing(hd, False)
+    Tr = bd.stacklstm_steps_run(hd)  # T, or the virtual steps of the push-only mode
 
     peaks, src = load_peaks()
     sms = torch.cuda.get_device_properties(dev).multi_processor_count
@@ -329,8 +337,8 @@ def measure_workload(w, steps, warmup, min_seconds=0.0):
     # a persistent or cluster step kernel is one launch over all T steps; the per-step
     # kernels are T (or 2T) launches of B instance-steps each; dx and dW are one
     # contraction over all T * B rows (dW: plus its fixed-order reduction of the partials)
-    launches_per_pass = {"T": w.T, "2T": 2 * w.T}.get(lpp, lpp)
-    per_launch_units = w.B * w.T / launches_per_pass
+    launches_per_pass = {"T": Tr, "2T": 2 * Tr}.get(lpp, lpp)
+    per_launch_units = w.B * Tr / launches_per_pass
     launch_s = phase_ms[dom] / 1e3 / launches_per_pass
     fl, by = wk[dom]["flops"], wk[dom]["bytes"]
     m = re.search(r"dx CTAs (\d+)", plan)
@@ -344,13 +352,14 @@ def measure_workload(w, steps, warmup, min_seconds=0.0):
                "unit_of_work": "instance-step", "algorithmic_flops_per_unit": fl,
                "algorithmic_bytes_per_unit": by, "traffic": kernel_traffic(kname, kfile, wkey(w))})
     sec = total_ms / 1e3 / steps
-    srf = roofline_of(wk["step"]["flops"] * w.B * w.T, wk["step"]["bytes"] * w.B * w.T, sec, peaks, src, w.dtype, sms)
+    srf = roofline_of(wk["step"]["flops"] * w.B * Tr, wk["step"]["bytes"] * w.B * Tr, sec, peaks, src, w.dtype, sms)
     res = {"value": w.B * w.T * steps / (total_ms / 1e3), "ms_per_step": total_ms / steps, "steps": steps,
            "roofline": rf, "step_roofline": srf, "phases_ms_per_step": {p: round(v, 4) for p, v in phase_ms.items()},
-           "step_latency_us": {"forward": 1e3 * phase_ms["forward"] / w.T,
-                               "backward": 1e3 * (phase_ms["backward"] + phase_ms["dx"]) / w.T},
-           "plan": plan, "gpu_launches": int(n_launch), "clocks": clocks.summary()}
-    res["e2e"] = measure_e2e(w, hd, ins, out, steps, flush)
+           "step_latency_us": {"forward": 1e3 * phase_ms["forward"] / Tr,
+                               "backward": 1e3 * (phase_ms["backward"] + phase_ms["dx"]) / Tr},
+           "steps_run": Tr, "plan": plan, "gpu_launches": int(n_launch), "clocks": clocks.summary()}
+    if with_e2e:
+        res["e2e"] = measure_e2e(w, hd, ins, out, steps, flush)
     hd.destroy()
     del ins, out, flush
     torch.cuda.empty_cache()

@@ -141,6 +141,39 @@ sl_status stacklstm_backward(stacklstm_t s, const float *d_top_h, const float *d
                              float *dh0, float *dc0, float *dW, float *dbias);
 
 /*
+ * Modes of the step computation.
+ *   SL_MODE_HOMOGENIZED (default): Algorithm 1 as written. Every instance runs the LSTM
+ *     cell at every step, whatever its op, and writes slot p + 1.
+ *   SL_MODE_PUSH_ONLY: dead writes skipped. By Observation 2 of Sec. 3 a pop or hold step
+ *     writes slot p + 1 above the new top, and the next push overwrites that slot before
+ *     the pointer reaches it, so only push steps' writes are ever read. This mode runs
+ *     the cell for push steps only: virtual step k of instance b is its k-th push, and
+ *     the step kernels run max_b(pushes of b) steps instead of T. p_final, p_traj, src,
+ *     y and every gradient are those of the homogenized mode (y and dx bit for bit; dW
+ *     and dbias are sums in another order). h_stack / c_stack hold the stack of the
+ *     push/pop definition of Sec. 2: each slot the state last pushed into it (0 if
+ *     none). They equal the homogenized mode's on the live part (slots 0 .. p_final);
+ *     above the top, Algorithm 1 leaves what a pop or hold step wrote last, states
+ *     nothing reads. bf16 path only.
+ *     Its forward synchronizes the handle's stream once, after the index prepass, to
+ *     learn the number of virtual steps (also in async mode).
+ */
+typedef enum { SL_MODE_HOMOGENIZED = 0, SL_MODE_PUSH_ONLY = 1 } sl_mode;
+
+/*
+ * stacklstm_set_mode -- choose the mode of later forward calls. Switching modes needs a
+ * new forward before backward (SL_ERR_STATE otherwise). The first switch to
+ * SL_MODE_PUSH_ONLY allocates its workspace (about (T + 1) B 24 + T B 2 I bytes):
+ * SL_ERR_OOM if that fails; SL_ERR_UNSUPPORTED on the fp32 path. Synchronizes the
+ * handle's stream.
+ */
+sl_status stacklstm_set_mode(stacklstm_t s, sl_mode mode);
+
+/* Number of steps the step kernels ran in the last forward: T in the homogenized mode,
+ * the most pushes of any instance (at least 1) in the push-only mode. */
+sl_status stacklstm_steps_run(stacklstm_t s, int *steps);
+
+/*
  * Phases of a forward + backward, as stacklstm_get_timing reports them. Each phase is a
  * contiguous run of kernel launches on the handle's stream.
  */

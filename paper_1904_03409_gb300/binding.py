@@ -16,6 +16,7 @@ from typing import Optional
 from . import build as _build
 
 SL_FP32, SL_BF16 = 0, 1
+SL_MODE_HOMOGENIZED, SL_MODE_PUSH_ONLY = 0, 1
 STATUS = {0: "SL_OK", 1: "SL_ERR_ARG", 2: "SL_ERR_OP", 3: "SL_ERR_UNDERFLOW", 4: "SL_ERR_STATE",
           5: "SL_ERR_CUDA", 6: "SL_ERR_TIMEOUT", 7: "SL_ERR_UNSUPPORTED", 8: "SL_ERR_OOM"}
 HEADER = os.path.join(_build.ROOT, "include", "stacklstm.h")
@@ -59,6 +60,8 @@ def load(path: Optional[str] = None):
     lib.stacklstm_get_timing.argtypes = [vp, vp, vp, i]
     lib.stacklstm_pointers_noalloc.argtypes = [i, i, vp, vp, vp, vp]
     lib.stacklstm_pointers_noalloc.restype = ctypes.c_int
+    lib.stacklstm_set_mode.argtypes = [vp, i]
+    lib.stacklstm_steps_run.argtypes = [vp, vp]
     lib.stacklstm_plan.argtypes = [vp]
     lib.stacklstm_plan.restype = ctypes.c_char_p
     lib.stacklstm_last_error.argtypes = [vp]
@@ -72,7 +75,7 @@ def load(path: Optional[str] = None):
     lib.stacklstm_head_last_error.restype = ctypes.c_char_p
     for fn in ("stacklstm_create", "stacklstm_forward", "stacklstm_backward", "stacklstm_set_stream",
                "stacklstm_set_async", "stacklstm_status", "stacklstm_destroy", "stacklstm_set_timing",
-               "stacklstm_get_timing", "stacklstm_head_create", "stacklstm_head_run", "stacklstm_head_add_h0_grads",
+               "stacklstm_get_timing", "stacklstm_set_mode", "stacklstm_steps_run", "stacklstm_head_create", "stacklstm_head_run", "stacklstm_head_add_h0_grads",
                "stacklstm_head_status", "stacklstm_head_destroy"):
         getattr(lib, fn).restype = ctypes.c_int
     _lib = lib
@@ -149,6 +152,19 @@ def stacklstm_set_stream(hd: StackLSTMHandle, stream):
 
 def stacklstm_set_async(hd: StackLSTMHandle, on: bool):
     _check(hd.h, load().stacklstm_set_async(hd.h, int(bool(on))), "stacklstm_set_async")
+
+
+def stacklstm_set_mode(hd: StackLSTMHandle, mode: int):
+    """SL_MODE_HOMOGENIZED (Algorithm 1) or SL_MODE_PUSH_ONLY (dead writes skipped)."""
+    _check(hd.h, load().stacklstm_set_mode(hd.h, int(mode)), "stacklstm_set_mode")
+
+
+def stacklstm_steps_run(hd: StackLSTMHandle) -> int:
+    """Steps the step kernels ran in the last forward (T, or the most pushes of any
+    instance in push-only mode)."""
+    n = ctypes.c_int(0)
+    _check(hd.h, load().stacklstm_steps_run(hd.h, ctypes.byref(n)), "stacklstm_steps_run")
+    return n.value
 
 
 def stacklstm_status(hd: StackLSTMHandle):

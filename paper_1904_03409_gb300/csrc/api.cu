@@ -187,6 +187,7 @@ sl_status stacklstm_create(stacklstm_t *out, int T, int B, int I, int H, sl_dtyp
     stacklstm *s = new (std::nothrow) stacklstm;
     if (!s) return SL_ERR_OOM;
     s->T = T; s->B = B; s->I = I; s->H = H; s->dt = dtype; s->device = device;
+    s->Tr = T;
     s->stream = (cudaStream_t)stream;
     if (cudaDeviceGetAttribute(&s->num_sms, cudaDevAttrMultiProcessorCount, device) != cudaSuccess) {
         delete s;
@@ -254,6 +255,11 @@ sl_status stacklstm_forward(stacklstm_t s, const void *x, const int8_t *ops, con
     {
         Phase ph(s, SL_PHASE_PREPASS);
         if ((e = sl::launch_prepass(s, ops))) return cuda_fail(s, e, "prepass");
+        s->Tr = T;
+        // push-only mode: each instance's pushes as a virtual timeline; the step count the
+        // kernels run is read back here (the one synchronization of this mode's forward)
+        if (s->push_only && ((e = sl::launch_compact(s)) || (e = sl::read_virtual_steps(s))))
+            return cuda_fail(s, e, "push-only indices");
     }
     {
         Phase ph(s, SL_PHASE_FWD_SETUP);
@@ -293,11 +299,14 @@ sl_status stacklstm_forward(stacklstm_t s, const void *x, const int8_t *ops, con
         if (src && (e = cudaMemcpyAsync(src, s->top, sizeof(int32_t) * (T + 1) * B, cudaMemcpyDeviceToDevice,
                                         s->stream)))
             return cuda_fail(s, e, "src");
-        if (y && (e = sl::launch_gather_rows(s, s->top + B, T * B, es, s->hist_h, y, H)))
+        // history index of the top after each step and of each slot's last write (in
+        // push-only mode: virtual indices, and each slot's last push, as in Sec. 2)
+        const int32_t *ytop = s->push_only ? s->vy : s->top, *slots = s->push_only ? s->vslot : s->slot_last;
+        if (y && (e = sl::launch_gather_rows(s, ytop + B, T * B, es, s->hist_h, y, H)))
             return cuda_fail(s, e, "y");
-        if (h_stack && (e = sl::launch_gather_rows(s, s->slot_last, (T + 1) * B, es, s->hist_h, h_stack, H)))
+        if (h_stack && (e = sl::launch_gather_rows(s, slots, (T + 1) * B, es, s->hist_h, h_stack, H)))
             return cuda_fail(s, e, "h_stack");
-        if (c_stack && (e = sl::launch_gather_rows(s, s->slot_last, (T + 1) * B, 4, s->hist_c, c_stack, H)))
+        if (c_stack && (e = sl::launch_gather_rows(s, slots, (T + 1) * B, 4, s->hist_c, c_stack, H)))
             return cuda_fail(s, e, "c_stack");
     }
     s->fwd_done = 1;
@@ -331,6 +340,11 @@ sl_status stacklstm_backward(stacklstm_t s, const float *d_top_h, const float *d
         if (s->dt == SL_BF16 && (e = sl::bf16_backward_setup(s))) return cuda_fail(s, e, "backward setup");
     }
     bool dx_done = false;  // computed by the step launch on otherwise idle SMs
+    if (s->push_only) {
+        // the dx rows of steps that do not push are zero; the contraction writes the others
+        Phase ph(s, SL_PHASE_BWD_SETUP);
+        if ((e = sl::launch_zero_nonpush_rows(s, dx))) return cuda_fail(s, e, "dx rows");
+    }
     {
         Phase ph(s, SL_PHASE_BACKWARD);
         e = s->dt == SL_FP32 ? sl::fp32_backward_steps(s) : sl::bf16_backward_steps(s, dx, &dx_done);
@@ -352,6 +366,43 @@ sl_status stacklstm_backward(stacklstm_t s, const float *d_top_h, const float *d
     if (dc0 && (e = cudaMemcpyAsync(dc0, s->dhist_c, sizeof(float) * B * H, cudaMemcpyDeviceToDevice, s->stream)))
         return cuda_fail(s, e, "dc0");
     return s->async ? SL_OK : read_status(s);
+}
+
+sl_status stacklstm_set_mode(stacklstm_t s, sl_mode mode)
+{
+    if (!s || (mode != SL_MODE_HOMOGENIZED && mode != SL_MODE_PUSH_ONLY)) return SL_ERR_ARG;
+    s->last_error.clear();
+    if (mode == SL_MODE_PUSH_ONLY && s->dt != SL_BF16)
+        return fail(s, SL_ERR_UNSUPPORTED, "push-only mode runs on the bf16 path");
+    DeviceGuard g(s->device);
+    cudaError_t e = cudaStreamSynchronize(s->stream);
+    if (e != cudaSuccess) return cuda_fail(s, e, "synchronize");
+    if (mode == SL_MODE_PUSH_ONLY && !s->vtop) {
+        const size_t T1B = (size_t)(s->T + 1) * s->B, TB = (size_t)s->T * s->B;
+        bool ok = alloc(s, &s->vtop, T1B * 4) && alloc(s, &s->vmap, T1B * 4) && alloc(s, &s->vy, T1B * 4) &&
+                  alloc(s, &s->vslot, T1B * 4) && alloc(s, &s->xidx, TB * 4) && alloc(s, &s->vstep, TB * 4) &&
+                  alloc(s, &s->x_push, TB * s->I * 2) && alloc(s, &s->kmax, 16);
+        if (ok && cudaMallocHost(&s->kmax_host, sizeof(int32_t)) != cudaSuccess) {
+            cudaGetLastError();
+            s->kmax_host = nullptr;
+            ok = false;
+        }
+        if (!ok) return fail(s, SL_ERR_OOM, "push-only workspace");
+    }
+    if (mode != (s->push_only ? SL_MODE_PUSH_ONLY : SL_MODE_HOMOGENIZED)) s->fwd_done = 0;
+    s->push_only = mode == SL_MODE_PUSH_ONLY;
+    const std::string tag = "; push-only steps (dead writes skipped)";
+    const size_t at = s->plan.find(tag);
+    if (s->push_only && at == std::string::npos) s->plan += tag;
+    if (!s->push_only && at != std::string::npos) s->plan.erase(at);
+    return SL_OK;
+}
+
+sl_status stacklstm_steps_run(stacklstm_t s, int *steps)
+{
+    if (!s || !steps) return SL_ERR_ARG;
+    *steps = s->Tr;
+    return SL_OK;
 }
 
 sl_status stacklstm_set_timing(stacklstm_t s, int on)
@@ -405,6 +456,7 @@ sl_status stacklstm_destroy(stacklstm_t s)
         collect_timing(s);
         for (cudaEvent_t ev : s->event_pool) cudaEventDestroy(ev);
         s->event_pool.clear();
+        if (s->kmax_host) cudaFreeHost(s->kmax_host);
         free_all(s);
         cudaGetLastError();
     }

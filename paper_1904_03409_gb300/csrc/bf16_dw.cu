@@ -291,20 +291,21 @@ cudaError_t bf16_launch_dw(stacklstm *s, const CUtensorMap &tm_x, const CUtensor
                            float *dW, float *dbias)
 {
     DwWsArgs w;
-    w.R = s->T * s->B;
+    w.R = s->Tr * s->B;
     w.I = s->I;
     w.H = s->H;
     w.kbx = (int)ceil_div(s->I, 64);
     w.kbh = (int)ceil_div(s->H, 64);
     w.n_nt = s->dw_nt;
-    w.split = s->dw_split;
+    // every split keeps at least 16 chunks of 64 rows (fewer rows than planned: push-only mode)
+    w.split = (int)std::min<size_t>(s->dw_split, std::max<size_t>(1, ceil_div((size_t)w.R, 64) / 16));
     w.S = s->sw;
     w.part = s->dw_part;
     w.ld_part = (size_t)s->dw_nt * s->dw_ntile;
     w.rows_part = (size_t)s->dw_mt * 128 + 1;
     w.limit = s->wait_limit;
     w.err = s->err;
-    const dim3 grid(s->dw_mt * s->dw_nt, s->dw_split);
+    const dim3 grid(s->dw_mt * s->dw_nt, w.split);
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = grid;
     cfg.blockDim = dim3(kDwThreads);

@@ -346,6 +346,8 @@ struct DxArgs {
     int I, KC, S;
     const uint8_t *wpack;
     float *dx;  // [R][I]
+    const int32_t *xidx;  // push-only mode: real step of each virtual row's step (-1: none), else null
+    int B;
     long long limit;
     int32_t *err;
 };
@@ -371,13 +373,22 @@ __global__ void __launch_bounds__(kThreads, 1) dx_tc(const __grid_constant__ CUt
     mainloop<false>(c, a.S, a.KC, -1, a.limit, a.err, tma, no_gather, issue);
     if (!*c.abort) {
         const size_t row = row0 + tid;
+        // the dx row this accumulator row belongs to: the same row, or (push-only mode)
+        // the real step of this virtual row's push; rows past an instance's pushes have none
+        bool out = row < a.R;
+        size_t orow = row;
+        if (out && a.xidx) {
+            const int t = a.xidx[row];
+            out = t >= 0;
+            orow = (size_t)t * a.B + row % a.B;
+        }
         const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
 #pragma unroll 1
         for (int cu = 0; cu < N / 8; ++cu) {
             float v[8];
             tc::tmem_ld8(trow + cu * 8, v);
             const int col = ct * N + cu * 8;
-            if (row < a.R && col < a.I) st8f(a.dx + row * a.I + col, v);
+            if (out && col < a.I) st8f(a.dx + orow * a.I + col, v);
         }
     }
     finish(c, tmem, kCols);
@@ -432,6 +443,19 @@ __global__ void pack_rows(const __nv_bfloat16 *__restrict__ W, int H, int row0, 
         const __nv_bfloat16 v = (m < nrows && k < G) ? W[(size_t)(row0 + m) * G + k] : __float2bfloat16(0.0f);
         const size_t byte = tile * NB * 128 + sw128(row, col >> 3) + (col & 7) * 2;
         out[byte / 2] = v;
+    }
+}
+
+// Push-only mode: the input of each virtual step, x_push[k][b] = x[xidx[k][b]][b] (zero
+// rows past the instance's pushes), 16-byte pieces (I % 8 == 0).
+__global__ void gather_push_x(size_t rows, int B, int I8, const int32_t *__restrict__ xidx, const uint4 *__restrict__ x,
+                              uint4 *__restrict__ out)
+{
+    const size_t n = rows * I8;
+    for (size_t e = blockIdx.x * (size_t)blockDim.x + threadIdx.x; e < n; e += (size_t)gridDim.x * blockDim.x) {
+        const size_t r = e / I8;
+        const int t = xidx[r];
+        out[e] = t >= 0 ? x[((size_t)t * B + r % B) * I8 + e % I8] : make_uint4(0u, 0u, 0u, 0u);
     }
 }
 
@@ -528,9 +552,11 @@ unsigned grid_for(const stacklstm *s, size_t n)
 StepArgs step_args(stacklstm *s, const float *bias, const void *wpack, int kcx, int KC, int S)
 {
     StepArgs a;
-    a.T = s->T; a.B = s->B; a.I = s->I; a.H = s->H;
+    // the step kernels run over s->Tr steps: the real ones, or (push-only mode) the
+    // virtual timeline of each instance's pushes with its own read indices
+    a.T = s->Tr; a.B = s->B; a.I = s->I; a.H = s->H;
     a.kcx = kcx; a.KC = KC; a.S = S;
-    a.top = s->top;
+    a.top = s->push_only ? s->vtop : s->top;
     a.hist_h = (__nv_bfloat16 *)s->hist_h; a.hr = (__nv_bfloat16 *)s->hr;
     a.hist_c = s->hist_c; a.gates = (__half *)s->gates; a.gates_blk = 0;
     a.bias = bias; a.wpack = (const uint8_t *)wpack;
@@ -663,6 +689,11 @@ cudaError_t bf16_forward_setup(stacklstm *s, const __nv_bfloat16 *x, const __nv_
 {
     const int T = s->T, B = s->B, I = s->I, H = s->H;
     cudaError_t e;
+    if (s->push_only) {
+        // the forward and the weight gradient read the inputs of the virtual steps
+        if ((e = bf16_gather_push_x(s, x))) return e;
+        x = (const __nv_bfloat16 *)s->x_push;
+    }
     s->x_saved = x;
     if ((e = make_map(s->tmaps[kMapX128], x, (uint64_t)T * B, I, kRows))) return e;
     if ((e = make_map(s->tmaps[kMapX64], x, (uint64_t)T * B, I, kChunk))) return e;
@@ -684,9 +715,18 @@ cudaError_t bf16_forward_setup(stacklstm *s, const __nv_bfloat16 *x, const __nv_
     return cudaGetLastError();
 }
 
+cudaError_t bf16_gather_push_x(stacklstm *s, const __nv_bfloat16 *x)
+{
+    const size_t rows = (size_t)s->Tr * s->B;
+    gather_push_x<<<grid_for(s, rows * (s->I / 8)), 256, 0, s->stream>>>(rows, s->B, s->I / 8, s->xidx,
+                                                                          (const uint4 *)x, (uint4 *)s->x_push);
+    s->launches += 1;
+    return cudaGetLastError();
+}
+
 cudaError_t bf16_forward_steps(stacklstm *s, const float *bias)
 {
-    const int T = s->T, B = s->B, H = s->H;
+    const int T = s->Tr, B = s->B, H = s->H;
     const int nctf = std::max((int)ceil_div(H, s->uf), s->pf.on ? s->pf.n_ct : 0);
     cudaError_t e;
     if (s->fc.on)
@@ -727,7 +767,7 @@ cudaError_t bf16_backward_setup(stacklstm *s)
 cudaError_t bf16_backward_steps(stacklstm *s, float *dx, bool *dx_done)
 {
     *dx_done = false;
-    const int T = s->T, B = s->B, H = s->H;
+    const int T = s->Tr, B = s->B, H = s->H;
     cudaError_t e;
     const StepArgs a = step_args(s, nullptr, s->w_bwd, 0, s->kcb, s->sb);
     if (s->bc.on) return bf16_launch_bwd_cluster(s, step_args(s, nullptr, s->w_bcl, 0, s->kcb, 0));
@@ -754,10 +794,12 @@ cudaError_t bf16_backward_steps(stacklstm *s, float *dx, bool *dx_done)
 cudaError_t bf16_dx(stacklstm *s, float *dx)
 {
     if (!dx) return cudaSuccess;
-    const size_t R = (size_t)s->T * s->B;
+    const size_t R = (size_t)s->Tr * s->B;
     DxArgs d;
     d.R = R; d.I = s->I; d.KC = s->kcb; d.S = s->sx;
     d.wpack = (const uint8_t *)s->w_dx; d.dx = dx; d.limit = s->wait_limit; d.err = s->err;
+    d.xidx = s->push_only ? s->xidx : nullptr;
+    d.B = s->B;
     const dim3 g(s->nxt, ceil_div(R, kRows));
     const size_t smem = smem_bytes(s->sx, s->nx);
     const CUtensorMap &tmg = map(s, kMapG128);

@@ -52,6 +52,7 @@ struct WsArgs {
     int dx_v8;               // dx is 32-byte aligned (whole-sector row stores)
     int nxt;                 // 256-column tiles of dx
     float *dx;               // [T B][I]
+    const int32_t *dx_xidx;  // push-only mode: real step of each virtual row's step (-1: none), else null
     const uint8_t *wdx;      // W_x packed as [nxt][KC][256 rows][64], 128-byte swizzled rows
 };
 
@@ -805,14 +806,23 @@ __device__ __forceinline__ void dx_role(const CUtensorMap *tm_g, const WsArgs &p
             tc::tc_fence_after();
             const size_t row = (size_t)row0 + q * 32 + lane;
             const uint32_t taddr = tmem + acc * kDxN + ((uint32_t)(q * 32) << 16) + part * CPT;
-            float *drow = p.dx + row * I;
+            // the dx row of this accumulator row: the same row, or (push-only mode) the
+            // real step of this virtual row's push; rows past an instance's pushes have none
+            bool out = row < R;
+            size_t orow = row;
+            if (out && p.dx_xidx) {
+                const int tr = p.dx_xidx[row];
+                out = tr >= 0;
+                orow = (size_t)tr * B + row % B;
+            }
+            float *drow = p.dx + orow * I;
 #pragma unroll 1
             for (int cg = 0; cg < CPT / 16; ++cg) {
                 uint32_t v[16];
                 tmem_cols<16>(taddr + cg * 16, v);
                 tc::tmem_wait_ld();
                 const int col = xt * kDxN + part * CPT + cg * 16;
-                if (row < R) {
+                if (out) {
 #pragma unroll
                     for (int h = 0; h < 2; ++h)
                         if (col + 8 * h < I) {  // I is a multiple of 8
@@ -1299,6 +1309,7 @@ cudaError_t bf16_launch_bwd_persist(stacklstm *s, const StepArgs &a, const CUten
     p.dx_v8 = ((uintptr_t)dx & 31) == 0;
     p.nxt = s->nxt;
     p.dx = dx;
+    p.dx_xidx = s->push_only ? s->xidx : nullptr;
     p.wdx = (const uint8_t *)s->w_dx;
     cudaError_t e = cudaMemsetAsync(p.cnt, 0, sizeof(int32_t) * p.n_rt * p.cs, s->stream);
     if (e) return e;

@@ -53,6 +53,21 @@ struct stacklstm {
     int32_t *slot_scratch = nullptr;  // global slot-tag stack when it does not fit on chip
     int32_t *err = nullptr;           // device-detected status (first error wins)
 
+    // push-only mode (stacklstm_set_mode): the step kernels run over a virtual timeline
+    // in which virtual step k of instance b is its k-th push; only push steps' writes are
+    // ever read (Sec. 3, Observation 2), so the other steps need no computation
+    int push_only = 0;
+    int Tr = 0;                  // steps the step kernels run: T, or the most pushes of any instance
+    int32_t *vtop = nullptr;     // [T+1][B] virtual history index each virtual step reads
+    int32_t *vmap = nullptr;     // [T+1][B] real history index -> virtual index (-1: a non-push write)
+    int32_t *vy = nullptr;       // [T+1][B] vmap[top[t][b]]: virtual index of the top at real time t
+    int32_t *vslot = nullptr;    // [T+1][B] virtual index of the state last pushed into each slot (-1: none)
+    int32_t *xidx = nullptr;     // [T][B] real step of virtual step k (-1: past the instance's pushes)
+    int32_t *vstep = nullptr;    // [T][B] virtual step of real step t (-1: not a push)
+    void *x_push = nullptr;      // [T][B][I] bf16: x of each virtual step (zero past the pushes)
+    int32_t *kmax = nullptr;     // device: the most pushes of any instance
+    int32_t *kmax_host = nullptr;  // pinned host copy
+
     // forward state, write-once history: index 0 = initial state, t+1 = written at step t
     void *hist_h = nullptr;  // [T+1][B][H] dtype
     void *hr = nullptr;      // bf16: [T+1][B][H] h operand of each step, hr[t][b] = hist_h[top[t][b]][b]
@@ -123,6 +138,12 @@ cudaError_t smem_at_least(const void *fn, size_t bytes);
 cudaError_t launch_gather_rows(stacklstm *s, const int32_t *idx, int rows, size_t elem_bytes,
                                const void *hist, void *out, int row_elems);
 cudaError_t launch_seed_grads(stacklstm *s, const float *d_top_h, const float *dy);
+// push-only mode: the virtual timeline's indices from the prepass's (kernel), and the
+// number of virtual steps (read back to the host: synchronizes the stream)
+cudaError_t launch_compact(stacklstm *s);
+cudaError_t read_virtual_steps(stacklstm *s);
+// push-only mode: zero the rows of dx [T][B][I] that belong to non-push steps
+cudaError_t launch_zero_nonpush_rows(stacklstm *s, float *dx);
 
 // ---- fp32 CUDA-core path (fp32_path.cu)
 cudaError_t fp32_forward_setup(stacklstm *s, const float *h0, const float *c0, const float *W);
@@ -140,6 +161,8 @@ cudaError_t bf16_backward_setup(stacklstm *s);
 cudaError_t bf16_backward_steps(stacklstm *s, float *dx, bool *dx_done);
 cudaError_t bf16_dx(stacklstm *s, float *dx);
 cudaError_t bf16_dw(stacklstm *s, float *dW, float *dbias);
+// push-only mode: x of each virtual step into s->x_push (bf16 rows)
+cudaError_t bf16_gather_push_x(stacklstm *s, const __nv_bfloat16 *x);
 size_t bf16_workspace_bytes(int T, int B, int I, int H, int num_sms);
 const char *bf16_unsupported(int T, int B, int I, int H);
 std::string bf16_describe(const stacklstm *s);

@@ -98,7 +98,101 @@ __global__ void seed_grads_kernel(int T, int B, int H, const int32_t *__restrict
     }
 }
 
+// Push-only mode: the virtual timeline of each instance. By Observation 2 of Sec. 3 only
+// a push step's write is ever read (a pop or hold writes slot p + 1 above the new top,
+// and the next push overwrites it before the pointer gets there), so instance b's
+// computation is the chain of its push steps alone: virtual step k is its k-th push, it
+// reads the virtual state of the push that wrote the slot it reads (or the initial state,
+// virtual index 0) and writes virtual history row k + 1. One thread per instance walks its
+// steps in order, so every index it looks up was set at an earlier step. Virtual steps
+// past an instance's last push read the initial state and their writes are never read.
+// A step is a push when its pointer moves up by one (ops the prepass rejected ran as
+// holds). vslot is the stack of Sec. 2's definition: each slot's last pushed state.
+// kmax (zero on entry) receives the most pushes of any instance.
+__global__ void __launch_bounds__(kPrepassThreads)
+compact_kernel(int T, int B, const int32_t *__restrict__ p_traj, const int32_t *__restrict__ top,
+               int32_t *__restrict__ vtop, int32_t *__restrict__ vmap,
+               int32_t *__restrict__ vy, int32_t *__restrict__ vslot, int32_t *__restrict__ xidx,
+               int32_t *__restrict__ vstep, int32_t *__restrict__ kmax)
+{
+    const int b = blockIdx.x * kPrepassThreads + threadIdx.x;
+    if (b >= B) return;
+    // virtual index of the state at real history index j (written at step j - 1, or the
+    // initial state at j = 0); a state that is read is always a push write or the initial
+    // state, so the clamp never applies to valid prepass output
+    auto vof = [&](int j) { return max(0, vmap[(size_t)j * B + b]); };
+    vmap[b] = 0;
+    vslot[b] = 0;  // slot 0: the initial state
+    for (int sl = 1; sl <= T; ++sl) vslot[(size_t)sl * B + b] = -1;
+    int k = 0;
+    for (int t = 0; t < T; ++t) {
+        const size_t i = (size_t)t * B + b;
+        const int rd = vof(top[i]);
+        vy[i] = rd;
+        if (p_traj[i + B] - p_traj[i] == 1) {
+            xidx[(size_t)k * B + b] = t;
+            vtop[(size_t)k * B + b] = rd;
+            vstep[i] = k;
+            vmap[i + B] = k + 1;
+            vslot[(size_t)(p_traj[i] + 1) * B + b] = k + 1;
+            ++k;
+        } else {
+            vstep[i] = -1;
+            vmap[i + B] = -1;
+        }
+    }
+    vy[(size_t)T * B + b] = vof(top[(size_t)T * B + b]);
+    for (int kk = k; kk < T; ++kk) {
+        xidx[(size_t)kk * B + b] = -1;
+        vtop[(size_t)kk * B + b] = 0;
+    }
+    vtop[(size_t)T * B + b] = 0;
+    atomicMax(kmax, k);
+}
+
+// Push-only mode: dx rows of the steps that do not push are zero (a state no step reads
+// has zero gradient); the push rows are written by the input-gradient contraction.
+__global__ void zero_nonpush_rows_kernel(size_t rows, int I4, const int32_t *__restrict__ vstep,
+                                         float4 *__restrict__ dx)
+{
+    const size_t n = rows * I4;
+    for (size_t e = blockIdx.x * (size_t)blockDim.x + threadIdx.x; e < n; e += (size_t)gridDim.x * blockDim.x)
+        if (vstep[e / I4] < 0) dx[e] = make_float4(0.f, 0.f, 0.f, 0.f);
+}
+
 }  // namespace
+
+cudaError_t launch_compact(stacklstm *s)
+{
+    cudaError_t e = cudaMemsetAsync(s->kmax, 0, sizeof(int32_t), s->stream);
+    if (e) return e;
+    compact_kernel<<<ceil_div(s->B, kPrepassThreads), kPrepassThreads, 0, s->stream>>>(
+        s->T, s->B, s->p_traj, s->top, s->vtop, s->vmap, s->vy, s->vslot, s->xidx, s->vstep, s->kmax);
+    s->launches += 1;
+    return cudaGetLastError();
+}
+
+cudaError_t read_virtual_steps(stacklstm *s)
+{
+    cudaError_t e = cudaMemcpyAsync(s->kmax_host, s->kmax, sizeof(int32_t), cudaMemcpyDeviceToHost, s->stream);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s->stream);
+    if (e) return e;
+    // at least one step, so that every kernel has work of its usual shape (a batch with no
+    // push at all runs one virtual step whose write nobody reads)
+    s->Tr = std::max(1, std::min(s->T, (int)*s->kmax_host));
+    return cudaSuccess;
+}
+
+cudaError_t launch_zero_nonpush_rows(stacklstm *s, float *dx)
+{
+    if (!dx) return cudaSuccess;
+    const size_t rows = (size_t)s->T * s->B;
+    const int I4 = s->I / 4;  // the bf16 path has I % 8 == 0
+    const unsigned grid = (unsigned)std::min<size_t>(ceil_div(rows * I4, 256), (size_t)s->num_sms * 16);
+    zero_nonpush_rows_kernel<<<grid, 256, 0, s->stream>>>(rows, I4, s->vstep, (float4 *)dx);
+    s->launches += 1;
+    return cudaGetLastError();
+}
 
 cudaError_t smem_at_least(const void *fn, size_t bytes)
 {
@@ -164,7 +258,9 @@ cudaError_t launch_seed_grads(stacklstm *s, const float *d_top_h, const float *d
     if (!d_top_h && !dy) return cudaSuccess;
     const size_t n = (size_t)s->B * s->H;
     const unsigned grid = (unsigned)std::min<size_t>(ceil_div(n, 256), (size_t)s->num_sms * 16);
-    seed_grads_kernel<<<grid, 256, 0, s->stream>>>(s->T, s->B, s->H, s->top, d_top_h, dy, s->dhist_h);
+    // the (virtual, in push-only mode) history index of the top at each real time
+    seed_grads_kernel<<<grid, 256, 0, s->stream>>>(s->T, s->B, s->H, s->push_only ? s->vy : s->top, d_top_h, dy,
+                                                   s->dhist_h);
     s->launches += 1;
     return cudaGetLastError();
 }

@@ -54,11 +54,14 @@ def to_numpy(out: dict) -> dict:
     return res
 
 
-def run(w, device: int = 0, d_top_h: Optional[np.ndarray] = None) -> dict:
-    """Forward + backward of workload ``w`` on ``cuda:device``; numpy results."""
+def run(w, device: int = 0, d_top_h: Optional[np.ndarray] = None, mode: int = bd.SL_MODE_HOMOGENIZED) -> dict:
+    """Forward + backward of workload ``w`` on ``cuda:device`` in the given mode; numpy
+    results (plus ``steps_run``, the steps the step kernels ran)."""
     import torch
     hd = bd.stacklstm_create(w.T, w.B, w.I, w.H, bd.SL_BF16 if w.dtype == "bf16" else bd.SL_FP32, device)
     try:
+        if mode != bd.SL_MODE_HOMOGENIZED:
+            bd.stacklstm_set_mode(hd, mode)
         ins = upload(w, device)
         out = alloc_outputs(w, device)
         for v in out.values():  # an element the path does not write cannot match the oracle
@@ -68,7 +71,9 @@ def run(w, device: int = 0, d_top_h: Optional[np.ndarray] = None) -> dict:
             ins["x"].device)
         forward_backward(hd, ins, out, d_top_h=seed)
         torch.cuda.synchronize(device)
-        return to_numpy(out)
+        res = to_numpy(out)
+        res["steps_run"] = bd.stacklstm_steps_run(hd)
+        return res
     finally:
         hd.destroy()
 

@@ -10,6 +10,8 @@ calls in a row (the second call runs on the scratch the first one left behind), 
 call changes neither torch's allocated memory nor the device's free memory, and that
 sizes beyond its limit are refused. The file is named to be collected last.
 """
+import gc
+
 import numpy as np
 import pytest
 import torch
@@ -55,12 +57,19 @@ def test_a_call_allocates_no_device_memory():
     s = torch.empty(w.T + 1, w.B, dtype=torch.int32, device=dev)
     bd.stacklstm_pointers_noalloc(ops, p, s)  # the device's one-time set-up happens here
     torch.cuda.synchronize(dev)
-    for _ in range(2):
-        alloc0, free0 = torch.cuda.memory_allocated(dev), torch.cuda.mem_get_info(dev)[0]
-        bd.stacklstm_pointers_noalloc(ops, p, s)
-        torch.cuda.synchronize(dev)
-        assert torch.cuda.memory_allocated(dev) == alloc0
-        assert torch.cuda.mem_get_info(dev)[0] == free0
+    # tensors of earlier tests are collected first, and no collection runs during the
+    # measurement, so the counts change only if the call itself allocated
+    gc.collect()
+    gc.disable()
+    try:
+        for _ in range(2):
+            alloc0, free0 = torch.cuda.memory_allocated(dev), torch.cuda.mem_get_info(dev)[0]
+            bd.stacklstm_pointers_noalloc(ops, p, s)
+            torch.cuda.synchronize(dev)
+            assert torch.cuda.memory_allocated(dev) == alloc0
+            assert torch.cuda.mem_get_info(dev)[0] == free0
+    finally:
+        gc.enable()
 
 
 def test_refuses_sizes_beyond_its_scratch():
