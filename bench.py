@@ -137,7 +137,9 @@ def phase_kernel(plan, phase, dtype):
                 "backward": ("bwd_pointwise_f32+bwd_contract_f32", "fp32_path.cu", "2T"),
                 "dx": ("dx_f32", "fp32_path.cu", 1), "dw": ("dw_f32", "fp32_path.cu", 1)}[phase]
     if phase in ("forward", "backward"):
-        m = re.search(phase + r" (persistent|per-step|cluster) U=(\d+)", plan)
+        m = re.search(phase + r" (persistent|per-step|cluster|cuda-core) U=(\d+)", plan)
+        if m and m.group(1) == "cuda-core":
+            return "%s<BT>" % ("step_ccf" if phase == "forward" else "step_ccb"), "bf16_small.cu", 1
         if m and m.group(1) == "cluster":
             return ("%s<U=%s,%s>" % ("step_cl" if phase == "forward" else "step_clb", m.group(2), phase),
                     "bf16_cluster.cu", 1)
@@ -368,8 +370,9 @@ def measure_workload(w, steps, warmup, min_seconds=0.0, push_only=False, with_e2
 
 def measure_group(name, steps, warmup):
     """The three StackLSTMs of an arc-hybrid parser batch (stack, buffer, action history),
-    forward + backward at the same time, one stream each; against the same three timed one
-    at a time. value = instance-steps of all three / second."""
+    forward + backward through the grouped calls (their step kernels as one launch each
+    way); beside it, the same three as separate calls on three streams, and each timed
+    alone. value = instance-steps of all three / second through the grouped calls."""
     import torch
     from paper_1904_03409_gb300 import runner, workloads as wl
 
@@ -391,7 +394,9 @@ def measure_group(name, steps, warmup):
             flush.zero_()
             a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             a.record(cur)
-            if members is None:
+            if members == "one_call":
+                runner.group_forward_backward_one_call(hds, ins, outs)
+            elif members is None:
                 runner.group_forward_backward(hds, ins, outs)
             else:
                 hd, st = hds[members]
@@ -407,8 +412,9 @@ def measure_group(name, steps, warmup):
     clocks = ClockSampler(0)
     time.sleep(0.3)
     clocks.start()
-    ms = timed(None)
+    ms = timed("one_call")
     clocks.stop()
+    ms_streams = timed(None)
     alone = {k: timed(k) for k in runner.GROUP_MEMBERS}
     units = sum(g[k].B * g[k].T for k in runner.GROUP_MEMBERS)
     peaks, src = load_peaks()
@@ -420,7 +426,8 @@ def measure_group(name, steps, warmup):
                            g["action"].T, g["action"].I, g["stack"].H, g["stack"].seed),
            "value": units / (ms / 1e3), "unit": "instance-steps/s (three StackLSTMs)",
            "transitions_per_s": g["stack"].B * g["stack"].T / (ms / 1e3),
-           "ms_per_step": ms, "ms_one_at_a_time": {k: round(v, 4) for k, v in alone.items()},
+           "ms_per_step": ms, "ms_three_streams_separate_calls": ms_streams,
+           "ms_one_at_a_time": {k: round(v, 4) for k, v in alone.items()},
            "overlap_speedup": round(sum(alone.values()) / ms, 3), "steps": steps, "warmup": warmup,
            "step_roofline": roofline_of(fl, by, ms / 1e3, peaks, src), "clocks": clocks.summary()}
     for hd, _ in hds.values():

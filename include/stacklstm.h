@@ -53,6 +53,9 @@
  *                                  over k CTAs per 64-unit column tile (k = 4)
  *   STACKLSTM_DX_SPARE=0 | k       dx in its own launch (0), or by at most k extra CTAs of
  *                                  the persistent backward launch
+ *   STACKLSTM_CUDA_CORE=0 | 1      small batches (B <= 32, H <= 256): never (0), or
+ *                                  whenever the shape allows (1), the CUDA-core cluster
+ *                                  kernels instead of the tensor-core ones
  */
 #ifndef STACKLSTM_H
 #define STACKLSTM_H
@@ -172,6 +175,49 @@ sl_status stacklstm_set_mode(stacklstm_t s, sl_mode mode);
 /* Number of steps the step kernels ran in the last forward: T in the homogenized mode,
  * the most pushes of any instance (at least 1) in the push-only mode. */
 sl_status stacklstm_steps_run(stacklstm_t s, int *steps);
+
+/*
+ * Grouped calls: the forward (backward) of up to 4 handles on one device in one call. A
+ * transition-based parser runs several StackLSTMs over one batch (the stack, the buffer
+ * and the action history of Sec. 4.1; Table 1 gives each transition's stack and buffer
+ * ops); with the transitions known, their recurrences are independent of one another.
+ * The result is that of calling stacklstm_forward (stacklstm_backward) on each handle,
+ * each on its own stream. When every handle runs the one-row-tile cluster kernels (B <= 64)
+ * with the same cluster size (the same H), their step kernels run as ONE launch of one
+ * thread-block cluster per handle, on the first handle's stream; each handle's stream
+ * joins that stream before the launch and waits for it afterwards. Otherwise each handle
+ * launches its own. The work before and after the steps stays on each handle's stream.
+ * Timing: the one launch counts in the first handle's forward (backward) phase.
+ * Returns the first failing handle's status (SL_ERR_ARG: n outside 1..4, a null or
+ * repeated handle, handles on different devices).
+ */
+typedef struct {
+    const void *x;        /* as stacklstm_forward's arguments of the same names */
+    const int8_t *ops;
+    const void *h0;
+    const float *c0;
+    const void *W;
+    const float *bias;
+    void *h_stack;
+    float *c_stack;
+    int32_t *p_final;
+    int32_t *p_traj;
+    int32_t *src;
+    void *y;
+} sl_forward_args;
+
+typedef struct {
+    const float *d_top_h;  /* as stacklstm_backward's arguments of the same names */
+    const float *dy;
+    float *dx;
+    float *dh0;
+    float *dc0;
+    float *dW;
+    float *dbias;
+} sl_backward_args;
+
+sl_status stacklstm_forward_group(int n, const stacklstm_t *hs, const sl_forward_args *args);
+sl_status stacklstm_backward_group(int n, const stacklstm_t *hs, const sl_backward_args *args);
 
 /*
  * Phases of a forward + backward, as stacklstm_get_timing reports them. Each phase is a

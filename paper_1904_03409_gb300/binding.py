@@ -60,6 +60,8 @@ def load(path: Optional[str] = None):
     lib.stacklstm_get_timing.argtypes = [vp, vp, vp, i]
     lib.stacklstm_pointers_noalloc.argtypes = [i, i, vp, vp, vp, vp]
     lib.stacklstm_pointers_noalloc.restype = ctypes.c_int
+    lib.stacklstm_forward_group.argtypes = [i, vp, vp]
+    lib.stacklstm_backward_group.argtypes = [i, vp, vp]
     lib.stacklstm_set_mode.argtypes = [vp, i]
     lib.stacklstm_steps_run.argtypes = [vp, vp]
     lib.stacklstm_plan.argtypes = [vp]
@@ -75,7 +77,7 @@ def load(path: Optional[str] = None):
     lib.stacklstm_head_last_error.restype = ctypes.c_char_p
     for fn in ("stacklstm_create", "stacklstm_forward", "stacklstm_backward", "stacklstm_set_stream",
                "stacklstm_set_async", "stacklstm_status", "stacklstm_destroy", "stacklstm_set_timing",
-               "stacklstm_get_timing", "stacklstm_set_mode", "stacklstm_steps_run", "stacklstm_head_create", "stacklstm_head_run", "stacklstm_head_add_h0_grads",
+               "stacklstm_get_timing", "stacklstm_forward_group", "stacklstm_backward_group", "stacklstm_set_mode", "stacklstm_steps_run", "stacklstm_head_create", "stacklstm_head_run", "stacklstm_head_add_h0_grads",
                "stacklstm_head_status", "stacklstm_head_destroy"):
         getattr(lib, fn).restype = ctypes.c_int
     _lib = lib
@@ -171,30 +173,77 @@ def stacklstm_status(hd: StackLSTMHandle):
     _check(hd.h, load().stacklstm_status(hd.h), "stacklstm_status")
 
 
+FWD_FIELDS = ("x", "ops", "h0", "c0", "W", "bias", "h_stack", "c_stack", "p_final", "p_traj", "src", "y")
+BWD_FIELDS = ("d_top_h", "dy", "dx", "dh0", "dc0", "dW", "dbias")
+
+
+class _FwdArgs(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_void_p) for n in FWD_FIELDS]
+
+
+class _BwdArgs(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_void_p) for n in BWD_FIELDS]
+
+
 def stacklstm_forward(hd: StackLSTMHandle, x, ops, h0, c0, W, bias, h_stack=None, c_stack=None, p_final=None,
                       p_traj=None, src=None, y=None):
     """Forward over all T steps; see include/stacklstm.h for the layout of each tensor."""
+    args = _forward_ptrs(hd, x, ops, h0, c0, W, bias, h_stack, c_stack, p_final, p_traj, src, y)
+    _check(hd.h, load().stacklstm_forward(hd.h, *args), "stacklstm_forward")
+
+
+def _forward_ptrs(hd, x, ops, h0, c0, W, bias, h_stack=None, c_stack=None, p_final=None, p_traj=None, src=None,
+                  y=None):
     import torch
     T, B, I, H, d, dt = hd.T, hd.B, hd.I, hd.H, hd.device, hd.tdtype
-    args = [
+    return [
         _ptr(x, d, dt, (T, B, I), "x"), _ptr(ops, d, torch.int8, (T, B), "ops"), _ptr(h0, d, dt, (B, H), "h0"),
         _ptr(c0, d, torch.float32, (B, H), "c0"), _ptr(W, d, dt, (I + H, 4 * H), "W"),
         _ptr(bias, d, torch.float32, (4 * H,), "bias"), _ptr(h_stack, d, dt, (T + 1, B, H), "h_stack"),
         _ptr(c_stack, d, torch.float32, (T + 1, B, H), "c_stack"), _ptr(p_final, d, torch.int32, (B,), "p_final"),
         _ptr(p_traj, d, torch.int32, (T + 1, B), "p_traj"), _ptr(src, d, torch.int32, (T + 1, B), "src"),
         _ptr(y, d, dt, (T, B, H), "y")]
-    _check(hd.h, load().stacklstm_forward(hd.h, *args), "stacklstm_forward")
 
 
 def stacklstm_backward(hd: StackLSTMHandle, d_top_h=None, dy=None, dx=None, dh0=None, dc0=None, dW=None,
                        dbias=None):
     """Backward of the last forward; gradients are overwritten."""
+    args = _backward_ptrs(hd, d_top_h, dy, dx, dh0, dc0, dW, dbias)
+    _check(hd.h, load().stacklstm_backward(hd.h, *args), "stacklstm_backward")
+
+
+def _backward_ptrs(hd, d_top_h=None, dy=None, dx=None, dh0=None, dc0=None, dW=None, dbias=None):
     import torch
     T, B, I, H, d, f = hd.T, hd.B, hd.I, hd.H, hd.device, torch.float32
-    args = [_ptr(d_top_h, d, f, (B, H), "d_top_h"), _ptr(dy, d, f, (T, B, H), "dy"),
+    return [_ptr(d_top_h, d, f, (B, H), "d_top_h"), _ptr(dy, d, f, (T, B, H), "dy"),
             _ptr(dx, d, f, (T, B, I), "dx"), _ptr(dh0, d, f, (B, H), "dh0"), _ptr(dc0, d, f, (B, H), "dc0"),
             _ptr(dW, d, f, (I + H, 4 * H), "dW"), _ptr(dbias, d, f, (4 * H,), "dbias")]
-    _check(hd.h, load().stacklstm_backward(hd.h, *args), "stacklstm_backward")
+
+
+def _group_call(fn, hds, args, ptrs_of, Struct, fields, where):
+    n = len(hds)
+    handles = (ctypes.c_void_p * n)(*[hd.h for hd in hds])
+    arr = (Struct * n)()
+    for i, (hd, a) in enumerate(zip(hds, args)):
+        for name, p in zip(fields, ptrs_of(hd, **a)):
+            setattr(arr[i], name, p.value if p is not None else None)
+    st = fn(n, handles, arr)
+    if st != 0:
+        msg = "; ".join(m for m in (load().stacklstm_last_error(hd.h).decode() for hd in hds) if m)
+        raise StackLSTMError(st, where, msg)
+
+
+def stacklstm_forward_group(hds, args):
+    """Forward of several handles in one call (include/stacklstm.h): ``args`` holds, per
+    handle, a dict of stacklstm_forward's keyword arguments."""
+    _group_call(load().stacklstm_forward_group, hds, args, _forward_ptrs, _FwdArgs, FWD_FIELDS,
+                "stacklstm_forward_group")
+
+
+def stacklstm_backward_group(hds, args):
+    """Backward of several handles in one call: ``args`` as for stacklstm_backward."""
+    _group_call(load().stacklstm_backward_group, hds, args, _backward_ptrs, _BwdArgs, BWD_FIELDS,
+                "stacklstm_backward_group")
 
 
 def stacklstm_pointers_noalloc(ops, p_traj, src, stream=None):

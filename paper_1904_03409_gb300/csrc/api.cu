@@ -140,6 +140,182 @@ sl_status read_status(stacklstm *s)
     return SL_OK;
 }
 
+// ---- the phases of a forward and a backward call, shared by the single and grouped calls
+
+// Argument checks, the index prepass and the forward setup (weight packing, initial state).
+sl_status fwd_begin(stacklstm *s, const sl_forward_args &a)
+{
+    s->last_error.clear();
+    if (!a.x || !a.ops || !a.h0 || !a.c0 || !a.W || !a.bias || !a.p_final)
+        return fail(s, SL_ERR_ARG, "x, ops, h0, c0, W, bias and p_final are required");
+    const void *ptrs[] = {a.x, a.h0, a.c0, a.W, a.bias, a.h_stack, a.c_stack, a.p_final, a.p_traj, a.src, a.y};
+    for (const void *p : ptrs)
+        if (p && !aligned16(p)) return fail(s, SL_ERR_ARG, "tensor pointers must be 16-byte aligned");
+    cudaError_t e;
+    s->fwd_done = 0;
+    {
+        Phase ph(s, SL_PHASE_PREPASS);
+        if ((e = sl::launch_prepass(s, a.ops))) return cuda_fail(s, e, "prepass");
+        s->Tr = s->T;
+        // push-only mode: each instance's pushes as a virtual timeline; the step count the
+        // kernels run is read back here (the one synchronization of this mode's forward)
+        if (s->push_only && ((e = sl::launch_compact(s)) || (e = sl::read_virtual_steps(s))))
+            return cuda_fail(s, e, "push-only indices");
+    }
+    {
+        Phase ph(s, SL_PHASE_FWD_SETUP);
+        if (s->dt == SL_FP32)
+            e = sl::fp32_forward_setup(s, (const float *)a.h0, a.c0, (const float *)a.W);
+        else
+            e = sl::bf16_forward_setup(s, (const __nv_bfloat16 *)a.x, (const __nv_bfloat16 *)a.h0, a.c0,
+                                       (const __nv_bfloat16 *)a.W);
+        if (e) return cuda_fail(s, e, "forward setup");
+    }
+    return SL_OK;
+}
+
+// The gradient history is cleared on the side stream while the forward runs (the forward
+// leaves most of the memory bandwidth unused); the side stream first waits for `side_go`,
+// recorded on the caller's stream before the forward steps (a previous backward reads it).
+sl_status fwd_clear(stacklstm *s)
+{
+    const size_t hist_bytes = sizeof(float) * (size_t)(s->T + 1) * s->B * s->H;
+    cudaError_t e;
+    if ((e = cudaStreamWaitEvent(s->side, s->side_go, 0)) ||
+        (e = cudaMemsetAsync(s->dhist_h, 0, hist_bytes, s->side)) ||
+        (e = cudaMemsetAsync(s->dhist_c, 0, hist_bytes, s->side)) || (e = cudaEventRecord(s->cleared, s->side)))
+        return cuda_fail(s, e, "clear");
+    s->clear_queued = 1;
+    return SL_OK;
+}
+
+sl_status fwd_steps(stacklstm *s, const sl_forward_args &a)
+{
+    Phase ph(s, SL_PHASE_FORWARD);
+    cudaError_t e;
+    if ((e = cudaEventRecord(s->side_go, s->stream))) return cuda_fail(s, e, "forward");
+    if (s->dt == SL_FP32)
+        e = sl::fp32_forward_steps(s, (const float *)a.x, (const float *)a.W, a.bias);
+    else
+        e = sl::bf16_forward_steps(s, a.bias);
+    if (e) return cuda_fail(s, e, "forward");
+    return fwd_clear(s);
+}
+
+// The optional outputs: final pointers, trajectories, provenance, y, the slot-indexed stack.
+sl_status fwd_end(stacklstm *s, const sl_forward_args &a)
+{
+    const int T = s->T, B = s->B, H = s->H;
+    const size_t es = elem_size(s->dt);
+    cudaError_t e;
+    {
+        Phase ph(s, SL_PHASE_OUTPUTS);
+        if ((e = cudaMemcpyAsync(a.p_final, s->p_traj + (size_t)T * B, sizeof(int32_t) * B,
+                                 cudaMemcpyDeviceToDevice, s->stream)))
+            return cuda_fail(s, e, "p_final");
+        if (a.p_traj && (e = cudaMemcpyAsync(a.p_traj, s->p_traj, sizeof(int32_t) * (T + 1) * B,
+                                             cudaMemcpyDeviceToDevice, s->stream)))
+            return cuda_fail(s, e, "p_traj");
+        if (a.src && (e = cudaMemcpyAsync(a.src, s->top, sizeof(int32_t) * (T + 1) * B, cudaMemcpyDeviceToDevice,
+                                          s->stream)))
+            return cuda_fail(s, e, "src");
+        // history index of the top after each step and of each slot's last write (in
+        // push-only mode: virtual indices, and each slot's last push, as in Sec. 2)
+        const int32_t *ytop = s->push_only ? s->vy : s->top, *slots = s->push_only ? s->vslot : s->slot_last;
+        if (a.y && (e = sl::launch_gather_rows(s, ytop + B, T * B, es, s->hist_h, a.y, H)))
+            return cuda_fail(s, e, "y");
+        if (a.h_stack && (e = sl::launch_gather_rows(s, slots, (T + 1) * B, es, s->hist_h, a.h_stack, H)))
+            return cuda_fail(s, e, "h_stack");
+        if (a.c_stack && (e = sl::launch_gather_rows(s, slots, (T + 1) * B, 4, s->hist_c, a.c_stack, H)))
+            return cuda_fail(s, e, "c_stack");
+    }
+    s->fwd_done = 1;
+    return SL_OK;
+}
+
+// Argument checks, the cleared and seeded gradient history, the last step's pointwise
+// backward (and, push-only mode, the zero dx rows of non-push steps).
+sl_status bwd_begin(stacklstm *s, const sl_backward_args &a)
+{
+    s->last_error.clear();
+    if (!s->fwd_done) return fail(s, SL_ERR_STATE, "backward needs a completed forward on this handle");
+    const void *ptrs[] = {a.d_top_h, a.dy, a.dx, a.dh0, a.dc0, a.dW, a.dbias};
+    for (const void *p : ptrs)
+        if (p && !aligned16(p)) return fail(s, SL_ERR_ARG, "tensor pointers must be 16-byte aligned");
+    const size_t hist_bytes = sizeof(float) * (size_t)(s->T + 1) * s->B * s->H;
+    cudaError_t e;
+    Phase ph(s, SL_PHASE_BWD_SETUP);
+    if (s->clear_queued) {
+        // cleared on the side stream during the forward
+        if ((e = cudaStreamWaitEvent(s->stream, s->cleared, 0))) return cuda_fail(s, e, "clear");
+        s->clear_queued = 0;
+    } else {
+        if ((e = cudaMemsetAsync(s->dhist_h, 0, hist_bytes, s->stream))) return cuda_fail(s, e, "clear");
+        if ((e = cudaMemsetAsync(s->dhist_c, 0, hist_bytes, s->stream))) return cuda_fail(s, e, "clear");
+    }
+    if ((e = sl::launch_seed_grads(s, a.d_top_h, a.dy))) return cuda_fail(s, e, "seed");
+    if (s->dt == SL_BF16 && (e = sl::bf16_backward_setup(s))) return cuda_fail(s, e, "backward setup");
+    // push-only mode: the dx rows of steps that do not push are zero; the contraction
+    // writes the others
+    if (s->push_only && (e = sl::launch_zero_nonpush_rows(s, a.dx))) return cuda_fail(s, e, "dx rows");
+    return SL_OK;
+}
+
+sl_status bwd_steps(stacklstm *s, const sl_backward_args &a, bool *dx_done)
+{
+    Phase ph(s, SL_PHASE_BACKWARD);
+    cudaError_t e = s->dt == SL_FP32 ? sl::fp32_backward_steps(s) : sl::bf16_backward_steps(s, a.dx, dx_done);
+    return e ? cuda_fail(s, e, "backward") : SL_OK;
+}
+
+// dx (unless the step launch computed it on otherwise idle SMs), dW and dbias, dh0 and dc0.
+sl_status bwd_end(stacklstm *s, const sl_backward_args &a, bool dx_done)
+{
+    const int B = s->B, H = s->H;
+    cudaError_t e;
+    if (!dx_done) {
+        Phase ph(s, SL_PHASE_DX);
+        e = s->dt == SL_FP32 ? sl::fp32_dx(s, a.dx) : sl::bf16_dx(s, a.dx);
+        if (e) return cuda_fail(s, e, "dx");
+    }
+    {
+        Phase ph(s, SL_PHASE_DW);
+        e = s->dt == SL_FP32 ? sl::fp32_dw(s, a.dW, a.dbias) : sl::bf16_dw(s, a.dW, a.dbias);
+        if (e) return cuda_fail(s, e, "dW");
+    }
+    // slot 0 always holds the initial state, which is history row 0
+    if (a.dh0 && (e = cudaMemcpyAsync(a.dh0, s->dhist_h, sizeof(float) * B * H, cudaMemcpyDeviceToDevice, s->stream)))
+        return cuda_fail(s, e, "dh0");
+    if (a.dc0 && (e = cudaMemcpyAsync(a.dc0, s->dhist_c, sizeof(float) * B * H, cudaMemcpyDeviceToDevice, s->stream)))
+        return cuda_fail(s, e, "dc0");
+    return SL_OK;
+}
+
+// Grouped calls: the members' streams join the first member's stream before the one step
+// launch (before = true), and wait for it afterwards.
+sl_status join_streams(stacklstm *const *hs, int n, bool before)
+{
+    cudaError_t e;
+    for (int m = 1; m < n; ++m) {
+        stacklstm *from = before ? hs[m] : hs[0], *to = before ? hs[0] : hs[m];
+        if ((e = cudaEventRecord(from->join, from->stream)) || (e = cudaStreamWaitEvent(to->stream, from->join, 0)))
+            return cuda_fail(hs[m], e, "stream join");
+    }
+    return SL_OK;
+}
+
+sl_status check_group(int n, const stacklstm_t *hs, const void *args)
+{
+    if (n < 1 || n > kMaxGroup || !hs || !args) return SL_ERR_ARG;
+    for (int m = 0; m < n; ++m) {
+        if (!hs[m]) return SL_ERR_ARG;
+        for (int k = 0; k < m; ++k)
+            if (hs[k] == hs[m]) return fail(hs[m], SL_ERR_ARG, "a handle appears twice in the group");
+        if (hs[m]->device != hs[0]->device) return fail(hs[m], SL_ERR_ARG, "the group's handles share one device");
+    }
+    return SL_OK;
+}
+
 }  // namespace
 
 namespace sl {
@@ -207,11 +383,13 @@ sl_status stacklstm_create(stacklstm_t *out, int T, int B, int I, int H, sl_dtyp
     if (ok) ok = cudaMemset(s->err, 0, 16) == cudaSuccess;
     if (ok) ok = cudaStreamCreateWithFlags(&s->side, cudaStreamNonBlocking) == cudaSuccess &&
                  cudaEventCreateWithFlags(&s->side_go, cudaEventDisableTiming) == cudaSuccess &&
-                 cudaEventCreateWithFlags(&s->cleared, cudaEventDisableTiming) == cudaSuccess;
+                 cudaEventCreateWithFlags(&s->cleared, cudaEventDisableTiming) == cudaSuccess &&
+                 cudaEventCreateWithFlags(&s->join, cudaEventDisableTiming) == cudaSuccess;
     if (!ok) {
         if (s->side) cudaStreamDestroy(s->side);
         if (s->side_go) cudaEventDestroy(s->side_go);
         if (s->cleared) cudaEventDestroy(s->cleared);
+        if (s->join) cudaEventDestroy(s->join);
         cudaGetLastError();
         free_all(s);
         delete s;
@@ -241,75 +419,10 @@ sl_status stacklstm_forward(stacklstm_t s, const void *x, const int8_t *ops, con
                             int32_t *p_traj, int32_t *src, void *y)
 {
     if (!s) return SL_ERR_ARG;
-    s->last_error.clear();
-    if (!x || !ops || !h0 || !c0 || !W || !bias || !p_final)
-        return fail(s, SL_ERR_ARG, "x, ops, h0, c0, W, bias and p_final are required");
-    const void *ptrs[] = {x, h0, c0, W, bias, h_stack, c_stack, p_final, p_traj, src, y};
-    for (const void *p : ptrs)
-        if (p && !aligned16(p)) return fail(s, SL_ERR_ARG, "tensor pointers must be 16-byte aligned");
     DeviceGuard g(s->device);
-    const int T = s->T, B = s->B, H = s->H;
-    const size_t es = elem_size(s->dt);
-    cudaError_t e;
-    s->fwd_done = 0;
-    {
-        Phase ph(s, SL_PHASE_PREPASS);
-        if ((e = sl::launch_prepass(s, ops))) return cuda_fail(s, e, "prepass");
-        s->Tr = T;
-        // push-only mode: each instance's pushes as a virtual timeline; the step count the
-        // kernels run is read back here (the one synchronization of this mode's forward)
-        if (s->push_only && ((e = sl::launch_compact(s)) || (e = sl::read_virtual_steps(s))))
-            return cuda_fail(s, e, "push-only indices");
-    }
-    {
-        Phase ph(s, SL_PHASE_FWD_SETUP);
-        if (s->dt == SL_FP32)
-            e = sl::fp32_forward_setup(s, (const float *)h0, c0, (const float *)W);
-        else
-            e = sl::bf16_forward_setup(s, (const __nv_bfloat16 *)x, (const __nv_bfloat16 *)h0, c0,
-                                       (const __nv_bfloat16 *)W);
-        if (e) return cuda_fail(s, e, "forward setup");
-    }
-    {
-        Phase ph(s, SL_PHASE_FORWARD);
-        // the gradient history is cleared on the side stream while the forward runs (the
-        // forward leaves most of the memory bandwidth unused); the side stream first waits
-        // for everything queued on the caller's stream so far (a previous backward reads it)
-        if ((e = cudaEventRecord(s->side_go, s->stream))) return cuda_fail(s, e, "forward");
-        if (s->dt == SL_FP32)
-            e = sl::fp32_forward_steps(s, (const float *)x, (const float *)W, bias);
-        else
-            e = sl::bf16_forward_steps(s, bias);
-        if (e) return cuda_fail(s, e, "forward");
-        const size_t hist_bytes = sizeof(float) * (size_t)(T + 1) * B * H;
-        if ((e = cudaStreamWaitEvent(s->side, s->side_go, 0)) ||
-            (e = cudaMemsetAsync(s->dhist_h, 0, hist_bytes, s->side)) ||
-            (e = cudaMemsetAsync(s->dhist_c, 0, hist_bytes, s->side)) || (e = cudaEventRecord(s->cleared, s->side)))
-            return cuda_fail(s, e, "clear");
-        s->clear_queued = 1;
-    }
-    {
-        Phase ph(s, SL_PHASE_OUTPUTS);
-        if ((e = cudaMemcpyAsync(p_final, s->p_traj + (size_t)T * B, sizeof(int32_t) * B,
-                                 cudaMemcpyDeviceToDevice, s->stream)))
-            return cuda_fail(s, e, "p_final");
-        if (p_traj && (e = cudaMemcpyAsync(p_traj, s->p_traj, sizeof(int32_t) * (T + 1) * B,
-                                           cudaMemcpyDeviceToDevice, s->stream)))
-            return cuda_fail(s, e, "p_traj");
-        if (src && (e = cudaMemcpyAsync(src, s->top, sizeof(int32_t) * (T + 1) * B, cudaMemcpyDeviceToDevice,
-                                        s->stream)))
-            return cuda_fail(s, e, "src");
-        // history index of the top after each step and of each slot's last write (in
-        // push-only mode: virtual indices, and each slot's last push, as in Sec. 2)
-        const int32_t *ytop = s->push_only ? s->vy : s->top, *slots = s->push_only ? s->vslot : s->slot_last;
-        if (y && (e = sl::launch_gather_rows(s, ytop + B, T * B, es, s->hist_h, y, H)))
-            return cuda_fail(s, e, "y");
-        if (h_stack && (e = sl::launch_gather_rows(s, slots, (T + 1) * B, es, s->hist_h, h_stack, H)))
-            return cuda_fail(s, e, "h_stack");
-        if (c_stack && (e = sl::launch_gather_rows(s, slots, (T + 1) * B, 4, s->hist_c, c_stack, H)))
-            return cuda_fail(s, e, "c_stack");
-    }
-    s->fwd_done = 1;
+    const sl_forward_args a{x, ops, h0, c0, W, bias, h_stack, c_stack, p_final, p_traj, src, y};
+    sl_status st;
+    if ((st = fwd_begin(s, a)) || (st = fwd_steps(s, a)) || (st = fwd_end(s, a))) return st;
     return s->async ? SL_OK : read_status(s);
 }
 
@@ -317,55 +430,78 @@ sl_status stacklstm_backward(stacklstm_t s, const float *d_top_h, const float *d
                              float *dc0, float *dW, float *dbias)
 {
     if (!s) return SL_ERR_ARG;
-    s->last_error.clear();
-    if (!s->fwd_done) return fail(s, SL_ERR_STATE, "backward needs a completed forward on this handle");
-    const void *ptrs[] = {d_top_h, dy, dx, dh0, dc0, dW, dbias};
-    for (const void *p : ptrs)
-        if (p && !aligned16(p)) return fail(s, SL_ERR_ARG, "tensor pointers must be 16-byte aligned");
     DeviceGuard g(s->device);
-    const int T = s->T, B = s->B, H = s->H;
-    const size_t hist_bytes = sizeof(float) * (size_t)(T + 1) * B * H;
-    cudaError_t e;
-    {
-        Phase ph(s, SL_PHASE_BWD_SETUP);
-        if (s->clear_queued) {
-            // cleared on the side stream during the forward
-            if ((e = cudaStreamWaitEvent(s->stream, s->cleared, 0))) return cuda_fail(s, e, "clear");
-            s->clear_queued = 0;
-        } else {
-            if ((e = cudaMemsetAsync(s->dhist_h, 0, hist_bytes, s->stream))) return cuda_fail(s, e, "clear");
-            if ((e = cudaMemsetAsync(s->dhist_c, 0, hist_bytes, s->stream))) return cuda_fail(s, e, "clear");
-        }
-        if ((e = sl::launch_seed_grads(s, d_top_h, dy))) return cuda_fail(s, e, "seed");
-        if (s->dt == SL_BF16 && (e = sl::bf16_backward_setup(s))) return cuda_fail(s, e, "backward setup");
-    }
-    bool dx_done = false;  // computed by the step launch on otherwise idle SMs
-    if (s->push_only) {
-        // the dx rows of steps that do not push are zero; the contraction writes the others
-        Phase ph(s, SL_PHASE_BWD_SETUP);
-        if ((e = sl::launch_zero_nonpush_rows(s, dx))) return cuda_fail(s, e, "dx rows");
-    }
-    {
-        Phase ph(s, SL_PHASE_BACKWARD);
-        e = s->dt == SL_FP32 ? sl::fp32_backward_steps(s) : sl::bf16_backward_steps(s, dx, &dx_done);
-        if (e) return cuda_fail(s, e, "backward");
-    }
-    if (!dx_done) {
-        Phase ph(s, SL_PHASE_DX);
-        e = s->dt == SL_FP32 ? sl::fp32_dx(s, dx) : sl::bf16_dx(s, dx);
-        if (e) return cuda_fail(s, e, "dx");
-    }
-    {
-        Phase ph(s, SL_PHASE_DW);
-        e = s->dt == SL_FP32 ? sl::fp32_dw(s, dW, dbias) : sl::bf16_dw(s, dW, dbias);
-        if (e) return cuda_fail(s, e, "dW");
-    }
-    // slot 0 always holds the initial state, which is history row 0
-    if (dh0 && (e = cudaMemcpyAsync(dh0, s->dhist_h, sizeof(float) * B * H, cudaMemcpyDeviceToDevice, s->stream)))
-        return cuda_fail(s, e, "dh0");
-    if (dc0 && (e = cudaMemcpyAsync(dc0, s->dhist_c, sizeof(float) * B * H, cudaMemcpyDeviceToDevice, s->stream)))
-        return cuda_fail(s, e, "dc0");
+    const sl_backward_args a{d_top_h, dy, dx, dh0, dc0, dW, dbias};
+    bool dx_done = false;
+    sl_status st;
+    if ((st = bwd_begin(s, a)) || (st = bwd_steps(s, a, &dx_done)) || (st = bwd_end(s, a, dx_done))) return st;
     return s->async ? SL_OK : read_status(s);
+}
+
+sl_status stacklstm_forward_group(int n, const stacklstm_t *hs, const sl_forward_args *args)
+{
+    sl_status st = check_group(n, hs, args);
+    if (st) return st;
+    DeviceGuard g(hs[0]->device);
+    stacklstm *h[kMaxGroup];
+    for (int m = 0; m < n; ++m) {
+        h[m] = hs[m];
+        if ((st = fwd_begin(h[m], args[m]))) return st;
+    }
+    if (n > 1 && sl::bf16_can_group(h, n, true)) {
+        const float *bias[kMaxGroup];
+        cudaError_t e;
+        for (int m = 0; m < n; ++m) {
+            bias[m] = args[m].bias;
+            if ((e = cudaEventRecord(h[m]->side_go, h[m]->stream))) return cuda_fail(h[m], e, "forward");
+        }
+        if ((st = join_streams(h, n, true))) return st;
+        {
+            Phase ph(h[0], SL_PHASE_FORWARD);
+            if ((e = sl::bf16_forward_steps_group(h, n, bias, h[0]->stream))) return cuda_fail(h[0], e, "forward");
+        }
+        if ((st = join_streams(h, n, false))) return st;
+        for (int m = 0; m < n; ++m)
+            if ((st = fwd_clear(h[m]))) return st;
+    } else {
+        for (int m = 0; m < n; ++m)
+            if ((st = fwd_steps(h[m], args[m]))) return st;
+    }
+    for (int m = 0; m < n; ++m)
+        if ((st = fwd_end(h[m], args[m]))) return st;
+    for (int m = 0; m < n; ++m)
+        if (!h[m]->async && (st = read_status(h[m]))) return st;
+    return SL_OK;
+}
+
+sl_status stacklstm_backward_group(int n, const stacklstm_t *hs, const sl_backward_args *args)
+{
+    sl_status st = check_group(n, hs, args);
+    if (st) return st;
+    DeviceGuard g(hs[0]->device);
+    stacklstm *h[kMaxGroup];
+    bool dx_done[kMaxGroup] = {};
+    for (int m = 0; m < n; ++m) {
+        h[m] = hs[m];
+        if ((st = bwd_begin(h[m], args[m]))) return st;
+    }
+    if (n > 1 && sl::bf16_can_group(h, n, false)) {
+        if ((st = join_streams(h, n, true))) return st;
+        {
+            Phase ph(h[0], SL_PHASE_BACKWARD);
+            cudaError_t e = sl::bf16_backward_steps_group(h, n, h[0]->stream);
+            if (e) return cuda_fail(h[0], e, "backward");
+        }
+        if ((st = join_streams(h, n, false))) return st;
+    } else {
+        for (int m = 0; m < n; ++m)
+            if ((st = bwd_steps(h[m], args[m], &dx_done[m]))) return st;
+    }
+    for (int m = 0; m < n; ++m)
+        if ((st = bwd_end(h[m], args[m], dx_done[m]))) return st;
+    for (int m = 0; m < n; ++m)
+        if (!h[m]->async && (st = read_status(h[m]))) return st;
+    return SL_OK;
 }
 
 sl_status stacklstm_set_mode(stacklstm_t s, sl_mode mode)
@@ -453,6 +589,7 @@ sl_status stacklstm_destroy(stacklstm_t s)
         }
         if (s->side_go) cudaEventDestroy(s->side_go);
         if (s->cleared) cudaEventDestroy(s->cleared);
+        if (s->join) cudaEventDestroy(s->join);
         collect_timing(s);
         for (cudaEvent_t ev : s->event_pool) cudaEventDestroy(ev);
         s->event_pool.clear();

@@ -159,7 +159,7 @@ __device__ __forceinline__ void deliver_slice(const ClCtl &c, uint8_t *blk, int 
 constexpr int kClFwdThreads = 224;  // 4 epilogue warps, producer, two MMA issuers
 
 template <int U>
-__global__ void __launch_bounds__(kClFwdThreads, 1) step_cl(const __grid_constant__ CUtensorMap tm_x, ClArgs p)
+__device__ __forceinline__ void step_cl_body(const CUtensorMap *tmx, const ClArgs &p)
 {
     static_assert(U == 16, "one h slice (two 8-unit core matrices) per CTA");
     constexpr int NB = 4 * U;
@@ -214,7 +214,7 @@ __global__ void __launch_bounds__(kClFwdThreads, 1) step_cl(const __grid_constan
                 }
                 tc::mbar_arrive_expect_tx(&c.xfull[b], (uint32_t)kcx * kC64);
                 for (int j = 0; j < kcx; ++j)
-                    tc::tma_load_2d(c.x0 + (b * kcx + j) * kC64, &tm_x, j * kChunk, t * B, &c.xfull[b]);
+                    tc::tma_load_2d(c.x0 + (b * kcx + j) * kC64, tmx, j * kChunk, t * B, &c.xfull[b]);
                 last = t;
             }
             // copies still in flight after an abort land before the CTA exits (each buffer's
@@ -542,7 +542,7 @@ constexpr int kClbIssuers = 4;                          // MMA issue warps
 constexpr int kClBwdThreads = (4 + kClbIssuers) * 32;  // and 4 epilogue warps
 
 template <int U>
-__global__ void __launch_bounds__(kClBwdThreads, 1) step_clb(ClArgs p)
+__device__ __forceinline__ void step_clb_body(const ClArgs &p)
 {
     static_assert(U == 16, "four 16-unit gate slices per CTA");
     constexpr int NI = kClbIssuers;
@@ -784,6 +784,39 @@ __global__ void __launch_bounds__(kClBwdThreads, 1) step_clb(ClArgs p)
     if (warp == E) tc::tmem_dealloc(tmem, 2 * kCols);
 }
 
+// One launch of the forward / backward cluster kernel for one handle.
+template <int U>
+__global__ void __launch_bounds__(kClFwdThreads, 1) step_cl(const __grid_constant__ CUtensorMap tm_x, ClArgs p)
+{
+    step_cl_body<U>(&tm_x, p);
+}
+template <int U>
+__global__ void __launch_bounds__(kClBwdThreads, 1) step_clb(ClArgs p)
+{
+    step_clb_body<U>(p);
+}
+
+// Several handles' recurrences in one launch: cluster m (CTAs m n_ct .. m n_ct + n_ct - 1)
+// runs member m's steps with its own arguments, workspace and step count. The members are
+// independent (each has its own inputs and op stream), so no barrier spans clusters; each
+// keeps its own per-step operand exchange.
+struct ClGroup {
+    CUtensorMap tm[kMaxGroup];  // forward: each member's x map
+    ClArgs p[kMaxGroup];
+};
+template <int U>
+__global__ void __launch_bounds__(kClFwdThreads, 1) step_cl_group(const __grid_constant__ ClGroup g)
+{
+    const int m = (int)blockIdx.x / g.p[0].n_ct;
+    step_cl_body<U>(&g.tm[m], g.p[m]);
+}
+template <int U>
+__global__ void __launch_bounds__(kClBwdThreads, 1) step_clb_group(const __grid_constant__ ClGroup g)
+{
+    const int m = (int)blockIdx.x / g.p[0].n_ct;
+    step_clb_body<U>(g.p[m]);
+}
+
 }  // namespace
 
 // One row tile (B <= 64), at most 16 column tiles of 16 units, the footprint within the
@@ -947,6 +980,60 @@ cudaError_t bf16_launch_bwd_cluster(stacklstm *s, const StepArgs &a)
     if (e) return e;
     s->launches += 1;
     return cudaGetLastError();
+}
+
+// Several handles' forward (or backward) recurrences as one launch of n clusters: the
+// dynamic shared memory is the largest member's, each cluster carves its own layout.
+template <bool kFwd>
+cudaError_t launch_cluster_group(stacklstm *const *hs, const StepArgs *as, const CUtensorMap *const *tms, int n,
+                                 cudaStream_t st)
+{
+    ClGroup g{};
+    size_t smem = 0;
+    const int n_ct = (kFwd ? hs[0]->fc : hs[0]->bc).n_ct;
+    for (int m = 0; m < n; ++m) {
+        stacklstm *s = hs[m];
+        const PersistPlan &pl = kFwd ? s->fc : s->bc;
+        if (!pl.on || pl.n_ct != n_ct) return cudaErrorInvalidValue;
+        ClArgs &p = g.p[m];
+        p.s = as[m];
+        p.s.gates_blk = kFwd ? s->bc.on : s->fc.on;
+        p.n_ct = n_ct;
+        p.gscr = (uint8_t *)(kFwd ? s->g_fcl : s->g_bcl);
+        if (kFwd) g.tm[m] = *tms[m];
+        smem = std::max<size_t>(smem, pl.smem);
+    }
+    const void *fn = kFwd ? (const void *)step_cl_group<kClU> : (const void *)step_clb_group<kClU>;
+    cudaError_t e = smem_at_least(fn, smem);
+    if (e) return e;
+    if (n_ct > 8 && (e = cudaFuncSetAttribute(fn, cudaFuncAttributeNonPortableClusterSizeAllowed, 1))) return e;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(n * n_ct);
+    cfg.blockDim = dim3(kFwd ? kClFwdThreads : kClBwdThreads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeClusterDimension;
+    at[0].val.clusterDim.x = n_ct;
+    at[0].val.clusterDim.y = 1;
+    at[0].val.clusterDim.z = 1;
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
+    void *argv[] = {(void *)&g};
+    if ((e = cudaLaunchKernelExC(&cfg, fn, argv))) return e;
+    hs[0]->launches += 1;
+    return cudaGetLastError();
+}
+
+cudaError_t bf16_launch_fwd_cluster_group(stacklstm *const *hs, const StepArgs *as, const CUtensorMap *const *tms, int n,
+                                          cudaStream_t st)
+{
+    return launch_cluster_group<true>(hs, as, tms, n, st);
+}
+
+cudaError_t bf16_launch_bwd_cluster_group(stacklstm *const *hs, const StepArgs *as, int n, cudaStream_t st)
+{
+    return launch_cluster_group<false>(hs, as, nullptr, n, st);
 }
 
 }  // namespace sl

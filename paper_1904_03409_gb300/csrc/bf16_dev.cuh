@@ -207,6 +207,9 @@ bool bf16_plan_bwd_cluster(stacklstm *s, PersistPlan *pl);
 size_t bf16_bwd_cluster_weight_bytes(int H);
 cudaError_t bf16_pack_bwd_cluster(stacklstm *s, const __nv_bfloat16 *W, __nv_bfloat16 *out);
 cudaError_t bf16_launch_bwd_cluster(stacklstm *s, const StepArgs &a);
+cudaError_t bf16_launch_fwd_cluster_group(stacklstm *const *hs, const StepArgs *as, const CUtensorMap *const *tms, int n,
+                                          cudaStream_t st);
+cudaError_t bf16_launch_bwd_cluster_group(stacklstm *const *hs, const StepArgs *as, int n, cudaStream_t st);
 size_t bf16_bwd_cluster_block_bytes(int T, int H);
 size_t bf16_fwd_cluster_block_bytes(int T, int H);
 cudaError_t bf16_launch_fwd_persist(stacklstm *s, const StepArgs &a, const CUtensorMap &tm_x, const CUtensorMap &tm_h,
@@ -214,6 +217,13 @@ cudaError_t bf16_launch_fwd_persist(stacklstm *s, const StepArgs &a, const CUten
                                     const CUtensorMap &tm_hc);
 cudaError_t bf16_launch_bwd_persist(stacklstm *s, const StepArgs &a, const CUtensorMap &tm_g, float *dx,
                                     bool *dx_done);
+
+// ---- small batches on CUDA cores (bf16_small.cu)
+bool bf16_plan_small(stacklstm *s, PersistPlan *pl);
+size_t bf16_small_weight_bytes(int I, int H, bool fwd);
+cudaError_t bf16_pack_small(stacklstm *s, const __nv_bfloat16 *W);
+cudaError_t bf16_launch_fwd_small(stacklstm *s, const StepArgs &a);
+cudaError_t bf16_launch_bwd_small(stacklstm *s, const StepArgs &a);
 
 // ---- weight / bias gradients (bf16_dw.cu)
 cudaError_t bf16_plan_dw(stacklstm *s);

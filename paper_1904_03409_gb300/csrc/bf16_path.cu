@@ -571,7 +571,7 @@ std::string bf16_describe(const stacklstm *s)
 {
     char buf[1024];
     const int rt = (int)ceil_div(s->B, kRows);
-    const PersistPlan &f = s->fc.on ? s->fc : s->pf, &b = s->bc.on ? s->bc : s->pb;
+    const PersistPlan &f = s->cc.on ? s->cc : s->fc.on ? s->fc : s->pf, &b = s->cc.on ? s->cc : s->bc.on ? s->bc : s->pb;
     snprintf(buf, sizeof buf,
              "bf16 tcgen05; row tiles %d; chunks fwd %d (x %d) bwd %d; "
              "forward %s U=%d [EP %d G %d ring %d slots %d cluster %d col tiles %d w_res %d smem %u threads %d "
@@ -580,8 +580,8 @@ std::string bf16_describe(const stacklstm *s)
              "per SM %d "
              "contraction parts %d dx CTAs %d ring %d]; "
              "step rings fwd %d bwd %d; dx N=%d x%d ring %d; dW %dx%d tiles of 128x%d x%d splits ring %d",
-             rt, s->kcf, s->kcx, s->kcb, s->fc.on ? "cluster" : f.on ? "persistent" : "per-step", s->uf, f.EP, f.G, f.S, f.slot, f.cl, f.n_ct,
-             f.w_res, f.smem, f.threads, f.per_sm, s->bc.on ? "cluster" : b.on ? "persistent" : "per-step", s->bc.on ? s->bc.U : s->ub, b.EP, b.G, b.S, b.slot, b.cl, b.n_ct,
+             rt, s->kcf, s->kcx, s->kcb, s->cc.on ? "cuda-core" : s->fc.on ? "cluster" : f.on ? "persistent" : "per-step", s->uf, f.EP, f.G, f.S, f.slot, f.cl, f.n_ct,
+             f.w_res, f.smem, f.threads, f.per_sm, s->cc.on ? "cuda-core" : s->bc.on ? "cluster" : b.on ? "persistent" : "per-step", s->bc.on ? s->bc.U : s->ub, b.EP, b.G, b.S, b.slot, b.cl, b.n_ct,
              b.w_res, b.smem, b.threads, b.per_sm, b.KS, b.n_dx, b.dx_S, s->sf, s->sb, s->nx, s->nxt, s->sx, s->dw_mt, s->dw_nt, s->dw_ntile, s->dw_split, s->sw);
     return buf;
 }
@@ -626,6 +626,11 @@ cudaError_t bf16_prepare(stacklstm *s)
             s->pf.on = 0;
         }
         bf16_plan_bwd_cluster(s, &s->bc);  // (the persistent plan stays as the fallback)
+        // small batches: both directions on CUDA cores instead
+        if (bf16_plan_small(s, &s->cc)) {
+            s->pf.on = s->pb.on = s->fc.on = s->bc.on = 0;
+            s->uf = s->ub = s->cc.U;
+        }
     }
     s->sf = pick_stages(s->kcf, 4 * s->uf, ceil_div(H, s->uf) * (size_t)rt, sms);
     s->sb = pick_stages(s->kcb, s->ub, ceil_div(H, s->ub) * (size_t)rt, sms);
@@ -652,6 +657,12 @@ cudaError_t bf16_prepare(stacklstm *s)
         s->allocs.push_back(p); s->w_bcl = p;
         if ((e = cudaMalloc(&p, bf16_bwd_cluster_block_bytes(T, H)))) return e;
         s->allocs.push_back(p); s->g_bcl = p;
+    }
+    if (s->cc.on) {
+        if ((e = cudaMalloc(&p, bf16_small_weight_bytes(I, H, true)))) return e;
+        s->allocs.push_back(p); s->w_ccf = p;
+        if ((e = cudaMalloc(&p, bf16_small_weight_bytes(I, H, false)))) return e;
+        s->allocs.push_back(p); s->w_ccb = p;
     }
     if ((e = cudaMalloc(&p, s->dw_part_elems * sizeof(float)))) return e;
     s->allocs.push_back(p); s->dw_part = (float *)p;
@@ -704,13 +715,18 @@ cudaError_t bf16_forward_setup(stacklstm *s, const __nv_bfloat16 *x, const __nv_
     if ((e = cudaMemcpyAsync(s->hist_c, c0, sizeof(float) * B * H, cudaMemcpyDeviceToDevice, s->stream))) return e;
     const int nctf = std::max((int)ceil_div(H, s->uf), s->pf.on ? s->pf.n_ct : 0);
     const int nctb = std::max((int)ceil_div(H, s->ub), s->pb.on ? s->pb.n_ct : 0);
-    pack_fwd<<<grid_for(s, (size_t)nctf * s->kcf * 4 * s->uf * kChunk), 256, 0, s->stream>>>(
-        W, I, H, s->uf, s->kcx, s->kcf, nctf, (__nv_bfloat16 *)s->w_fwd);
-    pack_rows<<<grid_for(s, (size_t)nctb * s->kcb * s->ub * kChunk), 256, 0, s->stream>>>(
-        W, H, I, H, s->ub, s->kcb, nctb, (__nv_bfloat16 *)s->w_bwd);
+    if (s->cc.on) {
+        if ((e = bf16_pack_small(s, W))) return e;
+    } else {
+        pack_fwd<<<grid_for(s, (size_t)nctf * s->kcf * 4 * s->uf * kChunk), 256, 0, s->stream>>>(
+            W, I, H, s->uf, s->kcx, s->kcf, nctf, (__nv_bfloat16 *)s->w_fwd);
+        pack_rows<<<grid_for(s, (size_t)nctb * s->kcb * s->ub * kChunk), 256, 0, s->stream>>>(
+            W, H, I, H, s->ub, s->kcb, nctb, (__nv_bfloat16 *)s->w_bwd);
+        s->launches += 2;
+    }
     pack_rows<<<grid_for(s, (size_t)s->nxt * s->kcb * s->nx * kChunk), 256, 0, s->stream>>>(
         W, H, 0, I, s->nx, s->kcb, s->nxt, (__nv_bfloat16 *)s->w_dx);
-    s->launches += 3;
+    s->launches += 1;
     if (s->bc.on && (e = bf16_pack_bwd_cluster(s, W, (__nv_bfloat16 *)s->w_bcl))) return e;
     return cudaGetLastError();
 }
@@ -729,6 +745,7 @@ cudaError_t bf16_forward_steps(stacklstm *s, const float *bias)
     const int T = s->Tr, B = s->B, H = s->H;
     const int nctf = std::max((int)ceil_div(H, s->uf), s->pf.on ? s->pf.n_ct : 0);
     cudaError_t e;
+    if (s->cc.on) return bf16_launch_fwd_small(s, step_args(s, bias, s->w_ccf, s->kcx, s->kcf, 0));
     if (s->fc.on)
         return bf16_launch_fwd_cluster(s, step_args(s, bias, s->w_fwd, s->kcx, s->kcf, 0), map(s, kMapX64));
     if (s->pf.on)
@@ -770,6 +787,7 @@ cudaError_t bf16_backward_steps(stacklstm *s, float *dx, bool *dx_done)
     const int T = s->Tr, B = s->B, H = s->H;
     cudaError_t e;
     const StepArgs a = step_args(s, nullptr, s->w_bwd, 0, s->kcb, s->sb);
+    if (s->cc.on) return bf16_launch_bwd_small(s, step_args(s, nullptr, s->w_ccb, 0, s->kcb, 0));
     if (s->bc.on) return bf16_launch_bwd_cluster(s, step_args(s, nullptr, s->w_bcl, 0, s->kcb, 0));
     // one row tile of at most 64 instances: 64-row boxes (the rest of each stage is never
     // loaded and only feeds accumulator rows that are not stored)
@@ -789,6 +807,36 @@ cudaError_t bf16_backward_steps(stacklstm *s, float *dx, bool *dx_done)
         s->launches += 1;
     }
     return cudaGetLastError();
+}
+
+bool bf16_can_group(stacklstm *const *hs, int n, bool fwd)
+{
+    for (int m = 0; m < n; ++m) {
+        const stacklstm *s = hs[m];
+        const PersistPlan &pl = fwd ? s->fc : s->bc;
+        if (s->dt != SL_BF16 || s->cc.on || !pl.on || pl.n_ct != (fwd ? hs[0]->fc : hs[0]->bc).n_ct ||
+            s->device != hs[0]->device)
+            return false;
+    }
+    return true;
+}
+
+cudaError_t bf16_forward_steps_group(stacklstm *const *hs, int n, const float *const *bias, cudaStream_t st)
+{
+    StepArgs as[kMaxGroup];
+    const CUtensorMap *tms[kMaxGroup];
+    for (int m = 0; m < n; ++m) {
+        as[m] = step_args(hs[m], bias[m], hs[m]->w_fwd, hs[m]->kcx, hs[m]->kcf, 0);
+        tms[m] = &map(hs[m], kMapX64);
+    }
+    return bf16_launch_fwd_cluster_group(hs, as, tms, n, st);
+}
+
+cudaError_t bf16_backward_steps_group(stacklstm *const *hs, int n, cudaStream_t st)
+{
+    StepArgs as[kMaxGroup];
+    for (int m = 0; m < n; ++m) as[m] = step_args(hs[m], nullptr, hs[m]->w_bcl, 0, hs[m]->kcb, 0);
+    return bf16_launch_bwd_cluster_group(hs, as, n, st);
 }
 
 cudaError_t bf16_dx(stacklstm *s, float *dx)

@@ -11,6 +11,9 @@
 
 #include "../../include/stacklstm.h"
 
+// Most handles one grouped call (stacklstm_forward_group / _backward_group) takes.
+constexpr int kMaxGroup = 4;
+
 // A planned persistent step kernel: one cooperative launch runs all T steps.
 struct PersistPlan {
     int on = 0;         // 1: persistent; 0: one launch per step
@@ -40,6 +43,7 @@ struct stacklstm {
     // the caller's stream before the forward steps, `cleared` the end of the clearing
     cudaStream_t side = nullptr;
     cudaEvent_t side_go = nullptr, cleared = nullptr;
+    cudaEvent_t join = nullptr;  // grouped calls: marks this handle's stream for the others
     int clear_queued = 0;
     int async = 0;
     int fwd_done = 0;
@@ -98,6 +102,8 @@ struct stacklstm {
     PersistPlan fc;                // forward as one thread-block cluster (one row tile; bf16_cluster.cu)
     void *g_fcl = nullptr;         // its h slice blocks [T][column tiles][2 KB]
     PersistPlan bc;                // backward as one thread-block cluster (one row tile; bf16_cluster.cu)
+    PersistPlan cc;                // small batches: both directions on CUDA cores (bf16_small.cu)
+    void *w_ccf = nullptr, *w_ccb = nullptr;  // their weight slices
     void *w_bcl = nullptr;         // its weight chunks
     void *g_bcl = nullptr;         // its swizzled dG blocks [T][column tiles][8 KB]
     int32_t *rowcnt = nullptr;     // [2][row tiles][cnt_stride] completed steps per row tile
@@ -159,6 +165,11 @@ cudaError_t bf16_forward_setup(stacklstm *s, const __nv_bfloat16 *x, const __nv_
 cudaError_t bf16_forward_steps(stacklstm *s, const float *bias);
 cudaError_t bf16_backward_setup(stacklstm *s);
 cudaError_t bf16_backward_steps(stacklstm *s, float *dx, bool *dx_done);
+// Grouped calls: true when the n handles' step kernels can run as one launch (every one
+// on the one-row-tile cluster kernels of the same cluster size); that launch, on `st`.
+bool bf16_can_group(stacklstm *const *hs, int n, bool fwd);
+cudaError_t bf16_forward_steps_group(stacklstm *const *hs, int n, const float *const *bias, cudaStream_t st);
+cudaError_t bf16_backward_steps_group(stacklstm *const *hs, int n, cudaStream_t st);
 cudaError_t bf16_dx(stacklstm *s, float *dx);
 cudaError_t bf16_dw(stacklstm *s, float *dW, float *dbias);
 // push-only mode: x of each virtual step into s->x_push (bf16 rows)

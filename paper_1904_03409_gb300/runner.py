@@ -108,14 +108,35 @@ def group_forward_backward(hds: dict, ins: dict, outs: dict):
         cur.wait_stream(hds[k][1])
 
 
+def group_forward_backward_one_call(hds: dict, ins: dict, outs: dict):
+    """The same as ``group_forward_backward`` through the grouped calls: one forward call
+    and one backward call for the three StackLSTMs, whose step kernels then run as one
+    launch each way."""
+    import torch
+    cur = torch.cuda.current_stream()
+    hs = [hds[k][0] for k in GROUP_MEMBERS]
+    for k in GROUP_MEMBERS:
+        hds[k][1].wait_stream(cur)
+    fwd = [dict(x=ins[k]["x"], ops=ins[k]["ops"], h0=ins[k]["h0"], c0=ins[k]["c0"], W=ins[k]["W"], bias=ins[k]["bias"],
+                h_stack=outs[k].get("h_stack"), c_stack=outs[k].get("c_stack"), p_final=outs[k]["p_final"],
+                p_traj=outs[k].get("p_traj"), src=outs[k].get("src"), y=outs[k].get("y")) for k in GROUP_MEMBERS]
+    bwd = [dict(d_top_h=ins[k]["d_top_h"], dy=ins[k].get("dy"), dx=outs[k].get("dx"), dh0=outs[k].get("dh0"),
+                dc0=outs[k].get("dc0"), dW=outs[k].get("dW"), dbias=outs[k].get("dbias")) for k in GROUP_MEMBERS]
+    bd.stacklstm_forward_group(hs, fwd)
+    bd.stacklstm_backward_group(hs, bwd)
+    for k in GROUP_MEMBERS:
+        cur.wait_stream(hds[k][1])
+
+
 def group_status(hds: dict):
     for hd, _ in hds.values():
         bd.stacklstm_status(hd)
 
 
-def run_group(group: dict, device: int = 0) -> dict:
+def run_group(group: dict, device: int = 0, one_call: bool = False) -> dict:
     """Forward + backward of the three StackLSTMs of a parser workload group at the same
-    time (one stream each), into NaN-filled outputs; numpy results per member."""
+    time (one stream each; with ``one_call`` through the grouped calls), into NaN-filled
+    outputs; numpy results per member."""
     import torch
     hds = create_group(group, device)
     try:
@@ -125,7 +146,7 @@ def run_group(group: dict, device: int = 0) -> dict:
             for v in o.values():
                 if v.is_floating_point():
                     v.fill_(float("nan"))
-        group_forward_backward(hds, ins, outs)
+        (group_forward_backward_one_call if one_call else group_forward_backward)(hds, ins, outs)
         torch.cuda.synchronize(device)
         group_status(hds)
         return {k: to_numpy(outs[k]) for k in GROUP_MEMBERS}

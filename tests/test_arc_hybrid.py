@@ -162,6 +162,79 @@ def test_arc_hybrid_three_stacklstms_at_once_match_oracle():
     torch.cuda.empty_cache()
 
 
+@pytest.mark.gpu
+def test_grouped_calls_run_one_step_launch_and_match_oracle():
+    """The three StackLSTMs through stacklstm_forward_group / stacklstm_backward_group: their
+    step kernels run as one launch each way (counted in the first handle's forward and
+    backward phases, none in the others'), and the results equal the oracle's and, bit for
+    bit, those of separate calls."""
+    import torch
+    from paper_1904_03409_gb300 import binding as bd
+    from paper_1904_03409_gb300 import runner
+    g = wl.make_arc_hybrid(**wl.GROUPS["arc_hybrid64"])
+    got = runner.run_group(g, one_call=True)
+    sep = runner.run_group(g)
+    for k in runner.GROUP_MEMBERS:
+        w = g[k]
+        compare(got[k], oracle.run(w.x, w.ops, w.h0, w.c0, w.W, w.bias, d_top_h=w.d_top_h), "bf16")
+        for name in ("dx", "dW", "dbias", "dh0", "dc0", "y", "h_stack", "c_stack", "p_traj", "src"):
+            assert np.array_equal(got[k][name], sep[k][name], equal_nan=True), (k, name)
+    hds = runner.create_group(g)
+    try:
+        ins = {k: runner.upload(g[k]) for k in runner.GROUP_MEMBERS}
+        outs = {k: runner.alloc_outputs(g[k], forward_outputs=False) for k in runner.GROUP_MEMBERS}
+        for hd, _ in hds.values():
+            bd.stacklstm_set_timing(hd, True)
+        runner.group_forward_backward_one_call(hds, ins, outs)
+        torch.cuda.synchronize()
+        steps = [(bd.stacklstm_get_timing(hds[k][0])["forward"][1], bd.stacklstm_get_timing(hds[k][0])["backward"][1])
+                 for k in runner.GROUP_MEMBERS]
+        assert steps == [(1, 1), (0, 0), (0, 0)], steps
+    finally:
+        for hd, _ in hds.values():
+            hd.destroy()
+    torch.cuda.empty_cache()
+
+
+@pytest.mark.gpu
+def test_grouped_calls_fall_back_when_the_members_differ():
+    """Handles that cannot share one launch (different hidden widths, a persistent plan)
+    still give the results of separate calls."""
+    import torch
+    from paper_1904_03409_gb300 import binding as bd
+    from paper_1904_03409_gb300 import runner
+    ws = [wl.make_workload("m%d" % i, T=T, B=B, I=I, H=H, dtype="bf16", seed=60 + i, ops_kind="random_walk",
+                           probs=(0.5, 0.3, 0.2), dy_scale=0.5)
+          for i, (T, B, I, H) in enumerate([(12, 40, 24, 48), (9, 40, 16, 32), (10, 130, 16, 48)])]
+    hds = [bd.stacklstm_create(w.T, w.B, w.I, w.H, bd.SL_BF16, 0) for w in ws]
+    try:
+        ins = [runner.upload(w) for w in ws]
+        outs = [runner.alloc_outputs(w) for w in ws]
+        for o in outs:
+            for v in o.values():
+                if v.is_floating_point():
+                    v.fill_(float("nan"))
+        fwd = [dict(x=i["x"], ops=i["ops"], h0=i["h0"], c0=i["c0"], W=i["W"], bias=i["bias"], h_stack=o["h_stack"],
+                    c_stack=o["c_stack"], p_final=o["p_final"], p_traj=o["p_traj"], src=o["src"], y=o["y"])
+               for i, o in zip(ins, outs)]
+        bwd = [dict(d_top_h=i["d_top_h"], dy=i["dy"], dx=o["dx"], dh0=o["dh0"], dc0=o["dc0"], dW=o["dW"],
+                    dbias=o["dbias"]) for i, o in zip(ins, outs)]
+        bd.stacklstm_forward_group(hds, fwd)
+        bd.stacklstm_backward_group(hds, bwd)
+        torch.cuda.synchronize()
+        for w, o in zip(ws, outs):
+            got = runner.to_numpy(o)
+            alone = runner.run(w)
+            for name in ("dx", "dW", "dbias", "dh0", "dc0", "y", "h_stack", "p_traj"):
+                assert np.array_equal(got[name], alone[name], equal_nan=True), (w.name, name)
+        with pytest.raises(bd.StackLSTMError) as e:
+            bd.stacklstm_forward_group([hds[0], hds[0]], fwd[:1] * 2)
+        assert e.value.status == 1
+    finally:
+        for hd in hds:
+            hd.destroy()
+
+
 def parser_oracle(g, got):
     """The oracle of one parser step, stage by stage on the inputs the GPU stage saw:
     each StackLSTM's forward; the head on the GPU's StackLSTM outputs; each StackLSTM's
