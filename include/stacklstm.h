@@ -308,13 +308,16 @@ sl_status stacklstm_pointers_noalloc(int T, int B, const int8_t *ops, int32_t *p
  * z = Wz p + q over the A transitions, and the row loss logsumexp(z) - z[gold[k, b]].
  * Transitions k >= L[b] are padding: no loss, no gradient. The paper fixes only the
  * state width; the ReLU layer and the softmax follow the parser architecture its
- * experiments reuse. bf16 inputs, fp32 arithmetic (CUDA cores); deterministic.
+ * experiments reuse. bf16 inputs; the contractions U Wp^T, dP Wp and dP^T U over all rows
+ * on the tensor cores (bf16 operands, dP rounded to bf16, fp32 accumulation), the rest in
+ * fp32; deterministic.
  *
  * stacklstm_head_create -- a head for T transitions (the stack and action StackLSTMs'
  *   step count), a buffer StackLSTM of Tb steps, B instances, hidden width H (a multiple
- *   of 8), state width P (<= 256) and A transitions (2..8). Owns its workspace: about
- *   T B (6H + 8P + 4A) bytes for the gathered tops, states and gradients, plus up to
- *   16 x P x 3H floats of weight-gradient partial sums. Calls are ordered on `stream`;
+ *   of 8), state width P (a multiple of 8, <= 256) and A transitions (2..8). Owns its
+ *   workspace: about T B (24 H + 8 P + 16) bytes for the gathered tops, the states and the
+ *   gradients, plus up to 32 x 3H x P floats of weight-gradient partial sums. Calls are
+ *   ordered on `stream`;
  *   SL_ERR_ARG (bad size or device), SL_ERR_UNSUPPORTED or SL_ERR_OOM on failure,
  *   leaving *out NULL.
  */

@@ -362,24 +362,29 @@ __global__ void __launch_bounds__(kThreads, 1) dx_tc(const __grid_constant__ CUt
     const int ct = blockIdx.x;
     const size_t row0 = (size_t)blockIdx.y * kRows;
     const uint32_t tmem = prologue(c, a.S, kCols);
-    const uint8_t *bpack = a.wpack + (size_t)ct * a.KC * c.b_bytes;
+    // split contraction (grid z > 1): part z takes chunks [kc0, kc1) and writes its partial
+    // product to slab z of the output
+    const int kz = blockIdx.z, nz = gridDim.z;
+    const int kc0 = (int)((long long)a.KC * kz / nz), kc1 = (int)((long long)a.KC * (kz + 1) / nz);
+    float *out = a.dx + (size_t)kz * a.R * a.I;
+    const uint8_t *bpack = a.wpack + ((size_t)ct * a.KC + kc0) * c.b_bytes;
     auto tma = [&](int it, int s, uint64_t *bar) {
         tc::mbar_arrive_expect_tx(bar, kAStage + c.b_bytes);
-        tc::tma_load_2d(c.a0 + s * kAStage, &tm_g, it * kChunk, (int)row0, bar);
+        tc::tma_load_2d(c.a0 + s * kAStage, &tm_g, (kc0 + it) * kChunk, (int)row0, bar);
         tc::bulk_g2s(c.b0 + s * c.b_bytes, bpack + (size_t)it * c.b_bytes, c.b_bytes, bar);
     };
     auto no_gather = [](int, int) {};
     auto issue = [&](int s, int j) { issue_kmajor<N>(tmem, c.a0 + s * kAStage, c.b0 + s * c.b_bytes, j); };
-    mainloop<false>(c, a.S, a.KC, -1, a.limit, a.err, tma, no_gather, issue);
+    mainloop<false>(c, a.S, kc1 - kc0, -1, a.limit, a.err, tma, no_gather, issue);
     if (!*c.abort) {
         const size_t row = row0 + tid;
         // the dx row this accumulator row belongs to: the same row, or (push-only mode)
         // the real step of this virtual row's push; rows past an instance's pushes have none
-        bool out = row < a.R;
+        bool ok_row = row < a.R;
         size_t orow = row;
-        if (out && a.xidx) {
+        if (ok_row && a.xidx) {
             const int t = a.xidx[row];
-            out = t >= 0;
+            ok_row = t >= 0;
             orow = (size_t)t * a.B + row % a.B;
         }
         const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
@@ -388,7 +393,7 @@ __global__ void __launch_bounds__(kThreads, 1) dx_tc(const __grid_constant__ CUt
             float v[8];
             tc::tmem_ld8(trow + cu * 8, v);
             const int col = ct * N + cu * 8;
-            if (out && col < a.I) st8f(a.dx + orow * a.I + col, v);
+            if (ok_row && col < a.I) st8f(out + orow * a.I + col, v);
         }
     }
     finish(c, tmem, kCols);
@@ -459,6 +464,27 @@ __global__ void gather_push_x(size_t rows, int B, int I8, const int32_t *__restr
     }
 }
 
+// Generic K-major operand tiles [n tiles][KC][NB rows][64], 128-byte swizzled rows: row n
+// of the operand is src row n (trans = false: src[n][k]) or src column n (trans = true:
+// src[k][n]), zero past N and K.
+__global__ void pack_kmajor(const __nv_bfloat16 *__restrict__ src, size_t ld, int trans, int N, int K, int NB, int KC,
+                            int n_tiles, __nv_bfloat16 *__restrict__ out)
+{
+    const size_t n_el = (size_t)n_tiles * KC * NB * kChunk;
+    for (size_t e = blockIdx.x * (size_t)blockDim.x + threadIdx.x; e < n_el; e += (size_t)gridDim.x * blockDim.x) {
+        const int col = (int)(e % kChunk);
+        const size_t rowi = e / kChunk;
+        const int row = (int)(rowi % NB);
+        const size_t tile = rowi / NB;
+        const int kc = (int)(tile % KC), nt = (int)(tile / KC);
+        const int n = nt * NB + row, k = kc * kChunk + col;
+        __nv_bfloat16 v = __float2bfloat16(0.0f);
+        if (n < N && k < K) v = trans ? src[(size_t)k * ld + n] : src[(size_t)n * ld + k];
+        const size_t byte = tile * NB * 128 + sw128(row, col >> 3) + (col & 7) * 2;
+        out[byte / 2] = v;
+    }
+}
+
 // ------------------------------------------------------------------ host side
 PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
 
@@ -474,12 +500,13 @@ cudaError_t get_encoder()
     return cudaSuccess;
 }
 
-// Row-major bf16 matrix [rows][cols] read in boxes of 64 columns x box_rows rows with
-// 128-byte swizzling; out-of-range elements read as zero.
-cudaError_t make_map(void *slot, const void *base, uint64_t rows, uint64_t cols, uint32_t box_rows)
+// Row-major bf16 matrix [rows][cols] (rows `ld` elements apart, ld = cols unless given)
+// read in boxes of 64 columns x box_rows rows with 128-byte swizzling; out-of-range
+// elements read as zero.
+cudaError_t make_map(void *slot, const void *base, uint64_t rows, uint64_t cols, uint32_t box_rows, uint64_t ld = 0)
 {
     cuuint64_t dims[2] = {cols, rows};
-    cuuint64_t strides[1] = {cols * 2};
+    cuuint64_t strides[1] = {(ld ? ld : cols) * 2};
     cuuint32_t box[2] = {(cuuint32_t)kChunk, box_rows};
     cuuint32_t es[2] = {1, 1};
     CUresult r = g_encode((CUtensorMap *)slot, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(base), dims,
@@ -867,6 +894,55 @@ cudaError_t bf16_dw(stacklstm *s, float *dW, float *dbias)
 {
     if (!dW && !dbias) return cudaSuccess;
     return bf16_launch_dw(s, map(s, kMapX64), map(s, kMapH64), map(s, kMapG64), dW, dbias);
+}
+
+// ------------------------------------------------------------ generic contraction
+// D = A B^T on the tensor cores, for the parser head: A [R][K] bf16 row-major (rows lda
+// elements apart, 16-byte aligned) read by TMA, B given as K-major tiles by
+// bf16_pack_kmajor, D [splits][R][N] fp32 (split contraction: slab z holds the product of
+// the z-th part of the K chunks; splits = 1 gives D itself).
+size_t bf16_kmajor_bytes(int N, int K)
+{
+    const int nx = pick_dx_n(N);
+    return (size_t)ceil_div(N, nx) * ceil_div(K, kChunk) * nx * 128;
+}
+
+cudaError_t bf16_pack_kmajor(const __nv_bfloat16 *src, size_t ld, bool trans, int N, int K, void *out,
+                             cudaStream_t st, int num_sms)
+{
+    const int nx = pick_dx_n(N), KC = (int)ceil_div(K, kChunk), nt = (int)ceil_div(N, nx);
+    const size_t n = (size_t)nt * KC * nx * kChunk;
+    pack_kmajor<<<(unsigned)std::max<size_t>(1, std::min<size_t>(ceil_div(n, 256), (size_t)num_sms * 16)), 256, 0,
+                  st>>>(src, ld, trans ? 1 : 0, N, K, nx, KC, nt, (__nv_bfloat16 *)out);
+    return cudaGetLastError();
+}
+
+cudaError_t bf16_gemm(const __nv_bfloat16 *A, size_t lda, int R, int K, const void *bpack, int N, float *D, int splits,
+                      cudaStream_t st, int num_sms, long long limit, int32_t *err)
+{
+    cudaError_t e;
+    if ((e = get_encoder())) return e;
+    alignas(64) unsigned char tm[128];
+    if ((e = make_map(tm, A, (uint64_t)R, (uint64_t)K, kRows, lda))) return e;
+    const int nx = pick_dx_n(N), KC = (int)ceil_div(K, kChunk), nt = (int)ceil_div(N, nx);
+    splits = std::max(1, std::min(splits, KC));
+    const size_t ctas = (size_t)nt * ceil_div(R, kRows) * splits;
+    DxArgs d;
+    d.R = (size_t)R; d.I = N; d.KC = KC;
+    d.S = pick_stages(KC, nx, ctas, num_sms);
+    d.wpack = (const uint8_t *)bpack; d.dx = D; d.limit = limit; d.err = err;
+    d.xidx = nullptr;
+    d.B = 1;
+    const dim3 g(nt, ceil_div(R, kRows), splits);
+    const size_t smem = smem_bytes(d.S, nx);
+    const CUtensorMap &tmg = *(const CUtensorMap *)tm;
+    switch (nx) {
+    case 32: e = allow_smem(dx_tc<32>); if (!e) e = launch(dx_tc<32>, g, smem, st, false, tmg, d); break;
+    case 64: e = allow_smem(dx_tc<64>); if (!e) e = launch(dx_tc<64>, g, smem, st, false, tmg, d); break;
+    case 128: e = allow_smem(dx_tc<128>); if (!e) e = launch(dx_tc<128>, g, smem, st, false, tmg, d); break;
+    default: e = allow_smem(dx_tc<256>); if (!e) e = launch(dx_tc<256>, g, smem, st, false, tmg, d); break;
+    }
+    return e ? e : cudaGetLastError();
 }
 
 }  // namespace sl

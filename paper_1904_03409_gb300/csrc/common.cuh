@@ -178,6 +178,15 @@ size_t bf16_workspace_bytes(int T, int B, int I, int H, int num_sms);
 const char *bf16_unsupported(int T, int B, int I, int H);
 std::string bf16_describe(const stacklstm *s);
 
+// generic tensor-core contraction (bf16_path.cu): D [splits][R][N] fp32 = A [R][K] B^T,
+// A bf16 row-major (rows lda apart), B packed by bf16_pack_kmajor from src (rows n of
+// length K, or with trans the columns of a [K][N] src)
+size_t bf16_kmajor_bytes(int N, int K);
+cudaError_t bf16_pack_kmajor(const __nv_bfloat16 *src, size_t ld, bool trans, int N, int K, void *out,
+                             cudaStream_t st, int num_sms);
+cudaError_t bf16_gemm(const __nv_bfloat16 *A, size_t lda, int R, int K, const void *bpack, int N, float *D, int splits,
+                      cudaStream_t st, int num_sms, long long limit, int32_t *err);
+
 inline unsigned ceil_div(size_t a, size_t b) { return (unsigned)((a + b - 1) / b); }
 
 }  // namespace sl

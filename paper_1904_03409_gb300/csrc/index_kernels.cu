@@ -98,6 +98,27 @@ __global__ void seed_grads_kernel(int T, int B, int H, const int32_t *__restrict
     }
 }
 
+// The same seeding with per-step gradients dy, for one instance and 32 units per block:
+// the T + 1 rows' sums of those units accumulate in shared memory in the same order as
+// above (final top, then t = T-1..0), then every row is written once. The gradient
+// history is zero before the seeding, so writing the sums equals adding them.
+__global__ void __launch_bounds__(32) seed_grads_dy_kernel(int T, int B, int H, const int32_t *__restrict__ top,
+                                                            const float *__restrict__ d_top_h,
+                                                            const float *__restrict__ dy, float *__restrict__ dhist_h)
+{
+    extern __shared__ float acc[];  // [T + 1][32]
+    const int b = blockIdx.x, lane = threadIdx.x, j = blockIdx.y * 32 + lane;
+    for (int s = 0; s <= T; ++s) acc[s * 32 + lane] = 0.0f;
+    __syncwarp();
+    if (j < H) {
+        const size_t n = (size_t)B * H, e = (size_t)b * H + j;
+        if (d_top_h) acc[top[(size_t)T * B + b] * 32 + lane] += d_top_h[e];
+#pragma unroll 8
+        for (int t = T - 1; t >= 0; --t) acc[top[(size_t)(t + 1) * B + b] * 32 + lane] += dy[(size_t)t * n + e];
+        for (int s = 0; s <= T; ++s) dhist_h[((size_t)s * B + b) * H + j] = acc[s * 32 + lane];
+    }
+}
+
 // Push-only mode: the virtual timeline of each instance. By Observation 2 of Sec. 3 only
 // a push step's write is ever read (a pop or hold writes slot p + 1 above the new top,
 // and the next push overwrites it before the pointer gets there), so instance b's
@@ -256,11 +277,20 @@ cudaError_t launch_gather_rows(stacklstm *s, const int32_t *idx, int rows, size_
 cudaError_t launch_seed_grads(stacklstm *s, const float *d_top_h, const float *dy)
 {
     if (!d_top_h && !dy) return cudaSuccess;
+    const int32_t *top = s->push_only ? s->vy : s->top;
+    const size_t acc_bytes = (size_t)(s->T + 1) * 32 * sizeof(float);
+    if (dy && acc_bytes <= 200 * 1024) {
+        cudaError_t e = acc_bytes > 48 * 1024 ? smem_at_least((const void *)seed_grads_dy_kernel, acc_bytes) : cudaSuccess;
+        if (e) return e;
+        seed_grads_dy_kernel<<<dim3(s->B, ceil_div(s->H, 32)), 32, acc_bytes, s->stream>>>(s->T, s->B, s->H, top,
+                                                                                           d_top_h, dy, s->dhist_h);
+        s->launches += 1;
+        return cudaGetLastError();
+    }
     const size_t n = (size_t)s->B * s->H;
     const unsigned grid = (unsigned)std::min<size_t>(ceil_div(n, 256), (size_t)s->num_sms * 16);
     // the (virtual, in push-only mode) history index of the top at each real time
-    seed_grads_kernel<<<grid, 256, 0, s->stream>>>(s->T, s->B, s->H, s->push_only ? s->vy : s->top, d_top_h, dy,
-                                                   s->dhist_h);
+    seed_grads_kernel<<<grid, 256, 0, s->stream>>>(s->T, s->B, s->H, top, d_top_h, dy, s->dhist_h);
     s->launches += 1;
     return cudaGetLastError();
 }

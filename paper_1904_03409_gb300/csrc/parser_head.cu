@@ -9,33 +9,44 @@
 // (the 200-wide parser state of Sec. 4.1), z = Wz p + q, and the row's loss is
 // logsumexp(z) - z[gold]. Rows k >= L_b are padding and contribute nothing.
 //
-// Kernels (CUDA cores, fp32 accumulation; bf16 inputs):
-//   head_rows      R rows (transitions) per CTA: gathers u = [s; bu; a] into shared
-//                  memory, pre = u Wp^T + dp, p = ReLU(pre), z, the softmax cross-entropy
-//                  and dz, dP = (dz Wz) * (pre > 0), du = dP Wp, and stores du into the
-//                  gradients of the StackLSTM outputs (each output row has one source row,
-//                  so plain stores after a zero fill); p, dP, dz and u go to the workspace.
-//   head_dwp_part  dWp partial sums over one of S row ranges; head_small_part the same for
-//                  dWz, ddp and dq; head_reduce sums the partials in range order, so every
-//                  gradient is bitwise reproducible.
+// The three contractions over all NR = T B rows run on the tensor cores (tcgen05, bf16
+// operands, fp32 accumulation; the generic contraction of bf16_path.cu):
+//   pre = U Wp^T         U [NR][3H] the gathered tops (zero rows for padding)
+//   du  = dP Wp          dP [NR][P] in bf16, scattered into the gradients of the rows read
+//   dWp^T = U^T dP       a split contraction over the rows, the parts summed in order
+// and the row-wise work on CUDA cores:
+//   head_gather    U and each row's (transition, instance, buffer row, label)
+//   head_epi       32 rows per CTA: p = ReLU(pre + dp), z, the softmax cross-entropy and
+//                  dz, dP = (dz Wz) * (pre > 0); partial sums of dWz, ddp and dq over the
+//                  CTA's rows in row order
+//   head_scatter   du rows into dy_stack / dy_buffer / dy_action (each output row has one
+//                  source row, so plain stores after a zero fill)
+//   head_reduce    partial sums in a fixed order: every gradient is bitwise reproducible.
 #include <stdio.h>
 
+#include <algorithm>
+#include <new>
 #include <string>
 
 #include "common.cuh"
 
 struct stacklstm_head {
-    int T, Tb, B, H, P, A, R;
-    int device;
+    int T, Tb, B, H, P, A;
+    int device, num_sms;
     cudaStream_t stream;
-    int S;                    // row ranges of the weight-gradient partial sums
-    __nv_bfloat16 *wpt = nullptr;  // [3H][P] Wp transposed
-    __nv_bfloat16 *u = nullptr;    // [T B][3H] gathered tops
-    float *p = nullptr, *dP = nullptr, *dz = nullptr;  // [T B][P], [T B][P], [T B][A]
-    float *dh0 = nullptr;     // [2][B][H] gradients of the k = 0 reads (stack, action)
-    float *part = nullptr;    // [S][P][3H] dWp partials, then [S2][A P + P + A]
+    int S3;                         // parts of the dWp contraction over the rows
+    int NR8;                        // NR rounded up to 8 (row length of U^T)
+    __nv_bfloat16 *u = nullptr;     // [NR][3H] gathered tops
+    __nv_bfloat16 *ut = nullptr;    // [3H][NR8] the same, transposed
+    __nv_bfloat16 *dpb = nullptr;   // [NR][P] dP in bf16
+    int4 *meta = nullptr;           // [NR] (k or -1, b, buffer row, label) of each row
+    float *pre = nullptr;           // [NR][P] U Wp^T
+    float *du = nullptr;            // [NR][3H] dP Wp
+    float *part3 = nullptr;         // [S3][3H][P] dWp^T parts
+    float *part = nullptr;          // [row blocks][A P + P + A] dWz, ddp, dq partials
+    void *wp_k = nullptr, *wpt_k = nullptr, *dpt_k = nullptr;  // packed operands: Wp, Wp^T, dP^T
+    float *dh0 = nullptr;           // [2][B][H] gradients of the k = 0 reads (stack, action)
     int32_t *err = nullptr;
-    size_t smem = 0;
     std::string last_error;
 };
 
@@ -43,266 +54,167 @@ namespace sl {
 namespace {
 
 constexpr int kHeadThreads = 256;
-constexpr int kSmallChunks = 64;  // row ranges of the dWz / ddp / dq partials
-constexpr int kDwpJ = 8;          // Wp rows per dWp CTA
+constexpr int kEpiRows = 32;  // rows per head_epi CTA
 
-__host__ __device__ constexpr size_t head_smem_bytes(int R, int H, int P, int A)
+// One warp per row: the row's transition, instance, buffer row and label (k = -1 for
+// padding or a bad length or label, which is recorded), and its U row [s; bu; a].
+__global__ void __launch_bounds__(kHeadThreads)
+head_gather(int T, int Tb, int B, int H, int A, const __nv_bfloat16 *__restrict__ y_stack,
+            const __nv_bfloat16 *__restrict__ h0_stack, const __nv_bfloat16 *__restrict__ y_buffer,
+            const __nv_bfloat16 *__restrict__ y_action, const __nv_bfloat16 *__restrict__ h0_action,
+            const int32_t *__restrict__ n, const int32_t *__restrict__ L, const int8_t *__restrict__ gold,
+            __nv_bfloat16 *__restrict__ u, int4 *__restrict__ meta, int32_t *err)
 {
-    // u [3H][R] bf16, p [R][P], dP [P][R], Wz [A][P], z and dz [R][A], row info [R]
-    return (size_t)3 * H * R * 2 + (size_t)R * P * 4 * 2 + (size_t)A * P * 4 + (size_t)R * A * 4 * 2 + (size_t)R * 16;
-}
-
-struct HeadArgs {
-    int T, Tb, B, H, P, A;
-    const __nv_bfloat16 *y_stack, *h0_stack, *y_buffer, *y_action, *h0_action;
-    const int32_t *n, *L;
-    const int8_t *gold;
-    const __nv_bfloat16 *Wp, *wpt;
-    const float *dp, *Wz, *q;
-    float *loss_rows, *dy_stack, *dy_buffer, *dy_action, *dh0;
-    __nv_bfloat16 *u;
-    float *p, *dP, *dz;
-    int32_t *err;
-};
-
-__global__ void head_pack_wpt(const __nv_bfloat16 *__restrict__ Wp, int P, int K, __nv_bfloat16 *__restrict__ wpt)
-{
-    const size_t n = (size_t)P * K;
-    for (size_t e = blockIdx.x * (size_t)blockDim.x + threadIdx.x; e < n; e += (size_t)gridDim.x * blockDim.x) {
-        const int j = (int)(e / K), c = (int)(e % K);
-        wpt[(size_t)c * P + j] = Wp[e];
-    }
-}
-
-template <int R>
-__global__ void __launch_bounds__(kHeadThreads) head_rows(HeadArgs a)
-{
-    extern __shared__ __align__(16) uint8_t sm[];
-    const int H = a.H, P = a.P, A = a.A, B = a.B, K = 3 * H;
-    __nv_bfloat16 *u_s = (__nv_bfloat16 *)sm;                 // [K][R]
-    float *p_s = (float *)(sm + (size_t)K * R * 2);           // [R][P]
-    float *dP_s = p_s + R * P;                                // [P][R]
-    float *wz_s = dP_s + P * R;                               // [A][P]
-    float *z_s = wz_s + A * P;                                // [R][A]
-    float *dz_s = z_s + R * A;                                // [R][A]
-    int *row_k = (int *)(dz_s + R * A);                       // [R] transition, -1 if padding
-    int *row_b = row_k + R;
-    int *row_tb = row_b + R;                                  // buffer output row read
-    int *row_g = row_tb + R;                                  // gold transition
-    const int tid = threadIdx.x;
-    const int row0 = blockIdx.x * R;
-    const int NR = a.T * B;
-
-    for (int i = tid; i < A * P; i += blockDim.x) wz_s[i] = a.Wz[i];
-    if (tid < R) {
-        const int row = row0 + tid;
-        int k = -1, b = 0, tb = 0, g = 0;
-        if (row < NR) {
-            k = row / B;
-            b = row % B;
-            const int nb = a.n[b], Lb = a.L[b];
-            if (k < Lb) {
-                tb = nb - 1 + k;
-                g = a.gold[row];
-                if (nb < 1 || Lb > a.T || tb >= a.Tb || g < 0 || g >= A) {
-                    atomicCAS(a.err, 0, (int)SL_ERR_ARG);  // bad lengths or label: the row is skipped
-                    k = -1;
-                }
-            } else {
-                k = -1;
-            }
+    const int NR = T * B, K = 3 * H, lane = threadIdx.x & 31;
+    const int row = blockIdx.x * (kHeadThreads / 32) + (threadIdx.x >> 5);
+    if (row >= NR) return;
+    const int kk = row / B, b = row % B;
+    int k = -1, tb = 0, g = 0;
+    const int nb = n[b], Lb = L[b];
+    if (kk < Lb) {
+        k = kk;
+        tb = nb - 1 + kk;
+        g = gold[row];
+        if (nb < 1 || Lb > T || tb >= Tb || g < 0 || g >= A) {
+            if (lane == 0) atomicCAS(err, 0, (int)SL_ERR_ARG);  // the row is skipped
+            k = -1;
         }
-        row_k[tid] = k;
-        row_b[tid] = b;
-        row_tb[tid] = tb;
-        row_g[tid] = g;
     }
-    __syncthreads();
-
-    // ---- gather u = [s; bu; a] (16-byte pieces; zeros for padding rows), also to the workspace
-    const int pieces = K / 8;
-    for (int e = tid; e < R * pieces; e += blockDim.x) {
-        const int r = e / pieces, pc = e % pieces, c0 = pc * 8;
-        const int k = row_k[r], b = row_b[r];
+    if (lane == 0) meta[row] = make_int4(k, b, tb, g);
+    for (int pc = lane; pc < K / 8; pc += 32) {
+        const int c0 = pc * 8, part = c0 / H, cc = c0 % H;
         uint4 v = make_uint4(0u, 0u, 0u, 0u);
         if (k >= 0) {
-            const int part = c0 / H, cc = c0 % H;
             const __nv_bfloat16 *src;
             if (part == 0)
-                src = k >= 1 ? a.y_stack + ((size_t)(k - 1) * B + b) * H : a.h0_stack + (size_t)b * H;
+                src = k >= 1 ? y_stack + ((size_t)(k - 1) * B + b) * H : h0_stack + (size_t)b * H;
             else if (part == 1)
-                src = a.y_buffer + ((size_t)row_tb[r] * B + b) * H;
+                src = y_buffer + ((size_t)tb * B + b) * H;
             else
-                src = k >= 1 ? a.y_action + ((size_t)(k - 1) * B + b) * H : a.h0_action + (size_t)b * H;
+                src = k >= 1 ? y_action + ((size_t)(k - 1) * B + b) * H : h0_action + (size_t)b * H;
             v = *(const uint4 *)(src + cc);
         }
-        if (row0 + r < NR) *(uint4 *)(a.u + (size_t)(row0 + r) * K + c0) = v;
-        const __nv_bfloat16 *vh = (const __nv_bfloat16 *)&v;
-#pragma unroll
-        for (int i = 0; i < 8; ++i) u_s[(size_t)(c0 + i) * R + r] = vh[i];
+        *(uint4 *)(u + (size_t)row * K + c0) = v;
+    }
+}
+
+// ut[c][r] = u[r][c] (r < rows), zero for rows .. ld: 32 x 32 tiles through shared memory.
+__global__ void head_transpose(const __nv_bfloat16 *__restrict__ u, int rows, int K, int ld,
+                               __nv_bfloat16 *__restrict__ ut)
+{
+    __shared__ __nv_bfloat16 tile[32][33];
+    const int r0 = blockIdx.x * 32, c0 = blockIdx.y * 32, tx = threadIdx.x, ty = threadIdx.y;
+    for (int i = ty; i < 32; i += blockDim.y) {
+        const int r = r0 + i, c = c0 + tx;
+        tile[i][tx] = (r < rows && c < K) ? u[(size_t)r * K + c] : __float2bfloat16(0.0f);
     }
     __syncthreads();
+    for (int i = ty; i < 32; i += blockDim.y) {
+        const int c = c0 + i, r = r0 + tx;
+        if (c < K && r < ld) ut[(size_t)c * ld + r] = tile[tx][i];
+    }
+}
 
-    // ---- pre = u Wp^T + dp; p = ReLU(pre)   (thread j: column j of all R rows)
-    for (int j = tid; j < P; j += blockDim.x) {
-        float acc[R];
-        const float dpj = a.dp[j];
-#pragma unroll
-        for (int r = 0; r < R; ++r) acc[r] = dpj;
-        for (int c = 0; c < K; ++c) {
-            const float w = __bfloat162float(a.wpt[(size_t)c * P + j]);
-            const uint4 *ur = (const uint4 *)(u_s + (size_t)c * R);
-#pragma unroll
-            for (int q8 = 0; q8 < R / 8; ++q8) {
-                const uint4 v = ur[q8];
-                const __nv_bfloat16 *vh = (const __nv_bfloat16 *)&v;
-#pragma unroll
-                for (int i = 0; i < 8; ++i) acc[q8 * 8 + i] = fmaf(__bfloat162float(vh[i]), w, acc[q8 * 8 + i]);
-            }
-        }
-#pragma unroll
-        for (int r = 0; r < R; ++r) {
-            const float pv = fmaxf(acc[r], 0.0f);
-            p_s[r * P + j] = pv;
-            if (row0 + r < NR) a.p[(size_t)(row0 + r) * P + j] = pv;
-        }
+// kEpiRows rows per CTA: p = ReLU(pre + dp), z = Wz p + q, the row's softmax cross-entropy
+// and dz, dP = (dz Wz) * (pre > 0) stored in bf16; the CTA's partial sums of dWz [A][P],
+// ddp [P] and dq [A] over its rows in row order, to part[blockIdx.x].
+__global__ void __launch_bounds__(kHeadThreads)
+head_epi(int NR, int P, int A, const float *__restrict__ pre, const float *__restrict__ dp,
+         const float *__restrict__ Wz, const float *__restrict__ q, const int4 *__restrict__ meta,
+         float *__restrict__ loss_rows, __nv_bfloat16 *__restrict__ dpb, float *__restrict__ part)
+{
+    extern __shared__ __align__(16) float es[];
+    float *p_s = es;                       // [rows][P]
+    float *dP_s = p_s + kEpiRows * P;      // [rows][P]
+    float *wz_s = dP_s + kEpiRows * P;     // [A][P]
+    float *z_s = wz_s + A * P;             // [rows][8]
+    float *dz_s = z_s + kEpiRows * 8;      // [rows][8]
+    const int tid = threadIdx.x, row0 = blockIdx.x * kEpiRows;
+    const int nrow = min(kEpiRows, NR - row0);
+    for (int i = tid; i < A * P; i += kHeadThreads) wz_s[i] = Wz[i];
+    for (int e = tid; e < kEpiRows * P; e += kHeadThreads) {
+        const int r = e / P, j = e % P;
+        p_s[e] = r < nrow ? fmaxf(pre[(size_t)(row0 + r) * P + j] + dp[j], 0.0f) : 0.0f;
     }
     __syncthreads();
-
-    // ---- z = Wz p + q
-    for (int t = tid; t < R * A; t += blockDim.x) {
-        const int r = t / A, o = t % A;
-        float acc = a.q[o];
+    if (tid < kEpiRows * A) {
+        const int r = tid / A, o = tid % A;
+        float acc = q[o];
         for (int j = 0; j < P; ++j) acc = fmaf(wz_s[o * P + j], p_s[r * P + j], acc);
-        z_s[t] = acc;
+        z_s[r * 8 + o] = acc;
     }
     __syncthreads();
-
-    // ---- softmax cross-entropy of each row and dz
-    if (tid < R) {
+    if (tid < kEpiRows) {
         const int r = tid, row = row0 + r;
-        float m = -INFINITY;
-        for (int o = 0; o < A; ++o) m = fmaxf(m, z_s[r * A + o]);
-        float s = 0.0f;
-        for (int o = 0; o < A; ++o) s += __expf(z_s[r * A + o] - m);
-        const float lse = m + __logf(s);
-        const bool valid = row_k[r] >= 0;
-        for (int o = 0; o < A; ++o) {
-            const float d = valid ? __expf(z_s[r * A + o] - lse) - (o == row_g[r] ? 1.0f : 0.0f) : 0.0f;
-            dz_s[r * A + o] = d;
-            if (row < NR) a.dz[(size_t)row * A + o] = d;
-        }
-        if (row < NR) a.loss_rows[row] = valid ? lse - z_s[r * A + row_g[r]] : 0.0f;
+        const int4 m = r < nrow ? meta[row] : make_int4(-1, 0, 0, 0);
+        float mx = -INFINITY;
+        for (int o = 0; o < A; ++o) mx = fmaxf(mx, z_s[r * 8 + o]);
+        float sum = 0.0f;
+        for (int o = 0; o < A; ++o) sum += __expf(z_s[r * 8 + o] - mx);
+        const float lse = mx + __logf(sum);
+        const bool valid = m.x >= 0;
+        for (int o = 0; o < A; ++o)
+            dz_s[r * 8 + o] = valid ? __expf(z_s[r * 8 + o] - lse) - (o == m.w ? 1.0f : 0.0f) : 0.0f;
+        if (r < nrow) loss_rows[row] = valid ? lse - z_s[r * 8 + m.w] : 0.0f;
     }
     __syncthreads();
-
-    // ---- dP = (dz Wz) * (pre > 0)   (thread j)
-    for (int j = tid; j < P; j += blockDim.x) {
-        for (int r = 0; r < R; ++r) {
-            float acc = 0.0f;
-            for (int o = 0; o < A; ++o) acc = fmaf(dz_s[r * A + o], wz_s[o * P + j], acc);
-            const float d = p_s[r * P + j] > 0.0f ? acc : 0.0f;
-            dP_s[j * R + r] = d;
-            if (row0 + r < NR) a.dP[(size_t)(row0 + r) * P + j] = d;
-        }
+    for (int e = tid; e < kEpiRows * P; e += kHeadThreads) {
+        const int r = e / P, j = e % P;
+        float acc = 0.0f;
+        for (int o = 0; o < A; ++o) acc = fmaf(dz_s[r * 8 + o], wz_s[o * P + j], acc);
+        const float d = p_s[e] > 0.0f ? acc : 0.0f;
+        dP_s[e] = d;
+        if (r < nrow) dpb[(size_t)(row0 + r) * P + j] = __float2bfloat16(d);
     }
     __syncthreads();
-
-    // ---- du = dP Wp, stored into the gradients of the rows the head read
-    for (int c = tid; c < K; c += blockDim.x) {
-        float acc[R];
-#pragma unroll
-        for (int r = 0; r < R; ++r) acc[r] = 0.0f;
-        for (int j = 0; j < P; ++j) {
-            const float w = __bfloat162float(a.Wp[(size_t)j * K + c]);
-            const float4 *dr = (const float4 *)(dP_s + (size_t)j * R);
-#pragma unroll
-            for (int q4 = 0; q4 < R / 4; ++q4) {
-                const float4 v = dr[q4];
-                acc[4 * q4 + 0] = fmaf(v.x, w, acc[4 * q4 + 0]);
-                acc[4 * q4 + 1] = fmaf(v.y, w, acc[4 * q4 + 1]);
-                acc[4 * q4 + 2] = fmaf(v.z, w, acc[4 * q4 + 2]);
-                acc[4 * q4 + 3] = fmaf(v.w, w, acc[4 * q4 + 3]);
-            }
-        }
-        const int part = c / H, cc = c % H;
-#pragma unroll
-        for (int r = 0; r < R; ++r) {
-            const int k = row_k[r], b = row_b[r];
-            if (k < 0) continue;
-            float *dst;
-            if (part == 0)
-                dst = k >= 1 ? a.dy_stack + ((size_t)(k - 1) * B + b) * H : a.dh0 + (size_t)b * H;
-            else if (part == 1)
-                dst = a.dy_buffer + ((size_t)row_tb[r] * B + b) * H;
-            else
-                dst = k >= 1 ? a.dy_action + ((size_t)(k - 1) * B + b) * H : a.dh0 + ((size_t)B + b) * H;
-            dst[cc] = acc[r];
-        }
-    }
-}
-
-// dWp partial sums over row range s: part[s][j][c] = sum over its rows of dP[row][j] u[row][c].
-__global__ void __launch_bounds__(kHeadThreads) head_dwp_part(const float *__restrict__ dP,
-                                                              const __nv_bfloat16 *__restrict__ u, int NR, int P, int K,
-                                                              int S, float *__restrict__ part)
-{
-    __shared__ float d_s[32][kDwpJ];
-    const int tid = threadIdx.x;
-    const int j0 = blockIdx.x * kDwpJ, c = blockIdx.y * blockDim.x + tid, s = blockIdx.z;
-    const int r_lo = (int)((long long)NR * s / S), r_hi = (int)((long long)NR * (s + 1) / S);
-    float acc[kDwpJ];
-#pragma unroll
-    for (int i = 0; i < kDwpJ; ++i) acc[i] = 0.0f;
-    for (int r0 = r_lo; r0 < r_hi; r0 += 32) {
-        {
-            const int rr = tid / kDwpJ, jj = tid % kDwpJ, row = r0 + rr;
-            d_s[rr][jj] = (row < r_hi && j0 + jj < P) ? dP[(size_t)row * P + j0 + jj] : 0.0f;
-        }
-        __syncthreads();
-        const int nr = min(32, r_hi - r0);
-        if (c < K)
-            for (int rr = 0; rr < nr; ++rr) {
-                const float uv = __bfloat162float(u[(size_t)(r0 + rr) * K + c]);
-#pragma unroll
-                for (int i = 0; i < kDwpJ; ++i) acc[i] = fmaf(d_s[rr][i], uv, acc[i]);
-            }
-        __syncthreads();
-    }
-    if (c < K)
-#pragma unroll
-        for (int i = 0; i < kDwpJ; ++i)
-            if (j0 + i < P) part[((size_t)s * P + j0 + i) * K + c] = acc[i];
-}
-
-// Partial sums over row range s of dWz [A][P], ddp [P], dq [A]: part[s][A P + P + A].
-__global__ void __launch_bounds__(kHeadThreads) head_small_part(const float *__restrict__ p, const float *__restrict__ dP,
-                                                                const float *__restrict__ dz, int NR, int P, int A,
-                                                                float *__restrict__ part)
-{
-    const int s = blockIdx.x, S = gridDim.x, tid = threadIdx.x;
-    const int r_lo = (int)((long long)NR * s / S), r_hi = (int)((long long)NR * (s + 1) / S);
     const size_t W = (size_t)A * P + P + A;
-    for (int j = tid; j < P; j += blockDim.x) {
+    float *pc = part + (size_t)blockIdx.x * W;
+    for (int j = tid; j < P; j += kHeadThreads) {
         float aw[8], ad = 0.0f;
 #pragma unroll
         for (int o = 0; o < 8; ++o) aw[o] = 0.0f;
-        for (int row = r_lo; row < r_hi; ++row) {
-            const float pv = p[(size_t)row * P + j];
-            ad += dP[(size_t)row * P + j];
+        for (int r = 0; r < nrow; ++r) {
+            const float pv = p_s[r * P + j];
+            ad += dP_s[r * P + j];
 #pragma unroll
             for (int o = 0; o < 8; ++o)
-                if (o < A) aw[o] = fmaf(dz[(size_t)row * A + o], pv, aw[o]);
+                if (o < A) aw[o] = fmaf(dz_s[r * 8 + o], pv, aw[o]);
         }
 #pragma unroll
         for (int o = 0; o < 8; ++o)
-            if (o < A) part[s * W + (size_t)o * P + j] = aw[o];
-        part[s * W + (size_t)A * P + j] = ad;
+            if (o < A) pc[(size_t)o * P + j] = aw[o];
+        pc[(size_t)A * P + j] = ad;
     }
     if (tid < A) {
         float aq = 0.0f;
-        for (int row = r_lo; row < r_hi; ++row) aq += dz[(size_t)row * A + tid];
-        part[s * W + (size_t)A * P + P + tid] = aq;
+        for (int r = 0; r < nrow; ++r) aq += dz_s[r * 8 + tid];
+        pc[(size_t)A * P + P + tid] = aq;
+    }
+}
+
+// du rows into the gradients of the StackLSTM outputs the head read (the k = 0 reads of
+// the initial states into dh0); one warp per row, 16-byte pieces.
+__global__ void __launch_bounds__(kHeadThreads)
+head_scatter(int NR, int B, int H, const float *__restrict__ du, const int4 *__restrict__ meta,
+             float *__restrict__ dy_stack, float *__restrict__ dy_buffer, float *__restrict__ dy_action,
+             float *__restrict__ dh0)
+{
+    const int lane = threadIdx.x & 31, row = blockIdx.x * (kHeadThreads / 32) + (threadIdx.x >> 5);
+    if (row >= NR) return;
+    const int4 m = meta[row];
+    const int k = m.x, b = m.y;
+    if (k < 0) return;
+    const int K = 3 * H;
+    for (int pc = lane; pc < K / 4; pc += 32) {
+        const int c0 = pc * 4, part = c0 / H, cc = c0 % H;
+        float *dst;
+        if (part == 0)
+            dst = k >= 1 ? dy_stack + ((size_t)(k - 1) * B + b) * H : dh0 + (size_t)b * H;
+        else if (part == 1)
+            dst = dy_buffer + ((size_t)m.z * B + b) * H;
+        else
+            dst = k >= 1 ? dy_action + ((size_t)(k - 1) * B + b) * H : dh0 + ((size_t)B + b) * H;
+        *(float4 *)(dst + cc) = *(const float4 *)(du + (size_t)row * K + c0);
     }
 }
 
@@ -321,6 +233,18 @@ __global__ void head_reduce(const float *__restrict__ part, int S, size_t n0, si
             out1[i - n0] = acc;
         else
             out2[i - n0 - n1] = acc;
+    }
+}
+
+// dWp [P][K] = the sum over s of the parts of dWp^T [s][K][P], in s order.
+__global__ void head_reduce_t(const float *__restrict__ part, int S, int P, int K, float *__restrict__ dWp)
+{
+    const size_t n = (size_t)P * K;
+    for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < n; i += (size_t)gridDim.x * blockDim.x) {
+        const int j = (int)(i / K), c = (int)(i % K);
+        float acc = 0.0f;
+        for (int s = 0; s < S; ++s) acc += part[((size_t)s * K + c) * P + j];
+        dWp[i] = acc;
     }
 }
 
@@ -352,6 +276,10 @@ bool al16(const void *p) { return ((uintptr_t)p & 15u) == 0; }
 
 unsigned grid_n(size_t n) { return (unsigned)std::max<size_t>(1, std::min<size_t>((n + 255) / 256, 4096)); }
 
+size_t epi_smem(int P, int A) { return ((size_t)2 * kEpiRows * P + (size_t)A * P + 2 * kEpiRows * 8) * 4; }
+
+constexpr long long kHeadWaitLimit = 4000000000LL;  // clock cycles one bounded wait of the contraction may spin
+
 }  // namespace
 }  // namespace sl
 
@@ -365,35 +293,33 @@ sl_status stacklstm_head_create(stacklstm_head_t *out, int T, int Tb, int B, int
     if (!out) return SL_ERR_ARG;
     *out = nullptr;
     if (T < 1 || Tb < 1 || B < 1 || H < 1 || P < 1 || A < 2) return SL_ERR_ARG;
-    if (H % 8 || P > kHeadThreads || A > 8 || (long long)T * B > (1LL << 30)) return SL_ERR_UNSUPPORTED;
-    int R = 32;
-    while (R >= 8 && head_smem_bytes(R, H, P, A) > 200 * 1024) R /= 2;
-    if (R < 8) return SL_ERR_UNSUPPORTED;
+    if (H % 8 || P % 8 || P > kHeadThreads || A > 8 || (long long)T * B > (1LL << 30)) return SL_ERR_UNSUPPORTED;
     stacklstm_head *h = new (std::nothrow) stacklstm_head;
     if (!h) return SL_ERR_OOM;
-    h->T = T; h->Tb = Tb; h->B = B; h->H = H; h->P = P; h->A = A; h->R = R;
+    h->T = T; h->Tb = Tb; h->B = B; h->H = H; h->P = P; h->A = A;
     h->device = device;
     h->stream = (cudaStream_t)stream;
-    h->S = std::max(1, std::min(16, (T * B) / 512));
-    h->smem = head_smem_bytes(R, H, P, A);
     int prev = -1;
     cudaGetDevice(&prev);
-    if (cudaSetDevice(device) != cudaSuccess) {
+    if (cudaSetDevice(device) != cudaSuccess ||
+        cudaDeviceGetAttribute(&h->num_sms, cudaDevAttrMultiProcessorCount, device) != cudaSuccess) {
         cudaGetLastError();
         delete h;
         return SL_ERR_ARG;  // no such device
     }
     const size_t NR = (size_t)T * B, K = 3 * (size_t)H;
-    const size_t part = std::max((size_t)h->S * P * K, (size_t)kSmallChunks * ((size_t)A * P + P + A));
-    bool ok = cudaMalloc(&h->wpt, K * P * 2) == cudaSuccess && cudaMalloc(&h->u, NR * K * 2) == cudaSuccess &&
-              cudaMalloc(&h->p, NR * P * 4) == cudaSuccess && cudaMalloc(&h->dP, NR * P * 4) == cudaSuccess &&
-              cudaMalloc(&h->dz, NR * A * 4) == cudaSuccess && cudaMalloc(&h->dh0, 2 * (size_t)B * H * 4) == cudaSuccess &&
-              cudaMalloc(&h->part, part * 4) == cudaSuccess && cudaMalloc(&h->err, 16) == cudaSuccess;
+    h->NR8 = (int)((NR + 7) / 8 * 8);
+    h->S3 = std::max(1, std::min(32, (int)ceil_div(NR, 64) / 8));
+    const size_t nblk = ceil_div(NR, kEpiRows), W = (size_t)A * P + P + A;
+    auto get = [&](auto **p, size_t bytes) { return cudaMalloc((void **)p, std::max<size_t>(bytes, 16)) == cudaSuccess; };
+    bool ok = get(&h->u, NR * K * 2) && get(&h->ut, K * h->NR8 * 2) && get(&h->dpb, NR * P * 2) &&
+              get(&h->meta, NR * 16) && get(&h->pre, NR * P * 4) && get(&h->du, NR * K * 4) &&
+              get(&h->part3, (size_t)h->S3 * K * P * 4) && get(&h->part, nblk * W * 4) &&
+              get(&h->wp_k, bf16_kmajor_bytes(P, (int)K)) && get(&h->wpt_k, bf16_kmajor_bytes((int)K, P)) &&
+              get(&h->dpt_k, bf16_kmajor_bytes(P, (int)NR)) && get(&h->dh0, 2 * (size_t)B * H * 4) &&
+              get(&h->err, 16);
     if (ok) ok = cudaMemset(h->err, 0, 16) == cudaSuccess;
-    if (ok) {
-        const void *fn = R == 32 ? (const void *)head_rows<32> : R == 16 ? (const void *)head_rows<16> : (const void *)head_rows<8>;
-        ok = smem_at_least(fn, h->smem) == cudaSuccess;
-    }
+    if (ok) ok = smem_at_least((const void *)head_epi, epi_smem(P, A)) == cudaSuccess;
     if (prev >= 0) cudaSetDevice(prev);
     if (!ok) {
         cudaGetLastError();
@@ -416,48 +342,50 @@ sl_status stacklstm_head_run(stacklstm_head_t h, const void *y_stack, const void
                           loss_rows, dy_stack, dy_buffer, dy_action, dWp, ddp, dWz, dq};
     for (const void *p : need)
         if (!p) return head_fail(h, SL_ERR_ARG, "null pointer");
-    const void *vec[] = {y_stack, h0_stack, y_buffer, y_action, h0_action};
+    const void *vec[] = {y_stack, h0_stack, y_buffer, y_action, h0_action, Wp, dy_stack, dy_buffer, dy_action};
     for (const void *p : vec)
-        if (!al16(p)) return head_fail(h, SL_ERR_ARG, "StackLSTM outputs must be 16-byte aligned");
+        if (!al16(p)) return head_fail(h, SL_ERR_ARG, "StackLSTM outputs, Wp and dy must be 16-byte aligned");
     int prev = -1;
     cudaGetDevice(&prev);
     cudaSetDevice(h->device);
-    const int T = h->T, B = h->B, H = h->H, P = h->P, A = h->A, K = 3 * H;
-    const size_t NR = (size_t)T * B;
+    const int T = h->T, B = h->B, H = h->H, P = h->P, A = h->A, K = 3 * H, NR = T * B, sms = h->num_sms;
+    const unsigned nblk = ceil_div(NR, kEpiRows), wrows = ceil_div(NR, kHeadThreads / 32);
+    const __nv_bfloat16 *wp = (const __nv_bfloat16 *)Wp;
     cudaStream_t st = h->stream;
     cudaError_t e = cudaSuccess;
-    // outputs the row kernel does not write everywhere start at zero
-    if (!e) e = cudaMemsetAsync(dy_stack, 0, NR * H * 4, st);
-    if (!e) e = cudaMemsetAsync(dy_action, 0, NR * H * 4, st);
+    // rows of the StackLSTM output gradients the head does not read stay zero
+    if (!e) e = cudaMemsetAsync(dy_stack, 0, (size_t)NR * H * 4, st);
+    if (!e) e = cudaMemsetAsync(dy_action, 0, (size_t)NR * H * 4, st);
     if (!e) e = cudaMemsetAsync(dy_buffer, 0, (size_t)h->Tb * B * H * 4, st);
     if (!e) e = cudaMemsetAsync(h->dh0, 0, 2 * (size_t)B * H * 4, st);
+    // the weights as contraction operands: Wp rows (pre = U Wp^T) and its columns (du = dP Wp)
+    if (!e) e = bf16_pack_kmajor(wp, K, false, P, K, h->wp_k, st, sms);
+    if (!e) e = bf16_pack_kmajor(wp, K, true, K, P, h->wpt_k, st, sms);
     if (!e) {
-        head_pack_wpt<<<grid_n((size_t)P * K), 256, 0, st>>>((const __nv_bfloat16 *)Wp, P, K, h->wpt);
-        HeadArgs a;
-        a.T = T; a.Tb = h->Tb; a.B = B; a.H = H; a.P = P; a.A = A;
-        a.y_stack = (const __nv_bfloat16 *)y_stack; a.h0_stack = (const __nv_bfloat16 *)h0_stack;
-        a.y_buffer = (const __nv_bfloat16 *)y_buffer; a.y_action = (const __nv_bfloat16 *)y_action;
-        a.h0_action = (const __nv_bfloat16 *)h0_action;
-        a.n = n; a.L = L; a.gold = gold;
-        a.Wp = (const __nv_bfloat16 *)Wp; a.wpt = h->wpt; a.dp = dp; a.Wz = Wz; a.q = q;
-        a.loss_rows = loss_rows; a.dy_stack = dy_stack; a.dy_buffer = dy_buffer; a.dy_action = dy_action;
-        a.dh0 = h->dh0; a.u = h->u; a.p = h->p; a.dP = h->dP; a.dz = h->dz; a.err = h->err;
-        const unsigned grid = (unsigned)((NR + h->R - 1) / h->R);
-        if (h->R == 32)
-            head_rows<32><<<grid, kHeadThreads, h->smem, st>>>(a);
-        else if (h->R == 16)
-            head_rows<16><<<grid, kHeadThreads, h->smem, st>>>(a);
-        else
-            head_rows<8><<<grid, kHeadThreads, h->smem, st>>>(a);
-        head_dwp_part<<<dim3((P + kDwpJ - 1) / kDwpJ, (K + kHeadThreads - 1) / kHeadThreads, h->S), kHeadThreads, 0,
-                        st>>>(h->dP, h->u, (int)NR, P, K, h->S, h->part);
-        head_reduce<<<grid_n((size_t)P * K), 256, 0, st>>>(h->part, h->S, (size_t)P * K, 0, 0, dWp, nullptr, nullptr);
+        head_gather<<<wrows, kHeadThreads, 0, st>>>(T, h->Tb, B, H, A, (const __nv_bfloat16 *)y_stack,
+                                                    (const __nv_bfloat16 *)h0_stack, (const __nv_bfloat16 *)y_buffer,
+                                                    (const __nv_bfloat16 *)y_action, (const __nv_bfloat16 *)h0_action,
+                                                    n, L, gold, h->u, h->meta, h->err);
         e = cudaGetLastError();
     }
+    if (!e) e = bf16_gemm(h->u, K, NR, K, h->wp_k, P, h->pre, 1, st, sms, kHeadWaitLimit, h->err);
     if (!e) {
-        // dWz, ddp, dq reuse the partial buffer after dWp's reduction (same stream)
-        head_small_part<<<kSmallChunks, kHeadThreads, 0, st>>>(h->p, h->dP, h->dz, (int)NR, P, A, h->part);
-        head_reduce<<<grid_n((size_t)A * P + P + A), 256, 0, st>>>(h->part, kSmallChunks, (size_t)A * P, (size_t)P,
+        head_epi<<<nblk, kHeadThreads, epi_smem(P, A), st>>>(NR, P, A, h->pre, dp, Wz, q, h->meta, loss_rows, h->dpb,
+                                                             h->part);
+        e = cudaGetLastError();
+    }
+    if (!e) e = bf16_gemm(h->dpb, P, NR, P, h->wpt_k, K, h->du, 1, st, sms, kHeadWaitLimit, h->err);
+    if (!e) {
+        head_scatter<<<wrows, kHeadThreads, 0, st>>>(NR, B, H, h->du, h->meta, dy_stack, dy_buffer, dy_action, h->dh0);
+        head_transpose<<<dim3(ceil_div(h->NR8, 32), ceil_div(K, 32)), dim3(32, 8), 0, st>>>(h->u, NR, K, h->NR8, h->ut);
+        e = cudaGetLastError();
+    }
+    // dWp^T = U^T dP: a split contraction over the rows, then the parts summed in order
+    if (!e) e = bf16_pack_kmajor(h->dpb, P, true, P, NR, h->dpt_k, st, sms);
+    if (!e) e = bf16_gemm(h->ut, h->NR8, K, NR, h->dpt_k, P, h->part3, h->S3, st, sms, kHeadWaitLimit, h->err);
+    if (!e) {
+        head_reduce_t<<<grid_n((size_t)P * K), 256, 0, st>>>(h->part3, h->S3, P, K, dWp);
+        head_reduce<<<grid_n((size_t)A * P + P + A), 256, 0, st>>>(h->part, (int)nblk, (size_t)A * P, (size_t)P,
                                                                    (size_t)A, dWz, ddp, dq);
         e = cudaGetLastError();
     }
@@ -490,6 +418,7 @@ sl_status stacklstm_head_status(stacklstm_head_t h)
     if (!e && v) e = cudaMemset(h->err, 0, 4);
     if (prev >= 0) cudaSetDevice(prev);
     if (e) return head_cuda(h, e, "stacklstm_head_status");
+    if (v == SL_ERR_TIMEOUT) return head_fail(h, SL_ERR_TIMEOUT, "a device-side wait of a contraction ran out");
     if (v) return head_fail(h, (sl_status)v, "a transition with a bad length or label was skipped");
     return SL_OK;
 }
@@ -501,7 +430,8 @@ sl_status stacklstm_head_destroy(stacklstm_head_t h)
     cudaGetDevice(&prev);
     cudaSetDevice(h->device);
     if (h->stream) cudaStreamSynchronize(h->stream);
-    void *ps[] = {h->wpt, h->u, h->p, h->dP, h->dz, h->dh0, h->part, h->err};
+    void *ps[] = {h->u, h->ut, h->dpb, h->meta, h->pre, h->du, h->part3, h->part, h->wp_k, h->wpt_k, h->dpt_k,
+                  h->dh0, h->err};
     for (void *p : ps)
         if (p) cudaFree(p);
     if (prev >= 0) cudaSetDevice(prev);
