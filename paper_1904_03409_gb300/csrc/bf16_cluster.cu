@@ -159,7 +159,7 @@ __device__ __forceinline__ void deliver_slice(const ClCtl &c, uint8_t *blk, int 
 constexpr int kClFwdThreads = 224;  // 4 epilogue warps, producer, two MMA issuers
 
 template <int U>
-__device__ __forceinline__ void step_cl_body(const CUtensorMap *tmx, const ClArgs &p)
+__device__ __forceinline__ void step_cl_body(const CUtensorMap *tmx, const ClArgs &p, int row0)
 {
     static_assert(U == 16, "one h slice (two 8-unit core matrices) per CTA");
     constexpr int NB = 4 * U;
@@ -170,6 +170,9 @@ __device__ __forceinline__ void step_cl_body(const CUtensorMap *tmx, const ClArg
     __shared__ float s_bias[4 * U];
     const int T = a.T, B = a.B, H = a.H, KC = a.KC, kcx = a.kcx;
     const uint32_t ct = tc::cluster_rank(), n_ct = (uint32_t)p.n_ct;
+    // this cluster's row tile: rows row0 .. row0 + nrows - 1 of the batch, and its slice blocks
+    const int nrows = min(64, B - row0);
+    uint8_t *gscr = p.gscr + (size_t)(row0 / 64) * T * n_ct * kSlice;
     const ClCtl c = cl_carve(smem_raw, KC, kcx, NB, (int)n_ct);
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const long long limit = a.limit;
@@ -214,7 +217,7 @@ __device__ __forceinline__ void step_cl_body(const CUtensorMap *tmx, const ClArg
                 }
                 tc::mbar_arrive_expect_tx(&c.xfull[b], (uint32_t)kcx * kC64);
                 for (int j = 0; j < kcx; ++j)
-                    tc::tma_load_2d(c.x0 + (b * kcx + j) * kC64, tmx, j * kChunk, t * B, &c.xfull[b]);
+                    tc::tma_load_2d(c.x0 + (b * kcx + j) * kC64, tmx, j * kChunk, t * B + row0, &c.xfull[b]);
                 last = t;
             }
             // copies still in flight after an abort land before the CTA exits (each buffer's
@@ -275,8 +278,9 @@ __device__ __forceinline__ void step_cl_body(const CUtensorMap *tmx, const ClArg
         // ------------------------------------------------------------ epilogue
         // M = 64 accumulator: rows 16 w .. 16 w + 15 in lanes 0..15 of TMEM lane quadrant w
         const int row = lane < 16 ? warp * 16 + lane : 64;  // lanes 16..31 hold no row
-        const bool row_ok = row < B;
-        const bool warp_rows = warp * 16 < B;
+        const int grow = row0 + row;                          // the row of the whole batch
+        const bool row_ok = row < nrows;
+        const bool warp_rows = warp * 16 < nrows;
         const int u0 = (int)ct * U;
         const bool v0 = row_ok && u0 < H, v1 = row_ok && u0 + 8 < H;  // the two 8-unit groups (H % 8 == 0)
         const uint32_t taddr0 = tmem + ((uint32_t)(warp * 32) << 16);
@@ -288,21 +292,21 @@ __device__ __forceinline__ void step_cl_body(const CUtensorMap *tmx, const ClArg
         int s_nxt = 0, s_2 = 0;
         uint4 h0v[2];
         if (v0) {
-            const int s_cur = a.top[row];
-            s_nxt = T >= 1 ? a.top[(size_t)B + row] : 0;
-            s_2 = T >= 2 ? a.top[(size_t)2 * B + row] : 0;
+            const int s_cur = a.top[grow];
+            s_nxt = T >= 1 ? a.top[(size_t)B + grow] : 0;
+            s_2 = T >= 2 ? a.top[(size_t)2 * B + grow] : 0;
 #pragma unroll
             for (int i = 0; i < 2; ++i) {
                 if (i == 1 && !v1) break;
                 float v[8];
-                ld8f_a32(a.hist_c + ((size_t)s_cur * B + row) * H + u0 + 8 * i, v);
+                ld8f_a32(a.hist_c + ((size_t)s_cur * B + grow) * H + u0 + 8 * i, v);
 #pragma unroll
                 for (int k = 0; k < 8; ++k) crv[8 * i + k] = v[k];
-                hold[i] = __ldcg((const uint4 *)(a.hr + ((size_t)s_nxt * B + row) * H + u0 + 8 * i));
-                h0v[i] = __ldcg((const uint4 *)(a.hr + (size_t)row * H + u0 + 8 * i));  // h_read(0)
+                hold[i] = __ldcg((const uint4 *)(a.hr + ((size_t)s_nxt * B + grow) * H + u0 + 8 * i));
+                h0v[i] = __ldcg((const uint4 *)(a.hr + (size_t)grow * H + u0 + 8 * i));  // h_read(0)
             }
         }
-        deliver_slice(c, p.gscr + (size_t)ct * kSlice, 0, row, h0v, v0, v1, ct, n_ct, tid);
+        deliver_slice(c, gscr + (size_t)ct * kSlice, 0, row, h0v, v0, v1, ct, n_ct, tid);
         for (int t = 0; t < T; ++t) {
             const int b = t & 1;
             // the next step's operands that rows written before this step hold: issued now,
@@ -312,17 +316,17 @@ __device__ __forceinline__ void step_cl_body(const CUtensorMap *tmx, const ClArg
             uint4 hold_n[2];
             int s_3 = 0;
             if (v0 && t + 1 < T) {
-                if (t + 3 <= T) s_3 = a.top[(size_t)(t + 3) * B + row];
+                if (t + 3 <= T) s_3 = a.top[(size_t)(t + 3) * B + grow];
 #pragma unroll
                 for (int i = 0; i < 2; ++i) {
                     if (i == 1 && !v1) break;
                     if (s_nxt != t + 1) {
                         float v[8];
-                        ld8f_a32(a.hist_c + ((size_t)s_nxt * B + row) * H + u0 + 8 * i, v);
+                        ld8f_a32(a.hist_c + ((size_t)s_nxt * B + grow) * H + u0 + 8 * i, v);
 #pragma unroll
                         for (int k = 0; k < 8; ++k) cr_n[8 * i + k] = v[k];
                     }
-                    if (s_2 <= t) hold_n[i] = __ldcg((const uint4 *)(a.hr + ((size_t)s_2 * B + row) * H + u0 + 8 * i));
+                    if (s_2 <= t) hold_n[i] = __ldcg((const uint4 *)(a.hr + ((size_t)s_2 * B + grow) * H + u0 + 8 * i));
                 }
             }
             const bool ok = tc::mbar_wait(&c.tfull[b], (t >> 1) & 1, limit, c.abort);
@@ -371,11 +375,11 @@ __device__ __forceinline__ void step_cl_body(const CUtensorMap *tmx, const ClArg
                 hop[i] = is_new ? hb[i] : hold[i];
             }
             if (t + 1 < T)
-                deliver_slice(c, p.gscr + ((size_t)(t + 1) * n_ct + ct) * kSlice, (t + 1) & 1, row, hop, v0, v1, ct, n_ct,
+                deliver_slice(c, gscr + ((size_t)(t + 1) * n_ct + ct) * kSlice, (t + 1) & 1, row, hop, v0, v1, ct, n_ct,
                               tid);
             if (v0) {
                 // history row t + 1, the h operand row t + 1 (for the weight gradient), the gates
-                const size_t w = ((size_t)(t + 1) * B + row) * H + u0;
+                const size_t w = ((size_t)(t + 1) * B + grow) * H + u0;
 #pragma unroll
                 for (int i = 0; i < 2; ++i) {
                     if (i == 1 && !v1) break;
@@ -385,7 +389,7 @@ __device__ __forceinline__ void step_cl_body(const CUtensorMap *tmx, const ClArg
                 }
                 if (a.gates_blk) {
                     // this CTA's 4 x 16 gates of the row: one 128-byte block, a 32-byte store a gate
-                    __half *gt = a.gates + (((size_t)t * B + row) * n_ct + ct) * 4 * U;
+                    __half *gt = a.gates + (((size_t)t * B + grow) * n_ct + ct) * 4 * U;
 #pragma unroll
                     for (int g = 0; g < 4; ++g) {
                         const uint4 lo = pack8_f16(*(const float(*)[8])(gv[g])), hi = pack8_f16(*(const float(*)[8])(gv[g] + 8));
@@ -393,7 +397,7 @@ __device__ __forceinline__ void step_cl_body(const CUtensorMap *tmx, const ClArg
                         st8u_a32(gt + g * U, q);
                     }
                 } else {
-                    __half *gt = a.gates + ((size_t)t * B + row) * 4 * H + u0;
+                    __half *gt = a.gates + ((size_t)t * B + grow) * 4 * H + u0;
 #pragma unroll
                     for (int i = 0; i < 2; ++i) {
                         if (i == 1 && !v1) break;
@@ -426,7 +430,8 @@ __device__ __forceinline__ void step_cl_body(const CUtensorMap *tmx, const ClArg
     if (warp == E) tc::tmem_dealloc(tmem, 2 * kCols);
 }
 
-constexpr int kClU = 16;  // hidden units per CTA
+constexpr int kClU = 16;        // hidden units per CTA
+constexpr int kClMaxTiles = 8;  // row tiles (clusters) of one launch
 
 // ====================================================================== backward
 // The reverse-time backward (Sec. 5) for one row tile (B <= 64) as one thread-block
@@ -542,7 +547,7 @@ constexpr int kClbIssuers = 4;                          // MMA issue warps
 constexpr int kClBwdThreads = (4 + kClbIssuers) * 32;  // and 4 epilogue warps
 
 template <int U>
-__device__ __forceinline__ void step_clb_body(const ClArgs &p)
+__device__ __forceinline__ void step_clb_body(const ClArgs &p, int row0)
 {
     static_assert(U == 16, "four 16-unit gate slices per CTA");
     constexpr int NI = kClbIssuers;
@@ -553,6 +558,9 @@ __device__ __forceinline__ void step_clb_body(const ClArgs &p)
     extern __shared__ uint8_t smem_raw[];
     const int T = a.T, B = a.B, H = a.H;
     const uint32_t ct = tc::cluster_rank(), n_ct = (uint32_t)p.n_ct;
+    // this cluster's row tile: rows row0 .. row0 + nrows - 1 of the batch, and its dG blocks
+    const int nrows = min(64, B - row0);
+    uint8_t *gscr = p.gscr + (size_t)(row0 / 64) * T * n_ct * kGBlock;
     const ClbCtl c = clb_carve(smem_raw, (int)n_ct);
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const long long limit = a.limit;
@@ -628,8 +636,9 @@ __device__ __forceinline__ void step_clb_body(const ClArgs &p)
         // ------------------------------------------------------------ epilogue
         // M = 64 accumulator: rows 16 w .. 16 w + 15 in lanes 0..15 of TMEM lane quadrant w
         const int row = lane < 16 ? warp * 16 + lane : 64;  // lanes 16..31 hold no row
-        const bool row_ok = row < B;
-        const bool warp_rows = warp * 16 < B;
+        const int grow = row0 + row;                          // the row of the whole batch
+        const bool row_ok = row < nrows;
+        const bool warp_rows = warp * 16 < nrows;
         const int u0 = (int)ct * U;
         const bool v0 = row_ok && u0 < H, v1 = row_ok && u0 + 8 < H;  // the two 8-unit groups (H % 8 == 0)
         const uint32_t taddr0 = tmem + ((uint32_t)(warp * 32) << 16);
@@ -642,16 +651,16 @@ __device__ __forceinline__ void step_clb_body(const ClArgs &p)
 #pragma unroll
                     for (int i = 0; i < 2; ++i)
                         if (i == 0 || v1)
-                            g0v[g][i] = __ldcg((const uint4 *)(a.dG + ((size_t)(T - 1) * B + row) * 4 * H + g * H + u0 + 8 * i));
-            uint8_t *blk = p.gscr + ((size_t)(T - 1) * n_ct + ct) * kGBlock;
+                            g0v[g][i] = __ldcg((const uint4 *)(a.dG + ((size_t)(T - 1) * B + grow) * 4 * H + g * H + u0 + 8 * i));
+            uint8_t *blk = gscr + ((size_t)(T - 1) * n_ct + ct) * kGBlock;
             store_dg_block(blk, row, g0v, v0, v1);
             deliver_dg(c, blk, -1, ct, n_ct, tid, limit, a.err);
         }
         // the state step t reads (src) and the one step t - 1 read (s1): a step ahead
         int src = 0, s1 = 0;
         if (row_ok) {
-            src = a.top[(size_t)(T - 1) * B + row];
-            s1 = T >= 2 ? a.top[(size_t)(T - 2) * B + row] : 0;
+            src = a.top[(size_t)(T - 1) * B + grow];
+            s1 = T >= 2 ? a.top[(size_t)(T - 2) * B + grow] : 0;
         }
         for (int k = 0; k < T; ++k) {
             const int t = T - 1 - k, acc = k & 1;
@@ -660,31 +669,31 @@ __device__ __forceinline__ void step_clb_body(const ClArgs &p)
             uint4 gq[4][2];
             int src_n = 0, s1_n = 0;
             if (row_ok && t >= 1) {
-                src_n = a.top[(size_t)(t - 1) * B + row];
-                s1_n = t >= 2 ? a.top[(size_t)(t - 2) * B + row] : 0;
+                src_n = a.top[(size_t)(t - 1) * B + grow];
+                s1_n = t >= 2 ? a.top[(size_t)(t - 2) * B + grow] : 0;
             }
             if (v0)
 #pragma unroll
                 for (int i = 0; i < 2; ++i) {
                     if (i == 1 && !v1) break;
-                    const size_t us = ((size_t)src * B + row) * H + u0 + 8 * i;
+                    const size_t us = ((size_t)src * B + grow) * H + u0 + 8 * i;
                     ld8f_a32(a.dhist_h + us, *(float(*)[8])(dh_src + 8 * i));
                     if (t >= 1) {
-                        const size_t wr = ((size_t)t * B + row) * H + u0 + 8 * i, rd = ((size_t)s1 * B + row) * H + u0 + 8 * i;
+                        const size_t wr = ((size_t)t * B + grow) * H + u0 + 8 * i, rd = ((size_t)s1 * B + grow) * H + u0 + 8 * i;
                         ld8f_a32(a.dhist_h + wr, *(float(*)[8])(dh_t + 8 * i));
                         ld8f_a32(a.dhist_c + wr, *(float(*)[8])(dc_t + 8 * i));
                         ld8f_a32(a.hist_c + wr, *(float(*)[8])(cn + 8 * i));
                         ld8f_a32(a.hist_c + rd, *(float(*)[8])(cr + 8 * i));
                         ld8f_a32(a.dhist_c + rd, *(float(*)[8])(dc_rd + 8 * i));
                         if (!a.gates_blk) {
-                            const __half *gt = a.gates + ((size_t)(t - 1) * B + row) * 4 * H + u0 + 8 * i;
+                            const __half *gt = a.gates + ((size_t)(t - 1) * B + grow) * 4 * H + u0 + 8 * i;
 #pragma unroll
                             for (int g = 0; g < 4; ++g) gq[g][i] = __ldcg((const uint4 *)(gt + (size_t)g * H));
                         }
                     }
                 }
             if (v0 && t >= 1 && a.gates_blk) {
-                const __half *gt = a.gates + (((size_t)(t - 1) * B + row) * n_ct + ct) * 4 * U;
+                const __half *gt = a.gates + (((size_t)(t - 1) * B + grow) * n_ct + ct) * 4 * U;
 #pragma unroll
                 for (int g = 0; g < 4; ++g) {
                     uint32_t q[8];
@@ -749,7 +758,7 @@ __device__ __forceinline__ void step_clb_body(const ClArgs &p)
 #pragma unroll
                     for (int i = 0; i < 2; ++i) dg[g][i] = pack8_bf16(*(const float(*)[8])(d[g] + 8 * i));
                 // dG_{t-1}: its block to global memory, then (multicast bulk copy) to every CTA
-                uint8_t *blk = p.gscr + ((size_t)(t - 1) * n_ct + ct) * kGBlock;
+                uint8_t *blk = gscr + ((size_t)(t - 1) * n_ct + ct) * kGBlock;
                 store_dg_block(blk, row, dg, v0, v1);
                 deliver_dg(c, blk, k & 1, ct, n_ct, tid, limit, a.err);
                 // and in the [T B][4H] layout (for the input and weight gradients), after the delivery
@@ -757,7 +766,7 @@ __device__ __forceinline__ void step_clb_body(const ClArgs &p)
 #pragma unroll
                     for (int i = 0; i < 2; ++i) {
                         if (i == 1 && !v1) break;
-                        __nv_bfloat16 *gp = a.dG + ((size_t)(t - 1) * B + row) * 4 * H + u0 + 8 * i;
+                        __nv_bfloat16 *gp = a.dG + ((size_t)(t - 1) * B + grow) * 4 * H + u0 + 8 * i;
 #pragma unroll
                         for (int g = 0; g < 4; ++g) *(uint4 *)(gp + (size_t)g * H) = dg[g][i];
                     }
@@ -766,8 +775,8 @@ __device__ __forceinline__ void step_clb_body(const ClArgs &p)
 #pragma unroll
                 for (int i = 0; i < 2; ++i) {
                     if (i == 1 && !v1) break;
-                    st8f_a32(a.dhist_h + ((size_t)src * B + row) * H + u0 + 8 * i, *(const float(*)[8])(v + 8 * i));
-                    if (t >= 1) st8f_a32(a.dhist_c + ((size_t)s1 * B + row) * H + u0 + 8 * i, *(const float(*)[8])(dcr + 8 * i));
+                    st8f_a32(a.dhist_h + ((size_t)src * B + grow) * H + u0 + 8 * i, *(const float(*)[8])(v + 8 * i));
+                    if (t >= 1) st8f_a32(a.dhist_c + ((size_t)s1 * B + grow) * H + u0 + 8 * i, *(const float(*)[8])(dcr + 8 * i));
                 }
             src = src_n;
             s1 = s1_n;
@@ -788,12 +797,12 @@ __device__ __forceinline__ void step_clb_body(const ClArgs &p)
 template <int U>
 __global__ void __launch_bounds__(kClFwdThreads, 1) step_cl(const __grid_constant__ CUtensorMap tm_x, ClArgs p)
 {
-    step_cl_body<U>(&tm_x, p);
+    step_cl_body<U>(&tm_x, p, (int)(blockIdx.x / p.n_ct) * 64);  // cluster m: row tile m
 }
 template <int U>
 __global__ void __launch_bounds__(kClBwdThreads, 1) step_clb(ClArgs p)
 {
-    step_clb_body<U>(p);
+    step_clb_body<U>(p, (int)(blockIdx.x / p.n_ct) * 64);
 }
 
 // Several handles' recurrences in one launch: cluster m (CTAs m n_ct .. m n_ct + n_ct - 1)
@@ -808,27 +817,29 @@ template <int U>
 __global__ void __launch_bounds__(kClFwdThreads, 1) step_cl_group(const __grid_constant__ ClGroup g)
 {
     const int m = (int)blockIdx.x / g.p[0].n_ct;
-    step_cl_body<U>(&g.tm[m], g.p[m]);
+    step_cl_body<U>(&g.tm[m], g.p[m], 0);
 }
 template <int U>
 __global__ void __launch_bounds__(kClBwdThreads, 1) step_clb_group(const __grid_constant__ ClGroup g)
 {
     const int m = (int)blockIdx.x / g.p[0].n_ct;
-    step_clb_body<U>(g.p[m]);
+    step_clb_body<U>(g.p[m], 0);
 }
 
 }  // namespace
 
-// One row tile (B <= 64), at most 16 column tiles of 16 units, the footprint within the
-// shared-memory cap, and a cluster of that size co-resident on this GPU;
-// STACKLSTM_FWD_CLUSTER=0 turns it off (test hook, include/stacklstm.h).
+// Row tiles of 64 instances (instances are independent, so each tile is its own cluster
+// of the one launch) up to kClMaxTiles, at most 16 column tiles of 16 units, the footprint
+// within the shared-memory cap, and every tile's cluster co-resident on this GPU (a tile
+// waiting for SMs would wait for another's whole recurrence); STACKLSTM_FWD_CLUSTER=0
+// turns it off (test hook, include/stacklstm.h).
 bool bf16_plan_fwd_cluster(stacklstm *s, PersistPlan *pl)
 {
     pl->on = 0;
     const char *env = getenv("STACKLSTM_FWD_CLUSTER");
     if (env && atoi(env) == 0) return false;
-    const int n_ct = (int)ceil_div(s->H, kClU);
-    if (s->B > 64 || n_ct > 16) return false;
+    const int n_ct = (int)ceil_div(s->H, kClU), tiles = (int)ceil_div(s->B, 64);
+    if (tiles > kClMaxTiles || n_ct > 16) return false;
     const int NB = 4 * kClU;
     const uint32_t smem = cl_smem_bytes(s->kcf, s->kcx, NB, n_ct);
     if (smem > kSmemCap) return false;
@@ -850,7 +861,7 @@ bool bf16_plan_fwd_cluster(stacklstm *s, PersistPlan *pl)
     cfg.attrs = at;
     cfg.numAttrs = 1;
     int clusters = 0;
-    if (cudaOccupancyMaxActiveClusters(&clusters, fn, &cfg) != cudaSuccess || clusters < 1) {
+    if (cudaOccupancyMaxActiveClusters(&clusters, fn, &cfg) != cudaSuccess || clusters < tiles) {
         cudaGetLastError();
         return false;
     }
@@ -859,7 +870,7 @@ bool bf16_plan_fwd_cluster(stacklstm *s, PersistPlan *pl)
     pl->EP = 1;
     pl->n_ct = n_ct;
     pl->cl = n_ct;
-    pl->slot = 1;
+    pl->slot = tiles;
     pl->smem = smem;
     pl->threads = kClFwdThreads;
     return true;
@@ -874,7 +885,7 @@ cudaError_t bf16_launch_fwd_cluster(stacklstm *s, const StepArgs &a, const CUten
     p.n_ct = pl.n_ct;
     p.gscr = (uint8_t *)s->g_fcl;
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(pl.n_ct);
+    cfg.gridDim = dim3(pl.n_ct * pl.slot);  // one cluster per row tile
     cfg.blockDim = dim3(pl.threads);
     cfg.dynamicSmemBytes = pl.smem;
     cfg.stream = s->stream;
@@ -891,9 +902,9 @@ cudaError_t bf16_launch_fwd_cluster(stacklstm *s, const StepArgs &a, const CUten
     return cudaGetLastError();
 }
 
-// The backward of one row tile as a cluster: B <= 64, at most 16 column tiles of 16 units,
-// a co-resident cluster of that size; STACKLSTM_BWD_CLUSTER=0 turns it off (test hook,
-// include/stacklstm.h). (Copying each CTA's 8 KB of dG into every CTA with bulk copies instead of
+// The backward as one cluster per row tile of 64 instances (as the forward above); at most
+// 16 column tiles of 16 units, every tile's cluster co-resident; STACKLSTM_BWD_CLUSTER=0
+// turns it off (test hook, include/stacklstm.h). (Copying each CTA's 8 KB of dG into every CTA with bulk copies instead of
 // the multicast tensor loads ran 30 % slower than the persistent backward at B = 64,
 // H = 200: n_ct^2 copies a step, issued one after another by one thread of each CTA.)
 bool bf16_plan_bwd_cluster(stacklstm *s, PersistPlan *pl)
@@ -901,8 +912,8 @@ bool bf16_plan_bwd_cluster(stacklstm *s, PersistPlan *pl)
     pl->on = 0;
     const char *env = getenv("STACKLSTM_BWD_CLUSTER");
     if (env && atoi(env) == 0) return false;
-    const int n_ct = (int)ceil_div(s->H, kClU);
-    if (s->B > 64 || n_ct > 16) return false;
+    const int n_ct = (int)ceil_div(s->H, kClU), tiles = (int)ceil_div(s->B, 64);
+    if (tiles > kClMaxTiles || n_ct > 16) return false;
     const uint32_t smem = clb_smem_bytes(n_ct);
     if (smem > kSmemCap) return false;
     const void *fn = (const void *)step_clb<kClU>;
@@ -923,7 +934,7 @@ bool bf16_plan_bwd_cluster(stacklstm *s, PersistPlan *pl)
     cfg.attrs = at;
     cfg.numAttrs = 1;
     int clusters = 0;
-    if (cudaOccupancyMaxActiveClusters(&clusters, fn, &cfg) != cudaSuccess || clusters < 1) {
+    if (cudaOccupancyMaxActiveClusters(&clusters, fn, &cfg) != cudaSuccess || clusters < tiles) {
         cudaGetLastError();
         return false;
     }
@@ -932,14 +943,20 @@ bool bf16_plan_bwd_cluster(stacklstm *s, PersistPlan *pl)
     pl->EP = 1;
     pl->n_ct = n_ct;
     pl->cl = n_ct;
-    pl->slot = 1;
+    pl->slot = tiles;
     pl->smem = smem;
     pl->threads = kClBwdThreads;
     return true;
 }
 
-size_t bf16_fwd_cluster_block_bytes(int T, int H) { return (size_t)T * ceil_div(H, kClU) * kSlice; }
-size_t bf16_bwd_cluster_block_bytes(int T, int H) { return (size_t)T * ceil_div(H, kClU) * kGBlock; }
+size_t bf16_fwd_cluster_block_bytes(int T, int B, int H)
+{
+    return ceil_div(B, 64) * (size_t)T * ceil_div(H, kClU) * kSlice;
+}
+size_t bf16_bwd_cluster_block_bytes(int T, int B, int H)
+{
+    return ceil_div(B, 64) * (size_t)T * ceil_div(H, kClU) * kGBlock;
+}
 
 size_t bf16_bwd_cluster_weight_bytes(int H)
 {
@@ -965,7 +982,7 @@ cudaError_t bf16_launch_bwd_cluster(stacklstm *s, const StepArgs &a)
     p.n_ct = pl.n_ct;
     p.gscr = (uint8_t *)s->g_bcl;
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(pl.n_ct);
+    cfg.gridDim = dim3(pl.n_ct * pl.slot);  // one cluster per row tile
     cfg.blockDim = dim3(pl.threads);
     cfg.dynamicSmemBytes = pl.smem;
     cfg.stream = s->stream;
@@ -994,7 +1011,7 @@ cudaError_t launch_cluster_group(stacklstm *const *hs, const StepArgs *as, const
     for (int m = 0; m < n; ++m) {
         stacklstm *s = hs[m];
         const PersistPlan &pl = kFwd ? s->fc : s->bc;
-        if (!pl.on || pl.n_ct != n_ct) return cudaErrorInvalidValue;
+        if (!pl.on || pl.n_ct != n_ct || pl.slot != 1) return cudaErrorInvalidValue;
         ClArgs &p = g.p[m];
         p.s = as[m];
         p.s.gates_blk = kFwd ? s->bc.on : s->fc.on;

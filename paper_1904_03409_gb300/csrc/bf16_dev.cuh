@@ -210,8 +210,8 @@ cudaError_t bf16_launch_bwd_cluster(stacklstm *s, const StepArgs &a);
 cudaError_t bf16_launch_fwd_cluster_group(stacklstm *const *hs, const StepArgs *as, const CUtensorMap *const *tms, int n,
                                           cudaStream_t st);
 cudaError_t bf16_launch_bwd_cluster_group(stacklstm *const *hs, const StepArgs *as, int n, cudaStream_t st);
-size_t bf16_bwd_cluster_block_bytes(int T, int H);
-size_t bf16_fwd_cluster_block_bytes(int T, int H);
+size_t bf16_bwd_cluster_block_bytes(int T, int B, int H);
+size_t bf16_fwd_cluster_block_bytes(int T, int B, int H);
 cudaError_t bf16_launch_fwd_persist(stacklstm *s, const StepArgs &a, const CUtensorMap &tm_x, const CUtensorMap &tm_h,
                                     const CUtensorMap &tm_gates, const CUtensorMap &tm_hh,
                                     const CUtensorMap &tm_hc);

@@ -676,13 +676,13 @@ cudaError_t bf16_prepare(stacklstm *s)
     if ((e = cudaMalloc(&p, dx_bytes))) return e;
     s->allocs.push_back(p); s->w_dx = p;
     if (s->fc.on) {
-        if ((e = cudaMalloc(&p, bf16_fwd_cluster_block_bytes(T, H)))) return e;
+        if ((e = cudaMalloc(&p, bf16_fwd_cluster_block_bytes(T, B, H)))) return e;
         s->allocs.push_back(p); s->g_fcl = p;
     }
     if (s->bc.on) {
         if ((e = cudaMalloc(&p, bf16_bwd_cluster_weight_bytes(H)))) return e;
         s->allocs.push_back(p); s->w_bcl = p;
-        if ((e = cudaMalloc(&p, bf16_bwd_cluster_block_bytes(T, H)))) return e;
+        if ((e = cudaMalloc(&p, bf16_bwd_cluster_block_bytes(T, B, H)))) return e;
         s->allocs.push_back(p); s->g_bcl = p;
     }
     if (s->cc.on) {
@@ -841,7 +841,7 @@ bool bf16_can_group(stacklstm *const *hs, int n, bool fwd)
     for (int m = 0; m < n; ++m) {
         const stacklstm *s = hs[m];
         const PersistPlan &pl = fwd ? s->fc : s->bc;
-        if (s->dt != SL_BF16 || s->cc.on || !pl.on || pl.n_ct != (fwd ? hs[0]->fc : hs[0]->bc).n_ct ||
+        if (s->dt != SL_BF16 || s->cc.on || !pl.on || pl.slot != 1 || pl.n_ct != (fwd ? hs[0]->fc : hs[0]->bc).n_ct ||
             s->device != hs[0]->device)
             return false;
     }

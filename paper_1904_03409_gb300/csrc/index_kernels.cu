@@ -37,8 +37,14 @@ prepass_kernel(int T, int B, const int8_t *__restrict__ ops, int32_t *__restrict
     tag(0) = 0;
     for (int slot = 1; slot <= T; ++slot) tag(slot) = -1;
     int p = 0, e = SL_OK;
+    // the ops of 8 steps are loaded before they are used, so that the loads do not wait on
+    // one another
+    int8_t opq[8];
     for (int t = 0; t < T; ++t) {
-        int op = ops[(size_t)t * B + b];
+        if ((t & 7) == 0)
+#pragma unroll
+            for (int i = 0; i < 8; ++i) opq[i] = t + i < T ? ops[(size_t)(t + i) * B + b] : 0;
+        int op = opq[t & 7];
         if (op < -1 || op > 1) {  // recorded, then run as a hold so indices stay in range
             if (e == SL_OK) e = SL_ERR_OP;
             op = 0;
@@ -130,36 +136,52 @@ __global__ void __launch_bounds__(32) seed_grads_dy_kernel(int T, int B, int H, 
 // A step is a push when its pointer moves up by one (ops the prepass rejected ran as
 // holds). vslot is the stack of Sec. 2's definition: each slot's last pushed state.
 // kmax (zero on entry) receives the most pushes of any instance.
+template <bool kOnChip>
 __global__ void __launch_bounds__(kPrepassThreads)
 compact_kernel(int T, int B, const int32_t *__restrict__ p_traj, const int32_t *__restrict__ top,
-               int32_t *__restrict__ vtop, int32_t *__restrict__ vmap,
+               int32_t *__restrict__ vtop, int32_t *__restrict__ gvmap,
                int32_t *__restrict__ vy, int32_t *__restrict__ vslot, int32_t *__restrict__ xidx,
                int32_t *__restrict__ vstep, int32_t *__restrict__ kmax)
 {
-    const int b = blockIdx.x * kPrepassThreads + threadIdx.x;
+    extern __shared__ int32_t s_vmap[];
+    const int lane = threadIdx.x, b = blockIdx.x * kPrepassThreads + lane;
     if (b >= B) return;
-    // virtual index of the state at real history index j (written at step j - 1, or the
-    // initial state at j = 0); a state that is read is always a push write or the initial
-    // state, so the clamp never applies to valid prepass output
-    auto vof = [&](int j) { return max(0, vmap[(size_t)j * B + b]); };
-    vmap[b] = 0;
+    // vmap: the virtual index of the state at real history index j (written at step j - 1,
+    // or the initial state at j = 0), -1 for a non-push write; in shared memory when it fits
+    auto vmap = [&](int j) -> int32_t & {
+        return kOnChip ? s_vmap[j * kPrepassThreads + lane] : gvmap[(size_t)j * B + b];
+    };
+    // a state that is read is always a push write or the initial state, so the clamp never
+    // applies to valid prepass output
+    auto vof = [&](int j) { return max(0, vmap(j)); };
+    vmap(0) = 0;
     vslot[b] = 0;  // slot 0: the initial state
     for (int sl = 1; sl <= T; ++sl) vslot[(size_t)sl * B + b] = -1;
     int k = 0;
+    // the tops and pointers of 8 steps are loaded before they are used
+    int tq[8], pq[9];
     for (int t = 0; t < T; ++t) {
+        if ((t & 7) == 0) {
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+                tq[i] = t + i < T ? top[(size_t)(t + i) * B + b] : 0;
+                pq[i] = t + i <= T ? p_traj[(size_t)(t + i) * B + b] : 0;
+            }
+            pq[8] = t + 8 <= T ? p_traj[(size_t)(t + 8) * B + b] : 0;
+        }
         const size_t i = (size_t)t * B + b;
-        const int rd = vof(top[i]);
+        const int rd = vof(tq[t & 7]);
         vy[i] = rd;
-        if (p_traj[i + B] - p_traj[i] == 1) {
+        if (pq[(t & 7) + 1] - pq[t & 7] == 1) {
             xidx[(size_t)k * B + b] = t;
             vtop[(size_t)k * B + b] = rd;
             vstep[i] = k;
-            vmap[i + B] = k + 1;
-            vslot[(size_t)(p_traj[i] + 1) * B + b] = k + 1;
+            vmap(t + 1) = k + 1;
+            vslot[(size_t)(pq[t & 7] + 1) * B + b] = k + 1;
             ++k;
         } else {
             vstep[i] = -1;
-            vmap[i + B] = -1;
+            vmap(t + 1) = -1;
         }
     }
     vy[(size_t)T * B + b] = vof(top[(size_t)T * B + b]);
@@ -187,8 +209,18 @@ cudaError_t launch_compact(stacklstm *s)
 {
     cudaError_t e = cudaMemsetAsync(s->kmax, 0, sizeof(int32_t), s->stream);
     if (e) return e;
-    compact_kernel<<<ceil_div(s->B, kPrepassThreads), kPrepassThreads, 0, s->stream>>>(
-        s->T, s->B, s->p_traj, s->top, s->vtop, s->vmap, s->vy, s->vslot, s->xidx, s->vstep, s->kmax);
+    // the index table on chip when the prepass's slot-tag stack is (the same size)
+    const unsigned grid = ceil_div(s->B, kPrepassThreads);
+    if (s->prepass_smem > 0) {
+        if (s->prepass_smem > 48 * 1024 &&
+            (e = smem_at_least((const void *)compact_kernel<true>, (size_t)s->prepass_smem)))
+            return e;
+        compact_kernel<true><<<grid, kPrepassThreads, s->prepass_smem, s->stream>>>(
+            s->T, s->B, s->p_traj, s->top, s->vtop, s->vmap, s->vy, s->vslot, s->xidx, s->vstep, s->kmax);
+    } else {
+        compact_kernel<false><<<grid, kPrepassThreads, 0, s->stream>>>(
+            s->T, s->B, s->p_traj, s->top, s->vtop, s->vmap, s->vy, s->vslot, s->xidx, s->vstep, s->kmax);
+    }
     s->launches += 1;
     return cudaGetLastError();
 }

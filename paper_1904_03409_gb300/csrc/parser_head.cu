@@ -137,11 +137,27 @@ head_epi(int NR, int P, int A, const float *__restrict__ pre, const float *__res
         p_s[e] = r < nrow ? fmaxf(pre[(size_t)(row0 + r) * P + j] + dp[j], 0.0f) : 0.0f;
     }
     __syncthreads();
-    if (tid < kEpiRows * A) {
-        const int r = tid / A, o = tid % A;
-        float acc = q[o];
-        for (int j = 0; j < P; ++j) acc = fmaf(wz_s[o * P + j], p_s[r * P + j], acc);
-        z_s[r * 8 + o] = acc;
+    // z: warp w takes rows w, w + 8, ...; its lanes split the state columns, then a fixed
+    // butterfly sums the lanes
+    for (int r = tid >> 5; r < kEpiRows; r += kHeadThreads / 32) {
+        const int lane = tid & 31;
+        float acc[8];
+#pragma unroll
+        for (int o = 0; o < 8; ++o) acc[o] = 0.0f;
+        for (int j = lane; j < P; j += 32) {
+            const float pv = p_s[r * P + j];
+#pragma unroll
+            for (int o = 0; o < 8; ++o)
+                if (o < A) acc[o] = fmaf(wz_s[o * P + j], pv, acc[o]);
+        }
+#pragma unroll
+        for (int o = 0; o < 8; ++o) {
+            if (o >= A) break;
+            float v = acc[o];
+#pragma unroll
+            for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
+            if (lane == 0) z_s[r * 8 + o] = v + q[o];
+        }
     }
     __syncthreads();
     if (tid < kEpiRows) {
@@ -225,8 +241,15 @@ __global__ void head_reduce(const float *__restrict__ part, int S, size_t n0, si
 {
     const size_t n = n0 + n1 + n2;
     for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < n; i += (size_t)gridDim.x * blockDim.x) {
-        float acc = 0.0f;
-        for (int s = 0; s < S; ++s) acc += part[(size_t)s * n + i];
+        // four interleaved partial sums (part s goes to sum s mod 4), added in that order:
+        // a fixed order, with four independent chains of loads
+        float a4[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+        int s = 0;
+        for (; s + 4 <= S; s += 4)
+#pragma unroll
+            for (int k = 0; k < 4; ++k) a4[k] += part[(size_t)(s + k) * n + i];
+        for (; s < S; ++s) a4[s & 3] += part[(size_t)s * n + i];
+        const float acc = (a4[0] + a4[1]) + (a4[2] + a4[3]);
         if (i < n0)
             out0[i] = acc;
         else if (i < n0 + n1)

@@ -198,7 +198,7 @@ def test_grouped_calls_run_one_step_launch_and_match_oracle():
 
 @pytest.mark.gpu
 def test_grouped_calls_fall_back_when_the_members_differ():
-    """Handles that cannot share one launch (different hidden widths, a persistent plan)
+    """Handles that cannot share one launch (different hidden widths, several row tiles)
     still give the results of separate calls."""
     import torch
     from paper_1904_03409_gb300 import binding as bd

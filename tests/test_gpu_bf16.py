@@ -114,17 +114,27 @@ def test_stress_config_sampled():
     sampled_check(w, [0, 1, 127, 128, 2047, 3000, 4094, 4095])
 
 
-@pytest.mark.parametrize("B", [130, 40])
-def test_wait_timeout_is_reported_and_context_survives(B):
+PERSISTENT = {"STACKLSTM_FWD_CLUSTER": "0", "STACKLSTM_BWD_CLUSTER": "0"}
+
+
+@pytest.mark.parametrize("B,env", [(130, PERSISTENT), (40, {}), (130, {})])
+def test_wait_timeout_is_reported_and_context_survives(B, env):
     """With a zero wait budget the bounded device-side waits run out: forward (persistent
-    kernel at B = 130, thread-block cluster at B = 40) reports SL_ERR_TIMEOUT instead of
-    hanging, and the device stays usable."""
+    kernel at B = 130, thread-block clusters at B = 40 and at B = 130, three row tiles)
+    reports SL_ERR_TIMEOUT instead of hanging, and the device stays usable."""
     w = case(4, B, 16, 32, 9)
+    old = {k: os.environ.get(k) for k in env}
+    os.environ.update(env)
     os.environ["STACKLSTM_WAIT_LIMIT_CYCLES"] = "0"
     try:
         hd = bd.stacklstm_create(w.T, w.B, w.I, w.H, bd.SL_BF16, 0)
     finally:
         del os.environ["STACKLSTM_WAIT_LIMIT_CYCLES"]
+        for k, v in old.items():
+            if v is None:
+                os.environ.pop(k, None)
+            else:
+                os.environ[k] = v
     try:
         ins = runner.upload(w)
         out = runner.alloc_outputs(w)
@@ -157,6 +167,7 @@ def test_split_contraction_backward_matches_oracle(T, B, I, H, seed):
     of unequal length (H = 200: 13 chunks over 4 parts)."""
     w = case(T, B, I, H, seed, bias_scale=0.3, h0_scale=0.5, c0_scale=0.5, dy_scale=0.5)
     os.environ["STACKLSTM_BWD_SPLIT"] = "4"
+    os.environ.update(PERSISTENT)
     try:
         hd = bd.stacklstm_create(w.T, w.B, w.I, w.H, bd.SL_BF16, 0)
         plan = bd.stacklstm_plan(hd)
@@ -165,6 +176,8 @@ def test_split_contraction_backward_matches_oracle(T, B, I, H, seed):
         again = runner.run(w)
     finally:
         del os.environ["STACKLSTM_BWD_SPLIT"]
+        for k in PERSISTENT:
+            del os.environ[k]
     assert "backward persistent U=64" in plan and "contraction parts 4" in plan, plan
     compare(got, oracle_all(w), "bf16")
     for k in ("dx", "dW", "dbias", "dh0", "dc0"):
@@ -207,27 +220,29 @@ def test_input_gradient_on_spare_sms_matches_oracle(T, B, I, H, seed):
     matches the oracle and equals bit for bit the separate dx launch (same contraction
     chunk order). A single extra CTA, trailing the whole chain, too."""
     w = case(T, B, I, H, seed, bias_scale=0.3, h0_scale=0.5, c0_scale=0.5, dy_scale=0.5)
-    plan, got = run_nan_filled(w, {})
+    plan, got = run_nan_filled(w, dict(PERSISTENT))
     m = re.search(r"dx CTAs (\d+)", plan)
     assert m and int(m.group(1)) >= 4, plan
     compare(got, oracle_all(w), "bf16")
-    plan0, sep = run_nan_filled(w, {"STACKLSTM_DX_SPARE": "0"})
+    plan0, sep = run_nan_filled(w, dict(PERSISTENT, STACKLSTM_DX_SPARE="0"))
     assert "dx CTAs 0" in plan0, plan0
     assert np.array_equal(got["dx"], sep["dx"])
-    plan1, one = run_nan_filled(w, {"STACKLSTM_DX_SPARE": "1"})
+    plan1, one = run_nan_filled(w, dict(PERSISTENT, STACKLSTM_DX_SPARE="1"))
     assert "dx CTAs 1" in plan1, plan1
     assert np.array_equal(one["dx"], sep["dx"])
 
 
 @pytest.mark.parametrize("T,B,I,H,seed", [(17, 40, 8, 16, 19), (24, 64, 200, 200, 20), (9, 8, 64, 136, 21),
-                                         (12, 37, 24, 40, 22)])
-def test_cluster_kernels_for_one_row_tile_match_oracle(T, B, I, H, seed):
-    """One row tile (B <= 64): the forward and the backward as one thread-block cluster each,
-    their defaults, into NaN-filled outputs, match the oracle, as do the persistent kernels
-    they replace."""
+                                         (12, 37, 24, 40, 22), (14, 100, 24, 40, 23), (10, 200, 64, 136, 24),
+                                         (8, 450, 16, 32, 25)])
+def test_cluster_kernels_match_oracle(T, B, I, H, seed):
+    """Up to 8 row tiles of 64 instances: the forward and the backward as one thread-block
+    cluster per row tile, their defaults (a ragged last tile: B = 100, 200, 450), into
+    NaN-filled outputs, match the oracle, as do the persistent kernels they replace."""
     w = case(T, B, I, H, seed, bias_scale=0.3, h0_scale=0.5, c0_scale=0.5, dy_scale=0.5)
     plan, got = run_nan_filled(w, {})
     assert "forward cluster U=16" in plan and "backward cluster U=16" in plan, plan
+    assert "slots %d" % ((B + 63) // 64) in plan, plan
     ref = oracle_all(w)
     compare(got, ref, "bf16")
     plan_p, per = run_nan_filled(w, {"STACKLSTM_BWD_CLUSTER": "0", "STACKLSTM_FWD_CLUSTER": "0"})

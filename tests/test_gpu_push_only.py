@@ -24,6 +24,7 @@ from parity import compare
 pytestmark = pytest.mark.gpu
 NTHREADS = max(1, len(os.sched_getaffinity(0)))
 PUSH = bd.SL_MODE_PUSH_ONLY
+PERSISTENT = {"STACKLSTM_FWD_CLUSTER": "0", "STACKLSTM_BWD_CLUSTER": "0"}
 
 
 def definition(w, d_top_h=None, inst=None):
@@ -70,12 +71,13 @@ def check_against_homogenized(w, got, env=None):
 @pytest.mark.parametrize("T,B,I,H,seed,env", [
     (17, 40, 8, 16, 31, {}),                                  # one row tile: thread-block cluster kernels
     (24, 64, 200, 200, 32, {}),                               # parser widths, cluster kernels
-    (20, 200, 24, 40, 33, {}),                                # persistent kernels, ragged tiles
-    (30, 300, 136, 72, 34, {}),                               # three row tiles
-    (11, 200, 264, 64, 35, {}),                               # dx on the spare SMs of the backward launch
-    (12, 200, 64, 256, 36, {"STACKLSTM_BWD_SPLIT": "4"}),     # split-contraction backward
+    (20, 200, 24, 40, 33, {}),                                # clusters, four row tiles
+    (20, 200, 24, 40, 33, dict(PERSISTENT)),                  # persistent kernels, ragged tiles
+    (30, 300, 136, 72, 34, dict(PERSISTENT)),                 # three row tiles
+    (11, 200, 264, 64, 35, dict(PERSISTENT)),                 # dx on the spare SMs of the backward launch
+    (12, 200, 64, 256, 36, dict(PERSISTENT, STACKLSTM_BWD_SPLIT="4")),  # split-contraction backward
     (20, 200, 24, 40, 37, {"STACKLSTM_STEP_KERNELS": "1"}),   # one launch per step
-    (11, 200, 264, 64, 38, {"STACKLSTM_DX_SPARE": "0"}),      # dx in its own launch
+    (11, 200, 264, 64, 38, dict(PERSISTENT, STACKLSTM_DX_SPARE="0")),   # dx in its own launch
 ])
 def test_push_only_matches_definition_mode(T, B, I, H, seed, env):
     w = case(T, B, I, H, seed, bias_scale=0.3, h0_scale=0.5, c0_scale=0.5, dy_scale=0.5)
