@@ -153,6 +153,24 @@ sl_status fwd_begin(stacklstm *s, const sl_forward_args &a)
         if (p && !aligned16(p)) return fail(s, SL_ERR_ARG, "tensor pointers must be 16-byte aligned");
     cudaError_t e;
     s->fwd_done = 0;
+    // bf16, homogenized mode: the forward setup (weight packing, the initial state) does not
+    // depend on the index prepass, so it runs on the side stream at the same time; the
+    // caller's stream waits for it before the forward steps
+    const bool overlap = s->dt == SL_BF16 && !s->push_only;
+    if (overlap) {
+        if ((e = cudaEventRecord(s->aux_go, s->stream)) || (e = cudaStreamWaitEvent(s->side, s->aux_go, 0)))
+            return cuda_fail(s, e, "forward setup");
+        const cudaStream_t main = s->stream;
+        s->stream = s->side;
+        {
+            Phase ph(s, SL_PHASE_FWD_SETUP);
+            e = sl::bf16_forward_setup(s, (const __nv_bfloat16 *)a.x, (const __nv_bfloat16 *)a.h0, a.c0,
+                                       (const __nv_bfloat16 *)a.W);
+        }
+        s->stream = main;
+        if (e) return cuda_fail(s, e, "forward setup");
+        if ((e = cudaEventRecord(s->aux_done, s->side))) return cuda_fail(s, e, "forward setup");
+    }
     {
         Phase ph(s, SL_PHASE_PREPASS);
         if ((e = sl::launch_prepass(s, a.ops))) return cuda_fail(s, e, "prepass");
@@ -161,6 +179,10 @@ sl_status fwd_begin(stacklstm *s, const sl_forward_args &a)
         // kernels run is read back here (the one synchronization of this mode's forward)
         if (s->push_only && ((e = sl::launch_compact(s)) || (e = sl::read_virtual_steps(s))))
             return cuda_fail(s, e, "push-only indices");
+    }
+    if (overlap) {
+        if ((e = cudaStreamWaitEvent(s->stream, s->aux_done, 0))) return cuda_fail(s, e, "forward setup");
+        return SL_OK;
     }
     {
         Phase ph(s, SL_PHASE_FWD_SETUP);
@@ -273,7 +295,22 @@ sl_status bwd_end(stacklstm *s, const sl_backward_args &a, bool dx_done)
 {
     const int B = s->B, H = s->H;
     cudaError_t e;
-    if (!dx_done) {
+    // bf16: dx and dW both only read the gate gradients, so dx runs on the side stream at
+    // the same time as dW; the caller's stream waits for it
+    const bool side_dx = !dx_done && a.dx && s->dt == SL_BF16;
+    if (side_dx) {
+        if ((e = cudaEventRecord(s->aux_go, s->stream)) || (e = cudaStreamWaitEvent(s->side, s->aux_go, 0)))
+            return cuda_fail(s, e, "dx");
+        const cudaStream_t main = s->stream;
+        s->stream = s->side;
+        {
+            Phase ph(s, SL_PHASE_DX);
+            e = sl::bf16_dx(s, a.dx);
+        }
+        s->stream = main;
+        if (e) return cuda_fail(s, e, "dx");
+        if ((e = cudaEventRecord(s->aux_done, s->side))) return cuda_fail(s, e, "dx");
+    } else if (!dx_done) {
         Phase ph(s, SL_PHASE_DX);
         e = s->dt == SL_FP32 ? sl::fp32_dx(s, a.dx) : sl::bf16_dx(s, a.dx);
         if (e) return cuda_fail(s, e, "dx");
@@ -283,6 +320,7 @@ sl_status bwd_end(stacklstm *s, const sl_backward_args &a, bool dx_done)
         e = s->dt == SL_FP32 ? sl::fp32_dw(s, a.dW, a.dbias) : sl::bf16_dw(s, a.dW, a.dbias);
         if (e) return cuda_fail(s, e, "dW");
     }
+    if (side_dx && (e = cudaStreamWaitEvent(s->stream, s->aux_done, 0))) return cuda_fail(s, e, "dx");
     // slot 0 always holds the initial state, which is history row 0
     if (a.dh0 && (e = cudaMemcpyAsync(a.dh0, s->dhist_h, sizeof(float) * B * H, cudaMemcpyDeviceToDevice, s->stream)))
         return cuda_fail(s, e, "dh0");
@@ -384,12 +422,16 @@ sl_status stacklstm_create(stacklstm_t *out, int T, int B, int I, int H, sl_dtyp
     if (ok) ok = cudaStreamCreateWithFlags(&s->side, cudaStreamNonBlocking) == cudaSuccess &&
                  cudaEventCreateWithFlags(&s->side_go, cudaEventDisableTiming) == cudaSuccess &&
                  cudaEventCreateWithFlags(&s->cleared, cudaEventDisableTiming) == cudaSuccess &&
-                 cudaEventCreateWithFlags(&s->join, cudaEventDisableTiming) == cudaSuccess;
+                 cudaEventCreateWithFlags(&s->join, cudaEventDisableTiming) == cudaSuccess &&
+                 cudaEventCreateWithFlags(&s->aux_go, cudaEventDisableTiming) == cudaSuccess &&
+                 cudaEventCreateWithFlags(&s->aux_done, cudaEventDisableTiming) == cudaSuccess;
     if (!ok) {
         if (s->side) cudaStreamDestroy(s->side);
         if (s->side_go) cudaEventDestroy(s->side_go);
         if (s->cleared) cudaEventDestroy(s->cleared);
         if (s->join) cudaEventDestroy(s->join);
+        if (s->aux_go) cudaEventDestroy(s->aux_go);
+        if (s->aux_done) cudaEventDestroy(s->aux_done);
         cudaGetLastError();
         free_all(s);
         delete s;
@@ -590,6 +632,8 @@ sl_status stacklstm_destroy(stacklstm_t s)
         if (s->side_go) cudaEventDestroy(s->side_go);
         if (s->cleared) cudaEventDestroy(s->cleared);
         if (s->join) cudaEventDestroy(s->join);
+        if (s->aux_go) cudaEventDestroy(s->aux_go);
+        if (s->aux_done) cudaEventDestroy(s->aux_done);
         collect_timing(s);
         for (cudaEvent_t ev : s->event_pool) cudaEventDestroy(ev);
         s->event_pool.clear();

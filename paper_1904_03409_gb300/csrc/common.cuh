@@ -44,6 +44,9 @@ struct stacklstm {
     cudaStream_t side = nullptr;
     cudaEvent_t side_go = nullptr, cleared = nullptr;
     cudaEvent_t join = nullptr;  // grouped calls: marks this handle's stream for the others
+    // work overlapped on the side stream (the forward setup beside the prepass, dx beside
+    // dW): `aux_go` marks the caller's stream before it, `aux_done` its end
+    cudaEvent_t aux_go = nullptr, aux_done = nullptr;
     int clear_queued = 0;
     int async = 0;
     int fwd_done = 0;
