@@ -153,10 +153,10 @@ sl_status fwd_begin(stacklstm *s, const sl_forward_args &a)
         if (p && !aligned16(p)) return fail(s, SL_ERR_ARG, "tensor pointers must be 16-byte aligned");
     cudaError_t e;
     s->fwd_done = 0;
-    // bf16, homogenized mode: the forward setup (weight packing, the initial state) does not
-    // depend on the index prepass, so it runs on the side stream at the same time; the
-    // caller's stream waits for it before the forward steps
-    const bool overlap = s->dt == SL_BF16 && !s->push_only;
+    // bf16: the initial state and the weight packing do not depend on the index prepass, so
+    // they run on the side stream at the same time; the caller's stream waits for them
+    // before the forward steps
+    const bool overlap = s->dt == SL_BF16;
     if (overlap) {
         if ((e = cudaEventRecord(s->aux_go, s->stream)) || (e = cudaStreamWaitEvent(s->side, s->aux_go, 0)))
             return cuda_fail(s, e, "forward setup");
@@ -164,8 +164,7 @@ sl_status fwd_begin(stacklstm *s, const sl_forward_args &a)
         s->stream = s->side;
         {
             Phase ph(s, SL_PHASE_FWD_SETUP);
-            e = sl::bf16_forward_setup(s, (const __nv_bfloat16 *)a.x, (const __nv_bfloat16 *)a.h0, a.c0,
-                                       (const __nv_bfloat16 *)a.W);
+            e = sl::bf16_forward_setup_state(s, (const __nv_bfloat16 *)a.h0, a.c0, (const __nv_bfloat16 *)a.W);
         }
         s->stream = main;
         if (e) return cuda_fail(s, e, "forward setup");
@@ -180,19 +179,16 @@ sl_status fwd_begin(stacklstm *s, const sl_forward_args &a)
         if (s->push_only && ((e = sl::launch_compact(s)) || (e = sl::read_virtual_steps(s))))
             return cuda_fail(s, e, "push-only indices");
     }
-    if (overlap) {
-        if ((e = cudaStreamWaitEvent(s->stream, s->aux_done, 0))) return cuda_fail(s, e, "forward setup");
-        return SL_OK;
-    }
     {
         Phase ph(s, SL_PHASE_FWD_SETUP);
-        if (s->dt == SL_FP32)
-            e = sl::fp32_forward_setup(s, (const float *)a.h0, a.c0, (const float *)a.W);
+        // push-only mode: the virtual steps' inputs, gathered after the compaction
+        if (overlap)
+            e = sl::bf16_forward_setup_x(s, (const __nv_bfloat16 *)a.x);
         else
-            e = sl::bf16_forward_setup(s, (const __nv_bfloat16 *)a.x, (const __nv_bfloat16 *)a.h0, a.c0,
-                                       (const __nv_bfloat16 *)a.W);
+            e = sl::fp32_forward_setup(s, (const float *)a.h0, a.c0, (const float *)a.W);
         if (e) return cuda_fail(s, e, "forward setup");
     }
+    if (overlap && (e = cudaStreamWaitEvent(s->stream, s->aux_done, 0))) return cuda_fail(s, e, "forward setup");
     return SL_OK;
 }
 
@@ -201,7 +197,8 @@ sl_status fwd_begin(stacklstm *s, const sl_forward_args &a)
 // recorded on the caller's stream before the forward steps (a previous backward reads it).
 sl_status fwd_clear(stacklstm *s)
 {
-    const size_t hist_bytes = sizeof(float) * (size_t)(s->T + 1) * s->B * s->H;
+    // the rows the kernels use: T + 1, or in push-only mode the virtual steps' Tr + 1
+    const size_t hist_bytes = sizeof(float) * (size_t)(s->Tr + 1) * s->B * s->H;
     cudaError_t e;
     if ((e = cudaStreamWaitEvent(s->side, s->side_go, 0)) ||
         (e = cudaMemsetAsync(s->dhist_h, 0, hist_bytes, s->side)) ||
@@ -264,7 +261,8 @@ sl_status bwd_begin(stacklstm *s, const sl_backward_args &a)
     const void *ptrs[] = {a.d_top_h, a.dy, a.dx, a.dh0, a.dc0, a.dW, a.dbias};
     for (const void *p : ptrs)
         if (p && !aligned16(p)) return fail(s, SL_ERR_ARG, "tensor pointers must be 16-byte aligned");
-    const size_t hist_bytes = sizeof(float) * (size_t)(s->T + 1) * s->B * s->H;
+    // the rows the kernels use: T + 1, or in push-only mode the virtual steps' Tr + 1
+    const size_t hist_bytes = sizeof(float) * (size_t)(s->Tr + 1) * s->B * s->H;
     cudaError_t e;
     Phase ph(s, SL_PHASE_BWD_SETUP);
     if (s->clear_queued) {
@@ -278,7 +276,8 @@ sl_status bwd_begin(stacklstm *s, const sl_backward_args &a)
     if ((e = sl::launch_seed_grads(s, a.d_top_h, a.dy))) return cuda_fail(s, e, "seed");
     if (s->dt == SL_BF16 && (e = sl::bf16_backward_setup(s))) return cuda_fail(s, e, "backward setup");
     // push-only mode: the dx rows of steps that do not push are zero; the contraction
-    // writes the others
+    // writes the others. (Zeroing them on the side stream during the step launch slowed
+    // the weight gradient that follows by twice the zeroing's own time.)
     if (s->push_only && (e = sl::launch_zero_nonpush_rows(s, a.dx))) return cuda_fail(s, e, "dx rows");
     return SL_OK;
 }

@@ -722,10 +722,9 @@ cudaError_t bf16_prepare(stacklstm *s)
     return cudaSuccess;
 }
 
-cudaError_t bf16_forward_setup(stacklstm *s, const __nv_bfloat16 *x, const __nv_bfloat16 *h0, const float *c0,
-                               const __nv_bfloat16 *W)
+cudaError_t bf16_forward_setup_x(stacklstm *s, const __nv_bfloat16 *x)
 {
-    const int T = s->T, B = s->B, I = s->I, H = s->H;
+    const int T = s->T, B = s->B, I = s->I;
     cudaError_t e;
     if (s->push_only) {
         // the forward and the weight gradient read the inputs of the virtual steps
@@ -734,7 +733,13 @@ cudaError_t bf16_forward_setup(stacklstm *s, const __nv_bfloat16 *x, const __nv_
     }
     s->x_saved = x;
     if ((e = make_map(s->tmaps[kMapX128], x, (uint64_t)T * B, I, kRows))) return e;
-    if ((e = make_map(s->tmaps[kMapX64], x, (uint64_t)T * B, I, kChunk))) return e;
+    return make_map(s->tmaps[kMapX64], x, (uint64_t)T * B, I, kChunk);
+}
+
+cudaError_t bf16_forward_setup_state(stacklstm *s, const __nv_bfloat16 *h0, const float *c0, const __nv_bfloat16 *W)
+{
+    const int B = s->B, I = s->I, H = s->H;
+    cudaError_t e;
     if ((e = cudaMemcpyAsync(s->hist_h, h0, sizeof(__nv_bfloat16) * B * H, cudaMemcpyDeviceToDevice, s->stream)))
         return e;
     if ((e = cudaMemcpyAsync(s->hr, h0, sizeof(__nv_bfloat16) * B * H, cudaMemcpyDeviceToDevice, s->stream)))

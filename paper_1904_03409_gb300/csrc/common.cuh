@@ -163,8 +163,10 @@ cudaError_t fp32_dw(stacklstm *s, float *dW, float *dbias);
 
 // ---- bf16 tensor-core path (bf16_path.cu)
 cudaError_t bf16_prepare(stacklstm *s);
-cudaError_t bf16_forward_setup(stacklstm *s, const __nv_bfloat16 *x, const __nv_bfloat16 *h0,
-                               const float *c0, const __nv_bfloat16 *W);
+// the forward's inputs: the virtual steps' x gathered (push-only mode), the x tensor maps
+cudaError_t bf16_forward_setup_x(stacklstm *s, const __nv_bfloat16 *x);
+// the initial state into history row 0, the weight tiles packed (needs no index)
+cudaError_t bf16_forward_setup_state(stacklstm *s, const __nv_bfloat16 *h0, const float *c0, const __nv_bfloat16 *W);
 cudaError_t bf16_forward_steps(stacklstm *s, const float *bias);
 cudaError_t bf16_backward_setup(stacklstm *s);
 cudaError_t bf16_backward_steps(stacklstm *s, float *dx, bool *dx_done);
