@@ -65,7 +65,12 @@ constexpr uint32_t kBarBytes = (2 * kMaxStages + 6) * 8 + 16;
 // staged for the tensor stores that write it out: the activated gates (4 gates x 128 rows
 // x U units, fp16), then h' (128 x U, bf16), then c' (128 x U, fp32); each block is laid
 // out [unit part][row][units of the part]
-__host__ __device__ constexpr uint32_t ws_stg_bytes(bool fwd, int U) { return fwd ? 128u * U * (8 + 2 + 4) : 0u; }
+// backward with 32-unit tiles: the accumulator rows pass through a [128 rows][32 units]
+// fp32 tile on their way from one row per lane to four lanes per row (epilogue_loop)
+__host__ __device__ constexpr uint32_t ws_stg_bytes(bool fwd, int U)
+{
+    return fwd ? 128u * U * (8 + 2 + 4) : U == 32 ? 128u * 32 * 4 : 0u;
+}
 
 __host__ __device__ constexpr uint32_t ws_stage_bytes(int G, int NB, int w_res)
 {
@@ -200,6 +205,10 @@ __device__ __forceinline__ void ld_v4(const void *p, uint32_t *w)
     const uint4 v = __ldcg((const uint4 *)p);
     w[0] = v.x; w[1] = v.y; w[2] = v.z; w[3] = v.w;
 }
+__device__ __forceinline__ void ld_shared_v4(uint32_t addr, uint32_t *w)
+{
+    asm volatile("ld.shared.v4.b32 {%0,%1,%2,%3}, [%4];" : "=r"(w[0]), "=r"(w[1]), "=r"(w[2]), "=r"(w[3]) : "r"(addr));
+}
 // NG 16-bit values (raw words, NG / 2 of them)
 template <int NG>
 __device__ __forceinline__ void st_h(void *p, const uint32_t *w)
@@ -329,6 +338,8 @@ __device__ __forceinline__ void epilogue_loop(const StepArgs &a, const WsArgs &p
     int cur0 = 0, cur1 = 0;
     if (e.n_tiles > 0) tile_rows(0, cur0, cur1);
     constexpr bool kLatePfBwd = UE > 16;  // backward: operands taken group by group (below)
+    // backward, 32 units a thread, unsplit contraction: four lanes per row (below)
+    constexpr bool kRows4 = !kFwd && KS == 1 && EP == 1 && UE == 32 && defer_dhist<EP>();
     for (int k = 0; k < e.n_tiles; ++k) {
         const int ks = k / e.n_mine, rt = e.slot + (k % e.n_mine) * p.n_slot;
         const int t = kFwd ? ks : T - 1 - ks;
@@ -377,6 +388,9 @@ __device__ __forceinline__ void epilogue_loop(const StepArgs &a, const WsArgs &p
         constexpr bool kDeferDhist = !kFwd && defer_dhist<EP>();
         float dfh[kDeferDhist ? UE : 1], dfc[kDeferDhist ? UE : 1];
         int d_src = 0, d_s1 = 0;
+        // four lanes per row (below): the rows' history indices, by round
+        int r_src[kRows4 ? 4 : 1], r_s1[kRows4 ? 4 : 1];
+        bool r_ok[kRows4 ? 4 : 1];
         if constexpr (kFwd) {
             // operands this thread wrote itself at earlier steps (same rows and units):
             // c_read, and the older top the next step reads when step t does not push
@@ -478,6 +492,106 @@ __device__ __forceinline__ void epilogue_loop(const StepArgs &a, const WsArgs &p
 #pragma unroll
                     for (int i = 0; i < NG / 8; ++i)
                         tc::st_shared_v4(tile + stg_swz<UE * 2>(srow, cg * NG / 8 + i), gw + 4 * i);
+                }
+            }
+        } else if constexpr (kRows4) {
+            // Four lanes per row. The accumulator comes out of tensor memory one row per lane
+            // (lane = row); each row's 32 values go through a shared-memory tile so that in
+            // round j lane l takes row 8 j + l / 4 of the warp's 32, units 8 (l % 4) .. + 7.
+            // Every global access of a round then covers eight rows with four lanes on each
+            // row's 128-byte line, a quarter of the L1 wavefronts of one row per lane. The
+            // history indices of a round's row come from the lane that loaded them.
+            const uint32_t xb = e.c.stg + (uint32_t)e.q * 4096u;  // this warp's 32 rows x 128 B
+            const int sub = e.lane & 3, us = u0 + 8 * sub;
+            float dr[4][8];
+            const bool ok = tc::mbar_wait(&e.c.tfull[acc], (k >> 1) & 1, e.limit, e.c.abort);
+            if (!ok) ws_abort(e.c, a.err);
+            __syncwarp();
+            if (tc::bar_any(1, E * 32, !ok || *e.c.abort)) break;
+            tc::tc_fence_after();
+            {
+                uint32_t v[UE];
+                tmem_cols<UE>(taddr, v);
+                tc::tmem_wait_ld();
+                tc::tc_fence_before();
+                __syncwarp();
+                if (e.lane == 0) tc::mbar_arrive(&e.c.tempty[acc]);
+                // row = lane, 16-byte piece i at piece i ^ (row mod 8): conflict-free both ways
+#pragma unroll
+                for (int i = 0; i < 8; ++i)
+                    tc::st_shared_v4(xb + (uint32_t)e.lane * 128u + (uint32_t)((i ^ (e.lane & 7)) * 16), v + 4 * i);
+            }
+            __syncwarp();
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                const int rr = 8 * j + (e.lane >> 2);
+                r_src[j] = __shfl_sync(0xffffffffu, cur0, rr);
+                r_s1[j] = __shfl_sync(0xffffffffu, cur1, rr);
+                r_ok[j] = rt * kRows + e.q * 32 + rr < B && us < H;
+                uint32_t w[8];
+                ld_shared_v4(xb + (uint32_t)rr * 128u + (uint32_t)(((2 * sub) ^ (rr & 7)) * 16), w);
+                ld_shared_v4(xb + (uint32_t)rr * 128u + (uint32_t)(((2 * sub + 1) ^ (rr & 7)) * 16), w + 4);
+#pragma unroll
+                for (int i = 0; i < 8; ++i) dr[j][i] = __uint_as_float(w[i]);
+            }
+            // two rounds' operands in flight at a time
+#pragma unroll
+            for (int jp = 0; jp < 4; jp += 2) {
+                float dh_src[2][8], dh_t[2][8], dc_t[2][8], cn[2][8], cr[2][8], dc_rd[2][8];
+                uint32_t gq[2][4][4];
+#pragma unroll
+                for (int h = 0; h < 2; ++h) {
+                    const int j = jp + h;
+                    if (!r_ok[j]) continue;
+                    const int bj = rt * kRows + e.q * 32 + 8 * j + (e.lane >> 2);
+                    ld_f<8>(a.dhist_h + ((size_t)r_src[j] * B + bj) * H + us, dh_src[h]);
+                    if (t >= 1) {
+                        const size_t wr = ((size_t)t * B + bj) * H + us, rd = ((size_t)r_s1[j] * B + bj) * H + us;
+                        ld_f<8>(a.dhist_h + wr, dh_t[h]);
+                        ld_f<8>(a.dhist_c + wr, dc_t[h]);
+                        ld_f<8>(a.hist_c + wr, cn[h]);
+                        ld_f<8>(a.hist_c + rd, cr[h]);
+                        ld_f<8>(a.dhist_c + rd, dc_rd[h]);
+                        const __half *gt = a.gates + ((size_t)(t - 1) * B + bj) * 4 * H + us;
+#pragma unroll
+                        for (int g = 0; g < 4; ++g) ld_v4(gt + (size_t)g * H, gq[h][g]);
+                    }
+                }
+#pragma unroll
+                for (int h = 0; h < 2; ++h) {
+                    const int j = jp + h;
+                    if (!r_ok[j]) continue;
+                    float v[8];
+#pragma unroll
+                    for (int i = 0; i < 8; ++i) v[i] = dh_src[h][i] + dr[j][i];
+#pragma unroll
+                    for (int i = 0; i < 8; ++i) dfh[8 * j + i] = v[i];
+                    if (t >= 1) {
+                        const int bj = rt * kRows + e.q * 32 + 8 * j + (e.lane >> 2);
+                        float ig[8], fg[8], gg[8], og[8], d[4][8];
+                        unpack_f16<8>(gq[h][0], ig);
+                        unpack_f16<8>(gq[h][1], fg);
+                        unpack_f16<8>(gq[h][2], gg);
+                        unpack_f16<8>(gq[h][3], og);
+#pragma unroll
+                        for (int i = 0; i < 8; ++i) {
+                            const float dh = r_src[j] == t ? v[i] : dh_t[h][i];  // the state read at t is row t
+                            const float tcn = tanh_hw(cn[h][i]);
+                            const float dc = dc_t[h][i] + dh * og[i] * (1.0f - tcn * tcn);
+                            d[0][i] = dc * gg[i] * ig[i] * (1.0f - ig[i]);
+                            d[1][i] = dc * cr[h][i] * fg[i] * (1.0f - fg[i]);
+                            d[2][i] = dc * ig[i] * (1.0f - gg[i] * gg[i]);
+                            d[3][i] = dh * tcn * og[i] * (1.0f - og[i]);
+                            dfc[8 * j + i] = dc_rd[h][i] + dc * fg[i];
+                        }
+                        __nv_bfloat16 *dg = a.dG + ((size_t)(t - 1) * B + bj) * 4 * H + us;
+#pragma unroll
+                        for (int g = 0; g < 4; ++g) {
+                            uint32_t w[4];
+                            pack_bf16<8>(d[g], w);
+                            st_v4(dg + (size_t)g * H, w);
+                        }
+                    }
                 }
             }
         } else {
@@ -624,7 +738,16 @@ __device__ __forceinline__ void epilogue_loop(const StepArgs &a, const WsArgs &p
         __syncwarp();
         tc::bar_sync(2, E * 32);
         if (e.tid == 0) tc::red_release_gpu_add(p.cnt + rt * p.cs, 1);
-        if constexpr (kDeferDhist) {
+        if constexpr (kRows4) {
+            const int sub = e.lane & 3, us = u0 + 8 * sub;
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                if (!r_ok[j]) continue;
+                const int bj = rt * kRows + e.q * 32 + 8 * j + (e.lane >> 2);
+                st_f<8>(a.dhist_h + ((size_t)r_src[j] * B + bj) * H + us, dfh + 8 * j);
+                if (t >= 1) st_f<8>(a.dhist_c + ((size_t)r_s1[j] * B + bj) * H + us, dfc + 8 * j);
+            }
+        } else if constexpr (kDeferDhist) {
             if (row_ok) {
 #pragma unroll
                 for (int cg = 0; cg < UE / NG; ++cg) {

@@ -114,6 +114,25 @@ def test_stress_config_sampled():
     sampled_check(w, [0, 1, 127, 128, 2047, 3000, 4094, 4095])
 
 
+@pytest.mark.parametrize("T,B,I,H,seed", [(16, 4096, 256, 256, 26), (16, 4000, 256, 248, 27)])
+def test_four_lanes_per_row_backward_epilogue(T, B, I, H, seed):
+    """The persistent backward with 32-unit column tiles and one epilogue warp group takes
+    each row's units four lanes at a time, after a shared-memory transpose of the
+    accumulator rows. The stress shape, and a ragged one (B = 4000: the last row tile a
+    quarter full; H = 248: the last column tile 24 units); the oracle on instances at
+    every warp, round and lane position of a row tile, in three row tiles."""
+    w = case(T, B, I, H, seed, probs=(0.6, 0.3, 0.1), bias_scale=0.3, h0_scale=0.5, c0_scale=0.5)
+    hd = bd.stacklstm_create(w.T, w.B, w.I, w.H, bd.SL_BF16, 0)
+    try:
+        plan = bd.stacklstm_plan(hd)
+    finally:
+        hd.destroy()
+    assert "backward persistent U=32 [EP 1" in plan and "contraction parts 1" in plan, plan
+    last = (B - 1) // 128 * 128
+    inst = sorted({base + r for base in (0, 17 * 128, last) for r in range(0, 128, 9) if base + r < B} | {B - 1})
+    sampled_check(w, inst)
+
+
 PERSISTENT = {"STACKLSTM_FWD_CLUSTER": "0", "STACKLSTM_BWD_CLUSTER": "0"}
 
 
