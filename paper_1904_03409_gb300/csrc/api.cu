@@ -154,12 +154,20 @@ sl_status fwd_begin(stacklstm *s, const sl_forward_args &a)
     cudaError_t e;
     s->fwd_done = 0;
     // bf16: the initial state and the weight packing do not depend on the index prepass, so
-    // they run on the side stream at the same time; the caller's stream waits for them
-    // before the forward steps
+    // they run on the side stream at the same time (launched after the prepass, whose few
+    // blocks then reach the SMs first); the caller's stream waits for them before the
+    // forward steps
     const bool overlap = s->dt == SL_BF16;
+    if (overlap && (e = cudaEventRecord(s->aux_go, s->stream))) return cuda_fail(s, e, "forward setup");
+    {
+        Phase ph(s, SL_PHASE_PREPASS);
+        if ((e = sl::launch_prepass(s, a.ops))) return cuda_fail(s, e, "prepass");
+        s->Tr = s->T;
+        // push-only mode: each instance's pushes as a virtual timeline
+        if (s->push_only && (e = sl::launch_compact(s))) return cuda_fail(s, e, "push-only indices");
+    }
     if (overlap) {
-        if ((e = cudaEventRecord(s->aux_go, s->stream)) || (e = cudaStreamWaitEvent(s->side, s->aux_go, 0)))
-            return cuda_fail(s, e, "forward setup");
+        if ((e = cudaStreamWaitEvent(s->side, s->aux_go, 0))) return cuda_fail(s, e, "forward setup");
         const cudaStream_t main = s->stream;
         s->stream = s->side;
         {
@@ -170,14 +178,11 @@ sl_status fwd_begin(stacklstm *s, const sl_forward_args &a)
         if (e) return cuda_fail(s, e, "forward setup");
         if ((e = cudaEventRecord(s->aux_done, s->side))) return cuda_fail(s, e, "forward setup");
     }
-    {
+    if (s->push_only) {
+        // the step count the kernels run is read back here (the one synchronization of this
+        // mode's forward)
         Phase ph(s, SL_PHASE_PREPASS);
-        if ((e = sl::launch_prepass(s, a.ops))) return cuda_fail(s, e, "prepass");
-        s->Tr = s->T;
-        // push-only mode: each instance's pushes as a virtual timeline; the step count the
-        // kernels run is read back here (the one synchronization of this mode's forward)
-        if (s->push_only && ((e = sl::launch_compact(s)) || (e = sl::read_virtual_steps(s))))
-            return cuda_fail(s, e, "push-only indices");
+        if ((e = sl::read_virtual_steps(s))) return cuda_fail(s, e, "push-only indices");
     }
     {
         Phase ph(s, SL_PHASE_FWD_SETUP);

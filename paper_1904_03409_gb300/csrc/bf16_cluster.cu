@@ -452,7 +452,7 @@ constexpr int kClMaxTiles = 8;  // row tiles (clusters) of one launch
 // them, each into its own accumulator.
 //
 // [weight chunks n_ct x 2 KB][dG buffer n_ct x 8 KB][barriers]
-constexpr uint32_t kWChunkB = 16 * 128;  // one weight chunk: 16 rows x 64 K
+// (kWChunkB, one weight chunk of 16 rows x 64 K, and its packing: bf16_dev.cuh)
 constexpr uint32_t kGBlock = 64 * 128;   // one CTA's dG block: 64 rows x 64 K
 __host__ __device__ constexpr uint32_t clb_smem_bytes(int n_ct)
 {
@@ -487,23 +487,6 @@ __device__ __forceinline__ ClbCtl clb_carve(uint8_t *raw, int n_ct)
 }
 
 }  // namespace
-
-// Weight chunks of the cluster backward: for CTA ct, chunk j, the 16 x 64 block
-// B[n][16 g + e] = W[I + 16 ct + n][g H + 16 j + e] (zero past H), 128-byte swizzled rows;
-// out is [n_ct][n_ct chunks][16 rows][64].
-__global__ void pack_bwd_slices(const __nv_bfloat16 *__restrict__ W, int I, int H, int n_ct,
-                                __nv_bfloat16 *__restrict__ out)
-{
-    const size_t n = (size_t)n_ct * n_ct * 16 * 64;
-    for (size_t e = blockIdx.x * (size_t)blockDim.x + threadIdx.x; e < n; e += (size_t)gridDim.x * blockDim.x) {
-        const int kk = (int)(e % 64), nn = (int)((e / 64) % 16);
-        const int blk = (int)(e / (64 * 16)), j = blk % n_ct, ct = blk / n_ct;
-        const int g = kk / 16, unit = 16 * ct + nn, ku = 16 * j + kk % 16;
-        const __nv_bfloat16 v = (unit < H && ku < H) ? W[(size_t)(I + unit) * 4 * H + g * H + ku] : __float2bfloat16(0.0f);
-        const uint32_t byte = sw128((uint32_t)nn, (uint32_t)kk >> 3) + (uint32_t)(kk & 7) * 2;
-        out[((size_t)blk * kWChunkB + byte) / 2] = v;
-    }
-}
 
 namespace {
 // This thread's row of a dG block (4 gates x 16 units, zero past H or B) into the swizzled
@@ -962,15 +945,6 @@ size_t bf16_bwd_cluster_weight_bytes(int H)
 {
     const size_t n_ct = ceil_div(H, kClU);
     return n_ct * n_ct * kWChunkB;
-}
-
-cudaError_t bf16_pack_bwd_cluster(stacklstm *s, const __nv_bfloat16 *W, __nv_bfloat16 *out)
-{
-    const int n_ct = s->bc.n_ct;
-    const size_t n = (size_t)n_ct * n_ct * 16 * 64;
-    pack_bwd_slices<<<(unsigned)std::min<size_t>((n + 255) / 256, 4096), 256, 0, s->stream>>>(W, s->I, s->H, n_ct, out);
-    s->launches += 1;
-    return cudaGetLastError();
 }
 
 cudaError_t bf16_launch_bwd_cluster(stacklstm *s, const StepArgs &a)

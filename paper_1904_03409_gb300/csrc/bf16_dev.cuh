@@ -22,6 +22,66 @@ constexpr uint32_t kAStage = kRows * 128;
 constexpr int kMaxStages = 16;
 constexpr long long kDrainLimit = 4000000000LL;  // wait for own copies / MMAs before exit
 
+// ---- weight packing (one output element each; the forward setup runs all of them in one
+// launch, bf16_path.cu)
+// Forward operand: for column tile ct, rows n = g * U + j hold gate g of hidden unit
+// ct * U + j; each row is the matching column of W over the contraction
+// [x padded to 64 ; h padded to 64], in 64-element chunks of 128-byte swizzled rows.
+// Element e of [n_ct][KC][4U rows][64].
+__device__ __forceinline__ void pack_gate_cols_elem(size_t e, const __nv_bfloat16 *__restrict__ W, int I, int H, int U,
+                                                    int kcx, int KC, __nv_bfloat16 *__restrict__ out)
+{
+    const int NB = 4 * U, G = 4 * H;
+    const int col = (int)(e % kChunk);
+    const size_t rowi = e / kChunk;  // (ct * KC + kc) * NB + row
+    const int row = (int)(rowi % NB);
+    const size_t tile = rowi / NB;
+    const int kc = (int)(tile % KC), ct = (int)(tile / KC);
+    const int g = row / U, unit = ct * U + row % U;
+    int wrow = -1;
+    if (kc < kcx) {
+        const int k = kc * kChunk + col;
+        if (k < I) wrow = k;
+    } else {
+        const int k = (kc - kcx) * kChunk + col;
+        if (k < H) wrow = I + k;
+    }
+    const __nv_bfloat16 v = (unit < H && wrow >= 0) ? W[(size_t)wrow * G + g * H + unit] : __float2bfloat16(0.0f);
+    const size_t byte = tile * NB * 128 + sw128(row, col >> 3) + (col & 7) * 2;
+    out[byte / 2] = v;
+}
+// Backward operands: for column tile ct, row m is W row (row0 + ct * NB + m) over the 4H
+// gate columns (zero padded): W_h rows (row0 = I, rows < I + H) for dh_read, W_x rows
+// (row0 = 0, rows < I) for dx. Element e of [n_ct][KC][NB rows][64].
+__device__ __forceinline__ void pack_w_rows_elem(size_t e, const __nv_bfloat16 *__restrict__ W, int H, int row0,
+                                                 int nrows, int NB, int KC, __nv_bfloat16 *__restrict__ out)
+{
+    const int G = 4 * H;
+    const int col = (int)(e % kChunk);
+    const size_t rowi = e / kChunk;
+    const int row = (int)(rowi % NB);
+    const size_t tile = rowi / NB;
+    const int kc = (int)(tile % KC), ct = (int)(tile / KC);
+    const int m = ct * NB + row, k = kc * kChunk + col;
+    const __nv_bfloat16 v = (m < nrows && k < G) ? W[(size_t)(row0 + m) * G + k] : __float2bfloat16(0.0f);
+    const size_t byte = tile * NB * 128 + sw128(row, col >> 3) + (col & 7) * 2;
+    out[byte / 2] = v;
+}
+// Weight chunks of the cluster backward (bf16_cluster.cu): for CTA ct, chunk j, the 16 x 64
+// block B[n][16 g + e] = W[I + 16 ct + n][g H + 16 j + e] (zero past H), 128-byte swizzled
+// rows. Element e of [n_ct][n_ct chunks][16 rows][64].
+constexpr uint32_t kWChunkB = 16 * 128;  // one weight chunk: 16 rows x 64 K
+__device__ __forceinline__ void pack_bwd_slice_elem(size_t e, const __nv_bfloat16 *__restrict__ W, int I, int H,
+                                                    int n_ct, __nv_bfloat16 *__restrict__ out)
+{
+    const int kk = (int)(e % 64), nn = (int)((e / 64) % 16);
+    const int blk = (int)(e / (64 * 16)), j = blk % n_ct, ct = blk / n_ct;
+    const int g = kk / 16, unit = 16 * ct + nn, ku = 16 * j + kk % 16;
+    const __nv_bfloat16 v = (unit < H && ku < H) ? W[(size_t)(I + unit) * 4 * H + g * H + ku] : __float2bfloat16(0.0f);
+    const uint32_t byte = sw128((uint32_t)nn, (uint32_t)kk >> 3) + (uint32_t)(kk & 7) * 2;
+    out[((size_t)blk * kWChunkB + byte) / 2] = v;
+}
+
 template <int N>
 struct TmemCols {
     static constexpr uint32_t value = N <= 32 ? 32 : N <= 64 ? 64 : N <= 128 ? 128 : 256;
@@ -205,7 +265,6 @@ bool bf16_plan_fwd_cluster(stacklstm *s, PersistPlan *pl);
 cudaError_t bf16_launch_fwd_cluster(stacklstm *s, const StepArgs &a, const CUtensorMap &tm_x);
 bool bf16_plan_bwd_cluster(stacklstm *s, PersistPlan *pl);
 size_t bf16_bwd_cluster_weight_bytes(int H);
-cudaError_t bf16_pack_bwd_cluster(stacklstm *s, const __nv_bfloat16 *W, __nv_bfloat16 *out);
 cudaError_t bf16_launch_bwd_cluster(stacklstm *s, const StepArgs &a);
 cudaError_t bf16_launch_fwd_cluster_group(stacklstm *const *hs, const StepArgs *as, const CUtensorMap *const *tms, int n,
                                           cudaStream_t st);

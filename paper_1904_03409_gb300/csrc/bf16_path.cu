@@ -400,54 +400,53 @@ __global__ void __launch_bounds__(kThreads, 1) dx_tc(const __grid_constant__ CUt
 }
 
 // ------------------------------------------------------------------ packing
-// Forward operand: for column tile ct, rows n = g * U + j hold gate g of hidden unit
-// ct * U + j; each row is the matching column of W over the contraction
-// [x padded to 64 ; h padded to 64], in 64-element chunks of 128-byte swizzled rows.
-__global__ void pack_fwd(const __nv_bfloat16 *__restrict__ W, int I, int H, int U, int kcx, int KC, int n_ct,
-                         __nv_bfloat16 *__restrict__ out)
-{
-    const int NB = 4 * U, G = 4 * H;
-    const size_t n = (size_t)n_ct * KC * NB * kChunk;
-    for (size_t e = blockIdx.x * (size_t)blockDim.x + threadIdx.x; e < n; e += (size_t)gridDim.x * blockDim.x) {
-        const int col = (int)(e % kChunk);
-        const size_t rowi = e / kChunk;  // (ct * KC + kc) * NB + row
-        const int row = (int)(rowi % NB);
-        const size_t tile = rowi / NB;
-        const int kc = (int)(tile % KC), ct = (int)(tile / KC);
-        const int g = row / U, unit = ct * U + row % U;
-        int wrow = -1;
-        if (kc < kcx) {
-            const int k = kc * kChunk + col;
-            if (k < I) wrow = k;
-        } else {
-            const int k = (kc - kcx) * kChunk + col;
-            if (k < H) wrow = I + k;
-        }
-        const __nv_bfloat16 v =
-            (unit < H && wrow >= 0) ? W[(size_t)wrow * G + g * H + unit] : __float2bfloat16(0.0f);
-        const size_t byte = tile * NB * 128 + sw128(row, col >> 3) + (col & 7) * 2;
-        out[byte / 2] = v;
-    }
-}
+// The forward setup in one launch: the initial state into history row 0 (h0 also as the
+// first h operand) and every weight tile the launches that follow read, each job a range of
+// a flat element index (pack_*_elem, bf16_dev.cuh).
+struct SetupArgs {
+    const __nv_bfloat16 *W;
+    int I, H;
+    __nv_bfloat16 *wf;  // forward gate columns (n_f elements; 0: packed elsewhere)
+    int uf, kcx, kcf;
+    __nv_bfloat16 *wb;  // persistent / per-step backward rows (n_b; 0: not needed)
+    int ub, kcb;
+    __nv_bfloat16 *wdx;  // input-gradient rows (n_dx)
+    int nx;
+    __nv_bfloat16 *wcl;  // cluster backward slices (n_cl; 0: not needed)
+    int n_ctc;
+    const uint4 *h0, *c0;  // 16-byte pieces: n_h of h0, n_c of c0
+    uint4 *hist_h, *hr, *hist_c;
+    size_t n_f, n_b, n_dx, n_cl, n_h, n_c;
+};
 
-// Backward operands: for column tile ct, row m is W row (row0 + ct * NB + m) over the 4H
-// gate columns (zero padded): W_h rows (row0 = I, rows < I + H) for dh_read, W_x rows
-// (row0 = 0, rows < I) for dx.
-__global__ void pack_rows(const __nv_bfloat16 *__restrict__ W, int H, int row0, int nrows, int NB, int KC,
-                          int n_ct, __nv_bfloat16 *__restrict__ out)
+__global__ void setup_kernel(SetupArgs a)
 {
-    const int G = 4 * H;
-    const size_t n = (size_t)n_ct * KC * NB * kChunk;
+    const size_t n = a.n_h + a.n_c + a.n_f + a.n_b + a.n_dx + a.n_cl;
     for (size_t e = blockIdx.x * (size_t)blockDim.x + threadIdx.x; e < n; e += (size_t)gridDim.x * blockDim.x) {
-        const int col = (int)(e % kChunk);
-        const size_t rowi = e / kChunk;
-        const int row = (int)(rowi % NB);
-        const size_t tile = rowi / NB;
-        const int kc = (int)(tile % KC), ct = (int)(tile / KC);
-        const int m = ct * NB + row, k = kc * kChunk + col;
-        const __nv_bfloat16 v = (m < nrows && k < G) ? W[(size_t)(row0 + m) * G + k] : __float2bfloat16(0.0f);
-        const size_t byte = tile * NB * 128 + sw128(row, col >> 3) + (col & 7) * 2;
-        out[byte / 2] = v;
+        size_t r = e;
+        if (r < a.n_h) {
+            const uint4 v = a.h0[r];
+            a.hist_h[r] = v;
+            a.hr[r] = v;
+            continue;
+        }
+        if ((r -= a.n_h) < a.n_c) {
+            a.hist_c[r] = a.c0[r];
+            continue;
+        }
+        if ((r -= a.n_c) < a.n_f) {
+            pack_gate_cols_elem(r, a.W, a.I, a.H, a.uf, a.kcx, a.kcf, a.wf);
+            continue;
+        }
+        if ((r -= a.n_f) < a.n_b) {
+            pack_w_rows_elem(r, a.W, a.H, a.I, a.H, a.ub, a.kcb, a.wb);
+            continue;
+        }
+        if ((r -= a.n_b) < a.n_dx) {
+            pack_w_rows_elem(r, a.W, a.H, 0, a.I, a.nx, a.kcb, a.wdx);
+            continue;
+        }
+        pack_bwd_slice_elem(r - a.n_dx, a.W, a.I, a.H, a.n_ctc, a.wcl);
     }
 }
 
@@ -740,30 +739,48 @@ cudaError_t bf16_forward_setup_state(stacklstm *s, const __nv_bfloat16 *h0, cons
 {
     const int B = s->B, I = s->I, H = s->H;
     cudaError_t e;
-    if ((e = cudaMemcpyAsync(s->hist_h, h0, sizeof(__nv_bfloat16) * B * H, cudaMemcpyDeviceToDevice, s->stream)))
-        return e;
-    if ((e = cudaMemcpyAsync(s->hr, h0, sizeof(__nv_bfloat16) * B * H, cudaMemcpyDeviceToDevice, s->stream)))
-        return e;
-    if ((e = cudaMemcpyAsync(s->hist_c, c0, sizeof(float) * B * H, cudaMemcpyDeviceToDevice, s->stream))) return e;
-    const int nctf = std::max((int)ceil_div(H, s->uf), s->pf.on ? s->pf.n_ct : 0);
-    const int nctb = std::max((int)ceil_div(H, s->ub), s->pb.on ? s->pb.n_ct : 0);
-    if (s->cc.on) {
-        if ((e = bf16_pack_small(s, W))) return e;
-    } else {
-        pack_fwd<<<grid_for(s, (size_t)nctf * s->kcf * 4 * s->uf * kChunk), 256, 0, s->stream>>>(
-            W, I, H, s->uf, s->kcx, s->kcf, nctf, (__nv_bfloat16 *)s->w_fwd);
-        s->launches += 1;
+    SetupArgs a{};
+    a.W = W;
+    a.I = I;
+    a.H = H;
+    // the CUDA-core kernels have weight layouts of their own
+    if (s->cc.on && (e = bf16_pack_small(s, W))) return e;
+    if (!s->cc.on) {
+        const int nctf = std::max((int)ceil_div(H, s->uf), s->pf.on ? s->pf.n_ct : 0);
+        a.wf = (__nv_bfloat16 *)s->w_fwd;
+        a.uf = s->uf;
+        a.kcx = s->kcx;
+        a.kcf = s->kcf;
+        a.n_f = (size_t)nctf * s->kcf * 4 * s->uf * kChunk;
         // the persistent and per-step backward's weight tiles (the cluster backward has its own)
         if (!s->bc.on) {
-            pack_rows<<<grid_for(s, (size_t)nctb * s->kcb * s->ub * kChunk), 256, 0, s->stream>>>(
-                W, H, I, H, s->ub, s->kcb, nctb, (__nv_bfloat16 *)s->w_bwd);
-            s->launches += 1;
+            const int nctb = std::max((int)ceil_div(H, s->ub), s->pb.on ? s->pb.n_ct : 0);
+            a.wb = (__nv_bfloat16 *)s->w_bwd;
+            a.ub = s->ub;
+            a.n_b = (size_t)nctb * s->kcb * s->ub * kChunk;
         }
     }
-    pack_rows<<<grid_for(s, (size_t)s->nxt * s->kcb * s->nx * kChunk), 256, 0, s->stream>>>(
-        W, H, 0, I, s->nx, s->kcb, s->nxt, (__nv_bfloat16 *)s->w_dx);
+    a.kcb = s->kcb;
+    a.wdx = (__nv_bfloat16 *)s->w_dx;
+    a.nx = s->nx;
+    a.n_dx = (size_t)s->nxt * s->kcb * s->nx * kChunk;
+    if (s->bc.on) {
+        a.wcl = (__nv_bfloat16 *)s->w_bcl;
+        a.n_ctc = s->bc.n_ct;
+        a.n_cl = (size_t)s->bc.n_ct * s->bc.n_ct * 16 * 64;
+    }
+    a.h0 = (const uint4 *)h0;
+    a.c0 = (const uint4 *)c0;
+    a.hist_h = (uint4 *)s->hist_h;
+    a.hr = (uint4 *)s->hr;
+    a.hist_c = (uint4 *)s->hist_c;
+    a.n_h = (size_t)B * H / 8;  // H % 8 == 0: whole 16-byte pieces
+    a.n_c = (size_t)B * H / 4;
+    // a few blocks per SM: the prepass, launched just before on the caller's stream, keeps its SMs
+    const size_t n = a.n_h + a.n_c + a.n_f + a.n_b + a.n_dx + a.n_cl;
+    setup_kernel<<<(unsigned)std::max<size_t>(1, std::min<size_t>(ceil_div(n, 256), (size_t)s->num_sms * 4)), 256, 0,
+                   s->stream>>>(a);
     s->launches += 1;
-    if (s->bc.on && (e = bf16_pack_bwd_cluster(s, W, (__nv_bfloat16 *)s->w_bcl))) return e;
     return cudaGetLastError();
 }
 

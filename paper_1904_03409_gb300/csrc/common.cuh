@@ -52,6 +52,8 @@ struct stacklstm {
     int fwd_done = 0;
     int num_sms = 0;
     int prepass_smem = 0;  // dynamic shared memory of the index prepass (0: global scratch)
+    int walk_push_smem = 0;      // the same for the push-only walk (slot tags and index map; 0: separate kernels)
+    int walk_built_virtual = 0;  // the last prepass also built the push-only timeline
 
     // integer bookkeeping, written by the prepass (all [T+1][B] int32)
     int32_t *p_traj = nullptr;     // pointer before step t (t = T: after the last step)

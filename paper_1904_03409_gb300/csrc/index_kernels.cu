@@ -17,23 +17,23 @@ namespace sl {
 namespace {
 
 constexpr int kPrepassThreads = 32;
+// shared-memory staging of prepass_walk_vec_kernel: four [32][32] int32 blocks and the ops
+constexpr size_t kWalkStageBytes = 4 * 32 * 32 * 4 + 32 * 32;
 
-// One thread per instance. The per-instance stack of slot tags lives in a column of
-// shared memory (slot-major, so the 32 threads of a warp hit 32 distinct banks) or, for
-// long sequences, in a global [T+1][B] scratch with the same coalesced layout.
-template <bool kOnChip>
+// One thread per instance, walking its steps in order with the instance's stack of slot
+// tags. This kernel keeps the stack in a global [T+1][B] scratch (coalesced: slot-major)
+// for sequences too long for shared memory and for the allocation-free entry point;
+// prepass_walk_kernel below keeps it in a column of shared memory (slot-major, so the 32
+// threads of a warp hit 32 distinct banks).
 __global__ void __launch_bounds__(kPrepassThreads)
 prepass_kernel(int T, int B, const int8_t *__restrict__ ops, int32_t *__restrict__ p_traj,
                int32_t *__restrict__ top, int32_t *__restrict__ slot_last,
                int32_t *__restrict__ gscratch, int32_t *__restrict__ err)
 {
-    extern __shared__ int32_t s_tag[];
     const int lane = threadIdx.x;
     const int b = blockIdx.x * kPrepassThreads + lane;
     if (b >= B) return;
-    auto tag = [&](int slot) -> int32_t & {
-        return kOnChip ? s_tag[slot * kPrepassThreads + lane] : gscratch[(size_t)slot * B + b];
-    };
+    auto tag = [&](int slot) -> int32_t & { return gscratch[(size_t)slot * B + b]; };
     tag(0) = 0;
     for (int slot = 1; slot <= T; ++slot) tag(slot) = -1;
     int p = 0, e = SL_OK;
@@ -61,6 +61,214 @@ prepass_kernel(int T, int B, const int8_t *__restrict__ ops, int32_t *__restrict
     p_traj[(size_t)T * B + b] = p;
     top[(size_t)T * B + b] = tag(p);
     for (int slot = 0; slot <= T; ++slot) slot_last[(size_t)slot * B + b] = tag(slot);
+    if (e != SL_OK) atomicCAS(err, 0, e);
+}
+
+// The push-only mode's virtual timeline (compact_kernel below), when the walk builds it.
+struct VirtOut {
+    int32_t *vtop, *vy, *vslot, *xidx, *vstep, *kmax;
+};
+
+// The same walk as prepass_kernel with the slot-tag stack in shared memory, its ops loaded
+// 32 steps ahead. With kPush it also builds the push-only mode's virtual timeline in the
+// same walk (what compact_kernel computes from the prepass's outputs), its real-to-virtual
+// index map in shared memory beside the slot tags. (Batches of whole 32-instance blocks
+// take prepass_walk_vec_kernel below.)
+template <bool kPush>
+__global__ void __launch_bounds__(kPrepassThreads)
+prepass_walk_kernel(int T, int B, const int8_t *__restrict__ ops, int32_t *__restrict__ p_traj,
+                    int32_t *__restrict__ top, int32_t *__restrict__ slot_last, int32_t *__restrict__ err, VirtOut v)
+{
+    constexpr int kBlk = 32;
+    extern __shared__ int32_t s_tag[];  // [T + 1][32] slot tags, then (kPush) [T + 1][32] vmap
+    const int lane = threadIdx.x;
+    const int b = blockIdx.x * kPrepassThreads + lane;
+    if (b >= B) return;
+    int32_t *s_vmap = s_tag + (size_t)(T + 1) * kPrepassThreads;
+    auto tag = [&](int slot) -> int32_t & { return s_tag[slot * kPrepassThreads + lane]; };
+    // virtual index of the state at real history index j (-1: a write no step reads)
+    auto vmap = [&](int j) -> int32_t & { return s_vmap[j * kPrepassThreads + lane]; };
+    tag(0) = 0;
+    for (int slot = 1; slot <= T; ++slot) tag(slot) = -1;
+    if (kPush) {
+        vmap(0) = 0;
+        for (int sl = 0; sl <= T; ++sl) v.vslot[(size_t)sl * B + b] = sl == 0 ? 0 : -1;
+    }
+    auto load = [&](int t0, int (&q)[kBlk]) {
+#pragma unroll
+        for (int i = 0; i < kBlk; ++i) q[i] = t0 + i < T ? (int)ops[(size_t)(t0 + i) * B + b] : 0;
+    };
+    int cur[kBlk], nxt[kBlk];
+    load(0, cur);
+    int p = 0, e = SL_OK, k = 0;
+    for (int t0 = 0; t0 < T; t0 += kBlk) {
+        if (t0 + kBlk < T) load(t0 + kBlk, nxt);
+#pragma unroll
+        for (int i = 0; i < kBlk; ++i) {
+            const int t = t0 + i;
+            if (t >= T) break;
+            int op = cur[i];
+            if (op < -1 || op > 1) {  // recorded, then run as a hold so indices stay in range
+                if (e == SL_OK) e = SL_ERR_OP;
+                op = 0;
+            }
+            if (p + op < 0) {
+                if (e == SL_OK) e = SL_ERR_UNDERFLOW;
+                op = 0;
+            }
+            const size_t ti = (size_t)t * B + b;
+            const int tp = tag(p);
+            p_traj[ti] = p;
+            top[ti] = tp;
+            tag(p + 1) = t + 1;  // Algorithm 1: every step writes slot p + 1
+            if (kPush) {
+                // a state that is read is a push write or the initial state (clamp never applies)
+                const int rd = max(0, vmap(tp));
+                v.vy[ti] = rd;
+                if (op == 1) {
+                    v.xidx[(size_t)k * B + b] = t;
+                    v.vtop[(size_t)k * B + b] = rd;
+                    v.vstep[ti] = k;
+                    vmap(t + 1) = k + 1;
+                    v.vslot[(size_t)(p + 1) * B + b] = k + 1;
+                    ++k;
+                } else {
+                    v.vstep[ti] = -1;
+                    vmap(t + 1) = -1;
+                }
+            }
+            p += op;
+        }
+#pragma unroll
+        for (int i = 0; i < kBlk; ++i) cur[i] = nxt[i];
+    }
+    const int tp = tag(p);
+    p_traj[(size_t)T * B + b] = p;
+    top[(size_t)T * B + b] = tp;
+    for (int slot = 0; slot <= T; ++slot) slot_last[(size_t)slot * B + b] = tag(slot);
+    if (kPush) {
+        v.vy[(size_t)T * B + b] = max(0, vmap(tp));
+        for (int kk = k; kk < T; ++kk) {
+            v.xidx[(size_t)kk * B + b] = -1;
+            v.vtop[(size_t)kk * B + b] = 0;
+        }
+        v.vtop[(size_t)T * B + b] = 0;
+        atomicMax(v.kmax, k);
+    }
+    if (e != SL_OK) atomicCAS(err, 0, e);
+}
+
+// prepass_walk_kernel for batches of whole 32-instance blocks (B % 32 == 0, ops 4-byte
+// aligned), its global traffic in 16-byte pieces: the walk costs about as much per memory
+// instruction of the block's one warp as per step, so the warp loads a block of 32 steps'
+// ops as 4-byte words (eight lanes a row) into shared memory, walks it there, stages the
+// block's pointers and tops (and virtual indices) in shared memory, and writes them four
+// rows per instruction; the slot tags go out the same way, and the push-only tables that
+// are mostly -1 / 0 are written so before the walk (__syncwarp orders those stores before
+// the walk's own stores to the same rows).
+template <bool kPush>
+__global__ void __launch_bounds__(kPrepassThreads)
+prepass_walk_vec_kernel(int T, int B, const int8_t *__restrict__ ops, int32_t *__restrict__ p_traj,
+                        int32_t *__restrict__ top, int32_t *__restrict__ slot_last, int32_t *__restrict__ err,
+                        VirtOut v)
+{
+    constexpr int kBlk = 32;
+    // [T + 1][32] slot tags, (kPush) [T + 1][32] vmap, then the block staging:
+    // pointer, top, (kPush) vy, vstep, each [32 steps][32], and the ops [32 steps][32 bytes]
+    extern __shared__ int32_t s_tag[];
+    const int lane = threadIdx.x, b0 = blockIdx.x * kPrepassThreads, b = b0 + lane;
+    const int rq = lane >> 3, pc = 4 * (lane & 7);  // row of four, 16-byte piece: the vector pattern
+    int32_t *s_vmap = s_tag + (size_t)(T + 1) * kPrepassThreads;
+    int32_t *st_p = s_tag + (size_t)(kPush ? 2 : 1) * (T + 1) * kPrepassThreads;
+    int32_t *st_t = st_p + kBlk * 32, *st_y = st_t + kBlk * 32, *st_v = st_y + kBlk * 32;
+    uint32_t *st_o = (uint32_t *)(st_v + kBlk * 32);  // [32 steps][8 words]
+    auto tag = [&](int slot) -> int32_t & { return s_tag[slot * kPrepassThreads + lane]; };
+    auto vmap = [&](int j) -> int32_t & { return s_vmap[j * kPrepassThreads + lane]; };
+    // rows [r0, r1) of a [rows][B] int32 table: this block's 32 columns, four rows at a time
+    auto fill = [&](int32_t *dst, int r0, int r1, int val) {
+        const uint4 w = make_uint4(val, val, val, val);
+        for (int r = r0 + rq; r < r1; r += 4) *(uint4 *)(dst + (size_t)r * B + b0 + pc) = w;
+    };
+    auto flush = [&](int32_t *dst, const int32_t *src, int r0, int nrows) {  // src: [nrows][32]
+        for (int r = rq; r < nrows; r += 4) *(uint4 *)(dst + (size_t)(r0 + r) * B + b0 + pc) = *(const uint4 *)(src + r * 32 + pc);
+    };
+    auto load = [&](int t0, uint32_t (&q)[8]) {
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+            const int t = t0 + rq + 4 * j;
+            q[j] = t < T ? *(const uint32_t *)(ops + (size_t)t * B + b0 + pc) : 0u;
+        }
+    };
+    tag(0) = 0;
+    for (int slot = 1; slot <= T; ++slot) tag(slot) = -1;
+    if (kPush) {
+        vmap(0) = 0;
+        fill(v.vslot, 0, 1, 0);
+        fill(v.vslot, 1, T + 1, -1);
+        fill(v.xidx, 0, T, -1);
+        fill(v.vtop, 0, T + 1, 0);
+        __syncwarp();
+    }
+    uint32_t cur[8], nxt[8];
+    load(0, cur);
+    int p = 0, e = SL_OK, k = 0;
+    for (int t0 = 0; t0 < T; t0 += kBlk) {
+        if (t0 + kBlk < T) load(t0 + kBlk, nxt);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) st_o[(rq + 4 * j) * 8 + (lane & 7)] = cur[j];
+        __syncwarp();
+        const int n = min(kBlk, T - t0);
+        const int8_t *ob = (const int8_t *)st_o;
+        for (int i = 0; i < n; ++i) {
+            const int t = t0 + i;
+            int op = ob[i * 32 + lane];
+            if (op < -1 || op > 1) {  // recorded, then run as a hold so indices stay in range
+                if (e == SL_OK) e = SL_ERR_OP;
+                op = 0;
+            }
+            if (p + op < 0) {
+                if (e == SL_OK) e = SL_ERR_UNDERFLOW;
+                op = 0;
+            }
+            const int tp = tag(p);
+            st_p[i * 32 + lane] = p;
+            st_t[i * 32 + lane] = tp;
+            tag(p + 1) = t + 1;  // Algorithm 1: every step writes slot p + 1
+            if (kPush) {
+                // a state that is read is a push write or the initial state (clamp never applies)
+                const int rd = max(0, vmap(tp));
+                st_y[i * 32 + lane] = rd;
+                st_v[i * 32 + lane] = op == 1 ? k : -1;
+                vmap(t + 1) = op == 1 ? k + 1 : -1;
+                if (op == 1) {
+                    v.xidx[(size_t)k * B + b] = t;
+                    v.vtop[(size_t)k * B + b] = rd;
+                    v.vslot[(size_t)(p + 1) * B + b] = k + 1;
+                    ++k;
+                }
+            }
+            p += op;
+        }
+        __syncwarp();
+        flush(p_traj, st_p, t0, n);
+        flush(top, st_t, t0, n);
+        if (kPush) {
+            flush(v.vy, st_y, t0, n);
+            flush(v.vstep, st_v, t0, n);
+        }
+        __syncwarp();  // the staging is read before the next block overwrites it
+#pragma unroll
+        for (int j = 0; j < 8; ++j) cur[j] = nxt[j];
+    }
+    const int tp = tag(p);
+    p_traj[(size_t)T * B + b] = p;
+    top[(size_t)T * B + b] = tp;
+    if (kPush) {
+        v.vy[(size_t)T * B + b] = max(0, vmap(tp));
+        atomicMax(v.kmax, k);
+    }
+    __syncwarp();
+    flush(slot_last, s_tag, 0, T + 1);
     if (e != SL_OK) atomicCAS(err, 0, e);
 }
 
@@ -207,6 +415,7 @@ __global__ void zero_nonpush_rows_kernel(size_t rows, int I4, const int32_t *__r
 
 cudaError_t launch_compact(stacklstm *s)
 {
+    if (s->walk_built_virtual) return cudaSuccess;  // the prepass's walk built the timeline
     cudaError_t e = cudaMemsetAsync(s->kmax, 0, sizeof(int32_t), s->stream);
     if (e) return e;
     // the index table on chip when the prepass's slot-tag stack is (the same size)
@@ -270,9 +479,19 @@ cudaError_t configure_prepass(stacklstm *s)
     cudaError_t e = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, s->device);
     if (e) return e;
     s->prepass_smem = 0;
-    if (bytes + 1024 <= (size_t)optin) {
-        if (bytes > 48 * 1024 && (e = smem_at_least((const void *)prepass_kernel<true>, bytes))) return e;
+    s->walk_push_smem = 0;
+    if (bytes + kWalkStageBytes + 1024 <= (size_t)optin) {
+        if ((e = smem_at_least((const void *)prepass_walk_kernel<false>, bytes)) ||
+            (e = smem_at_least((const void *)prepass_walk_vec_kernel<false>, bytes + kWalkStageBytes)))
+            return e;
         s->prepass_smem = (int)bytes;
+        // the push-only walk keeps the real-to-virtual index map beside the slot tags
+        if (2 * bytes + kWalkStageBytes + 1024 <= (size_t)optin) {
+            if ((e = smem_at_least((const void *)prepass_walk_kernel<true>, 2 * bytes)) ||
+                (e = smem_at_least((const void *)prepass_walk_vec_kernel<true>, 2 * bytes + kWalkStageBytes)))
+                return e;
+            s->walk_push_smem = (int)(2 * bytes);
+        }
     }
     return cudaSuccess;
 }
@@ -280,12 +499,31 @@ cudaError_t configure_prepass(stacklstm *s)
 cudaError_t launch_prepass(stacklstm *s, const int8_t *ops)
 {
     const unsigned grid = ceil_div(s->B, kPrepassThreads);
-    if (s->prepass_smem > 0)
-        prepass_kernel<true><<<grid, kPrepassThreads, s->prepass_smem, s->stream>>>(
-            s->T, s->B, ops, s->p_traj, s->top, s->slot_last, nullptr, s->err);
-    else
-        prepass_kernel<false><<<grid, kPrepassThreads, 0, s->stream>>>(
-            s->T, s->B, ops, s->p_traj, s->top, s->slot_last, s->slot_scratch, s->err);
+    s->walk_built_virtual = 0;
+    // whole 32-instance blocks and word-aligned ops: the walk's traffic in 16-byte pieces
+    const bool vec = s->B % kPrepassThreads == 0 && ((uintptr_t)ops & 3) == 0;
+    if (s->push_only && s->walk_push_smem > 0) {
+        cudaError_t e = cudaMemsetAsync(s->kmax, 0, sizeof(int32_t), s->stream);
+        if (e) return e;
+        const VirtOut v{s->vtop, s->vy, s->vslot, s->xidx, s->vstep, s->kmax};
+        if (vec)
+            prepass_walk_vec_kernel<true><<<grid, kPrepassThreads, s->walk_push_smem + kWalkStageBytes, s->stream>>>(
+                s->T, s->B, ops, s->p_traj, s->top, s->slot_last, s->err, v);
+        else
+            prepass_walk_kernel<true><<<grid, kPrepassThreads, s->walk_push_smem, s->stream>>>(
+                s->T, s->B, ops, s->p_traj, s->top, s->slot_last, s->err, v);
+        s->walk_built_virtual = 1;
+    } else if (s->prepass_smem > 0) {
+        if (vec)
+            prepass_walk_vec_kernel<false><<<grid, kPrepassThreads, s->prepass_smem + kWalkStageBytes, s->stream>>>(
+                s->T, s->B, ops, s->p_traj, s->top, s->slot_last, s->err, VirtOut{});
+        else
+            prepass_walk_kernel<false><<<grid, kPrepassThreads, s->prepass_smem, s->stream>>>(
+                s->T, s->B, ops, s->p_traj, s->top, s->slot_last, s->err, VirtOut{});
+    } else {
+        prepass_kernel<<<grid, kPrepassThreads, 0, s->stream>>>(s->T, s->B, ops, s->p_traj, s->top, s->slot_last,
+                                                                s->slot_scratch, s->err);
+    }
     s->launches += 1;
     return cudaGetLastError();
 }
@@ -378,8 +616,7 @@ extern "C" sl_status stacklstm_pointers_noalloc(int T, int B, const int8_t *ops,
         cudaGetLastError();
         return SL_ERR_CUDA;
     }
-    prepass_kernel<false><<<ceil_div(B, kPrepassThreads), kPrepassThreads, 0, st>>>(T, B, ops, p_traj, src, last,
-                                                                                   tags, err);
+    prepass_kernel<<<ceil_div(B, kPrepassThreads), kPrepassThreads, 0, st>>>(T, B, ops, p_traj, src, last, tags, err);
     int32_t h = 0;
     cudaError_t e = cudaGetLastError();
     if (e == cudaSuccess) e = cudaMemcpyAsync(&h, err, sizeof h, cudaMemcpyDeviceToHost, st);

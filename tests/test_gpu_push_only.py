@@ -86,6 +86,22 @@ def test_push_only_matches_definition_mode(T, B, I, H, seed, env):
     check_against_homogenized(w, got, env)
 
 
+@pytest.mark.parametrize("T,B", [(900, 40), (900, 64), (2000, 64)])
+def test_long_sequences_take_every_index_prepass(T, B):
+    """The index prepass has three forms by sequence length: up to several hundred steps one
+    kernel walks the ops with its slot tags (and, push-only mode, the real-to-virtual index
+    map) on chip; at T = 900 the push-only map no longer fits beside the tags and the
+    compaction runs as a kernel of its own; at T = 2000 the slot tags live in a global
+    scratch. Each with a ragged 32-instance block (B = 40) or whole ones (B = 64), both modes."""
+    w = case(T, B, 8, 16, 42 + T + B, probs=(0.45, 0.35, 0.2), bias_scale=0.3, h0_scale=0.5)
+    ptr = oracle.pointers(w.ops)
+    hom = runner.run(w)
+    assert np.array_equal(hom["p_traj"], ptr["p_traj"]) and np.array_equal(hom["src"], ptr["src"])
+    got = runner.run(w, mode=PUSH)
+    compare(got, definition(w), "bf16")
+    check_against_homogenized(w, got)
+
+
 def test_no_push_at_all_runs_one_unread_step():
     w = case(16, 40, 16, 24, 39, probs=(0.0, 0.0, 1.0), h0_scale=0.5)
     got = runner.run(w, mode=PUSH)
