@@ -489,22 +489,12 @@ __device__ __forceinline__ ClbCtl clb_carve(uint8_t *raw, int n_ct)
 }  // namespace
 
 namespace {
-// This thread's row of a dG block (4 gates x 16 units, zero past H or B) into the swizzled
-// global block `blk` (64 rows x 128 bytes).
-// The 16-byte pieces 2g and 2g + 1 of a row (gate g) land in one aligned 32-byte pair under
-// the 128-byte swizzle, in swapped order on odd rows: one 32-byte store a gate.
-__device__ __forceinline__ void store_dg_block(uint8_t *blk, int row, const uint4 (&v)[4][2], bool v0, bool v1)
+// One lane's half of a row of a dG block: gate g's units 8 h .. 8 h + 7 (zero past H or B)
+// to 16-byte piece 2 g + h of the row in the 128-byte-swizzled global block `blk`.
+__device__ __forceinline__ void store_dg_half(uint8_t *blk, int row, int h, const uint4 (&v)[4])
 {
-    if (row >= 64) return;
-    const uint4 z = make_uint4(0u, 0u, 0u, 0u);
-    const bool odd = row & 1;
 #pragma unroll
-    for (int g = 0; g < 4; ++g) {
-        const uint4 lo = v0 ? v[g][0] : z, hi = v1 ? v[g][1] : z;
-        const uint4 a = odd ? hi : lo, b = odd ? lo : hi;
-        const uint32_t w[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
-        st8u_a32(blk + (sw128((uint32_t)row, (uint32_t)(2 * g)) & ~31u), w);
-    }
+    for (int g = 0; g < 4; ++g) *(uint4 *)(blk + sw128((uint32_t)row, (uint32_t)(2 * g + h))) = v[g];
 }
 
 // After every epilogue warp has stored its rows of the block: thread 0 waits until every
@@ -617,26 +607,28 @@ __device__ __forceinline__ void step_clb_body(const ClArgs &p, int row0)
         __syncwarp();
     } else {
         // ------------------------------------------------------------ epilogue
-        // M = 64 accumulator: rows 16 w .. 16 w + 15 in lanes 0..15 of TMEM lane quadrant w
-        const int row = lane < 16 ? warp * 16 + lane : 64;  // lanes 16..31 hold no row
-        const int grow = row0 + row;                          // the row of the whole batch
+        // M = 64 accumulator: rows 16 w .. 16 w + 15 in lanes 0..15 of TMEM lane quadrant w.
+        // Two lanes per row: lane l takes row 16 w + l % 16 and units 8 h .. 8 h + 7 of this
+        // CTA's 16, h = l / 16; lanes 16..31 take their accumulator values from lane l - 16
+        // by shuffles. Both halves of a row's piece then sit on one line, so every global
+        // access of a warp covers its 16 rows in half the L1 wavefronts of one lane per row.
+        const int hf = lane >> 4;
+        const int row = warp * 16 + (lane & 15);
+        const int grow = row0 + row;          // the row of the whole batch
         const bool row_ok = row < nrows;
         const bool warp_rows = warp * 16 < nrows;
-        const int u0 = (int)ct * U;
-        const bool v0 = row_ok && u0 < H, v1 = row_ok && u0 + 8 < H;  // the two 8-unit groups (H % 8 == 0)
+        const int u0 = (int)ct * U, uh = u0 + 8 * hf;
+        const bool vh = row_ok && uh < H;  // this lane's 8 units (H % 8 == 0)
         const uint32_t taddr0 = tmem + ((uint32_t)(warp * 32) << 16);
+        const uint4 z4 = make_uint4(0u, 0u, 0u, 0u);
         // dG of step T - 1 (written before the launch) into every CTA's dG buffer
         {
-            uint4 g0v[4][2];
-            if (v0)
+            uint4 g0v[4];
 #pragma unroll
-                for (int g = 0; g < 4; ++g)
-#pragma unroll
-                    for (int i = 0; i < 2; ++i)
-                        if (i == 0 || v1)
-                            g0v[g][i] = __ldcg((const uint4 *)(a.dG + ((size_t)(T - 1) * B + grow) * 4 * H + g * H + u0 + 8 * i));
+            for (int g = 0; g < 4; ++g)
+                g0v[g] = vh ? __ldcg((const uint4 *)(a.dG + ((size_t)(T - 1) * B + grow) * 4 * H + g * H + uh)) : z4;
             uint8_t *blk = gscr + ((size_t)(T - 1) * n_ct + ct) * kGBlock;
-            store_dg_block(blk, row, g0v, v0, v1);
+            store_dg_half(blk, row, hf, g0v);
             deliver_dg(c, blk, -1, ct, n_ct, tid, limit, a.err);
         }
         // the state step t reads (src) and the one step t - 1 read (s1): a step ahead
@@ -648,41 +640,28 @@ __device__ __forceinline__ void step_clb_body(const ClArgs &p, int row0)
         for (int k = 0; k < T; ++k) {
             const int t = T - 1 - k, acc = k & 1;
             // this step's operands (rows this thread wrote at later steps, or the forward's)
-            float dh_src[U], dh_t[U], dc_t[U], cn[U], cr[U], dc_rd[U];
-            uint4 gq[4][2];
+            float dh_src[8], dh_t[8], dc_t[8], cn[8], cr[8], dc_rd[8];
+            uint4 gq[4];
             int src_n = 0, s1_n = 0;
             if (row_ok && t >= 1) {
                 src_n = a.top[(size_t)(t - 1) * B + grow];
                 s1_n = t >= 2 ? a.top[(size_t)(t - 2) * B + grow] : 0;
             }
-            if (v0)
+            if (vh) {
+                ld8f_a32(a.dhist_h + ((size_t)src * B + grow) * H + uh, dh_src);
+                if (t >= 1) {
+                    const size_t wr = ((size_t)t * B + grow) * H + uh, rd = ((size_t)s1 * B + grow) * H + uh;
+                    ld8f_a32(a.dhist_h + wr, dh_t);
+                    ld8f_a32(a.dhist_c + wr, dc_t);
+                    ld8f_a32(a.hist_c + wr, cn);
+                    ld8f_a32(a.hist_c + rd, cr);
+                    ld8f_a32(a.dhist_c + rd, dc_rd);
+                    const __half *gt = a.gates_blk
+                                           ? a.gates + (((size_t)(t - 1) * B + grow) * n_ct + ct) * 4 * U + 8 * hf
+                                           : a.gates + ((size_t)(t - 1) * B + grow) * 4 * H + uh;
+                    const size_t gs = a.gates_blk ? (size_t)U : (size_t)H;  // gate stride
 #pragma unroll
-                for (int i = 0; i < 2; ++i) {
-                    if (i == 1 && !v1) break;
-                    const size_t us = ((size_t)src * B + grow) * H + u0 + 8 * i;
-                    ld8f_a32(a.dhist_h + us, *(float(*)[8])(dh_src + 8 * i));
-                    if (t >= 1) {
-                        const size_t wr = ((size_t)t * B + grow) * H + u0 + 8 * i, rd = ((size_t)s1 * B + grow) * H + u0 + 8 * i;
-                        ld8f_a32(a.dhist_h + wr, *(float(*)[8])(dh_t + 8 * i));
-                        ld8f_a32(a.dhist_c + wr, *(float(*)[8])(dc_t + 8 * i));
-                        ld8f_a32(a.hist_c + wr, *(float(*)[8])(cn + 8 * i));
-                        ld8f_a32(a.hist_c + rd, *(float(*)[8])(cr + 8 * i));
-                        ld8f_a32(a.dhist_c + rd, *(float(*)[8])(dc_rd + 8 * i));
-                        if (!a.gates_blk) {
-                            const __half *gt = a.gates + ((size_t)(t - 1) * B + grow) * 4 * H + u0 + 8 * i;
-#pragma unroll
-                            for (int g = 0; g < 4; ++g) gq[g][i] = __ldcg((const uint4 *)(gt + (size_t)g * H));
-                        }
-                    }
-                }
-            if (v0 && t >= 1 && a.gates_blk) {
-                const __half *gt = a.gates + (((size_t)(t - 1) * B + grow) * n_ct + ct) * 4 * U;
-#pragma unroll
-                for (int g = 0; g < 4; ++g) {
-                    uint32_t q[8];
-                    ld8u_a32(gt + g * U, q);
-                    gq[g][0] = make_uint4(q[0], q[1], q[2], q[3]);
-                    gq[g][1] = make_uint4(q[4], q[5], q[6], q[7]);
+                    for (int g = 0; g < 4; ++g) gq[g] = __ldcg((const uint4 *)(gt + g * gs));
                 }
             }
             const bool ok = tc::mbar_wait(&c.tfull[acc], (k >> 1) & 1, limit, c.abort);
@@ -693,74 +672,67 @@ __device__ __forceinline__ void step_clb_body(const ClArgs &p, int row0)
             __syncwarp();
             if (tc::bar_any(1, E * 32, !ok || *c.abort)) break;
             tc::tc_fence_after();
-            float v[U];  // dh_src + the issuers' partial sums, added in issuer order
+            float v[8];  // dh_src + the issuers' partial sums, added in issuer order
+            {
+                float sum[U];
 #pragma unroll
-            for (int j = 0; j < U; ++j) v[j] = 0.0f;
-            if (warp_rows)
+                for (int j = 0; j < U; ++j) sum[j] = 0.0f;
+                if (warp_rows)
 #pragma unroll
-                for (int q2 = 0; q2 < NI; q2 += 2) {
-                    uint32_t dr[2][U];
-                    tc::tmem_ld16_async(taddr0 + acc * kCols + q2 * U, dr[0]);
-                    tc::tmem_ld16_async(taddr0 + acc * kCols + (q2 + 1) * U, dr[1]);
-                    tc::tmem_wait_ld();
+                    for (int q2 = 0; q2 < NI; q2 += 2) {
+                        uint32_t dr[2][U];
+                        tc::tmem_ld16_async(taddr0 + acc * kCols + q2 * U, dr[0]);
+                        tc::tmem_ld16_async(taddr0 + acc * kCols + (q2 + 1) * U, dr[1]);
+                        tc::tmem_wait_ld();
 #pragma unroll
-                    for (int j = 0; j < U; ++j) v[j] += __uint_as_float(dr[0][j]) + __uint_as_float(dr[1][j]);
+                        for (int j = 0; j < U; ++j) sum[j] += __uint_as_float(dr[0][j]) + __uint_as_float(dr[1][j]);
+                    }
+                tc::tc_fence_before();
+                __syncwarp();
+                if (lane == 0) tc::mbar_arrive(&c.tempty[acc]);
+#pragma unroll
+                for (int i = 0; i < 8; ++i) {
+                    const float up = __shfl_sync(0xffffffffu, sum[8 + i], lane & 15);
+                    v[i] = (hf ? up : sum[i]) + dh_src[i];
                 }
-            tc::tc_fence_before();
-            __syncwarp();
-            if (lane == 0) tc::mbar_arrive(&c.tempty[acc]);
-#pragma unroll
-            for (int j = 0; j < U; ++j) v[j] += dh_src[j];
-            float dcr[U];
+            }
+            float dcr[8];
             if (t >= 1) {
                 // the pointwise backward of step t - 1 (lanes without a row compute and discard)
-                float d[4][U];
+                float d[4][8], ig[8], fg[8], gg[8], og[8];
+                unpack8_f16(gq[0], ig);
+                unpack8_f16(gq[1], fg);
+                unpack8_f16(gq[2], gg);
+                unpack8_f16(gq[3], og);
 #pragma unroll
-                for (int i = 0; i < 2; ++i) {
-                    float ig[8], fg[8], gg[8], og[8];
-                    unpack8_f16(gq[0][i], ig);
-                    unpack8_f16(gq[1][i], fg);
-                    unpack8_f16(gq[2][i], gg);
-                    unpack8_f16(gq[3][i], og);
-#pragma unroll
-                    for (int e = 0; e < 8; ++e) {
-                        const int q = 8 * i + e;
-                        const float dh = src == t ? v[q] : dh_t[q];  // the state read at t is row t
-                        const float tcn = tanh_hw(cn[q]);
-                        const float dc = dc_t[q] + dh * og[e] * (1.0f - tcn * tcn);
-                        d[0][q] = dc * gg[e] * ig[e] * (1.0f - ig[e]);
-                        d[1][q] = dc * cr[q] * fg[e] * (1.0f - fg[e]);
-                        d[2][q] = dc * ig[e] * (1.0f - gg[e] * gg[e]);
-                        d[3][q] = dh * tcn * og[e] * (1.0f - og[e]);
-                        dcr[q] = dc_rd[q] + dc * fg[e];
-                    }
+                for (int q = 0; q < 8; ++q) {
+                    const float dh = src == t ? v[q] : dh_t[q];  // the state read at t is row t
+                    const float tcn = tanh_hw(cn[q]);
+                    const float dc = dc_t[q] + dh * og[q] * (1.0f - tcn * tcn);
+                    d[0][q] = dc * gg[q] * ig[q] * (1.0f - ig[q]);
+                    d[1][q] = dc * cr[q] * fg[q] * (1.0f - fg[q]);
+                    d[2][q] = dc * ig[q] * (1.0f - gg[q] * gg[q]);
+                    d[3][q] = dh * tcn * og[q] * (1.0f - og[q]);
+                    dcr[q] = dc_rd[q] + dc * fg[q];
                 }
-                uint4 dg[4][2];
+                uint4 dg[4];
 #pragma unroll
-                for (int g = 0; g < 4; ++g)
-#pragma unroll
-                    for (int i = 0; i < 2; ++i) dg[g][i] = pack8_bf16(*(const float(*)[8])(d[g] + 8 * i));
+                for (int g = 0; g < 4; ++g) dg[g] = vh ? pack8_bf16(d[g]) : z4;
                 // dG_{t-1}: its block to global memory, then (multicast bulk copy) to every CTA
                 uint8_t *blk = gscr + ((size_t)(t - 1) * n_ct + ct) * kGBlock;
-                store_dg_block(blk, row, dg, v0, v1);
+                store_dg_half(blk, row, hf, dg);
                 deliver_dg(c, blk, k & 1, ct, n_ct, tid, limit, a.err);
                 // and in the [T B][4H] layout (for the input and weight gradients), after the delivery
-                if (v0)
+                if (vh) {
+                    __nv_bfloat16 *gp = a.dG + ((size_t)(t - 1) * B + grow) * 4 * H + uh;
 #pragma unroll
-                    for (int i = 0; i < 2; ++i) {
-                        if (i == 1 && !v1) break;
-                        __nv_bfloat16 *gp = a.dG + ((size_t)(t - 1) * B + grow) * 4 * H + u0 + 8 * i;
-#pragma unroll
-                        for (int g = 0; g < 4; ++g) *(uint4 *)(gp + (size_t)g * H) = dg[g][i];
-                    }
-            }
-            if (v0)
-#pragma unroll
-                for (int i = 0; i < 2; ++i) {
-                    if (i == 1 && !v1) break;
-                    st8f_a32(a.dhist_h + ((size_t)src * B + grow) * H + u0 + 8 * i, *(const float(*)[8])(v + 8 * i));
-                    if (t >= 1) st8f_a32(a.dhist_c + ((size_t)s1 * B + grow) * H + u0 + 8 * i, *(const float(*)[8])(dcr + 8 * i));
+                    for (int g = 0; g < 4; ++g) *(uint4 *)(gp + (size_t)g * H) = dg[g];
                 }
+            }
+            if (vh) {
+                st8f_a32(a.dhist_h + ((size_t)src * B + grow) * H + uh, v);
+                if (t >= 1) st8f_a32(a.dhist_c + ((size_t)s1 * B + grow) * H + uh, dcr);
+            }
             src = src_n;
             s1 = s1_n;
         }
