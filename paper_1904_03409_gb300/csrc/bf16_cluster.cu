@@ -136,18 +136,14 @@ __device__ __forceinline__ uint64_t slice_desc(uint32_t addr)
 // byte offset of 16-byte piece k (units 8k .. 8k + 7) of row r in an h slice
 __host__ __device__ constexpr uint32_t slice_off(uint32_t r, uint32_t k) { return (r >> 3) * 256 + k * 128 + (r & 7) * 16; }
 
-// Writes this thread's row of h_read(s) (16 units, zero past H or B) into its global slice
-// block `blk` (2 KB, the slice layout), then (once every epilogue warp has) one multicast
-// bulk copy loads the block into every CTA's h buffer `buf` at this CTA's slice position,
-// completing on that CTA's hready[buf]: one L2 read delivered to all CTAs.
-__device__ __forceinline__ void deliver_slice(const ClCtl &c, uint8_t *blk, int buf, int row, const uint4 (&v)[2],
-                                              bool valid0, bool valid1, uint32_t ct, uint32_t n_ct, int tid)
+// Writes this lane's half of its row of h_read(s) (units 8 h .. 8 h + 7, zero past H or B)
+// into its global slice block `blk` (2 KB, the slice layout), then (once every epilogue warp
+// has) one multicast bulk copy loads the block into every CTA's h buffer `buf` at this CTA's
+// slice position, completing on that CTA's hready[buf]: one L2 read delivered to all CTAs.
+__device__ __forceinline__ void deliver_slice(const ClCtl &c, uint8_t *blk, int buf, int row, int h, const uint4 &v,
+                                              uint32_t ct, uint32_t n_ct, int tid)
 {
-    if (row < 64) {
-        const uint4 z = make_uint4(0u, 0u, 0u, 0u);
-        *(uint4 *)(blk + slice_off((uint32_t)row, 0)) = valid0 ? v[0] : z;
-        *(uint4 *)(blk + slice_off((uint32_t)row, 1)) = valid1 ? v[1] : z;
-    }
+    *(uint4 *)(blk + slice_off((uint32_t)row, (uint32_t)h)) = v;
     tc::fence_proxy_async_global();  // this thread's block stores -> the bulk copy
     __syncwarp();
     tc::bar_sync(2, 4 * 32);
@@ -276,144 +272,122 @@ __device__ __forceinline__ void step_cl_body(const CUtensorMap *tmx, const ClArg
         __syncwarp();
     } else {
         // ------------------------------------------------------------ epilogue
-        // M = 64 accumulator: rows 16 w .. 16 w + 15 in lanes 0..15 of TMEM lane quadrant w
-        const int row = lane < 16 ? warp * 16 + lane : 64;  // lanes 16..31 hold no row
-        const int grow = row0 + row;                          // the row of the whole batch
+        // M = 64 accumulator: rows 16 w .. 16 w + 15 in lanes 0..15 of TMEM lane quadrant w.
+        // Two lanes per row: lane l takes row 16 w + l % 16 and units 8 h .. 8 h + 7 of this
+        // CTA's 16, h = l / 16; lanes 16..31 take their pre-activations from lane l - 16 by
+        // shuffles. Both halves of a row's piece then sit on one line, so every global access
+        // of a warp covers its 16 rows in half the L1 wavefronts of one lane per row.
+        const int hf = lane >> 4;
+        const int row = warp * 16 + (lane & 15);
+        const int grow = row0 + row;  // the row of the whole batch
         const bool row_ok = row < nrows;
         const bool warp_rows = warp * 16 < nrows;
-        const int u0 = (int)ct * U;
-        const bool v0 = row_ok && u0 < H, v1 = row_ok && u0 + 8 < H;  // the two 8-unit groups (H % 8 == 0)
+        const int u0 = (int)ct * U, uh = u0 + 8 * hf;
+        const bool vh = row_ok && uh < H;  // this lane's 8 units (H % 8 == 0)
         const uint32_t taddr0 = tmem + ((uint32_t)(warp * 32) << 16);
+        const float *bias_h = s_bias + 8 * hf;  // gate g's bias of this lane's units: bias_h[g U + j]
         // c of the state step t reads, and (when step t does not push) the h of the older
         // state that becomes the next step's h operand
-        float crv[U];
-        uint4 hold[2];
+        float crv[8];
+        uint4 hold = make_uint4(0u, 0u, 0u, 0u);
         // top[t + 1][row] and top[t + 2][row] at step t (indices loaded two steps ahead)
         int s_nxt = 0, s_2 = 0;
-        uint4 h0v[2];
-        if (v0) {
+        uint4 h0v = make_uint4(0u, 0u, 0u, 0u);
+        if (vh) {
             const int s_cur = a.top[grow];
             s_nxt = T >= 1 ? a.top[(size_t)B + grow] : 0;
             s_2 = T >= 2 ? a.top[(size_t)2 * B + grow] : 0;
-#pragma unroll
-            for (int i = 0; i < 2; ++i) {
-                if (i == 1 && !v1) break;
-                float v[8];
-                ld8f_a32(a.hist_c + ((size_t)s_cur * B + grow) * H + u0 + 8 * i, v);
-#pragma unroll
-                for (int k = 0; k < 8; ++k) crv[8 * i + k] = v[k];
-                hold[i] = __ldcg((const uint4 *)(a.hr + ((size_t)s_nxt * B + grow) * H + u0 + 8 * i));
-                h0v[i] = __ldcg((const uint4 *)(a.hr + (size_t)grow * H + u0 + 8 * i));  // h_read(0)
-            }
+            ld8f_a32(a.hist_c + ((size_t)s_cur * B + grow) * H + uh, crv);
+            hold = __ldcg((const uint4 *)(a.hr + ((size_t)s_nxt * B + grow) * H + uh));
+            h0v = __ldcg((const uint4 *)(a.hr + (size_t)grow * H + uh));  // h_read(0)
         }
-        deliver_slice(c, gscr + (size_t)ct * kSlice, 0, row, h0v, v0, v1, ct, n_ct, tid);
+        deliver_slice(c, gscr + (size_t)ct * kSlice, 0, row, hf, h0v, ct, n_ct, tid);
         for (int t = 0; t < T; ++t) {
             const int b = t & 1;
             // the next step's operands that rows written before this step hold: issued now,
             // used after this step's cell (c_read of step t + 1 unless step t pushes; the
             // older top that is step t + 2's h operand unless it is this step's new state)
-            float cr_n[U];
-            uint4 hold_n[2];
+            float cr_n[8];
+            uint4 hold_n = make_uint4(0u, 0u, 0u, 0u);
             int s_3 = 0;
-            if (v0 && t + 1 < T) {
+            if (vh && t + 1 < T) {
                 if (t + 3 <= T) s_3 = a.top[(size_t)(t + 3) * B + grow];
-#pragma unroll
-                for (int i = 0; i < 2; ++i) {
-                    if (i == 1 && !v1) break;
-                    if (s_nxt != t + 1) {
-                        float v[8];
-                        ld8f_a32(a.hist_c + ((size_t)s_nxt * B + grow) * H + u0 + 8 * i, v);
-#pragma unroll
-                        for (int k = 0; k < 8; ++k) cr_n[8 * i + k] = v[k];
-                    }
-                    if (s_2 <= t) hold_n[i] = __ldcg((const uint4 *)(a.hr + ((size_t)s_2 * B + grow) * H + u0 + 8 * i));
-                }
+                if (s_nxt != t + 1) ld8f_a32(a.hist_c + ((size_t)s_nxt * B + grow) * H + uh, cr_n);
+                if (s_2 <= t) hold_n = __ldcg((const uint4 *)(a.hr + ((size_t)s_2 * B + grow) * H + uh));
             }
             const bool ok = tc::mbar_wait(&c.tfull[b], (t >> 1) & 1, limit, c.abort);
             if (!ok) cl_abort(c, a.err);
             __syncwarp();
             if (tc::bar_any(1, E * 32, !ok || *c.abort)) break;
             tc::tc_fence_after();
-            uint32_t zr[4][U];
-            if (warp_rows) {
+            float z[4][8];  // this lane's units of the four gates' pre-activations
+            {
+                uint32_t zr[4][U];
+                if (warp_rows) {
 #pragma unroll
-                for (int g = 0; g < 4; ++g) tc::tmem_ld16_async(taddr0 + b * kCols + g * U, zr[g]);
-                tc::tmem_wait_ld();
-#pragma unroll
-                for (int h2 = 0; h2 < 2; ++h2) {  // the second issuer's accumulator, two gates at a time
-                    uint32_t z1[2][U];
-#pragma unroll
-                    for (int g = 0; g < 2; ++g) tc::tmem_ld16_async(taddr0 + b * kCols + NB + (2 * h2 + g) * U, z1[g]);
+                    for (int g = 0; g < 4; ++g) tc::tmem_ld16_async(taddr0 + b * kCols + g * U, zr[g]);
                     tc::tmem_wait_ld();
 #pragma unroll
-                    for (int g = 0; g < 2; ++g)
+                    for (int h2 = 0; h2 < 2; ++h2) {  // the second issuer's accumulator, two gates at a time
+                        uint32_t z1[2][U];
 #pragma unroll
-                        for (int j = 0; j < U; ++j)
-                            zr[2 * h2 + g][j] = __float_as_uint(__uint_as_float(zr[2 * h2 + g][j]) + __uint_as_float(z1[g][j]));
+                        for (int g = 0; g < 2; ++g)
+                            tc::tmem_ld16_async(taddr0 + b * kCols + NB + (2 * h2 + g) * U, z1[g]);
+                        tc::tmem_wait_ld();
+#pragma unroll
+                        for (int g = 0; g < 2; ++g)
+#pragma unroll
+                            for (int j = 0; j < U; ++j)
+                                zr[2 * h2 + g][j] =
+                                    __float_as_uint(__uint_as_float(zr[2 * h2 + g][j]) + __uint_as_float(z1[g][j]));
+                    }
                 }
-            }
-            tc::tc_fence_before();
-            __syncwarp();
-            if (lane == 0) tc::mbar_arrive(&c.tempty[b]);
-            // the cell (lanes without a row compute and discard)
-            float cn[U], hn[U], gv[4][U];
+                tc::tc_fence_before();
+                __syncwarp();
+                if (lane == 0) tc::mbar_arrive(&c.tempty[b]);
 #pragma unroll
-            for (int j = 0; j < U; ++j) {
-                const float ig = sigm(__uint_as_float(zr[0][j]) + s_bias[j]);
-                const float fg = sigm(__uint_as_float(zr[1][j]) + s_bias[U + j]);
-                const float gg = tanh_hw(__uint_as_float(zr[2][j]) + s_bias[2 * U + j]);
-                const float og = sigm(__uint_as_float(zr[3][j]) + s_bias[3 * U + j]);
+                for (int g = 0; g < 4; ++g)
+#pragma unroll
+                    for (int j = 0; j < 8; ++j) {
+                        const uint32_t up = __shfl_sync(0xffffffffu, zr[g][8 + j], lane & 15);
+                        z[g][j] = __uint_as_float(hf ? up : zr[g][j]);
+                    }
+            }
+            // the cell (lanes without a row compute and discard)
+            float cn[8], hn[8], gv[4][8];
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+                const float ig = sigm(z[0][j] + bias_h[j]);
+                const float fg = sigm(z[1][j] + bias_h[U + j]);
+                const float gg = tanh_hw(z[2][j] + bias_h[2 * U + j]);
+                const float og = sigm(z[3][j] + bias_h[3 * U + j]);
                 cn[j] = fmaf(fg, crv[j], ig * gg);
                 hn[j] = og * tanh_hw(cn[j]);
                 gv[0][j] = ig; gv[1][j] = fg; gv[2][j] = gg; gv[3][j] = og;
             }
             const bool is_new = s_nxt == t + 1;  // step t pushed: h' is the next step's operand
-            uint4 hb[2], hop[2];
-#pragma unroll
-            for (int i = 0; i < 2; ++i) {
-                hb[i] = pack8_bf16(*(const float(*)[8])(hn + 8 * i));
-                hop[i] = is_new ? hb[i] : hold[i];
-            }
+            const uint4 hb = pack8_bf16(hn), hop = is_new ? hb : hold;
             if (t + 1 < T)
-                deliver_slice(c, gscr + ((size_t)(t + 1) * n_ct + ct) * kSlice, (t + 1) & 1, row, hop, v0, v1, ct, n_ct,
-                              tid);
-            if (v0) {
+                deliver_slice(c, gscr + ((size_t)(t + 1) * n_ct + ct) * kSlice, (t + 1) & 1, row, hf,
+                              vh ? hop : make_uint4(0u, 0u, 0u, 0u), ct, n_ct, tid);
+            if (vh) {
                 // history row t + 1, the h operand row t + 1 (for the weight gradient), the gates
-                const size_t w = ((size_t)(t + 1) * B + grow) * H + u0;
+                const size_t w = ((size_t)(t + 1) * B + grow) * H + uh;
+                *(uint4 *)(a.hist_h + w) = hb;
+                *(uint4 *)(a.hr + w) = hop;
+                st8f_a32(a.hist_c + w, cn);
+                // this CTA's 4 x 16 gates of the row: one 128-byte block ([gate][16 units]) or
+                // the row-major [4][H] layout
+                __half *gt = a.gates_blk ? a.gates + (((size_t)t * B + grow) * n_ct + ct) * 4 * U + 8 * hf
+                                         : a.gates + ((size_t)t * B + grow) * 4 * H + uh;
+                const size_t gs = a.gates_blk ? (size_t)U : (size_t)H;  // gate stride
 #pragma unroll
-                for (int i = 0; i < 2; ++i) {
-                    if (i == 1 && !v1) break;
-                    *(uint4 *)(a.hist_h + w + 8 * i) = hb[i];
-                    *(uint4 *)(a.hr + w + 8 * i) = hop[i];
-                    st8f_a32(a.hist_c + w + 8 * i, *(const float(*)[8])(cn + 8 * i));
-                }
-                if (a.gates_blk) {
-                    // this CTA's 4 x 16 gates of the row: one 128-byte block, a 32-byte store a gate
-                    __half *gt = a.gates + (((size_t)t * B + grow) * n_ct + ct) * 4 * U;
-#pragma unroll
-                    for (int g = 0; g < 4; ++g) {
-                        const uint4 lo = pack8_f16(*(const float(*)[8])(gv[g])), hi = pack8_f16(*(const float(*)[8])(gv[g] + 8));
-                        const uint32_t q[8] = {lo.x, lo.y, lo.z, lo.w, hi.x, hi.y, hi.z, hi.w};
-                        st8u_a32(gt + g * U, q);
-                    }
-                } else {
-                    __half *gt = a.gates + ((size_t)t * B + grow) * 4 * H + u0;
-#pragma unroll
-                    for (int i = 0; i < 2; ++i) {
-                        if (i == 1 && !v1) break;
-#pragma unroll
-                        for (int g = 0; g < 4; ++g)
-                            *(uint4 *)(gt + (size_t)g * H + 8 * i) = pack8_f16(*(const float(*)[8])(gv[g] + 8 * i));
-                    }
-                }
+                for (int g = 0; g < 4; ++g) *(uint4 *)(gt + g * gs) = pack8_f16(gv[g]);
             }
             if (t + 1 < T) {
 #pragma unroll
-                for (int i = 0; i < 2; ++i) {
-#pragma unroll
-                    for (int k = 0; k < 8; ++k) crv[8 * i + k] = s_nxt == t + 1 ? cn[8 * i + k] : cr_n[8 * i + k];
-                    hold[i] = s_2 == t + 1 ? hb[i] : hold_n[i];
-                }
+                for (int k = 0; k < 8; ++k) crv[k] = s_nxt == t + 1 ? cn[k] : cr_n[k];
+                hold = s_2 == t + 1 ? hb : hold_n;
                 s_nxt = s_2;
                 s_2 = s_3;
             }
