@@ -161,7 +161,7 @@ sl_status fwd_begin(stacklstm *s, const sl_forward_args &a)
     if (overlap && (e = cudaEventRecord(s->aux_go, s->stream))) return cuda_fail(s, e, "forward setup");
     {
         Phase ph(s, SL_PHASE_PREPASS);
-        if ((e = sl::launch_prepass(s, a.ops))) return cuda_fail(s, e, "prepass");
+        if ((e = sl::launch_prepass(s, a.ops, a.p_final))) return cuda_fail(s, e, "prepass");
         s->Tr = s->T;
         // push-only mode: each instance's pushes as a virtual timeline
         if (s->push_only && (e = sl::launch_compact(s))) return cuda_fail(s, e, "push-only indices");
@@ -234,7 +234,7 @@ sl_status fwd_end(stacklstm *s, const sl_forward_args &a)
     cudaError_t e;
     {
         Phase ph(s, SL_PHASE_OUTPUTS);
-        if ((e = cudaMemcpyAsync(a.p_final, s->p_traj + (size_t)T * B, sizeof(int32_t) * B,
+        if (!s->pfinal_written && (e = cudaMemcpyAsync(a.p_final, s->p_traj + (size_t)T * B, sizeof(int32_t) * B,
                                  cudaMemcpyDeviceToDevice, s->stream)))
             return cuda_fail(s, e, "p_final");
         if (a.p_traj && (e = cudaMemcpyAsync(a.p_traj, s->p_traj, sizeof(int32_t) * (T + 1) * B,

@@ -54,6 +54,7 @@ struct stacklstm {
     int prepass_smem = 0;  // dynamic shared memory of the index prepass (0: global scratch)
     int walk_push_smem = 0;      // the same for the push-only walk (slot tags and index map; 0: separate kernels)
     int walk_built_virtual = 0;  // the last prepass also built the push-only timeline
+    int pfinal_written = 0;      // the last prepass also wrote the caller's final pointers
 
     // integer bookkeeping, written by the prepass (all [T+1][B] int32)
     int32_t *p_traj = nullptr;     // pointer before step t (t = T: after the last step)
@@ -141,7 +142,9 @@ struct stacklstm {
 namespace sl {
 
 // ---- index / gather kernels (index_kernels.cu)
-cudaError_t launch_prepass(stacklstm *s, const int8_t *ops);
+// also writes the final pointers to p_final (if given) when the walk runs on chip
+// (s->pfinal_written)
+cudaError_t launch_prepass(stacklstm *s, const int8_t *ops, int32_t *p_final);
 // Raise kernel `fn`'s dynamic shared-memory limit on the current device to at least
 // `bytes`. The limit belongs to the function, not to a handle, so handles of different
 // sizes (created in any order, used from any stream) only ever raise it.

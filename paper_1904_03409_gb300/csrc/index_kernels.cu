@@ -68,6 +68,7 @@ prepass_kernel(int T, int B, const int8_t *__restrict__ ops, int32_t *__restrict
 struct VirtOut {
     int32_t *vtop, *vy, *vslot, *xidx, *vstep, *kmax;
 };
+// (both walks also write the caller's final pointers, p_final, when it is given)
 
 // The same walk as prepass_kernel with the slot-tag stack in shared memory, its ops loaded
 // 32 steps ahead. With kPush it also builds the push-only mode's virtual timeline in the
@@ -77,7 +78,8 @@ struct VirtOut {
 template <bool kPush>
 __global__ void __launch_bounds__(kPrepassThreads)
 prepass_walk_kernel(int T, int B, const int8_t *__restrict__ ops, int32_t *__restrict__ p_traj,
-                    int32_t *__restrict__ top, int32_t *__restrict__ slot_last, int32_t *__restrict__ err, VirtOut v)
+                    int32_t *__restrict__ top, int32_t *__restrict__ slot_last, int32_t *__restrict__ err, VirtOut v,
+                    int32_t *__restrict__ p_final)
 {
     constexpr int kBlk = 32;
     extern __shared__ int32_t s_tag[];  // [T + 1][32] slot tags, then (kPush) [T + 1][32] vmap
@@ -145,6 +147,7 @@ prepass_walk_kernel(int T, int B, const int8_t *__restrict__ ops, int32_t *__res
     const int tp = tag(p);
     p_traj[(size_t)T * B + b] = p;
     top[(size_t)T * B + b] = tp;
+    if (p_final) p_final[b] = p;
     for (int slot = 0; slot <= T; ++slot) slot_last[(size_t)slot * B + b] = tag(slot);
     if (kPush) {
         v.vy[(size_t)T * B + b] = max(0, vmap(tp));
@@ -170,7 +173,7 @@ template <bool kPush>
 __global__ void __launch_bounds__(kPrepassThreads)
 prepass_walk_vec_kernel(int T, int B, const int8_t *__restrict__ ops, int32_t *__restrict__ p_traj,
                         int32_t *__restrict__ top, int32_t *__restrict__ slot_last, int32_t *__restrict__ err,
-                        VirtOut v)
+                        VirtOut v, int32_t *__restrict__ p_final)
 {
     constexpr int kBlk = 32;
     // [T + 1][32] slot tags, (kPush) [T + 1][32] vmap, then the block staging:
@@ -263,6 +266,7 @@ prepass_walk_vec_kernel(int T, int B, const int8_t *__restrict__ ops, int32_t *_
     const int tp = tag(p);
     p_traj[(size_t)T * B + b] = p;
     top[(size_t)T * B + b] = tp;
+    if (p_final) p_final[b] = p;
     if (kPush) {
         v.vy[(size_t)T * B + b] = max(0, vmap(tp));
         atomicMax(v.kmax, k);
@@ -496,10 +500,11 @@ cudaError_t configure_prepass(stacklstm *s)
     return cudaSuccess;
 }
 
-cudaError_t launch_prepass(stacklstm *s, const int8_t *ops)
+cudaError_t launch_prepass(stacklstm *s, const int8_t *ops, int32_t *p_final)
 {
     const unsigned grid = ceil_div(s->B, kPrepassThreads);
     s->walk_built_virtual = 0;
+    s->pfinal_written = s->prepass_smem > 0;  // the walks write it; prepass_kernel does not
     // whole 32-instance blocks and word-aligned ops: the walk's traffic in 16-byte pieces
     const bool vec = s->B % kPrepassThreads == 0 && ((uintptr_t)ops & 3) == 0;
     if (s->push_only && s->walk_push_smem > 0) {
@@ -508,18 +513,18 @@ cudaError_t launch_prepass(stacklstm *s, const int8_t *ops)
         const VirtOut v{s->vtop, s->vy, s->vslot, s->xidx, s->vstep, s->kmax};
         if (vec)
             prepass_walk_vec_kernel<true><<<grid, kPrepassThreads, s->walk_push_smem + kWalkStageBytes, s->stream>>>(
-                s->T, s->B, ops, s->p_traj, s->top, s->slot_last, s->err, v);
+                s->T, s->B, ops, s->p_traj, s->top, s->slot_last, s->err, v, p_final);
         else
             prepass_walk_kernel<true><<<grid, kPrepassThreads, s->walk_push_smem, s->stream>>>(
-                s->T, s->B, ops, s->p_traj, s->top, s->slot_last, s->err, v);
+                s->T, s->B, ops, s->p_traj, s->top, s->slot_last, s->err, v, p_final);
         s->walk_built_virtual = 1;
     } else if (s->prepass_smem > 0) {
         if (vec)
             prepass_walk_vec_kernel<false><<<grid, kPrepassThreads, s->prepass_smem + kWalkStageBytes, s->stream>>>(
-                s->T, s->B, ops, s->p_traj, s->top, s->slot_last, s->err, VirtOut{});
+                s->T, s->B, ops, s->p_traj, s->top, s->slot_last, s->err, VirtOut{}, p_final);
         else
             prepass_walk_kernel<false><<<grid, kPrepassThreads, s->prepass_smem, s->stream>>>(
-                s->T, s->B, ops, s->p_traj, s->top, s->slot_last, s->err, VirtOut{});
+                s->T, s->B, ops, s->p_traj, s->top, s->slot_last, s->err, VirtOut{}, p_final);
     } else {
         prepass_kernel<<<grid, kPrepassThreads, 0, s->stream>>>(s->T, s->B, ops, s->p_traj, s->top, s->slot_last,
                                                                 s->slot_scratch, s->err);
