@@ -451,15 +451,18 @@ __global__ void setup_kernel(SetupArgs a)
 }
 
 // Push-only mode: the input of each virtual step, x_push[k][b] = x[xidx[k][b]][b] (zero
-// rows past the instance's pushes), 16-byte pieces (I % 8 == 0).
-__global__ void gather_push_x(size_t rows, int B, int I8, const int32_t *__restrict__ xidx, const uint4 *__restrict__ x,
+// rows past the instance's pushes), 16-byte pieces (I % 8 == 0), one a thread. IDX is the
+// index type: 32-bit whenever the pieces number fewer than 2^32 (its divisions are a
+// fraction of the 64-bit ones).
+template <typename IDX>
+__global__ void gather_push_x(IDX rows, IDX B, IDX I8, const int32_t *__restrict__ xidx, const uint4 *__restrict__ x,
                               uint4 *__restrict__ out)
 {
-    const size_t n = rows * I8;
-    for (size_t e = blockIdx.x * (size_t)blockDim.x + threadIdx.x; e < n; e += (size_t)gridDim.x * blockDim.x) {
-        const size_t r = e / I8;
+    const IDX n = rows * I8;
+    for (IDX e = blockIdx.x * (IDX)blockDim.x + threadIdx.x; e < n; e += (IDX)gridDim.x * blockDim.x) {
+        const IDX r = e / I8;
         const int t = xidx[r];
-        out[e] = t >= 0 ? x[((size_t)t * B + r % B) * I8 + e % I8] : make_uint4(0u, 0u, 0u, 0u);
+        out[e] = t >= 0 ? x[((size_t)t * B + r % B) * I8 + (e - r * I8)] : make_uint4(0u, 0u, 0u, 0u);
     }
 }
 
@@ -787,8 +790,14 @@ cudaError_t bf16_forward_setup_state(stacklstm *s, const __nv_bfloat16 *h0, cons
 cudaError_t bf16_gather_push_x(stacklstm *s, const __nv_bfloat16 *x)
 {
     const size_t rows = (size_t)s->Tr * s->B;
-    gather_push_x<<<grid_for(s, rows * (s->I / 8)), 256, 0, s->stream>>>(rows, s->B, s->I / 8, s->xidx,
-                                                                          (const uint4 *)x, (uint4 *)s->x_push);
+    const size_t n = rows * (s->I / 8);
+    if (n < ((size_t)1 << 32) - (size_t)s->num_sms * 16 * 256)
+        gather_push_x<uint32_t><<<grid_for(s, n), 256, 0, s->stream>>>((uint32_t)rows, (uint32_t)s->B,
+                                                                        (uint32_t)(s->I / 8), s->xidx,
+                                                                        (const uint4 *)x, (uint4 *)s->x_push);
+    else
+        gather_push_x<size_t><<<grid_for(s, n), 256, 0, s->stream>>>(rows, (size_t)s->B, (size_t)(s->I / 8), s->xidx,
+                                                                      (const uint4 *)x, (uint4 *)s->x_push);
     s->launches += 1;
     return cudaGetLastError();
 }

@@ -407,12 +407,18 @@ compact_kernel(int T, int B, const int32_t *__restrict__ p_traj, const int32_t *
 
 // Push-only mode: dx rows of the steps that do not push are zero (a state no step reads
 // has zero gradient); the push rows are written by the input-gradient contraction.
+// A warp per row: the row's step index is read once, its 16-byte pieces written by the
+// warp's lanes side by side.
 __global__ void zero_nonpush_rows_kernel(size_t rows, int I4, const int32_t *__restrict__ vstep,
                                          float4 *__restrict__ dx)
 {
-    const size_t n = rows * I4;
-    for (size_t e = blockIdx.x * (size_t)blockDim.x + threadIdx.x; e < n; e += (size_t)gridDim.x * blockDim.x)
-        if (vstep[e / I4] < 0) dx[e] = make_float4(0.f, 0.f, 0.f, 0.f);
+    const int lane = threadIdx.x & 31;
+    const size_t warps = (size_t)gridDim.x * (blockDim.x >> 5);
+    for (size_t r = (size_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); r < rows; r += warps) {
+        if (vstep[r] >= 0) continue;
+        float4 *row = dx + r * I4;
+        for (int i = lane; i < I4; i += 32) row[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+    }
 }
 
 }  // namespace
@@ -454,7 +460,7 @@ cudaError_t launch_zero_nonpush_rows(stacklstm *s, float *dx)
     if (!dx) return cudaSuccess;
     const size_t rows = (size_t)s->T * s->B;
     const int I4 = s->I / 4;  // the bf16 path has I % 8 == 0
-    const unsigned grid = (unsigned)std::min<size_t>(ceil_div(rows * I4, 256), (size_t)s->num_sms * 16);
+    const unsigned grid = (unsigned)std::max<size_t>(1, std::min<size_t>(ceil_div(rows, 8), (size_t)s->num_sms * 16));
     zero_nonpush_rows_kernel<<<grid, 256, 0, s->stream>>>(rows, I4, s->vstep, (float4 *)dx);
     s->launches += 1;
     return cudaGetLastError();
