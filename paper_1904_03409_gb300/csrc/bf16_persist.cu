@@ -401,8 +401,8 @@ __device__ __forceinline__ void epilogue_loop(const StepArgs &a, const WsArgs &p
             if (k >= e.n_mine) {
                 // c' leaves by tensor store: the stores of this row tile's previous step
                 // (n_mine tiles back, so every group but possibly the latest) have completed
-                // before its rows are read back
-                if (e.tid == 0) {
+                // before its rows are read back (each warp's lane 0 issued some of them)
+                if (e.lane == 0) {
                     if (e.n_mine == 1)
                         tc::bulk_wait();
                     else
@@ -420,7 +420,7 @@ __device__ __forceinline__ void epilogue_loop(const StepArgs &a, const WsArgs &p
                 }
             }
             if (pf_early) prefetch_next();
-            if (e.tid == 0) tc::bulk_wait_read();  // the previous tile's gate stores read the staging tile
+            if (e.lane == 0) tc::bulk_wait_read();  // the previous tile's stores read the staging tiles
             const bool ok = tc::mbar_wait(&e.c.tfull[acc], (k >> 1) & 1, e.limit, e.c.abort);
             if (!ok) ws_abort(e.c, a.err);
             __syncwarp();
@@ -759,19 +759,24 @@ __device__ __forceinline__ void epilogue_loop(const StepArgs &a, const WsArgs &p
             }
         }
         if constexpr (kFwd) {
-            if (e.tid == 0) {
-#pragma unroll
-                for (int g = 0; g < 4; ++g)
-#pragma unroll
-                    for (int q = 0; q < EP; ++q)
+            // the tile's 6 EP tensor stores (4 EP gate blocks, EP h' and EP c' blocks), issued
+            // by lane 0 of the epilogue warps, store w, w + E, ... each
+            if (e.lane == 0) {
+                const int w = e.part * 4 + e.q;
+                for (int st = w; st < 6 * EP; st += E) {
+                    if (st < 4 * EP) {
+                        const int g = st / EP, q = st % EP;
                         tc::tma_store_4d(tm_gates, e.c.stg + (uint32_t)((g * EP + q) * kRows * UE * 2),
                                          e.ct * U + q * UE, g, rt * kRows, t);
-#pragma unroll
-                for (int q = 0; q < EP; ++q) {
-                    tc::tma_store_3d(tm_hh, e.c.stg + 8u * U * kRows + (uint32_t)(q * kRows * UE * 2), e.ct * U + q * UE,
-                                     rt * kRows, t + 1);
-                    tc::tma_store_3d(tm_hc, e.c.stg + 10u * U * kRows + (uint32_t)(q * kRows * UE * 4),
-                                     e.ct * U + q * UE, rt * kRows, t + 1);
+                    } else if (st < 5 * EP) {
+                        const int q = st - 4 * EP;
+                        tc::tma_store_3d(tm_hh, e.c.stg + 8u * U * kRows + (uint32_t)(q * kRows * UE * 2),
+                                         e.ct * U + q * UE, rt * kRows, t + 1);
+                    } else {
+                        const int q = st - 5 * EP;
+                        tc::tma_store_3d(tm_hc, e.c.stg + 10u * U * kRows + (uint32_t)(q * kRows * UE * 4),
+                                         e.ct * U + q * UE, rt * kRows, t + 1);
+                    }
                 }
                 tc::bulk_commit();
             }
@@ -780,7 +785,7 @@ __device__ __forceinline__ void epilogue_loop(const StepArgs &a, const WsArgs &p
         cur1 = nx1;
     }
     if constexpr (kFwd)
-        if (e.tid == 0) tc::bulk_wait();  // the history stores completed before the CTA exits
+        if (e.lane == 0) tc::bulk_wait();  // the history stores completed before the CTA exits
 }
 
 // ------------------------------------------------------------------ input gradient
