@@ -46,7 +46,7 @@
  *                                  (default 4e9); 0 makes every wait run out at once, so
  *                                  calls report SL_ERR_TIMEOUT
  *   STACKLSTM_STEP_KERNELS=1       one launch per time step instead of the persistent and
- *                                  cluster kernels
+ *                                  cluster kernels (fp32: instead of one CTA for all steps)
  *   STACKLSTM_FWD_CLUSTER=0        no thread-block-cluster forward for one row tile
  *   STACKLSTM_BWD_CLUSTER=0        no thread-block-cluster backward for one row tile
  *   STACKLSTM_BWD_SPLIT=k          the persistent backward with its 4H contraction split

@@ -153,12 +153,10 @@ sl_status fwd_begin(stacklstm *s, const sl_forward_args &a)
         if (p && !aligned16(p)) return fail(s, SL_ERR_ARG, "tensor pointers must be 16-byte aligned");
     cudaError_t e;
     s->fwd_done = 0;
-    // bf16: the initial state and the weight packing do not depend on the index prepass, so
-    // they run on the side stream at the same time (launched after the prepass, whose few
-    // blocks then reach the SMs first); the caller's stream waits for them before the
-    // forward steps
-    const bool overlap = s->dt == SL_BF16;
-    if (overlap && (e = cudaEventRecord(s->aux_go, s->stream))) return cuda_fail(s, e, "forward setup");
+    // the initial state and the weight packing do not depend on the index prepass, so they
+    // run on the side stream at the same time (launched after the prepass, whose few blocks
+    // then reach the SMs first); the caller's stream waits for them before the forward steps
+    if ((e = cudaEventRecord(s->aux_go, s->stream))) return cuda_fail(s, e, "forward setup");
     {
         Phase ph(s, SL_PHASE_PREPASS);
         if ((e = sl::launch_prepass(s, a.ops, a.p_final))) return cuda_fail(s, e, "prepass");
@@ -166,13 +164,15 @@ sl_status fwd_begin(stacklstm *s, const sl_forward_args &a)
         // push-only mode: each instance's pushes as a virtual timeline
         if (s->push_only && (e = sl::launch_compact(s))) return cuda_fail(s, e, "push-only indices");
     }
-    if (overlap) {
+    {
         if ((e = cudaStreamWaitEvent(s->side, s->aux_go, 0))) return cuda_fail(s, e, "forward setup");
         const cudaStream_t main = s->stream;
         s->stream = s->side;
         {
             Phase ph(s, SL_PHASE_FWD_SETUP);
-            e = sl::bf16_forward_setup_state(s, (const __nv_bfloat16 *)a.h0, a.c0, (const __nv_bfloat16 *)a.W);
+            e = s->dt == SL_BF16
+                    ? sl::bf16_forward_setup_state(s, (const __nv_bfloat16 *)a.h0, a.c0, (const __nv_bfloat16 *)a.W)
+                    : sl::fp32_forward_setup(s, (const float *)a.h0, a.c0, (const float *)a.W);
         }
         s->stream = main;
         if (e) return cuda_fail(s, e, "forward setup");
@@ -184,16 +184,13 @@ sl_status fwd_begin(stacklstm *s, const sl_forward_args &a)
         Phase ph(s, SL_PHASE_PREPASS);
         if ((e = sl::read_virtual_steps(s))) return cuda_fail(s, e, "push-only indices");
     }
-    {
+    if (s->dt == SL_BF16) {
         Phase ph(s, SL_PHASE_FWD_SETUP);
-        // push-only mode: the virtual steps' inputs, gathered after the compaction
-        if (overlap)
-            e = sl::bf16_forward_setup_x(s, (const __nv_bfloat16 *)a.x);
-        else
-            e = sl::fp32_forward_setup(s, (const float *)a.h0, a.c0, (const float *)a.W);
-        if (e) return cuda_fail(s, e, "forward setup");
+        // the x tensor maps (push-only mode: the virtual steps' inputs, gathered after the
+        // compaction)
+        if ((e = sl::bf16_forward_setup_x(s, (const __nv_bfloat16 *)a.x))) return cuda_fail(s, e, "forward setup");
     }
-    if (overlap && (e = cudaStreamWaitEvent(s->stream, s->aux_done, 0))) return cuda_fail(s, e, "forward setup");
+    if ((e = cudaStreamWaitEvent(s->stream, s->aux_done, 0))) return cuda_fail(s, e, "forward setup");
     return SL_OK;
 }
 
@@ -299,9 +296,9 @@ sl_status bwd_end(stacklstm *s, const sl_backward_args &a, bool dx_done)
 {
     const int B = s->B, H = s->H;
     cudaError_t e;
-    // bf16: dx and dW both only read the gate gradients, so dx runs on the side stream at
-    // the same time as dW; the caller's stream waits for it
-    const bool side_dx = !dx_done && a.dx && s->dt == SL_BF16;
+    // dx and dW both only read the gate gradients, so dx runs on the side stream at the same
+    // time as dW; the caller's stream waits for it
+    const bool side_dx = !dx_done && a.dx;
     if (side_dx) {
         if ((e = cudaEventRecord(s->aux_go, s->stream)) || (e = cudaStreamWaitEvent(s->side, s->aux_go, 0)))
             return cuda_fail(s, e, "dx");
@@ -309,7 +306,7 @@ sl_status bwd_end(stacklstm *s, const sl_backward_args &a, bool dx_done)
         s->stream = s->side;
         {
             Phase ph(s, SL_PHASE_DX);
-            e = sl::bf16_dx(s, a.dx);
+            e = s->dt == SL_FP32 ? sl::fp32_dx(s, a.dx) : sl::bf16_dx(s, a.dx);
         }
         s->stream = main;
         if (e) return cuda_fail(s, e, "dx");
@@ -441,7 +438,7 @@ sl_status stacklstm_create(stacklstm_t *out, int T, int B, int I, int H, sl_dtyp
         delete s;
         return SL_ERR_OOM;
     }
-    s->plan = dtype == SL_BF16 ? sl::bf16_describe(s) : "fp32 CUDA cores; one launch per step";
+    s->plan = dtype == SL_BF16 ? sl::bf16_describe(s) : sl::fp32_describe(s);
     *out = s;
     return SL_OK;
 }

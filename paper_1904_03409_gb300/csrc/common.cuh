@@ -54,6 +54,7 @@ struct stacklstm {
     int prepass_smem = 0;  // dynamic shared memory of the index prepass (0: global scratch)
     int walk_push_smem = 0;      // the same for the push-only walk (slot tags and index map; 0: separate kernels)
     int walk_built_virtual = 0;  // the last prepass also built the push-only timeline
+    int fp32_one_cta = 0;        // fp32: every step of each direction in one CTA (small B * H)
     int pfinal_written = 0;      // the last prepass also wrote the caller's final pointers
 
     // integer bookkeeping, written by the prepass (all [T+1][B] int32)
@@ -160,6 +161,8 @@ cudaError_t read_virtual_steps(stacklstm *s);
 cudaError_t launch_zero_nonpush_rows(stacklstm *s, float *dx);
 
 // ---- fp32 CUDA-core path (fp32_path.cu)
+// plans the fp32 path (s->fp32_one_cta) and describes it
+std::string fp32_describe(stacklstm *s);
 cudaError_t fp32_forward_setup(stacklstm *s, const float *h0, const float *c0, const float *W);
 cudaError_t fp32_forward_steps(stacklstm *s, const float *x, const float *W, const float *bias);
 cudaError_t fp32_backward_steps(stacklstm *s);

@@ -1,6 +1,7 @@
 // fp32_path.cu -- the fp32 homogenized StackLSTM step on CUDA cores (no tensor cores,
 // no TF32). It serves small problems, where B * 4H is too small for a dense tensor-core
-// contraction, and is the full-precision counterpart of the bf16 path.
+// contraction, and is the full-precision counterpart of the bf16 path. With B * H <= 1024
+// each direction runs all its steps in one CTA (fwd_seq_f32, bwd_seq_f32); otherwise:
 //
 // Forward, one launch per step t (Algorithm 1): every instance reads history row
 // top[t] (the state at its stack top), computes z = [x_t ; h_read] W + bias, applies the
@@ -11,7 +12,10 @@
 // gradient history has exactly one writer per launch, so no atomics are needed and the
 // summation order is fixed. dx = dG W_x^T, dW = [x ; h_read]^T dG and dbias = sum dG are
 // taken after the loop in a fixed order.
+#include <stdlib.h>
+
 #include <algorithm>
+#include <string>
 
 #include "common.cuh"
 
@@ -155,12 +159,174 @@ __global__ void dw_f32(size_t R, int K, int G, const float *__restrict__ a_rm, c
     }
 }
 
+// Small problems (B * H <= 1024 threads, and the whole history in shared memory): all T
+// steps of a direction in one CTA, thread (b, j) = (tid / H, tid % H), __syncthreads()
+// between the phases of a step instead of a launch per step, and every row a step reads
+// taken from shared memory (the rows go to global memory as they are written). The
+// arithmetic of each element is that of the per-step kernels above (the same operands, k
+// and n ascending with fmaf), so both give the same bits.
+// Shared memory: forward [B][K] operands, [K][4H] W, [T+1][B][H] h and c, [T][B][I] x,
+// [T+1][B] tops;
+// backward [4H][H] W_h^T, [T+1][B][H] c, dh and dc, [B][4H] the step's dG, [T+1][B] tops.
+size_t fwd_seq_smem(int T, int B, int I, int H)
+{
+    const size_t K = (size_t)I + H, G = 4 * (size_t)H, R = (size_t)(T + 1) * B;
+    return sizeof(float) * ((size_t)B * K + K * G + 2 * R * H + (size_t)T * B * I) + sizeof(int32_t) * R;
+}
+size_t bwd_seq_smem(int T, int B, int H)
+{
+    const size_t G = 4 * (size_t)H, R = (size_t)(T + 1) * B;
+    return sizeof(float) * (G * H + 3 * R * H + (size_t)B * G) + sizeof(int32_t) * R;
+}
+
+__global__ void __launch_bounds__(1024) fwd_seq_f32(int T, int B, int I, int H, const float *__restrict__ x,
+                                                    const float *__restrict__ W, const float *__restrict__ bias,
+                                                    const int32_t *__restrict__ top, float *__restrict__ hist_h,
+                                                    float *__restrict__ hist_c, float *__restrict__ gates,
+                                                    float *__restrict__ a_rm)
+{
+    extern __shared__ float sm[];
+    const int K = I + H, G = 4 * H, tid = threadIdx.x, b = tid / H, j = tid - b * H;
+    const bool mine = tid < B * H;
+    const size_t R = (size_t)(T + 1) * B;
+    float *a_s = sm, *w_s = a_s + (size_t)B * K, *h_s = w_s + (size_t)K * G, *c_s = h_s + R * H;
+    float *x_s = c_s + R * H;
+    int32_t *top_s = (int32_t *)(x_s + (size_t)T * B * I);
+    for (size_t e = tid; e < (size_t)K * G; e += blockDim.x) w_s[e] = W[e];
+    for (size_t e = tid; e < (size_t)T * B * I; e += blockDim.x) x_s[e] = x[e];
+    for (size_t e = tid; e < R; e += blockDim.x) top_s[e] = top[e];
+    for (int e = tid; e < B * H; e += blockDim.x) {  // row 0: the initial state
+        h_s[e] = hist_h[e];
+        c_s[e] = hist_c[e];
+    }
+    __syncthreads();
+    for (int t = 0; t < T; ++t) {
+        for (int e = tid; e < B * K; e += blockDim.x) {
+            const int bb = e / K, k = e - bb * K;
+            const int src = top_s[t * B + bb];
+            const float v = k < I ? x_s[((size_t)t * B + bb) * I + k] : h_s[((size_t)src * B + bb) * H + (k - I)];
+            a_s[e] = v;
+            a_rm[((size_t)t * B + bb) * K + k] = v;
+        }
+        __syncthreads();
+        if (mine) {
+            const float *as = a_s + (size_t)b * K;
+            float zi = bias[j], zf = bias[H + j], zg = bias[2 * H + j], zo = bias[3 * H + j];
+            for (int k = 0; k < K; ++k) {
+                const float av = as[k];
+                const float *Wk = w_s + (size_t)k * G;
+                zi = fmaf(av, Wk[j], zi);
+                zf = fmaf(av, Wk[H + j], zf);
+                zg = fmaf(av, Wk[2 * H + j], zg);
+                zo = fmaf(av, Wk[3 * H + j], zo);
+            }
+            const float ig = sigmoidf(zi), fg = sigmoidf(zf), gg = tanhf(zg), og = sigmoidf(zo);
+            const int src = top_s[t * B + b];
+            const float cr = c_s[((size_t)src * B + b) * H + j];
+            const float cn = fmaf(fg, cr, ig * gg);
+            const float hn = og * tanhf(cn);
+            const size_t w = ((size_t)(t + 1) * B + b) * H + j;
+            h_s[w] = hn;
+            c_s[w] = cn;
+            hist_h[w] = hn;
+            hist_c[w] = cn;
+            float *gt = gates + ((size_t)t * B + b) * G;
+            gt[j] = ig;
+            gt[H + j] = fg;
+            gt[2 * H + j] = gg;
+            gt[3 * H + j] = og;
+        }
+        __syncthreads();  // row t + 1 is complete before a later step reads it
+    }
+}
+
+__global__ void __launch_bounds__(1024) bwd_seq_f32(int T, int B, int I, int H, const int32_t *__restrict__ top,
+                                                    const float *__restrict__ gates, const float *__restrict__ hist_c,
+                                                    const float *__restrict__ WT, float *__restrict__ dhist_h,
+                                                    float *__restrict__ dhist_c, float *__restrict__ dG)
+{
+    extern __shared__ float sm[];
+    const int K = I + H, G = 4 * H, tid = threadIdx.x, b = tid / H, j = tid - b * H;
+    const bool mine = tid < B * H;
+    const size_t R = (size_t)(T + 1) * B;
+    float *wh_s = sm, *c_s = wh_s + (size_t)G * H, *dh_s = c_s + R * H, *dc_s = dh_s + R * H;
+    float *dg_s = dc_s + R * H;  // [B][4H]: dG of the current step
+    int32_t *top_s = (int32_t *)(dg_s + (size_t)B * G);
+    for (int e = tid; e < G * H; e += blockDim.x) wh_s[e] = WT[(size_t)(e / H) * K + I + e % H];
+    for (size_t e = tid; e < R * H; e += blockDim.x) {
+        c_s[e] = hist_c[e];
+        dh_s[e] = dhist_h[e];  // the seeded loss gradients (zero elsewhere)
+        dc_s[e] = dhist_c[e];
+    }
+    for (size_t e = tid; e < R; e += blockDim.x) top_s[e] = top[e];
+    // this thread's four activated gates of the next step processed (loaded a step ahead)
+    float gn[4] = {0.f, 0.f, 0.f, 0.f};
+    if (mine && T >= 1)
+        for (int g = 0; g < 4; ++g) gn[g] = gates[((size_t)(T - 1) * B + b) * G + g * H + j];
+    __syncthreads();
+    for (int t = T - 1; t >= 0; --t) {
+        const int src = mine ? top_s[t * B + b] : 0;
+        if (mine) {
+            // pointwise backward of step t (bwd_pointwise_f32)
+            const float ig = gn[0], fg = gn[1], gg = gn[2], og = gn[3];
+            if (t >= 1)
+                for (int g = 0; g < 4; ++g) gn[g] = gates[((size_t)(t - 1) * B + b) * G + g * H + j];
+            const size_t wr = ((size_t)(t + 1) * B + b) * H + j, rd = ((size_t)src * B + b) * H + j;
+            const float dh = dh_s[wr], dcn = dc_s[wr];
+            const float tc = tanhf(c_s[wr]);
+            const float dc = dcn + dh * og * (1.0f - tc * tc);
+            float *dg = dg_s + (size_t)b * G;
+            float *dgo = dG + ((size_t)t * B + b) * G;
+            dgo[j] = dg[j] = dc * gg * ig * (1.0f - ig);
+            dgo[H + j] = dg[H + j] = dc * c_s[rd] * fg * (1.0f - fg);
+            dgo[2 * H + j] = dg[2 * H + j] = dc * ig * (1.0f - gg * gg);
+            dgo[3 * H + j] = dg[3 * H + j] = dh * tc * og * (1.0f - og);
+            dc_s[rd] += dc * fg;
+        }
+        __syncthreads();  // dG_t complete
+        if (mine) {
+            // dh_read = dG_t W_h^T added to the row step t read (bwd_contract_f32)
+            const float *dg = dg_s + (size_t)b * G;
+            float acc = 0.0f;
+            for (int n = 0; n < G; ++n) acc = fmaf(dg[n], wh_s[n * H + j], acc);
+            dh_s[((size_t)src * B + b) * H + j] += acc;
+        }
+        __syncthreads();  // the row's gradient is complete before step t - 1 reads it
+    }
+    // out: the gradient history (rows 0..T: dh0, dc0 among them)
+    for (size_t e = tid; e < R * H; e += blockDim.x) {
+        dhist_h[e] = dh_s[e];
+        dhist_c[e] = dc_s[e];
+    }
+}
+
 unsigned grid_for(const stacklstm *s, size_t n, int threads)
 {
     return (unsigned)std::max<size_t>(1, std::min<size_t>(ceil_div(n, threads), (size_t)s->num_sms * 32));
 }
 
 }  // namespace
+
+std::string fp32_describe(stacklstm *s)
+{
+    // test hook (include/stacklstm.h): STACKLSTM_STEP_KERNELS=1 keeps one launch per step
+    const char *per_step = getenv("STACKLSTM_STEP_KERNELS");
+    int optin = 0;
+    if (cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, s->device) != cudaSuccess) {
+        cudaGetLastError();
+        optin = 48 * 1024;
+    }
+    const size_t cap = (size_t)optin - 1024;
+    s->fp32_one_cta = s->B * s->H <= 1024 && fwd_seq_smem(s->T, s->B, s->I, s->H) <= cap &&
+                      bwd_seq_smem(s->T, s->B, s->H) <= cap && !(per_step && atoi(per_step) != 0);
+    if (s->fp32_one_cta && (smem_at_least((const void *)fwd_seq_f32, fwd_seq_smem(s->T, s->B, s->I, s->H)) ||
+                            smem_at_least((const void *)bwd_seq_f32, bwd_seq_smem(s->T, s->B, s->H)))) {
+        cudaGetLastError();
+        s->fp32_one_cta = 0;
+    }
+    return s->fp32_one_cta ? "fp32 CUDA cores; every step of each direction in one CTA"
+                           : "fp32 CUDA cores; one launch per step";
+}
 
 cudaError_t fp32_forward_setup(stacklstm *s, const float *h0, const float *c0, const float *W)
 {
@@ -179,6 +345,13 @@ cudaError_t fp32_forward_setup(stacklstm *s, const float *h0, const float *c0, c
 cudaError_t fp32_forward_steps(stacklstm *s, const float *x, const float *W, const float *bias)
 {
     const int T = s->T, B = s->B, I = s->I, H = s->H, K = I + H;
+    if (s->fp32_one_cta) {
+        (void)K;
+        fwd_seq_f32<<<1, (unsigned)ceil_div(B * H, 32) * 32, fwd_seq_smem(T, B, I, H), s->stream>>>(
+            T, B, I, H, x, W, bias, s->top, (float *)s->hist_h, s->hist_c, (float *)s->gates, (float *)s->a_rm);
+        s->launches += 1;
+        return cudaGetLastError();
+    }
     const int threads = std::min(128, ((H + 31) / 32) * 32);
     const dim3 grid(ceil_div(H, threads), B);
     const size_t smem = sizeof(float) * K;
@@ -194,6 +367,12 @@ cudaError_t fp32_backward_steps(stacklstm *s)
     const int T = s->T, B = s->B, I = s->I, H = s->H, G = 4 * H;
     const float *WT = (const float *)s->w_fwd;
     float *dG = (float *)s->dG;
+    if (s->fp32_one_cta) {
+        bwd_seq_f32<<<1, (unsigned)ceil_div(B * H, 32) * 32, bwd_seq_smem(T, B, H), s->stream>>>(T, B, I, H, s->top, (const float *)s->gates,
+                                                                         s->hist_c, WT, s->dhist_h, s->dhist_c, dG);
+        s->launches += 1;
+        return cudaGetLastError();
+    }
     const int threads = std::min(128, ((H + 31) / 32) * 32);
     const unsigned pw_grid = grid_for(s, (size_t)B * H, 256);
     for (int t = T - 1; t >= 0; --t) {

@@ -36,6 +36,35 @@ def test_random_cases(T, B, I, H, seed, probs):
     compare(got, oracle_of(w), "fp32")
 
 
+@pytest.mark.parametrize("T,B,I,H,seed", [(12, 4, 16, 16, 10), (20, 16, 16, 32, 11), (9, 20, 8, 48, 12)])
+def test_one_cta_and_per_step_kernels_agree_bit_for_bit(T, B, I, H, seed):
+    """Small problems run each direction's steps in one CTA; the per-step kernels
+    (STACKLSTM_STEP_KERNELS=1) do the same arithmetic per element, so every output is
+    bit-identical, and both match the oracle."""
+    import os
+    w = wl.make_workload("case", T=T, B=B, I=I, H=H, dtype="fp32", seed=seed, ops_kind="random_walk",
+                         probs=(0.5, 0.3, 0.2), bias_scale=0.3, h0_scale=0.5, c0_scale=0.5, dy_scale=0.5)
+    hd = bd.stacklstm_create(T, B, I, H, bd.SL_FP32, 0)
+    try:
+        assert "one CTA" in bd.stacklstm_plan(hd)
+    finally:
+        hd.destroy()
+    one = runner.run(w)
+    os.environ["STACKLSTM_STEP_KERNELS"] = "1"
+    try:
+        hd = bd.stacklstm_create(T, B, I, H, bd.SL_FP32, 0)
+        try:
+            assert "one launch per step" in bd.stacklstm_plan(hd)
+        finally:
+            hd.destroy()
+        per = runner.run(w)
+    finally:
+        os.environ.pop("STACKLSTM_STEP_KERNELS", None)
+    for k in ("y", "h_stack", "c_stack", "dx", "dW", "dbias", "dh0", "dc0"):
+        assert np.array_equal(one[k], per[k], equal_nan=False), k
+    compare(one, oracle_of(w), "fp32")
+
+
 def test_holds_only_and_all_push():
     for probs in ((0.0, 0.0, 1.0), (1.0, 0.0, 0.0)):
         w = wl.make_workload("case", T=16, B=9, I=8, H=12, dtype="fp32", seed=7, ops_kind="random_walk",
