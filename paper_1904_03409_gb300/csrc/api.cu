@@ -275,8 +275,12 @@ sl_status bwd_begin(stacklstm *s, const sl_backward_args &a)
         if ((e = cudaMemsetAsync(s->dhist_h, 0, hist_bytes, s->stream))) return cuda_fail(s, e, "clear");
         if ((e = cudaMemsetAsync(s->dhist_c, 0, hist_bytes, s->stream))) return cuda_fail(s, e, "clear");
     }
-    if ((e = sl::launch_seed_grads(s, a.d_top_h, a.dy))) return cuda_fail(s, e, "seed");
-    if (s->dt == SL_BF16 && (e = sl::bf16_backward_setup(s))) return cuda_fail(s, e, "backward setup");
+    // bf16 without per-step dy: the final tops' seeds go in with the last step's pointwise
+    // backward (the same element owners, one launch fewer)
+    const bool seed_in_pointwise = s->dt == SL_BF16 && !a.dy;
+    if (!seed_in_pointwise && (e = sl::launch_seed_grads(s, a.d_top_h, a.dy))) return cuda_fail(s, e, "seed");
+    if (s->dt == SL_BF16 && (e = sl::bf16_backward_setup(s, seed_in_pointwise ? a.d_top_h : nullptr)))
+        return cuda_fail(s, e, "backward setup");
     // push-only mode: the dx rows of steps that do not push are zero; the contraction
     // writes the others. (Zeroing them on the side stream during the step launch slowed
     // the weight gradient that follows by twice the zeroing's own time.)

@@ -281,13 +281,24 @@ __device__ __forceinline__ void pointwise8(const StepArgs &a, int tp, int b, int
     st8f(a.dhist_c + rd, acc);
 }
 
-// Pointwise backward of the last step (t = T - 1), before the reverse loop.
-__global__ void pointwise_last(StepArgs a)
+// Pointwise backward of the last step (t = T - 1), before the reverse loop. With d_top_h
+// (and no per-step dy) it first adds the loss gradient of the final top to that state's
+// gradient-history row, ftop[b] (the seeding, done by the thread that owns the elements).
+__global__ void pointwise_last(StepArgs a, const float *__restrict__ d_top_h, const int32_t *__restrict__ ftop)
 {
     const int groups = a.H / 8;
     const size_t n = (size_t)a.B * groups;
     for (size_t e = blockIdx.x * (size_t)blockDim.x + threadIdx.x; e < n; e += (size_t)gridDim.x * blockDim.x) {
         const int b = (int)(e / groups), u = (int)(e - (size_t)b * groups) * 8;
+        if (d_top_h) {
+            float *row = a.dhist_h + ((size_t)ftop[b] * a.B + b) * a.H + u;
+            float acc[8], sd[8];
+            ld8f_cg(row, acc);
+            ld8f_cg(d_top_h + (size_t)b * a.H + u, sd);
+#pragma unroll
+            for (int i = 0; i < 8; ++i) acc[i] += sd[i];
+            st8f(row, acc);
+        }
         pointwise8(a, a.T - 1, b, u);
     }
 }
@@ -833,11 +844,13 @@ cudaError_t bf16_forward_steps(stacklstm *s, const float *bias)
 }
 
 // Pointwise backward of the last step, before the reverse loop.
-cudaError_t bf16_backward_setup(stacklstm *s)
+cudaError_t bf16_backward_setup(stacklstm *s, const float *d_top_h)
 {
     StepArgs a = step_args(s, nullptr, s->w_bwd, 0, s->kcb, s->sb);
     a.gates_blk = s->fc.on && s->bc.on;  // the layout the cluster forward wrote for the cluster backward
-    pointwise_last<<<grid_for(s, (size_t)s->B * (s->H / 8)), 256, 0, s->stream>>>(a);
+    // the final top's history row of each instance (virtual, in push-only mode)
+    const int32_t *ftop = (s->push_only ? s->vy : s->top) + (size_t)s->T * s->B;
+    pointwise_last<<<grid_for(s, (size_t)s->B * (s->H / 8)), 256, 0, s->stream>>>(a, d_top_h, ftop);
     s->launches += 1;
     return cudaGetLastError();
 }

@@ -176,7 +176,9 @@ cudaError_t bf16_forward_setup_x(stacklstm *s, const __nv_bfloat16 *x);
 // the initial state into history row 0, the weight tiles packed (needs no index)
 cudaError_t bf16_forward_setup_state(stacklstm *s, const __nv_bfloat16 *h0, const float *c0, const __nv_bfloat16 *W);
 cudaError_t bf16_forward_steps(stacklstm *s, const float *bias);
-cudaError_t bf16_backward_setup(stacklstm *s);
+// the last step's pointwise backward; with d_top_h it also seeds the final tops' gradients
+// (the caller seeds them itself when the loss also has per-step terms)
+cudaError_t bf16_backward_setup(stacklstm *s, const float *d_top_h);
 cudaError_t bf16_backward_steps(stacklstm *s, float *dx, bool *dx_done);
 // Grouped calls: true when the n handles' step kernels can run as one launch (every one
 // on the one-row-tile cluster kernels of the same cluster size); that launch, on `st`.
