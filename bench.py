@@ -133,6 +133,9 @@ def phase_kernel(plan, phase, dtype):
     """(kernel name, source file, launches per pass) of the kernel that does a phase's
     work, from the plan."""
     if dtype == "fp32":
+        if "one CTA" in plan:
+            return {"forward": ("fwd_seq_f32", "fp32_path.cu", 1), "backward": ("bwd_seq_f32", "fp32_path.cu", 1),
+                    "dx": ("dx_f32", "fp32_path.cu", 1), "dw": ("dw_f32", "fp32_path.cu", 1)}[phase]
         return {"forward": ("fwd_step_f32", "fp32_path.cu", "T"),
                 "backward": ("bwd_pointwise_f32+bwd_contract_f32", "fp32_path.cu", "2T"),
                 "dx": ("dx_f32", "fp32_path.cu", 1), "dw": ("dw_f32", "fp32_path.cu", 1)}[phase]
