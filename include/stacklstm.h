@@ -51,8 +51,12 @@
  *   STACKLSTM_BWD_CLUSTER=0        no thread-block-cluster backward for one row tile
  *   STACKLSTM_BWD_SPLIT=k          the persistent backward with its 4H contraction split
  *                                  over k CTAs per 64-unit column tile (k = 4)
+ *   STACKLSTM_SPLIT_CLUSTER=0      the parts of a split contraction trade their partial
+ *                                  sums through an L2 scratch, not as a thread-block
+ *                                  cluster in shared memory
  *   STACKLSTM_DX_SPARE=0 | k       dx in its own launch (0), or by at most k extra CTAs of
- *                                  the persistent backward launch
+ *                                  the persistent backward launch (whole clusters of it,
+ *                                  when that launch is a cluster launch)
  *   STACKLSTM_CUDA_CORE=0 | 1      small batches (B <= 32, H <= 256): never (0), or
  *                                  whenever the shape allows (1), the CUDA-core cluster
  *                                  kernels instead of the tensor-core ones

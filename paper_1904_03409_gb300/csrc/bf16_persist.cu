@@ -54,12 +54,14 @@ struct WsArgs {
     float *dx;               // [T B][I]
     const int32_t *dx_xidx;  // push-only mode: real step of each virtual row's step (-1: none), else null
     const uint8_t *wdx;      // W_x packed as [nxt][KC][256 rows][64], 128-byte swizzled rows
+    int cl;                  // 1, or KS: the KS parts of a column tile form a thread-block
+                             // cluster and trade their partial sums in shared memory
 };
 
 // Dynamic shared memory: [weight tile (w_res)][S stages: G A chunks, then G weight
-// chunks unless resident][forward: gate staging tile][barriers], based at the first
-// 1024-byte boundary.
-constexpr uint32_t kBarBytes = (2 * kMaxStages + 6) * 8 + 16;
+// chunks unless resident][forward: gate staging tile][split contraction in a cluster:
+// partial-sum exchange tile][barriers], based at the first 1024-byte boundary.
+constexpr uint32_t kBarBytes = (2 * kMaxStages + 7) * 8 + 16;
 
 // forward: what one tile writes to the history apart from the h operand of the next step,
 // staged for the tensor stores that write it out: the activated gates (4 gates x 128 rows
@@ -71,6 +73,10 @@ __host__ __device__ constexpr uint32_t ws_stg_bytes(bool fwd, int U)
 {
     return fwd ? 128u * U * (8 + 2 + 4) : U == 32 ? 128u * 32 * 4 : 0u;
 }
+
+// split contraction in a cluster: what the other parts send one CTA, fp32 laid out
+// [sending part][4-unit group of the U / KS units the CTA finishes][128 rows][4 units]
+__host__ __device__ constexpr uint32_t ws_xch_bytes(int U) { return 128u * U * 4; }
 
 __host__ __device__ constexpr uint32_t ws_stage_bytes(int G, int NB, int w_res)
 {
@@ -85,13 +91,16 @@ __host__ __device__ constexpr uint32_t ws_smem_bytes(int S, int G, int NB, int K
 struct WCtl {
     uint32_t w0, ring0, stage;  // resident weight tile, stage 0, bytes per stage
     uint32_t stg;               // forward: gate staging tile
+    uint32_t xch;               // split contraction in a cluster: the partial sums received
     uint64_t *full, *empty, *tfull, *tempty, *wbar, *done;
+    uint64_t *rbar;  // one phase per tile: every thread of the other parts stored its partials
     uint32_t *tmem_slot;
     int *n_issued, *n_consumed;  // groups armed by the producer / consumed by the MMA warp
     volatile int *abort;
 };
 
-__device__ __forceinline__ WCtl wcarve(uint8_t *raw, int S, int G, int NB, int KC, int w_res, uint32_t stg)
+__device__ __forceinline__ WCtl wcarve(uint8_t *raw, int S, int G, int NB, int KC, int w_res, uint32_t stg,
+                                       uint32_t xch)
 {
     const uint32_t off = smem_u32(raw);
     uint8_t *base = raw + ((1024u - (off & 1023u)) & 1023u);
@@ -101,14 +110,16 @@ __device__ __forceinline__ WCtl wcarve(uint8_t *raw, int S, int G, int NB, int K
     c.w0 = smem_u32(base);
     c.ring0 = c.w0 + wbytes;
     c.stg = c.ring0 + S * c.stage;
-    uint64_t *bars = (uint64_t *)(base + wbytes + (size_t)S * c.stage + stg);
+    c.xch = c.stg + stg;
+    uint64_t *bars = (uint64_t *)(base + wbytes + (size_t)S * c.stage + stg + xch);
     c.full = bars;
     c.empty = bars + kMaxStages;
     c.tfull = bars + 2 * kMaxStages;
     c.tempty = c.tfull + 2;
     c.wbar = c.tempty + 2;
     c.done = c.wbar + 1;
-    c.tmem_slot = (uint32_t *)(c.done + 1);
+    c.rbar = c.done + 1;
+    c.tmem_slot = (uint32_t *)(c.rbar + 1);
     c.n_issued = (int *)(c.tmem_slot + 1);
     c.n_consumed = c.n_issued + 1;
     c.abort = (volatile int *)(c.n_consumed + 1);
@@ -303,9 +314,11 @@ struct EpiCtx {
 // units. Without a split contraction (KS = 1) the thread finishes units
 // ct * U + part * UE .. + UE straight from its accumulator lane. With KS > 1 (backward
 // only) the KS CTAs of a column tile each hold a partial dh_read over a quarter (half ...)
-// of the 4H contraction: every CTA writes its whole partial row to an L2 scratch, counts
-// it, waits for the other parts, then sums the parts in part order (deterministic) for the
-// U / KS units it finishes: ct * U + kp * U / KS .. + U / KS.
+// of the 4H contraction and finish U / KS units, ct * U + kp * U / KS .. + U / KS, summing
+// the parts in part order (deterministic). The parts trade their partials as one
+// thread-block cluster, each storing the other parts' units of its row into their shared
+// memory (p.cl = KS), or through an L2 scratch: every CTA writes its whole partial row,
+// counts it, waits for the other parts and reads back its units of each.
 template <int U, int EP, int NG, bool kFwd, int KS>
 __device__ __forceinline__ void epilogue_loop(const StepArgs &a, const WsArgs &p, const EpiCtx &e,
                                               const float *s_bias, const CUtensorMap *tm_gates,
@@ -634,35 +647,76 @@ __device__ __forceinline__ void epilogue_loop(const StepArgs &a, const WsArgs &p
             tc::tc_fence_after();
             float dsum[KS > 1 ? UE : 1];
             if constexpr (KS > 1) {
-                // the whole partial row of this lane to the scratch, then the sum of the parts
+                // this lane's whole partial row, then the sum of the parts for its units
                 uint32_t pr[U];
                 tmem_cols<U>(taddr, pr);
                 tc::tmem_wait_ld();
                 tc::tc_fence_before();
                 __syncwarp();
                 if (e.lane == 0) tc::mbar_arrive(&e.c.tempty[acc]);
-                const size_t grp = (size_t)rt * p.n_ct + e.ct;
-                float *prow = p.part + ((grp * KS + e.kp) * kRows + e.q * 32 + e.lane) * U;
-#pragma unroll
-                for (int i = 0; i < U / 8; ++i) st_v8(prow + 8 * i, pr + 8 * i);
-                __syncwarp();
-                tc::bar_sync(2, E * 32);
-                bool ok2 = true;
-                if (e.tid == 0) {
-                    tc::red_release_gpu_add(p.pcnt + grp, 1);
-                    ok2 = spin_until(p.pcnt + grp, KS * (ks + 1), e.limit, e.c.abort, a.err);
-                    if (!ok2) ws_abort(e.c, a.err);
-                }
-                __syncwarp();
-                if (tc::bar_any(1, E * 32, !ok2 || *e.c.abort)) break;
 #pragma unroll
                 for (int i = 0; i < UE; ++i) dsum[i] = 0.0f;
+                if (p.cl > 1) {
+                    // the parts form a cluster: this row's units of part j go straight into
+                    // CTA j's exchange tile, each thread releasing its stores with its
+                    // arrival; the tile's phase completes once every thread of the other
+                    // parts arrived (one row tile per CTA: a part stores a tile's partials
+                    // only after every CTA of the row tile released the step before, so
+                    // after this CTA read the previous ones)
+                    constexpr int G4 = UE / 4;
+                    const uint32_t r16 = (uint32_t)(e.q * 32 + e.lane) * 16u;
 #pragma unroll
-                for (int j = 0; j < KS; ++j) {
-                    float v[UE];
-                    ld_f<UE>(p.part + ((grp * KS + j) * kRows + e.q * 32 + e.lane) * U + e.kp * (U / KS), v);
+                    for (int j = 0; j < KS; ++j) {
+                        if (j == e.kp) continue;
+                        const uint32_t dst = tc::mapa(e.c.xch, (uint32_t)j) + (uint32_t)(e.kp * G4) * (kRows * 16u) + r16;
 #pragma unroll
-                    for (int i = 0; i < UE; ++i) dsum[i] += v[i];
+                        for (int g = 0; g < G4; ++g) tc::st_cluster_v4(dst + (uint32_t)g * (kRows * 16u), pr + j * UE + 4 * g);
+                        tc::mbar_arrive_remote(tc::mapa(tc::smem_u32(e.c.rbar), (uint32_t)j));
+                    }
+                    const bool ok2 = tc::mbar_wait_cluster(e.c.rbar, (uint32_t)(k & 1), e.limit, e.c.abort);
+                    if (!ok2) ws_abort(e.c, a.err);
+                    __syncwarp();
+                    if (tc::bar_any(1, E * 32, !ok2 || *e.c.abort)) break;
+                    // the sum in part order, as below
+#pragma unroll
+                    for (int j = 0; j < KS; ++j) {
+#pragma unroll
+                        for (int g = 0; g < G4; ++g) {
+                            uint32_t w[4];
+                            if (j == e.kp) {
+#pragma unroll
+                                for (int i = 0; i < 4; ++i) w[i] = pr[j * UE + 4 * g + i];
+                            } else {
+                                ld_shared_v4(e.c.xch + (uint32_t)(j * G4 + g) * (kRows * 16u) + r16, w);
+                            }
+#pragma unroll
+                            for (int i = 0; i < 4; ++i) dsum[4 * g + i] += __uint_as_float(w[i]);
+                        }
+                    }
+                } else {
+                    // the whole partial row of this lane to the L2 scratch, counted, then the
+                    // parts of this CTA's units read back once every part counted
+                    const size_t grp = (size_t)rt * p.n_ct + e.ct;
+                    float *prow = p.part + ((grp * KS + e.kp) * kRows + e.q * 32 + e.lane) * U;
+#pragma unroll
+                    for (int i = 0; i < U / 8; ++i) st_v8(prow + 8 * i, pr + 8 * i);
+                    __syncwarp();
+                    tc::bar_sync(2, E * 32);
+                    bool ok2 = true;
+                    if (e.tid == 0) {
+                        tc::red_release_gpu_add(p.pcnt + grp, 1);
+                        ok2 = spin_until(p.pcnt + grp, KS * (ks + 1), e.limit, e.c.abort, a.err);
+                        if (!ok2) ws_abort(e.c, a.err);
+                    }
+                    __syncwarp();
+                    if (tc::bar_any(1, E * 32, !ok2 || *e.c.abort)) break;
+#pragma unroll
+                    for (int j = 0; j < KS; ++j) {
+                        float v[UE];
+                        ld_f<UE>(p.part + ((grp * KS + j) * kRows + e.q * 32 + e.lane) * U + e.kp * (U / KS), v);
+#pragma unroll
+                        for (int i = 0; i < UE; ++i) dsum[i] += v[i];
+                    }
                 }
             }
 #pragma unroll
@@ -817,7 +871,7 @@ __device__ __forceinline__ void dx_role(const CUtensorMap *tm_g, const WsArgs &p
     const int did = (int)blockIdx.x - p.n_chain;
     const int n_mine = did < n_items ? (n_items - did + p.n_dx - 1) / p.n_dx : 0;
     const long long limit = a.limit;
-    const WCtl c = wcarve(smem_raw, S, 1, kDxN, KC, 0, 0u);
+    const WCtl c = wcarve(smem_raw, S, 1, kDxN, KC, 0, 0u, 0u);
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     if (tid == 0) {
         for (int s = 0; s < S; ++s) {
@@ -1009,7 +1063,9 @@ step_ws(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtens
     const int kp = (int)(blockIdx.x % KS), cidx = (int)(blockIdx.x / KS);
     const int k0 = KC * kp / KS, k1 = KC * (kp + 1) / KS;  // this CTA's contraction chunks
     const int dep_c = split > k0 ? split : k0;            // first chunk that needs step t - 1
-    const WCtl c = wcarve(smem_raw, S, G, NB, (KC + KS - 1) / KS, p.w_res, ws_stg_bytes(kFwd, U));
+    const bool xcl = KS > 1 && p.cl > 1;  // the parts trade partials in the cluster's shared memory
+    const WCtl c = wcarve(smem_raw, S, G, NB, (KC + KS - 1) / KS, p.w_res, ws_stg_bytes(kFwd, U),
+                          xcl ? ws_xch_bytes(U) : 0u);
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int ct = cidx % p.n_ct, slot = cidx / p.n_ct;
     const int n_mine = slot < p.n_rt ? (p.n_rt - slot + p.n_slot - 1) / p.n_slot : 0;
@@ -1031,6 +1087,8 @@ step_ws(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtens
         }
         tc::mbar_init(c.wbar, 1);
         tc::mbar_init(c.done, 1);
+        // every epilogue thread of each other part arrives once a tile
+        tc::mbar_init(c.rbar, KS > 1 ? (KS - 1) * E * 32 : 1);
         *c.n_issued = 0;
         *c.n_consumed = 0;
         *c.abort = 0;
@@ -1040,6 +1098,7 @@ step_ws(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtens
     tc::tc_fence_before();
     __syncthreads();
     tc::tc_fence_after();
+    if (xcl) tc::cluster_sync();  // the other parts' barriers are initialised before any arrival
     const uint32_t tmem = *c.tmem_slot;
     const uint8_t *wtile = a.wpack + (size_t)ct * KC * bchunk;
 
@@ -1155,6 +1214,8 @@ step_ws(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtens
     tc::tc_fence_before();
     __syncthreads();
     if (warp == E) tc::tmem_dealloc(tmem, 2 * kCols);
+    // no part leaves while another may still store into its shared memory
+    if (xcl) tc::cluster_sync();
 }
 
 // ------------------------------------------------------------------ planning
@@ -1206,6 +1267,28 @@ uint32_t pad_for_tmem(const void *fn, int threads, uint32_t smem, uint32_t kcols
     return kSmemCap;
 }
 
+// Co-resident thread-block clusters of cl CTAs at this footprint (0 on any error).
+int max_clusters(const void *fn, int threads, uint32_t smem, int cl)
+{
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(cl);
+    cfg.blockDim = dim3(threads);
+    cfg.dynamicSmemBytes = smem;
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeClusterDimension;
+    at[0].val.clusterDim.x = cl;
+    at[0].val.clusterDim.y = 1;
+    at[0].val.clusterDim.z = 1;
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, fn, &cfg) != cudaSuccess) {
+        cudaGetLastError();
+        return 0;
+    }
+    return n;
+}
+
 // Plans one variant: the weight tile resident or streamed, a two-stage ring. The grid is
 // sized from the number of co-resident CTAs of that footprint. Cost = row-tile rounds per
 // step x per-tile time (constants fitted to GB300 measurements); ties go to plans within
@@ -1249,6 +1332,21 @@ bool plan_variant(const Variant &v, bool fwd, int KC, int split, int n_rt, int H
         // slot then has (about) the same work, and the SMs left over take other work
         const int rounds = (n_rt + std::min(n_rt, resident / pad) - 1) / std::min(n_rt, resident / pad);
         const int sl = (n_rt + rounds - 1) / rounds;
+        // a split contraction whose CTAs each keep one row tile: its parts as one
+        // thread-block cluster, trading partial sums in shared memory, when the larger
+        // footprint and every cluster still fit. Test hook (include/stacklstm.h):
+        // STACKLSTM_SPLIT_CLUSTER = 0 keeps the L2 exchange
+        int cl = 1;
+        if (!fwd && v.KS > 1 && rounds == 1) {
+            const char *fc = getenv("STACKLSTM_SPLIT_CLUSTER");
+            const uint32_t sx = pad_for_tmem(v.fn, threads, ws_smem_bytes(S, v.G, NB, KCl, wr, stg + ws_xch_bytes(v.U)),
+                                             kcols2);
+            if ((!fc || atoi(fc) != 0) && sx && sx <= cap &&
+                max_clusters(v.fn, threads, sx, v.KS) * v.KS >= pad * sl) {
+                cl = v.KS;
+                smem = sx;
+            }
+        }
         // forward, per CTA and step: MMA issue plus the epilogue's ~16 B of stores per
         // (instance, unit) at about 30 B/cycle
         double c = rounds * (KC * 4 * mma_cycles(NB) + groups * kWaitCycles + 128.0 * v.U * 16 / 30);
@@ -1260,8 +1358,8 @@ bool plan_variant(const Variant &v, bool fwd, int KC, int split, int n_rt, int H
             // exchange of a split contraction
             const double ingest = (128.0 * KCl * 128 + (wr ? 0.0 : (double)NB * KCl * 128)) / 70;
             const double mma = KCl * 4 * mma_cycles(NB) + groups * 400.0;
-            const double epi = 128.0 * (v.U / v.KS) * 48 / 30 +
-                               (v.KS > 1 ? 2.0 * 128 * v.U * 4 / 30 + 3000 : 0.0);
+            const double xch = v.KS == 1 ? 0.0 : cl > 1 ? 1500.0 : 2.0 * 128 * v.U * 4 / 30 + 3000;
+            const double epi = 128.0 * (v.U / v.KS) * 48 / 30 + xch;
             // with two or more row tiles a CTA multiplies one while the epilogue
             // finishes the other (their chains are independent)
             const double mm = std::max(ingest, mma);
@@ -1281,7 +1379,7 @@ bool plan_variant(const Variant &v, bool fwd, int KC, int split, int n_rt, int H
             pl->S = S;
             pl->slot = sl;
             pl->w_res = wr;
-            pl->cl = 1;
+            pl->cl = cl;
             pl->KS = v.KS;
             pl->n_ct = n_ct;
             pl->smem = smem;
@@ -1345,14 +1443,17 @@ bool plan(stacklstm *s, bool fwd, PersistPlan *pl)
         const char *fx = getenv("STACKLSTM_DX_SPARE");
         int r = 0;
         const int n_chain = pl->n_ct * pl->KS * pl->slot;
-        const int spare = s->num_sms - n_chain;
+        // in a cluster launch the extra CTAs come in whole (co-resident) clusters too
+        const int spare = pl->cl > 1 ? (max_clusters(find_fn(false, *pl), pl->threads, pl->smem, pl->cl) * pl->cl - n_chain)
+                                     : s->num_sms - n_chain;
         const int S = (int)std::min<uint32_t>(kMaxStages, (pl->smem - 1024 - kBarBytes) / (kAStage + 256u * 128));
         if ((!fx || atoi(fx) != 0) && s->nx == 256 && s->B >= kRows && spare >= 4 && S >= 2 &&
             cudaOccupancyMaxActiveBlocksPerMultiprocessor(&r, find_fn(false, *pl), pl->threads, pl->smem) ==
                 cudaSuccess &&
             r == 1) {
             pl->n_dx = fx && atoi(fx) > 0 ? std::min(spare, atoi(fx)) : spare;
-            pl->dx_S = S;
+            pl->n_dx -= pl->n_dx % pl->cl;
+            pl->dx_S = pl->n_dx > 0 ? S : 0;
         }
         cudaGetLastError();
     }
@@ -1403,6 +1504,7 @@ cudaError_t bf16_launch_fwd_persist(stacklstm *s, const StepArgs &a, const CUten
     p.part = nullptr;
     p.pcnt = nullptr;
     p.a_rows = s->B <= 64 ? 64 : kRows;
+    p.cl = 1;
     cudaError_t e = cudaMemsetAsync(p.cnt, 0, sizeof(int32_t) * p.n_rt * p.cs, s->stream);
     if (e) return e;
     const void *fn = find_fn(true, pl);
@@ -1439,6 +1541,7 @@ cudaError_t bf16_launch_bwd_persist(stacklstm *s, const StepArgs &a, const CUten
     p.dx = dx;
     p.dx_xidx = s->push_only ? s->xidx : nullptr;
     p.wdx = (const uint8_t *)s->w_dx;
+    p.cl = pl.cl;
     cudaError_t e = cudaMemsetAsync(p.cnt, 0, sizeof(int32_t) * p.n_rt * p.cs, s->stream);
     if (e) return e;
     if (pl.KS > 1 && (e = cudaMemsetAsync(p.pcnt, 0, sizeof(int32_t) * p.n_rt * p.n_ct, s->stream))) return e;

@@ -23,7 +23,8 @@ struct PersistPlan {
     int S = 0;          // ring stages
     int slot = 0;       // CTAs per column tile (each takes every slot-th row tile)
     int w_res = 0;      // weight tile resident in shared memory
-    int cl = 1;         // thread-block cluster size (the one-row-tile cluster kernels; 1 otherwise)
+    int cl = 1;         // thread-block cluster size (the one-row-tile cluster kernels; the KS parts
+                        // of a split contraction; 1 otherwise)
     int KS = 1;         // contraction parts per column tile (backward split contraction)
     int n_ct = 0;       // column tiles, padded to a multiple of cl
     unsigned smem = 0;  // dynamic shared memory per CTA

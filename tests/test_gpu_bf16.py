@@ -179,27 +179,26 @@ def test_per_step_kernels_match_oracle(T, B, I, H, seed):
     compare(got, oracle_all(w), "bf16")
 
 
-@pytest.mark.parametrize("T,B,I,H,seed", [(12, 200, 64, 256, 14), (10, 130, 40, 200, 15)])
-def test_split_contraction_backward_matches_oracle(T, B, I, H, seed):
-    """The backward with its 4H contraction split over four CTAs per column tile (partial
-    sums exchanged through L2, summed in part order) stays parity-green, including parts
-    of unequal length (H = 200: 13 chunks over 4 parts)."""
+@pytest.mark.parametrize("T,B,I,H,seed,cl", [(12, 200, 64, 256, 14, 4), (10, 130, 40, 200, 15, 4),
+                                            (6, 1300, 16, 256, 26, 1)])
+def test_split_contraction_backward_matches_oracle(T, B, I, H, seed, cl):
+    """The backward with its 4H contraction split over four CTAs per column tile stays
+    parity-green, including parts of unequal length (H = 200: 13 chunks over 4 parts), into
+    NaN-filled outputs. Where each CTA keeps one row tile the four parts run as one
+    thread-block cluster and trade their partial sums in shared memory; with several row
+    tiles a CTA (B = 1300: 11 row tiles) they go through an L2 scratch. Both sum the parts in
+    part order, so the two exchanges agree bit for bit, and a rerun repeats them."""
     w = case(T, B, I, H, seed, bias_scale=0.3, h0_scale=0.5, c0_scale=0.5, dy_scale=0.5)
-    os.environ["STACKLSTM_BWD_SPLIT"] = "4"
-    os.environ.update(PERSISTENT)
-    try:
-        hd = bd.stacklstm_create(w.T, w.B, w.I, w.H, bd.SL_BF16, 0)
-        plan = bd.stacklstm_plan(hd)
-        hd.destroy()
-        got = runner.run(w)
-        again = runner.run(w)
-    finally:
-        del os.environ["STACKLSTM_BWD_SPLIT"]
-        for k in PERSISTENT:
-            del os.environ[k]
-    assert "backward persistent U=64" in plan and "contraction parts 4" in plan, plan
+    env = dict(PERSISTENT, STACKLSTM_BWD_SPLIT="4")
+    plan, got = run_nan_filled(w, env)
+    plan0, l2 = run_nan_filled(w, dict(env, STACKLSTM_SPLIT_CLUSTER="0"))
+    _, again = run_nan_filled(w, env)
+    bwd, bwd0 = plan.split("; backward ")[1], plan0.split("; backward ")[1]
+    assert "persistent U=64" in bwd and "contraction parts 4" in bwd and "cluster %d " % cl in bwd, plan
+    assert "contraction parts 4" in bwd0 and "cluster 1 " in bwd0, plan0
     compare(got, oracle_all(w), "bf16")
     for k in ("dx", "dW", "dbias", "dh0", "dc0"):
+        assert np.array_equal(got[k], l2[k]), k
         assert np.array_equal(got[k], again[k]), k
 
 
@@ -246,9 +245,13 @@ def test_input_gradient_on_spare_sms_matches_oracle(T, B, I, H, seed):
     plan0, sep = run_nan_filled(w, dict(PERSISTENT, STACKLSTM_DX_SPARE="0"))
     assert "dx CTAs 0" in plan0, plan0
     assert np.array_equal(got["dx"], sep["dx"])
-    plan1, one = run_nan_filled(w, dict(PERSISTENT, STACKLSTM_DX_SPARE="1"))
+    # one extra CTA is no whole cluster: a split contraction's parts then trade through L2
+    # (which may change the plan, so its own separate-launch dx is the reference)
+    l2 = dict(PERSISTENT, STACKLSTM_SPLIT_CLUSTER="0")
+    _, sep1 = run_nan_filled(w, dict(l2, STACKLSTM_DX_SPARE="0"))
+    plan1, one = run_nan_filled(w, dict(l2, STACKLSTM_DX_SPARE="1"))
     assert "dx CTAs 1" in plan1, plan1
-    assert np.array_equal(one["dx"], sep["dx"])
+    assert np.array_equal(one["dx"], sep1["dx"])
 
 
 @pytest.mark.parametrize("T,B,I,H,seed", [(17, 40, 8, 16, 19), (24, 64, 200, 200, 20), (9, 8, 64, 136, 21),
