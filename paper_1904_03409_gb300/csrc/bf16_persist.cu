@@ -93,7 +93,7 @@ struct WCtl {
     uint32_t stg;               // forward: gate staging tile
     uint32_t xch;               // split contraction in a cluster: the partial sums received
     uint64_t *full, *empty, *tfull, *tempty, *wbar, *done;
-    uint64_t *rbar;  // one phase per tile: every thread of the other parts stored its partials
+    uint64_t *rbar;  // one phase per tile: the other parts' partials have landed
     uint32_t *tmem_slot;
     int *n_issued, *n_consumed;  // groups armed by the producer / consumed by the MMA warp
     volatile int *abort;
@@ -658,20 +658,21 @@ __device__ __forceinline__ void epilogue_loop(const StepArgs &a, const WsArgs &p
                 for (int i = 0; i < UE; ++i) dsum[i] = 0.0f;
                 if (p.cl > 1) {
                     // the parts form a cluster: this row's units of part j go straight into
-                    // CTA j's exchange tile, each thread releasing its stores with its
-                    // arrival; the tile's phase completes once every thread of the other
-                    // parts arrived (one row tile per CTA: a part stores a tile's partials
-                    // only after every CTA of the row tile released the step before, so
-                    // after this CTA read the previous ones)
+                    // CTA j's exchange tile by asynchronous stores that count their bytes on
+                    // its barrier; this tile's phase completes once the other parts' bytes
+                    // landed and thread 0 arrived with their count (one row tile per CTA: a
+                    // part stores a tile's partials only after every CTA of the row tile
+                    // released the step before, so after this CTA read the previous ones)
                     constexpr int G4 = UE / 4;
                     const uint32_t r16 = (uint32_t)(e.q * 32 + e.lane) * 16u;
+                    if (e.tid == 0) tc::mbar_arrive_expect_tx(e.c.rbar, (uint32_t)(KS - 1) * kRows * UE * 4);
 #pragma unroll
                     for (int j = 0; j < KS; ++j) {
                         if (j == e.kp) continue;
                         const uint32_t dst = tc::mapa(e.c.xch, (uint32_t)j) + (uint32_t)(e.kp * G4) * (kRows * 16u) + r16;
+                        const uint32_t bar = tc::mapa(tc::smem_u32(e.c.rbar), (uint32_t)j);
 #pragma unroll
-                        for (int g = 0; g < G4; ++g) tc::st_cluster_v4(dst + (uint32_t)g * (kRows * 16u), pr + j * UE + 4 * g);
-                        tc::mbar_arrive_remote(tc::mapa(tc::smem_u32(e.c.rbar), (uint32_t)j));
+                        for (int g = 0; g < G4; ++g) tc::st_async_v4(dst + (uint32_t)g * (kRows * 16u), pr + j * UE + 4 * g, bar);
                     }
                     const bool ok2 = tc::mbar_wait_cluster(e.c.rbar, (uint32_t)(k & 1), e.limit, e.c.abort);
                     if (!ok2) ws_abort(e.c, a.err);
@@ -1087,8 +1088,8 @@ step_ws(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtens
         }
         tc::mbar_init(c.wbar, 1);
         tc::mbar_init(c.done, 1);
-        // every epilogue thread of each other part arrives once a tile
-        tc::mbar_init(c.rbar, KS > 1 ? (KS - 1) * E * 32 : 1);
+        // one arrival a tile (with the bytes the other parts store asynchronously)
+        tc::mbar_init(c.rbar, 1);
         *c.n_issued = 0;
         *c.n_consumed = 0;
         *c.abort = 0;

@@ -188,21 +188,18 @@ __device__ __forceinline__ uint32_t mapa(uint32_t addr, uint32_t rank)
     asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
     return r;
 }
-// 16-byte store to another CTA's shared memory (an address from mapa).
-__device__ __forceinline__ void st_cluster_v4(uint32_t addr, const uint32_t *w)
+// 16-byte asynchronous store to another CTA's shared memory (an address from mapa) whose
+// completion counts 16 bytes on that CTA's mbarrier `bar` (a cluster address too), with
+// release semantics at cluster scope: no fence and no arrival of the storing thread.
+__device__ __forceinline__ void st_async_v4(uint32_t addr, const uint32_t *w, uint32_t bar)
 {
-    asm volatile("st.shared::cluster.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(w[0]), "r"(w[1]), "r"(w[2]),
-                 "r"(w[3])
+    asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.v4.b32 [%0], {%1, %2, %3, %4}, [%5];" ::"r"(
+                     addr),
+                 "r"(w[0]), "r"(w[1]), "r"(w[2]), "r"(w[3]), "r"(bar)
                  : "memory");
 }
-// Arrival (count one) on an mbarrier of another CTA of the cluster, releasing this thread's
-// earlier writes at cluster scope.
-__device__ __forceinline__ void mbar_arrive_remote(uint32_t cluster_addr)
-{
-    asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
-}
-// mbar_wait with acquire semantics at cluster scope: what the arriving threads of other
-// CTAs wrote before their release arrivals is visible after it returns true.
+// mbar_wait with acquire semantics at cluster scope: what other CTAs of the cluster stored
+// with release (or release-completed asynchronous stores) is visible after it returns true.
 __device__ __forceinline__ bool mbar_wait_cluster(uint64_t *bar, uint32_t parity, long long limit,
                                                   volatile int *abort)
 {
