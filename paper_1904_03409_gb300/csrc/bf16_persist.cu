@@ -23,8 +23,9 @@
 // of the row tile wrote at the step before (forward: hr[t]; backward: dG_t). Each row tile
 // has a counter of completed steps, raised with release semantics after the epilogue's
 // stores and polled with acquire semantics (a bounded spin) by the producer before it
-// loads the dependent chunks. All CTAs are co-resident (cooperative launch), so the spins
-// end; every wait is bounded and a timeout aborts the whole grid through the error word.
+// loads the dependent chunks. All CTAs are co-resident (a cooperative launch, or a cluster
+// launch whose clusters the planner checked fit at once), so the spins end; every wait is
+// bounded and a timeout aborts the whole grid through the error word.
 #include <stdio.h>
 
 #include <algorithm>
@@ -1064,7 +1065,10 @@ step_ws(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtens
     const int kp = (int)(blockIdx.x % KS), cidx = (int)(blockIdx.x / KS);
     const int k0 = KC * kp / KS, k1 = KC * (kp + 1) / KS;  // this CTA's contraction chunks
     const int dep_c = split > k0 ? split : k0;            // first chunk that needs step t - 1
-    const bool xcl = KS > 1 && p.cl > 1;  // the parts trade partials in the cluster's shared memory
+    // the parts trade partials in the cluster's shared memory; a launch whose clusters are not
+    // the KS parts of a column tile (blockIdx.x % KS is the rank only then) takes the L2
+    // exchange instead, so no CTA ever addresses a peer that is not there
+    const bool xcl = KS > 1 && p.cl > 1 && tc::cluster_size() == (uint32_t)KS;
     const WCtl c = wcarve(smem_raw, S, G, NB, (KC + KS - 1) / KS, p.w_res, ws_stg_bytes(kFwd, U),
                           xcl ? ws_xch_bytes(U) : 0u);
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -1461,6 +1465,9 @@ bool plan(stacklstm *s, bool fwd, PersistPlan *pl)
     return true;
 }
 
+// A cooperative launch (every CTA co-resident, or the launch fails); a plan with clusters
+// launches with its cluster shape alone, the planner having checked that all of the grid's
+// clusters fit at once (cudaOccupancyMaxActiveClusters). Every spin is bounded either way.
 template <typename... Args>
 cudaError_t launch_coop(const void *fn, const PersistPlan &pl, int grid, cudaStream_t st, Args... args)
 {
@@ -1469,15 +1476,18 @@ cudaError_t launch_coop(const void *fn, const PersistPlan &pl, int grid, cudaStr
     cfg.blockDim = dim3(pl.threads);
     cfg.dynamicSmemBytes = pl.smem;
     cfg.stream = st;
-    cudaLaunchAttribute at[2];
-    at[0].id = cudaLaunchAttributeCooperative;
-    at[0].val.cooperative = 1;
-    at[1].id = cudaLaunchAttributeClusterDimension;
-    at[1].val.clusterDim.x = pl.cl;
-    at[1].val.clusterDim.y = 1;
-    at[1].val.clusterDim.z = 1;
+    cudaLaunchAttribute at[1];
+    if (pl.cl > 1) {
+        at[0].id = cudaLaunchAttributeClusterDimension;
+        at[0].val.clusterDim.x = pl.cl;
+        at[0].val.clusterDim.y = 1;
+        at[0].val.clusterDim.z = 1;
+    } else {
+        at[0].id = cudaLaunchAttributeCooperative;
+        at[0].val.cooperative = 1;
+    }
     cfg.attrs = at;
-    cfg.numAttrs = 2;
+    cfg.numAttrs = 1;
     void *argv[] = {(void *)&args...};
     return cudaLaunchKernelExC(&cfg, fn, argv);
 }

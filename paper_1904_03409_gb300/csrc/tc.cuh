@@ -176,6 +176,13 @@ __device__ __forceinline__ uint32_t cluster_rank()
     asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
     return r;
 }
+// CTAs in this CTA's cluster (1 when the launch has no cluster shape).
+__device__ __forceinline__ uint32_t cluster_size()
+{
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_nctarank;" : "=r"(r));
+    return r;
+}
 // Every thread of every CTA of the cluster arrives, then waits for all of them.
 __device__ __forceinline__ void cluster_sync()
 {
