@@ -57,6 +57,8 @@
  *   STACKLSTM_DX_SPARE=0 | k       dx in its own launch (0), or by at most k extra CTAs of
  *                                  the persistent backward launch (whole clusters of it,
  *                                  when that launch is a cluster launch)
+ *   STACKLSTM_DW_M=128 | 256       the weight gradient's tile: 128 or 256 rows of W (x 256
+ *                                  gate columns) per CTA
  *   STACKLSTM_CUDA_CORE=0 | 1      small batches (B <= 32, H <= 256): never (0), or
  *                                  whenever the shape allows (1), the CUDA-core cluster
  *                                  kernels instead of the tensor-core ones

@@ -6,11 +6,12 @@
 // caller's x, [T*B][I]), hr rows (the h operand of each step, [(T+1)*B][H]) and dG rows
 // ([T*B][4H]), 64 r-rows per contraction chunk. The M index is padded so that no 64-wide
 // block straddles x and h: blocks 0 .. kbx-1 are x columns, kbx .. kbx+kbh-1 are h
-// columns, anything after is a constant zero block. A CTA owns 128 m (two blocks) x NT
-// gate columns (NT = 512: two 256-column accumulators, all of tensor memory) over a range
-// of chunks. Warps: 0-3 epilogue, 4 TMA producer, 5 MMA issue. The epilogue warps of the
-// first m tile also sum the dG chunks they find in shared memory column by column: the
-// bias gradient, without an all-ones operand row.
+// columns, anything after is a constant zero block. A CTA owns MT m (MT / 64 blocks) x 256
+// gate columns over a range of chunks: MT = 128, one 256-column accumulator (two CTAs an
+// SM), or MT = 256, two accumulators over one shared dG operand (all of tensor memory, one
+// CTA an SM, a third fewer operand bytes per MMA). Warps: 0-3 epilogue, 4 TMA producer, 5
+// MMA issue. The epilogue warps of the first m tile also sum the dG chunks they find in
+// shared memory column by column: the bias gradient, without an all-ones operand row.
 #include <stdlib.h>
 
 #include <algorithm>
@@ -24,6 +25,7 @@ using tc::smem_u32;
 using tc::sw128;
 
 constexpr int kDwThreads = 192;
+constexpr int kDwN = 256;            // gate columns per tile
 constexpr uint32_t kBlk = 64 * 128;  // one MN-major block: 64 r-rows of 64 bf16 (128 bytes)
 
 struct DwWsArgs {
@@ -36,12 +38,12 @@ struct DwWsArgs {
     int32_t *err;
 };
 
-__host__ __device__ constexpr uint32_t dw_stage_bytes(int NT) { return 2 * kBlk + (uint32_t)NT * 128; }
+__host__ __device__ constexpr uint32_t dw_stage_bytes(int MT) { return (uint32_t)(MT / 64) * kBlk + kDwN * 128u; }
 constexpr uint32_t kDwBarBytes = (2 * kMaxStages + 1) * 8 + 16;
 constexpr uint32_t kDwBiasBytes = 128 * 8 * 4;
-__host__ __device__ constexpr uint32_t dw_smem_bytes(int S, int NT)
+__host__ __device__ constexpr uint32_t dw_smem_bytes(int S, int MT)
 {
-    return 1024 + (uint32_t)S * dw_stage_bytes(NT) + kDwBarBytes + kDwBiasBytes;
+    return 1024 + (uint32_t)S * dw_stage_bytes(MT) + kDwBarBytes + kDwBiasBytes;
 }
 
 // 8 fp32 values, one whole 32-byte sector (address 32-byte aligned)
@@ -52,14 +54,16 @@ __device__ __forceinline__ void st32f(float *p, const float *v)
                  : "memory");
 }
 
-template <int NT>
+template <int MT>
 __global__ void __launch_bounds__(kDwThreads, 1)
 dw_ws(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtensorMap tm_h,
       const __grid_constant__ CUtensorMap tm_g, DwWsArgs a)
 {
-    constexpr int NACC = NT / 256;
-    constexpr uint32_t kCols = NT;
-    constexpr uint32_t kStage = dw_stage_bytes(NT);
+    constexpr int NT = kDwN;
+    constexpr int MB = MT / 64;      // m blocks per tile
+    constexpr int NACC = MT / 128;   // accumulators: one per 128 m rows
+    constexpr uint32_t kCols = NACC * NT;
+    constexpr uint32_t kStage = dw_stage_bytes(MT);
     extern __shared__ uint8_t smem_raw[];
     uint8_t *base = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
     const int S = a.S;
@@ -80,10 +84,10 @@ dw_ws(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtensor
     const int KC = c_hi - c_lo;
     const bool do_bias = mt == 0;
     const long long limit = a.limit;
-    // kinds of the two m blocks: 0 x, 1 h, 2 zero
-    int kind[2], m0[2];
-    for (int j = 0; j < 2; ++j) {
-        const int blk = 2 * mt + j;
+    // kinds of the m blocks: 0 x, 1 h, 2 zero
+    int kind[MB], m0[MB];
+    for (int j = 0; j < MB; ++j) {
+        const int blk = MB * mt + j;
         kind[j] = blk < a.kbx ? 0 : blk < a.kbx + a.kbh ? 1 : 2;
         m0[j] = kind[j] == 0 ? blk * 64 : (blk - a.kbx) * 64;
     }
@@ -99,7 +103,7 @@ dw_ws(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtensor
         tc::fence_mbar_init();
     }
     // constant zero blocks, in every stage (never overwritten by a copy)
-    for (int j = 0; j < 2; ++j)
+    for (int j = 0; j < MB; ++j)
         if (kind[j] == 2)
             for (int s = 0; s < S; ++s)
                 for (uint32_t i = tid; i < kBlk / 16; i += kDwThreads)
@@ -118,7 +122,8 @@ dw_ws(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtensor
 
     if (warp == 4) {
         if (lane == 0) {
-            const uint32_t bytes = (uint32_t)((kind[0] != 2) + (kind[1] != 2)) * kBlk + NT * 128;
+            uint32_t bytes = NT * 128;
+            for (int j = 0; j < MB; ++j) bytes += kind[j] != 2 ? kBlk : 0u;
             int it = 0;
             for (; it < KC; ++it) {
                 const int s = it % S;
@@ -129,10 +134,10 @@ dw_ws(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtensor
                 const uint32_t st = ring0 + s * kStage;
                 const int r0 = (c_lo + it) * 64;
                 tc::mbar_arrive_expect_tx(&full[s], bytes);
-                for (int j = 0; j < 2; ++j)
+                for (int j = 0; j < MB; ++j)
                     if (kind[j] != 2) tc::tma_load_2d(st + j * kBlk, kind[j] == 0 ? &tm_x : &tm_h, m0[j], r0, &full[s]);
                 for (int nb = 0; nb < NT / 64; ++nb)
-                    tc::tma_load_2d(st + 2 * kBlk + nb * kBlk, &tm_g, nt * NT + nb * 64, r0, &full[s]);
+                    tc::tma_load_2d(st + MB * kBlk + nb * kBlk, &tm_g, nt * NT + nb * 64, r0, &full[s]);
             }
             *n_issued = it;
         }
@@ -148,13 +153,13 @@ dw_ws(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtensor
                     break;
                 }
                 tc::tc_fence_after();
-                const uint32_t as = ring0 + s * kStage, bs = as + 2 * kBlk;
+                const uint32_t as = ring0 + s * kStage, bs = as + MB * kBlk;
 #pragma unroll
                 for (int k = 0; k < 4; ++k)  // 16 r-rows (two 8-row groups, 2048 bytes) per MMA
 #pragma unroll
-                    for (int h = 0; h < NACC; ++h)
-                        tc::mma_bf16(tmem + h * 256, tc::smem_desc(as + k * 2048, kBlk, 1024),
-                                     tc::smem_desc(bs + h * 4 * kBlk + k * 2048, kBlk, 1024), idesc, (it | k) != 0);
+                    for (int h = 0; h < NACC; ++h)  // m rows 128 h .. + 127: blocks 2 h, 2 h + 1
+                        tc::mma_bf16(tmem + h * NT, tc::smem_desc(as + 2 * h * kBlk + k * 2048, kBlk, 1024),
+                                     tc::smem_desc(bs + k * 2048, kBlk, 1024), idesc, (it | k) != 0);
                 tc::mma_commit(&empty[s]);
             }
             *n_consumed = it;  // chunks whose copies this warp saw land
@@ -175,7 +180,7 @@ dw_ws(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtensor
                     fail();
                     break;
                 }
-                const uint8_t *blk = base + (size_t)s * kStage + 2 * kBlk + nb * kBlk;
+                const uint8_t *blk = base + (size_t)s * kStage + MB * kBlk + nb * kBlk;
 #pragma unroll 4
                 for (int r = sub * RPT; r < (sub + 1) * RPT; ++r) {
                     const uint4 v = *(const uint4 *)(blk + sw128(r, q));
@@ -196,18 +201,21 @@ dw_ws(const __grid_constant__ CUtensorMap tm_x, const __grid_constant__ CUtensor
         if (!ok) fail();
         tc::tc_fence_after();
         if (ok && !*abort) {
-            const size_t m = (size_t)mt * 128 + warp * 32 + lane;
-            float *dst = a.part + ((size_t)sp * a.rows_part + m) * a.ld_part + (size_t)nt * NT;
-            const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
 #pragma unroll 1
-            for (int c16 = 0; c16 < NT / 16; ++c16) {
-                float v[16];
-                tc::tmem_ld16(trow + c16 * 16, v);
-                if (KC == 0)
+            for (int h = 0; h < NACC; ++h) {
+                const size_t m = (size_t)mt * MT + h * 128 + warp * 32 + lane;
+                float *dst = a.part + ((size_t)sp * a.rows_part + m) * a.ld_part + (size_t)nt * NT;
+                const uint32_t trow = tmem + h * NT + ((uint32_t)(warp * 32) << 16);
+#pragma unroll 1
+                for (int c16 = 0; c16 < NT / 16; ++c16) {
+                    float v[16];
+                    tc::tmem_ld16(trow + c16 * 16, v);
+                    if (KC == 0)
 #pragma unroll
-                    for (int i = 0; i < 16; ++i) v[i] = 0.0f;
-                st32f(dst + c16 * 16, v);
-                st32f(dst + c16 * 16 + 8, v + 8);
+                        for (int i = 0; i < 16; ++i) v[i] = 0.0f;
+                    st32f(dst + c16 * 16, v);
+                    st32f(dst + c16 * 16 + 8, v + 8);
+                }
             }
         }
         if (do_bias) {
@@ -263,27 +271,56 @@ __global__ void dw_reduce_pad(int I, int H, int kbx, int split, const float *__r
 
 }  // namespace
 
-// Tile width, splits and ring depth, as measured best on this GPU: 256-column tiles with
-// a two-stage ring, so that two CTAs share an SM and one's partial-sum epilogue overlaps
-// the other's contraction; splits enough for about two waves of such pairs (at least 16
-// chunks per CTA). 512-column tiles (one CTA per SM) and fewer, longer splits measured
-// slower (stress: 2.03 ms against 1.82 ms; large: 0.68 ms against 0.52 ms).
+// Tile shape, splits and ring depth. 128 x 256 tiles run two CTAs an SM (one's partial-sum
+// epilogue overlaps the other's contraction) with a two-stage ring, splits for about two
+// waves of such pairs (at least 16 chunks per CTA); their MMAs need about 94 bytes of
+// operands a cycle per SM at the full tensor rate, more than TMA delivers (they ran at
+// 70-81 % of it). 256 x 256 tiles share one dG operand between two accumulators: one CTA
+// an SM, a three-stage ring, and about 62 bytes a cycle. Cost (cycles) = waves x chunks per
+// CTA x cycles per chunk (measured) + the split partial sums written and read back at the
+// HBM rate; the split count with the least; 512-column tiles and fewer, longer splits
+// measured slower. Test hook (include/stacklstm.h): STACKLSTM_DW_M = 128 or 256 fixes the
+// tile's m size.
 cudaError_t bf16_plan_dw(stacklstm *s)
 {
     const int I = s->I, H = s->H, sms = s->num_sms;
     const size_t R = (size_t)s->T * s->B, RC = ceil_div(R, 64);
     const int kbx = (int)ceil_div(I, 64), kbh = (int)ceil_div(H, 64);
-    const int n_mt = (kbx + kbh + 1) / 2;
-    s->dw_ntile = 256;
-    s->dw_nt = (int)ceil_div(4 * H, 256);
-    const size_t tiles = (size_t)n_mt * s->dw_nt, want = 4 * (size_t)sms;  // two waves of two CTAs per SM
     const size_t max_split = std::max<size_t>(1, RC / 16);
-    s->dw_split = (int)std::min(max_split, std::max<size_t>(1, ceil_div(want, tiles)));
-    s->dw_mt = n_mt;
-    s->sw = 2;
-    s->dw_part_elems = (size_t)s->dw_split * ((size_t)n_mt * 128 + 1) * ((size_t)s->dw_nt * s->dw_ntile);
+    s->dw_ntile = kDwN;
+    s->dw_nt = (int)ceil_div(4 * H, kDwN);
+    // partial sums of `sp` splits over `rows` padded m rows: written, then read by the reduction
+    auto part_cycles = [&](size_t sp, size_t rows) {
+        return (double)sp * rows * s->dw_nt * kDwN * 4 * 2 / 6.8e12 * 1.92e9;
+    };
+    // 128 x 256, two CTAs an SM: splits for about two waves of pairs
+    const int mt128 = (kbx + kbh + 1) / 2;
+    const size_t tiles128 = (size_t)mt128 * s->dw_nt;
+    const size_t split128 = std::min(max_split, std::max<size_t>(1, ceil_div(4 * (size_t)sms, tiles128)));
+    const double cost128 = (double)ceil_div(tiles128 * split128, 2 * (size_t)sms) * ceil_div(RC, split128) * 1460.0 +
+                           part_cycles(split128, (size_t)mt128 * 128);
+    // 256 x 256, one CTA an SM: the split count with the fewest waves x chunks
+    const int mt256 = (kbx + kbh + 3) / 4;
+    const size_t tiles256 = (size_t)mt256 * s->dw_nt;
+    size_t split256 = 1;
+    double cost256 = 1e300;
+    for (size_t sp = 1; sp <= max_split; ++sp) {
+        const double c = (double)ceil_div(tiles256 * sp, (size_t)sms) * ceil_div(RC, sp) * 1140.0 +
+                         part_cycles(sp, (size_t)mt256 * 256);
+        if (c < cost256 * 0.999) {
+            cost256 = c;
+            split256 = sp;
+        }
+    }
+    const char *fm = getenv("STACKLSTM_DW_M");
+    const bool big = fm ? atoi(fm) == 256 : cost256 < cost128;
+    s->dw_mtile = big ? 256 : 128;
+    s->dw_mt = big ? mt256 : mt128;
+    s->dw_split = (int)(big ? split256 : split128);
+    s->sw = big ? 3 : 2;
+    s->dw_part_elems = (size_t)s->dw_split * ((size_t)s->dw_mt * s->dw_mtile + 1) * ((size_t)s->dw_nt * kDwN);
     cudaError_t e;
-    if ((e = allow_smem(dw_ws<512>)) || (e = allow_smem(dw_ws<256>))) return e;
+    if ((e = allow_smem(dw_ws<256>)) || (e = allow_smem(dw_ws<128>))) return e;
     return cudaSuccess;
 }
 
@@ -302,17 +339,17 @@ cudaError_t bf16_launch_dw(stacklstm *s, const CUtensorMap &tm_x, const CUtensor
     w.S = s->sw;
     w.part = s->dw_part;
     w.ld_part = (size_t)s->dw_nt * s->dw_ntile;
-    w.rows_part = (size_t)s->dw_mt * 128 + 1;
+    w.rows_part = (size_t)s->dw_mt * s->dw_mtile + 1;
     w.limit = s->wait_limit;
     w.err = s->err;
     const dim3 grid(s->dw_mt * s->dw_nt, w.split);
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = grid;
     cfg.blockDim = dim3(kDwThreads);
-    cfg.dynamicSmemBytes = dw_smem_bytes(s->sw, s->dw_ntile);
+    cfg.dynamicSmemBytes = dw_smem_bytes(s->sw, s->dw_mtile);
     cfg.stream = s->stream;
-    cudaError_t e = s->dw_ntile == 512 ? cudaLaunchKernelEx(&cfg, dw_ws<512>, tm_x, tm_h, tm_g, w)
-                                       : cudaLaunchKernelEx(&cfg, dw_ws<256>, tm_x, tm_h, tm_g, w);
+    cudaError_t e = s->dw_mtile == 256 ? cudaLaunchKernelEx(&cfg, dw_ws<256>, tm_x, tm_h, tm_g, w)
+                                       : cudaLaunchKernelEx(&cfg, dw_ws<128>, tm_x, tm_h, tm_g, w);
     if (e) return e;
     const size_t n = (size_t)(s->I + s->H + 1) * s->H;
     const unsigned blocks = (unsigned)std::max<size_t>(1, std::min<size_t>(ceil_div(n, 256), (size_t)s->num_sms * 16));

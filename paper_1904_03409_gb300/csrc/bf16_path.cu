@@ -619,10 +619,10 @@ std::string bf16_describe(const stacklstm *s)
              "backward %s U=%d [EP %d G %d ring %d slots %d cluster %d col tiles %d w_res %d smem %u threads %d "
              "per SM %d "
              "contraction parts %d dx CTAs %d ring %d]; "
-             "step rings fwd %d bwd %d; dx N=%d x%d ring %d; dW %dx%d tiles of 128x%d x%d splits ring %d",
+             "step rings fwd %d bwd %d; dx N=%d x%d ring %d; dW %dx%d tiles of %dx%d x%d splits ring %d",
              rt, s->kcf, s->kcx, s->kcb, s->cc.on ? "cuda-core" : s->fc.on ? "cluster" : f.on ? "persistent" : "per-step", s->uf, f.EP, f.G, f.S, f.slot, f.cl, f.n_ct,
              f.w_res, f.smem, f.threads, f.per_sm, s->cc.on ? "cuda-core" : s->bc.on ? "cluster" : b.on ? "persistent" : "per-step", s->bc.on ? s->bc.U : s->ub, b.EP, b.G, b.S, b.slot, b.cl, b.n_ct,
-             b.w_res, b.smem, b.threads, b.per_sm, b.KS, b.n_dx, b.dx_S, s->sf, s->sb, s->nx, s->nxt, s->sx, s->dw_mt, s->dw_nt, s->dw_ntile, s->dw_split, s->sw);
+             b.w_res, b.smem, b.threads, b.per_sm, b.KS, b.n_dx, b.dx_S, s->sf, s->sb, s->nx, s->nxt, s->sx, s->dw_mt, s->dw_nt, s->dw_mtile, s->dw_ntile, s->dw_split, s->sw);
     return buf;
 }
 

@@ -121,6 +121,7 @@ struct stacklstm {
     int nx = 0, nxt = 0;     // input gradient: columns per tile, number of column tiles
     int dw_mt = 0, dw_nt = 0, dw_split = 0;  // weight gradient: m tiles, column tiles, splits
     int dw_ntile = 0;                        // weight gradient: gate columns per tile
+    int dw_mtile = 0;                        // weight gradient: m rows per tile (128 or 256)
     long long wait_limit = 0;  // clock cycles one bounded device-side wait may spin
 
     // launch accounting and optional per-phase event timing (api.cu)

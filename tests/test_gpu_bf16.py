@@ -202,6 +202,20 @@ def test_split_contraction_backward_matches_oracle(T, B, I, H, seed, cl):
         assert np.array_equal(got[k], again[k]), k
 
 
+@pytest.mark.parametrize("T,B,I,H,seed", [(20, 200, 24, 40, 27), (9, 300, 136, 72, 28), (12, 130, 264, 64, 29)])
+def test_weight_gradient_tile_shapes_match_oracle(T, B, I, H, seed):
+    """The weight gradient with 128 x 256 tiles (two CTAs an SM) and with 256 x 256 tiles
+    (two accumulators over one dG operand, one CTA an SM), into NaN-filled outputs: x and h
+    blocks of W in one tile, constant zero blocks past I + H (I = 264: five x blocks and one
+    h block), ragged gate columns (4H = 160, 288)."""
+    w = case(T, B, I, H, seed, bias_scale=0.3, h0_scale=0.5, c0_scale=0.5, dy_scale=0.5)
+    ref = oracle_all(w)
+    for m in ("128", "256"):
+        plan, got = run_nan_filled(w, {"STACKLSTM_DW_M": m})
+        assert "tiles of %sx256" % m in plan, plan
+        compare(got, ref, "bf16")
+
+
 def run_nan_filled(w, env):
     """Forward + backward with every output buffer filled with NaN first (an element the
     path fails to write cannot pass), under extra environment settings; (plan, dx)."""
