@@ -14,6 +14,8 @@
 //     two tensor-memory accumulators, so tile k + 1 is multiplied while tile k's epilogue
 //     runs. An mbarrier wait between MMAs stalls MMA issue for a few hundred cycles, so a
 //     wait covers a whole stage;
+//   release (warp 4 EP + 2): raises the row tile's step counter once the epilogue warps
+//     have written a tile (its release fence waits for their writes, off their path);
 //   epilogue (warps 0 .. 4 EP - 1): warp w reads accumulator lanes 32 (w mod 4) .. + 31
 //     (rows) for unit part w / 4. Forward: the LSTM cell, history row t + 1 and the h
 //     operand of step t + 1. Backward: adds dh_read to the gradient of the state step t
@@ -62,7 +64,7 @@ struct WsArgs {
 // Dynamic shared memory: [weight tile (w_res)][S stages: G A chunks, then G weight
 // chunks unless resident][forward: gate staging tile][split contraction in a cluster:
 // partial-sum exchange tile][barriers], based at the first 1024-byte boundary.
-constexpr uint32_t kBarBytes = (2 * kMaxStages + 7) * 8 + 16;
+constexpr uint32_t kBarBytes = (2 * kMaxStages + 7) * 8 + 32;
 
 // forward: what one tile writes to the history apart from the h operand of the next step,
 // staged for the tensor stores that write it out: the activated gates (4 gates x 128 rows
@@ -98,6 +100,7 @@ struct WCtl {
     uint32_t *tmem_slot;
     int *n_issued, *n_consumed;  // groups armed by the producer / consumed by the MMA warp
     volatile int *abort;
+    volatile int *rel_end;  // tiles the epilogue completed, written before its last barrier with the release warp
 };
 
 __device__ __forceinline__ WCtl wcarve(uint8_t *raw, int S, int G, int NB, int KC, int w_res, uint32_t stg,
@@ -124,6 +127,7 @@ __device__ __forceinline__ WCtl wcarve(uint8_t *raw, int S, int G, int NB, int K
     c.n_issued = (int *)(c.tmem_slot + 1);
     c.n_consumed = c.n_issued + 1;
     c.abort = (volatile int *)(c.n_consumed + 1);
+    c.rel_end = c.abort + 1;
     return c;
 }
 
@@ -303,6 +307,20 @@ __device__ __forceinline__ uint32_t stg_swz(uint32_t r, uint32_t q)
 }
 
 // ------------------------------------------------------------------ epilogue
+// Named barrier of the epilogue warps with the release warp, once a tile. The release
+// (`red.release.gpu`) waits for every earlier memory operation to be performed, about
+// 1.4-1.8 K cycles. The backward whose epilogue is its bottleneck (32-unit tiles, four lanes
+// a row, several row tiles a CTA) hands it to a warp of its own, off the epilogue's path
+// (-4.7 %). Elsewhere thread 0 of the epilogue releases: there the counter is on the step
+// chain, and the fence of a separate warp also waited for the stores and loads the
+// epilogue issued after the barrier (large backward +5.6 %, stress forward +6 %).
+constexpr int kRelBar = 4;
+template <int U, int EP, bool kFwd, int KS>
+__host__ __device__ constexpr bool rel_warp()
+{
+    return !kFwd && KS == 1 && EP == 1 && U == 32 && defer_dhist<EP>();
+}
+
 struct EpiCtx {
     WCtl c;
     uint32_t tmem;
@@ -354,7 +372,8 @@ __device__ __forceinline__ void epilogue_loop(const StepArgs &a, const WsArgs &p
     constexpr bool kLatePfBwd = UE > 16;  // backward: operands taken group by group (below)
     // backward, 32 units a thread, unsplit contraction: four lanes per row (below)
     constexpr bool kRows4 = !kFwd && KS == 1 && EP == 1 && UE == 32 && defer_dhist<EP>();
-    for (int k = 0; k < e.n_tiles; ++k) {
+    int k = 0;
+    for (; k < e.n_tiles; ++k) {
         const int ks = k / e.n_mine, rt = e.slot + (k % e.n_mine) * p.n_slot;
         const int t = kFwd ? ks : T - 1 - ks;
         const int b = rt * kRows + e.q * 32 + e.lane;
@@ -787,13 +806,18 @@ __device__ __forceinline__ void epilogue_loop(const StepArgs &a, const WsArgs &p
             d_s1 = s1;
         }
         if (kFwd ? !pf_early : kLatePfBwd) prefetch_next();
-        // the next step reads these rows by TMA: generic writes -> async proxy, then
-        // release the step for this row tile
+        // the next step reads these rows by TMA: generic writes -> async proxy; then, with
+        // the release warp, which releases the step for this row tile while this tile's
+        // remaining stores go out and the next tile starts
         tc::fence_proxy_async_global();
         if constexpr (kFwd) tc::fence_proxy_async();  // staging-tile writes -> the tensor store
         __syncwarp();
-        tc::bar_sync(2, E * 32);
-        if (e.tid == 0) tc::red_release_gpu_add(p.cnt + rt * p.cs, 1);
+        if constexpr (rel_warp<U, EP, kFwd, KS>()) {
+            tc::bar_sync(kRelBar, (E + 1) * 32);
+        } else {
+            tc::bar_sync(2, E * 32);
+            if (e.tid == 0) tc::red_release_gpu_add(p.cnt + rt * p.cs, 1);
+        }
         if constexpr (kRows4) {
             const int sub = e.lane & 3, us = u0 + 8 * sub;
 #pragma unroll
@@ -839,6 +863,12 @@ __device__ __forceinline__ void epilogue_loop(const StepArgs &a, const WsArgs &p
         }
         cur0 = nx0;
         cur1 = nx1;
+    }
+    // the release warp's last barrier, after every tile (or after an abort, at the tile the
+    // epilogue left): the tiles completed, k, tell it that this one releases nothing
+    if constexpr (rel_warp<U, EP, kFwd, KS>()) {
+        if (e.tid == 0) *e.c.rel_end = k;
+        tc::bar_sync(kRelBar, (E + 1) * 32);
     }
     if constexpr (kFwd)
         if (e.lane == 0) tc::bulk_wait();  // the history stores completed before the CTA exits
@@ -975,7 +1005,7 @@ __device__ __forceinline__ void dx_role(const CUtensorMap *tm_g, const WsArgs &p
             tc::mma_commit(c.done);
         }
         __syncwarp();
-    } else {
+    } else if (warp < E) {
         // ------------------------------------------------------------ epilogue
         const int q = warp & 3, part = warp >> 2;
         for (int j = 0; j < n_mine; ++j) {
@@ -1042,7 +1072,7 @@ __device__ __forceinline__ void dx_role(const CUtensorMap *tm_g, const WsArgs &p
 // KS > 1 (backward): the KS CTAs blockIdx = (slot, ct, kp) split the contraction; part kp
 // takes chunks [KC kp / KS, KC (kp + 1) / KS) and keeps only that slice of the weight tile.
 template <int U, int EP, int G, bool kFwd, int KS>
-__global__ void __launch_bounds__(32 * (4 * EP + 2), 1)
+__global__ void __launch_bounds__(32 * (4 * EP + 3), 1)
 step_ws(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtensorMap tm_b,
         const __grid_constant__ CUtensorMap tm_gates, const __grid_constant__ CUtensorMap tm_hh,
         const __grid_constant__ CUtensorMap tm_hc, WsArgs p)
@@ -1097,6 +1127,7 @@ step_ws(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtens
         *c.n_issued = 0;
         *c.n_consumed = 0;
         *c.abort = 0;
+        *c.rel_end = 0x7fffffff;
         tc::fence_mbar_init();
     }
     if (warp == E) tc::tmem_alloc(c.tmem_slot, 2 * kCols);
@@ -1226,6 +1257,21 @@ step_ws(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtens
             tc::mma_commit(c.done);  // arrives once every MMA issued above has completed
         }
         __syncwarp();
+    } else if (warp == E + 2) {
+        // ------------------------------------------------------------ release
+        // (only where rel_warp: see kRelBar) once the epilogue warps of tile k have written
+        // and fenced its rows (their barrier), count the step done for the tile's row tile,
+        // with release semantics. The epilogue ends with one more barrier, before which it
+        // records the tiles it completed: that barrier (k == *rel_end) releases nothing and
+        // ends this loop, also after an abort
+        if constexpr (rel_warp<U, EP, kFwd, KS>()) {
+            for (int k = 0;; ++k) {
+                tc::bar_sync(kRelBar, (E + 1) * 32);
+                if (k >= *c.rel_end) break;
+                if (lane == 0) tc::red_release_gpu_add(p.cnt + (slot + (k % n_mine) * p.n_slot) * p.cs, 1);
+                __syncwarp();
+            }
+        }
     } else {
         // ------------------------------------------------------------ epilogue
         constexpr int NG = UE % 16 == 0 ? 16 : 8;
@@ -1331,7 +1377,7 @@ bool plan_variant(const Variant &v, bool fwd, int KC, int split, int n_rt, int H
                   PersistPlan *pl, double *cost)
 {
     const int NB = fwd ? 4 * v.U : v.U, n_ct = (H + v.U - 1) / v.U;
-    const int threads = 32 * (4 * v.EP + 2);
+    const int threads = 32 * (4 * v.EP + 3);  // epilogue warps, producer, MMA issue, release
     const uint32_t kcols2 = 2u * (NB <= 32 ? 32 : NB <= 64 ? 64 : NB <= 128 ? 128 : 256);
     const int KCl = (KC + v.KS - 1) / v.KS;  // chunks of one contraction part
     const int groups = (split + v.G - 1) / v.G + (KCl - split + v.G - 1) / v.G;
