@@ -45,6 +45,9 @@
  *   STACKLSTM_WAIT_LIMIT_CYCLES=n  clock budget of one bounded device-side wait
  *                                  (default 4e9); 0 makes every wait run out at once, so
  *                                  calls report SL_ERR_TIMEOUT
+ *   STACKLSTM_WAIT_LIMIT_BWD_CYCLES=n  the same budget for the backward's kernels only
+ *                                  (default: STACKLSTM_WAIT_LIMIT_CYCLES), so that a
+ *                                  forward can complete before the backward times out
  *   STACKLSTM_STEP_KERNELS=1       one launch per time step instead of the persistent and
  *                                  cluster kernels (fp32: instead of one CTA for all steps)
  *   STACKLSTM_FWD_CLUSTER=0        no thread-block-cluster forward for one row tile

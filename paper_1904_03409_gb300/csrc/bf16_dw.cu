@@ -340,7 +340,7 @@ cudaError_t bf16_launch_dw(stacklstm *s, const CUtensorMap &tm_x, const CUtensor
     w.part = s->dw_part;
     w.ld_part = (size_t)s->dw_nt * s->dw_ntile;
     w.rows_part = (size_t)s->dw_mt * s->dw_mtile + 1;
-    w.limit = s->wait_limit;
+    w.limit = s->wait_limit_bwd;
     w.err = s->err;
     const dim3 grid(s->dw_mt * s->dw_nt, w.split);
     cudaLaunchConfig_t cfg = {};

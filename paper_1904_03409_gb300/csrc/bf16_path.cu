@@ -604,6 +604,13 @@ StepArgs step_args(stacklstm *s, const float *bias, const void *wpack, int kcx, 
     a.limit = s->wait_limit; a.err = s->err;
     return a;
 }
+// the backward's step arguments: as step_args, with the backward's wait budget
+StepArgs bwd_args(stacklstm *s, const void *wpack, int KC, int S)
+{
+    StepArgs a = step_args(s, nullptr, wpack, 0, KC, S);
+    a.limit = s->wait_limit_bwd;
+    return a;
+}
 
 }  // namespace
 
@@ -649,6 +656,9 @@ cudaError_t bf16_prepare(stacklstm *s)
     // test hook (include/stacklstm.h): the clock budget of one device-side wait
     const char *lim = getenv("STACKLSTM_WAIT_LIMIT_CYCLES");
     s->wait_limit = lim ? atoll(lim) : 4000000000LL;
+    // test hook: the backward's kernels alone (so that a forward can run before they time out)
+    const char *limb = getenv("STACKLSTM_WAIT_LIMIT_BWD_CYCLES");
+    s->wait_limit_bwd = limb ? atoll(limb) : s->wait_limit;
     if ((e = allow_smem(fwd_step_tc<32>)) || (e = allow_smem(fwd_step_tc<16>)) || (e = allow_smem(fwd_step_tc<8>)) ||
         (e = allow_smem(bwd_step_tc<32>)) || (e = allow_smem(bwd_step_tc<16>)) || (e = allow_smem(dx_tc<32>)) ||
         (e = allow_smem(dx_tc<64>)) || (e = allow_smem(dx_tc<128>)) || (e = allow_smem(dx_tc<256>)))
@@ -846,7 +856,7 @@ cudaError_t bf16_forward_steps(stacklstm *s, const float *bias)
 // Pointwise backward of the last step, before the reverse loop.
 cudaError_t bf16_backward_setup(stacklstm *s, const float *d_top_h)
 {
-    StepArgs a = step_args(s, nullptr, s->w_bwd, 0, s->kcb, s->sb);
+    StepArgs a = bwd_args(s, s->w_bwd, s->kcb, s->sb);
     a.gates_blk = s->fc.on && s->bc.on;  // the layout the cluster forward wrote for the cluster backward
     // the final top's history row of each instance (virtual, in push-only mode)
     const int32_t *ftop = (s->push_only ? s->vy : s->top) + (size_t)s->T * s->B;
@@ -861,13 +871,13 @@ cudaError_t bf16_backward_steps(stacklstm *s, float *dx, bool *dx_done)
     *dx_done = false;
     const int T = s->Tr, B = s->B, H = s->H;
     cudaError_t e;
-    const StepArgs a = step_args(s, nullptr, s->w_bwd, 0, s->kcb, s->sb);
-    if (s->cc.on) return bf16_launch_bwd_small(s, step_args(s, nullptr, s->w_ccb, 0, s->kcb, 0));
-    if (s->bc.on) return bf16_launch_bwd_cluster(s, step_args(s, nullptr, s->w_bcl, 0, s->kcb, 0));
+    const StepArgs a = bwd_args(s, s->w_bwd, s->kcb, s->sb);
+    if (s->cc.on) return bf16_launch_bwd_small(s, bwd_args(s, s->w_ccb, s->kcb, 0));
+    if (s->bc.on) return bf16_launch_bwd_cluster(s, bwd_args(s, s->w_bcl, s->kcb, 0));
     // one row tile of at most 64 instances: 64-row boxes (the rest of each stage is never
     // loaded and only feeds accumulator rows that are not stored)
     if (s->pb.on)
-        return bf16_launch_bwd_persist(s, step_args(s, nullptr, s->w_bwd, 0, s->kcb, s->pb.S),
+        return bf16_launch_bwd_persist(s, bwd_args(s, s->w_bwd, s->kcb, s->pb.S),
                                        map(s, B <= 64 ? kMapG64 : kMapG128), dx, dx_done);
     const dim3 grid(ceil_div(H, s->ub), ceil_div(B, kRows));
     const size_t smem = smem_bytes(s->sb, s->ub);
@@ -910,7 +920,7 @@ cudaError_t bf16_forward_steps_group(stacklstm *const *hs, int n, const float *c
 cudaError_t bf16_backward_steps_group(stacklstm *const *hs, int n, cudaStream_t st)
 {
     StepArgs as[kMaxGroup];
-    for (int m = 0; m < n; ++m) as[m] = step_args(hs[m], nullptr, hs[m]->w_bcl, 0, hs[m]->kcb, 0);
+    for (int m = 0; m < n; ++m) as[m] = bwd_args(hs[m], hs[m]->w_bcl, hs[m]->kcb, 0);
     return bf16_launch_bwd_cluster_group(hs, as, n, st);
 }
 
@@ -920,7 +930,7 @@ cudaError_t bf16_dx(stacklstm *s, float *dx)
     const size_t R = (size_t)s->Tr * s->B;
     DxArgs d;
     d.R = R; d.I = s->I; d.KC = s->kcb; d.S = s->sx;
-    d.wpack = (const uint8_t *)s->w_dx; d.dx = dx; d.limit = s->wait_limit; d.err = s->err;
+    d.wpack = (const uint8_t *)s->w_dx; d.dx = dx; d.limit = s->wait_limit_bwd; d.err = s->err;
     d.xidx = s->push_only ? s->xidx : nullptr;
     d.B = s->B;
     const dim3 g(s->nxt, ceil_div(R, kRows));

@@ -123,6 +123,7 @@ struct stacklstm {
     int dw_ntile = 0;                        // weight gradient: gate columns per tile
     int dw_mtile = 0;                        // weight gradient: m rows per tile (128 or 256)
     long long wait_limit = 0;  // clock cycles one bounded device-side wait may spin
+    long long wait_limit_bwd = 0;  // the same for the backward's kernels (its own test hook)
 
     // launch accounting and optional per-phase event timing (api.cu)
     long long launches = 0;  // kernel launches of this library, running total

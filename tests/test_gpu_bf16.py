@@ -166,6 +166,55 @@ def test_wait_timeout_is_reported_and_context_survives(B, env):
     compare(runner.run(w), oracle_all(w), "bf16")
 
 
+@pytest.mark.parametrize("T,B,I,H,env,want", [
+    (6, 200, 64, 256, dict(PERSISTENT, STACKLSTM_BWD_SPLIT="4"), "cluster 4 "),  # split contraction, clusters
+    (4, 4096, 256, 256, {}, "U=32 [EP 1"),                                      # the release warp's plan
+    (6, 200, 64, 256, dict(PERSISTENT, STACKLSTM_BWD_SPLIT="4", STACKLSTM_SPLIT_CLUSTER="0"), "cluster 1 "),
+    (6, 40, 64, 64, {}, "cluster U=16 ["),                                       # one-row-tile cluster
+])
+def test_backward_wait_timeout_is_reported_and_context_survives(T, B, I, H, env, want):
+    """With a zero wait budget for the backward's kernels only, the forward completes and the
+    backward reports SL_ERR_TIMEOUT instead of hanging: the persistent backward with its
+    contraction split in thread-block clusters (partials in flight between the parts) or
+    through L2, the one whose release warp waits at a barrier with the epilogue, and the
+    cluster backward. The device stays usable: a new handle then reproduces a normal run
+    bit for bit."""
+    w = case(T, B, I, H, 10, bias_scale=0.3, h0_scale=0.5)
+
+    def with_env(extra, fn):
+        keys = dict(env, **extra)
+        old = {k: os.environ.get(k) for k in keys}
+        os.environ.update(keys)
+        try:
+            return fn()
+        finally:
+            for k, v in old.items():
+                if v is None:
+                    os.environ.pop(k, None)
+                else:
+                    os.environ[k] = v
+
+    ref = with_env({}, lambda: runner.run(w))
+    hd = with_env({"STACKLSTM_WAIT_LIMIT_BWD_CYCLES": "0"},
+                  lambda: bd.stacklstm_create(w.T, w.B, w.I, w.H, bd.SL_BF16, 0))
+    try:
+        assert want in bd.stacklstm_plan(hd).split("; backward ")[1], bd.stacklstm_plan(hd)
+        ins, out = runner.upload(w), runner.alloc_outputs(w)
+        bd.stacklstm_forward(hd, ins["x"], ins["ops"], ins["h0"], ins["c0"], ins["W"], ins["bias"],
+                             p_final=out["p_final"])
+        bd.stacklstm_status(hd)
+        with pytest.raises(bd.StackLSTMError) as e:
+            bd.stacklstm_backward(hd, ins["d_top_h"], None, out["dx"], out["dh0"], out["dc0"], out["dW"],
+                                  out["dbias"])
+            bd.stacklstm_status(hd)
+        assert e.value.status == 6
+    finally:
+        hd.destroy()
+    again = with_env({}, lambda: runner.run(w))
+    for k in ("y", "h_stack", "c_stack", "dx", "dW", "dbias", "dh0", "dc0"):
+        assert np.array_equal(again[k], ref[k]), k
+
+
 @pytest.mark.parametrize("T,B,I,H,seed", [(20, 200, 24, 40, 12), (9, 300, 136, 72, 13)])
 def test_per_step_kernels_match_oracle(T, B, I, H, seed):
     """The one-launch-per-step kernels (used when a persistent grid cannot be
