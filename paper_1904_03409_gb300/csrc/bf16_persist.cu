@@ -1,6 +1,6 @@
 // bf16_persist.cu -- persistent, warp-specialised step kernels of the bf16 path: one
-// cooperative launch runs all T steps of the forward (Algorithm 1) or of the reverse-time
-// backward (Sec. 5).
+// launch (cooperative, or a cluster launch whose clusters all fit at once) runs all T steps
+// of the forward (Algorithm 1) or of the reverse-time backward (Sec. 5).
 //
 // Each CTA keeps one column tile ct (U hidden units: forward, the 4U gate columns of those
 // units; backward, U columns of dh_read = dG_t W_h^T) and a fixed set of row tiles
