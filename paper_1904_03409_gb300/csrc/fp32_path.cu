@@ -65,12 +65,22 @@ __global__ void fwd_step_f32(int t, int B, int I, int H, const float *__restrict
     gt[3 * H + j] = og;
 }
 
-__global__ void transpose_f32(int R, int C, const float *__restrict__ in, float *__restrict__ out)
+// The forward setup in one launch: history row 0 = (h0, c0), the initial state (stack
+// slot 0), and W^T (out[c][r] = in[r][c], R x C) for the backward contractions, so that the
+// backward needs nothing the caller owns.
+__global__ void setup_f32(int n0, const float *__restrict__ h0, const float *__restrict__ c0,
+                          float *__restrict__ hist_h, float *__restrict__ hist_c, int R, int C,
+                          const float *__restrict__ in, float *__restrict__ out)
 {
-    const size_t n = (size_t)R * C;
-    for (size_t e = blockIdx.x * (size_t)blockDim.x + threadIdx.x; e < n; e += (size_t)gridDim.x * blockDim.x) {
-        const size_t r = e / C, c = e - r * C;
-        out[c * R + r] = in[e];
+    const size_t n = (size_t)R * C, stride = (size_t)gridDim.x * blockDim.x;
+    for (size_t e = blockIdx.x * (size_t)blockDim.x + threadIdx.x; e < n + n0; e += stride) {
+        if (e < (size_t)n0) {
+            hist_h[e] = h0[e];
+            hist_c[e] = c0[e];
+        } else {
+            const size_t f = e - n0, r = f / C, c = f - r * C;
+            out[c * R + r] = in[f];
+        }
     }
 }
 
@@ -101,8 +111,9 @@ __global__ void bwd_pointwise_f32(int t, int B, int H, const int32_t *__restrict
     }
 }
 
-// dh_read = dG_t W_h^T added to row top[t]; grid (ceil(H / blockDim.x), B).
-__global__ void bwd_contract_f32(int t, int B, int I, int H, const int32_t *__restrict__ top,
+// dh_read = dG_t W_h^T added to row top[t]; grid (ceil(H / blockDim.x), B). P (1, 2 or 4,
+// from the shape: fwd_seq_threads_per_unit) is the one-CTA backward's split of the 4H sum.
+__global__ void bwd_contract_f32(int t, int B, int I, int H, int P, const int32_t *__restrict__ top,
                                  const float *__restrict__ WT, const float *__restrict__ dG,
                                  float *__restrict__ dhist_h)
 {
@@ -113,8 +124,14 @@ __global__ void bwd_contract_f32(int t, int B, int I, int H, const int32_t *__re
     __syncthreads();
     const int k = blockIdx.x * blockDim.x + threadIdx.x;
     if (k >= H) return;
+    // P partial sums over consecutive quarters (halves, the whole) of the 4H gate columns,
+    // added in part order: the one-CTA backward's split, in one thread
     float acc = 0.0f;
-    for (int n = 0; n < G; ++n) acc = fmaf(g_s[n], WT[(size_t)n * K + I + k], acc);
+    for (int p = 0; p < P; ++p) {
+        float sp = 0.0f;
+        for (int n = p * (G / P); n < (p + 1) * (G / P); ++n) sp = fmaf(g_s[n], WT[(size_t)n * K + I + k], sp);
+        acc = p == 0 ? sp : acc + sp;
+    }
     const int src = top[(size_t)t * B + b];
     dhist_h[((size_t)src * B + b) * H + k] += acc;
 }
@@ -159,12 +176,14 @@ __global__ void dw_f32(size_t R, int K, int G, const float *__restrict__ a_rm, c
     }
 }
 
-// Small problems (B * H <= 1024 threads, and the whole history in shared memory): all T
-// steps of a direction in one CTA, thread (b, j) = (tid / H, tid % H), __syncthreads()
-// between the phases of a step instead of a launch per step, and every row a step reads
-// taken from shared memory (the rows go to global memory as they are written). The
-// arithmetic of each element is that of the per-step kernels above (the same operands, k
-// and n ascending with fmaf), so both give the same bits.
+// Small problems (B * H <= 1024, and the whole history in shared memory): all T steps of a
+// direction in one CTA, P threads per (instance b, unit j) (as many of 4, 2, 1 as 1024 threads
+// allow), __syncthreads() between the phases of a step instead of a launch per step, and
+// every row a step reads taken from shared memory (the rows go to global memory as they are
+// written). The forward's P threads of a unit split its four gates' dot products, the
+// backward's its 4H-long contraction (in P consecutive parts, added in part order). The
+// arithmetic of each element is that of the per-step kernels above (the same operands, k and
+// n ascending with fmaf, the same P parts), so both give the same bits.
 // Shared memory: forward [B][K] operands, [K][4H] W, [T+1][B][H] h and c, [T][B][I] x,
 // [T+1][B] tops;
 // backward [4H][H] W_h^T, [T+1][B][H] c, dh and dc, [B][4H] the step's dG, [T+1][B] tops.
@@ -178,16 +197,23 @@ size_t bwd_seq_smem(int T, int B, int H)
     const size_t G = 4 * (size_t)H, R = (size_t)(T + 1) * B;
     return sizeof(float) * (G * H + 3 * R * H + (size_t)B * G) + sizeof(int32_t) * R;
 }
+// threads per (instance, unit) of the one-CTA forward: as many of 4, 2, 1 as 1024 allow
+int fwd_seq_threads_per_unit(int B, int H) { return B * H * 4 <= 1024 ? 4 : B * H * 2 <= 1024 ? 2 : 1; }
 
-__global__ void __launch_bounds__(1024) fwd_seq_f32(int T, int B, int I, int H, const float *__restrict__ x,
+// P threads per (instance, unit), P in {1, 2, 4}: each runs the dot products of 4 / P of the
+// unit's gates (every gate's fmaf chain as in fwd_step_f32, so the results are the same bit for
+// bit), and the first of them collects the four by shuffles for the cell.
+__global__ void __launch_bounds__(1024) fwd_seq_f32(int T, int B, int I, int H, int P, const float *__restrict__ x,
                                                     const float *__restrict__ W, const float *__restrict__ bias,
                                                     const int32_t *__restrict__ top, float *__restrict__ hist_h,
                                                     float *__restrict__ hist_c, float *__restrict__ gates,
                                                     float *__restrict__ a_rm)
 {
     extern __shared__ float sm[];
-    const int K = I + H, G = 4 * H, tid = threadIdx.x, b = tid / H, j = tid - b * H;
-    const bool mine = tid < B * H;
+    const int K = I + H, G = 4 * H, tid = threadIdx.x, u = tid / P, part = tid - u * P, GP = 4 / P;
+    const int b = u / H, j = u - b * H;
+    const bool mine = u < B * H;
+    const int lane = tid & 31;
     const size_t R = (size_t)(T + 1) * B;
     float *a_s = sm, *w_s = a_s + (size_t)B * K, *h_s = w_s + (size_t)K * G, *c_s = h_s + R * H;
     float *x_s = c_s + R * H;
@@ -209,17 +235,30 @@ __global__ void __launch_bounds__(1024) fwd_seq_f32(int T, int B, int I, int H, 
             a_rm[((size_t)t * B + bb) * K + k] = v;
         }
         __syncthreads();
+        float z[4] = {0.f, 0.f, 0.f, 0.f};  // gates part * GP .. + GP - 1 of unit (b, j)
         if (mine) {
             const float *as = a_s + (size_t)b * K;
-            float zi = bias[j], zf = bias[H + j], zg = bias[2 * H + j], zo = bias[3 * H + j];
-            for (int k = 0; k < K; ++k) {
-                const float av = as[k];
-                const float *Wk = w_s + (size_t)k * G;
-                zi = fmaf(av, Wk[j], zi);
-                zf = fmaf(av, Wk[H + j], zf);
-                zg = fmaf(av, Wk[2 * H + j], zg);
-                zo = fmaf(av, Wk[3 * H + j], zo);
-            }
+#pragma unroll
+            for (int i = 0; i < 4; ++i)
+                if (i < GP) {
+                    const int gc = (part * GP + i) * H + j;
+                    float zz = bias[gc];
+                    for (int k = 0; k < K; ++k) zz = fmaf(as[k], w_s[(size_t)k * G + gc], zz);
+                    z[i] = zz;
+                }
+        }
+        // gate g of the unit is value g mod GP of its part g / GP: to the unit's first thread
+        float zg4[4];
+#pragma unroll
+        for (int g = 0; g < 4; ++g) {
+            float v = z[0];
+#pragma unroll
+            for (int i = 1; i < 4; ++i)
+                if (g % GP == i) v = z[i];
+            zg4[g] = __shfl_sync(0xffffffffu, v, (lane & ~(P - 1)) + g / GP);
+        }
+        if (mine && part == 0) {
+            const float zi = zg4[0], zf = zg4[1], zg = zg4[2], zo = zg4[3];
             const float ig = sigmoidf(zi), fg = sigmoidf(zf), gg = tanhf(zg), og = sigmoidf(zo);
             const int src = top_s[t * B + b];
             const float cr = c_s[((size_t)src * B + b) * H + j];
@@ -240,14 +279,17 @@ __global__ void __launch_bounds__(1024) fwd_seq_f32(int T, int B, int I, int H, 
     }
 }
 
-__global__ void __launch_bounds__(1024) bwd_seq_f32(int T, int B, int I, int H, const int32_t *__restrict__ top,
+__global__ void __launch_bounds__(1024) bwd_seq_f32(int T, int B, int I, int H, int P, const int32_t *__restrict__ top,
                                                     const float *__restrict__ gates, const float *__restrict__ hist_c,
                                                     const float *__restrict__ WT, float *__restrict__ dhist_h,
                                                     float *__restrict__ dhist_c, float *__restrict__ dG)
 {
     extern __shared__ float sm[];
-    const int K = I + H, G = 4 * H, tid = threadIdx.x, b = tid / H, j = tid - b * H;
-    const bool mine = tid < B * H;
+    // P threads per (instance, unit): the unit's first runs the pointwise backward; all P the
+    // contraction, part p over gate columns [p G / P, (p + 1) G / P), summed in part order
+    const int K = I + H, G = 4 * H, tid = threadIdx.x, u = tid / P, part = tid - u * P;
+    const int b = u / H, j = u - b * H, lane = tid & 31;
+    const bool unit = u < B * H, mine = unit && part == 0;
     const size_t R = (size_t)(T + 1) * B;
     float *wh_s = sm, *c_s = wh_s + (size_t)G * H, *dh_s = c_s + R * H, *dc_s = dh_s + R * H;
     float *dg_s = dc_s + R * H;  // [B][4H]: dG of the current step
@@ -265,7 +307,7 @@ __global__ void __launch_bounds__(1024) bwd_seq_f32(int T, int B, int I, int H, 
         for (int g = 0; g < 4; ++g) gn[g] = gates[((size_t)(T - 1) * B + b) * G + g * H + j];
     __syncthreads();
     for (int t = T - 1; t >= 0; --t) {
-        const int src = mine ? top_s[t * B + b] : 0;
+        const int src = unit ? top_s[t * B + b] : 0;
         if (mine) {
             // pointwise backward of step t (bwd_pointwise_f32)
             const float ig = gn[0], fg = gn[1], gg = gn[2], og = gn[3];
@@ -284,13 +326,15 @@ __global__ void __launch_bounds__(1024) bwd_seq_f32(int T, int B, int I, int H, 
             dc_s[rd] += dc * fg;
         }
         __syncthreads();  // dG_t complete
-        if (mine) {
-            // dh_read = dG_t W_h^T added to the row step t read (bwd_contract_f32)
+        // dh_read = dG_t W_h^T added to the row step t read (bwd_contract_f32)
+        float sp = 0.0f;
+        if (unit) {
             const float *dg = dg_s + (size_t)b * G;
-            float acc = 0.0f;
-            for (int n = 0; n < G; ++n) acc = fmaf(dg[n], wh_s[n * H + j], acc);
-            dh_s[((size_t)src * B + b) * H + j] += acc;
+            for (int n = part * (G / P); n < (part + 1) * (G / P); ++n) sp = fmaf(dg[n], wh_s[n * H + j], sp);
         }
+        float acc = sp;
+        for (int p = 1; p < P; ++p) acc = acc + __shfl_sync(0xffffffffu, sp, (lane & ~(P - 1)) + p);
+        if (mine) dh_s[((size_t)src * B + b) * H + j] += acc;
         __syncthreads();  // the row's gradient is complete before step t - 1 reads it
     }
     // out: the gradient history (rows 0..T: dh0, dc0 among them)
@@ -331,13 +375,8 @@ std::string fp32_describe(stacklstm *s)
 cudaError_t fp32_forward_setup(stacklstm *s, const float *h0, const float *c0, const float *W)
 {
     const int B = s->B, I = s->I, H = s->H, K = I + H, G = 4 * H;
-    cudaError_t e;
-    // history row 0 = the initial state (stack slot 0)
-    if ((e = cudaMemcpyAsync(s->hist_h, h0, sizeof(float) * B * H, cudaMemcpyDeviceToDevice, s->stream))) return e;
-    if ((e = cudaMemcpyAsync(s->hist_c, c0, sizeof(float) * B * H, cudaMemcpyDeviceToDevice, s->stream)))
-        return e;
-    // W^T for the backward contractions (so backward needs nothing the caller owns)
-    transpose_f32<<<grid_for(s, (size_t)K * G, 256), 256, 0, s->stream>>>(K, G, W, (float *)s->w_fwd);
+    setup_f32<<<grid_for(s, (size_t)K * G + (size_t)B * H, 256), 256, 0, s->stream>>>(
+        B * H, h0, c0, (float *)s->hist_h, s->hist_c, K, G, W, (float *)s->w_fwd);
     s->launches += 1;
     return cudaGetLastError();
 }
@@ -347,8 +386,9 @@ cudaError_t fp32_forward_steps(stacklstm *s, const float *x, const float *W, con
     const int T = s->T, B = s->B, I = s->I, H = s->H, K = I + H;
     if (s->fp32_one_cta) {
         (void)K;
-        fwd_seq_f32<<<1, (unsigned)ceil_div(B * H, 32) * 32, fwd_seq_smem(T, B, I, H), s->stream>>>(
-            T, B, I, H, x, W, bias, s->top, (float *)s->hist_h, s->hist_c, (float *)s->gates, (float *)s->a_rm);
+        const int P = fwd_seq_threads_per_unit(B, H);
+        fwd_seq_f32<<<1, (unsigned)ceil_div(B * H * P, 32) * 32, fwd_seq_smem(T, B, I, H), s->stream>>>(
+            T, B, I, H, P, x, W, bias, s->top, (float *)s->hist_h, s->hist_c, (float *)s->gates, (float *)s->a_rm);
         s->launches += 1;
         return cudaGetLastError();
     }
@@ -368,7 +408,8 @@ cudaError_t fp32_backward_steps(stacklstm *s)
     const float *WT = (const float *)s->w_fwd;
     float *dG = (float *)s->dG;
     if (s->fp32_one_cta) {
-        bwd_seq_f32<<<1, (unsigned)ceil_div(B * H, 32) * 32, bwd_seq_smem(T, B, H), s->stream>>>(T, B, I, H, s->top, (const float *)s->gates,
+        const int P = fwd_seq_threads_per_unit(B, H);
+        bwd_seq_f32<<<1, (unsigned)ceil_div(B * H * P, 32) * 32, bwd_seq_smem(T, B, H), s->stream>>>(T, B, I, H, P, s->top, (const float *)s->gates,
                                                                          s->hist_c, WT, s->dhist_h, s->dhist_c, dG);
         s->launches += 1;
         return cudaGetLastError();
@@ -379,7 +420,7 @@ cudaError_t fp32_backward_steps(stacklstm *s)
         bwd_pointwise_f32<<<pw_grid, 256, 0, s->stream>>>(t, B, H, s->top, (const float *)s->gates, s->hist_c,
                                                           s->dhist_h, s->dhist_c, dG);
         bwd_contract_f32<<<dim3(ceil_div(H, threads), B), threads, sizeof(float) * G, s->stream>>>(
-            t, B, I, H, s->top, WT, dG, s->dhist_h);
+            t, B, I, H, fwd_seq_threads_per_unit(B, H), s->top, WT, dG, s->dhist_h);
     }
     s->launches += 2 * T;
     return cudaGetLastError();
