@@ -148,7 +148,14 @@ __global__ void dx_f32(int I, int H, const float *__restrict__ WT, const float *
     const int k = blockIdx.x * blockDim.x + threadIdx.x;
     if (k >= I) return;
     float acc = 0.0f;
-    for (int n = 0; n < G; ++n) acc = fmaf(g_s[n], WT[(size_t)n * K + k], acc);
+    for (int n0 = 0; n0 < G; n0 += 8) {  // eight weights loaded, then used in order
+        float wv[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) wv[i] = n0 + i < G ? WT[(size_t)(n0 + i) * K + k] : 0.0f;
+#pragma unroll
+        for (int i = 0; i < 8; ++i)
+            if (n0 + i < G) acc = fmaf(g_s[n0 + i], wv[i], acc);
+    }
     dx[r * I + k] = acc;
 }
 
@@ -161,12 +168,25 @@ __global__ void dw_f32(size_t R, int K, int G, const float *__restrict__ a_rm, c
     for (size_t e = blockIdx.x * (size_t)blockDim.x + threadIdx.x; e < n_out; e += (size_t)gridDim.x * blockDim.x) {
         const int k = (int)(e / G), n = (int)(e - (size_t)k * G);
         float acc = 0.0f, comp = 0.0f;
-        for (size_t r = 0; r < R; ++r) {
-            const float term = (k < K ? a_rm[r * K + k] : 1.0f) * dG[r * G + n];
-            const float y = term - comp;
-            const float t = acc + y;
-            comp = (t - acc) - y;
-            acc = t;
+        // eight rows' operands loaded before they are summed (in row order), so that their
+        // loads are in flight together
+        for (size_t r0 = 0; r0 < R; r0 += 8) {
+            float av[8], gv[8];
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+                const size_t r = r0 + i;
+                av[i] = r < R && k < K ? a_rm[r * K + k] : 1.0f;
+                gv[i] = r < R ? dG[r * G + n] : 0.0f;
+            }
+#pragma unroll
+            for (int i = 0; i < 8; ++i)
+                if (r0 + i < R) {
+                    const float term = av[i] * gv[i];
+                    const float y = term - comp;
+                    const float t = acc + y;
+                    comp = (t - acc) - y;
+                    acc = t;
+                }
         }
         if (k < K) {
             if (dW) dW[(size_t)k * G + n] = acc;
@@ -409,8 +429,8 @@ cudaError_t fp32_backward_steps(stacklstm *s)
     float *dG = (float *)s->dG;
     if (s->fp32_one_cta) {
         const int P = fwd_seq_threads_per_unit(B, H);
-        bwd_seq_f32<<<1, (unsigned)ceil_div(B * H * P, 32) * 32, bwd_seq_smem(T, B, H), s->stream>>>(T, B, I, H, P, s->top, (const float *)s->gates,
-                                                                         s->hist_c, WT, s->dhist_h, s->dhist_c, dG);
+        bwd_seq_f32<<<1, (unsigned)ceil_div(B * H * P, 32) * 32, bwd_seq_smem(T, B, H), s->stream>>>(
+            T, B, I, H, P, s->top, (const float *)s->gates, s->hist_c, WT, s->dhist_h, s->dhist_c, dG);
         s->launches += 1;
         return cudaGetLastError();
     }
