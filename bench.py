@@ -508,9 +508,30 @@ def hd_launches(hd):
     return sum(v[1] for v in bd.stacklstm_get_timing(hd).values())
 
 
+def packed(tensors: dict, keys, device=None, align: int = 256):
+    """One buffer (pinned host memory, or device memory) holding the given tensors back to
+    back at 256-byte-aligned offsets; returns (buffer, {key: view of the buffer with that
+    tensor's dtype and shape})."""
+    import torch
+    offs, n = {}, 0
+    for k in keys:
+        t = tensors[k]
+        n = (n + align - 1) // align * align
+        offs[k] = n
+        n += t.numel() * t.element_size()
+    buf = (torch.empty(n, dtype=torch.uint8, device=device) if device is not None
+           else torch.empty(n, dtype=torch.uint8).pin_memory())
+    views = {k: buf[offs[k]:offs[k] + tensors[k].numel() * tensors[k].element_size()].view(tensors[k].dtype)
+             .view(tensors[k].shape) for k in keys}
+    return buf, views
+
+
 def measure_e2e(w, hd, ins, out, steps, flush):
     """Same metric through the ABI with the step's inputs copied from pinned host memory
-    and its results (all gradients, final pointers) read back, inside the timed events."""
+    and its results (all gradients, final pointers) read back, inside the timed events. The
+    inputs live in one pinned host buffer and one device buffer, and so do the results (each
+    tensor a 256-byte-aligned view the library reads or writes in place): one copy each way
+    a step, the same bytes as a copy per tensor, without a copy's fixed cost per tensor."""
     import torch
     from paper_1904_03409_gb300 import runner
 
@@ -518,21 +539,25 @@ def measure_e2e(w, hd, ins, out, steps, flush):
     stream = torch.cuda.current_stream(dev)
     keys_in = ["x", "ops", "h0", "c0", "W", "bias", "d_top_h"]
     keys_out = ["p_final", "dx", "dh0", "dc0", "dW", "dbias"]
-    host_in = {k: ins[k].cpu().pin_memory() for k in keys_in}
-    host_out = {k: torch.empty(out[k].shape, dtype=out[k].dtype).pin_memory() for k in keys_out}
-    h2d = sum(t.numel() * t.element_size() for t in host_in.values())
-    d2h = sum(t.numel() * t.element_size() for t in host_out.values())
+    host_in_buf, host_in = packed(ins, keys_in)
+    for k in keys_in:
+        host_in[k].copy_(ins[k].cpu())
+    dev_in_buf, dev_in = packed(ins, keys_in, dev)
+    host_out_buf, _ = packed(out, keys_out)
+    dev_out_buf, dev_out = packed(out, keys_out, dev)
+    ins_e = dict(ins, **dev_in)
+    out_e = dict(out, **dev_out)
+    h2d = host_in_buf.numel()
+    d2h = host_out_buf.numel()
     n = max(3, min(steps, 50))
     evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n)]
     torch.cuda.synchronize(dev)
     for i in range(n):
         flush.zero_()
         evs[i][0].record(stream)
-        for k in keys_in:
-            ins[k].copy_(host_in[k], non_blocking=True)
-        runner.forward_backward(hd, ins, out)
-        for k in keys_out:
-            host_out[k].copy_(out[k], non_blocking=True)
+        dev_in_buf.copy_(host_in_buf, non_blocking=True)
+        runner.forward_backward(hd, ins_e, out_e)
+        host_out_buf.copy_(dev_out_buf, non_blocking=True)
         evs[i][1].record(stream)
     torch.cuda.synchronize(dev)
     total = sum(a.elapsed_time(b) for a, b in evs)
