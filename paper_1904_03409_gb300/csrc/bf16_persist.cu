@@ -316,9 +316,15 @@ __device__ __forceinline__ uint32_t stg_swz(uint32_t r, uint32_t q)
 // epilogue issued after the barrier (large backward +5.6 %, stress forward +6 %).
 constexpr int kRelBar = 4;
 template <int U, int EP, bool kFwd, int KS>
-__host__ __device__ constexpr bool rel_warp()
+__host__ __device__ constexpr bool rel_warp_variant()
 {
     return !kFwd && KS == 1 && EP == 1 && U == 32 && defer_dhist<EP>();
+}
+// the same for every thread of the launch: that variant, with more row tiles than slots
+template <int U, int EP, bool kFwd, int KS>
+__device__ __forceinline__ bool rel_warp(const WsArgs &p)
+{
+    return rel_warp_variant<U, EP, kFwd, KS>() && p.n_rt > p.n_slot;
 }
 
 struct EpiCtx {
@@ -812,7 +818,7 @@ __device__ __forceinline__ void epilogue_loop(const StepArgs &a, const WsArgs &p
         tc::fence_proxy_async_global();
         if constexpr (kFwd) tc::fence_proxy_async();  // staging-tile writes -> the tensor store
         __syncwarp();
-        if constexpr (rel_warp<U, EP, kFwd, KS>()) {
+        if (rel_warp<U, EP, kFwd, KS>(p)) {
             tc::bar_sync(kRelBar, (E + 1) * 32);
         } else {
             tc::bar_sync(2, E * 32);
@@ -866,7 +872,7 @@ __device__ __forceinline__ void epilogue_loop(const StepArgs &a, const WsArgs &p
     }
     // the release warp's last barrier, after every tile (or after an abort, at the tile the
     // epilogue left): the tiles completed, k, tell it that this one releases nothing
-    if constexpr (rel_warp<U, EP, kFwd, KS>()) {
+    if (rel_warp<U, EP, kFwd, KS>(p)) {
         if (e.tid == 0) *e.c.rel_end = k;
         tc::bar_sync(kRelBar, (E + 1) * 32);
     }
@@ -1264,7 +1270,7 @@ step_ws(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtens
         // with release semantics. The epilogue ends with one more barrier, before which it
         // records the tiles it completed: that barrier (k == *rel_end) releases nothing and
         // ends this loop, also after an abort
-        if constexpr (rel_warp<U, EP, kFwd, KS>()) {
+        if (rel_warp<U, EP, kFwd, KS>(p)) {
             for (int k = 0;; ++k) {
                 tc::bar_sync(kRelBar, (E + 1) * 32);
                 if (k >= *c.rel_end) break;
