@@ -234,40 +234,73 @@ head_scatter(int NR, int B, int H, const float *__restrict__ du, const int4 *__r
     }
 }
 
-// out[i] = sum over s of part[s][i], in s order; element i goes to out0 below n0, else
-// out1 below n0 + n1, else out2.
-__global__ void head_reduce(const float *__restrict__ part, int S, size_t n0, size_t n1, size_t n2, float *out0,
-                            float *out1, float *out2)
+// out[i] = (a0 + a1) + (a2 + a3), a_k the sum over the parts s = k mod 4 in s order; element
+// i goes to out0 below n0, else out1 below n0 + n1, else out2. A CTA takes 32 elements (one
+// per lane) and its warp k the chain a_k, with 16 loads in flight per pass, so the CTAs of a
+// narrow output need not walk all S parts one load at a time.
+__global__ void __launch_bounds__(128)
+head_reduce(const float *__restrict__ part, int S, size_t n0, size_t n1, size_t n2, float *out0, float *out1,
+            float *out2)
 {
+    __shared__ float chain[4][32];
     const size_t n = n0 + n1 + n2;
-    for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < n; i += (size_t)gridDim.x * blockDim.x) {
-        // four interleaved partial sums (part s goes to sum s mod 4), added in that order:
-        // a fixed order, with four independent chains of loads
-        float a4[4] = {0.0f, 0.0f, 0.0f, 0.0f};
-        int s = 0;
-        for (; s + 4 <= S; s += 4)
+    const int lane = threadIdx.x & 31, k = threadIdx.x >> 5;
+    const size_t i = blockIdx.x * (size_t)32 + lane;
+    float acc = 0.0f;
+    if (i < n) {
+        int s = k;
+        for (; s + 4 * 15 < S; s += 4 * 16) {
+            float v[16];
 #pragma unroll
-            for (int k = 0; k < 4; ++k) a4[k] += part[(size_t)(s + k) * n + i];
-        for (; s < S; ++s) a4[s & 3] += part[(size_t)s * n + i];
-        const float acc = (a4[0] + a4[1]) + (a4[2] + a4[3]);
+            for (int u = 0; u < 16; ++u) v[u] = part[(size_t)(s + 4 * u) * n + i];
+#pragma unroll
+            for (int u = 0; u < 16; ++u) acc += v[u];
+        }
+        for (; s < S; s += 4) acc += part[(size_t)s * n + i];
+    }
+    chain[k][lane] = acc;
+    __syncthreads();
+    if (k == 0 && i < n) {
+        const float a = (chain[0][lane] + chain[1][lane]) + (chain[2][lane] + chain[3][lane]);
         if (i < n0)
-            out0[i] = acc;
+            out0[i] = a;
         else if (i < n0 + n1)
-            out1[i - n0] = acc;
+            out1[i - n0] = a;
         else
-            out2[i - n0 - n1] = acc;
+            out2[i - n0 - n1] = a;
     }
 }
 
-// dWp [P][K] = the sum over s of the parts of dWp^T [s][K][P], in s order.
-__global__ void head_reduce_t(const float *__restrict__ part, int S, int P, int K, float *__restrict__ dWp)
+// dWp [P][K] = the sum over s of the parts of dWp^T [s][K][P], in s order. A CTA (32 x 8
+// threads) takes a 32 x 32 tile: its lanes read 32 consecutive j of a part row, each thread
+// sums four columns c, and the tile is written transposed through shared memory.
+__global__ void __launch_bounds__(256)
+head_reduce_t(const float *__restrict__ part, int S, int P, int K, float *__restrict__ dWp)
 {
-    const size_t n = (size_t)P * K;
-    for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < n; i += (size_t)gridDim.x * blockDim.x) {
-        const int j = (int)(i / K), c = (int)(i % K);
-        float acc = 0.0f;
-        for (int s = 0; s < S; ++s) acc += part[((size_t)s * K + c) * P + j];
-        dWp[i] = acc;
+    __shared__ float tile[32][33];  // [c][j]
+    const int c0 = blockIdx.x * 32, j0 = blockIdx.y * 32, tx = threadIdx.x, ty = threadIdx.y;
+    const int j = j0 + tx;
+    float acc[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+    if (j < P) {
+#pragma unroll 4
+        for (int s = 0; s < S; ++s) {
+            float v[4];
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const int c = c0 + ty + 8 * u;
+                v[u] = c < K ? part[((size_t)s * K + c) * P + j] : 0.0f;
+            }
+#pragma unroll
+            for (int u = 0; u < 4; ++u) acc[u] += v[u];
+        }
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u) tile[ty + 8 * u][tx] = acc[u];
+    __syncthreads();
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+        const int jj = j0 + ty + 8 * u, c = c0 + tx;
+        if (jj < P && c < K) dWp[(size_t)jj * K + c] = tile[tx][ty + 8 * u];
     }
 }
 
@@ -407,9 +440,9 @@ sl_status stacklstm_head_run(stacklstm_head_t h, const void *y_stack, const void
     if (!e) e = bf16_pack_kmajor(h->dpb, P, true, P, NR, h->dpt_k, st, sms);
     if (!e) e = bf16_gemm(h->ut, h->NR8, K, NR, h->dpt_k, P, h->part3, h->S3, st, sms, kHeadWaitLimit, h->err);
     if (!e) {
-        head_reduce_t<<<grid_n((size_t)P * K), 256, 0, st>>>(h->part3, h->S3, P, K, dWp);
-        head_reduce<<<grid_n((size_t)A * P + P + A), 256, 0, st>>>(h->part, (int)nblk, (size_t)A * P, (size_t)P,
-                                                                   (size_t)A, dWz, ddp, dq);
+        head_reduce_t<<<dim3(ceil_div(K, 32), ceil_div(P, 32)), dim3(32, 8), 0, st>>>(h->part3, h->S3, P, K, dWp);
+        head_reduce<<<ceil_div((size_t)A * P + P + A, 32), 128, 0, st>>>(h->part, (int)nblk, (size_t)A * P,
+                                                                         (size_t)P, (size_t)A, dWz, ddp, dq);
         e = cudaGetLastError();
     }
     if (prev >= 0) cudaSetDevice(prev);
